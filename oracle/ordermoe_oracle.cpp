@@ -1,0 +1,503 @@
+// OrderMoE CPU oracle.
+//
+// TEST INFRASTRUCTURE ONLY. This file is the slow, plain reference that the
+// CUDA library is checked against. Only the test suite, the smoke check in
+// __graft_entry__.py and the CPU-baseline leg of bench.py may load it. It
+// shares no code, header, table or helper with the CUDA library, and the CUDA
+// library never calls it.
+//
+// Paper: "OrderMoE: an expert similarity driven distributed edge MoE
+// inference" (arXiv 2607.17154). Every function names the section and
+// equation it follows. Floating point is fp64 unless a step is stated to run
+// in fp32 (the selection's cost compares, which the method decides in fp32
+// on both sides from identical fp32 tables). Build with -ffp-contract=off so
+// that no multiply-add is fused.
+//
+// Readings where the paper is silent or garbled (listed again in the design doc):
+//  * top-k > 1: the selection of Alg. 2 runs once per routed slot, in rank
+//    order; a substitute may not be an expert the token already routes to or
+//    has already been given (every token keeps k distinct experts).
+//  * the token location after a layer is the server of slot 0 (highest gate).
+//  * phi in Eq. 18 is the identity.
+//  * d_ref in Eq. 38 is the compute-only delay c/F_a on the home server a.
+//  * argmin ties in Eq. 43: lower cost, then exact before substitute, then
+//    the token's current server, then lower server id, then lower expert id.
+//  * grouping (Eqs. 24-25): experts in decreasing frequency (ties: lower
+//    index); argmax ties go to the earlier-created dominant; group id = the
+//    dominant's creation order.
+//  * placement (Eqs. 29-31): the within-layer order is memory demand desc,
+//    then importance desc, then index asc; score ties go to the lower server;
+//    the used memory b_m accumulates over layers (Alg. 1 initialises it once).
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <vector>
+
+namespace {
+
+float bf16_bits_to_float(uint16_t h) {
+  uint32_t u = static_cast<uint32_t>(h) << 16;
+  float f;
+  std::memcpy(&f, &u, sizeof f);
+  return f;
+}
+
+// Round-to-nearest-even fp32 -> bf16 (the rounding the bf16 format defines).
+uint16_t float_to_bf16_bits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, sizeof u);
+  if ((u & 0x7fffffffu) > 0x7f800000u) return static_cast<uint16_t>((u >> 16) | 0x0040u);
+  uint32_t lsb = (u >> 16) & 1u;
+  u += 0x7fffu + lsb;
+  return static_cast<uint16_t>(u >> 16);
+}
+
+double bf(const uint16_t* p, int64_t i) { return static_cast<double>(bf16_bits_to_float(p[i])); }
+
+// Rank order used for top-k: larger logit first, equal logits by lower index.
+bool ranks_before(float a, int ia, float b, int ib) {
+  if (a != b) return a > b;
+  return ia < ib;
+}
+
+}  // namespace
+
+extern "C" {
+
+// Status codes of this oracle (independent of the library's).
+enum { ORC_OK = 0, ORC_BAD_ARG = 1, ORC_NAN = 2, ORC_CAPACITY = 3 };
+
+// ---------------------------------------------------------------------------
+// Router logits, Eq. 3 written per token: logits[t][e] = sum_c X[t][c] W[e][c]
+// (the router's response; Alg. 2 obtains the target expert from it). fp64
+// accumulation, stored as fp32.
+int orc_router_logits(const uint16_t* X, const uint16_t* W, int T, int E, int d, float* logits) {
+  if (T < 0 || E <= 0 || d <= 0) return ORC_BAD_ARG;
+  for (int t = 0; t < T; ++t)
+    for (int e = 0; e < E; ++e) {
+      double acc = 0.0;
+      for (int c = 0; c < d; ++c) acc += bf(X, (int64_t)t * d + c) * bf(W, (int64_t)e * d + c);
+      logits[(int64_t)t * E + e] = static_cast<float>(acc);
+    }
+  return ORC_OK;
+}
+
+// Softmax over all E experts in fp64, then the k highest logits (ties: lower
+// index). Gate weight of slot j = p[idx_j], renormalised over the k slots when
+// renorm != 0. A NaN logit is an error.
+int orc_topk(const float* logits, int T, int E, int k, int renorm, int32_t* idx, float* w) {
+  if (T < 0 || E <= 0 || k <= 0 || k > E) return ORC_BAD_ARG;
+  std::vector<int> order(E);
+  std::vector<double> p(E);
+  for (int t = 0; t < T; ++t) {
+    const float* l = logits + (int64_t)t * E;
+    for (int e = 0; e < E; ++e)
+      if (std::isnan(l[e])) return ORC_NAN;
+    for (int e = 0; e < E; ++e) order[e] = e;
+    std::sort(order.begin(), order.end(),
+              [&](int a, int b) { return ranks_before(l[a], a, l[b], b); });
+    double mx = static_cast<double>(l[order[0]]);
+    double s = 0.0;
+    for (int e = 0; e < E; ++e) {
+      p[e] = std::exp(static_cast<double>(l[e]) - mx);
+      s += p[e];
+    }
+    for (int e = 0; e < E; ++e) p[e] /= s;
+    double ssel = 0.0;
+    for (int j = 0; j < k; ++j) ssel += p[order[j]];
+    for (int j = 0; j < k; ++j) {
+      idx[(int64_t)t * k + j] = order[j];
+      double wj = renorm ? p[order[j]] / ssel : p[order[j]];
+      w[(int64_t)t * k + j] = static_cast<float>(wj);
+    }
+  }
+  return ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Per-layer selection tables.
+//   Qtab[r][k] = Q_l(r,k) of Eq. 18 with phi = identity, in fp32:
+//                0 for k == r, else 0.5f * (1 - min(Sim,1)).
+//   Cq[r][k]   = omega_Q * Q_l(r,k) / Qbar (the quality term of Eq. 38),
+//                fp64 then rounded to fp32; 0 where Q_l = 0.
+//   subst[r]   = bit set of R_{l,r} (Eq. 7): k != r in r's group with
+//                Sim(r,k) >= theta.
+//   A[a][s][m] = omega_T * d(s,m) / d_ref(a) (the delay term of Eq. 38) with
+//                d(s,m) = 1(s != m)(z / B_{s,m} + tau_{s,m}) + c / F_m (Eq. 37)
+//                and d_ref(a) = c / F_a; fp64 then rounded to fp32.
+//   pmask[e]   = bit set of servers m with x_{m,e} = 1.
+int orc_tables(const float* sim, const int32_t* group, const uint8_t* placement, int E, int M,
+               float theta, float qbar, const double* F, const double* B, const double* tau,
+               double z, double c, double omega_T, double omega_Q, float* Qtab, float* Cq,
+               uint64_t* subst, float* A, uint32_t* pmask) {
+  if (E <= 0 || E > 64 || M <= 0 || M > 32 || !(qbar >= 0.0f)) return ORC_BAD_ARG;
+  for (int r = 0; r < E; ++r) {
+    uint64_t bits = 0;
+    for (int k = 0; k < E; ++k) {
+      float s = sim[r * E + k];
+      float q = 0.0f;
+      if (k != r) q = 0.5f * (1.0f - std::min(s, 1.0f));
+      Qtab[r * E + k] = q;
+      float cq = 0.0f;
+      if (q != 0.0f) cq = static_cast<float>(omega_Q * static_cast<double>(q) / static_cast<double>(qbar));
+      Cq[r * E + k] = cq;
+      if (k != r && group[k] == group[r] && s >= theta) bits |= (uint64_t)1 << k;
+    }
+    subst[r] = bits;
+  }
+  for (int a = 0; a < M; ++a) {
+    double dref = c / F[a];
+    for (int s = 0; s < M; ++s)
+      for (int m = 0; m < M; ++m) {
+        double comp = c / F[m];
+        double dl = comp;
+        if (s != m) {
+          double trans = z / B[s * M + m] + tau[s * M + m];
+          dl = trans + comp;
+        }
+        double num = omega_T * dl;
+        A[((int64_t)a * M + s) * M + m] = static_cast<float>(num / dref);
+      }
+  }
+  for (int e = 0; e < E; ++e) {
+    uint32_t bits = 0;
+    for (int m = 0; m < M; ++m)
+      if (placement[m * E + e]) bits |= 1u << m;
+    pmask[e] = bits;
+  }
+  return ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Online server-expert selection, Alg. 2 with horizon H = 1 (Phi = 0,
+// Section V-C), one routed slot at a time in rank order.
+//   s = loc[t] (Eq. 36: the home server a(i) before the first layer),
+//   feasible set (Eq. 40): (m, k) with x_{m,k} = 1, k in V_{l,r} (Eq. 8), and
+//     Qhat + Q_l(r,k) <= Qbar; a substitute must not be one of the token's
+//     routed experts nor a substitute already given to it;
+//   cost (Eq. 38) = A[a][s][m] + Cq[r][k] as one fp32 add;
+//   argmin (Eq. 43) with the tie rule listed at the top of this file;
+//   update (Eq. 44): Qhat += Q_l(r,k*); location = server of slot 0.
+// kind: 0 local exact, 1 local substitute, 2 remote exact, 3 remote substitute.
+int orc_select(const int32_t* idx, int T, int E, int k, int M, const float* Qtab, const float* Cq,
+               const uint64_t* subst, const float* A, const uint32_t* pmask, float qbar,
+               const uint8_t* home, uint8_t* loc, float* qhat, int32_t* chosen, uint8_t* server,
+               uint8_t* kind) {
+  if (E <= 0 || E > 64 || M <= 0 || M > 32 || k <= 0 || k > E) return ORC_BAD_ARG;
+  for (int t = 0; t < T; ++t) {
+    const int a = home[t];
+    const int s = loc[t];
+    if (a >= M || s >= M) return ORC_BAD_ARG;
+    float q = qhat[t];
+    uint64_t taken = 0;
+    for (int j = 0; j < k; ++j) taken |= (uint64_t)1 << idx[(int64_t)t * k + j];
+    int first_server = -1;
+    for (int j = 0; j < k; ++j) {
+      const int r = idx[(int64_t)t * k + j];
+      if (r < 0 || r >= E) return ORC_BAD_ARG;
+      bool have = false;
+      float best_cost = 0.0f;
+      int best_sub = 0, best_away = 0, best_m = 0, best_k = 0;
+      for (int kk = 0; kk < E; ++kk) {
+        const bool exact = (kk == r);
+        if (!exact) {
+          if (!((subst[r] >> kk) & 1u)) continue;           // e_k in R_{l,r}
+          if ((taken >> kk) & 1u) continue;                   // distinct experts
+          if (!(q + Qtab[r * E + kk] <= qbar)) continue;      // budget, Eq. 40
+        }
+        for (int m = 0; m < M; ++m) {
+          if (!((pmask[kk] >> m) & 1u)) continue;             // x_{m,k} = 1
+          const float cost = A[((int64_t)a * M + s) * M + m] + (exact ? 0.0f : Cq[r * E + kk]);
+          const int sub = exact ? 0 : 1;
+          const int away = (m != s) ? 1 : 0;
+          bool better;
+          if (!have) better = true;
+          else if (cost != best_cost) better = cost < best_cost;
+          else if (sub != best_sub) better = sub < best_sub;
+          else if (away != best_away) better = away < best_away;
+          else if (m != best_m) better = m < best_m;
+          else better = kk < best_k;
+          if (better) {
+            have = true;
+            best_cost = cost; best_sub = sub; best_away = away; best_m = m; best_k = kk;
+          }
+        }
+      }
+      if (!have) return ORC_BAD_ARG;  // Property 1 violated: target placed nowhere
+      chosen[(int64_t)t * k + j] = best_k;
+      server[(int64_t)t * k + j] = static_cast<uint8_t>(best_m);
+      kind[(int64_t)t * k + j] = static_cast<uint8_t>(2 * best_away + best_sub);
+      if (best_sub) {
+        taken |= (uint64_t)1 << best_k;
+        q = q + Qtab[r * E + best_k];
+      }
+      if (j == 0) first_server = best_m;
+    }
+    loc[t] = static_cast<uint8_t>(first_server);
+    qhat[t] = q;
+  }
+  return ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Token permutation: a stable counting sort of the T*k (token, slot) entries
+// by executed expert. offsets[e] = number of entries with expert < e;
+// entries of one expert keep their flat (t*k + j) order. row_token[row] = t,
+// row_of[t*k + j] = row.
+int orc_dispatch(const int32_t* chosen, int T, int k, int E, int32_t* offsets, int32_t* row_token,
+                 int32_t* row_of) {
+  const int64_t n = (int64_t)T * k;
+  std::vector<int64_t> count(E, 0);
+  for (int64_t i = 0; i < n; ++i) {
+    if (chosen[i] < 0 || chosen[i] >= E) return ORC_BAD_ARG;
+    count[chosen[i]]++;
+  }
+  offsets[0] = 0;
+  for (int e = 0; e < E; ++e) offsets[e + 1] = offsets[e] + static_cast<int32_t>(count[e]);
+  std::vector<int64_t> next(E);
+  for (int e = 0; e < E; ++e) next[e] = offsets[e];
+  for (int64_t i = 0; i < n; ++i) {
+    int64_t row = next[chosen[i]]++;
+    row_token[row] = static_cast<int32_t>(i / k);
+    row_of[i] = static_cast<int32_t>(row);
+  }
+  return ORC_OK;
+}
+
+// X_perm[row] = X[row_token[row]] (a copy of bf16 rows).
+int orc_gather_rows(const uint16_t* X, const int32_t* row_token, int64_t R, int d, uint16_t* Xp) {
+  for (int64_t r = 0; r < R; ++r)
+    std::memcpy(Xp + r * d, X + (int64_t)row_token[r] * d, sizeof(uint16_t) * d);
+  return ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// SwiGLU expert FFN (the Mixtral-shaped experts of Section VI-A), one row at
+// a time, rows given with their expert:
+//   g = x W1_e^T, u = x W3_e^T (fp64), h = bf16(fp32(silu(g) * u)),
+//   silu(g) = g / (1 + exp(-g)); y = bf16(fp32(h W2_e^T)) (fp64 accumulate).
+// W1, W3: [E][dff][d]; W2: [E][d][dff]; all bf16 bits.
+int orc_ffn_rows(const uint16_t* Xrows, const int32_t* row_expert, int64_t R, const uint16_t* W1,
+                 const uint16_t* W3, const uint16_t* W2, int E, int d, int dff, uint16_t* H,
+                 uint16_t* Y) {
+  if (E <= 0 || d <= 0 || dff <= 0) return ORC_BAD_ARG;
+#pragma omp parallel for schedule(dynamic, 1)
+  for (int64_t r = 0; r < R; ++r) {
+    const int e = row_expert[r];
+    if (e < 0 || e >= E) continue;
+    const uint16_t* x = Xrows + r * d;
+    uint16_t* h = H + r * dff;
+    for (int n = 0; n < dff; ++n) {
+      const uint16_t* w1 = W1 + ((int64_t)e * dff + n) * d;
+      const uint16_t* w3 = W3 + ((int64_t)e * dff + n) * d;
+      double g = 0.0, u = 0.0;
+      for (int c = 0; c < d; ++c) {
+        double xc = bf(x, c);
+        g += xc * bf(w1, c);
+        u += xc * bf(w3, c);
+      }
+      double silu = g / (1.0 + std::exp(-g));
+      h[n] = float_to_bf16_bits(static_cast<float>(silu * u));
+    }
+    for (int o = 0; o < d; ++o) {
+      const uint16_t* w2 = W2 + ((int64_t)e * d + o) * dff;
+      double acc = 0.0;
+      for (int n = 0; n < dff; ++n) acc += bf(h, n) * bf(w2, n);
+      Y[r * d + o] = float_to_bf16_bits(static_cast<float>(acc));
+    }
+  }
+  return ORC_OK;
+}
+
+// Weighted combine: y[t] = bf16(sum_j w[t][j] * Y_perm[row_of[t][j]]), fp64
+// accumulation over slots j = 0..k-1.
+int orc_combine(const uint16_t* Yp, const int32_t* row_of, const float* w, int T, int k, int d,
+                uint16_t* y) {
+  for (int t = 0; t < T; ++t)
+    for (int c = 0; c < d; ++c) {
+      double acc = 0.0;
+      for (int j = 0; j < k; ++j) {
+        int64_t row = row_of[(int64_t)t * k + j];
+        acc += static_cast<double>(w[(int64_t)t * k + j]) * bf(Yp, row * d + c);
+      }
+      y[(int64_t)t * d + c] = float_to_bf16_bits(static_cast<float>(acc));
+    }
+  return ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Expert similarity, Eqs. 3-4: H = W_r X_cal^T (fp64), Sim(i,j) = cosine of
+// rows i and j of H, fp64 then rounded to fp32; the diagonal is exactly 1 and
+// a pair with a zero-norm row has Sim 0. Also returns the fp32 H when Hout is
+// not null ([E][N]).
+int orc_similarity(const uint16_t* W, const uint16_t* Xc, int E, int d, int64_t N, float* sim,
+                   float* Hout) {
+  std::vector<double> H((size_t)E * N);
+#pragma omp parallel for schedule(static)
+  for (int64_t n = 0; n < N; ++n)
+    for (int e = 0; e < E; ++e) {
+      double acc = 0.0;
+      for (int c = 0; c < d; ++c) acc += bf(W, (int64_t)e * d + c) * bf(Xc, n * d + c);
+      H[(size_t)e * N + n] = acc;
+    }
+  if (Hout)
+    for (size_t i = 0; i < H.size(); ++i) Hout[i] = static_cast<float>(H[i]);
+  std::vector<double> norm(E);
+  for (int e = 0; e < E; ++e) {
+    double s = 0.0;
+    for (int64_t n = 0; n < N; ++n) s += H[(size_t)e * N + n] * H[(size_t)e * N + n];
+    norm[e] = std::sqrt(s);
+  }
+  for (int i = 0; i < E; ++i)
+    for (int j = 0; j < E; ++j) {
+      if (i == j) { sim[i * E + j] = 1.0f; continue; }
+      if (norm[i] == 0.0 || norm[j] == 0.0) { sim[i * E + j] = 0.0f; continue; }
+      double dot = 0.0;
+      for (int64_t n = 0; n < N; ++n) dot += H[(size_t)i * N + n] * H[(size_t)j * N + n];
+      sim[i * E + j] = static_cast<float>(dot / (norm[i] * norm[j]));
+    }
+  return ORC_OK;
+}
+
+// Activation counts n_j of Eq. 5 from given fp32 logits [N][E]: the number
+// of tokens whose top-kf experts (rank order of orc_topk) include j.
+int orc_expert_counts(const float* logits, int64_t N, int E, int kf, int32_t* count) {
+  if (kf <= 0 || kf > E) return ORC_BAD_ARG;
+  for (int e = 0; e < E; ++e) count[e] = 0;
+  std::vector<int> order(E);
+  for (int64_t n = 0; n < N; ++n) {
+    const float* l = logits + n * E;
+    for (int e = 0; e < E; ++e) order[e] = e;
+    std::sort(order.begin(), order.end(),
+              [&](int a, int b) { return ranks_before(l[a], a, l[b], b); });
+    for (int j = 0; j < kf; ++j) count[order[j]]++;
+  }
+  return ORC_OK;
+}
+
+// Depth-aware threshold, Eq. 6, layers l = 1..N. The formula divides by
+// N - 1, so a single-layer model takes theta_single instead.
+float orc_theta(int l, int N, double theta_min, double theta_max, double theta_single) {
+  if (N <= 1) return static_cast<float>(theta_single);
+  double frac = static_cast<double>(N - l) / static_cast<double>(N - 1);
+  return static_cast<float>(theta_min + (theta_max - theta_min) * frac);
+}
+
+// Greedy representative-cover grouping, Eqs. 24-26 (Alg. 1, grouping loop).
+// Experts are visited by decreasing count (ties: lower index). dominant[g] is
+// the dominant (centre) of group g.
+int orc_group(const float* sim, const int32_t* count, int E, float theta, int32_t* group,
+              int32_t* n_groups, int32_t* dominant) {
+  std::vector<int> order(E);
+  for (int e = 0; e < E; ++e) order[e] = e;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return count[a] > count[b]; });
+  int K = 0;
+  for (int pos = 0; pos < E; ++pos) {
+    const int j = order[pos];
+    int best_g = -1;
+    float best_s = 0.0f;
+    for (int g = 0; g < K; ++g) {
+      float s = sim[j * E + dominant[g]];
+      if (best_g < 0 || s > best_s) { best_g = g; best_s = s; }
+    }
+    if (best_g < 0 || best_s < theta) {
+      dominant[K] = j;
+      group[j] = K;
+      ++K;
+    } else {
+      group[j] = best_g;
+    }
+  }
+  *n_groups = K;
+  return ORC_OK;
+}
+
+// Importance, Eqs. 27-28: rho_j = mean of Sim(j,k) over k in j's group (j
+// itself included), I_j = alpha_f f_j + alpha_r rho_j, f_j = n_j / sum n.
+int orc_importance(const float* sim, const int32_t* count, const int32_t* group, int E,
+                   double alpha_f, double alpha_r, double* importance) {
+  double total = 0.0;
+  for (int e = 0; e < E; ++e) total += count[e];
+  for (int j = 0; j < E; ++j) {
+    double s = 0.0;
+    int size = 0;
+    for (int k = 0; k < E; ++k)
+      if (group[k] == group[j]) { s += sim[j * E + k]; ++size; }
+    double rho = s / size;
+    double f = total > 0.0 ? count[j] / total : 0.0;
+    importance[j] = alpha_f * f + alpha_r * rho;
+  }
+  return ORC_OK;
+}
+
+// Mandatory placement over L layers, Eqs. 29-31 and Alg. 1's placement loop:
+// per layer, experts in order (p desc, I desc, index asc); feasible servers
+// b_m + p <= C_m; score = lambda1 b_m / C_m + lambda2 eta (eta = experts of
+// the same group already on m in this layer); argmin, ties lower m. Experts
+// with no feasible server wait and then go to the server with the largest
+// C_m - b_m (ties lower m). b_m accumulates over layers.
+// placement: [L][M][E] u8. Returns ORC_CAPACITY if sum C < sum p, or if a
+// waiting-list expert overflowed its server.
+int orc_place(const int32_t* group, const double* importance, const double* p, int L, int E,
+              int M, const double* C, double lambda1, double lambda2, uint8_t* placement,
+              double* used) {
+  double needed = 0.0, have = 0.0;
+  for (int i = 0; i < L * E; ++i) needed += p[i];
+  for (int m = 0; m < M; ++m) have += C[m];
+  std::memset(placement, 0, (size_t)L * M * E);
+  std::vector<double> b(M, 0.0);
+  bool overflow = needed > have;
+  for (int l = 0; l < L; ++l) {
+    const int32_t* g = group + (int64_t)l * E;
+    const double* I = importance + (int64_t)l * E;
+    const double* pl = p + (int64_t)l * E;
+    uint8_t* x = placement + (int64_t)l * M * E;
+    std::vector<int> order(E);
+    for (int e = 0; e < E; ++e) order[e] = e;
+    std::sort(order.begin(), order.end(), [&](int a, int c) {
+      if (pl[a] != pl[c]) return pl[a] > pl[c];
+      if (I[a] != I[c]) return I[a] > I[c];
+      return a < c;
+    });
+    std::vector<int> waiting;
+    for (int j : order) {
+      int best = -1;
+      double best_score = 0.0;
+      for (int m = 0; m < M; ++m) {
+        if (!(b[m] + pl[j] <= C[m])) continue;
+        int eta = 0;
+        for (int k = 0; k < E; ++k)
+          if (g[k] == g[j] && x[m * E + k]) ++eta;
+        double score = lambda1 * (b[m] / C[m]) + lambda2 * static_cast<double>(eta);
+        if (best < 0 || score < best_score) { best = m; best_score = score; }
+      }
+      if (best < 0) { waiting.push_back(j); continue; }
+      x[best * E + j] = 1;
+      b[best] += pl[j];
+    }
+    for (int j : waiting) {
+      int best = 0;
+      for (int m = 1; m < M; ++m)
+        if (C[m] - b[m] > C[best] - b[best]) best = m;
+      x[best * E + j] = 1;
+      b[best] += pl[j];
+      if (b[best] > C[best]) overflow = true;
+    }
+  }
+  for (int m = 0; m < M; ++m) used[m] = b[m];
+  return overflow ? ORC_CAPACITY : ORC_OK;
+}
+
+// Local group coverage, Eq. 32 (indices read as y_{m,l,g} = 1 when server m
+// hosts at least one expert of group g in layer l). cover: [M][K].
+int orc_coverage(const uint8_t* placement_l, const int32_t* group_l, int E, int M, int K,
+                 uint8_t* cover) {
+  std::memset(cover, 0, (size_t)M * K);
+  for (int m = 0; m < M; ++m)
+    for (int e = 0; e < E; ++e)
+      if (placement_l[m * E + e]) cover[m * K + group_l[e]] = 1;
+  return ORC_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,644 @@
+"""Pins for the CPU oracle: each check ties an oracle function to something
+other than itself (exact arithmetic, a library routine on a special case, a
+closed form, an invariant the paper states, or brute-force enumeration on a
+tiny input), chosen so that a dropped term, a wrong sign or index, or a
+transposed operand fails at least one of them.
+"""
+import itertools
+from fractions import Fraction
+
+import numpy as np
+import pytest
+import scipy.special
+import torch
+from scipy.spatial.distance import cdist
+
+pytestmark = pytest.mark.filterwarnings("ignore::RuntimeWarning")
+
+
+def bf16_bits(a):
+    """float array -> bf16 bit patterns (torch's round-to-nearest-even)."""
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16)
+    return t.view(torch.int16).numpy().view(np.uint16)
+
+
+def bits_to_f(b):
+    return (np.asarray(b, np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def rnd_bf16(rng, shape, std=1.0):
+    return bf16_bits(rng.standard_normal(shape) * std)
+
+
+# --------------------------------------------------------------------------
+# Router logits (Eq. 3 per token)
+
+def test_router_logits_exact_rational(orc):
+    rng = np.random.default_rng(1)
+    X = rnd_bf16(rng, (5, 7)); W = rnd_bf16(rng, (3, 7))
+    got = orc.router_logits(X, W)
+    xf, wf = bits_to_f(X), bits_to_f(W)
+    for t in range(5):
+        for e in range(3):
+            exact = sum(Fraction(float(xf[t, c])) * Fraction(float(wf[e, c])) for c in range(7))
+            assert got[t, e] == np.float32(float(exact))
+
+
+def test_router_logits_one_hot_tokens_pick_weight_columns(orc):
+    rng = np.random.default_rng(2)
+    E, d = 3, 11
+    W = rnd_bf16(rng, (E, d))
+    cols = np.array([0, 4, 10, 7])
+    X = np.zeros((4, d), np.float32); X[np.arange(4), cols] = 1.0
+    got = orc.router_logits(bf16_bits(X), W)
+    np.testing.assert_array_equal(got, bits_to_f(W)[:, cols].T)
+
+
+# --------------------------------------------------------------------------
+# Softmax + top-k
+
+def brute_topk(l, k):
+    E = len(l)
+    rank = [sum(1 for f in range(E) if l[f] > l[e] or (l[f] == l[e] and f < e)) for e in range(E)]
+    return [rank.index(j) for j in range(k)]
+
+
+def test_topk_brute_force_and_library_softmax(orc):
+    rng = np.random.default_rng(3)
+    for E, k in [(4, 1), (6, 2), (8, 3), (5, 5)]:
+        logits = rng.standard_normal((20, E)).astype(np.float32)
+        logits[0, :] = 0.5          # all tied
+        logits[1, 1] = logits[1, 3]  # a tie inside
+        for renorm in (0, 1):
+            idx, w = orc.topk(logits, k, renorm)
+            p = scipy.special.softmax(logits.astype(np.float64), axis=1)
+            for t in range(20):
+                sel = brute_topk(list(logits[t]), k)
+                assert list(idx[t]) == sel
+                ref = p[t, sel] / (p[t, sel].sum() if renorm else 1.0)
+                np.testing.assert_allclose(w[t], ref, rtol=1e-6)
+
+
+def test_topk_nan_is_an_error(orc):
+    logits = np.zeros((2, 4), np.float32); logits[1, 2] = np.nan
+    with pytest.raises(orc.OracleError):
+        orc.topk(logits, 2)
+
+
+# --------------------------------------------------------------------------
+# Tables (Eqs. 7, 18, 37, 38)
+
+def _params(rng, M):
+    F = rng.uniform(20e12, 110e12, M)
+    B = rng.uniform(1e9, 1e10, (M, M)); B = (B + B.T) / 2
+    tau = rng.uniform(2e-4, 2e-2, (M, M)); tau = (tau + tau.T) / 2
+    return F, B, tau
+
+
+def test_tables_delay_term_closed_forms(orc):
+    rng = np.random.default_rng(4)
+    M, E = 4, 3
+    F, B, tau = _params(rng, M)
+    sim = np.eye(E, dtype=np.float32); group = np.arange(E, dtype=np.int32)
+    x = np.ones((M, E), np.uint8)
+    z, c, wT = 8192.0, 3.5e8, 0.5
+    tab = orc.tables(sim, group, x, 0.5, 0.1, F, B, tau, z, c, wT, 0.5)
+    A = tab.A.astype(np.float64)
+    for a in range(M):
+        # home server, no move: the delay equals d_ref, so the term is omega_T
+        assert tab.A[a, a, a] == np.float32(wT)
+        for s in range(M):
+            # staying on s: omega_T * F_a / F_s (Eq. 37 with no transfer)
+            np.testing.assert_allclose(A[a, s, s], wT * F[a] / F[s], rtol=1e-6)
+            for m in range(M):
+                if m == s:
+                    continue
+                # moving s -> m costs omega_T * F_a / c * (z / B_sm + tau_sm) extra
+                extra = wT * F[a] / c * (z / B[s, m] + tau[s, m])
+                np.testing.assert_allclose(A[a, s, m] - A[a, m, m], extra, rtol=1e-5)
+    # no transfer cost at all: the term depends on the executing server only
+    tab0 = orc.tables(sim, group, x, 0.5, 0.1, F, B, tau * 0, 0.0, c, wT, 0.5)
+    for a, s, m in itertools.product(range(M), repeat=3):
+        np.testing.assert_allclose(tab0.A[a, s, m], wT * F[a] / F[m], rtol=1e-6)
+
+
+def test_tables_quality_terms_closed_forms(orc):
+    E = 4
+    sim = np.array([[1.0, 0.5, -1.0, 0.75],
+                    [0.5, 1.0, 0.0, 1.25],   # 1.25: rounding overshoot, clamps to zero loss
+                    [-1.0, 0.0, 1.0, 0.5],
+                    [0.75, 1.25, 0.5, 1.0]], np.float32)
+    group = np.array([0, 0, 1, 0], np.int32)
+    x = np.ones((2, E), np.uint8)
+    F = np.array([1e13, 2e13]); B = np.ones((2, 2)) * 1e9; tau = np.zeros((2, 2))
+    tab = orc.tables(sim, group, x, 0.6, 0.25, F, B, tau, 1.0, 1.0, 0.5, 0.5)
+    expect_Q = np.array([[0, 0.25, 1.0, 0.125],
+                         [0.25, 0, 0.5, 0.0],
+                         [1.0, 0.5, 0, 0.25],
+                         [0.125, 0.0, 0.25, 0]], np.float32)
+    np.testing.assert_array_equal(tab.Qtab, expect_Q)
+    # Cq = omega_Q * Q / Qbar = 0.5 * Q / 0.25 = 2 Q
+    np.testing.assert_array_equal(tab.Cq, 2 * expect_Q)
+    # R_{l,r}: same group, k != r, Sim >= 0.6
+    subst = [int(v) for v in tab.subst]
+    assert subst[0] == (1 << 3)              # 1: Sim 0.5 < 0.6; 3: 0.75
+    assert subst[1] == (1 << 3)              # 3: Sim 1.25 >= 0.6
+    assert subst[2] == 0                     # alone in group 1
+    assert subst[3] == (1 << 0) | (1 << 1)
+
+
+def test_tables_placement_mask(orc):
+    E, M = 5, 3
+    x = np.zeros((M, E), np.uint8); x[0, 0] = x[2, 0] = x[1, 3] = x[2, 4] = x[0, 1] = x[1, 2] = 1
+    F = np.ones(M) * 1e13; B = np.ones((M, M)) * 1e9; tau = np.zeros((M, M))
+    tab = orc.tables(np.eye(E, dtype=np.float32), np.arange(E, dtype=np.int32), x, 0.5, 0.1,
+                     F, B, tau, 1.0, 1.0, 0.5, 0.5)
+    assert [int(v) for v in tab.pmask] == [0b101, 0b001, 0b010, 0b010, 0b100]
+
+
+# --------------------------------------------------------------------------
+# Selection (Alg. 2, H = 1) against brute-force enumeration of every
+# (server, expert) pair, following Eqs. 7, 8, 18, 37, 38, 40, 43, 44.
+
+def brute_select(idx, sim, group, x, theta, qbar, F, B, tau, z, c, wT, wQ, home, loc, qhat):
+    T, k = idx.shape
+    M, E = x.shape
+    f32 = np.float32
+    chosen = np.zeros((T, k), np.int32); server = np.zeros((T, k), np.uint8)
+    kind = np.zeros((T, k), np.uint8)
+    loc2 = loc.copy(); q2 = qhat.copy()
+
+    def quality(r, kk):  # Eq. 18, phi = identity, fp32
+        if kk == r:
+            return f32(0)
+        return f32(f32(0.5) * (f32(1) - min(f32(sim[r, kk]), f32(1))))
+
+    def delay_term(a, s, m):  # Eqs. 37-38 delay term, fp64 -> fp32
+        dl = c / F[m] if s == m else (z / B[s, m] + tau[s, m]) + c / F[m]
+        return f32(wT * dl / (c / F[a]))
+
+    for t in range(T):
+        a, s, q = int(home[t]), int(loc[t]), f32(qhat[t])
+        used = set(int(v) for v in idx[t])
+        for j in range(k):
+            r = int(idx[t, j])
+            cands = []
+            for m in range(M):
+                for kk in range(E):
+                    if not x[m, kk]:
+                        continue
+                    if kk != r:
+                        if group[kk] != group[r] or not (sim[r, kk] >= f32(theta)):
+                            continue
+                        if kk in used:
+                            continue
+                        if not (f32(q + quality(r, kk)) <= f32(qbar)):
+                            continue
+                    Q = quality(r, kk)
+                    qterm = f32(0) if Q == 0 else f32(wQ * float(Q) / float(f32(qbar)))
+                    cost = f32(delay_term(a, s, m) + (f32(0) if kk == r else qterm))
+                    cands.append((cost, kk != r, m != s, m, kk))
+            best = min(cands)
+            _, sub, away, m, kk = best
+            chosen[t, j] = kk; server[t, j] = m; kind[t, j] = 2 * away + sub
+            if sub:
+                used.add(kk)
+                q = f32(q + quality(r, kk))
+            if j == 0:
+                loc2[t] = m
+        q2[t] = q
+    return chosen, server, kind, loc2, q2
+
+
+def random_case(rng, E, M, k, T, kgroups):
+    Wt = rng.standard_normal((E, 5))
+    Wt[:, 0] += 3.0 * (np.arange(E) % kgroups)  # correlate same-group rows
+    sim = (1 - cdist(Wt, Wt, "cosine")).astype(np.float32)
+    np.fill_diagonal(sim, 1.0)
+    group = (np.arange(E) % kgroups).astype(np.int32)
+    x = (rng.random((M, E)) < 0.4).astype(np.uint8)
+    for e in range(E):
+        if not x[:, e].any():
+            x[rng.integers(M), e] = 1
+    F, B, tau = _params(rng, M)
+    if rng.random() < 0.5:   # cheap links so that remote candidates compete
+        tau = tau * 1e-4
+    theta = float(rng.choice([-0.5, 0.0, 0.3, 0.6]))
+    qbar = float(rng.choice([0.0, 0.1, 0.3, 1.0]))
+    logits = rng.standard_normal((T, E)).astype(np.float32)
+    idx = np.argsort(-logits, axis=1, kind="stable")[:, :k].astype(np.int32)
+    home = rng.integers(0, M, T).astype(np.uint8)
+    loc = np.where(rng.random(T) < 0.5, home, rng.integers(0, M, T)).astype(np.uint8)
+    qhat = (rng.random(T) * qbar * 0.8).astype(np.float32)
+    return dict(idx=idx, sim=sim, group=group, x=x, theta=theta, qbar=qbar, F=F, B=B, tau=tau,
+                z=2048.0, c=1e9, wT=float(rng.choice([0.0, 0.3, 0.5])), wQ=0.5,
+                home=home, loc=loc, qhat=qhat)
+
+
+def run_oracle_select(orc, cs):
+    tab = orc.tables(cs["sim"], cs["group"], cs["x"], cs["theta"], cs["qbar"], cs["F"], cs["B"],
+                     cs["tau"], cs["z"], cs["c"], cs["wT"], cs["wQ"])
+    return orc.select(cs["idx"], tab, cs["home"], cs["loc"], cs["qhat"]), tab
+
+
+def test_select_matches_brute_force(orc):
+    rng = np.random.default_rng(5)
+    n = 0
+    for trial in range(300):
+        E = int(rng.integers(2, 7)); M = int(rng.integers(1, 4)); k = int(rng.integers(1, min(E, 3) + 1))
+        cs = random_case(rng, E, M, k, 6, int(rng.integers(1, 3)))
+        (ch, sv, kd, loc, q), _ = run_oracle_select(orc, cs)
+        bch, bsv, bkd, bloc, bq = brute_select(**cs)
+        np.testing.assert_array_equal(ch, bch)
+        np.testing.assert_array_equal(sv, bsv)
+        np.testing.assert_array_equal(kd, bkd)
+        np.testing.assert_array_equal(loc, bloc)
+        np.testing.assert_array_equal(q, bq)
+        n += int((kd % 2 == 1).sum())
+    assert n > 50   # substitutes were exercised
+
+
+def test_select_invariants(orc):
+    rng = np.random.default_rng(6)
+    for trial in range(200):
+        E = int(rng.integers(2, 9)); M = int(rng.integers(1, 5)); k = int(rng.integers(1, min(E, 4) + 1))
+        cs = random_case(rng, E, M, k, 16, int(rng.integers(1, 4)))
+        (ch, sv, kd, loc, q), tab = run_oracle_select(orc, cs)
+        for t in range(16):
+            assert len(set(ch[t])) == k                                  # k distinct experts
+            for j in range(k):
+                r, kk, m = cs["idx"][t, j], ch[t, j], sv[t, j]
+                assert cs["x"][m, kk] == 1                               # c.6
+                if kk != r:                                              # c.7 / Eq. 7
+                    assert cs["group"][kk] == cs["group"][r]
+                    assert cs["sim"][r, kk] >= np.float32(cs["theta"])
+                assert (kd[t, j] & 1) == (kk != r)
+                assert (kd[t, j] >> 1) == (m != cs["loc"][t])
+            assert q[t] <= np.float32(cs["qbar"])                        # Property 2
+            assert loc[t] == sv[t, 0]
+
+
+def test_select_identity_when_every_expert_is_everywhere(orc):
+    rng = np.random.default_rng(7)
+    cs = random_case(rng, 6, 3, 2, 32, 2)
+    cs["x"] = np.ones((3, 6), np.uint8)
+    cs["qbar"] = 1.0; cs["theta"] = -1.0; cs["wT"] = 0.5
+    cs["F"], cs["B"], cs["tau"] = _params(rng, 3)      # testbed links: >= 0.2 ms per move
+    (ch, sv, kd, loc, q), _ = run_oracle_select(orc, cs)
+    np.testing.assert_array_equal(ch, cs["idx"])
+    assert (kd == 0).all() and (sv == cs["loc"][:, None]).all()
+    assert (q == cs["qhat"]).all()
+
+
+def test_select_no_budget_or_high_threshold_is_pure_exact(orc):
+    rng = np.random.default_rng(8)
+    for over in ({"qbar": 0.0}, {"theta": 1.5}):
+        cs = random_case(rng, 6, 3, 2, 32, 2)
+        cs["qhat"] = np.zeros(32, np.float32)
+        cs.update(over)
+        (ch, sv, kd, loc, q), _ = run_oracle_select(orc, cs)
+        np.testing.assert_array_equal(ch, cs["idx"])
+        assert (kd % 2 == 0).all()
+
+
+def test_select_ties_prefer_current_then_lower_server(orc):
+    E, M = 3, 3
+    sim = np.eye(E, dtype=np.float32)
+    x = np.zeros((M, E), np.uint8); x[1, 0] = x[2, 0] = 1; x[0, 1] = x[0, 2] = 1
+    F = np.ones(M) * 1e13; B = np.ones((M, M)) * 1e9; tau = np.ones((M, M)) * 1e-3
+    tab = orc.tables(sim, np.arange(E, dtype=np.int32), x, 0.5, 0.1, F, B, tau, 1.0, 1.0, 0.0, 0.5)
+    idx = np.array([[0], [0]], np.int32)          # omega_T = 0: every exact costs 0
+    ch, sv, kd, loc, q = orc.select(idx, tab, np.array([2, 0], np.uint8),
+                                    np.array([2, 0], np.uint8), np.zeros(2, np.float32))
+    assert list(sv[:, 0]) == [2, 1]               # stay on 2; else lowest server 1
+    assert list(kd[:, 0]) == [0, 2]
+
+
+def test_select_local_first_with_testbed_parameters(orc):
+    """With the testbed's ranges (Section VI-A) every remote move costs more
+    than any local candidate, so the choice is: keep the target if local, else
+    the most similar feasible local substitute, else a remote candidate."""
+    from paper_2607_17154_gb300 import synth
+    rng = np.random.default_rng(9)
+    E, M, k, d, dff = 8, 4, 2, 4096, 14336
+    sp = synth.server_params(M, d, dff, seed=3)
+    Wt = rng.standard_normal((E, 6)); Wt[:, 0] += 4 * (np.arange(E) // 4)
+    sim = (1 - cdist(Wt, Wt, "cosine")).astype(np.float32); np.fill_diagonal(sim, 1)
+    group = (np.arange(E) // 4).astype(np.int32)
+    x = np.zeros((M, E), np.uint8)
+    for e in range(E):
+        x[e % M, e] = 1
+    theta, qbar = 0.0, 0.4
+    tab = orc.tables(sim, group, x, theta, qbar, sp.F, sp.B, sp.tau, sp.z, sp.c, 0.5, 0.5)
+    T = 64
+    idx = np.array([rng.permutation(E)[:k] for _ in range(T)], np.int32)
+    home = rng.integers(0, M, T).astype(np.uint8)
+    ch, sv, kd, loc, q = orc.select(idx, tab, home, home.copy(), np.zeros(T, np.float32))
+    for t in range(T):
+        s = home[t]; used = set(idx[t]); qq = np.float32(0)
+        for j in range(k):
+            r = idx[t, j]
+            if x[s, r]:
+                assert ch[t, j] == r and sv[t, j] == s
+                continue
+            local = [kk for kk in range(E) if x[s, kk] and kk != r and group[kk] == group[r]
+                     and sim[r, kk] >= theta and kk not in used
+                     and np.float32(qq + tab.Qtab[r, kk]) <= np.float32(qbar)]
+            if local:
+                best = max(local, key=lambda kk: (sim[r, kk], -kk))
+                assert ch[t, j] == best and sv[t, j] == s
+                used.add(best); qq = np.float32(qq + tab.Qtab[r, best])
+            else:
+                # no local candidate: the token moves (to the target, or to a
+                # substitute on a server with a cheaper link)
+                assert sv[t, j] != s
+                if ch[t, j] != r:
+                    used.add(ch[t, j]); qq = np.float32(qq + tab.Qtab[r, ch[t, j]])
+
+
+# --------------------------------------------------------------------------
+# Permutation
+
+def test_dispatch_is_a_stable_counting_sort(orc):
+    rng = np.random.default_rng(10)
+    for T, k, E in [(1, 1, 1), (7, 2, 5), (100, 3, 8), (33, 6, 64)]:
+        chosen = rng.integers(0, E, (T, k)).astype(np.int32)
+        if E > 3:
+            chosen[chosen == 2] = 1       # an expert with no rows
+        off, row_token, row_of = orc.dispatch(chosen, E)
+        order = np.argsort(chosen.ravel(), kind="stable")
+        np.testing.assert_array_equal(row_token, order // k)
+        np.testing.assert_array_equal(off, np.concatenate([[0], np.cumsum(np.bincount(chosen.ravel(), minlength=E))]))
+        inv = np.empty(T * k, np.int64); inv[order] = np.arange(T * k)
+        np.testing.assert_array_equal(row_of.ravel(), inv)
+        assert sorted(row_of.ravel()) == list(range(T * k))      # bijection
+
+
+def test_gather_rows(orc):
+    rng = np.random.default_rng(11)
+    X = rnd_bf16(rng, (9, 16)); rt = rng.integers(0, 9, 20).astype(np.int32)
+    np.testing.assert_array_equal(orc.gather_rows(X, rt), X[rt])
+
+
+# --------------------------------------------------------------------------
+# SwiGLU FFN
+
+def test_ffn_one_hot_reduces_to_silu(orc):
+    """x = e_0, W1[:, 0] = a, W3[:, 0] = 1, W2 a selection matrix: the expert
+    output is bf16(silu(a)) routed through W2's selection, so the gate, the
+    up projection, their order and both matrix orientations are all pinned."""
+    rng = np.random.default_rng(12)
+    E, d, dff = 2, 6, 10
+    a = rng.standard_normal((E, dff)) * 3
+    W1 = np.zeros((E, dff, d)); W1[:, :, 0] = a
+    W1[:, :, 1:] = rng.standard_normal((E, dff, d - 1))   # never multiplied (x_c = 0)
+    W3 = np.zeros((E, dff, d)); W3[:, :, 0] = 1.0; W3[:, :, 2] = 5.0
+    W2 = np.zeros((E, d, dff))
+    perm = [rng.permutation(dff)[:d] for _ in range(E)]
+    for e in range(E):
+        W2[e, np.arange(d), perm[e]] = 1.0
+    X = np.zeros((4, d)); X[:, 0] = 1.0
+    rows_e = np.array([0, 1, 1, 0], np.int32)
+    W1b, W3b, W2b = bf16_bits(W1), bf16_bits(W3), bf16_bits(W2)
+    H, Y = orc.ffn_rows(bf16_bits(X), rows_e, W1b, W3b, W2b)
+    ab = bits_to_f(W1b)[:, :, 0].astype(np.float64)
+    silu = ab * scipy.special.expit(ab)
+    for r, e in enumerate(rows_e):
+        np.testing.assert_array_equal(H[r], bf16_bits(silu[e]))
+        np.testing.assert_array_equal(Y[r], H[r][perm[e]])
+
+
+def test_ffn_zero_input_and_power_of_two_scaling(orc):
+    rng = np.random.default_rng(13)
+    E, d, dff = 3, 8, 12
+    W1, W3, W2 = (rnd_bf16(rng, s, 0.5) for s in [(E, dff, d), (E, dff, d), (E, d, dff)])
+    X = rnd_bf16(rng, (5, d)); re = np.array([0, 1, 2, 2, 0], np.int32)
+    H0, Y0 = orc.ffn_rows(np.zeros_like(X), re, W1, W3, W2)
+    assert (H0 == 0).all() and (bits_to_f(Y0) == 0).all()
+    H, Y = orc.ffn_rows(X, re, W1, W3, W2)
+    H2, Y2 = orc.ffn_rows(X, re, W1, W3, bf16_bits(bits_to_f(W2) * 4.0))
+    np.testing.assert_array_equal(H2, H)
+    np.testing.assert_array_equal(bits_to_f(Y2), bits_to_f(Y) * 4.0)
+    # swapping the gate and up matrices changes the output (silu is not symmetric)
+    Hs, Ys = orc.ffn_rows(X, re, W3, W1, W2)
+    assert not np.array_equal(Hs, H)
+
+
+def test_ffn_row_uses_its_own_expert(orc):
+    rng = np.random.default_rng(14)
+    E, d, dff = 3, 8, 16
+    W1, W3, W2 = (rnd_bf16(rng, s, 0.5) for s in [(E, dff, d), (E, dff, d), (E, d, dff)])
+    X = rnd_bf16(rng, (1, d))
+    outs = [orc.ffn_rows(X, np.array([e], np.int32), W1, W3, W2)[1] for e in range(E)]
+    for e in range(E):
+        # the same row through expert e equals the row through a model whose
+        # only expert is e
+        solo = orc.ffn_rows(X, np.array([0], np.int32), W1[e:e + 1], W3[e:e + 1], W2[e:e + 1])[1]
+        np.testing.assert_array_equal(outs[e], solo)
+    assert not np.array_equal(outs[0], outs[1])
+
+
+# --------------------------------------------------------------------------
+# Combine
+
+def test_combine_special_cases(orc):
+    rng = np.random.default_rng(15)
+    T, d = 6, 10
+    Y = rnd_bf16(rng, (T, d))
+    rof = np.arange(T, dtype=np.int32)[:, None]
+    np.testing.assert_array_equal(orc.combine(Y, rof, np.ones((T, 1), np.float32)), Y)
+    # two slots, small-integer rows and dyadic weights: exact
+    Yi = bf16_bits(rng.integers(-8, 8, (2 * T, d)).astype(np.float32))
+    rof2 = np.stack([np.arange(T), T + (np.arange(T) + 1) % T], 1).astype(np.int32)
+    w = np.tile(np.array([0.75, 0.25], np.float32), (T, 1))
+    yf = bits_to_f(orc.combine(Yi, rof2, w))
+    Yf = bits_to_f(Yi)
+    np.testing.assert_array_equal(yf, 0.75 * Yf[rof2[:, 0]] + 0.25 * Yf[rof2[:, 1]])
+
+
+# --------------------------------------------------------------------------
+# Similarity (Eqs. 3-4) and activation counts (Eq. 5)
+
+def test_similarity_identity_calibration_is_cosine_of_router_rows(orc):
+    rng = np.random.default_rng(16)
+    E, d = 6, 12
+    W = rnd_bf16(rng, (E, d))
+    Wf = bits_to_f(W).astype(np.float64)
+    sim = orc.similarity(W, bf16_bits(np.eye(d)))
+    ref = 1 - cdist(Wf, Wf, "cosine")
+    np.fill_diagonal(ref, 1.0)
+    np.testing.assert_allclose(sim, ref, atol=1e-6)
+
+
+def test_similarity_diagonal_calibration_scales_feature_columns(orc):
+    rng = np.random.default_rng(17)
+    E, d = 5, 9
+    W = rnd_bf16(rng, (E, d)); s = np.array([1, 2, 0.5, 4, 1, 0.25, 8, 1, 2], np.float32)
+    sim = orc.similarity(W, bf16_bits(np.diag(s)))
+    Ws = bits_to_f(W).astype(np.float64) * s
+    ref = 1 - cdist(Ws, Ws, "cosine"); np.fill_diagonal(ref, 1.0)
+    np.testing.assert_allclose(sim, ref, atol=1e-6)
+
+
+def test_similarity_invariants(orc):
+    rng = np.random.default_rng(18)
+    E, d, N = 7, 16, 40
+    W = rnd_bf16(rng, (E, d)); Xc = rnd_bf16(rng, (N, d))
+    Wf = bits_to_f(W).copy()
+    Wf[3] = Wf[1]              # identical rows
+    Wf[5] = -2 * Wf[2]         # opposite direction
+    Wf[6] = 0                  # a dead expert
+    W = bf16_bits(Wf)
+    sim = orc.similarity(W, Xc)
+    np.testing.assert_array_equal(sim, sim.T)
+    assert (np.diag(sim) == 1).all() and (np.abs(sim) <= 1 + 1e-6).all()
+    assert sim[1, 3] == pytest.approx(1.0, abs=1e-6)
+    assert sim[2, 5] == pytest.approx(-1.0, abs=1e-6)
+    assert (sim[6, :6] == 0).all()
+    Ws = Wf.copy(); Ws[0] *= 4
+    np.testing.assert_allclose(orc.similarity(bf16_bits(Ws), Xc), sim, atol=1e-6)
+    # duplicating every calibration token leaves the cosine unchanged
+    np.testing.assert_allclose(orc.similarity(W, np.concatenate([Xc, Xc])), sim, atol=1e-6)
+
+
+def test_expert_counts_brute_force(orc):
+    rng = np.random.default_rng(19)
+    logits = rng.standard_normal((50, 6)).astype(np.float32)
+    logits[3] = 1.0
+    for kf in (1, 2, 6):
+        cnt = orc.expert_counts(logits, kf)
+        ref = np.zeros(6, np.int64)
+        for t in range(50):
+            for e in brute_topk(list(logits[t]), kf):
+                ref[e] += 1
+        np.testing.assert_array_equal(cnt, ref)
+        assert cnt.sum() == 50 * kf
+
+
+# --------------------------------------------------------------------------
+# Threshold, grouping, importance, placement (Eqs. 6, 24-31)
+
+def test_theta_endpoints_and_monotone(orc):
+    N = 24
+    th = [float(orc.theta(l, N, 0.5, 0.9, 0.7)) for l in range(1, N + 1)]
+    assert th[0] == pytest.approx(0.9) and th[-1] == pytest.approx(0.5)
+    assert all(a > b for a, b in zip(th, th[1:]))
+    assert float(orc.theta(1, 1, 0.5, 0.9, 0.7)) == pytest.approx(0.7)
+    assert th[11] == pytest.approx(0.5 + 0.4 * 12 / 23, abs=1e-7)
+
+
+def test_group_hand_example(orc):
+    # counts order: 2 (9), 0 (7), 4 (5), 1 (3), 3 (1)
+    sim = np.array([[1, .9, .2, .1, .3],
+                    [.9, 1, .1, .3, .6],
+                    [.2, .1, 1, .8, .1],
+                    [.1, .3, .8, 1, .4],
+                    [.3, .6, .1, .4, 1]], np.float32)
+    cnt = np.array([7, 3, 9, 1, 5], np.int32)
+    g, K, dom = orc.group(sim, cnt, 0.5)
+    # 2 -> new group 0; 0: sim to 2 is .2 < .5 -> group 1; 4: max(.1, .3) < .5 -> group 2;
+    # 1: sims .1 (2), .9 (0), .6 (4) -> joins 0's group 1; 3: .8 (2), .1, .4 -> group 0
+    assert K == 3 and list(dom) == [2, 0, 4]
+    assert list(g) == [1, 1, 0, 0, 2]
+    g2, K2, _ = orc.group(sim, cnt, -1.01)
+    assert K2 == 1 and (g2 == 0).all()
+    g3, K3, _ = orc.group(sim, cnt, 1.01)
+    assert K3 == 5 and sorted(g3) == list(range(5))
+
+
+def test_group_rule_holds_on_random_inputs(orc):
+    rng = np.random.default_rng(20)
+    for _ in range(100):
+        E = int(rng.integers(2, 12))
+        Wt = rng.standard_normal((E, 4))
+        sim = (1 - cdist(Wt, Wt, "cosine")).astype(np.float32); np.fill_diagonal(sim, 1)
+        cnt = rng.integers(0, 5, E).astype(np.int32)
+        th = float(rng.uniform(-0.5, 1.0))
+        g, K, dom = orc.group(sim, cnt, th)
+        order = sorted(range(E), key=lambda e: (-cnt[e], e))
+        made = []
+        for j in order:
+            if j in dom:
+                assert all(sim[j, c] < np.float32(th) for c in made)       # Eq. 24
+                assert g[j] == len(made); made.append(j)
+            else:
+                best = max(sim[j, c] for c in made)
+                assert best >= np.float32(th)
+                first = next(c for c in made if sim[j, c] == best)          # Eq. 25, tie: earliest
+                assert g[j] == made.index(first)
+
+
+def test_group_clustered_generator_recovers_clusters(orc):
+    from paper_2607_17154_gb300 import synth
+    E, d, K = 16, 256, 4
+    Wr = synth.router_weights(E, d, K, seed=5)
+    Xc = synth.calibration(2048, d, seed=5)
+    sim = orc.similarity(synth.bits(Wr), synth.bits(Xc))
+    cnt = np.ones(E, np.int32)
+    for th in (0.3, 0.5, 0.7, 0.9):
+        g, KK, _ = orc.group(sim, cnt, th)
+        assert KK == K
+        cl = synth.cluster_of(E, K)
+        for i in range(E):
+            for j in range(E):
+                assert (g[i] == g[j]) == (cl[i] == cl[j])
+
+
+def test_importance_closed_forms(orc):
+    sim = np.array([[1, .6, 0], [.6, 1, 0], [0, 0, 1]], np.float32)
+    group = np.array([0, 0, 1], np.int32)
+    cnt = np.array([2, 1, 1], np.int32)
+    I = orc.importance(sim, cnt, group, 0.5, 0.5)
+    np.testing.assert_allclose(I, [0.5 * 0.5 + 0.5 * 0.8, 0.5 * 0.25 + 0.5 * 0.8, 0.5 * 0.25 + 0.5],
+                               rtol=1e-7)
+
+
+def test_place_hand_example_disperses_groups(orc):
+    # 4 experts in 2 groups, 2 servers with room for 2 each
+    group = np.array([[0, 0, 1, 1]], np.int32)
+    I = np.array([[0.9, 0.8, 0.7, 0.6]])
+    p = np.ones((1, 4)); C = np.array([2.0, 2.0])
+    x, used, rc = orc.place(group, I, p, C)
+    assert rc == 0
+    # 0 -> server 0 (tie, lower m); 1 -> server 1 (eta); 2 -> server 0 (b/C tie -> eta 0 both, lower);
+    # 3 -> server 1 (server 0 full)
+    np.testing.assert_array_equal(x[0], [[1, 0, 1, 0], [0, 1, 0, 1]])
+    np.testing.assert_array_equal(used, [2, 2])
+
+
+def test_place_waiting_list_and_capacity(orc):
+    group = np.array([[0, 1, 2]], np.int32)
+    I = np.array([[0.5, 0.5, 0.5]])
+    p = np.array([[2.0, 2.0, 3.0]]); C = np.array([3.0, 4.0])
+    x, used, rc = orc.place(group, I, p, C)
+    # order by p desc: 2 (3) -> score 0 both -> server 0; 0 (2): feasible {1} -> 1;
+    # 1 (2): feasible {1}? b1 = 2, 2+2 <= 4 yes -> 1
+    np.testing.assert_array_equal(x[0], [[0, 0, 1], [1, 1, 0]])
+    assert rc == 0
+    p2 = np.array([[2.0, 2.0, 2.0]]); C2 = np.array([3.0, 3.0])
+    x2, used2, rc2 = orc.place(group, I, p2, C2)
+    assert x2[0].sum(axis=0).tolist() == [1, 1, 1]          # c.2 still met
+    assert rc2 == orc.CAPACITY                               # sum C < sum p
+
+
+def test_place_invariants_over_layers(orc):
+    rng = np.random.default_rng(21)
+    for _ in range(50):
+        L, E, M = int(rng.integers(1, 5)), int(rng.integers(2, 10)), int(rng.integers(1, 6))
+        group = rng.integers(0, 3, (L, E)).astype(np.int32)
+        I = rng.random((L, E)); p = rng.integers(1, 4, (L, E)).astype(np.float64)
+        C = np.full(M, p.sum() / M * 1.5)
+        x, used, rc = orc.place(group, I, p, C)
+        assert (x.sum(axis=1) == 1).all()                                   # c.2, one copy
+        load = np.einsum("lme,le->m", x.astype(np.float64), p)
+        np.testing.assert_allclose(load, used)
+        if rc == 0:
+            assert (load <= C + 1e-9).all()                                 # c.1
+        else:   # only the waiting list may overflow a server
+            assert rc == orc.CAPACITY and (load > C).any()
+
+
+def test_coverage(orc):
+    x = np.array([[1, 0, 1, 0], [0, 1, 0, 0]], np.uint8)
+    g = np.array([0, 0, 1, 1], np.int32)
+    np.testing.assert_array_equal(orc.coverage(x, g, 2), [[1, 1], [1, 0]])
