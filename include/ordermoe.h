@@ -1,0 +1,198 @@
+/*
+ * ordermoe.h - C ABI of the GB300 (sm_103a) OrderMoE hot-path library.
+ *
+ * The library computes one MoE layer forward with similarity-aware expert
+ * substitution, after "OrderMoE: an expert similarity driven distributed edge
+ * MoE inference" (arXiv 2607.17154), plus the offline similarity, grouping and
+ * placement that feed it. Edge servers are a logical expert-to-server
+ * placement map on one GPU: no data moves between servers.
+ *
+ * Conventions for every call below:
+ *  - Pointers are DEVICE pointers owned by the caller unless a parameter says
+ *    "host". The library keeps no pointer after a call returns.
+ *  - bf16 tensors are passed as uint16_t bit patterns, row-major, dense.
+ *  - Every call only enqueues work on `stream` (NULL = the legacy default
+ *    stream) and returns; nothing is synchronised and nothing is read back to
+ *    the host, except where a call says so.
+ *  - Return value: ORDERMOE_OK, or an error code; ordermoe_last_error() then
+ *    gives a message (thread-local). Argument errors are detected on the host
+ *    before anything is enqueued. Errors found by a kernel (an index out of
+ *    range, a NaN logit, a bounded wait that ran out) set a device error word
+ *    that ordermoe_device_error() reads.
+ *  - Limits: E <= 64 experts, M <= 32 servers, k <= 8 slots per token.
+ */
+#ifndef ORDERMOE_H
+#define ORDERMOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t / CUstream. */
+typedef struct CUstream_st* ordermoe_stream_t;
+
+enum {
+  ORDERMOE_OK = 0,
+  ORDERMOE_ERR_INVALID_ARG = 1,       /* null pointer, bad size, bad alignment  */
+  ORDERMOE_ERR_UNSUPPORTED_SHAPE = 2, /* outside the limits stated per call      */
+  ORDERMOE_ERR_CAPACITY = 3,          /* placement: sum C_m < sum p, or overflow */
+  ORDERMOE_ERR_CUDA = 4,              /* a CUDA runtime/driver call failed       */
+  ORDERMOE_ERR_DEVICE_CHECK = 5       /* a kernel reported an error (see below)  */
+};
+
+/* Device error word values (ordermoe_device_error). */
+enum {
+  ORDERMOE_DEV_OK = 0,
+  ORDERMOE_DEV_NAN_LOGIT = 1,     /* route_select: a logit was NaN             */
+  ORDERMOE_DEV_BAD_INDEX = 2,     /* an expert/server index out of range       */
+  ORDERMOE_DEV_NO_CANDIDATE = 3,  /* selection: target expert placed nowhere   */
+  ORDERMOE_DEV_WAIT_TIMEOUT = 4   /* a bounded pipeline wait ran out           */
+};
+
+#define ORDERMOE_MAX_EXPERTS 64
+#define ORDERMOE_MAX_SERVERS 32
+#define ORDERMOE_MAX_TOPK 8
+
+/* Message for the last error returned on this host thread. */
+const char* ordermoe_last_error(void);
+
+/* Library version, major * 10000 + minor * 100 + patch. */
+int ordermoe_version(void);
+
+/* Reads and clears the device error word of the current device. This call
+ * synchronises the device. *code (host) receives an ORDERMOE_DEV_* value and
+ * *detail (host, nullable) a kernel-specific detail (e.g. the token index).
+ * Returns ORDERMOE_ERR_DEVICE_CHECK when *code != 0, else ORDERMOE_OK. */
+int ordermoe_device_error(int* code, int* detail);
+
+/* Sets the limit, in nanoseconds, of every bounded device-side wait in kernels
+ * launched afterwards on this host thread (default 2e9 = 2 s). A wait that runs
+ * out sets ORDERMOE_DEV_WAIT_TIMEOUT and the kernel returns early. */
+int ordermoe_set_wait_limit_ns(uint64_t limit_ns);
+
+/* Launches one kernel whose single bounded wait is on an mbarrier that nothing
+ * arrives at, so that the wait runs out after `limit_ns`. Used to test that
+ * bounded waits end and report ORDERMOE_DEV_WAIT_TIMEOUT. */
+int ordermoe_selftest_wait_timeout(uint64_t limit_ns, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Per-layer selection tables.
+ *
+ * A device buffer of ordermoe_tables_bytes(E, M) bytes, written by
+ * ordermoe_build_tables and read by ordermoe_route_select. Layout (byte
+ * offsets; all little-endian):
+ *     0  int32  magic 0x4f4d5442, E, M, reserved
+ *    16  float  theta, qbar
+ *    64  uint32 pmask[64]   bit m set <=> x_{m,e} = 1          (placement)
+ *   320  uint64 subst[64]   bit k set <=> e_k in R_{l,e} (Eq. 7)
+ *   832  float  Qtab[E][E]  Q_l(r,k) of Eq. 18, phi = identity
+ *        float  Cq[E][E]    omega_Q Q_l(r,k) / Qbar (quality term of Eq. 38)
+ *        float  A[M][M][M]  A[a][s][m] = omega_T d(s,m) / d_ref(a) (delay term
+ *                           of Eq. 38; d of Eq. 37; d_ref(a) = c / F_a)
+ * ------------------------------------------------------------------------ */
+size_t ordermoe_tables_bytes(int E, int M);
+
+/* Builds the selection tables of one layer (Sections III-B, III-D, III-E and
+ * V-A: Eqs. 7, 18, 37, 38).
+ *   sim        [E][E] f32   expert similarity Sim_l (Eq. 4)
+ *   group      [E] i32      similarity group of each expert (Eq. 26)
+ *   placement  [M][E] u8    x_{m,l,e} (1 = expert e deployed on server m)
+ *   theta      similarity threshold theta_l of the layer (Eq. 6 / Eq. 7)
+ *   qbar       per-token quality budget Qbar (Eq. 39), >= 0
+ *   F [M], B [M][M], tau [M][M]  f64: server compute (flop/s), link bandwidth
+ *              (bytes/s) and latency (s); the diagonals are not read
+ *   z          bytes moved when a token changes server (z_l of Eq. 37)
+ *   c          flop of one expert on one token (c_l of Eq. 15)
+ *   omega_T, omega_Q  cost weights of Eq. 38
+ *   tables     out, device buffer of tables_bytes >= ordermoe_tables_bytes(E,M)
+ * fp64 terms are computed with correctly rounded IEEE operations (no fused
+ * multiply-add) and rounded once to fp32. */
+int ordermoe_build_tables(const float* sim, const int32_t* group, const uint8_t* placement,
+                          int E, int M, float theta, float qbar, const double* F, const double* B,
+                          const double* tau, double z, double c, double omega_T, double omega_Q,
+                          void* tables, size_t tables_bytes, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Router + softmax + top-k + server-expert selection (Alg. 2 with horizon
+ * H = 1, Section V; the router output is the "target expert from the local
+ * router" of Alg. 2).
+ *   X          [T][d] bf16  token representations (ignored if logits_in)
+ *   W_r        [E][d] bf16  router weights (ignored if logits_in)
+ *   logits_in  [T][E] f32, nullable: when given, the router GEMM is skipped
+ *              and these logits are used
+ *   renorm     1: top-k gate weights renormalised to sum to 1 over the k slots
+ *   tables     the layer's tables (ordermoe_build_tables)
+ *   home       [T] u8   home (access) server a(i) of each token
+ *   loc        [T] u8   in/out: server holding the token before / after the
+ *              layer (Eq. 36, Eq. 44); set loc = home before the first layer
+ *   qhat       [T] f32  in/out: accumulated quality loss (Eq. 44); 0 at start
+ *   logits_out [T][E] f32, nullable: the router logits
+ *   topk_idx   [T][k] i32  routed (target) experts, rank order
+ *   topk_w     [T][k] f32  gate weights of the routed slots
+ *   chosen_expert [T][k] i32  executed expert k* per slot (Eq. 43)
+ *   chosen_server [T][k] u8   executing server m* per slot
+ *   kind       [T][k] u8   0 local exact, 1 local substitute, 2 remote exact,
+ *              3 remote substitute (Section VI-C's execution types)
+ *   counters   [4] i32, nullable: += number of slots of each kind
+ * Readings of the paper: with k > 1 the selection runs per slot in rank
+ * order; a substitute is never one of the token's routed experts nor a
+ * substitute already given to it; the token's new location is the server of
+ * slot 0; ties in Eq. 43 go to lower cost, exact, current server, lower
+ * server, lower expert. Shapes: 1 <= E <= 64, 1 <= k <= min(E, 8),
+ * d % 8 == 0 (X and W_r 16-byte aligned) unless logits_in is given. */
+int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, const float* logits_in, int T,
+                          int E, int d, int k, int renorm, const void* tables, size_t tables_bytes,
+                          const uint8_t* home, uint8_t* loc, float* qhat, float* logits_out,
+                          int32_t* topk_idx, float* topk_w, int32_t* chosen_expert,
+                          uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
+                          ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Token permutation: histogram + prefix sum + stable scatter of the T*k
+ * (token, slot) entries by executed expert, and the row gather of X into
+ * expert-contiguous order (the grouped layout the expert FFN consumes).
+ *   chosen_expert [T][k] i32 (0 <= e < E)
+ *   X          [T][d] bf16
+ *   offsets    [E+1] i32 out: rows of expert e are offsets[e] .. offsets[e+1]-1
+ *   row_token  [T*k] i32 out: token of each permuted row
+ *   row_of     [T][k] i32 out: permuted row of each (token, slot)
+ *   X_perm     [T*k][d] bf16 out: X_perm[row] = X[row_token[row]]
+ *   workspace  device scratch of ordermoe_dispatch_workspace_bytes(T,k,E) bytes
+ * Within one expert, rows keep the flat (t*k + j) order: the result is
+ * unique. d % 8 == 0 and 16-byte aligned X / X_perm. */
+size_t ordermoe_dispatch_workspace_bytes(int T, int k, int E);
+int ordermoe_dispatch(const int32_t* chosen_expert, const uint16_t* X, int T, int k, int E, int d,
+                      int32_t* offsets, int32_t* row_token, int32_t* row_of, uint16_t* X_perm,
+                      void* workspace, size_t workspace_bytes, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Grouped SwiGLU expert FFN over the permuted rows (the Mixtral-style experts
+ * of Section VI-A):
+ *   H[row] = bf16( silu(x W1_e^T) * (x W3_e^T) ),  Y_perm[row] = bf16( H[row] W2_e^T )
+ * for every row of expert e (offsets from ordermoe_dispatch, read on the
+ * device: no host synchronisation). fp32 accumulation on tcgen05 tensor cores.
+ *   X_perm [R][d] bf16, offsets [E+1] i32 (offsets[E] == R)
+ *   W1, W3 [E][dff][d] bf16;  W2 [E][d][dff] bf16
+ *   H      [R][dff] bf16 out (the SwiGLU activations; caller-owned scratch)
+ *   Y_perm [R][d] bf16 out
+ * Shapes: d % 256 == 0, dff % 128 == 0, all pointers 16-byte aligned. */
+int ordermoe_expert_ffn(const uint16_t* X_perm, const int32_t* offsets, int R, const uint16_t* W1,
+                        const uint16_t* W3, const uint16_t* W2, int E, int d, int dff, uint16_t* H,
+                        uint16_t* Y_perm, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Weighted combine: y[t] = bf16( sum_{j=0..k-1} topk_w[t][j] * Y_perm[row_of[t][j]] )
+ * with fp32 accumulation in slot order.
+ *   Y_perm [T*k][d] bf16, row_of [T][k] i32, topk_w [T][k] f32, y [T][d] bf16 out.
+ * d % 8 == 0, 16-byte aligned Y_perm / y. */
+int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of, const float* topk_w, int T,
+                     int k, int d, uint16_t* y, ordermoe_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ORDERMOE_H */

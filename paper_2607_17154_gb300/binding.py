@@ -1,0 +1,180 @@
+"""ctypes binding of libordermoe.so: one Python function per C-ABI entry point,
+with the same names. Arguments are torch tensors on the current CUDA device;
+the binding only checks dtypes/devices and passes pointers, sizes and the
+current stream. Every step of the path runs in the library's kernels; there
+is no fallback: if the library is missing the call raises.
+"""
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libordermoe.so")
+
+OK = 0
+ERR_INVALID_ARG, ERR_UNSUPPORTED_SHAPE, ERR_CAPACITY, ERR_CUDA, ERR_DEVICE_CHECK = 1, 2, 3, 4, 5
+DEV_OK, DEV_NAN_LOGIT, DEV_BAD_INDEX, DEV_NO_CANDIDATE, DEV_WAIT_TIMEOUT = 0, 1, 2, 3, 4
+
+_lib = None
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_F = ctypes.c_float
+_D = ctypes.c_double
+_SZ = ctypes.c_size_t
+_U64 = ctypes.c_uint64
+_I64 = ctypes.c_int64
+
+_SIGNATURES = {
+    "ordermoe_version": ([], _I),
+    "ordermoe_last_error": ([], ctypes.c_char_p),
+    "ordermoe_device_error": ([_P, _P], _I),
+    "ordermoe_set_wait_limit_ns": ([_U64], _I),
+    "ordermoe_selftest_wait_timeout": ([_U64, _P], _I),
+    "ordermoe_tables_bytes": ([_I, _I], _SZ),
+    "ordermoe_build_tables": ([_P, _P, _P, _I, _I, _F, _F, _P, _P, _P, _D, _D, _D, _D, _P, _SZ, _P], _I),
+    "ordermoe_route_select": ([_P, _P, _P, _I, _I, _I, _I, _I, _P, _SZ, _P, _P, _P, _P, _P, _P, _P,
+                               _P, _P, _P, _P], _I),
+    "ordermoe_dispatch_workspace_bytes": ([_I, _I, _I], _SZ),
+    "ordermoe_dispatch": ([_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "ordermoe_expert_ffn": ([_P, _P, _I, _P, _P, _P, _I, _I, _I, _P, _P, _P], _I),
+    "ordermoe_combine": ([_P, _P, _P, _I, _I, _I, _P, _P], _I),
+}
+
+
+class OrderMoEError(RuntimeError):
+    def __init__(self, name, code, msg):
+        super().__init__("%s failed with status %d: %s" % (name, code, msg))
+        self.code = code
+
+
+def lib():
+    """Load libordermoe.so (built in-tree by build.py / __graft_entry__.build())."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libordermoe.so is not built (%s); run __graft_entry__.build()"
+                               % LIB_PATH)
+        L = ctypes.CDLL(LIB_PATH)
+        for name, (args, res) in _SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = L
+    return _lib
+
+
+def _check(name, rc):
+    if rc != OK:
+        msg = lib().ordermoe_last_error()
+        raise OrderMoEError(name, rc, msg.decode() if msg else "")
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch.Tensor")
+    if not t.is_cuda:
+        raise ValueError("tensor must be on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError("tensor must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _dt(t, dtype, name):
+    if t is not None and t.dtype != dtype:
+        raise TypeError("%s must be %s, got %s" % (name, dtype, t.dtype))
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+# ------------------------------------------------------------------ entry points
+
+def ordermoe_version():
+    return lib().ordermoe_version()
+
+
+def ordermoe_device_error():
+    """Synchronises; returns (code, detail) of the device error word and clears it."""
+    code = ctypes.c_int(0); detail = ctypes.c_int(0)
+    lib().ordermoe_device_error(ctypes.byref(code), ctypes.byref(detail))
+    return code.value, detail.value
+
+
+def ordermoe_set_wait_limit_ns(limit_ns):
+    _check("ordermoe_set_wait_limit_ns", lib().ordermoe_set_wait_limit_ns(int(limit_ns)))
+
+
+def ordermoe_selftest_wait_timeout(limit_ns, stream=None):
+    _check("ordermoe_selftest_wait_timeout",
+           lib().ordermoe_selftest_wait_timeout(int(limit_ns), _stream(stream)))
+
+
+def ordermoe_tables_bytes(E, M):
+    return int(lib().ordermoe_tables_bytes(E, M))
+
+
+def ordermoe_build_tables(sim, group, placement, theta, qbar, F, B, tau, z, c, omega_T, omega_Q,
+                          tables, stream=None):
+    _dt(sim, torch.float32, "sim"); _dt(group, torch.int32, "group")
+    _dt(placement, torch.uint8, "placement"); _dt(tables, torch.uint8, "tables")
+    for n, t in (("F", F), ("B", B), ("tau", tau)):
+        _dt(t, torch.float64, n)
+    E = sim.shape[0]; M = placement.shape[0]
+    rc = lib().ordermoe_build_tables(_ptr(sim), _ptr(group), _ptr(placement), E, M, float(theta),
+                                     float(qbar), _ptr(F), _ptr(B), _ptr(tau), float(z), float(c),
+                                     float(omega_T), float(omega_Q), _ptr(tables), tables.numel(),
+                                     _stream(stream))
+    _check("ordermoe_build_tables", rc)
+
+
+def ordermoe_route_select(X, W_r, logits_in, T, E, d, k, renorm, tables, home, loc, qhat,
+                          logits_out, topk_idx, topk_w, chosen_expert, chosen_server, kind,
+                          counters=None, stream=None):
+    _dt(X, torch.bfloat16, "X"); _dt(W_r, torch.bfloat16, "W_r"); _dt(logits_in, torch.float32, "logits_in")
+    _dt(home, torch.uint8, "home"); _dt(loc, torch.uint8, "loc"); _dt(qhat, torch.float32, "qhat")
+    _dt(topk_idx, torch.int32, "topk_idx"); _dt(topk_w, torch.float32, "topk_w")
+    _dt(chosen_expert, torch.int32, "chosen_expert"); _dt(chosen_server, torch.uint8, "chosen_server")
+    _dt(kind, torch.uint8, "kind"); _dt(counters, torch.int32, "counters")
+    rc = lib().ordermoe_route_select(_ptr(X), _ptr(W_r), _ptr(logits_in), T, E, d, k, int(renorm),
+                                     _ptr(tables), tables.numel(), _ptr(home), _ptr(loc), _ptr(qhat),
+                                     _ptr(logits_out), _ptr(topk_idx), _ptr(topk_w),
+                                     _ptr(chosen_expert), _ptr(chosen_server), _ptr(kind),
+                                     _ptr(counters), _stream(stream))
+    _check("ordermoe_route_select", rc)
+
+
+def ordermoe_dispatch_workspace_bytes(T, k, E):
+    return int(lib().ordermoe_dispatch_workspace_bytes(T, k, E))
+
+
+def ordermoe_dispatch(chosen_expert, X, T, k, E, d, offsets, row_token, row_of, X_perm, workspace,
+                      stream=None):
+    _dt(chosen_expert, torch.int32, "chosen_expert"); _dt(X, torch.bfloat16, "X")
+    _dt(offsets, torch.int32, "offsets"); _dt(row_token, torch.int32, "row_token")
+    _dt(row_of, torch.int32, "row_of"); _dt(X_perm, torch.bfloat16, "X_perm")
+    rc = lib().ordermoe_dispatch(_ptr(chosen_expert), _ptr(X), T, k, E, d, _ptr(offsets),
+                                 _ptr(row_token), _ptr(row_of), _ptr(X_perm), _ptr(workspace),
+                                 workspace.numel() * workspace.element_size(), _stream(stream))
+    _check("ordermoe_dispatch", rc)
+
+
+def ordermoe_expert_ffn(X_perm, offsets, R, W1, W3, W2, E, d, dff, H, Y_perm, stream=None):
+    for n, t in (("X_perm", X_perm), ("W1", W1), ("W3", W3), ("W2", W2), ("H", H), ("Y_perm", Y_perm)):
+        _dt(t, torch.bfloat16, n)
+    _dt(offsets, torch.int32, "offsets")
+    rc = lib().ordermoe_expert_ffn(_ptr(X_perm), _ptr(offsets), R, _ptr(W1), _ptr(W3), _ptr(W2),
+                                   E, d, dff, _ptr(H), _ptr(Y_perm), _stream(stream))
+    _check("ordermoe_expert_ffn", rc)
+
+
+def ordermoe_combine(Y_perm, row_of, topk_w, T, k, d, y, stream=None):
+    _dt(Y_perm, torch.bfloat16, "Y_perm"); _dt(row_of, torch.int32, "row_of")
+    _dt(topk_w, torch.float32, "topk_w"); _dt(y, torch.bfloat16, "y")
+    rc = lib().ordermoe_combine(_ptr(Y_perm), _ptr(row_of), _ptr(topk_w), T, k, d, _ptr(y),
+                                _stream(stream))
+    _check("ordermoe_combine", rc)

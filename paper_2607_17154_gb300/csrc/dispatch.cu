@@ -1,0 +1,217 @@
+// Token permutation (histogram, prefix sum, stable scatter + row gather) and
+// the weighted combine.
+//
+// The (token, slot) entries i = t*k + j are cut into chunks of kChunk = 256
+// consecutive entries, one block each:
+//   1. chunk_hist: per-chunk expert histogram -> hist[chunk][E]
+//   2. chunk_scan: one block; for every expert the exclusive prefix of its
+//      count over chunks, plus the expert offsets (exclusive prefix over
+//      experts) -> base[chunk][e] = offsets[e] + entries of e in earlier chunks
+//   3. rank_gather: stable rank inside the chunk (per-warp match + per-warp
+//      counts), row = base + rank; then each warp copies its 32 rows of X into
+//      X_perm with 16-byte loads and stores.
+// Rows of one expert therefore keep the flat entry order: the permutation
+// is unique and deterministic.
+#include "common.cuh"
+
+namespace om {
+
+static __device__ unsigned long long g_err_dispatch = 0;
+
+int read_clear_err_dispatch(unsigned long long* out) {
+  unsigned long long zero = 0;
+  OM_CUDA(cudaMemcpyFromSymbol(out, g_err_dispatch, sizeof(*out)));
+  OM_CUDA(cudaMemcpyToSymbol(g_err_dispatch, &zero, sizeof(zero)));
+  return ORDERMOE_OK;
+}
+
+constexpr int kChunk = 256;
+
+__global__ void __launch_bounds__(kChunk) chunk_hist_kernel(const int32_t* __restrict__ chosen,
+                                                            int64_t n, int E,
+                                                            int32_t* __restrict__ hist) {
+  __shared__ int h[64];
+  if (threadIdx.x < 64) h[threadIdx.x] = 0;
+  __syncthreads();
+  const int64_t i = (int64_t)blockIdx.x * kChunk + threadIdx.x;
+  if (i < n) {
+    const int e = chosen[i];
+    if (e >= 0 && e < E) atomicAdd(&h[e], 1);
+    else report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, static_cast<int>(i));
+  }
+  __syncthreads();
+  if (threadIdx.x < E) hist[(size_t)blockIdx.x * E + threadIdx.x] = h[threadIdx.x];
+}
+
+// One block of 64 threads: thread e walks the chunks of expert e.
+__global__ void chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks, int E,
+                                  int32_t* __restrict__ offsets) {
+  __shared__ int total[64];
+  __shared__ int start[65];
+  const int e = threadIdx.x;
+  int run = 0;
+  if (e < E) {
+    for (int b = 0; b < nchunks; ++b) {
+      const int v = hist[(size_t)b * E + e];
+      hist[(size_t)b * E + e] = run;
+      run += v;
+    }
+    total[e] = run;
+  }
+  __syncthreads();
+  if (e == 0) {
+    int s = 0;
+    for (int x = 0; x < E; ++x) {
+      start[x] = s;
+      s += total[x];
+    }
+    start[E] = s;
+  }
+  __syncthreads();
+  if (e <= E) offsets[e] = start[e];
+  if (e < E)
+    for (int b = 0; b < nchunks; ++b) hist[(size_t)b * E + e] += start[e];
+}
+
+__global__ void __launch_bounds__(kChunk) rank_gather_kernel(
+    const int32_t* __restrict__ chosen, int64_t n, int k, int E, int d,
+    const int32_t* __restrict__ base, const uint16_t* __restrict__ X, int32_t* __restrict__ row_token,
+    int32_t* __restrict__ row_of, uint16_t* __restrict__ X_perm) {
+  constexpr int kWarps = kChunk / 32;
+  __shared__ int cnt[kWarps][64];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int i = threadIdx.x; i < kWarps * 64; i += kChunk) (&cnt[0][0])[i] = 0;
+  __syncthreads();
+  const int64_t i = (int64_t)blockIdx.x * kChunk + threadIdx.x;
+  const bool live = i < n;
+  int e = live ? chosen[i] : -1;
+  if (e >= E || e < -1) e = -1;  // reported by chunk_hist_kernel
+  const unsigned peers = __match_any_sync(0xffffffffu, e);
+  const int rank_in_warp = __popc(peers & ((1u << lane) - 1u));
+  if (e >= 0 && rank_in_warp == 0) cnt[warp][e] = __popc(peers);
+  __syncthreads();
+  int row = -1;
+  if (e >= 0) {
+    int before = 0;
+    for (int w = 0; w < warp; ++w) before += cnt[w][e];
+    row = base[(size_t)blockIdx.x * E + e] + before + rank_in_warp;
+    row_of[i] = row;
+    row_token[row] = static_cast<int32_t>(i / k);
+  }
+  // each warp copies the rows of its 32 entries
+  const int nvec = d >> 3;  // 16-byte vectors per row
+  for (int src = 0; src < 32; ++src) {
+    const int r = __shfl_sync(0xffffffffu, row, src);
+    if (r < 0) continue;
+    const int64_t ii = (int64_t)blockIdx.x * kChunk + warp * 32 + src;
+    const int64_t t = ii / k;
+    const uint4* in = reinterpret_cast<const uint4*>(X + t * d);
+    uint4* out = reinterpret_cast<uint4*>(X_perm + (int64_t)r * d);
+    for (int v = lane; v < nvec; v += 32) out[v] = __ldg(in + v);
+  }
+}
+
+// One warp per token; lane l handles the 16-byte vectors l, l + 32, ...
+__global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict__ Yp,
+                                                      const int32_t* __restrict__ row_of,
+                                                      const float* __restrict__ w, int T, int k,
+                                                      int d, uint16_t* __restrict__ y) {
+  const int lane = threadIdx.x & 31;
+  const int warps_total = gridDim.x * (blockDim.x >> 5);
+  const int nvec = d >> 3;
+  for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < T; t += warps_total) {
+    int rows[ORDERMOE_MAX_TOPK];
+    float ws[ORDERMOE_MAX_TOPK];
+    for (int j = 0; j < k; ++j) {
+      rows[j] = row_of[(size_t)t * k + j];
+      ws[j] = w[(size_t)t * k + j];
+    }
+    for (int v = lane; v < nvec; v += 32) {
+      float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+      for (int j = 0; j < k; ++j) {
+        const uint4 yv = __ldg(reinterpret_cast<const uint4*>(Yp + (size_t)rows[j] * d) + v);
+        const float wj = ws[j];
+        acc[0] = fmaf(wj, bf16_lo(yv.x), acc[0]); acc[1] = fmaf(wj, bf16_hi(yv.x), acc[1]);
+        acc[2] = fmaf(wj, bf16_lo(yv.y), acc[2]); acc[3] = fmaf(wj, bf16_hi(yv.y), acc[3]);
+        acc[4] = fmaf(wj, bf16_lo(yv.z), acc[4]); acc[5] = fmaf(wj, bf16_hi(yv.z), acc[5]);
+        acc[6] = fmaf(wj, bf16_lo(yv.w), acc[6]); acc[7] = fmaf(wj, bf16_hi(yv.w), acc[7]);
+      }
+      uint4 o;
+      o.x = pack_bf16x2(acc[0], acc[1]); o.y = pack_bf16x2(acc[2], acc[3]);
+      o.z = pack_bf16x2(acc[4], acc[5]); o.w = pack_bf16x2(acc[6], acc[7]);
+      reinterpret_cast<uint4*>(y + (size_t)t * d)[v] = o;
+    }
+  }
+}
+
+size_t dispatch_workspace_bytes(int64_t n, int E) {
+  const int64_t nchunks = (n + kChunk - 1) / kChunk;
+  return (size_t)((nchunks > 0 ? nchunks : 1) * E * sizeof(int32_t) + 255) & ~size_t(255);
+}
+
+int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int E, int d,
+                    int32_t* offsets, int32_t* row_token, int32_t* row_of, uint16_t* X_perm,
+                    int32_t* hist, cudaStream_t stream) {
+  const int64_t n = (int64_t)T * k;
+  const int nchunks = static_cast<int>((n + kChunk - 1) / kChunk);
+  if (n == 0) {
+    OM_CUDA(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), stream));
+    return ORDERMOE_OK;
+  }
+  chunk_hist_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, E, hist);
+  OM_LAUNCHED("chunk_hist_kernel");
+  chunk_scan_kernel<<<1, 96, 0, stream>>>(hist, nchunks, E, offsets);
+  OM_LAUNCHED("chunk_scan_kernel");
+  rank_gather_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, d, hist, X, row_token,
+                                                     row_of, X_perm);
+  OM_LAUNCHED("rank_gather_kernel");
+  return ORDERMOE_OK;
+}
+
+}  // namespace om
+
+using namespace om;
+
+extern "C" size_t ordermoe_dispatch_workspace_bytes(int T, int k, int E) {
+  if (T < 0 || k <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS) return 0;
+  return om::dispatch_workspace_bytes((int64_t)T * k, E);
+}
+
+extern "C" int ordermoe_dispatch(const int32_t* chosen_expert, const uint16_t* X, int T, int k,
+                                 int E, int d, int32_t* offsets, int32_t* row_token,
+                                 int32_t* row_of, uint16_t* X_perm, void* workspace,
+                                 size_t workspace_bytes, ordermoe_stream_t stream) {
+  if (T < 0 || k <= 0 || k > ORDERMOE_MAX_TOPK || E <= 0 || E > ORDERMOE_MAX_EXPERTS)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "dispatch: need T >= 0, 1 <= k <= 8, 1 <= E <= 64");
+  if (d <= 0 || d % 8 != 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "dispatch: d must be a positive multiple of 8");
+  if (!offsets) return fail(ORDERMOE_ERR_INVALID_ARG, "dispatch: null offsets");
+  if (T > 0 && (!chosen_expert || !X || !row_token || !row_of || !X_perm || !workspace))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "dispatch: null pointer");
+  if ((int64_t)T * k > INT32_MAX) return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "dispatch: T*k too large");
+  if (T > 0 && (!aligned16(X) || !aligned16(X_perm)))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "dispatch: X and X_perm must be 16-byte aligned");
+  if (workspace_bytes < om::dispatch_workspace_bytes((int64_t)T * k, E))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "dispatch: workspace too small");
+  return dispatch_launch(chosen_expert, X, T, k, E, d, offsets, row_token, row_of, X_perm,
+                         static_cast<int32_t*>(workspace), stream);
+}
+
+extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,
+                                const float* topk_w, int T, int k, int d, uint16_t* y,
+                                ordermoe_stream_t stream) {
+  if (T < 0 || k <= 0 || k > ORDERMOE_MAX_TOPK)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "combine: need T >= 0, 1 <= k <= 8");
+  if (d <= 0 || d % 8 != 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "combine: d must be a positive multiple of 8");
+  if (T == 0) return ORDERMOE_OK;
+  if (!Y_perm || !row_of || !topk_w || !y) return fail(ORDERMOE_ERR_INVALID_ARG, "combine: null pointer");
+  if (!aligned16(Y_perm) || !aligned16(y))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "combine: Y_perm and y must be 16-byte aligned");
+  int blocks = (T + 7) / 8;
+  const int cap = num_sms() * 8;
+  if (blocks > cap) blocks = cap;
+  combine_kernel<<<blocks, 256, 0, stream>>>(Y_perm, row_of, topk_w, T, k, d, y);
+  OM_LAUNCHED("combine_kernel");
+  return ORDERMOE_OK;
+}

@@ -1,0 +1,434 @@
+// Grouped SwiGLU expert FFN on sm_103a tensor cores (tcgen05 + TMEM + TMA).
+//
+// Two persistent warp-specialised kernels over the expert-contiguous rows of
+// ordermoe_dispatch, with the per-expert row ranges read on the device:
+//   gate/up: H[rows of e, n0:n0+128] = bf16(silu(X W1_e^T) * (X W3_e^T)) for a
+//            128-column slice n0 of d_ff. One tcgen05.mma of N = 256 computes
+//            the gate (TMEM columns 0..127) and up (128..255) projections from
+//            a B tile whose first 128 rows are W1_e rows and last 128 rows are
+//            W3_e rows; the epilogue fuses SwiGLU.
+//   down:    Y[rows of e, n0:n0+256] = bf16(H W2_e^T).
+// Tile = 128 rows x 256 accumulator columns, K step 64 (one 128-byte
+// swizzled TMA box per operand row), 4-stage shared-memory ring, two TMEM
+// accumulators (2 x 256 columns = all 512) so the epilogue of one tile
+// overlaps the main loop of the next.
+// Warp roles (192 threads): warp 0 = TMA producer, warp 1 = MMA issuer and
+// TMEM owner, warps 2-5 = epilogue (warp w reads TMEM lanes 32 (w % 4) ...).
+// Tile order: expert, then N slice, then M tile, so CTAs running at the same
+// time share the same weight slice through L2.
+// Every wait is bounded (globaltimer); a wait that runs out reports
+// ORDERMOE_DEV_WAIT_TIMEOUT, makes the other roles stop, drains the copies
+// and MMAs in flight (bounded too), frees TMEM and returns.
+#include <mutex>
+
+#include "common.cuh"
+
+namespace om {
+
+static __device__ unsigned long long g_err_gemm = 0;
+
+int read_clear_err_gemm(unsigned long long* out) {
+  unsigned long long zero = 0;
+  OM_CUDA(cudaMemcpyFromSymbol(out, g_err_gemm, sizeof(*out)));
+  OM_CUDA(cudaMemcpyToSymbol(g_err_gemm, &zero, sizeof(zero)));
+  return ORDERMOE_OK;
+}
+
+namespace gg {
+
+constexpr int BM = 128;
+constexpr int BN = 256;  // accumulator columns per tile
+constexpr int BK = 64;   // bf16 elements = 128 bytes
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int BOX_BYTES = 128 * BK * 2;  // one TMA box: 128 rows x 64 columns
+constexpr int THREADS = 192;
+constexpr int TMEM_COLS = 512;
+constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
+
+struct Smem {
+  uint64_t full[STAGES];
+  uint64_t empty[STAGES];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+  int zero;
+  int mt_start[ORDERMOE_MAX_EXPERTS + 1];
+  int offs[ORDERMOE_MAX_EXPERTS + 1];
+};
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + static_cast<int>(sizeof(Smem));
+
+enum { GATEUP = 0, DOWN = 1 };
+
+struct Args {
+  const int32_t* offsets;
+  int E;
+  int K;             // reduction length
+  int n_tiles;       // N slices per expert
+  int b_rows;        // weight rows per expert in the B tensor map (d_ff or d)
+  uint16_t* out;     // H [R][d_ff] or Y [R][d]
+  int ldo;           // row length of out
+  uint64_t limit_ns; // bounded-wait limit
+};
+
+struct Tile {
+  int e, m0, m_end, n;
+};
+
+__device__ __forceinline__ Tile decode(int tile, const Smem& s, int E, int n_tiles) {
+  int e = 0;
+  while (e < E - 1 && s.mt_start[e + 1] * n_tiles <= tile) ++e;
+  const int local = tile - s.mt_start[e] * n_tiles;
+  const int n_mt = s.mt_start[e + 1] - s.mt_start[e];
+  Tile t;
+  t.e = e;
+  t.n = local / n_mt;
+  t.m0 = s.offs[e] + (local - t.n * n_mt) * BM;
+  t.m_end = s.offs[e + 1];
+  return t;
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(THREADS, 1)
+    ffn_gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB0,
+                    const __grid_constant__ CUtensorMap mapB1, Args args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* tiles = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  Smem& s = *reinterpret_cast<Smem*>(tiles + STAGES * STAGE_BYTES);
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+
+  if (tid == 0) {
+    for (int i = 0; i < STAGES; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s.tfull[i], 1);
+      mbar_init(&s.tempty[i], 128);
+    }
+    mbar_init(&s.drain, 1);
+    s.abort = 0;
+    s.zero = 0;
+    int acc = 0;
+    for (int e = 0; e <= args.E; ++e) {
+      const int o = args.offsets[e];
+      s.offs[e] = o;
+      if (e > 0) {
+        const int rows = o - s.offs[e - 1];
+        acc += rows > 0 ? (rows + BM - 1) / BM : 0;
+      }
+      s.mt_start[e] = acc;
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&mapA);
+    tma_prefetch_map(&mapB0);
+    if (MODE == GATEUP) tma_prefetch_map(&mapB1);
+  }
+  if (warp == 1) {
+    tmem_alloc(&s.tmem_base, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = s.tmem_base;
+  const int total = s.mt_start[args.E] * args.n_tiles;
+  const int kblocks = args.K / BK;
+  volatile int* abort = &s.abort;
+
+  // per-role bookkeeping for the drain after an abort
+  uint32_t issued_mask = 0, last_phase_bits = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x) {
+        const Tile t = decode(tile, s, args.E, args.n_tiles);
+        const int brow = t.e * args.b_rows + t.n * (MODE == GATEUP ? 128 : 256);
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
+            if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 1);
+            *abort = 1;
+            break;
+          }
+          uint8_t* sa = tiles + stage * STAGE_BYTES;
+          uint8_t* sb = sa + A_BYTES;
+          mbar_arrive_expect_tx(&s.full[stage], STAGE_BYTES);
+          tma_load_2d(sa, &mapA, &s.full[stage], kb * BK, t.m0);
+          if (MODE == GATEUP) {
+            tma_load_2d(sb, &mapB0, &s.full[stage], kb * BK, brow);
+            tma_load_2d(sb + BOX_BYTES, &mapB1, &s.full[stage], kb * BK, brow);
+          } else {
+            tma_load_2d(sb, &mapB0, &s.full[stage], kb * BK, brow);
+            tma_load_2d(sb + BOX_BYTES, &mapB0, &s.full[stage], kb * BK, brow + 128);
+          }
+          issued_mask |= 1u << stage;
+          last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x, ++it) {
+        const int slot = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!mbar_wait(&s.tempty[slot], acc_phase ^ 1u, args.limit_ns, abort)) {
+          if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 2);
+          *abort = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + slot * BN;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&s.full[stage], phase, args.limit_ns, abort)) {
+            if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 3);
+            *abort = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(tiles + stage * STAGE_BYTES);
+          const uint32_t b0 = a0 + A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk) {
+            mma_bf16(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
+                     IDESC, (kb | kk) != 0 ? 1u : 0u);
+          }
+          mma_issued = true;
+          mma_commit(&s.empty[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        mma_commit(&s.tfull[slot]);
+      }
+    }
+  } else {
+    // epilogue: warps 2..5 -> TMEM lane quarter (warp % 4)
+    const int q = warp & 3;
+    const int lrow = q * 32 + lane;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+      // warp-uniform control flow: tcgen05.ld below is .sync.aligned
+      if (__any_sync(0xffffffffu, *abort != 0)) break;
+      const int slot = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&s.tfull[slot], acc_phase, args.limit_ns, abort));
+      if (!ok) {
+        if (lane == 0 && !*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 4);
+        *abort = 1;
+        break;
+      }
+      tc_fence_after();
+      const Tile t = decode(tile, s, args.E, args.n_tiles);
+      const int row = t.m0 + lrow;
+      const bool valid = row < t.m_end;
+      const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
+      if (MODE == GATEUP) {
+        uint16_t* orow = args.out + (size_t)row * args.ldo + t.n * 128;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t g[32], u[32];
+          tmem_ld32(tb + c * 32, g);
+          tmem_ld32(tb + 128 + c * 32, u);
+          tmem_ld_wait();
+          if (valid) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+              const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+              const float h0 = g0 / (1.0f + __expf(-g0)) * u0;
+              const float h1 = g1 / (1.0f + __expf(-g1)) * u1;
+              pk[i] = pack_bf16x2(h0, h1);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+          }
+        }
+      } else {
+        uint16_t* orow = args.out + (size_t)row * args.ldo + t.n * 256;
+#pragma unroll 1
+        for (int c = 0; c < 8; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tb + c * 32, v);
+          tmem_ld_wait();
+          if (valid) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+              pk[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&s.tempty[slot]);
+    }
+  }
+
+  __syncthreads();
+  if (s.abort) {
+    volatile int* never = &s.zero;
+    if (warp == 0 && lane == 0) {
+      // wait for every TMA copy this CTA issued (bounded)
+      for (int st = 0; st < STAGES; ++st)
+        if ((issued_mask >> st) & 1u)
+          mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, args.limit_ns, never);
+    }
+    if (warp == 1 && lane == 0 && mma_issued) {
+      mma_commit(&s.drain);
+      mbar_wait(&s.drain, 0, args.limit_ns, never);
+    }
+    __syncthreads();
+  }
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+// ------------------------------------------------------------------- host
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 row-major [rows][cols] map with a 64 x 128 box and 128-byte swizzle.
+int make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return fail(ORDERMOE_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {BK, 128};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(ORDERMOE_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  return ORDERMOE_OK;
+}
+
+}  // namespace gg
+
+int ffn_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const uint16_t* W1,
+               const uint16_t* W3, const uint16_t* W2, int E, int d, int dff, uint16_t* H,
+               uint16_t* Y, cudaStream_t stream) {
+  using namespace gg;
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<GATEUP>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<DOWN>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(ffn_gemm_kernel)");
+  CUtensorMap mX, mW1, mW3, mH, mW2;
+  int rc;
+  if ((rc = make_map(&mX, X_perm, R, d))) return rc;
+  if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
+  if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
+  if ((rc = make_map(&mH, H, R, dff))) return rc;
+  if ((rc = make_map(&mW2, W2, (uint64_t)E * d, dff))) return rc;
+  const int sms = num_sms();
+  const long long mt_max = (R + BM - 1) / BM + E;
+  Args a{};
+  a.offsets = offsets;
+  a.E = E;
+  a.limit_ns = wait_limit_ns();
+  // gate/up
+  a.K = d; a.n_tiles = dff / 128; a.b_rows = dff; a.out = H; a.ldo = dff;
+  long long tiles = mt_max * a.n_tiles;
+  int grid = static_cast<int>(tiles < sms ? tiles : sms);
+  ffn_gemm_kernel<GATEUP><<<grid, THREADS, SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
+  OM_LAUNCHED("ffn_gemm_kernel<gate_up>");
+  // down
+  a.K = dff; a.n_tiles = d / 256; a.b_rows = d; a.out = Y; a.ldo = d;
+  tiles = mt_max * a.n_tiles;
+  grid = static_cast<int>(tiles < sms ? tiles : sms);
+  ffn_gemm_kernel<DOWN><<<grid, THREADS, SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
+  OM_LAUNCHED("ffn_gemm_kernel<down>");
+  return ORDERMOE_OK;
+}
+
+// ---------------------------------------------------------- wait self-test
+__global__ void wait_timeout_kernel(uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    // nothing ever arrives on `bar`: the wait must run out
+    if (!mbar_wait(&bar, 0, limit_ns, reinterpret_cast<volatile int*>(&abort_flag)))
+      report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 99);
+  }
+}
+
+int selftest_wait_timeout(uint64_t limit_ns, cudaStream_t stream) {
+  wait_timeout_kernel<<<1, 32, 0, stream>>>(limit_ns);
+  OM_LAUNCHED("wait_timeout_kernel");
+  return ORDERMOE_OK;
+}
+
+}  // namespace om
+
+using namespace om;
+
+extern "C" int ordermoe_expert_ffn(const uint16_t* X_perm, const int32_t* offsets, int R,
+                                   const uint16_t* W1, const uint16_t* W3, const uint16_t* W2,
+                                   int E, int d, int dff, uint16_t* H, uint16_t* Y_perm,
+                                   ordermoe_stream_t stream) {
+  if (R < 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_ffn: need R >= 0 and 1 <= E <= 64");
+  if (d <= 0 || d % 256 != 0 || dff <= 0 || dff % 128 != 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_ffn: need d %% 256 == 0 and dff %% 128 == 0");
+  if (R == 0) return ORDERMOE_OK;
+  if (!X_perm || !offsets || !W1 || !W3 || !W2 || !H || !Y_perm)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "expert_ffn: null pointer");
+  if (!aligned16(X_perm) || !aligned16(W1) || !aligned16(W3) || !aligned16(W2) || !aligned16(H) ||
+      !aligned16(Y_perm))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "expert_ffn: pointers must be 16-byte aligned");
+  if ((long long)E * dff > INT32_MAX || (long long)E * d > INT32_MAX)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_ffn: weight rows exceed 2^31");
+  return ffn_launch(X_perm, offsets, R, W1, W3, W2, E, d, dff, H, Y_perm, stream);
+}

@@ -1,0 +1,57 @@
+"""Test-side helpers: run the oracle's offline plan (Eqs. 3-6, 24-31) and the
+oracle's per-token forward for sampled tokens."""
+import numpy as np
+
+import oracle
+from paper_2607_17154_gb300 import synth
+
+
+def bits_to_f(b):
+    return (np.asarray(b, np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def oracle_plan(Wr_bits, Xcal_bits, k, M, theta, p_unit=1.0):
+    """Similarity, counts, groups and placement of one layer by the oracle."""
+    E = Wr_bits.shape[0]
+    sim, H = oracle.similarity(Wr_bits, Xcal_bits, return_H=True)
+    counts = oracle.expert_counts(np.ascontiguousarray(H.T), k)
+    group, K, _ = oracle.group(sim, counts, theta)
+    imp = oracle.importance(sim, counts, group)
+    p = np.full((1, E), p_unit)
+    C = np.full(M, E * p_unit / M)
+    x, used, rc = oracle.place(group[None], imp[None], p, C)
+    assert rc == 0
+    return dict(sim=sim, counts=counts, group=group, K=K, placement=x[0])
+
+
+def oracle_layer_tokens(tokens, X_bits, Wr_bits, W1, W3, W2, tab, home, loc, qhat, k, renorm=1):
+    """Oracle forward of the listed tokens through one layer.
+
+    Returns (y [n,d] bf16 bits, idx, w, chosen, server, kind, margin) where
+    margin is the oracle's logit gap around the k-th rank (small = near tie)."""
+    Xs = X_bits[tokens]
+    logits = oracle.router_logits(Xs, Wr_bits)
+    idx, w = oracle.topk(logits, k, renorm)
+    chosen, server, kind, loc2, q2 = oracle.select(idx, tab, home[tokens], loc[tokens], qhat[tokens])
+    srt = -np.sort(-logits.astype(np.float64), axis=1)
+    E = logits.shape[1]
+    gaps = np.abs(np.diff(srt[:, :min(k + 1, E)], axis=1))
+    margin = gaps.min(axis=1) if gaps.shape[1] else np.full(len(tokens), np.inf)
+    n = len(tokens)
+    rows = np.repeat(Xs, k, axis=0)
+    _, Y = oracle.ffn_rows(rows, chosen.reshape(-1).astype(np.int32), W1, W3, W2)
+    row_of = np.arange(n * k, dtype=np.int32).reshape(n, k)
+    y = oracle.combine(Y, row_of, w)
+    return dict(y=y, logits=logits, idx=idx, w=w, chosen=chosen, server=server, kind=kind,
+                loc=loc2, qhat=q2, margin=margin)
+
+
+def assert_close_bf16(got_bits, ref_bits, rtol=2e-2, atol=1e-2, what=""):
+    g = bits_to_f(got_bits).astype(np.float64)
+    r = bits_to_f(ref_bits).astype(np.float64)
+    bad = np.abs(g - r) > atol + rtol * np.abs(r)
+    if bad.any():
+        i = np.argwhere(bad)[:5]
+        raise AssertionError("%s: %d / %d elements outside rtol=%g atol=%g; first %s: got %s ref %s"
+                             % (what, bad.sum(), bad.size, rtol, atol, i.tolist(),
+                                g[tuple(i.T)].tolist(), r[tuple(i.T)].tolist()))
