@@ -1,0 +1,434 @@
+#!/usr/bin/env python
+"""Benchmark of the OrderMoE MoE-layer hot path on GB300.
+
+One step = one pass of the hot path over one batch: router + softmax + top-k
++ server-expert selection, permutation, grouped SwiGLU expert FFN (gate/up,
+down) and weighted combine -- seven kernels of libordermoe.so, nothing else.
+Default workload: the Mixtral-8x7B-shaped prefill layer (T = 4096 tokens,
+d = 4096, E = 8, top-2, d_ff = 14336, 4 logical servers), synthetic seeded
+inputs drawn on the device. The offline plan (similarity, grouping,
+placement, tables) runs once through the library before timing.
+
+Prints one JSON line (rank 0). `--impl reference` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "MoE-layer tokens/s on 1 GB300 (route+select+FFN) and % of tensor/HBM roofline"
+UNIT = "tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=500)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="mixtral_prefill")
+    p.add_argument("--seed", type=int, default=0)
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=15.0,
+                   help="target CPU seconds of the oracle baseline sample")
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.index = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1])); smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, v in zip(self.NAMES, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gpu_index(local_rank):
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        items = [v.strip() for v in vis.split(",") if v.strip()]
+        if local_rank < len(items):
+            return items[local_rank]
+    return str(local_rank)
+
+
+# ----------------------------------------------------------------- distributed
+class Dist:
+    """Replicas only: ranks share nothing on the data path; the process group
+    serves the timing barrier and the max-over-ranks reduction."""
+
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+        if self.world > 1:
+            import torch.distributed as dist
+            backend = os.environ.get("ORDERMOE_BENCH_BACKEND", "nccl")
+            dist.init_process_group(backend=backend)
+            self.pg = dist
+
+    def barrier(self, device=None):
+        if self.pg is not None:
+            if device is not None and self.pg.get_backend() == "nccl":
+                self.pg.barrier(device_ids=[device.index])
+            else:
+                self.pg.barrier()
+
+    def max(self, value, device=None):
+        if self.pg is None:
+            return value
+        import torch
+        t = torch.tensor([float(value)], dtype=torch.float64,
+                         device=device if self.pg.get_backend() == "nccl" else "cpu")
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def close(self):
+        if self.pg is not None:
+            self.pg.destroy_process_group()
+
+
+# ----------------------------------------------------------------- our arm
+def setup_gpu(w, seed, device):
+    """Inputs on the device, then the offline plan through the library."""
+    import torch
+    from paper_2607_17154_gb300 import binding as B
+    from paper_2607_17154_gb300 import synth
+
+    inp = synth.layer_inputs(w, seed=seed, device=device)
+    home = torch.as_tensor(inp["home"]).to(device)
+    Xcal = synth.calibration(w.n_cal, w.d, seed, device=device)
+    sim = torch.empty(1, w.E, w.E, dtype=torch.float32, device=device)
+    counts = torch.empty(1, w.E, dtype=torch.int32, device=device)
+    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(1, w.E, w.n_cal), dtype=torch.uint8,
+                     device=device)
+    t0 = time.perf_counter()
+    B.ordermoe_similarity(inp["Wr"], Xcal, 1, w.E, w.d, w.n_cal, w.k, sim, counts, ws)
+    group = torch.empty(1, w.E, dtype=torch.int32, device=device)
+    ngroups = torch.empty(1, dtype=torch.int32, device=device)
+    theta = torch.empty(1, dtype=torch.float32, device=device)
+    placement = torch.empty(1, w.M, w.E, dtype=torch.uint8, device=device)
+    used = torch.empty(w.M, dtype=torch.float64, device=device)
+    status = torch.empty(1, dtype=torch.int32, device=device)
+    p = torch.ones(1, w.E, dtype=torch.float64, device=device)
+    C = torch.full((w.M,), w.E / w.M, dtype=torch.float64, device=device)
+    B.ordermoe_place(sim, counts, 1, w.E, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5, 0.5,
+                     0.5, p, C, group, ngroups, theta, placement, used, status)
+    sp = synth.server_params(w.M, w.d, w.dff, seed)
+    f64 = lambda a: torch.as_tensor(a, dtype=torch.float64).to(device)
+    tables = torch.zeros(B.ordermoe_tables_bytes(w.E, w.M), dtype=torch.uint8, device=device)
+    B.ordermoe_build_tables(sim[0], group[0], placement[0], w.theta, w.qbar, f64(sp.F), f64(sp.B),
+                            f64(sp.tau), sp.z, sp.c, sp.omega_T, sp.omega_Q, tables)
+    torch.cuda.synchronize(device)
+    plan_ms = (time.perf_counter() - t0) * 1e3
+    code, detail = B.ordermoe_device_error()
+    if code:
+        raise RuntimeError("device error %d (%d) in the offline plan" % (code, detail))
+    return inp, home, tables, {"plan_ms": round(plan_ms, 3), "n_groups": int(ngroups.item()),
+                               "place_status": int(status.item())}
+
+
+def run_ours(args, dist):
+    import torch
+    from paper_2607_17154_gb300 import binding as B
+    from paper_2607_17154_gb300 import synth
+
+    device = torch.device("cuda", dist.local_rank)
+    torch.cuda.set_device(device)
+    B.lib()
+    w = synth.workload(args.workload)
+    if w.L != 1:
+        raise SystemExit("bench.py times single-layer workloads; %s has %d layers" % (w.name, w.L))
+    inp, home, tables, plan = setup_gpu(w, args.seed + 1000 * dist.rank, device)
+    T, E, d, k, dff = w.T, w.E, w.d, w.k, w.dff
+    R = T * k
+    X, Wr, W1, W3, W2 = (inp[n] for n in ("X", "Wr", "W1", "W3", "W2"))
+    f = lambda *s, dt: torch.empty(*s, dtype=dt, device=device)
+    idx, wts, ch = f(T, k, dt=torch.int32), f(T, k, dt=torch.float32), f(T, k, dt=torch.int32)
+    sv, kd = f(T, k, dt=torch.uint8), f(T, k, dt=torch.uint8)
+    counters = torch.zeros(4, dtype=torch.int32, device=device)
+    offsets, row_token, row_of = f(E + 1, dt=torch.int32), f(R, dt=torch.int32), f(T, k, dt=torch.int32)
+    Xp, H, Yp = f(R, d, dt=torch.bfloat16), f(R, dff, dt=torch.bfloat16), f(R, d, dt=torch.bfloat16)
+    y = f(T, d, dt=torch.bfloat16)
+    ws = f(B.ordermoe_dispatch_workspace_bytes(T, k, E), dt=torch.uint8)
+    stream = torch.cuda.current_stream(device)
+
+    def step(ev0=None, ev1=None, cnt=None):
+        B.ordermoe_route_select(X, Wr, None, T, E, d, k, 1, tables, home, None, None, None, idx,
+                                wts, ch, sv, kd, cnt)
+        B.ordermoe_dispatch(ch, X, T, k, E, d, offsets, row_token, row_of, Xp, ws)
+        if ev0 is not None:
+            ev0.record(stream)
+        B.ordermoe_expert_gate_up(Xp, offsets, R, W1, W3, E, d, dff, H)
+        if ev1 is not None:
+            ev1.record(stream)
+        B.ordermoe_expert_down(H, offsets, R, W2, E, d, dff, Yp)
+        B.ordermoe_combine(Yp, row_of, wts, T, k, d, y)
+
+    KERNELS_PER_STEP = 7   # route_select 1, dispatch 3, gate/up 1, down 1, combine 1
+    step(cnt=counters)     # one counted pass for the execution-type breakdown
+    for _ in range(max(args.warmup, 3)):
+        step()
+    ev0 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ev1 = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(gpu_index(dist.local_rank))
+    sampler.start()
+    dist.barrier(device)
+    torch.cuda.synchronize(device)
+    start.record(stream)
+    for i in range(args.steps):
+        step(ev0[i], ev1[i])
+    stop.record(stream)
+    torch.cuda.synchronize(device)
+    dist.barrier(device)
+    clocks = sampler.stop()
+    elapsed_ms = start.elapsed_time(stop)
+    gu_ms = statistics.mean(a.elapsed_time(b) for a, b in zip(ev0, ev1))
+    code, detail = B.ordermoe_device_error()
+    if code:
+        raise RuntimeError("device error %d (%d) during the timed steps" % (code, detail))
+    elapsed_ms = dist.max(elapsed_ms, device)
+    total_tokens = T * args.steps * dist.world
+    value = total_tokens / (elapsed_ms / 1e3)
+
+    # end to end through the C ABI with host buffers (pinned), copies timed
+    e2e = None
+    if not args.no_e2e:
+        scratch = torch.empty(B.ordermoe_layer_scratch_bytes(T, E, d, dff, k), dtype=torch.uint8,
+                              device=device)
+        desc = B.make_layer_desc(T, Wr, W1, W3, W2, tables, k, scratch)
+        Xh = X.cpu().pin_memory()
+        hh = home.cpu().pin_memory()
+        yh = torch.empty(T, d, dtype=torch.bfloat16).pin_memory()
+        for _ in range(max(args.warmup, 3)):
+            B.ordermoe_layer_forward(desc, T, Xh, hh, None, None, yh, None, host_io=1)
+        n_e2e = max(1, min(args.steps, 200))
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        dist.barrier(device)
+        torch.cuda.synchronize(device)
+        a.record(stream)
+        for _ in range(n_e2e):
+            B.ordermoe_layer_forward(desc, T, Xh, hh, None, None, yh, None, host_io=1)
+        b.record(stream)
+        torch.cuda.synchronize(device)
+        dist.barrier(device)
+        e_ms = dist.max(a.elapsed_time(b), device)
+        e2e = {"value": round(T * n_e2e * dist.world / (e_ms / 1e3), 1), "unit": UNIT,
+               "h2d_bytes_per_step": T * d * 2 + T, "d2h_bytes_per_step": T * d * 2,
+               "steps": n_e2e}
+        code, detail = B.ordermoe_device_error()
+        if code:
+            raise RuntimeError("device error %d (%d) during the e2e steps" % (code, detail))
+
+    pk, pk_kind = peaks()
+    gu_flop = 2.0 * R * d * 2 * dff
+    achieved = gu_flop / (gu_ms / 1e3) / 1e12
+    peak = float(pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    layer_flop = 2.0 * R * 3 * d * dff + 2.0 * T * d * E
+    out = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": dist.world,
+        "steps": args.steps, "warmup": max(args.warmup, 3),
+        "ms_per_step": round(elapsed_ms / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "T": T, "d": d, "E": E, "k": k, "d_ff": dff, "M": w.M,
+                   "similarity_groups": w.n_clusters, "theta": w.theta, "qbar": w.qbar,
+                   "home": w.home, "seed": args.seed, "parallelism": "replicas",
+                   "l2": "inputs larger than L2: %.2f GB of expert weights read every step"
+                         % (3 * E * d * dff * 2 / 1e9)},
+        "roofline": {"kernel": "ffn_gemm_kernel<gate_up> (tcgen05)", "bound": "tensor",
+                     "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
+                     "frac": round(achieved / peak, 4), "traffic": None,
+                     "peak_source": "%s bf16_tflops_sustained" % pk_kind,
+                     "flop_per_launch": gu_flop, "ms_per_launch": round(gu_ms, 4),
+                     "layer_tflops": round(layer_flop / (elapsed_ms / args.steps / 1e3) / 1e12, 1)},
+        "e2e": e2e,
+        "gpu_launches": KERNELS_PER_STEP * args.steps,
+        "clocks": clocks,
+        "exec_types": dict(zip(["local_exact", "local_sub", "remote_exact", "remote_sub"],
+                               counters.cpu().tolist())),
+        "plan": plan,
+    }
+    if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(w, inp, args.seed, args.cpu_seconds)
+    return out
+
+
+# ----------------------------------------------------------------- oracle side
+def oracle_setup(w, inp, seed):
+    """Host copies of the inputs and the oracle's own plan and tables."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_17154_gb300 import synth
+    bits = synth.bits
+    host = {n: bits(inp[n]) for n in ("X", "Wr", "W1", "W3", "W2")}
+    home = np.asarray(inp["home"].cpu() if hasattr(inp["home"], "cpu") else inp["home"], np.uint8)
+    Xcal = bits(synth.calibration(w.n_cal, w.d, seed, device=inp["X"].device))
+    sim, H = oracle.similarity(host["Wr"], Xcal, return_H=True)
+    counts = oracle.expert_counts(np.ascontiguousarray(H.T), w.k)
+    group, K, _ = oracle.group(sim, counts, w.theta)
+    imp = oracle.importance(sim, counts, group)
+    x, _, _ = oracle.place(group[None], imp[None], np.ones((1, w.E)), np.full(w.M, w.E / w.M))
+    sp = synth.server_params(w.M, w.d, w.dff, seed)
+    tab = oracle.tables(sim, group, x[0], w.theta, w.qbar, sp.F, sp.B, sp.tau, sp.z, sp.c,
+                        sp.omega_T, sp.omega_Q)
+    return host, home, tab
+
+
+def oracle_tokens(w, host, home, tab, toks):
+    """The oracle's whole hot path for the listed tokens."""
+    import numpy as np
+
+    import oracle
+    Xs = np.ascontiguousarray(host["X"][toks])
+    logits = oracle.router_logits(Xs, host["Wr"])
+    idx, wt = oracle.topk(logits, w.k)
+    h = home[toks]
+    chosen, _, _, _, _ = oracle.select(idx, tab, h, h.copy(), np.zeros(len(toks), np.float32))
+    off, rt, row_of = oracle.dispatch(chosen, w.E)
+    Xp = oracle.gather_rows(Xs, rt)
+    row_e = np.repeat(np.arange(w.E), np.diff(off)).astype(np.int32)
+    _, Y = oracle.ffn_rows(Xp, row_e, host["W1"], host["W3"], host["W2"])
+    return oracle.combine(Y, row_of, wt)
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(w, inp, seed, target_s):
+    import numpy as np
+    host, home, tab = oracle_setup(w, inp, seed)
+    rng = np.random.default_rng(seed)
+    t0 = time.perf_counter()
+    oracle_tokens(w, host, home, tab, np.sort(rng.choice(w.T, 4, replace=False)))
+    per_tok = max((time.perf_counter() - t0) / 4, 1e-6)
+    n = int(min(w.T, max(4, target_s / per_tok)))
+    toks = np.sort(rng.choice(w.T, n, replace=False))
+    t0 = time.perf_counter()
+    oracle_tokens(w, host, home, tab, toks)
+    dt = time.perf_counter() - t0
+    return {"value": round(n / dt, 3), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+            "sample": "%d of the %d tokens of one %s layer through the whole oracle path "
+                      "(router, top-k, selection, permutation, SwiGLU FFN, combine), %.1f s"
+                      % (n, w.T, w.name, dt)}
+
+
+def run_reference(args, dist):
+    """The CPU oracle as it stands, each step a bounded sample of the workload."""
+    import numpy as np
+    import torch
+    from paper_2607_17154_gb300 import synth
+    w = synth.workload(args.workload)
+    device = "cuda" if torch.cuda.is_available() else "cpu"
+    inp = synth.layer_inputs(w, seed=args.seed, device=device)
+    host, home, tab = oracle_setup(w, inp, args.seed)
+    rng = np.random.default_rng(args.seed)
+    t0 = time.perf_counter()
+    oracle_tokens(w, host, home, tab, np.sort(rng.choice(w.T, 2, replace=False)))
+    per_tok = max((time.perf_counter() - t0) / 2, 1e-6)
+    budget = 150.0
+    n = int(max(1, min(w.T, budget / max(1, args.steps + args.warmup) / per_tok)))
+    for _ in range(args.warmup):
+        oracle_tokens(w, host, home, tab, np.sort(rng.choice(w.T, n, replace=False)))
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_tokens(w, host, home, tab, np.sort(rng.choice(w.T, n, replace=False)))
+    dt = time.perf_counter() - t0
+    value = n * args.steps / dt
+    sample = ("%d of the %d tokens of one %s layer per step through the whole oracle path"
+              % (n, w.T, w.name))
+    return {
+        "impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
+        "n_gpus": dist.world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "T": w.T, "d": w.d, "E": w.E, "k": w.k, "d_ff": w.dff,
+                   "M": w.M, "tokens_per_step": n},
+        "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cpu_cores(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse()
+    dist = Dist()
+    try:
+        if args.impl == "reference":
+            if dist.rank != 0:
+                return
+            out = run_reference(args, dist)
+        else:
+            out = run_ours(args, dist)
+        if dist.rank == 0:
+            print(json.dumps(out), flush=True)
+    finally:
+        dist.close()
+
+
+if __name__ == "__main__":
+    main()

@@ -129,6 +129,9 @@ int ordermoe_build_tables(const float* sim, const int32_t* group, const uint8_t*
  *   loc        [T] u8   in/out: server holding the token before / after the
  *              layer (Eq. 36, Eq. 44); set loc = home before the first layer
  *   qhat       [T] f32  in/out: accumulated quality loss (Eq. 44); 0 at start
+ *              loc and qhat may both be NULL: every token then starts at its
+ *              home server with zero loss (the first layer) and the new state
+ *              is not written
  *   logits_out [T][E] f32, nullable: the router logits
  *   topk_idx   [T][k] i32  routed (target) experts, rank order
  *   topk_w     [T][k] f32  gate weights of the routed slots
@@ -183,6 +186,14 @@ int ordermoe_expert_ffn(const uint16_t* X_perm, const int32_t* offsets, int R, c
                         const uint16_t* W3, const uint16_t* W2, int E, int d, int dff, uint16_t* H,
                         uint16_t* Y_perm, ordermoe_stream_t stream);
 
+/* The two halves of ordermoe_expert_ffn as separate launches (same shapes,
+ * same rules): H = SwiGLU(X_perm W1^T, X_perm W3^T), then Y_perm = H W2^T. */
+int ordermoe_expert_gate_up(const uint16_t* X_perm, const int32_t* offsets, int R,
+                            const uint16_t* W1, const uint16_t* W3, int E, int d, int dff,
+                            uint16_t* H, ordermoe_stream_t stream);
+int ordermoe_expert_down(const uint16_t* H, const int32_t* offsets, int R, const uint16_t* W2,
+                         int E, int d, int dff, uint16_t* Y_perm, ordermoe_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * Weighted combine: y[t] = bf16( sum_{j=0..k-1} topk_w[t][j] * Y_perm[row_of[t][j]] )
  * with fp32 accumulation in slot order.
@@ -190,6 +201,95 @@ int ordermoe_expert_ffn(const uint16_t* X_perm, const int32_t* offsets, int R, c
  * d % 8 == 0, 16-byte aligned Y_perm / y. */
 int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of, const float* topk_w, int T,
                      int k, int d, uint16_t* y, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * One whole MoE layer: route_select, dispatch, expert_gate_up, expert_down and
+ * combine in order on `stream`, with all intermediates in `scratch`.
+ * The descriptor (host memory) holds device pointers owned by the caller:
+ *   W_r [E][d], W1/W3 [E][dff][d], W2 [E][d][dff] bf16; tables of the layer;
+ *   scratch: ordermoe_layer_scratch_bytes(T_max, E, d, dff, k) bytes,
+ *   256-byte aligned. */
+typedef struct {
+  int T_max, E, d, dff, k, renorm;
+  const uint16_t* W_r;
+  const uint16_t* W1;
+  const uint16_t* W3;
+  const uint16_t* W2;
+  const void* tables;
+  size_t tables_bytes;
+  void* scratch;
+  size_t scratch_bytes;
+} ordermoe_layer_desc;
+
+size_t ordermoe_layer_scratch_bytes(int T_max, int E, int d, int dff, int k);
+
+/* y[t] = MoE layer output of token t, t < T <= T_max.
+ *   X [T][d] bf16, home [T] u8, y [T][d] bf16 out.
+ *   loc [T] u8 and qhat [T] f32 in/out (Eq. 36 / Eq. 44), or both NULL: the
+ *   tokens then start at their home server with zero accumulated loss (the
+ *   first MoE layer) and the new state is not returned.
+ *   counters [4] i32 device, nullable (see ordermoe_route_select).
+ *   host_io = 0: X, home, loc, qhat, y are device pointers.
+ *   host_io = 1: they are HOST pointers (pinned for asynchronous copies); the
+ *   call enqueues the host -> device copies, the layer, and the device -> host
+ *   copies on `stream`; the caller synchronises before reading y.
+ * Shapes as ordermoe_route_select and ordermoe_expert_ffn. */
+int ordermoe_layer_forward(const ordermoe_layer_desc* layer, int T, const uint16_t* X,
+                           const uint8_t* home, uint8_t* loc, float* qhat, uint16_t* y,
+                           int32_t* counters, int host_io, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Offline expert similarity (Section III-B, Eqs. 3-5; Alg. 1 lines 3-5).
+ * For each layer l: H_l = W_r^l X_cal^T (router logits over the calibration
+ * tokens, fp32 accumulation on tcgen05 tensor cores),
+ * Sim_l(i,j) = <H_l,i, H_l,j> / (|H_l,i| |H_l,j|) (Eq. 4; diagonal exactly 1,
+ * 0 for a zero-norm row), and the activation counts n_l^j = number of
+ * calibration tokens whose top-k_freq experts include j (Eq. 5; ties to the
+ * lower index).
+ *   W_r      [L][E][d] bf16 (the L router matrices stacked)
+ *   X_cal    [N][d] bf16 calibration tokens
+ *   sim      [L][E][E] f32 out;  counts [L][E] i32 out
+ *   workspace  device scratch of ordermoe_similarity_workspace_bytes(L,E,N)
+ *              bytes, 256-byte aligned (holds H in fp32 and partial Grams)
+ * Shapes: d % 64 == 0, 1 <= k_freq <= E <= 64. Gram partial sums are reduced
+ * in a fixed order: results are deterministic. */
+size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N);
+int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d, int64_t N,
+                        int k_freq, float* sim, int32_t* counts, void* workspace,
+                        size_t workspace_bytes, ordermoe_stream_t stream);
+
+/* Activation counts of Eq. 5 from given logits [N][E] f32 (top-k_freq per
+ * token, ties to the lower index). counts [E] i32 out (overwritten). */
+int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq, int32_t* counts,
+                           ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Grouping and mandatory placement (Section IV-A/B; Alg. 1 lines 1-24), all
+ * layers in order:
+ *   theta_l = theta_min + (theta_max - theta_min)(L - l)/(L - 1), l = 1..L
+ *            (Eq. 6; L == 1 uses theta_single);
+ *   greedy representative cover (Eqs. 24-26): experts by decreasing count
+ *            (ties: lower index) become a new dominant when their largest Sim
+ *            to the existing dominants is < theta_l, else join the most similar
+ *            dominant's group (ties: the earlier dominant); group id = the
+ *            dominant's creation order;
+ *   importance I = alpha_f f + alpha_r rho (Eqs. 27-28);
+ *   placement (Eqs. 29-31): experts by (p desc, I desc, index asc), feasible
+ *            servers b_m + p <= C_m, score lambda1 b_m / C_m + lambda2 eta,
+ *            lowest score (ties: lower m); experts with no feasible server go,
+ *            after the layer, to the server with the most free memory. The
+ *            used memory b_m accumulates over the layers.
+ *   sim [L][E][E] f32, counts [L][E] i32, p [L][E] f64 (memory of each
+ *   expert), C [M] f64 (server capacities)
+ *   group [L][E] i32 out, n_groups [L] i32 out, theta [L] f32 out,
+ *   placement [L][M][E] u8 out, used [M] f64 out,
+ *   status [1] i32 out (device): ORDERMOE_OK, or ORDERMOE_ERR_CAPACITY when
+ *   sum C < sum p or a waiting-list expert overflowed its server. */
+int ordermoe_place(const float* sim, const int32_t* counts, int L, int E, int M, double theta_min,
+                   double theta_max, double theta_single, double alpha_f, double alpha_r,
+                   double lambda1, double lambda2, const double* p, const double* C,
+                   int32_t* group, int32_t* n_groups, float* theta, uint8_t* placement,
+                   double* used, int32_t* status, ordermoe_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -39,7 +39,23 @@ _SIGNATURES = {
     "ordermoe_dispatch": ([_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ordermoe_expert_ffn": ([_P, _P, _I, _P, _P, _P, _I, _I, _I, _P, _P, _P], _I),
     "ordermoe_combine": ([_P, _P, _P, _I, _I, _I, _P, _P], _I),
+    "ordermoe_similarity_workspace_bytes": ([_I, _I, _I64], _SZ),
+    "ordermoe_similarity": ([_P, _P, _I, _I, _I, _I64, _I, _P, _P, _P, _SZ, _P], _I),
+    "ordermoe_expert_counts": ([_P, _I64, _I, _I, _P, _P], _I),
+    "ordermoe_place": ([_P, _P, _I, _I, _I, _D, _D, _D, _D, _D, _D, _D, _P, _P, _P, _P, _P, _P,
+                        _P, _P, _P], _I),
+    "ordermoe_expert_gate_up": ([_P, _P, _I, _P, _P, _I, _I, _I, _P, _P], _I),
+    "ordermoe_expert_down": ([_P, _P, _I, _P, _I, _I, _I, _P, _P], _I),
+    "ordermoe_layer_scratch_bytes": ([_I, _I, _I, _I, _I], _SZ),
+    "ordermoe_layer_forward": ([_P, _I, _P, _P, _P, _P, _P, _P, _I, _P], _I),
 }
+
+
+class LayerDesc(ctypes.Structure):
+    """Mirror of ordermoe_layer_desc."""
+    _fields_ = [("T_max", _I), ("E", _I), ("d", _I), ("dff", _I), ("k", _I), ("renorm", _I),
+                ("W_r", _P), ("W1", _P), ("W3", _P), ("W2", _P), ("tables", _P),
+                ("tables_bytes", _SZ), ("scratch", _P), ("scratch_bytes", _SZ)]
 
 
 class OrderMoEError(RuntimeError):
@@ -178,3 +194,93 @@ def ordermoe_combine(Y_perm, row_of, topk_w, T, k, d, y, stream=None):
     rc = lib().ordermoe_combine(_ptr(Y_perm), _ptr(row_of), _ptr(topk_w), T, k, d, _ptr(y),
                                 _stream(stream))
     _check("ordermoe_combine", rc)
+
+
+def ordermoe_similarity_workspace_bytes(L, E, N):
+    return int(lib().ordermoe_similarity_workspace_bytes(L, E, N))
+
+
+def ordermoe_similarity(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, stream=None):
+    _dt(W_r, torch.bfloat16, "W_r"); _dt(X_cal, torch.bfloat16, "X_cal")
+    _dt(sim, torch.float32, "sim"); _dt(counts, torch.int32, "counts")
+    rc = lib().ordermoe_similarity(_ptr(W_r), _ptr(X_cal), L, E, d, N, k_freq, _ptr(sim),
+                                   _ptr(counts), _ptr(workspace),
+                                   workspace.numel() * workspace.element_size(), _stream(stream))
+    _check("ordermoe_similarity", rc)
+
+
+def ordermoe_expert_counts(logits, N, E, k_freq, counts, stream=None):
+    _dt(logits, torch.float32, "logits"); _dt(counts, torch.int32, "counts")
+    _check("ordermoe_expert_counts",
+           lib().ordermoe_expert_counts(_ptr(logits), N, E, k_freq, _ptr(counts), _stream(stream)))
+
+
+def ordermoe_place(sim, counts, L, E, M, theta_min, theta_max, theta_single, alpha_f, alpha_r,
+                   lambda1, lambda2, p, C, group, n_groups, theta, placement, used, status,
+                   stream=None):
+    _dt(sim, torch.float32, "sim"); _dt(counts, torch.int32, "counts")
+    _dt(p, torch.float64, "p"); _dt(C, torch.float64, "C"); _dt(group, torch.int32, "group")
+    _dt(n_groups, torch.int32, "n_groups"); _dt(theta, torch.float32, "theta")
+    _dt(placement, torch.uint8, "placement"); _dt(used, torch.float64, "used")
+    _dt(status, torch.int32, "status")
+    rc = lib().ordermoe_place(_ptr(sim), _ptr(counts), L, E, M, float(theta_min), float(theta_max),
+                              float(theta_single), float(alpha_f), float(alpha_r), float(lambda1),
+                              float(lambda2), _ptr(p), _ptr(C), _ptr(group), _ptr(n_groups),
+                              _ptr(theta), _ptr(placement), _ptr(used), _ptr(status), _stream(stream))
+    _check("ordermoe_place", rc)
+
+
+def ordermoe_expert_gate_up(X_perm, offsets, R, W1, W3, E, d, dff, H, stream=None):
+    for n, t in (("X_perm", X_perm), ("W1", W1), ("W3", W3), ("H", H)):
+        _dt(t, torch.bfloat16, n)
+    _dt(offsets, torch.int32, "offsets")
+    _check("ordermoe_expert_gate_up",
+           lib().ordermoe_expert_gate_up(_ptr(X_perm), _ptr(offsets), R, _ptr(W1), _ptr(W3), E, d,
+                                         dff, _ptr(H), _stream(stream)))
+
+
+def ordermoe_expert_down(H, offsets, R, W2, E, d, dff, Y_perm, stream=None):
+    for n, t in (("H", H), ("W2", W2), ("Y_perm", Y_perm)):
+        _dt(t, torch.bfloat16, n)
+    _dt(offsets, torch.int32, "offsets")
+    _check("ordermoe_expert_down",
+           lib().ordermoe_expert_down(_ptr(H), _ptr(offsets), R, _ptr(W2), E, d, dff, _ptr(Y_perm),
+                                      _stream(stream)))
+
+
+def ordermoe_layer_scratch_bytes(T_max, E, d, dff, k):
+    return int(lib().ordermoe_layer_scratch_bytes(T_max, E, d, dff, k))
+
+
+def make_layer_desc(T_max, W_r, W1, W3, W2, tables, k, scratch, renorm=1):
+    E, dff, d = W1.shape
+    for n, t in (("W_r", W_r), ("W1", W1), ("W3", W3), ("W2", W2)):
+        _dt(t, torch.bfloat16, n)
+    desc = LayerDesc(T_max, E, d, dff, k, int(renorm), _ptr(W_r), _ptr(W1), _ptr(W3), _ptr(W2),
+                     _ptr(tables), tables.numel(), _ptr(scratch),
+                     scratch.numel() * scratch.element_size())
+    desc._keep = (W_r, W1, W3, W2, tables, scratch)
+    return desc
+
+
+def _host_or_dev_ptr(t, host):
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensor must be contiguous")
+    if host and t.is_cuda:
+        raise ValueError("host_io=1 needs host tensors")
+    if not host and not t.is_cuda:
+        raise ValueError("host_io=0 needs CUDA tensors")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def ordermoe_layer_forward(desc, T, X, home, loc, qhat, y, counters=None, host_io=0, stream=None):
+    h = bool(host_io)
+    _dt(X, torch.bfloat16, "X"); _dt(y, torch.bfloat16, "y"); _dt(home, torch.uint8, "home")
+    _dt(loc, torch.uint8, "loc"); _dt(qhat, torch.float32, "qhat")
+    rc = lib().ordermoe_layer_forward(ctypes.byref(desc), T, _host_or_dev_ptr(X, h),
+                                      _host_or_dev_ptr(home, h), _host_or_dev_ptr(loc, h),
+                                      _host_or_dev_ptr(qhat, h), _host_or_dev_ptr(y, h),
+                                      _ptr(counters), int(host_io), _stream(stream))
+    _check("ordermoe_layer_forward", rc)

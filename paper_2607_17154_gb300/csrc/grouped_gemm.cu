@@ -19,6 +19,7 @@
 // Every wait is bounded (globaltimer); a wait that runs out reports
 // ORDERMOE_DEV_WAIT_TIMEOUT, makes the other roles stop, drains the copies
 // and MMAs in flight (bounded too), frees TMEM and returns.
+#include <initializer_list>
 #include <mutex>
 
 #include "common.cuh"
@@ -62,10 +63,13 @@ struct Smem {
 };
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + static_cast<int>(sizeof(Smem));
 
-enum { GATEUP = 0, DOWN = 1 };
+enum { GATEUP = 0, DOWN = 1, LOGITS = 2 };
 
 struct Args {
-  const int32_t* offsets;
+  const int32_t* offsets;  // [E+1] row ranges; null: one group of `rows` rows
+  int rows;
+  int n_valid;       // LOGITS: number of valid output columns
+  float* out_f32;    // LOGITS: H [rows][n_valid] fp32
   int E;
   int K;             // reduction length
   int n_tiles;       // N slices per expert
@@ -118,7 +122,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     s.zero = 0;
     int acc = 0;
     for (int e = 0; e <= args.E; ++e) {
-      const int o = args.offsets[e];
+      const int o = args.offsets ? args.offsets[e] : (e == 0 ? 0 : args.rows);
       s.offs[e] = o;
       if (e > 0) {
         const int rows = o - s.offs[e - 1];
@@ -155,7 +159,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t phase = 0;
       for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x) {
         const Tile t = decode(tile, s, args.E, args.n_tiles);
-        const int brow = t.e * args.b_rows + t.n * (MODE == GATEUP ? 128 : 256);
+        const int brow = t.e * args.b_rows + t.n * (MODE == GATEUP ? 128 : 256);  // LOGITS: e == 0
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
             if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 1);
@@ -263,6 +267,31 @@ __global__ void __launch_bounds__(THREADS, 1)
               dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
           }
         }
+      } else if (MODE == LOGITS) {
+        const int col0 = t.n * 256;
+        float* orow = args.out_f32 + (size_t)row * args.n_valid;
+        const bool vec = (args.n_valid & 3) == 0;
+#pragma unroll 1
+        for (int c = 0; c < 8; ++c) {
+          if (col0 + c * 32 >= args.n_valid) break;  // warp-uniform
+          uint32_t v[32];
+          tmem_ld32(tb + c * 32, v);
+          tmem_ld_wait();
+          if (valid) {
+            const int cb = col0 + c * 32;
+            if (vec && cb + 32 <= args.n_valid) {
+              float4* dst = reinterpret_cast<float4*>(orow + cb);
+#pragma unroll
+              for (int i = 0; i < 8; ++i)
+                dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
+                                     __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (cb + i < args.n_valid) orow[cb + i] = __uint_as_float(v[i]);
+            }
+          }
+        }
       } else {
         uint16_t* orow = args.out + (size_t)row * args.ldo + t.n * 256;
 #pragma unroll 1
@@ -345,9 +374,7 @@ int make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols) {
 
 }  // namespace gg
 
-int ffn_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const uint16_t* W1,
-               const uint16_t* W3, const uint16_t* W2, int E, int d, int dff, uint16_t* H,
-               uint16_t* Y, cudaStream_t stream) {
+static int ffn_attrs() {
   using namespace gg;
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
@@ -359,31 +386,89 @@ int ffn_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const uint
                                       cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   });
   if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(ffn_gemm_kernel)");
-  CUtensorMap mX, mW1, mW3, mH, mW2;
+  return ORDERMOE_OK;
+}
+
+// H = SwiGLU(X_perm W1^T, X_perm W3^T) over the expert row ranges.
+int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const uint16_t* W1,
+                   const uint16_t* W3, int E, int d, int dff, uint16_t* H, cudaStream_t stream) {
+  using namespace gg;
   int rc;
+  if ((rc = ffn_attrs())) return rc;
+  CUtensorMap mX, mW1, mW3;
   if ((rc = make_map(&mX, X_perm, R, d))) return rc;
   if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
   if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
-  if ((rc = make_map(&mH, H, R, dff))) return rc;
-  if ((rc = make_map(&mW2, W2, (uint64_t)E * d, dff))) return rc;
-  const int sms = num_sms();
-  const long long mt_max = (R + BM - 1) / BM + E;
   Args a{};
-  a.offsets = offsets;
-  a.E = E;
-  a.limit_ns = wait_limit_ns();
-  // gate/up
+  a.offsets = offsets; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = d; a.n_tiles = dff / 128; a.b_rows = dff; a.out = H; a.ldo = dff;
-  long long tiles = mt_max * a.n_tiles;
-  int grid = static_cast<int>(tiles < sms ? tiles : sms);
+  const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
+  const int sms = num_sms();
+  const int grid = static_cast<int>(tiles < sms ? tiles : sms);
   ffn_gemm_kernel<GATEUP><<<grid, THREADS, SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
   OM_LAUNCHED("ffn_gemm_kernel<gate_up>");
-  // down
+  return ORDERMOE_OK;
+}
+
+// Y_perm = H W2^T over the expert row ranges.
+int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t* W2, int E, int d,
+                int dff, uint16_t* Y, cudaStream_t stream) {
+  using namespace gg;
+  int rc;
+  if ((rc = ffn_attrs())) return rc;
+  CUtensorMap mH, mW2;
+  if ((rc = make_map(&mH, H, R, dff))) return rc;
+  if ((rc = make_map(&mW2, W2, (uint64_t)E * d, dff))) return rc;
+  Args a{};
+  a.offsets = offsets; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = dff; a.n_tiles = d / 256; a.b_rows = d; a.out = Y; a.ldo = d;
-  tiles = mt_max * a.n_tiles;
-  grid = static_cast<int>(tiles < sms ? tiles : sms);
+  const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
+  const int sms = num_sms();
+  const int grid = static_cast<int>(tiles < sms ? tiles : sms);
   ffn_gemm_kernel<DOWN><<<grid, THREADS, SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
   OM_LAUNCHED("ffn_gemm_kernel<down>");
+  return ORDERMOE_OK;
+}
+
+int ffn_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const uint16_t* W1,
+               const uint16_t* W3, const uint16_t* W2, int E, int d, int dff, uint16_t* H,
+               uint16_t* Y, cudaStream_t stream) {
+  int rc = gate_up_launch(X_perm, offsets, R, W1, W3, E, d, dff, H, stream);
+  if (rc) return rc;
+  return down_launch(H, offsets, R, W2, E, d, dff, Y, stream);
+}
+
+// H[n][c] = sum_k X[n][k] W[c][k] in fp32 for n < N, c < C (C = L*E stacked
+// router rows): the router-logit contraction of Eq. 3 over calibration tokens.
+int logits_gemm_launch(const uint16_t* X, int N, const uint16_t* W, int C, int d, float* H,
+                       cudaStream_t stream) {
+  using namespace gg;
+  static std::once_flag attr_once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(attr_once, [] {
+    attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<LOGITS>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(logits)");
+  CUtensorMap mX, mW;
+  int rc;
+  if ((rc = make_map(&mX, X, N, d))) return rc;
+  if ((rc = make_map(&mW, W, C, d))) return rc;
+  Args a{};
+  a.offsets = nullptr;
+  a.rows = N;
+  a.n_valid = C;
+  a.out_f32 = H;
+  a.E = 1;
+  a.K = d;
+  a.n_tiles = (C + 255) / 256;
+  a.b_rows = 0;
+  a.limit_ns = wait_limit_ns();
+  const long long tiles = (long long)((N + BM - 1) / BM) * a.n_tiles;
+  const int sms = num_sms();
+  const int grid = static_cast<int>(tiles < sms ? tiles : sms);
+  ffn_gemm_kernel<LOGITS><<<grid, THREADS, SMEM_BYTES, stream>>>(mX, mW, mW, a);
+  OM_LAUNCHED("ffn_gemm_kernel<logits>");
   return ORDERMOE_OK;
 }
 
@@ -414,21 +499,49 @@ int selftest_wait_timeout(uint64_t limit_ns, cudaStream_t stream) {
 
 using namespace om;
 
+static int ffn_check(const char* who, int R, int E, int d, int dff) {
+  if (R < 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "%s: need R >= 0 and 1 <= E <= 64", who);
+  if (d <= 0 || d % 256 != 0 || dff <= 0 || dff % 128 != 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "%s: need d %% 256 == 0 and dff %% 128 == 0", who);
+  if ((long long)E * dff > INT32_MAX || (long long)E * d > INT32_MAX || (long long)R * dff > INT32_MAX * 4LL)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "%s: sizes too large", who);
+  return ORDERMOE_OK;
+}
+
+static bool all_aligned(std::initializer_list<const void*> ps) {
+  for (const void* p : ps)
+    if (!p || !aligned16(p)) return false;
+  return true;
+}
+
 extern "C" int ordermoe_expert_ffn(const uint16_t* X_perm, const int32_t* offsets, int R,
                                    const uint16_t* W1, const uint16_t* W3, const uint16_t* W2,
                                    int E, int d, int dff, uint16_t* H, uint16_t* Y_perm,
                                    ordermoe_stream_t stream) {
-  if (R < 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS)
-    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_ffn: need R >= 0 and 1 <= E <= 64");
-  if (d <= 0 || d % 256 != 0 || dff <= 0 || dff % 128 != 0)
-    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_ffn: need d %% 256 == 0 and dff %% 128 == 0");
-  if (R == 0) return ORDERMOE_OK;
-  if (!X_perm || !offsets || !W1 || !W3 || !W2 || !H || !Y_perm)
-    return fail(ORDERMOE_ERR_INVALID_ARG, "expert_ffn: null pointer");
-  if (!aligned16(X_perm) || !aligned16(W1) || !aligned16(W3) || !aligned16(W2) || !aligned16(H) ||
-      !aligned16(Y_perm))
-    return fail(ORDERMOE_ERR_INVALID_ARG, "expert_ffn: pointers must be 16-byte aligned");
-  if ((long long)E * dff > INT32_MAX || (long long)E * d > INT32_MAX)
-    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_ffn: weight rows exceed 2^31");
+  int rc = ffn_check("expert_ffn", R, E, d, dff);
+  if (rc || R == 0) return rc;
+  if (!offsets || !all_aligned({X_perm, W1, W3, W2, H, Y_perm}))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "expert_ffn: null or not 16-byte aligned pointer");
   return ffn_launch(X_perm, offsets, R, W1, W3, W2, E, d, dff, H, Y_perm, stream);
+}
+
+extern "C" int ordermoe_expert_gate_up(const uint16_t* X_perm, const int32_t* offsets, int R,
+                                       const uint16_t* W1, const uint16_t* W3, int E, int d, int dff,
+                                       uint16_t* H, ordermoe_stream_t stream) {
+  int rc = ffn_check("expert_gate_up", R, E, d, dff);
+  if (rc || R == 0) return rc;
+  if (!offsets || !all_aligned({X_perm, W1, W3, H}))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "expert_gate_up: null or not 16-byte aligned pointer");
+  return gate_up_launch(X_perm, offsets, R, W1, W3, E, d, dff, H, stream);
+}
+
+extern "C" int ordermoe_expert_down(const uint16_t* H, const int32_t* offsets, int R,
+                                    const uint16_t* W2, int E, int d, int dff, uint16_t* Y_perm,
+                                    ordermoe_stream_t stream) {
+  int rc = ffn_check("expert_down", R, E, d, dff);
+  if (rc || R == 0) return rc;
+  if (!offsets || !all_aligned({H, W2, Y_perm}))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "expert_down: null or not 16-byte aligned pointer");
+  return down_launch(H, offsets, R, W2, E, d, dff, Y_perm, stream);
 }

@@ -1,0 +1,145 @@
+// One MoE layer forward through the hot path: route_select -> dispatch ->
+// expert gate/up -> expert down -> combine, with its scratch carved from one
+// caller-provided buffer. With host_io the inputs are copied host -> device
+// and the output device -> host on the same stream.
+#include "common.cuh"
+
+namespace om {
+int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int E, int d,
+                    int32_t* offsets, int32_t* row_token, int32_t* row_of, uint16_t* X_perm,
+                    int32_t* hist, cudaStream_t stream);
+size_t dispatch_workspace_bytes(int64_t n, int E);
+
+struct LayerScratch {
+  int32_t *topk_idx, *chosen, *offsets, *row_token, *row_of, *hist;
+  float *topk_w, *qhat;
+  uint8_t *server, *kind, *loc, *home;
+  uint16_t *X_perm, *H, *Y_perm, *X, *y;
+  size_t bytes;
+};
+
+static size_t up256(size_t v) { return (v + 255) & ~size_t(255); }
+
+// Carves the scratch; with base == nullptr only computes its size.
+static LayerScratch carve(uint8_t* base, int T, int E, int d, int dff, int k) {
+  LayerScratch s{};
+  size_t off = 0;
+  const size_t R = (size_t)T * k;
+  auto take = [&](size_t bytes) {
+    uint8_t* p = base ? base + off : nullptr;
+    off += up256(bytes);
+    return p;
+  };
+  s.topk_idx = reinterpret_cast<int32_t*>(take(R * 4));
+  s.topk_w = reinterpret_cast<float*>(take(R * 4));
+  s.chosen = reinterpret_cast<int32_t*>(take(R * 4));
+  s.server = take(R);
+  s.kind = take(R);
+  s.offsets = reinterpret_cast<int32_t*>(take((E + 1) * 4));
+  s.row_token = reinterpret_cast<int32_t*>(take(R * 4));
+  s.row_of = reinterpret_cast<int32_t*>(take(R * 4));
+  s.hist = reinterpret_cast<int32_t*>(take(dispatch_workspace_bytes((int64_t)R, E)));
+  s.X_perm = reinterpret_cast<uint16_t*>(take(R * d * 2));
+  s.H = reinterpret_cast<uint16_t*>(take(R * dff * 2));
+  s.Y_perm = reinterpret_cast<uint16_t*>(take(R * d * 2));
+  s.loc = take(T);
+  s.qhat = reinterpret_cast<float*>(take((size_t)T * 4));
+  s.home = take(T);
+  s.X = reinterpret_cast<uint16_t*>(take((size_t)T * d * 2));
+  s.y = reinterpret_cast<uint16_t*>(take((size_t)T * d * 2));
+  s.bytes = off;
+  return s;
+}
+
+int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const uint16_t* W1,
+                   const uint16_t* W3, int E, int d, int dff, uint16_t* H, cudaStream_t stream);
+int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t* W2, int E, int d,
+                int dff, uint16_t* Y, cudaStream_t stream);
+
+}  // namespace om
+
+using namespace om;
+
+extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, const float* logits_in,
+                                     int T, int E, int d, int k, int renorm, const void* tables,
+                                     size_t tables_bytes_, const uint8_t* home, uint8_t* loc,
+                                     float* qhat, float* logits_out, int32_t* topk_idx,
+                                     float* topk_w, int32_t* chosen_expert,
+                                     uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
+                                     ordermoe_stream_t stream);
+extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,
+                                const float* topk_w, int T, int k, int d, uint16_t* y,
+                                ordermoe_stream_t stream);
+
+extern "C" size_t ordermoe_layer_scratch_bytes(int T_max, int E, int d, int dff, int k) {
+  if (T_max <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || d <= 0 || dff <= 0 || k <= 0 ||
+      k > ORDERMOE_MAX_TOPK)
+    return 0;
+  return carve(nullptr, T_max, E, d, dff, k).bytes;
+}
+
+extern "C" int ordermoe_layer_forward(const ordermoe_layer_desc* L, int T, const uint16_t* X,
+                                      const uint8_t* home, uint8_t* loc, float* qhat, uint16_t* y,
+                                      int32_t* counters, int host_io, ordermoe_stream_t stream) {
+  if (!L) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: null layer");
+  if (T < 0 || T > L->T_max) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: need 0 <= T <= T_max");
+  if (!L->W_r || !L->W1 || !L->W3 || !L->W2 || !L->tables || !L->scratch)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: null pointer in the layer");
+  if ((reinterpret_cast<uintptr_t>(L->scratch) & 255u) != 0)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: scratch must be 256-byte aligned");
+  const size_t need = ordermoe_layer_scratch_bytes(L->T_max, L->E, L->d, L->dff, L->k);
+  if (need == 0 || L->scratch_bytes < need)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: scratch too small or bad shape");
+  if (L->d % 256 != 0 || L->dff % 128 != 0 || L->k > L->E)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "layer_forward: need d %% 256 == 0, dff %% 128 == 0, k <= E");
+  if (!aligned16(L->W_r) || !aligned16(L->W1) || !aligned16(L->W3) || !aligned16(L->W2))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: weights must be 16-byte aligned");
+  if (T == 0) return ORDERMOE_OK;
+  if (!X || !home || !y) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: null X/home/y");
+  if ((loc == nullptr) != (qhat == nullptr))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: give both loc and qhat, or neither");
+  const int E = L->E, d = L->d, dff = L->dff, k = L->k, R = T * k;
+  LayerScratch s = carve(static_cast<uint8_t*>(L->scratch), L->T_max, E, d, dff, k);
+  cudaStream_t st = stream;
+  const uint16_t* Xd = X;
+  const uint8_t* homed = home;
+  uint8_t* locd = loc;
+  float* qd = qhat;
+  uint16_t* yd = y;
+  if (!host_io && (!aligned16(X) || !aligned16(y)))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: X and y must be 16-byte aligned");
+  if (host_io) {
+    OM_CUDA(cudaMemcpyAsync(s.X, X, (size_t)T * d * 2, cudaMemcpyHostToDevice, st));
+    OM_CUDA(cudaMemcpyAsync(s.home, home, (size_t)T, cudaMemcpyHostToDevice, st));
+    Xd = s.X;
+    homed = s.home;
+    yd = s.y;
+    if (loc) {
+      OM_CUDA(cudaMemcpyAsync(s.loc, loc, (size_t)T, cudaMemcpyHostToDevice, st));
+      OM_CUDA(cudaMemcpyAsync(s.qhat, qhat, (size_t)T * 4, cudaMemcpyHostToDevice, st));
+      locd = s.loc;
+      qd = s.qhat;
+    }
+  }
+  int rc = ordermoe_route_select(Xd, L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
+                                 L->tables_bytes, homed, locd, qd, nullptr, s.topk_idx, s.topk_w,
+                                 s.chosen, s.server, s.kind, counters, stream);
+  if (rc) return rc;
+  rc = dispatch_launch(s.chosen, Xd, T, k, E, d, s.offsets, s.row_token, s.row_of, s.X_perm,
+                       s.hist, st);
+  if (rc) return rc;
+  rc = gate_up_launch(s.X_perm, s.offsets, R, L->W1, L->W3, E, d, dff, s.H, st);
+  if (rc) return rc;
+  rc = down_launch(s.H, s.offsets, R, L->W2, E, d, dff, s.Y_perm, st);
+  if (rc) return rc;
+  rc = ordermoe_combine(s.Y_perm, s.row_of, s.topk_w, T, k, d, yd, stream);
+  if (rc) return rc;
+  if (host_io) {
+    OM_CUDA(cudaMemcpyAsync(y, s.y, (size_t)T * d * 2, cudaMemcpyDeviceToHost, st));
+    if (loc) {
+      OM_CUDA(cudaMemcpyAsync(loc, s.loc, (size_t)T, cudaMemcpyDeviceToHost, st));
+      OM_CUDA(cudaMemcpyAsync(qhat, s.qhat, (size_t)T * 4, cudaMemcpyDeviceToHost, st));
+    }
+  }
+  return ORDERMOE_OK;
+}

@@ -243,13 +243,13 @@ __global__ void __launch_bounds__(256) route_select_kernel(
 
     // selection
     const int a = home[t];
-    const int s = loc[t];
+    const int s = (loc != nullptr) ? loc[t] : a;  // no state given: first layer (Eq. 36)
     if (a >= M || s >= M) {
       if (lane == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
       continue;
     }
     const float* Aas = gA + ((size_t)a * M + s) * M;
-    float q = qhat[t];
+    float q = (qhat != nullptr) ? qhat[t] : 0.0f;
     unsigned long long taken = used_targets;
     int first_server = s;
     for (int j = 0; j < k; ++j) {
@@ -306,7 +306,7 @@ __global__ void __launch_bounds__(256) route_select_kernel(
       }
       kind_count[kd]++;
     }
-    if (lane == 0) {
+    if (lane == 0 && loc != nullptr) {
       loc[t] = static_cast<uint8_t>(first_server);
       qhat[t] = q;
     }
@@ -363,9 +363,10 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
   if (T < 0) return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: T < 0");
   if (E <= 0 || E > ORDERMOE_MAX_EXPERTS || k <= 0 || k > ORDERMOE_MAX_TOPK || k > E)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select: need 1 <= k <= min(E, 8), E <= 64");
-  if (!tables || !home || !loc || !qhat || !topk_idx || !topk_w || !chosen_expert ||
-      !chosen_server || !kind)
+  if (!tables || !home || !topk_idx || !topk_w || !chosen_expert || !chosen_server || !kind)
     return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: null pointer");
+  if ((loc == nullptr) != (qhat == nullptr))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: give both loc and qhat, or neither");
   if (logits_in == nullptr) {
     if (!X || !W_r) return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: X/W_r null without logits_in");
     if (d <= 0 || d % 8 != 0)

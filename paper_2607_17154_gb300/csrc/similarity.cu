@@ -1,0 +1,344 @@
+// Offline planning on the GPU (Section IV, Alg. 1 grouping and placement):
+//   ordermoe_similarity: H = W_r X_cal^T (Eq. 3, tcgen05 GEMM into scratch),
+//     Sim = cosine of the rows of H (Eq. 4), activation counts n_j (Eq. 5);
+//   ordermoe_expert_counts: the counts of Eq. 5 from given logits;
+//   ordermoe_place: threshold (Eq. 6), greedy grouping (Eqs. 24-26),
+//     importance (Eqs. 27-28) and mandatory placement (Eqs. 29-31).
+#include "common.cuh"
+
+namespace om {
+
+int logits_gemm_launch(const uint16_t* X, int N, const uint16_t* W, int C, int d, float* H,
+                       cudaStream_t stream);
+
+static __device__ unsigned long long g_err_sim = 0;
+
+int read_clear_err_sim(unsigned long long* out) {
+  unsigned long long zero = 0;
+  OM_CUDA(cudaMemcpyFromSymbol(out, g_err_sim, sizeof(*out)));
+  OM_CUDA(cudaMemcpyToSymbol(g_err_sim, &zero, sizeof(zero)));
+  return ORDERMOE_OK;
+}
+
+constexpr int kSimChunk = 1024;  // calibration tokens per partial Gram
+constexpr int kSub = 32;         // tokens staged in shared memory at a time
+
+// Rank order used for top-k: larger logit first, equal logits by lower index.
+__device__ __forceinline__ void add_topk_counts(const float* l, int E, int kf, int* counts) {
+  unsigned long long used = 0;
+  for (int j = 0; j < kf; ++j) {
+    int best = -1;
+    float bv = 0.0f;
+    for (int e = 0; e < E; ++e) {
+      if ((used >> e) & 1ull) continue;
+      if (best < 0 || l[e] > bv) { best = e; bv = l[e]; }
+    }
+    used |= 1ull << best;
+    atomicAdd(&counts[best], 1);
+  }
+}
+
+// grid (chunks, L), 256 threads. Partial Gram of layer l over the tokens of
+// one chunk: thread (i, jb) accumulates G[i][16 jb .. 16 jb + 15] in fp32.
+__global__ void __launch_bounds__(256) gram_counts_kernel(const float* __restrict__ H, int64_t N,
+                                                          int L, int E, int kf,
+                                                          float* __restrict__ gpart,
+                                                          int32_t* __restrict__ cpart) {
+  __shared__ float sh[kSub][65];
+  __shared__ int cnt[64];
+  const int chunk = blockIdx.x, l = blockIdx.y;
+  const int nchunks = gridDim.x;
+  const int tid = threadIdx.x;
+  const int i = tid >> 2, j0 = (tid & 3) * 16;
+  const int LE = L * E;
+  float acc[16];
+#pragma unroll
+  for (int q = 0; q < 16; ++q) acc[q] = 0.0f;
+  if (tid < 64) cnt[tid] = 0;
+  const int64_t n_begin = (int64_t)chunk * kSimChunk;
+  int64_t n_end = n_begin + kSimChunk;
+  if (n_end > N) n_end = N;
+  for (int64_t n0 = n_begin; n0 < n_end; n0 += kSub) {
+    __syncthreads();
+    for (int x = tid; x < kSub * E; x += 256) {
+      const int r = x / E, c = x % E;
+      const int64_t n = n0 + r;
+      sh[r][c] = (n < n_end) ? H[n * LE + (int64_t)l * E + c] : 0.0f;
+    }
+    __syncthreads();
+    if (i < E) {
+      for (int r = 0; r < kSub; ++r) {
+        const float a = sh[r][i];
+#pragma unroll
+        for (int q = 0; q < 16; ++q) acc[q] = fmaf(a, sh[r][j0 + q], acc[q]);
+      }
+    }
+    if (tid < kSub && n0 + tid < n_end) add_topk_counts(&sh[tid][0], E, kf, cnt);
+  }
+  __syncthreads();
+  float* gp = gpart + ((size_t)l * nchunks + chunk) * 64 * 64;
+  if (i < E)
+#pragma unroll
+    for (int q = 0; q < 16; ++q) gp[i * 64 + j0 + q] = acc[q];
+  if (tid < E) cpart[((size_t)l * nchunks + chunk) * 64 + tid] = cnt[tid];
+}
+
+// grid L, 256 threads: G = sum of the partial Grams in chunk order (fp64),
+// Sim(i,j) = G_ij / (sqrt(G_ii) sqrt(G_jj)) (Eq. 4), diagonal 1, zero-norm 0.
+__global__ void __launch_bounds__(256) sim_finish_kernel(const float* __restrict__ gpart,
+                                                         const int32_t* __restrict__ cpart,
+                                                         int nchunks, int E, float* __restrict__ sim,
+                                                         int32_t* __restrict__ counts) {
+  __shared__ double G[64 * 64];
+  const int l = blockIdx.x;
+  for (int x = threadIdx.x; x < E * E; x += blockDim.x) {
+    const int i = x / E, j = x % E;
+    double s = 0.0;
+    for (int c = 0; c < nchunks; ++c)
+      s += static_cast<double>(gpart[((size_t)l * nchunks + c) * 4096 + i * 64 + j]);
+    G[i * 64 + j] = s;
+  }
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int s = 0;
+    for (int c = 0; c < nchunks; ++c) s += cpart[((size_t)l * nchunks + c) * 64 + e];
+    counts[(size_t)l * E + e] = s;
+  }
+  __syncthreads();
+  for (int x = threadIdx.x; x < E * E; x += blockDim.x) {
+    const int i = x / E, j = x % E;
+    float v;
+    if (i == j) {
+      v = 1.0f;
+    } else {
+      const double ni = sqrt(G[i * 64 + i]), nj = sqrt(G[j * 64 + j]);
+      v = (ni == 0.0 || nj == 0.0) ? 0.0f : __double2float_rn(G[i * 64 + j] / (ni * nj));
+    }
+    sim[(size_t)l * E * E + x] = v;
+  }
+}
+
+__global__ void counts_from_logits_kernel(const float* __restrict__ logits, int64_t N, int E,
+                                          int kf, int32_t* __restrict__ counts) {
+  __shared__ int cnt[64];
+  if (threadIdx.x < 64) cnt[threadIdx.x] = 0;
+  __syncthreads();
+  for (int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; n < N;
+       n += (int64_t)gridDim.x * blockDim.x) {
+    float l[64];
+    for (int e = 0; e < E; ++e) l[e] = logits[n * E + e];
+    add_topk_counts(l, E, kf, cnt);
+  }
+  __syncthreads();
+  if (threadIdx.x < E && cnt[threadIdx.x]) atomicAdd(&counts[threadIdx.x], cnt[threadIdx.x]);
+}
+
+// ---------------------------------------------------------------------------
+// Grouping and placement: one block of 64 threads, layers in order. Thread e
+// owns expert e in the parallel parts; the greedy loops are sequential in the
+// paper's order. fp64 arithmetic uses explicit round-to-nearest operations.
+struct PlaceParams {
+  double theta_min, theta_max, theta_single;
+  double alpha_f, alpha_r, lambda1, lambda2;
+};
+
+__global__ void __launch_bounds__(64) place_kernel(
+    const float* __restrict__ sim, const int32_t* __restrict__ counts, int L, int E, int M,
+    PlaceParams pp, const double* __restrict__ p, const double* __restrict__ C,
+    int32_t* __restrict__ group, int32_t* __restrict__ n_groups, float* __restrict__ theta_out,
+    uint8_t* __restrict__ placement, double* __restrict__ used, int32_t* __restrict__ status) {
+  __shared__ double b[32];
+  __shared__ double imp[64];
+  __shared__ int order[64];
+  __shared__ int dom[64];
+  __shared__ int grp[64];
+  __shared__ int waiting[64];
+  __shared__ int overflow;
+  const int t = threadIdx.x;
+  if (t < M) b[t] = 0.0;
+  if (t == 0) {
+    double need = 0.0, have = 0.0;
+    for (int i = 0; i < L * E; ++i) need = __dadd_rn(need, p[i]);
+    for (int m = 0; m < M; ++m) have = __dadd_rn(have, C[m]);
+    overflow = need > have ? 1 : 0;
+  }
+  __syncthreads();
+  for (int l = 0; l < L; ++l) {
+    const float* S = sim + (size_t)l * E * E;
+    const int32_t* cn = counts + (size_t)l * E;
+    const double* pl = p + (size_t)l * E;
+    uint8_t* x = placement + (size_t)l * M * E;
+    // Eq. 6 (layers numbered from 1)
+    float theta;
+    if (L <= 1) {
+      theta = __double2float_rn(pp.theta_single);
+    } else {
+      const double frac = __ddiv_rn(static_cast<double>(L - (l + 1)), static_cast<double>(L - 1));
+      theta = __double2float_rn(
+          __dadd_rn(pp.theta_min, __dmul_rn(__dsub_rn(pp.theta_max, pp.theta_min), frac)));
+    }
+    // visiting order: count desc, index asc
+    if (t < E) {
+      int r = 0;
+      for (int e = 0; e < E; ++e)
+        if (cn[e] > cn[t] || (cn[e] == cn[t] && e < t)) ++r;
+      order[r] = t;
+    }
+    for (int i = t; i < M * E; i += blockDim.x) x[i] = 0;
+    __syncthreads();
+    // Eqs. 24-26, sequential in the visiting order
+    if (t == 0) {
+      int k = 0;
+      for (int pos = 0; pos < E; ++pos) {
+        const int j = order[pos];
+        int bg = -1;
+        float bs = 0.0f;
+        for (int g = 0; g < k; ++g) {
+          const float s = S[j * E + dom[g]];
+          if (bg < 0 || s > bs) { bg = g; bs = s; }
+        }
+        if (bg < 0 || bs < theta) { dom[k] = j; grp[j] = k; ++k; }
+        else grp[j] = bg;
+      }
+      n_groups[l] = k;
+      theta_out[l] = theta;
+    }
+    __syncthreads();
+    // Eqs. 27-28
+    double total = 0.0;
+    for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cn[e]));
+    if (t < E) {
+      group[(size_t)l * E + t] = grp[t];
+      double s = 0.0;
+      int size = 0;
+      for (int k2 = 0; k2 < E; ++k2)
+        if (grp[k2] == grp[t]) { s = __dadd_rn(s, static_cast<double>(S[t * E + k2])); ++size; }
+      const double rho = __ddiv_rn(s, static_cast<double>(size));
+      const double f = total > 0.0 ? __ddiv_rn(static_cast<double>(cn[t]), total) : 0.0;
+      imp[t] = __dadd_rn(__dmul_rn(pp.alpha_f, f), __dmul_rn(pp.alpha_r, rho));
+    }
+    __syncthreads();
+    // placement order: p desc, I desc, index asc
+    if (t < E) {
+      int r = 0;
+      for (int e = 0; e < E; ++e) {
+        bool before;
+        if (pl[e] != pl[t]) before = pl[e] > pl[t];
+        else if (imp[e] != imp[t]) before = imp[e] > imp[t];
+        else before = e < t;
+        if (before) ++r;
+      }
+      order[r] = t;
+    }
+    __syncthreads();
+    // Eqs. 29-31, sequential; waiting list to the server with the most room
+    if (t == 0) {
+      int nw = 0;
+      for (int pos = 0; pos < E; ++pos) {
+        const int j = order[pos];
+        int best = -1;
+        double bsc = 0.0;
+        for (int m = 0; m < M; ++m) {
+          if (!(__dadd_rn(b[m], pl[j]) <= C[m])) continue;
+          int eta = 0;
+          for (int k2 = 0; k2 < E; ++k2)
+            if (grp[k2] == grp[j] && x[m * E + k2]) ++eta;
+          const double sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[m], C[m])),
+                                      __dmul_rn(pp.lambda2, static_cast<double>(eta)));
+          if (best < 0 || sc < bsc) { best = m; bsc = sc; }
+        }
+        if (best < 0) { waiting[nw++] = j; continue; }
+        x[best * E + j] = 1;
+        b[best] = __dadd_rn(b[best], pl[j]);
+      }
+      for (int w = 0; w < nw; ++w) {
+        const int j = waiting[w];
+        int best = 0;
+        for (int m = 1; m < M; ++m)
+          if (__dsub_rn(C[m], b[m]) > __dsub_rn(C[best], b[best])) best = m;
+        x[best * E + j] = 1;
+        b[best] = __dadd_rn(b[best], pl[j]);
+        if (b[best] > C[best]) overflow = 1;
+      }
+    }
+    __syncthreads();
+  }
+  if (t < M) used[t] = b[t];
+  if (t == 0) *status = overflow ? ORDERMOE_ERR_CAPACITY : ORDERMOE_OK;
+}
+
+}  // namespace om
+
+using namespace om;
+
+extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
+  if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || N <= 0) return 0;
+  const int64_t nchunks = (N + kSimChunk - 1) / kSimChunk;
+  const size_t h = (size_t)N * L * E * sizeof(float);
+  const size_t g = (size_t)L * nchunks * 64 * 64 * sizeof(float);
+  const size_t c = (size_t)L * nchunks * 64 * sizeof(int32_t);
+  auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
+  return up(h) + up(g) + up(c);
+}
+
+extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
+                                   int64_t N, int k_freq, float* sim, int32_t* counts,
+                                   void* workspace, size_t workspace_bytes,
+                                   ordermoe_stream_t stream) {
+  if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: need L >= 1, 1 <= k_freq <= E <= 64");
+  if (d <= 0 || d % 64 != 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: d must be a positive multiple of 64");
+  if (N <= 0 || N > INT32_MAX || (int64_t)L * E > INT32_MAX)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: bad N");
+  if (!W_r || !X_cal || !sim || !counts || !workspace)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: null pointer");
+  if (!aligned16(W_r) || !aligned16(X_cal) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: W_r/X_cal 16-byte and workspace 256-byte aligned");
+  if (workspace_bytes < ordermoe_similarity_workspace_bytes(L, E, N))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: workspace too small");
+  const int nchunks = static_cast<int>((N + kSimChunk - 1) / kSimChunk);
+  auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  float* H = reinterpret_cast<float*>(ws);
+  float* gpart = reinterpret_cast<float*>(ws + up((size_t)N * L * E * sizeof(float)));
+  int32_t* cpart = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(gpart) +
+                                              up((size_t)L * nchunks * 64 * 64 * sizeof(float)));
+  int rc = logits_gemm_launch(X_cal, static_cast<int>(N), W_r, L * E, d, H, stream);
+  if (rc) return rc;
+  gram_counts_kernel<<<dim3(nchunks, L), 256, 0, stream>>>(H, N, L, E, k_freq, gpart, cpart);
+  OM_LAUNCHED("gram_counts_kernel");
+  sim_finish_kernel<<<L, 256, 0, stream>>>(gpart, cpart, nchunks, E, sim, counts);
+  OM_LAUNCHED("sim_finish_kernel");
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq,
+                                      int32_t* counts, ordermoe_stream_t stream) {
+  if (E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E || N < 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_counts: need 1 <= k_freq <= E <= 64");
+  if (!counts || (N > 0 && !logits)) return fail(ORDERMOE_ERR_INVALID_ARG, "expert_counts: null pointer");
+  OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * E, stream));
+  if (N == 0) return ORDERMOE_OK;
+  int64_t blocks = (N + 255) / 256;
+  if (blocks > num_sms() * 4) blocks = num_sms() * 4;
+  counts_from_logits_kernel<<<static_cast<int>(blocks), 256, 0, stream>>>(logits, N, E, k_freq, counts);
+  OM_LAUNCHED("counts_from_logits_kernel");
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, int E, int M,
+                              double theta_min, double theta_max, double theta_single,
+                              double alpha_f, double alpha_r, double lambda1, double lambda2,
+                              const double* p, const double* C, int32_t* group, int32_t* n_groups,
+                              float* theta, uint8_t* placement, double* used, int32_t* status,
+                              ordermoe_stream_t stream) {
+  if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 || M > ORDERMOE_MAX_SERVERS)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "place: need L >= 1, 1 <= E <= 64, 1 <= M <= 32");
+  if (!sim || !counts || !p || !C || !group || !n_groups || !theta || !placement || !used || !status)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "place: null pointer");
+  PlaceParams pp{theta_min, theta_max, theta_single, alpha_f, alpha_r, lambda1, lambda2};
+  place_kernel<<<1, 64, 0, stream>>>(sim, counts, L, E, M, pp, p, C, group, n_groups, theta,
+                                     placement, used, status);
+  OM_LAUNCHED("place_kernel");
+  return ORDERMOE_OK;
+}

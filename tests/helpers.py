@@ -42,8 +42,8 @@ def oracle_layer_tokens(tokens, X_bits, Wr_bits, W1, W3, W2, tab, home, loc, qha
     _, Y = oracle.ffn_rows(rows, chosen.reshape(-1).astype(np.int32), W1, W3, W2)
     row_of = np.arange(n * k, dtype=np.int32).reshape(n, k)
     y = oracle.combine(Y, row_of, w)
-    return dict(y=y, logits=logits, idx=idx, w=w, chosen=chosen, server=server, kind=kind,
-                loc=loc2, qhat=q2, margin=margin)
+    return dict(y=y, Y=Y.reshape(n, k, -1), logits=logits, idx=idx, w=w, chosen=chosen,
+                server=server, kind=kind, loc=loc2, qhat=q2, margin=margin)
 
 
 def assert_close_bf16(got_bits, ref_bits, rtol=2e-2, atol=1e-2, what=""):
@@ -55,3 +55,19 @@ def assert_close_bf16(got_bits, ref_bits, rtol=2e-2, atol=1e-2, what=""):
         raise AssertionError("%s: %d / %d elements outside rtol=%g atol=%g; first %s: got %s ref %s"
                              % (what, bad.sum(), bad.size, rtol, atol, i.tolist(),
                                 g[tuple(i.T)].tolist(), r[tuple(i.T)].tolist()))
+
+
+def assert_close_combined(got_bits, ref_bits, w, Yref_bits, rtol=2e-2, atol=1e-2, what="y"):
+    """Weighted-sum check: y = sum_j w_j Y_j is compared with a tolerance that
+    scales with sum_j |w_j| |Y_j| (the magnitude the rounding of each Y_j
+    carries into y), since the slots can cancel."""
+    g = bits_to_f(got_bits).astype(np.float64)
+    r = bits_to_f(ref_bits).astype(np.float64)
+    scale = np.einsum("tk,tkd->td", np.abs(w).astype(np.float64),
+                      np.abs(bits_to_f(Yref_bits).astype(np.float64)))
+    bad = np.abs(g - r) > atol + rtol * scale
+    if bad.any():
+        i = np.argwhere(bad)[:5]
+        raise AssertionError("%s: %d / %d elements outside the combine bound; first %s: got %s ref %s"
+                             % (what, bad.sum(), bad.size, i.tolist(), g[tuple(i.T)].tolist(),
+                                r[tuple(i.T)].tolist()))

@@ -8,7 +8,8 @@ import oracle
 from paper_2607_17154_gb300 import binding as B
 from paper_2607_17154_gb300 import synth
 from paper_2607_17154_gb300.layer import MoELayer, build_tables
-from tests.helpers import assert_close_bf16, bits_to_f, oracle_layer_tokens, oracle_plan
+from tests.helpers import (assert_close_bf16, assert_close_combined, bits_to_f,
+                           oracle_layer_tokens, oracle_plan)
 
 pytestmark = pytest.mark.gpu
 
@@ -248,15 +249,35 @@ def run_layer_check(w, seed, sample=None):
     ref = oracle_layer_tokens(toks, gbits(inp["X"]), gbits(inp["Wr"]), gbits(inp["W1"]),
                               gbits(inp["W3"]), gbits(inp["W2"]), o_tab, h, h.copy(),
                               np.zeros(w.T, np.float32), w.k)
-    clear = ref["margin"] > 1e-3          # top-k not decided by a near tie
-    assert clear.mean() > 0.9
-    got_y = gbits(y)[toks]
-    assert_close_bf16(got_y[clear], ref["y"][clear], what="y")
+    # Router logits: fp32 tensor/CUDA-core sums vs the oracle's fp64 sums.
+    g_logits = layer.logits.cpu().numpy()[toks]
+    np.testing.assert_allclose(g_logits, ref["logits"], rtol=1e-3, atol=2e-3)
+    # A top-k decision is unique when every gap around the k-th rank exceeds
+    # the logit disagreement (8x the largest one seen); near ties are checked
+    # for validity instead.
+    delta = max(8.0 * float(np.abs(g_logits - ref["logits"]).max()), 1e-6)
+    clear = ref["margin"] > delta
+    assert clear.mean() > 0.5, (clear.mean(), delta)
     for name, t in (("idx", layer.topk_idx), ("chosen", layer.chosen), ("server", layer.server),
                     ("kind", layer.kind)):
         np.testing.assert_array_equal(t.cpu().numpy()[toks][clear], ref[name][clear], err_msg=name)
     np.testing.assert_array_equal(loc.cpu().numpy()[toks][clear], ref["loc"][clear])
     np.testing.assert_array_equal(qhat.cpu().numpy()[toks][clear], ref["qhat"][clear])
+    # expert outputs (the rows each slot's expert produced), spec tolerance
+    row_of = layer.row_of.cpu().numpy()[toks]
+    Yg = gbits(layer.Y_perm)[row_of]                     # [n, k, d]
+    assert_close_bf16(Yg[clear], ref["Y"][clear], what="expert outputs Y")
+    assert_close_combined(gbits(y)[toks][clear], ref["y"][clear], ref["w"][clear], ref["Y"][clear])
+    # near ties: the GPU's rank order agrees with the oracle's logits within delta
+    gidx = layer.topk_idx.cpu().numpy()[toks]
+    for t in np.where(~clear)[0]:
+        lo = ref["logits"][t]
+        sel = gidx[t]
+        assert len(set(sel)) == w.k
+        assert all(lo[sel[j]] >= lo[sel[j + 1]] - delta for j in range(w.k - 1))
+        rest = np.setdiff1d(np.arange(w.E), sel)
+        if len(rest):
+            assert lo[sel[-1]] >= lo[rest].max() - delta
     # permutation invariants at this size
     off = layer.offsets.cpu().numpy(); ch = layer.chosen.cpu().numpy()
     np.testing.assert_array_equal(off, np.concatenate([[0], np.cumsum(np.bincount(ch.ravel(), minlength=w.E))]))
