@@ -171,6 +171,22 @@ int ordermoe_dispatch(const int32_t* chosen_expert, const uint16_t* X, int T, in
                       int32_t* offsets, int32_t* row_token, int32_t* row_of, uint16_t* X_perm,
                       void* workspace, size_t workspace_bytes, ordermoe_stream_t stream);
 
+/* The permutation of ordermoe_dispatch, same arguments and results, for
+ * callers that cannot give the library device memory: a plugin whose host
+ * framework owns every device allocation through its own pool, or a serving
+ * loop that may not call cudaMalloc once it runs. (The paper has no
+ * counterpart; it is an interface convenience.) Its scratch is a fixed
+ * 256 KB device array inside the library, present on every GPU that loads the
+ * library until the process exits, so T*k is limited to 262144 entries
+ * (larger calls fail with ORDERMOE_ERR_UNSUPPORTED_SHAPE). The array's device
+ * address is looked up on the first call made on each device: make that
+ * first call before any stream capture. All calls share the array, so calls
+ * that overlap on the GPU (other streams, other host threads) race; nothing
+ * in it needs clearing between calls. The call allocates nothing. */
+int ordermoe_dispatch_noalloc(const int32_t* chosen_expert, const uint16_t* X, int T, int k,
+                              int E, int d, int32_t* offsets, int32_t* row_token, int32_t* row_of,
+                              uint16_t* X_perm, ordermoe_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * Grouped SwiGLU expert FFN over the permuted rows (the Mixtral-style experts
  * of Section VI-A):

@@ -48,6 +48,7 @@ _SIGNATURES = {
     "ordermoe_expert_down": ([_P, _P, _I, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_layer_scratch_bytes": ([_I, _I, _I, _I, _I], _SZ),
     "ordermoe_layer_forward": ([_P, _I, _P, _P, _P, _P, _P, _P, _I, _P], _I),
+    "ordermoe_dispatch_noalloc": ([_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P], _I),
 }
 
 
@@ -284,3 +285,16 @@ def ordermoe_layer_forward(desc, T, X, home, loc, qhat, y, counters=None, host_i
                                       _host_or_dev_ptr(qhat, h), _host_or_dev_ptr(y, h),
                                       _ptr(counters), int(host_io), _stream(stream))
     _check("ordermoe_layer_forward", rc)
+
+
+def ordermoe_dispatch_noalloc(chosen_expert, X, T, k, E, d, offsets, row_token, row_of, X_perm,
+                              stream=None):
+    """ordermoe_dispatch without a workspace argument: for callers that cannot
+    allocate device memory (the library keeps a fixed 256 KB scratch array)."""
+    _dt(chosen_expert, torch.int32, "chosen_expert"); _dt(X, torch.bfloat16, "X")
+    _dt(offsets, torch.int32, "offsets"); _dt(row_token, torch.int32, "row_token")
+    _dt(row_of, torch.int32, "row_of"); _dt(X_perm, torch.bfloat16, "X_perm")
+    rc = lib().ordermoe_dispatch_noalloc(_ptr(chosen_expert), _ptr(X), T, k, E, d, _ptr(offsets),
+                                         _ptr(row_token), _ptr(row_of), _ptr(X_perm),
+                                         _stream(stream))
+    _check("ordermoe_dispatch_noalloc", rc)
