@@ -7,9 +7,10 @@
 //   2. chunk_scan: one block; for every expert the exclusive prefix of its
 //      count over chunks, plus the expert offsets (exclusive prefix over
 //      experts) -> base[chunk][e] = offsets[e] + entries of e in earlier chunks
-//   3. rank_gather: stable rank inside the chunk (per-warp match + per-warp
-//      counts), row = base + rank; then each warp copies its 32 rows of X into
-//      X_perm with 16-byte loads and stores.
+//   3. rank: stable rank inside the chunk (per-warp match + per-warp
+//      counts), row = base + rank;
+//   4. gather_rows: one warp per permuted row copies X[row_token[row]] into
+//      X_perm with 16-byte loads and stores, over all SMs.
 // Rows of one expert therefore keep the flat entry order: the permutation
 // is unique and deterministic.
 #include "common.cuh"
@@ -43,40 +44,47 @@ __global__ void __launch_bounds__(kChunk) chunk_hist_kernel(const int32_t* __res
   if (threadIdx.x < E) hist[(size_t)blockIdx.x * E + threadIdx.x] = h[threadIdx.x];
 }
 
-// One block of 64 threads: thread e walks the chunks of expert e.
-__global__ void chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks, int E,
-                                  int32_t* __restrict__ offsets) {
+// One block of 1024 threads. Warp w scans the chunk counts of experts w and
+// w + 32 with warp shuffles (32 chunks at a time, carrying the running sum),
+// then the expert totals are scanned into offsets and added back.
+__global__ void __launch_bounds__(1024) chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks,
+                                                          int E, int32_t* __restrict__ offsets) {
   __shared__ int total[64];
   __shared__ int start[65];
-  const int e = threadIdx.x;
-  int run = 0;
-  if (e < E) {
-    for (int b = 0; b < nchunks; ++b) {
-      const int v = hist[(size_t)b * E + e];
-      hist[(size_t)b * E + e] = run;
-      run += v;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int e = warp; e < E; e += 32) {
+    int carry = 0;
+    for (int b0 = 0; b0 < nchunks; b0 += 32) {
+      const int b = b0 + lane;
+      const int v = (b < nchunks) ? hist[(size_t)b * E + e] : 0;
+      int incl = v;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += u;
+      }
+      if (b < nchunks) hist[(size_t)b * E + e] = carry + incl - v;
+      carry += __shfl_sync(0xffffffffu, incl, 31);
     }
-    total[e] = run;
+    if (lane == 0) total[e] = carry;
   }
   __syncthreads();
-  if (e == 0) {
-    int s = 0;
+  if (threadIdx.x == 0) {
+    int acc = 0;
     for (int x = 0; x < E; ++x) {
-      start[x] = s;
-      s += total[x];
+      start[x] = acc;
+      acc += total[x];
     }
-    start[E] = s;
+    start[E] = acc;
   }
   __syncthreads();
-  if (e <= E) offsets[e] = start[e];
-  if (e < E)
-    for (int b = 0; b < nchunks; ++b) hist[(size_t)b * E + e] += start[e];
+  if (threadIdx.x <= E) offsets[threadIdx.x] = start[threadIdx.x];
+  for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) hist[i] += start[i % E];
 }
 
-__global__ void __launch_bounds__(kChunk) rank_gather_kernel(
-    const int32_t* __restrict__ chosen, int64_t n, int k, int E, int d,
-    const int32_t* __restrict__ base, const uint16_t* __restrict__ X, int32_t* __restrict__ row_token,
-    int32_t* __restrict__ row_of, uint16_t* __restrict__ X_perm) {
+__global__ void __launch_bounds__(kChunk) rank_kernel(
+    const int32_t* __restrict__ chosen, int64_t n, int k, int E, const int32_t* __restrict__ base,
+    int32_t* __restrict__ row_token, int32_t* __restrict__ row_of) {
   constexpr int kWarps = kChunk / 32;
   __shared__ int cnt[kWarps][64];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -90,24 +98,51 @@ __global__ void __launch_bounds__(kChunk) rank_gather_kernel(
   const int rank_in_warp = __popc(peers & ((1u << lane) - 1u));
   if (e >= 0 && rank_in_warp == 0) cnt[warp][e] = __popc(peers);
   __syncthreads();
-  int row = -1;
   if (e >= 0) {
     int before = 0;
     for (int w = 0; w < warp; ++w) before += cnt[w][e];
-    row = base[(size_t)blockIdx.x * E + e] + before + rank_in_warp;
+    const int row = base[(size_t)blockIdx.x * E + e] + before + rank_in_warp;
     row_of[i] = row;
     row_token[row] = static_cast<int32_t>(i / k);
   }
-  // each warp copies the rows of its 32 entries
-  const int nvec = d >> 3;  // 16-byte vectors per row
-  for (int src = 0; src < 32; ++src) {
-    const int r = __shfl_sync(0xffffffffu, row, src);
-    if (r < 0) continue;
-    const int64_t ii = (int64_t)blockIdx.x * kChunk + warp * 32 + src;
-    const int64_t t = ii / k;
+}
+
+// X_perm[row] = X[row_token[row]]: one warp per row, kUnroll independent
+// 16-byte loads per lane in flight, grid over all SMs.
+// Only rows below offsets[E] were ranked (entries with a bad expert index are
+// skipped and reported by chunk_hist_kernel).
+__global__ void __launch_bounds__(256) gather_rows_kernel(const uint16_t* __restrict__ X,
+                                                          const int32_t* __restrict__ row_token,
+                                                          const int32_t* __restrict__ offsets,
+                                                          int E, int T, int d,
+                                                          uint16_t* __restrict__ X_perm) {
+  constexpr int kUnroll = 8;
+  const int lane = threadIdx.x & 31;
+  const int nvec = d >> 3;
+  const int64_t R = offsets[E];
+  const int64_t warps_total = (int64_t)gridDim.x * (blockDim.x >> 5);
+  for (int64_t r = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < R;
+       r += warps_total) {
+    const int64_t t = row_token[r];
+    if (t < 0 || t >= T) {
+      if (lane == 0) report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, static_cast<int>(r));
+      continue;
+    }
     const uint4* in = reinterpret_cast<const uint4*>(X + t * d);
-    uint4* out = reinterpret_cast<uint4*>(X_perm + (int64_t)r * d);
-    for (int v = lane; v < nvec; v += 32) out[v] = __ldg(in + v);
+    uint4* out = reinterpret_cast<uint4*>(X_perm + r * d);
+    for (int v0 = lane; v0 < nvec; v0 += 32 * kUnroll) {
+      uint4 buf[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int v = v0 + 32 * u;
+        if (v < nvec) buf[u] = __ldg(in + v);
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int v = v0 + 32 * u;
+        if (v < nvec) out[v] = buf[u];
+      }
+    }
   }
 }
 
@@ -122,9 +157,15 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict
   for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < T; t += warps_total) {
     int rows[ORDERMOE_MAX_TOPK];
     float ws[ORDERMOE_MAX_TOPK];
+    bool ok = true;
     for (int j = 0; j < k; ++j) {
       rows[j] = row_of[(size_t)t * k + j];
       ws[j] = w[(size_t)t * k + j];
+      if (rows[j] < 0 || (int64_t)rows[j] >= (int64_t)T * k) ok = false;
+    }
+    if (!ok) {  // a row index outside Y_perm: report, leave y[t] untouched
+      if (lane == 0) report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, t);
+      continue;
     }
     for (int v = lane; v < nvec; v += 32) {
       float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
@@ -160,11 +201,16 @@ int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int 
   }
   chunk_hist_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, E, hist);
   OM_LAUNCHED("chunk_hist_kernel");
-  chunk_scan_kernel<<<1, 96, 0, stream>>>(hist, nchunks, E, offsets);
+  chunk_scan_kernel<<<1, 1024, 0, stream>>>(hist, nchunks, E, offsets);
   OM_LAUNCHED("chunk_scan_kernel");
-  rank_gather_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, d, hist, X, row_token,
-                                                     row_of, X_perm);
-  OM_LAUNCHED("rank_gather_kernel");
+  rank_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, hist, row_token, row_of);
+  OM_LAUNCHED("rank_kernel");
+  int64_t blocks = (n + 7) / 8;
+  const int cap = num_sms() * 8;
+  if (blocks > cap) blocks = cap;
+  gather_rows_kernel<<<static_cast<int>(blocks), 256, 0, stream>>>(X, row_token, offsets, E, T, d,
+                                                                    X_perm);
+  OM_LAUNCHED("gather_rows_kernel");
   return ORDERMOE_OK;
 }
 

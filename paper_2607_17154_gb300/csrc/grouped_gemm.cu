@@ -66,7 +66,7 @@ constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + static_cast<int>(sizeof
 enum { GATEUP = 0, DOWN = 1, LOGITS = 2 };
 
 struct Args {
-  const int32_t* offsets;  // [E+1] row ranges; null: one group of `rows` rows
+  const int32_t* offsets;  // [E+1] row ranges (0 <= ... <= rows); null: one group of `rows` rows
   int rows;
   int n_valid;       // LOGITS: number of valid output columns
   float* out_f32;    // LOGITS: H [rows][n_valid] fp32
@@ -121,14 +121,21 @@ __global__ void __launch_bounds__(THREADS, 1)
     s.abort = 0;
     s.zero = 0;
     int acc = 0;
+    bool bad = false;
     for (int e = 0; e <= args.E; ++e) {
       const int o = args.offsets ? args.offsets[e] : (e == 0 ? 0 : args.rows);
       s.offs[e] = o;
+      if (e == 0 && o != 0) bad = true;
       if (e > 0) {
         const int rows = o - s.offs[e - 1];
+        if (rows < 0) bad = true;
         acc += rows > 0 ? (rows + BM - 1) / BM : 0;
       }
       s.mt_start[e] = acc;
+    }
+    if (bad || s.offs[args.E] > args.rows) {  // offsets must run 0 <= ... <= rows
+      if (blockIdx.x == 0) report(&g_err_gemm, ORDERMOE_DEV_BAD_INDEX, -2);
+      for (int e = 0; e <= args.E; ++e) s.mt_start[e] = 0;  // no tiles
     }
     fence_mbar_init();
   }
@@ -400,7 +407,7 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
   if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
   if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
   Args a{};
-  a.offsets = offsets; a.E = E; a.limit_ns = wait_limit_ns();
+  a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = d; a.n_tiles = dff / 128; a.b_rows = dff; a.out = H; a.ldo = dff;
   const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
   const int sms = num_sms();
@@ -420,7 +427,7 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   if ((rc = make_map(&mH, H, R, dff))) return rc;
   if ((rc = make_map(&mW2, W2, (uint64_t)E * d, dff))) return rc;
   Args a{};
-  a.offsets = offsets; a.E = E; a.limit_ns = wait_limit_ns();
+  a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = dff; a.n_tiles = d / 256; a.b_rows = d; a.out = Y; a.ldo = d;
   const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
   const int sms = num_sms();

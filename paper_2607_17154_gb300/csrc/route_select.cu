@@ -161,20 +161,35 @@ __global__ void __launch_bounds__(256) route_select_kernel(
 #pragma unroll
       for (int e = 0; e < EMAX; ++e) lg[e] = 0.0f;
       const uint4* xr = reinterpret_cast<const uint4*>(X + (size_t)t * d);
-      for (int c = lane; c < (d >> 3); c += 32) {
-        const uint4 xv = __ldg(xr + c);
-        const float x0 = bf16_lo(xv.x), x1 = bf16_hi(xv.x), x2 = bf16_lo(xv.y), x3 = bf16_hi(xv.y);
-        const float x4 = bf16_lo(xv.z), x5 = bf16_hi(xv.z), x6 = bf16_lo(xv.w), x7 = bf16_hi(xv.w);
+      const int nvec = d >> 3;
+      // X is streamed once from HBM: keep kBatch independent 16-byte loads
+      // per lane in flight before using them; W_r stays in L1.
+      constexpr int kBatch = 4;
+      for (int c0 = lane; c0 < nvec; c0 += 32 * kBatch) {
+        uint4 xv[kBatch];
 #pragma unroll
-        for (int e = 0; e < EMAX; ++e) {
-          if (e < E) {
-            const uint4 wv = __ldg(reinterpret_cast<const uint4*>(Wr + (size_t)e * d) + c);
-            float a = lg[e];
-            a = fmaf(x0, bf16_lo(wv.x), a); a = fmaf(x1, bf16_hi(wv.x), a);
-            a = fmaf(x2, bf16_lo(wv.y), a); a = fmaf(x3, bf16_hi(wv.y), a);
-            a = fmaf(x4, bf16_lo(wv.z), a); a = fmaf(x5, bf16_hi(wv.z), a);
-            a = fmaf(x6, bf16_lo(wv.w), a); a = fmaf(x7, bf16_hi(wv.w), a);
-            lg[e] = a;
+        for (int b = 0; b < kBatch; ++b) {
+          const int c = c0 + 32 * b;
+          xv[b] = (c < nvec) ? __ldg(xr + c) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int b = 0; b < kBatch; ++b) {
+          const int c = c0 + 32 * b;
+          if (c >= nvec) break;
+          const float x0 = bf16_lo(xv[b].x), x1 = bf16_hi(xv[b].x), x2 = bf16_lo(xv[b].y);
+          const float x3 = bf16_hi(xv[b].y), x4 = bf16_lo(xv[b].z), x5 = bf16_hi(xv[b].z);
+          const float x6 = bf16_lo(xv[b].w), x7 = bf16_hi(xv[b].w);
+#pragma unroll
+          for (int e = 0; e < EMAX; ++e) {
+            if (e < E) {
+              const uint4 wv = __ldg(reinterpret_cast<const uint4*>(Wr + (size_t)e * d) + c);
+              float a = lg[e];
+              a = fmaf(x0, bf16_lo(wv.x), a); a = fmaf(x1, bf16_hi(wv.x), a);
+              a = fmaf(x2, bf16_lo(wv.y), a); a = fmaf(x3, bf16_hi(wv.y), a);
+              a = fmaf(x4, bf16_lo(wv.z), a); a = fmaf(x5, bf16_hi(wv.z), a);
+              a = fmaf(x6, bf16_lo(wv.w), a); a = fmaf(x7, bf16_hi(wv.w), a);
+              lg[e] = a;
+            }
           }
         }
       }

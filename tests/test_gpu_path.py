@@ -345,3 +345,30 @@ def test_bounded_wait_runs_out_and_reports():
     # the context is still usable afterwards
     x = torch.ones(16, device=DEV)
     assert float(x.sum()) == 16.0
+
+
+def test_bad_row_index_in_combine_is_reported_not_read():
+    T, k, d = 16, 2, 64
+    Yp = torch.zeros(T * k, d, dtype=torch.bfloat16, device=DEV)
+    row_of = torch.arange(T * k, dtype=torch.int32, device=DEV).view(T, k).clone()
+    row_of[5, 1] = T * k + 1000                      # outside Y_perm
+    y = torch.full((T, d), 7.0, dtype=torch.bfloat16, device=DEV)
+    B.ordermoe_combine(Yp, row_of, torch.ones(T, k, device=DEV), T, k, d, y)
+    code, detail = B.ordermoe_device_error()
+    assert code == B.DEV_BAD_INDEX and detail == 5
+    yc = y.cpu().float()
+    assert (yc[5] == 7.0).all() and (yc[4] == 0).all()
+
+
+def test_bad_offsets_in_expert_ffn_are_reported_not_used():
+    E, R, d, dff = 3, 64, 256, 128
+    z = lambda *s: torch.zeros(*s, dtype=torch.bfloat16, device=DEV)
+    W1, W3, W2 = z(E, dff, d), z(E, dff, d), z(E, d, dff)
+    H = torch.full((R, dff), 3.0, dtype=torch.bfloat16, device=DEV)
+    Y = torch.full((R, d), 3.0, dtype=torch.bfloat16, device=DEV)
+    for bad in ([0, 40, 20, 64], [0, 10, 20, 4000], [5, 10, 20, 64]):
+        B.ordermoe_expert_ffn(z(R, d), torch.tensor(bad, dtype=torch.int32, device=DEV), R, W1, W3,
+                              W2, E, d, dff, H, Y)
+        code, detail = B.ordermoe_device_error()
+        assert code == B.DEV_BAD_INDEX and detail == -2, bad
+    assert (H.cpu().float() == 3.0).all() and (Y.cpu().float() == 3.0).all()
