@@ -28,6 +28,29 @@ METRIC = "MoE-layer tokens/s on 1 GB300 (route+select+FFN) and % of tensor/HBM r
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
+# DRAM bytes (read + write) per launch of the gate/up GEMM at the mixtral_prefill workload, from
+# the ncu capture summarised in profiles/ffn_gemm_gate_up_mixtral_prefill.md, valid only while the
+# kernel sources hash to the values recorded with it.
+GATE_UP_TRAFFIC = {
+    "bytes": 2173090816,
+    "sha256": {"paper_2607_17154_gb300/csrc/grouped_gemm.cu":
+               "54bf04f18e3bf96dce70b2c096b0a7dc19eda56fbe66bf983d119f040d63b634",
+               "paper_2607_17154_gb300/csrc/common.cuh":
+               "3df474ac82e60f13f0feed5b9c9d5dc72f79ef090734595e235722b2624e6103"},
+}
+
+
+def gate_up_traffic(workload):
+    """The recorded traffic if the kernel is unchanged since the capture, else None."""
+    import hashlib
+    if workload != "mixtral_prefill":
+        return None
+    for rel, digest in GATE_UP_TRAFFIC["sha256"].items():
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            if hashlib.sha256(f.read()).hexdigest() != digest:
+                return None
+    return GATE_UP_TRAFFIC["bytes"]
+
 
 def parse():
     p = argparse.ArgumentParser()
@@ -296,7 +319,7 @@ def run_ours(args, dist):
                          % (3 * E * d * dff * 2 / 1e9)},
         "roofline": {"kernel": "ffn_gemm_kernel<gate_up> (tcgen05)", "bound": "tensor",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
-                     "frac": round(achieved / peak, 4), "traffic": None,
+                     "frac": round(achieved / peak, 4), "traffic": gate_up_traffic(w.name),
                      "peak_source": "%s bf16_tflops_sustained" % pk_kind,
                      "flop_per_launch": gu_flop, "ms_per_launch": round(gu_ms, 4),
                      "layer_tflops": round(layer_flop / (elapsed_ms / args.steps / 1e3) / 1e12, 1)},

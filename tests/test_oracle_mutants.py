@@ -1,0 +1,89 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each case plants one mistake (a dropped term, a wrong sign or index, a
+transposed operand, a wrong tie rule) in a temporary copy of the oracle's
+source, builds it, loads it in place of the real oracle, and runs the pin
+tests against it: at least one pin must fail. The real oracle is never
+modified.
+"""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "ordermoe_oracle.cpp")
+
+# (name, original text, planted mistake)
+MUTANTS = [
+    ("router: W transposed", "acc += bf(X, (int64_t)t * d + c) * bf(W, (int64_t)e * d + c);",
+     "acc += bf(X, (int64_t)t * d + c) * bf(W, (int64_t)c * E + e);"),
+    ("topk: ties to higher index", "return ia < ib;", "return ia > ib;"),
+    ("topk: no renormalisation", "renorm ? p[order[j]] / ssel : p[order[j]]", "p[order[j]]"),
+    ("Eq. 18: sign of Sim", "q = 0.5f * (1.0f - std::min(s, 1.0f));", "q = 0.5f * (1.0f + std::min(s, 1.0f));"),
+    ("Eq. 38: quality term not divided by Qbar",
+     "omega_Q * static_cast<double>(q) / static_cast<double>(qbar)", "omega_Q * static_cast<double>(q)"),
+    ("Eq. 7: threshold ignored", "group[k] == group[r] && s >= theta", "group[k] == group[r]"),
+    ("Eq. 7: group ignored", "group[k] == group[r] && s >= theta", "s >= theta"),
+    ("Eq. 37: latency dropped", "z / B[s * M + m] + tau[s * M + m]", "z / B[s * M + m]"),
+    ("Eq. 37: compute on the source server", "double comp = c / F[m];", "double comp = c / F[s];"),
+    ("Eq. 38: d_ref of the executing server", "double dref = c / F[a];", "double dref = c / F[0];"),
+    ("Eq. 40: budget ignored", "if (!(q + Qtab[r * E + kk] <= qbar)) continue;", ""),
+    ("distinct experts ignored", "if ((taken >> kk) & 1u) continue;", ""),
+    ("tie: remote preferred", "better = away < best_away;", "better = away > best_away;"),
+    ("Eq. 44: loss not accumulated", "q = q + Qtab[r * E + best_k];", ""),
+    ("Eq. 44: location from the last slot", "if (j == 0) first_server = best_m;", "first_server = best_m;"),
+    ("permutation not stable", "row_token[row] = static_cast<int32_t>(i / k);",
+     "row_token[row] = static_cast<int32_t>((n - 1 - i) / k);"),
+    ("FFN: gate and up swapped", "double silu = g / (1.0 + std::exp(-g));\n      h[n] = float_to_bf16_bits(static_cast<float>(silu * u));",
+     "double silu = u / (1.0 + std::exp(-u));\n      h[n] = float_to_bf16_bits(static_cast<float>(silu * g));"),
+    ("FFN: W2 transposed", "W2 + ((int64_t)e * d + o) * dff", "W2 + (int64_t)e * d * dff + o"),
+    ("combine: weights dropped", "acc += static_cast<double>(w[(int64_t)t * k + j]) * bf(Yp, row * d + c);",
+     "acc += bf(Yp, row * d + c);"),
+    ("Eq. 4: not normalised", "dot / (norm[i] * norm[j])", "dot"),
+    ("Eq. 24: threshold inclusive", "best_s < theta", "best_s <= theta"),
+    ("Eq. 25: argmax ties to the later dominant", "if (best_g < 0 || s > best_s)", "if (best_g < 0 || s >= best_s)"),
+    ("Eq. 27: representativeness over all experts", "if (group[k] == group[j]) { s += sim[j * E + k]; ++size; }",
+     "{ s += sim[j * E + k]; ++size; }"),
+    ("Eq. 30: dispersion term dropped", "lambda2 * static_cast<double>(eta)", "0.0"),
+    ("Eq. 29: capacity ignored", "if (!(b[m] + pl[j] <= C[m])) continue;", ""),
+]
+
+
+CONFTEST = """
+import pytest
+
+
+@pytest.fixture(scope="session")
+def orc():
+    import oracle
+    assert "mutant" in oracle.__file__, oracle.__file__
+    oracle.lib()
+    return oracle
+"""
+
+
+@pytest.mark.parametrize("name,orig,bad", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_planted_mistake(name, orig, bad, tmp_path):
+    src = open(SRC).read()
+    assert src.count(orig) == 1, "mutation anchor not found once: %r" % orig
+    base = tmp_path / "mutant"
+    pkg = base / "oracle"
+    pkg.mkdir(parents=True)
+    for f in ("__init__.py", "build.py"):
+        shutil.copy(os.path.join(ROOT, "oracle", f), pkg / f)
+    (pkg / "ordermoe_oracle.cpp").write_text(src.replace(orig, bad))
+    subprocess.run([sys.executable, str(pkg / "build.py")], check=True, capture_output=True)
+    tdir = base / "pins"
+    tdir.mkdir()
+    shutil.copy(os.path.join(ROOT, "tests", "test_oracle_pins.py"), tdir / "test_oracle_pins.py")
+    (tdir / "conftest.py").write_text(CONFTEST)
+    env = dict(os.environ, PYTHONPATH=str(base) + os.pathsep + ROOT)
+    r = subprocess.run([sys.executable, "-m", "pytest", str(tdir), "-q", "-x", "-p", "no:cacheprovider",
+                        "--rootdir", str(base)],
+                       capture_output=True, text=True, env=env, cwd=str(base))
+    assert "mutant" not in r.stdout or "AssertionError: /" not in r.stdout
+    assert r.returncode == 1, "no pin caught the planted mistake %r (rc %d):\n%s" % (
+        name, r.returncode, r.stdout[-2000:])

@@ -642,3 +642,27 @@ def test_coverage(orc):
     x = np.array([[1, 0, 1, 0], [0, 1, 0, 0]], np.uint8)
     g = np.array([0, 0, 1, 1], np.int32)
     np.testing.assert_array_equal(orc.coverage(x, g, 2), [[1, 1], [1, 0]])
+
+
+def test_group_threshold_is_strict_and_ties_go_to_the_earlier_dominant(orc):
+    cnt = np.array([3, 2, 1], np.int32)            # visiting order 0, 1, 2
+    # Sim(1, 0) == theta: Eq. 24 needs max Sim < theta for a new dominant, so 1 joins 0
+    sim = np.array([[1, .5, .3], [.5, 1, .3], [.3, .3, 1]], np.float32)
+    g, K, dom = orc.group(sim, cnt, 0.5)
+    assert K == 2 and list(g) == [0, 0, 1]
+    # 0 and 1 are dominants (Sim .1 < .3); 2 is equally similar to both (.6):
+    # Eq. 25's argmax tie goes to the earlier dominant
+    sim2 = np.array([[1, .1, .6], [.1, 1, .6], [.6, .6, 1]], np.float32)
+    g2, K2, dom2 = orc.group(sim2, cnt, 0.3)
+    assert K2 == 2 and list(dom2) == [0, 1] and g2[2] == 0
+
+
+def test_place_disperses_same_group_experts_even_when_load_alone_would_not(orc):
+    # importance order 0 (g0), 2 (g1), 1 (g0), 3 (g1) on 2 servers of capacity 4:
+    # load balance alone would put 0 and 1 together; the eta term of Eq. 30
+    # sends each server one expert of each group
+    group = np.array([[0, 0, 1, 1]], np.int32)
+    I = np.array([[0.9, 0.7, 0.8, 0.6]])
+    x, used, rc = orc.place(group, I, np.ones((1, 4)), np.array([4.0, 4.0]))
+    assert rc == 0
+    np.testing.assert_array_equal(x[0], [[1, 0, 0, 1], [0, 1, 1, 0]])
