@@ -218,8 +218,10 @@ def run_ours(args, dist):
     torch.cuda.set_device(device)
     B.lib()
     w = synth.workload(args.workload)
-    if w.L != 1:
-        raise SystemExit("bench.py times single-layer workloads; %s has %d layers" % (w.name, w.L))
+    if w.name == "decode_stack":
+        return run_decode(args, dist, w, device)
+    if w.name == "similarity":
+        return run_similarity(args, dist, w, device)
     inp, home, tables, plan = setup_gpu(w, args.seed + 1000 * dist.rank, device)
     T, E, d, k, dff = w.T, w.E, w.d, w.k, w.dff
     R = T * k
@@ -333,6 +335,162 @@ def run_ours(args, dist):
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, inp, args.seed, args.cpu_seconds)
     return out
+
+
+def timed_region(args, dist, device, fn):
+    """W warm-up calls, then K timed calls between barriers and synchronizes,
+    CUDA events on the current stream; returns (max-over-ranks ms, clocks)."""
+    import torch
+    for _ in range(max(args.warmup, 3)):
+        fn()
+    stream = torch.cuda.current_stream(device)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(gpu_index(dist.local_rank))
+    sampler.start()
+    dist.barrier(device)
+    torch.cuda.synchronize(device)
+    a.record(stream)
+    for _ in range(args.steps):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize(device)
+    dist.barrier(device)
+    clocks = sampler.stop()
+    return dist.max(a.elapsed_time(b), device), clocks
+
+
+def run_decode(args, dist, w, device):
+    """Decode stack: one step = 32 MoE layers over a batch of 128 tokens, with
+    the selection state carried across layers; bound by streaming the expert
+    weights from HBM."""
+    import torch
+    from paper_2607_17154_gb300 import binding as B
+    from paper_2607_17154_gb300 import synth
+    from paper_2607_17154_gb300.layer import LayerStack
+    seed = args.seed + 1000 * dist.rank
+    L, E, M = w.L, w.E, w.M
+    layers = []
+    for l in range(L):
+        inp = synth.layer_inputs(w, seed=seed, layer=l, device=device)
+        layers.append({"W_r": inp["Wr"], "W1": inp["W1"], "W3": inp["W3"], "W2": inp["W2"]})
+    home = torch.as_tensor(synth.layer_inputs(w, seed=seed, with_ffn=False)["home"]).to(device)
+    # offline plan of all layers at once: theta_l of Eq. 6, b_m carried over the layers
+    Xcal = synth.calibration(w.n_cal, w.d, seed, device=device)
+    Wr = torch.stack([l["W_r"] for l in layers])
+    sim = torch.empty(L, E, E, dtype=torch.float32, device=device)
+    counts = torch.empty(L, E, dtype=torch.int32, device=device)
+    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, w.n_cal), dtype=torch.uint8,
+                     device=device)
+    B.ordermoe_similarity(Wr, Xcal, L, E, w.d, w.n_cal, w.k, sim, counts, ws)
+    group = torch.empty(L, E, dtype=torch.int32, device=device)
+    ng = torch.empty(L, dtype=torch.int32, device=device)
+    theta = torch.empty(L, dtype=torch.float32, device=device)
+    x = torch.empty(L, M, E, dtype=torch.uint8, device=device)
+    used = torch.empty(M, dtype=torch.float64, device=device)
+    st = torch.empty(1, dtype=torch.int32, device=device)
+    B.ordermoe_place(sim, counts, L, E, M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5, 0.5, 0.5,
+                     torch.ones(L, E, dtype=torch.float64, device=device),
+                     torch.full((M,), L * E / M, dtype=torch.float64, device=device),
+                     group, ng, theta, x, used, st)
+    sp = synth.server_params(M, w.d, w.dff, seed)
+    f64 = lambda a: torch.as_tensor(a, dtype=torch.float64).to(device)
+    th = theta.cpu().tolist()
+    tabs = []
+    for l in range(L):
+        t = torch.zeros(B.ordermoe_tables_bytes(E, M), dtype=torch.uint8, device=device)
+        B.ordermoe_build_tables(sim[l], group[l], x[l], th[l], w.qbar, f64(sp.F), f64(sp.B),
+                                f64(sp.tau), sp.z, sp.c, sp.omega_T, sp.omega_Q, t)
+        tabs.append(t)
+    stack = LayerStack(layers, tabs, w.k, w.T, device)
+    Xs = [synth.hidden(w.T, w.d, seed + 5000 + l, device=device) for l in range(w.L)]
+    ys = [torch.empty(w.T, w.d, dtype=torch.bfloat16, device=device) for _ in range(w.L)]
+    loc = home.clone()
+    qhat = torch.zeros(w.T, device=device)
+
+    def step():
+        loc.copy_(home)
+        qhat.zero_()
+        stack.step(Xs, home, loc, qhat, ys)
+
+    ms, clocks = timed_region(args, dist, device, step)
+    code, detail = B.ordermoe_device_error()
+    if code:
+        raise RuntimeError("device error %d (%d)" % (code, detail))
+    step_s = ms / args.steps / 1e3
+    wbytes = 3.0 * w.E * w.d * w.dff * 2 * w.L
+    pk, pk_kind = peaks()
+    achieved = wbytes / step_s / 1e9
+    peak = float(pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]))
+    return {
+        "metric": METRIC, "value": round(w.T * args.steps * dist.world / (ms / 1e3), 1), "unit": UNIT,
+        "n_gpus": dist.world, "steps": args.steps, "warmup": max(args.warmup, 3),
+        "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "layers": w.L, "T": w.T, "d": w.d, "E": w.E, "k": w.k,
+                   "d_ff": w.dff, "M": w.M, "l2": "inputs larger than L2: %.1f GB of expert weights"
+                   % (wbytes / 1e9)},
+        "roofline": {"kernel": "whole decode step (expert weight streaming)", "bound": "hbm",
+                     "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": None,
+                     "peak_source": "%s hbm_gbs" % pk_kind, "bytes_per_step": wbytes},
+        "gpu_launches": 8 * w.L * args.steps,
+        "clocks": clocks,
+    }
+
+
+def run_similarity(args, dist, w, device):
+    """Offline similarity of 24 layers x 64 experts over 262144 calibration
+    tokens (Eqs. 3-5), then grouping and placement (Eqs. 6, 24-31)."""
+    import torch
+    from paper_2607_17154_gb300 import binding as B
+    from paper_2607_17154_gb300 import synth
+    L, E, d, N = w.L, w.E, w.d, w.n_cal
+    seed = args.seed + 1000 * dist.rank
+    Wr = torch.stack([synth.router_weights(E, d, w.n_clusters, seed=seed + 500 + l, device=device)
+                      for l in range(L)])
+    Xcal = synth.calibration(N, d, seed, device=device)
+    sim = torch.empty(L, E, E, dtype=torch.float32, device=device)
+    counts = torch.empty(L, E, dtype=torch.int32, device=device)
+    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, N), dtype=torch.uint8, device=device)
+    group = torch.empty(L, E, dtype=torch.int32, device=device)
+    ng = torch.empty(L, dtype=torch.int32, device=device)
+    theta = torch.empty(L, dtype=torch.float32, device=device)
+    x = torch.empty(L, w.M, E, dtype=torch.uint8, device=device)
+    used = torch.empty(w.M, dtype=torch.float64, device=device)
+    st = torch.empty(1, dtype=torch.int32, device=device)
+    p = torch.ones(L, E, dtype=torch.float64, device=device)
+    C = torch.full((w.M,), L * E / w.M, dtype=torch.float64, device=device)
+
+    def step():
+        B.ordermoe_similarity(Wr, Xcal, L, E, d, N, w.k, sim, counts, ws)
+        B.ordermoe_place(sim, counts, L, E, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5,
+                         0.5, 0.5, p, C, group, ng, theta, x, used, st)
+
+    ms, clocks = timed_region(args, dist, device, step)
+    code, detail = B.ordermoe_device_error()
+    if code:
+        raise RuntimeError("device error %d (%d)" % (code, detail))
+    step_s = ms / args.steps / 1e3
+    flop = 2.0 * N * L * E * d + 2.0 * L * N * E * E
+    pk, pk_kind = peaks()
+    peak = float(pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    achieved = flop / step_s / 1e12
+    return {
+        "metric": "calibration tokens/s through the offline similarity + grouping + placement",
+        "value": round(N * args.steps * dist.world / (ms / 1e3), 1), "unit": "tokens/s",
+        "n_gpus": dist.world, "steps": args.steps, "warmup": max(args.warmup, 3),
+        "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "layers": L, "E": E, "d": d, "N": N, "groups": w.n_clusters,
+                   "M": w.M, "k_freq": w.k},
+        "roofline": {"kernel": "ordermoe_similarity + ordermoe_place (whole call)", "bound": "tensor",
+                     "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
+                     "frac": round(achieved / peak, 4), "traffic": None,
+                     "peak_source": "%s bf16_tflops (burst)" % pk_kind, "flop_per_step": flop},
+        "gpu_launches": 4 * args.steps,
+        "n_groups": ng.cpu().tolist()[:3], "place_status": int(st.item()),
+        "clocks": clocks,
+    }
 
 
 # ----------------------------------------------------------------- oracle side

@@ -59,3 +59,24 @@ def build_tables(sim, group, placement, theta, qbar, sp, device):
                             theta, qbar, f(sp.F, torch.float64), f(sp.B, torch.float64),
                             f(sp.tau, torch.float64), sp.z, sp.c, sp.omega_T, sp.omega_Q, t)
     return t
+
+
+class LayerStack:
+    """L MoE layers run through ordermoe_layer_forward with the token state
+    (location, accumulated loss; Eqs. 36 and 44) carried from layer to layer."""
+
+    def __init__(self, layers, tables, k, T_max, device):
+        # layers: list of dicts with W_r, W1, W3, W2 (device bf16); tables: list of device buffers
+        E, dff, d = layers[0]["W1"].shape
+        self.scratch = torch.empty(B.ordermoe_layer_scratch_bytes(T_max, E, d, dff, k),
+                                   dtype=torch.uint8, device=device)
+        self.descs = [B.make_layer_desc(T_max, l["W_r"], l["W1"], l["W3"], l["W2"], t, k,
+                                        self.scratch) for l, t in zip(layers, tables)]
+        self.d, self.T_max = d, T_max
+
+    def step(self, X_layers, home, loc, qhat, y_layers, counters=None, stream=None):
+        """Layer l reads X_layers[l] and writes y_layers[l]; loc/qhat carry the
+        trajectory (set loc = home, qhat = 0 before the first layer)."""
+        T = X_layers[0].shape[0]
+        for desc, X, y in zip(self.descs, X_layers, y_layers):
+            B.ordermoe_layer_forward(desc, T, X, home, loc, qhat, y, counters, 0, stream)
