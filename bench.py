@@ -319,7 +319,7 @@ def run_ours(args, dist):
                    "home": w.home, "seed": args.seed, "parallelism": "replicas",
                    "l2": "inputs larger than L2: %.2f GB of expert weights read every step"
                          % (3 * E * d * dff * 2 / 1e9)},
-        "roofline": {"kernel": "ffn_gemm_kernel<gate_up> (tcgen05)", "bound": "tensor",
+        "roofline": {"kernel": "ffn_gemm_pair_kernel<gate_up> (tcgen05, CTA pair)", "bound": "tensor",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(achieved / peak, 4), "traffic": gate_up_traffic(w.name),
                      "peak_source": "%s bf16_tflops_sustained" % pk_kind,
@@ -330,6 +330,7 @@ def run_ours(args, dist):
         "clocks": clocks,
         "exec_types": dict(zip(["local_exact", "local_sub", "remote_exact", "remote_sub"],
                                counters.cpu().tolist())),
+        "rows_per_expert": torch.diff(offsets).cpu().tolist(),
         "plan": plan,
     }
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:

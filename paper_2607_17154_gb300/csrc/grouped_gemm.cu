@@ -344,6 +344,274 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+// ------------------------------------------------- CTA-pair variant (gate/up, down)
+//
+// A cluster of 2 CTAs on 2 SMs computes a 256-row x 256-column tile with
+// tcgen05.mma.cta_group::2 issued by the even CTA: each CTA holds 128 rows
+// of A and 128 of the 256 B rows in its own shared memory (the same offsets in
+// both), and receives its 128 accumulator rows in its own TMEM. Per SM this
+// halves the B bytes loaded from L2 and written to shared memory per flop
+// compared with a one-CTA 128 x 256 tile. gate/up: B rows 0..127 (even CTA)
+// are W1_e rows, 128..255 (odd CTA) the same rows of W3_e, so accumulator
+// columns 0..127 are the gate and 128..255 the up projection.
+// Barriers: full[s] (even CTA, one arrive with the pair's bytes; both CTAs'
+// TMA loads complete on it), empty[s] and tfull[b] (both CTAs, arrived by the
+// even CTA's MMA commits multicast to the pair), tempty[b] (even CTA, one
+// arrive per epilogue warp of either CTA).
+constexpr int P_BM = 256;            // rows per CTA pair
+constexpr int P_STAGES = 6;
+constexpr int P_STAGE_BYTES = 2 * BOX_BYTES;  // 128 A rows + 128 B rows per CTA
+constexpr uint32_t P_IDESC = idesc_bf16_f32(256, 256);
+constexpr int P_SMEM_BYTES = P_STAGES * P_STAGE_BYTES + 1024 + static_cast<int>(sizeof(Smem));
+
+struct PSmem {
+  uint64_t full[P_STAGES];
+  uint64_t empty[P_STAGES];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+  int zero;
+  int mt_start[ORDERMOE_MAX_EXPERTS + 1];
+  int offs[ORDERMOE_MAX_EXPERTS + 1];
+};
+static_assert(sizeof(PSmem) <= sizeof(Smem) + 8 * 8, "PSmem size");
+
+__device__ __forceinline__ Tile decode_pair(int tile, const PSmem& s, int E, int n_tiles) {
+  int e = 0;
+  while (e < E - 1 && s.mt_start[e + 1] * n_tiles <= tile) ++e;
+  const int local = tile - s.mt_start[e] * n_tiles;
+  const int n_mt = s.mt_start[e + 1] - s.mt_start[e];
+  Tile t;
+  t.e = e;
+  t.n = local / n_mt;
+  t.m0 = s.offs[e] + (local - t.n * n_mt) * P_BM;
+  t.m_end = s.offs[e + 1];
+  return t;
+}
+
+template <int MODE>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+    ffn_gemm_pair_kernel(const __grid_constant__ CUtensorMap mapA,
+                         const __grid_constant__ CUtensorMap mapB0,
+                         const __grid_constant__ CUtensorMap mapB1, Args args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* tiles = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  PSmem& s = *reinterpret_cast<PSmem*>(tiles + P_STAGES * P_STAGE_BYTES);
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool even = (rank == 0);
+  const int cluster = blockIdx.x >> 1;
+  const int n_clusters = gridDim.x >> 1;
+
+  if (tid == 0) {
+    for (int i = 0; i < P_STAGES; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s.tfull[i], 1);
+      mbar_init(&s.tempty[i], 8);
+    }
+    mbar_init(&s.drain, 1);
+    s.abort = 0;
+    s.zero = 0;
+    int acc = 0;
+    bool bad = false;
+    for (int e = 0; e <= args.E; ++e) {
+      const int o = args.offsets[e];
+      s.offs[e] = o;
+      if (e == 0 && o != 0) bad = true;
+      if (e > 0) {
+        const int rows = o - s.offs[e - 1];
+        if (rows < 0) bad = true;
+        acc += rows > 0 ? (rows + P_BM - 1) / P_BM : 0;
+      }
+      s.mt_start[e] = acc;
+    }
+    if (bad || s.offs[args.E] > args.rows) {
+      if (blockIdx.x == 0) report(&g_err_gemm, ORDERMOE_DEV_BAD_INDEX, -2);
+      for (int e = 0; e <= args.E; ++e) s.mt_start[e] = 0;
+    }
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&mapA);
+    tma_prefetch_map(&mapB0);
+    if (MODE == GATEUP) tma_prefetch_map(&mapB1);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(&s.tmem_base, TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
+  tc_fence_after();
+  const uint32_t tmem_base = s.tmem_base;
+  const int total = s.mt_start[args.E] * args.n_tiles;
+  const int kblocks = args.K / BK;
+  volatile int* abort = &s.abort;
+  uint32_t issued_mask = 0, last_phase_bits = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int tile = cluster; tile < total && !*abort; tile += n_clusters) {
+        const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
+        const int arow = t.m0 + 128 * static_cast<int>(rank);
+        const int brow = (MODE == GATEUP) ? t.e * args.b_rows + t.n * 128
+                                          : t.e * args.b_rows + t.n * 256 + 128 * static_cast<int>(rank);
+        const CUtensorMap* mapB = (MODE == GATEUP && !even) ? &mapB1 : &mapB0;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
+            if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 11);
+            *abort = 1;
+            break;
+          }
+          uint8_t* sa = tiles + stage * P_STAGE_BYTES;
+          uint8_t* sb = sa + BOX_BYTES;
+          const uint32_t full_even = mapa_shared(smem_u32(&s.full[stage]), 0);
+          if (even) mbar_arrive_expect_tx(&s.full[stage], 2 * P_STAGE_BYTES);
+          tma_load_2d_pair(sa, &mapA, full_even, kb * BK, arow);
+          tma_load_2d_pair(sb, mapB, full_even, kb * BK, brow);
+          issued_mask |= 1u << stage;
+          last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
+          if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && even) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      for (int tile = cluster; tile < total && !*abort; tile += n_clusters, ++it) {
+        const int slot = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!mbar_wait(&s.tempty[slot], acc_phase ^ 1u, args.limit_ns, abort)) {
+          if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 12);
+          *abort = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + slot * BN;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&s.full[stage], phase, args.limit_ns, abort)) {
+            if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 13);
+            *abort = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(tiles + stage * P_STAGE_BYTES);
+          const uint32_t b0 = a0 + BOX_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32),
+                          sdesc_kmajor_sw128(b0 + kk * 32), P_IDESC, (kb | kk) != 0 ? 1u : 0u);
+          mma_issued = true;
+          mma_commit_pair(&s.empty[stage], 0x3);
+          if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        mma_commit_pair(&s.tfull[slot], 0x3);
+      }
+    }
+  } else {
+    const int q = warp & 3;
+    const int lrow = q * 32 + lane;
+    int it = 0;
+    for (int tile = cluster; tile < total; tile += n_clusters, ++it) {
+      if (__any_sync(0xffffffffu, *abort != 0)) break;
+      const int slot = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      const bool ok =
+          __all_sync(0xffffffffu, mbar_wait(&s.tfull[slot], acc_phase, args.limit_ns, abort));
+      if (!ok) {
+        if (lane == 0 && !*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 14);
+        *abort = 1;
+        break;
+      }
+      tc_fence_after();
+      const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
+      const int row = t.m0 + 128 * static_cast<int>(rank) + lrow;
+      const bool valid = row < t.m_end;
+      const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
+      if (MODE == GATEUP) {
+        uint16_t* orow = args.out + (size_t)row * args.ldo + t.n * 128;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t g[32], u[32];
+          tmem_ld32(tb + c * 32, g);
+          tmem_ld32(tb + 128 + c * 32, u);
+          tmem_ld_wait();
+          if (valid) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
+              const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
+              const float h0 = g0 / (1.0f + __expf(-g0)) * u0;
+              const float h1 = g1 / (1.0f + __expf(-g1)) * u1;
+              pk[i] = pack_bf16x2(h0, h1);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+          }
+        }
+      } else {
+        uint16_t* orow = args.out + (size_t)row * args.ldo + t.n * 256;
+#pragma unroll 1
+        for (int c = 0; c < 8; ++c) {
+          uint32_t v[32];
+          tmem_ld32(tb + c * 32, v);
+          tmem_ld_wait();
+          if (valid) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+              pk[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&s.tempty[slot]), 0));
+    }
+  }
+
+  __syncthreads();
+  if (s.abort) {
+    volatile int* never = &s.zero;
+    if (warp == 0 && lane == 0 && even) {
+      for (int st = 0; st < P_STAGES; ++st)
+        if ((issued_mask >> st) & 1u)
+          mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, args.limit_ns, never);
+    }
+    if (warp == 1 && lane == 0 && even && mma_issued) {
+      mma_commit_pair(&s.drain, 0x1);
+      mbar_wait(&s.drain, 0, args.limit_ns, never);
+    }
+  }
+  tc_fence_before();
+  cluster_sync();  // both CTAs finished: no more arrivals or copies into either
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+}
+
 // ------------------------------------------------------------------- host
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -386,14 +654,48 @@ static int ffn_attrs() {
   static std::once_flag attr_once;
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(attr_once, [] {
-    attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<GATEUP>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    attr_err = cudaFuncSetAttribute(ffn_gemm_pair_kernel<GATEUP>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
     if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<DOWN>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+      attr_err = cudaFuncSetAttribute(ffn_gemm_pair_kernel<DOWN>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
   });
-  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(ffn_gemm_kernel)");
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(ffn_gemm_pair_kernel)");
   return ORDERMOE_OK;
+}
+
+// CTA pairs that can be resident at once (not every SM may find a partner in
+// its GPC); the persistent grid never exceeds it, so no pair waits for another.
+static int max_resident_pairs() {
+  using namespace gg;
+  static std::once_flag once;
+  static int pairs = 0;
+  std::call_once(once, [] {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (num_sms() / 2), 1, 1);
+    cfg.blockDim = dim3(THREADS, 1, 1);
+    cfg.dynamicSmemBytes = P_SMEM_BYTES;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 2;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, ffn_gemm_pair_kernel<GATEUP>, &cfg) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = num_sms() / 2;
+    }
+    pairs = n < num_sms() / 2 ? n : num_sms() / 2;
+  });
+  return pairs;
+}
+
+static int pair_grid(long long tiles) {
+  const int pairs_max = max_resident_pairs();
+  const long long pairs = tiles < pairs_max ? tiles : pairs_max;
+  return static_cast<int>(2 * (pairs > 0 ? pairs : 1));
 }
 
 // H = SwiGLU(X_perm W1^T, X_perm W3^T) over the expert row ranges.
@@ -409,11 +711,9 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
   Args a{};
   a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = d; a.n_tiles = dff / 128; a.b_rows = dff; a.out = H; a.ldo = dff;
-  const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
-  const int sms = num_sms();
-  const int grid = static_cast<int>(tiles < sms ? tiles : sms);
-  ffn_gemm_kernel<GATEUP><<<grid, THREADS, SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
-  OM_LAUNCHED("ffn_gemm_kernel<gate_up>");
+  const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
+  ffn_gemm_pair_kernel<GATEUP><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
+  OM_LAUNCHED("ffn_gemm_pair_kernel<gate_up>");
   return ORDERMOE_OK;
 }
 
@@ -429,11 +729,9 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   Args a{};
   a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = dff; a.n_tiles = d / 256; a.b_rows = d; a.out = Y; a.ldo = d;
-  const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
-  const int sms = num_sms();
-  const int grid = static_cast<int>(tiles < sms ? tiles : sms);
-  ffn_gemm_kernel<DOWN><<<grid, THREADS, SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
-  OM_LAUNCHED("ffn_gemm_kernel<down>");
+  const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
+  ffn_gemm_pair_kernel<DOWN><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
+  OM_LAUNCHED("ffn_gemm_pair_kernel<down>");
   return ORDERMOE_OK;
 }
 
