@@ -20,8 +20,8 @@ int read_clear_err_sim(unsigned long long* out) {
   return ORDERMOE_OK;
 }
 
-constexpr int kSimChunk = 1024;  // calibration tokens per partial Gram
-constexpr int kSub = 32;         // tokens staged in shared memory at a time
+constexpr int kSimChunk = 4096;  // calibration tokens per partial Gram
+constexpr int kSub = 64;         // tokens staged in shared memory at a time
 
 // Rank order used for top-k: larger logit first, equal logits by lower index.
 __device__ __forceinline__ void add_topk_counts(const float* l, int E, int kf, int* counts) {
@@ -38,57 +38,105 @@ __device__ __forceinline__ void add_topk_counts(const float* l, int E, int kf, i
   }
 }
 
-// grid (chunks, L), 256 threads. Partial Gram of layer l over the tokens of
-// one chunk: thread (i, jb) accumulates G[i][16 jb .. 16 jb + 15] in fp32.
-__global__ void __launch_bounds__(256) gram_counts_kernel(const float* __restrict__ H, int64_t N,
-                                                          int L, int E, int kf,
-                                                          float* __restrict__ gpart,
-                                                          int32_t* __restrict__ cpart) {
-  __shared__ float sh[kSub][65];
-  __shared__ int cnt[64];
+// grid (chunks, L), 256 threads. Partial Gram of layer l over one chunk of
+// tokens: thread (ti, tj) of a 16 x 16 grid accumulates the 4 x 4 block
+// G[4 ti .. 4 ti + 3][4 tj .. 4 tj + 3] in fp32; each staged token costs two
+// float4 shared loads per 16 FMAs.
+__global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ H, int64_t N, int L,
+                                                   int E, float* __restrict__ gpart) {
+  __shared__ __align__(16) float sh[kSub][64];
   const int chunk = blockIdx.x, l = blockIdx.y;
   const int nchunks = gridDim.x;
   const int tid = threadIdx.x;
-  const int i = tid >> 2, j0 = (tid & 3) * 16;
+  const int ti = tid >> 4, tj = tid & 15;
   const int LE = L * E;
-  float acc[16];
+  float acc[4][4];
 #pragma unroll
-  for (int q = 0; q < 16; ++q) acc[q] = 0.0f;
-  if (tid < 64) cnt[tid] = 0;
+  for (int a = 0; a < 4; ++a)
+#pragma unroll
+    for (int b = 0; b < 4; ++b) acc[a][b] = 0.0f;
   const int64_t n_begin = (int64_t)chunk * kSimChunk;
   int64_t n_end = n_begin + kSimChunk;
   if (n_end > N) n_end = N;
+  const bool active = 4 * ti < E && 4 * tj < E;
   for (int64_t n0 = n_begin; n0 < n_end; n0 += kSub) {
     __syncthreads();
-    for (int x = tid; x < kSub * E; x += 256) {
-      const int r = x / E, c = x % E;
+    for (int x = tid; x < kSub * 64; x += 256) {
+      const int r = x >> 6, c = x & 63;
       const int64_t n = n0 + r;
-      sh[r][c] = (n < n_end) ? H[n * LE + (int64_t)l * E + c] : 0.0f;
+      sh[r][c] = (n < n_end && c < E) ? H[n * LE + (int64_t)l * E + c] : 0.0f;
     }
     __syncthreads();
-    if (i < E) {
+    if (active) {
+#pragma unroll 4
       for (int r = 0; r < kSub; ++r) {
-        const float a = sh[r][i];
-#pragma unroll
-        for (int q = 0; q < 16; ++q) acc[q] = fmaf(a, sh[r][j0 + q], acc[q]);
+        const float4 a = *reinterpret_cast<const float4*>(&sh[r][4 * ti]);
+        const float4 b = *reinterpret_cast<const float4*>(&sh[r][4 * tj]);
+#define OM_GRAM_ROW(p, ap)                       \
+  acc[p][0] = fmaf(ap, b.x, acc[p][0]);          \
+  acc[p][1] = fmaf(ap, b.y, acc[p][1]);          \
+  acc[p][2] = fmaf(ap, b.z, acc[p][2]);          \
+  acc[p][3] = fmaf(ap, b.w, acc[p][3]);
+        OM_GRAM_ROW(0, a.x) OM_GRAM_ROW(1, a.y) OM_GRAM_ROW(2, a.z) OM_GRAM_ROW(3, a.w)
+#undef OM_GRAM_ROW
       }
     }
-    if (tid < kSub && n0 + tid < n_end) add_topk_counts(&sh[tid][0], E, kf, cnt);
+  }
+  float* gp = gpart + ((size_t)l * nchunks + chunk) * 64 * 64;
+  if (active)
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) gp[(4 * ti + p) * 64 + 4 * tj + q] = acc[p][q];
+}
+
+// Eq. 5 counts from the token-major logits H[n][l E + e]: one warp per
+// (token, layer); lane e holds experts e and e + 32; k_freq warp-wide argmax
+// rounds (larger logit first, lower index on ties). Block totals are added
+// with integer atomics, so the result does not depend on the order.
+__global__ void __launch_bounds__(256) counts_kernel(const float* __restrict__ H, int64_t N, int L,
+                                                     int E, int kf, int32_t* __restrict__ counts) {
+  __shared__ int cnt[64];
+  const int lane = threadIdx.x & 31;
+  const int l = blockIdx.y;
+  if (threadIdx.x < 64) cnt[threadIdx.x] = 0;
+  __syncthreads();
+  const int64_t warps_total = (int64_t)gridDim.x * (blockDim.x >> 5);
+  const int LE = L * E;
+  for (int64_t n = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); n < N;
+       n += warps_total) {
+    const float* row = H + n * LE + (int64_t)l * E;
+    float v0 = lane < E ? row[lane] : -INFINITY;
+    float v1 = lane + 32 < E ? row[lane + 32] : -INFINITY;
+    bool u0 = lane >= E, u1 = lane + 32 >= E;  // used or absent
+    for (int j = 0; j < kf; ++j) {
+      // best of this lane: (value desc, index asc) over its unused entries
+      float bv = -INFINITY;
+      int bi = 1 << 30;
+      if (!u0) { bv = v0; bi = lane; }
+      if (!u1 && (bi == (1 << 30) || v1 > bv)) { bv = v1; bi = lane + 32; }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (oi != (1 << 30) && (bi == (1 << 30) || ov > bv || (ov == bv && oi < bi))) {
+          bv = ov;
+          bi = oi;
+        }
+      }
+      if (bi == lane) u0 = true;
+      if (bi == lane + 32) u1 = true;
+      if (lane == 0 && bi < E) atomicAdd(&cnt[bi], 1);
+    }
   }
   __syncthreads();
-  float* gp = gpart + ((size_t)l * nchunks + chunk) * 64 * 64;
-  if (i < E)
-#pragma unroll
-    for (int q = 0; q < 16; ++q) gp[i * 64 + j0 + q] = acc[q];
-  if (tid < E) cpart[((size_t)l * nchunks + chunk) * 64 + tid] = cnt[tid];
+  if (threadIdx.x < E && cnt[threadIdx.x]) atomicAdd(&counts[(size_t)l * E + threadIdx.x], cnt[threadIdx.x]);
 }
 
 // grid L, 256 threads: G = sum of the partial Grams in chunk order (fp64),
 // Sim(i,j) = G_ij / (sqrt(G_ii) sqrt(G_jj)) (Eq. 4), diagonal 1, zero-norm 0.
 __global__ void __launch_bounds__(256) sim_finish_kernel(const float* __restrict__ gpart,
-                                                         const int32_t* __restrict__ cpart,
-                                                         int nchunks, int E, float* __restrict__ sim,
-                                                         int32_t* __restrict__ counts) {
+                                                         int nchunks, int E, float* __restrict__ sim) {
   __shared__ double G[64 * 64];
   const int l = blockIdx.x;
   for (int x = threadIdx.x; x < E * E; x += blockDim.x) {
@@ -97,11 +145,6 @@ __global__ void __launch_bounds__(256) sim_finish_kernel(const float* __restrict
     for (int c = 0; c < nchunks; ++c)
       s += static_cast<double>(gpart[((size_t)l * nchunks + c) * 4096 + i * 64 + j]);
     G[i * 64 + j] = s;
-  }
-  for (int e = threadIdx.x; e < E; e += blockDim.x) {
-    int s = 0;
-    for (int c = 0; c < nchunks; ++c) s += cpart[((size_t)l * nchunks + c) * 64 + e];
-    counts[(size_t)l * E + e] = s;
   }
   __syncthreads();
   for (int x = threadIdx.x; x < E * E; x += blockDim.x) {
@@ -275,9 +318,8 @@ extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
   const int64_t nchunks = (N + kSimChunk - 1) / kSimChunk;
   const size_t h = (size_t)N * L * E * sizeof(float);
   const size_t g = (size_t)L * nchunks * 64 * 64 * sizeof(float);
-  const size_t c = (size_t)L * nchunks * 64 * sizeof(int32_t);
   auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
-  return up(h) + up(g) + up(c);
+  return up(h) + up(g);
 }
 
 extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
@@ -301,13 +343,16 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   float* H = reinterpret_cast<float*>(ws);
   float* gpart = reinterpret_cast<float*>(ws + up((size_t)N * L * E * sizeof(float)));
-  int32_t* cpart = reinterpret_cast<int32_t*>(reinterpret_cast<uint8_t*>(gpart) +
-                                              up((size_t)L * nchunks * 64 * 64 * sizeof(float)));
   int rc = logits_gemm_launch(X_cal, static_cast<int>(N), W_r, L * E, d, H, stream);
   if (rc) return rc;
-  gram_counts_kernel<<<dim3(nchunks, L), 256, 0, stream>>>(H, N, L, E, k_freq, gpart, cpart);
-  OM_LAUNCHED("gram_counts_kernel");
-  sim_finish_kernel<<<L, 256, 0, stream>>>(gpart, cpart, nchunks, E, sim, counts);
+  OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, stream));
+  int64_t cblocks = (N + 7) / 8;
+  if (cblocks > num_sms() * 8) cblocks = num_sms() * 8;
+  counts_kernel<<<dim3(static_cast<unsigned>(cblocks), L), 256, 0, stream>>>(H, N, L, E, k_freq, counts);
+  OM_LAUNCHED("counts_kernel");
+  gram_kernel<<<dim3(nchunks, L), 256, 0, stream>>>(H, N, L, E, gpart);
+  OM_LAUNCHED("gram_kernel");
+  sim_finish_kernel<<<L, 256, 0, stream>>>(gpart, nchunks, E, sim);
   OM_LAUNCHED("sim_finish_kernel");
   return ORDERMOE_OK;
 }
