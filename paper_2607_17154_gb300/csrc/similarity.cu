@@ -20,7 +20,7 @@ int read_clear_err_sim(unsigned long long* out) {
   return ORDERMOE_OK;
 }
 
-constexpr int kSimChunk = 4096;  // calibration tokens per partial Gram
+constexpr int kSimChunk = 1024;  // calibration tokens per partial Gram
 constexpr int kSub = 64;         // tokens staged in shared memory at a time
 
 // Rank order used for top-k: larger logit first, equal logits by lower index.
@@ -61,10 +61,24 @@ __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ H, 
   const bool active = 4 * ti < E && 4 * tj < E;
   for (int64_t n0 = n_begin; n0 < n_end; n0 += kSub) {
     __syncthreads();
-    for (int x = tid; x < kSub * 64; x += 256) {
-      const int r = x >> 6, c = x & 63;
-      const int64_t n = n0 + r;
-      sh[r][c] = (n < n_end && c < E) ? H[n * LE + (int64_t)l * E + c] : 0.0f;
+    if ((E & 3) == 0 && (LE & 3) == 0) {
+      // 16 float4 per token row; each thread stages 4 of the 1024 float4
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int x = tid + 256 * u;
+        const int r = x >> 4, c4 = (x & 15) * 4;
+        const int64_t n = n0 + r;
+        float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        if (n < n_end && c4 < E)
+          v = *reinterpret_cast<const float4*>(H + n * LE + (int64_t)l * E + c4);
+        *reinterpret_cast<float4*>(&sh[r][c4]) = v;
+      }
+    } else {
+      for (int x = tid; x < kSub * 64; x += 256) {
+        const int r = x >> 6, c = x & 63;
+        const int64_t n = n0 + r;
+        sh[r][c] = (n < n_end && c < E) ? H[n * LE + (int64_t)l * E + c] : 0.0f;
+      }
     }
     __syncthreads();
     if (active) {
@@ -190,14 +204,23 @@ __global__ void __launch_bounds__(64) place_kernel(
     int32_t* __restrict__ group, int32_t* __restrict__ n_groups, float* __restrict__ theta_out,
     uint8_t* __restrict__ placement, double* __restrict__ used, int32_t* __restrict__ status) {
   __shared__ double b[32];
+  __shared__ double Cs[32];
   __shared__ double imp[64];
+  __shared__ double pls[64];
   __shared__ int order[64];
   __shared__ int dom[64];
   __shared__ int grp[64];
+  __shared__ int cnt[64];
   __shared__ int waiting[64];
+  __shared__ uint8_t xs[32 * 64];   // placement of the current layer, [m][e]
+  __shared__ int eta[32 * 64];      // experts of group g already on server m, [m][g]
+  __shared__ float S[64 * 64];      // Sim of the current layer
   __shared__ int overflow;
   const int t = threadIdx.x;
-  if (t < M) b[t] = 0.0;
+  if (t < M) {
+    b[t] = 0.0;
+    Cs[t] = C[t];
+  }
   if (t == 0) {
     double need = 0.0, have = 0.0;
     for (int i = 0; i < L * E; ++i) need = __dadd_rn(need, p[i]);
@@ -206,10 +229,16 @@ __global__ void __launch_bounds__(64) place_kernel(
   }
   __syncthreads();
   for (int l = 0; l < L; ++l) {
-    const float* S = sim + (size_t)l * E * E;
-    const int32_t* cn = counts + (size_t)l * E;
-    const double* pl = p + (size_t)l * E;
-    uint8_t* x = placement + (size_t)l * M * E;
+    for (int i = t; i < E * E; i += blockDim.x) S[i] = sim[(size_t)l * E * E + i];
+    for (int i = t; i < M * 64; i += blockDim.x) {
+      xs[i] = 0;
+      eta[i] = 0;
+    }
+    if (t < E) {
+      cnt[t] = counts[(size_t)l * E + t];
+      pls[t] = p[(size_t)l * E + t];
+    }
+    __syncthreads();
     // Eq. 6 (layers numbered from 1)
     float theta;
     if (L <= 1) {
@@ -223,10 +252,9 @@ __global__ void __launch_bounds__(64) place_kernel(
     if (t < E) {
       int r = 0;
       for (int e = 0; e < E; ++e)
-        if (cn[e] > cn[t] || (cn[e] == cn[t] && e < t)) ++r;
+        if (cnt[e] > cnt[t] || (cnt[e] == cnt[t] && e < t)) ++r;
       order[r] = t;
     }
-    for (int i = t; i < M * E; i += blockDim.x) x[i] = 0;
     __syncthreads();
     // Eqs. 24-26, sequential in the visiting order
     if (t == 0) {
@@ -236,8 +264,8 @@ __global__ void __launch_bounds__(64) place_kernel(
         int bg = -1;
         float bs = 0.0f;
         for (int g = 0; g < k; ++g) {
-          const float s = S[j * E + dom[g]];
-          if (bg < 0 || s > bs) { bg = g; bs = s; }
+          const float sv = S[j * E + dom[g]];
+          if (bg < 0 || sv > bs) { bg = g; bs = sv; }
         }
         if (bg < 0 || bs < theta) { dom[k] = j; grp[j] = k; ++k; }
         else grp[j] = bg;
@@ -248,15 +276,15 @@ __global__ void __launch_bounds__(64) place_kernel(
     __syncthreads();
     // Eqs. 27-28
     double total = 0.0;
-    for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cn[e]));
+    for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cnt[e]));
     if (t < E) {
       group[(size_t)l * E + t] = grp[t];
-      double s = 0.0;
+      double sum = 0.0;
       int size = 0;
       for (int k2 = 0; k2 < E; ++k2)
-        if (grp[k2] == grp[t]) { s = __dadd_rn(s, static_cast<double>(S[t * E + k2])); ++size; }
-      const double rho = __ddiv_rn(s, static_cast<double>(size));
-      const double f = total > 0.0 ? __ddiv_rn(static_cast<double>(cn[t]), total) : 0.0;
+        if (grp[k2] == grp[t]) { sum = __dadd_rn(sum, static_cast<double>(S[t * E + k2])); ++size; }
+      const double rho = __ddiv_rn(sum, static_cast<double>(size));
+      const double f = total > 0.0 ? __ddiv_rn(static_cast<double>(cnt[t]), total) : 0.0;
       imp[t] = __dadd_rn(__dmul_rn(pp.alpha_f, f), __dmul_rn(pp.alpha_r, rho));
     }
     __syncthreads();
@@ -265,7 +293,7 @@ __global__ void __launch_bounds__(64) place_kernel(
       int r = 0;
       for (int e = 0; e < E; ++e) {
         bool before;
-        if (pl[e] != pl[t]) before = pl[e] > pl[t];
+        if (pls[e] != pls[t]) before = pls[e] > pls[t];
         else if (imp[e] != imp[t]) before = imp[e] > imp[t];
         else before = e < t;
         if (before) ++r;
@@ -273,36 +301,39 @@ __global__ void __launch_bounds__(64) place_kernel(
       order[r] = t;
     }
     __syncthreads();
-    // Eqs. 29-31, sequential; waiting list to the server with the most room
+    // Eqs. 29-31, sequential; eta from the per-(server, group) counts
     if (t == 0) {
       int nw = 0;
       for (int pos = 0; pos < E; ++pos) {
         const int j = order[pos];
+        const int g = grp[j];
         int best = -1;
         double bsc = 0.0;
         for (int m = 0; m < M; ++m) {
-          if (!(__dadd_rn(b[m], pl[j]) <= C[m])) continue;
-          int eta = 0;
-          for (int k2 = 0; k2 < E; ++k2)
-            if (grp[k2] == grp[j] && x[m * E + k2]) ++eta;
-          const double sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[m], C[m])),
-                                      __dmul_rn(pp.lambda2, static_cast<double>(eta)));
+          if (!(__dadd_rn(b[m], pls[j]) <= Cs[m])) continue;
+          const double sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[m], Cs[m])),
+                                      __dmul_rn(pp.lambda2, static_cast<double>(eta[m * 64 + g])));
           if (best < 0 || sc < bsc) { best = m; bsc = sc; }
         }
         if (best < 0) { waiting[nw++] = j; continue; }
-        x[best * E + j] = 1;
-        b[best] = __dadd_rn(b[best], pl[j]);
+        xs[best * 64 + j] = 1;
+        eta[best * 64 + g] += 1;
+        b[best] = __dadd_rn(b[best], pls[j]);
       }
       for (int w = 0; w < nw; ++w) {
         const int j = waiting[w];
         int best = 0;
         for (int m = 1; m < M; ++m)
-          if (__dsub_rn(C[m], b[m]) > __dsub_rn(C[best], b[best])) best = m;
-        x[best * E + j] = 1;
-        b[best] = __dadd_rn(b[best], pl[j]);
-        if (b[best] > C[best]) overflow = 1;
+          if (__dsub_rn(Cs[m], b[m]) > __dsub_rn(Cs[best], b[best])) best = m;
+        xs[best * 64 + j] = 1;
+        eta[best * 64 + grp[j]] += 1;
+        b[best] = __dadd_rn(b[best], pls[j]);
+        if (b[best] > Cs[best]) overflow = 1;
       }
     }
+    __syncthreads();
+    uint8_t* x = placement + (size_t)l * M * E;
+    for (int i = t; i < M * E; i += blockDim.x) x[i] = xs[(i / E) * 64 + (i % E)];
     __syncthreads();
   }
   if (t < M) used[t] = b[t];
