@@ -3,7 +3,7 @@
 
 One step = one pass of the hot path over one batch: router + softmax + top-k
 + server-expert selection, permutation, grouped SwiGLU expert FFN (gate/up,
-down) and weighted combine -- seven kernels of libordermoe.so, nothing else.
+down) and weighted combine -- eight kernels of libordermoe.so, nothing else.
 Default workload: the Mixtral-8x7B-shaped prefill layer (T = 4096 tokens,
 d = 4096, E = 8, top-2, d_ff = 14336, 4 logical servers), synthetic seeded
 inputs drawn on the device. The offline plan (similarity, grouping,
@@ -248,7 +248,19 @@ def run_ours(args, dist):
         B.ordermoe_expert_down(H, offsets, R, W2, E, d, dff, Yp)
         B.ordermoe_combine(Yp, row_of, wts, T, k, d, y)
 
-    KERNELS_PER_STEP = 7   # route_select 1, dispatch 3, gate/up 1, down 1, combine 1
+    def step_phases():
+        return [
+            ("route_select", lambda: B.ordermoe_route_select(X, Wr, None, T, E, d, k, 1, tables, home,
+                                                              None, None, None, idx, wts, ch, sv, kd,
+                                                              None)),
+            ("dispatch", lambda: B.ordermoe_dispatch(ch, X, T, k, E, d, offsets, row_token, row_of,
+                                                     Xp, ws)),
+            ("expert_gate_up", lambda: B.ordermoe_expert_gate_up(Xp, offsets, R, W1, W3, E, d, dff, H)),
+            ("expert_down", lambda: B.ordermoe_expert_down(H, offsets, R, W2, E, d, dff, Yp)),
+            ("combine", lambda: B.ordermoe_combine(Yp, row_of, wts, T, k, d, y)),
+        ]
+
+    KERNELS_PER_STEP = 8   # route_select 1, dispatch 4, gate/up 1, down 1, combine 1
     step(cnt=counters)     # one counted pass for the execution-type breakdown
     for _ in range(max(args.warmup, 3)):
         step()
@@ -272,6 +284,7 @@ def run_ours(args, dist):
     if code:
         raise RuntimeError("device error %d (%d) during the timed steps" % (code, detail))
     elapsed_ms = dist.max(elapsed_ms, device)
+    breakdown = phase_breakdown(step_phases, stream, reps=20)
     total_tokens = T * args.steps * dist.world
     value = total_tokens / (elapsed_ms / 1e3)
 
@@ -327,6 +340,7 @@ def run_ours(args, dist):
                      "layer_tflops": round(layer_flop / (elapsed_ms / args.steps / 1e3) / 1e12, 1)},
         "e2e": e2e,
         "gpu_launches": KERNELS_PER_STEP * args.steps,
+        "breakdown_ms": breakdown,
         "clocks": clocks,
         "exec_types": dict(zip(["local_exact", "local_sub", "remote_exact", "remote_sub"],
                                counters.cpu().tolist())),
@@ -336,6 +350,22 @@ def run_ours(args, dist):
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, inp, args.seed, args.cpu_seconds)
     return out
+
+
+def phase_breakdown(phases_fn, stream, reps=20):
+    """Mean time of each phase of a step (CUDA events around each C-ABI call),
+    measured after the timed region; informational, not part of `value`."""
+    import torch
+    names = [n for n, _ in phases_fn()]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)] for _ in range(reps)]
+    for r in range(reps):
+        ev[r][0].record(stream)
+        for i, (_, fn) in enumerate(phases_fn()):
+            fn()
+            ev[r][i + 1].record(stream)
+    torch.cuda.synchronize()
+    return {n: round(statistics.mean(ev[r][i].elapsed_time(ev[r][i + 1]) for r in range(reps)), 4)
+            for i, n in enumerate(names)}
 
 
 def timed_region(args, dist, device, fn):
