@@ -77,21 +77,29 @@ struct Args {
   uint16_t* out;     // H [R][d_ff] or Y [R][d]
   int ldo;           // row length of out
   uint64_t limit_ns; // bounded-wait limit
+  int m_major;       // 1: all N slices of an M tile back to back (A read once from HBM)
 };
 
 struct Tile {
   int e, m0, m_end, n;
 };
 
-__device__ __forceinline__ Tile decode(int tile, const Smem& s, int E, int n_tiles) {
+__device__ __forceinline__ Tile decode(int tile, const Smem& s, int E, int n_tiles, int m_major) {
   int e = 0;
   while (e < E - 1 && s.mt_start[e + 1] * n_tiles <= tile) ++e;
   const int local = tile - s.mt_start[e] * n_tiles;
   const int n_mt = s.mt_start[e + 1] - s.mt_start[e];
   Tile t;
   t.e = e;
-  t.n = local / n_mt;
-  t.m0 = s.offs[e] + (local - t.n * n_mt) * BM;
+  int mt;
+  if (m_major) {
+    mt = local / n_tiles;
+    t.n = local - mt * n_tiles;
+  } else {
+    t.n = local / n_mt;
+    mt = local - t.n * n_mt;
+  }
+  t.m0 = s.offs[e] + mt * BM;
   t.m_end = s.offs[e + 1];
   return t;
 }
@@ -165,7 +173,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x) {
-        const Tile t = decode(tile, s, args.E, args.n_tiles);
+        const Tile t = decode(tile, s, args.E, args.n_tiles, args.m_major);
         const int brow = t.e * args.b_rows + t.n * (MODE == GATEUP ? 128 : 256);  // LOGITS: e == 0
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
@@ -246,7 +254,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       tc_fence_after();
-      const Tile t = decode(tile, s, args.E, args.n_tiles);
+      const Tile t = decode(tile, s, args.E, args.n_tiles, args.m_major);
       const int row = t.m0 + lrow;
       const bool valid = row < t.m_end;
       const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
@@ -769,6 +777,7 @@ int logits_gemm_launch(const uint16_t* X, int N, const uint16_t* W, int C, int d
   a.n_tiles = (C + 255) / 256;
   a.b_rows = 0;
   a.limit_ns = wait_limit_ns();
+  a.m_major = 1;  // the stacked router rows (a few MB) stay in L2; X_cal streams once
   const long long tiles = (long long)((N + BM - 1) / BM) * a.n_tiles;
   const int sms = num_sms();
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);

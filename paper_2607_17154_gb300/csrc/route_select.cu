@@ -108,15 +108,18 @@ __global__ void __launch_bounds__(256) route_select_kernel(
     float* __restrict__ qhat, float* __restrict__ logits_out, int32_t* __restrict__ topk_idx,
     float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
     uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
-    int32_t* __restrict__ counters) {
+    int32_t* __restrict__ counters, int stage_w) {
   __shared__ uint32_t s_pmask[64];
   __shared__ unsigned long long s_subst[64];
   __shared__ uint8_t s_sublist[64 * 64];
   __shared__ int s_nsub[64];
   __shared__ int s_kind[4];
-  extern __shared__ float s_dyn[];  // Qtab[E*E], Cq[E*E]
+  extern __shared__ __align__(16) float s_dyn[];  // Qtab[E*E], Cq[E*E], then W_r if staged
   float* s_Q = s_dyn;
   float* s_Cq = s_dyn + E * E;
+  // W_r staged in shared memory when it fits (stage_w): every token of the
+  // block then reads it at shared-memory latency instead of from L2.
+  uint4* s_W = reinterpret_cast<uint4*>(s_dyn + ((2 * E * E + 3) & ~3));
 
   const int M = reinterpret_cast<const int32_t*>(tab)[2];
   if (reinterpret_cast<const int32_t*>(tab)[1] != E || M <= 0 || M > 32) {
@@ -143,6 +146,10 @@ __global__ void __launch_bounds__(256) route_select_kernel(
   for (int i = threadIdx.x; i < E * E; i += blockDim.x) {
     s_Q[i] = gQ[i];
     s_Cq[i] = gCq[i];
+  }
+  if (stage_w && logits_in == nullptr) {
+    const uint4* gw = reinterpret_cast<const uint4*>(Wr);
+    for (int i = threadIdx.x; i < E * (d >> 3); i += blockDim.x) s_W[i] = __ldg(gw + i);
   }
   if (threadIdx.x < 4) s_kind[threadIdx.x] = 0;
   __syncthreads();
@@ -182,7 +189,8 @@ __global__ void __launch_bounds__(256) route_select_kernel(
 #pragma unroll
           for (int e = 0; e < EMAX; ++e) {
             if (e < E) {
-              const uint4 wv = __ldg(reinterpret_cast<const uint4*>(Wr + (size_t)e * d) + c);
+              const uint4 wv = stage_w ? s_W[e * nvec + c]
+                                       : __ldg(reinterpret_cast<const uint4*>(Wr + (size_t)e * d) + c);
               float a = lg[e];
               a = fmaf(x0, bf16_lo(wv.x), a); a = fmaf(x1, bf16_hi(wv.x), a);
               a = fmaf(x2, bf16_lo(wv.y), a); a = fmaf(x3, bf16_hi(wv.y), a);
@@ -398,9 +406,14 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
   const int threads = 256;
   const int per_block = threads / 32;
   int blocks = (T + per_block - 1) / per_block;
-  const int cap = num_sms() * 8;
+  // Stage W_r in shared memory when it fits in 96 KB; the grid is then a few
+  // persistent blocks per SM so that each block loads it once.
+  const size_t tab_bytes = sizeof(float) * ((2 * E * E + 3) & ~3);
+  const size_t w_bytes = (size_t)E * d * 2;
+  const int stage_w = (logits_in == nullptr && w_bytes <= 96 * 1024) ? 1 : 0;
+  const int cap = num_sms() * (stage_w ? 2 : 8);
   if (blocks > cap) blocks = cap;
-  const size_t dyn = sizeof(float) * 2 * E * E;
+  const size_t dyn = tab_bytes + (stage_w ? w_bytes : 0);
   const uint8_t* tb = static_cast<const uint8_t*>(tables);
 #define OM_RS_LAUNCH(EM)                                                                        \
   do {                                                                                          \
@@ -408,7 +421,7 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
                          (int)dyn);                                                             \
     route_select_kernel<EM><<<blocks, threads, dyn, stream>>>(                                  \
         X, W_r, logits_in, T, E, d, k, renorm, tb, home, loc, qhat, logits_out, topk_idx,       \
-        topk_w, chosen_expert, chosen_server, kind, counters);                                  \
+        topk_w, chosen_expert, chosen_server, kind, counters, stage_w);                         \
   } while (0)
   if (E <= 8) OM_RS_LAUNCH(8);
   else if (E <= 16) OM_RS_LAUNCH(16);

@@ -147,20 +147,31 @@ __global__ void __launch_bounds__(256) counts_kernel(const float* __restrict__ H
   if (threadIdx.x < E && cnt[threadIdx.x]) atomicAdd(&counts[(size_t)l * E + threadIdx.x], cnt[threadIdx.x]);
 }
 
-// grid L, 256 threads: G = sum of the partial Grams in chunk order (fp64),
-// Sim(i,j) = G_ij / (sqrt(G_ii) sqrt(G_jj)) (Eq. 4), diagonal 1, zero-norm 0.
-__global__ void __launch_bounds__(256) sim_finish_kernel(const float* __restrict__ gpart,
-                                                         int nchunks, int E, float* __restrict__ sim) {
-  __shared__ double G[64 * 64];
+// grid (L, 16), 256 threads: block (l, b) reduces the 256 Gram entries
+// i * 64 + j in [256 b, 256 b + 256) over the chunks, in chunk order (fp64).
+__global__ void __launch_bounds__(256) gram_reduce_kernel(const float* __restrict__ gpart,
+                                                          int nchunks, double* __restrict__ G) {
   const int l = blockIdx.x;
-  for (int x = threadIdx.x; x < E * E; x += blockDim.x) {
-    const int i = x / E, j = x % E;
-    double s = 0.0;
-    for (int c = 0; c < nchunks; ++c)
-      s += static_cast<double>(gpart[((size_t)l * nchunks + c) * 4096 + i * 64 + j]);
-    G[i * 64 + j] = s;
+  const int x = blockIdx.y * 256 + threadIdx.x;
+  const float* src = gpart + (size_t)l * nchunks * 4096 + x;
+  double s = 0.0;
+  int c = 0;
+  for (; c + 8 <= nchunks; c += 8) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = src[(size_t)(c + u) * 4096];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) s += static_cast<double>(v[u]);
   }
-  __syncthreads();
+  for (; c < nchunks; ++c) s += static_cast<double>(src[(size_t)c * 4096]);
+  G[(size_t)l * 4096 + x] = s;
+}
+
+// grid L: Sim(i,j) = G_ij / (sqrt(G_ii) sqrt(G_jj)) (Eq. 4), diagonal 1, zero-norm 0.
+__global__ void __launch_bounds__(256) sim_finish_kernel(const double* __restrict__ Gall, int E,
+                                                         float* __restrict__ sim) {
+  const int l = blockIdx.x;
+  const double* G = Gall + (size_t)l * 4096;
   for (int x = threadIdx.x; x < E * E; x += blockDim.x) {
     const int i = x / E, j = x % E;
     float v;
@@ -349,8 +360,9 @@ extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
   const int64_t nchunks = (N + kSimChunk - 1) / kSimChunk;
   const size_t h = (size_t)N * L * E * sizeof(float);
   const size_t g = (size_t)L * nchunks * 64 * 64 * sizeof(float);
+  const size_t gd = (size_t)L * 64 * 64 * sizeof(double);
   auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
-  return up(h) + up(g);
+  return up(h) + up(g) + up(gd);
 }
 
 extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
@@ -374,6 +386,8 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   float* H = reinterpret_cast<float*>(ws);
   float* gpart = reinterpret_cast<float*>(ws + up((size_t)N * L * E * sizeof(float)));
+  double* G = reinterpret_cast<double*>(reinterpret_cast<uint8_t*>(gpart) +
+                                        up((size_t)L * nchunks * 64 * 64 * sizeof(float)));
   int rc = logits_gemm_launch(X_cal, static_cast<int>(N), W_r, L * E, d, H, stream);
   if (rc) return rc;
   OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, stream));
@@ -383,7 +397,9 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
   OM_LAUNCHED("counts_kernel");
   gram_kernel<<<dim3(nchunks, L), 256, 0, stream>>>(H, N, L, E, gpart);
   OM_LAUNCHED("gram_kernel");
-  sim_finish_kernel<<<L, 256, 0, stream>>>(gpart, nchunks, E, sim);
+  gram_reduce_kernel<<<dim3(L, 16), 256, 0, stream>>>(gpart, nchunks, G);
+  OM_LAUNCHED("gram_reduce_kernel");
+  sim_finish_kernel<<<L, 256, 0, stream>>>(G, E, sim);
   OM_LAUNCHED("sim_finish_kernel");
   return ORDERMOE_OK;
 }
