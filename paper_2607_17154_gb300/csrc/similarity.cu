@@ -104,43 +104,49 @@ __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ H, 
       for (int q = 0; q < 4; ++q) gp[(4 * ti + p) * 64 + 4 * tj + q] = acc[p][q];
 }
 
-// Eq. 5 counts from the token-major logits H[n][l E + e]: one warp per
-// (token, layer); lane e holds experts e and e + 32; k_freq warp-wide argmax
-// rounds (larger logit first, lower index on ties). Block totals are added
+// Eq. 5 counts from the token-major logits H[n][l E + e]: one thread per
+// (token, layer) holds the layer's E logits in registers and takes k_freq
+// passes (larger logit first, lower index on ties). Block totals are added
 // with integer atomics, so the result does not depend on the order.
+template <int EMAX>
 __global__ void __launch_bounds__(256) counts_kernel(const float* __restrict__ H, int64_t N, int L,
                                                      int E, int kf, int32_t* __restrict__ counts) {
   __shared__ int cnt[64];
-  const int lane = threadIdx.x & 31;
   const int l = blockIdx.y;
   if (threadIdx.x < 64) cnt[threadIdx.x] = 0;
   __syncthreads();
-  const int64_t warps_total = (int64_t)gridDim.x * (blockDim.x >> 5);
   const int LE = L * E;
-  for (int64_t n = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); n < N;
-       n += warps_total) {
+  const bool vec = (E & 3) == 0 && (LE & 3) == 0;
+  for (int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; n < N;
+       n += (int64_t)gridDim.x * blockDim.x) {
     const float* row = H + n * LE + (int64_t)l * E;
-    float v0 = lane < E ? row[lane] : -INFINITY;
-    float v1 = lane + 32 < E ? row[lane + 32] : -INFINITY;
-    bool u0 = lane >= E, u1 = lane + 32 >= E;  // used or absent
-    for (int j = 0; j < kf; ++j) {
-      // best of this lane: (value desc, index asc) over its unused entries
-      float bv = -INFINITY;
-      int bi = 1 << 30;
-      if (!u0) { bv = v0; bi = lane; }
-      if (!u1 && (bi == (1 << 30) || v1 > bv)) { bv = v1; bi = lane + 32; }
+    float v[EMAX];
+    if (vec) {
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-        if (oi != (1 << 30) && (bi == (1 << 30) || ov > bv || (ov == bv && oi < bi))) {
-          bv = ov;
-          bi = oi;
+      for (int e = 0; e < EMAX; e += 4) {
+        if (e < E) {
+          const float4 q = *reinterpret_cast<const float4*>(row + e);
+          v[e] = q.x; v[e + 1] = q.y; v[e + 2] = q.z; v[e + 3] = q.w;
         }
       }
-      if (bi == lane) u0 = true;
-      if (bi == lane + 32) u1 = true;
-      if (lane == 0 && bi < E) atomicAdd(&cnt[bi], 1);
+    } else {
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e)
+        if (e < E) v[e] = row[e];
+    }
+    unsigned long long used = 0;
+    for (int j = 0; j < kf; ++j) {
+      int best = -1;
+      float bv = 0.0f;
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e) {
+        if (e < E && !((used >> e) & 1ull) && (best < 0 || v[e] > bv)) {
+          best = e;
+          bv = v[e];
+        }
+      }
+      used |= 1ull << best;
+      atomicAdd(&cnt[best], 1);
     }
   }
   __syncthreads();
@@ -267,22 +273,40 @@ __global__ void __launch_bounds__(64) place_kernel(
       order[r] = t;
     }
     __syncthreads();
-    // Eqs. 24-26, sequential in the visiting order
-    if (t == 0) {
+    // Eqs. 24-26 in the visiting order; warp 0 scans the existing dominants
+    // in parallel (lane g takes dominants g and g + 32; argmax ties to the
+    // earlier dominant).
+    if (t < 32) {
       int k = 0;
       for (int pos = 0; pos < E; ++pos) {
         const int j = order[pos];
-        int bg = -1;
-        float bs = 0.0f;
-        for (int g = 0; g < k; ++g) {
+        float bs = -INFINITY;
+        int bg = 1 << 30;
+        for (int g = t; g < k; g += 32) {
           const float sv = S[j * E + dom[g]];
-          if (bg < 0 || sv > bs) { bg = g; bs = sv; }
+          if (bg == (1 << 30) || sv > bs) { bg = g; bs = sv; }
         }
-        if (bg < 0 || bs < theta) { dom[k] = j; grp[j] = k; ++k; }
-        else grp[j] = bg;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+          const int og = __shfl_xor_sync(0xffffffffu, bg, o);
+          if (og != (1 << 30) && (bg == (1 << 30) || os > bs || (os == bs && og < bg))) {
+            bs = os;
+            bg = og;
+          }
+        }
+        if (bg == (1 << 30) || bs < theta) {
+          if (t == 0) { dom[k] = j; grp[j] = k; }
+          ++k;
+        } else if (t == 0) {
+          grp[j] = bg;
+        }
+        __syncwarp();
       }
-      n_groups[l] = k;
-      theta_out[l] = theta;
+      if (t == 0) {
+        n_groups[l] = k;
+        theta_out[l] = theta;
+      }
     }
     __syncthreads();
     // Eqs. 27-28
@@ -312,34 +336,49 @@ __global__ void __launch_bounds__(64) place_kernel(
       order[r] = t;
     }
     __syncthreads();
-    // Eqs. 29-31, sequential; eta from the per-(server, group) counts
-    if (t == 0) {
+    // Eqs. 29-31 in the placement order; warp 0 scores the servers in
+    // parallel (lane m = server m) and takes the lowest score, ties to the
+    // lower server; eta comes from the per-(server, group) counts.
+    if (t < 32) {
       int nw = 0;
       for (int pos = 0; pos < E; ++pos) {
         const int j = order[pos];
         const int g = grp[j];
-        int best = -1;
-        double bsc = 0.0;
-        for (int m = 0; m < M; ++m) {
-          if (!(__dadd_rn(b[m], pls[j]) <= Cs[m])) continue;
-          const double sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[m], Cs[m])),
-                                      __dmul_rn(pp.lambda2, static_cast<double>(eta[m * 64 + g])));
-          if (best < 0 || sc < bsc) { best = m; bsc = sc; }
+        double sc = 0.0;
+        int m = (t < M && __dadd_rn(b[t], pls[j]) <= Cs[t]) ? t : (1 << 30);
+        if (m != (1 << 30))
+          sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[t], Cs[t])),
+                         __dmul_rn(pp.lambda2, static_cast<double>(eta[t * 64 + g])));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const double osc = __shfl_xor_sync(0xffffffffu, sc, o);
+          const int om_ = __shfl_xor_sync(0xffffffffu, m, o);
+          if (om_ != (1 << 30) && (m == (1 << 30) || osc < sc || (osc == sc && om_ < m))) {
+            sc = osc;
+            m = om_;
+          }
         }
-        if (best < 0) { waiting[nw++] = j; continue; }
-        xs[best * 64 + j] = 1;
-        eta[best * 64 + g] += 1;
-        b[best] = __dadd_rn(b[best], pls[j]);
+        if (m == (1 << 30)) {
+          if (t == 0) waiting[nw] = j;
+          ++nw;
+        } else if (t == 0) {
+          xs[m * 64 + j] = 1;
+          eta[m * 64 + g] += 1;
+          b[m] = __dadd_rn(b[m], pls[j]);
+        }
+        __syncwarp();
       }
-      for (int w = 0; w < nw; ++w) {
-        const int j = waiting[w];
-        int best = 0;
-        for (int m = 1; m < M; ++m)
-          if (__dsub_rn(Cs[m], b[m]) > __dsub_rn(Cs[best], b[best])) best = m;
-        xs[best * 64 + j] = 1;
-        eta[best * 64 + grp[j]] += 1;
-        b[best] = __dadd_rn(b[best], pls[j]);
-        if (b[best] > Cs[best]) overflow = 1;
+      if (t == 0) {
+        for (int w = 0; w < nw; ++w) {
+          const int j = waiting[w];
+          int best = 0;
+          for (int m2 = 1; m2 < M; ++m2)
+            if (__dsub_rn(Cs[m2], b[m2]) > __dsub_rn(Cs[best], b[best])) best = m2;
+          xs[best * 64 + j] = 1;
+          eta[best * 64 + grp[j]] += 1;
+          b[best] = __dadd_rn(b[best], pls[j]);
+          if (b[best] > Cs[best]) overflow = 1;
+        }
       }
     }
     __syncthreads();
@@ -391,9 +430,14 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
   int rc = logits_gemm_launch(X_cal, static_cast<int>(N), W_r, L * E, d, H, stream);
   if (rc) return rc;
   OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, stream));
-  int64_t cblocks = (N + 7) / 8;
-  if (cblocks > num_sms() * 8) cblocks = num_sms() * 8;
-  counts_kernel<<<dim3(static_cast<unsigned>(cblocks), L), 256, 0, stream>>>(H, N, L, E, k_freq, counts);
+  int64_t cblocks = (N + 255) / 256;
+  const int64_t ccap = (num_sms() * 8 + L - 1) / L;
+  if (cblocks > ccap) cblocks = ccap;
+  const dim3 cgrid(static_cast<unsigned>(cblocks), L);
+  if (E <= 8) counts_kernel<8><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
+  else if (E <= 16) counts_kernel<16><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
+  else if (E <= 32) counts_kernel<32><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
+  else counts_kernel<64><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
   OM_LAUNCHED("counts_kernel");
   gram_kernel<<<dim3(nchunks, L), 256, 0, stream>>>(H, N, L, E, gpart);
   OM_LAUNCHED("gram_kernel");
