@@ -300,12 +300,17 @@ int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq, in
  *   group [L][E] i32 out, n_groups [L] i32 out, theta [L] f32 out,
  *   placement [L][M][E] u8 out, used [M] f64 out,
  *   status [1] i32 out (device): ORDERMOE_OK, or ORDERMOE_ERR_CAPACITY when
- *   sum C < sum p or a waiting-list expert overflowed its server. */
+ *   sum C < sum p or a waiting-list expert overflowed its server.
+ *   workspace: device scratch of ordermoe_place_workspace_bytes(L, E) bytes
+ *   (the per-layer placement orders between the per-layer pass, which runs
+ *   the layers in parallel, and the placement pass, which runs them in order). */
+size_t ordermoe_place_workspace_bytes(int L, int E);
 int ordermoe_place(const float* sim, const int32_t* counts, int L, int E, int M, double theta_min,
                    double theta_max, double theta_single, double alpha_f, double alpha_r,
                    double lambda1, double lambda2, const double* p, const double* C,
                    int32_t* group, int32_t* n_groups, float* theta, uint8_t* placement,
-                   double* used, int32_t* status, ordermoe_stream_t stream);
+                   double* used, int32_t* status, void* workspace, size_t workspace_bytes,
+                   ordermoe_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -43,7 +43,8 @@ _SIGNATURES = {
     "ordermoe_similarity": ([_P, _P, _I, _I, _I, _I64, _I, _P, _P, _P, _SZ, _P], _I),
     "ordermoe_expert_counts": ([_P, _I64, _I, _I, _P, _P], _I),
     "ordermoe_place": ([_P, _P, _I, _I, _I, _D, _D, _D, _D, _D, _D, _D, _P, _P, _P, _P, _P, _P,
-                        _P, _P, _P], _I),
+                        _P, _P, _P, _SZ, _P], _I),
+    "ordermoe_place_workspace_bytes": ([_I, _I], _SZ),
     "ordermoe_expert_gate_up": ([_P, _P, _I, _P, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_expert_down": ([_P, _P, _I, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_layer_scratch_bytes": ([_I, _I, _I, _I, _I], _SZ),
@@ -216,9 +217,18 @@ def ordermoe_expert_counts(logits, N, E, k_freq, counts, stream=None):
            lib().ordermoe_expert_counts(_ptr(logits), N, E, k_freq, _ptr(counts), _stream(stream)))
 
 
+def ordermoe_place_workspace_bytes(L, E):
+    return int(lib().ordermoe_place_workspace_bytes(L, E))
+
+
 def ordermoe_place(sim, counts, L, E, M, theta_min, theta_max, theta_single, alpha_f, alpha_r,
                    lambda1, lambda2, p, C, group, n_groups, theta, placement, used, status,
-                   stream=None):
+                   workspace=None, stream=None):
+    """workspace: device scratch of ordermoe_place_workspace_bytes(L, E) bytes;
+    allocated here with torch when not given."""
+    if workspace is None:
+        workspace = torch.empty(ordermoe_place_workspace_bytes(L, E), dtype=torch.uint8,
+                                device=sim.device)
     _dt(sim, torch.float32, "sim"); _dt(counts, torch.int32, "counts")
     _dt(p, torch.float64, "p"); _dt(C, torch.float64, "C"); _dt(group, torch.int32, "group")
     _dt(n_groups, torch.int32, "n_groups"); _dt(theta, torch.float32, "theta")
@@ -227,7 +237,9 @@ def ordermoe_place(sim, counts, L, E, M, theta_min, theta_max, theta_single, alp
     rc = lib().ordermoe_place(_ptr(sim), _ptr(counts), L, E, M, float(theta_min), float(theta_max),
                               float(theta_single), float(alpha_f), float(alpha_r), float(lambda1),
                               float(lambda2), _ptr(p), _ptr(C), _ptr(group), _ptr(n_groups),
-                              _ptr(theta), _ptr(placement), _ptr(used), _ptr(status), _stream(stream))
+                              _ptr(theta), _ptr(placement), _ptr(used), _ptr(status),
+                              _ptr(workspace), workspace.numel() * workspace.element_size(),
+                              _stream(stream))
     _check("ordermoe_place", rc)
 
 

@@ -15,6 +15,10 @@ int fail(int code, const char* fmt, ...);         // sets the thread-local messa
 int cuda_fail(cudaError_t e, const char* what);   // ORDERMOE_ERR_CUDA with the CUDA message
 uint64_t wait_limit_ns();                          // per-thread limit for bounded waits
 int num_sms();                                     // SM count of the current device
+// 2-D bf16 row-major [rows][cols] tensor map, box of 64 columns x box_rows
+// rows, 128-byte swizzle, zero fill out of bounds.
+int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
+                   uint32_t box_rows);
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 

@@ -642,11 +642,18 @@ EncodeTiledFn encode_fn() {
 
 // 2-D bf16 row-major [rows][cols] map with a 64 x 128 box and 128-byte swizzle.
 int make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols) {
-  EncodeTiledFn enc = encode_fn();
+  return make_tmap_bf16(map, base, rows, cols, 128);
+}
+
+}  // namespace gg
+
+int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols,
+                   uint32_t box_rows) {
+  gg::EncodeTiledFn enc = gg::encode_fn();
   if (!enc) return fail(ORDERMOE_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {BK, 128};
+  cuuint32_t box[2] = {gg::BK, box_rows};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -654,8 +661,6 @@ int make_map(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols) {
   if (r != CUDA_SUCCESS) return fail(ORDERMOE_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
   return ORDERMOE_OK;
 }
-
-}  // namespace gg
 
 static int ffn_attrs() {
   using namespace gg;

@@ -86,214 +86,124 @@ __global__ void build_tables_kernel(const float* __restrict__ sim, const int32_t
 }
 
 // ---------------------------------------------------------------------------
-// Router + top-k + selection. One warp per token.
-//
-// Router: lane l accumulates the fp32 partial dot products of 8-element
-// chunks c = 8 l, 8 l + 256, ...; a butterfly reduction gives every lane all E
-// logits. Top-k and softmax are then computed redundantly by every lane (E
-// is at most 64), so the per-slot selection needs no further communication.
-//
-// Selection, per slot j in rank order (Eqs. 36-44): the candidates are the
-// pairs (m, k') with k' = r (exact) or k' in R_{l,r} (Eq. 7), x_{m,k'} = 1,
-// and for substitutes k' not yet used by the token and Qhat + Q(r,k') <= Qbar
-// (Eq. 40). Lanes take candidates c = lane, lane + 32, ...; the cost of Eq. 38
-// is A[a][s][m] + Cq[r][k'] (one fp32 add), packed with the tie-break fields
-// into a 64-bit key whose warp-wide minimum is the argmin of Eq. 43. Costs
-// are never negative, so the fp32 bit pattern orders them.
-template <int EMAX>
-__global__ void __launch_bounds__(256) route_select_kernel(
-    const uint16_t* __restrict__ X, const uint16_t* __restrict__ Wr,
-    const float* __restrict__ logits_in, int T, int E, int d, int k, int renorm,
-    const uint8_t* __restrict__ tab, const uint8_t* __restrict__ home, uint8_t* __restrict__ loc,
-    float* __restrict__ qhat, float* __restrict__ logits_out, int32_t* __restrict__ topk_idx,
-    float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
-    uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
-    int32_t* __restrict__ counters, int stage_w) {
-  __shared__ uint32_t s_pmask[64];
-  __shared__ unsigned long long s_subst[64];
-  __shared__ uint8_t s_sublist[64 * 64];
-  __shared__ int s_nsub[64];
-  __shared__ int s_kind[4];
-  extern __shared__ __align__(16) float s_dyn[];  // Qtab[E*E], Cq[E*E], then W_r if staged
-  float* s_Q = s_dyn;
-  float* s_Cq = s_dyn + E * E;
-  // W_r staged in shared memory when it fits (stage_w): every token of the
-  // block then reads it at shared-memory latency instead of from L2.
-  uint4* s_W = reinterpret_cast<uint4*>(s_dyn + ((2 * E * E + 3) & ~3));
+// Selection tables staged in shared memory (one copy per CTA).
+struct SelSmem {
+  uint32_t pmask[64];
+  int nsub[64];
+  int kind[4];
+  uint8_t sublist[64 * 64];
+};
 
+// Loads the layer's tables into shared memory (whole block). Returns false
+// if the header does not match E (reported once).
+__device__ bool load_tables(const uint8_t* __restrict__ tab, int E, SelSmem& sm, float* s_Q,
+                            float* s_Cq) {
   const int M = reinterpret_cast<const int32_t*>(tab)[2];
   if (reinterpret_cast<const int32_t*>(tab)[1] != E || M <= 0 || M > 32) {
     if (blockIdx.x == 0 && threadIdx.x == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, -1);
-    return;
+    return false;
   }
-  const float qbar = reinterpret_cast<const float*>(tab)[5];
   const float* gQ = reinterpret_cast<const float*>(tab + kOffQtab);
   const float* gCq = reinterpret_cast<const float*>(tab + off_cq(E));
-  const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
-
   for (int i = threadIdx.x; i < 64; i += blockDim.x) {
-    s_pmask[i] = reinterpret_cast<const uint32_t*>(tab + kOffPmask)[i];
+    sm.pmask[i] = reinterpret_cast<const uint32_t*>(tab + kOffPmask)[i];
     unsigned long long sb = reinterpret_cast<const unsigned long long*>(tab + kOffSubst)[i];
-    s_subst[i] = sb;
     int n = 0;
     while (sb) {
       const int b = __ffsll(static_cast<long long>(sb)) - 1;
-      s_sublist[i * 64 + n++] = static_cast<uint8_t>(b);
+      sm.sublist[i * 64 + n++] = static_cast<uint8_t>(b);
       sb &= sb - 1;
     }
-    s_nsub[i] = n;
+    sm.nsub[i] = n;
   }
   for (int i = threadIdx.x; i < E * E; i += blockDim.x) {
     s_Q[i] = gQ[i];
     s_Cq[i] = gCq[i];
   }
-  if (stage_w && logits_in == nullptr) {
-    const uint4* gw = reinterpret_cast<const uint4*>(Wr);
-    for (int i = threadIdx.x; i < E * (d >> 3); i += blockDim.x) s_W[i] = __ldg(gw + i);
+  if (threadIdx.x < 4) sm.kind[threadIdx.x] = 0;
+  return true;
+}
+
+// One token: softmax over E, top-k, then Alg. 2 (H = 1) per slot in rank
+// order (Eqs. 36-44). The logits are in registers (lg[e], e < E <= EMAX).
+// The argmin of Eq. 43 packs (fp32 cost bits, substitute, away, server,
+// expert) into a 64-bit key and keeps the smallest; costs are never
+// negative, so the bit pattern orders them like the values.
+template <int EMAX>
+__device__ __forceinline__ void select_token(
+    int t, const float (&lg)[EMAX], int E, int k, int renorm, int M, float qbar,
+    const float* __restrict__ gA, const SelSmem& sm, const float* s_Q, const float* s_Cq,
+    const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
+    int32_t* __restrict__ topk_idx, float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
+    uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out, int (&kind_count)[4]) {
+#pragma unroll
+  for (int e = 0; e < EMAX; ++e)
+    if (e < E && isnan(lg[e])) {
+      report(&g_err_route, ORDERMOE_DEV_NAN_LOGIT, t);
+      return;
+    }
+  // top-k by (logit desc, index asc)
+  int idx[ORDERMOE_MAX_TOPK];
+  float lsel[ORDERMOE_MAX_TOPK];
+  unsigned long long used_targets = 0;
+  for (int j = 0; j < k; ++j) {
+    int best = -1;
+    float bv = 0.0f;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E && !((used_targets >> e) & 1ull) && (best < 0 || lg[e] > bv)) {
+        best = e;
+        bv = lg[e];
+      }
+    idx[j] = best;
+    lsel[j] = bv;
+    used_targets |= 1ull << best;
   }
-  if (threadIdx.x < 4) s_kind[threadIdx.x] = 0;
-  __syncthreads();
-
-  const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
-  const int warps_total = gridDim.x * (blockDim.x >> 5);
-  int kind_count[4] = {0, 0, 0, 0};
-
-  for (int t = blockIdx.x * (blockDim.x >> 5) + warp; t < T; t += warps_total) {
-    float lg[EMAX];
-    if (logits_in != nullptr) {
+  // softmax over all E in fp32; gate weights of the k slots
+  const float lmax = lsel[0];
+  float denom = 0.0f;
 #pragma unroll
-      for (int e = 0; e < EMAX; ++e) lg[e] = (e < E) ? logits_in[(size_t)t * E + e] : 0.0f;
-    } else {
-#pragma unroll
-      for (int e = 0; e < EMAX; ++e) lg[e] = 0.0f;
-      const uint4* xr = reinterpret_cast<const uint4*>(X + (size_t)t * d);
-      const int nvec = d >> 3;
-      // X is streamed once from HBM: keep kBatch independent 16-byte loads
-      // per lane in flight before using them; W_r stays in L1.
-      constexpr int kBatch = 4;
-      for (int c0 = lane; c0 < nvec; c0 += 32 * kBatch) {
-        uint4 xv[kBatch];
-#pragma unroll
-        for (int b = 0; b < kBatch; ++b) {
-          const int c = c0 + 32 * b;
-          xv[b] = (c < nvec) ? __ldg(xr + c) : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int b = 0; b < kBatch; ++b) {
-          const int c = c0 + 32 * b;
-          if (c >= nvec) break;
-          const float x0 = bf16_lo(xv[b].x), x1 = bf16_hi(xv[b].x), x2 = bf16_lo(xv[b].y);
-          const float x3 = bf16_hi(xv[b].y), x4 = bf16_lo(xv[b].z), x5 = bf16_hi(xv[b].z);
-          const float x6 = bf16_lo(xv[b].w), x7 = bf16_hi(xv[b].w);
-#pragma unroll
-          for (int e = 0; e < EMAX; ++e) {
-            if (e < E) {
-              const uint4 wv = stage_w ? s_W[e * nvec + c]
-                                       : __ldg(reinterpret_cast<const uint4*>(Wr + (size_t)e * d) + c);
-              float a = lg[e];
-              a = fmaf(x0, bf16_lo(wv.x), a); a = fmaf(x1, bf16_hi(wv.x), a);
-              a = fmaf(x2, bf16_lo(wv.y), a); a = fmaf(x3, bf16_hi(wv.y), a);
-              a = fmaf(x4, bf16_lo(wv.z), a); a = fmaf(x5, bf16_hi(wv.z), a);
-              a = fmaf(x6, bf16_lo(wv.w), a); a = fmaf(x7, bf16_hi(wv.w), a);
-              lg[e] = a;
-            }
-          }
-        }
+  for (int e = 0; e < EMAX; ++e)
+    if (e < E) denom += expf(lg[e] - lmax);
+  float wsel[ORDERMOE_MAX_TOPK];
+  float ssel = 0.0f;
+  for (int j = 0; j < k; ++j) {
+    wsel[j] = expf(lsel[j] - lmax) / denom;
+    ssel += wsel[j];
+  }
+  for (int j = 0; j < k; ++j) {
+    topk_idx[(size_t)t * k + j] = idx[j];
+    topk_w[(size_t)t * k + j] = renorm ? wsel[j] / ssel : wsel[j];
+  }
+  // selection
+  const int a = home[t];
+  const int s = (loc != nullptr) ? loc[t] : a;  // no state given: first layer (Eq. 36)
+  if (a >= M || s >= M) {
+    report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
+    return;
+  }
+  const float* Aas = gA + ((size_t)a * M + s) * M;
+  float q = (qhat != nullptr) ? qhat[t] : 0.0f;
+  unsigned long long taken = used_targets;
+  int first_server = s;
+  for (int j = 0; j < k; ++j) {
+    const int r = idx[j];
+    const int nsub = sm.nsub[r];
+    unsigned long long best = ~0ull;
+    for (int ki = 0; ki <= nsub; ++ki) {
+      const int kk = (ki == 0) ? r : sm.sublist[r * 64 + ki - 1];
+      const bool sub = (ki != 0);
+      float cq = 0.0f;
+      if (sub) {
+        if ((taken >> kk) & 1ull) continue;
+        if (!(__fadd_rn(q, s_Q[r * E + kk]) <= qbar)) continue;  // Eq. 40 budget
+        cq = s_Cq[r * E + kk];
       }
-#pragma unroll
-      for (int e = 0; e < EMAX; ++e) {
-        float v = lg[e];
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-        lg[e] = v;
-      }
-    }
-    // logits out: lane e (and e + 32) writes expert e
-    if (logits_out != nullptr) {
-#pragma unroll
-      for (int e = 0; e < EMAX; ++e)
-        if (e < E && (e & 31) == lane) logits_out[(size_t)t * E + e] = lg[e];
-    }
-    bool bad = false;
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E && isnan(lg[e])) bad = true;
-    if (bad) {
-      if (lane == 0) report(&g_err_route, ORDERMOE_DEV_NAN_LOGIT, t);
-      continue;
-    }
-    // top-k by (logit desc, index asc)
-    int idx[ORDERMOE_MAX_TOPK];
-    unsigned long long used_targets = 0;
-    for (int j = 0; j < k; ++j) {
-      int best = -1;
-      float bv = 0.0f;
-#pragma unroll
-      for (int e = 0; e < EMAX; ++e) {
-        if (e < E && !((used_targets >> e) & 1ull)) {
-          if (best < 0 || lg[e] > bv) { best = e; bv = lg[e]; }
-        }
-      }
-      idx[j] = best;
-      used_targets |= 1ull << best;
-    }
-    // softmax over all E in fp32, gate weights of the k slots
-    float lmax = -INFINITY;
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) lmax = fmaxf(lmax, lg[e]);
-    float denom = 0.0f;
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E) denom += expf(lg[e] - lmax);
-    float wsel[ORDERMOE_MAX_TOPK];
-    float ssel = 0.0f;
-    for (int j = 0; j < k; ++j) {
-      float v = 0.0f;
-#pragma unroll
-      for (int e = 0; e < EMAX; ++e)
-        if (e == idx[j]) v = lg[e];
-      wsel[j] = expf(v - lmax) / denom;
-      ssel += wsel[j];
-    }
-    if (lane == 0) {
-      for (int j = 0; j < k; ++j) {
-        topk_idx[(size_t)t * k + j] = idx[j];
-        topk_w[(size_t)t * k + j] = renorm ? wsel[j] / ssel : wsel[j];
-      }
-    }
-
-    // selection
-    const int a = home[t];
-    const int s = (loc != nullptr) ? loc[t] : a;  // no state given: first layer (Eq. 36)
-    if (a >= M || s >= M) {
-      if (lane == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
-      continue;
-    }
-    const float* Aas = gA + ((size_t)a * M + s) * M;
-    float q = (qhat != nullptr) ? qhat[t] : 0.0f;
-    unsigned long long taken = used_targets;
-    int first_server = s;
-    for (int j = 0; j < k; ++j) {
-      const int r = idx[j];
-      const int nsub = s_nsub[r];
-      const int ncand = (1 + nsub) * M;
-      unsigned long long best = ~0ull;
-      for (int cidx = lane; cidx < ncand; cidx += 32) {
-        const int ki = cidx / M;
-        const int m = cidx - ki * M;
-        const int kk = (ki == 0) ? r : s_sublist[r * 64 + ki - 1];
-        if (!((s_pmask[kk] >> m) & 1u)) continue;
-        const bool sub = (ki != 0);
-        float cost = __ldg(Aas + m);
-        if (sub) {
-          if ((taken >> kk) & 1ull) continue;
-          if (!(__fadd_rn(q, s_Q[r * E + kk]) <= qbar)) continue;
-          cost = __fadd_rn(cost, s_Cq[r * E + kk]);
-        } else {
-          cost = __fadd_rn(cost, 0.0f);
-        }
+      uint32_t pm = sm.pmask[kk];
+      while (pm) {
+        const int m = __ffs(pm) - 1;
+        pm &= pm - 1;
+        const float cost = __fadd_rn(__ldg(Aas + m), cq);
         const unsigned long long key =
             (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
             (static_cast<unsigned long long>(sub ? 1u : 0u) << 31) |
@@ -301,45 +211,244 @@ __global__ void __launch_bounds__(256) route_select_kernel(
             (static_cast<unsigned long long>(m) << 8) | static_cast<unsigned long long>(kk);
         best = key < best ? key : best;
       }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
-        best = other < best ? other : best;
-      }
-      int kstar, mstar, kd;
-      if (best == ~0ull) {
-        if (lane == 0) report(&g_err_route, ORDERMOE_DEV_NO_CANDIDATE, t);
-        kstar = r; mstar = s; kd = 0;
-      } else {
-        kstar = static_cast<int>(best & 0xFFu);
-        mstar = static_cast<int>((best >> 8) & 0xFFu);
-        const int sub = static_cast<int>((best >> 31) & 1u);
-        const int away = static_cast<int>((best >> 30) & 1u);
-        kd = 2 * away + sub;
-        if (sub) {
-          taken |= 1ull << kstar;
-          q = __fadd_rn(q, s_Q[r * E + kstar]);
-        }
-      }
-      if (j == 0) first_server = mstar;
-      if (lane == 0) {
-        chosen_expert[(size_t)t * k + j] = kstar;
-        chosen_server[(size_t)t * k + j] = static_cast<uint8_t>(mstar);
-        kind_out[(size_t)t * k + j] = static_cast<uint8_t>(kd);
-      }
-      kind_count[kd]++;
     }
-    if (lane == 0 && loc != nullptr) {
-      loc[t] = static_cast<uint8_t>(first_server);
-      qhat[t] = q;
+    int kstar, mstar, kd;
+    if (best == ~0ull) {
+      report(&g_err_route, ORDERMOE_DEV_NO_CANDIDATE, t);
+      kstar = r; mstar = s; kd = 0;
+    } else {
+      kstar = static_cast<int>(best & 0xFFu);
+      mstar = static_cast<int>((best >> 8) & 0xFFu);
+      const int sub = static_cast<int>((best >> 31) & 1u);
+      const int away = static_cast<int>((best >> 30) & 1u);
+      kd = 2 * away + sub;
+      if (sub) {
+        taken |= 1ull << kstar;
+        q = __fadd_rn(q, s_Q[r * E + kstar]);
+      }
     }
+    if (j == 0) first_server = mstar;
+    chosen_expert[(size_t)t * k + j] = kstar;
+    chosen_server[(size_t)t * k + j] = static_cast<uint8_t>(mstar);
+    kind_out[(size_t)t * k + j] = static_cast<uint8_t>(kd);
+    kind_count[kd]++;
   }
-  if (counters != nullptr) {
-    if (lane == 0)
-      for (int i = 0; i < 4; ++i)
-        if (kind_count[i]) atomicAdd(&s_kind[i], kind_count[i]);
+  if (loc != nullptr) {
+    loc[t] = static_cast<uint8_t>(first_server);
+    qhat[t] = q;
+  }
+}
+
+__device__ __forceinline__ void flush_kind_counts(SelSmem& sm, const int (&kind_count)[4],
+                                                  int32_t* counters) {
+  if (counters == nullptr) return;
+  for (int i = 0; i < 4; ++i)
+    if (kind_count[i]) atomicAdd(&sm.kind[i], kind_count[i]);
+}
+
+// Selection from given logits: one thread per token.
+template <int EMAX>
+__global__ void __launch_bounds__(128) select_kernel(
+    const float* __restrict__ logits_in, int T, int E, int k, int renorm,
+    const uint8_t* __restrict__ tab, const uint8_t* __restrict__ home, uint8_t* __restrict__ loc,
+    float* __restrict__ qhat, float* __restrict__ logits_out, int32_t* __restrict__ topk_idx,
+    float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
+    uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
+    int32_t* __restrict__ counters) {
+  __shared__ SelSmem sm;
+  extern __shared__ __align__(16) float s_dyn[];
+  float* s_Q = s_dyn;
+  float* s_Cq = s_dyn + E * E;
+  if (!load_tables(tab, E, sm, s_Q, s_Cq)) return;
+  __syncthreads();
+  const int M = reinterpret_cast<const int32_t*>(tab)[2];
+  const float qbar = reinterpret_cast<const float*>(tab)[5];
+  const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
+  int kind_count[4] = {0, 0, 0, 0};
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t < T) {
+    float lg[EMAX];
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e) lg[e] = (e < E) ? logits_in[(size_t)t * E + e] : 0.0f;
+    if (logits_out != nullptr)
+      for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
+    select_token<EMAX>(t, lg, E, k, renorm, M, qbar, gA, sm, s_Q, s_Cq, home, loc, qhat, topk_idx,
+                       topk_w, chosen_expert, chosen_server, kind_out, kind_count);
+  }
+  flush_kind_counts(sm, kind_count, counters);
+  __syncthreads();
+  if (counters != nullptr && threadIdx.x < 4 && sm.kind[threadIdx.x])
+    atomicAdd(&counters[threadIdx.x], sm.kind[threadIdx.x]);
+}
+
+// ---------------------------------------------------------------------------
+// Router on tcgen05 + selection. One CTA per 128 tokens: logits = X W_r^T
+// (M = 128 tokens, N = NE >= E padded to a multiple of 16, K = d) accumulate
+// in TMEM; epilogue thread i of warp w (w = 2..5) owns token 32 (w % 4) + i,
+// reads its NE logits from TMEM lane 32 (w % 4) + i and runs select_token.
+// Warp 0 issues the TMA loads (X: 128 x 64 box; W_r: NE x 64 box, rows >= E
+// zero-filled), warp 1 the MMAs; 4-stage mbarrier ring; bounded waits.
+namespace rt {
+constexpr int BK = 64;
+constexpr int STAGES = 4;
+constexpr int A_BYTES = 128 * BK * 2;
+constexpr int THREADS = 192;
+}  // namespace rt
+
+template <int NE>
+struct RouterSmem {
+  uint64_t full[rt::STAGES];
+  uint64_t empty[rt::STAGES];
+  uint64_t tfull;
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+  int zero;
+};
+
+template <int NE>
+__global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
+    const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapW, int T,
+    int E, int d, int k, int renorm, const uint8_t* __restrict__ tab,
+    const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
+    float* __restrict__ logits_out, int32_t* __restrict__ topk_idx, float* __restrict__ topk_w,
+    int32_t* __restrict__ chosen_expert, uint8_t* __restrict__ chosen_server,
+    uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters, uint64_t limit_ns) {
+  constexpr int B_BYTES = NE * rt::BK * 2;
+  constexpr int STAGE_BYTES = rt::A_BYTES + B_BYTES;
+  constexpr int TMEM_COLS = NE <= 32 ? 32 : NE;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* tiles = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  RouterSmem<NE>& s = *reinterpret_cast<RouterSmem<NE>*>(tiles + rt::STAGES * STAGE_BYTES);
+  float* s_Q = reinterpret_cast<float*>(tiles + rt::STAGES * STAGE_BYTES + 256);
+  float* s_Cq = s_Q + E * E;
+  __shared__ SelSmem sm;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int m0 = blockIdx.x * 128;
+  const int kblocks = d / rt::BK;
+
+  if (tid == 0) {
+    for (int i = 0; i < rt::STAGES; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.empty[i], 1);
+    }
+    mbar_init(&s.tfull, 1);
+    mbar_init(&s.drain, 1);
+    s.abort = 0;
+    s.zero = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&mapX);
+    tma_prefetch_map(&mapW);
+  }
+  if (warp == 1) {
+    tmem_alloc(&s.tmem_base, TMEM_COLS);
+    tmem_relinquish();
+  }
+  const bool tables_ok = load_tables(tab, E, sm, s_Q, s_Cq);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = s.tmem_base;
+  volatile int* abort = &s.abort;
+  uint32_t issued_mask = 0, last_phase_bits = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      for (int kb = 0; kb < kblocks && !*abort; ++kb) {
+        const int stage = kb % rt::STAGES;
+        const uint32_t phase = (kb / rt::STAGES) & 1;
+        if (!mbar_wait(&s.empty[stage], phase ^ 1u, limit_ns, abort)) {
+          if (!*abort) report(&g_err_route, ORDERMOE_DEV_WAIT_TIMEOUT, 21);
+          *abort = 1;
+          break;
+        }
+        uint8_t* sa = tiles + stage * STAGE_BYTES;
+        mbar_arrive_expect_tx(&s.full[stage], STAGE_BYTES);
+        tma_load_2d(sa, &mapX, &s.full[stage], kb * rt::BK, m0);
+        tma_load_2d(sa + rt::A_BYTES, &mapW, &s.full[stage], kb * rt::BK, 0);
+        issued_mask |= 1u << stage;
+        last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      constexpr uint32_t IDESC = idesc_bf16_f32(128, NE);
+      bool ok = true;
+      for (int kb = 0; kb < kblocks && !*abort; ++kb) {
+        const int stage = kb % rt::STAGES;
+        const uint32_t phase = (kb / rt::STAGES) & 1;
+        if (!mbar_wait(&s.full[stage], phase, limit_ns, abort)) {
+          if (!*abort) report(&g_err_route, ORDERMOE_DEV_WAIT_TIMEOUT, 22);
+          *abort = 1;
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a0 = smem_u32(tiles + stage * STAGE_BYTES);
+        const uint32_t b0 = a0 + rt::A_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < rt::BK / 16; ++kk)
+          mma_bf16(tmem_base, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
+                   IDESC, (kb | kk) != 0 ? 1u : 0u);
+        mma_issued = true;
+        mma_commit(&s.empty[stage]);
+      }
+      if (ok && !*abort) mma_commit(&s.tfull);
+    }
+  } else {
+    const int q = warp & 3;
+    const int t = m0 + q * 32 + lane;
+    int kind_count[4] = {0, 0, 0, 0};
+    const bool ok = __all_sync(0xffffffffu, mbar_wait(&s.tfull, 0, limit_ns, abort));
+    if (!ok) {
+      if (lane == 0 && !*abort) report(&g_err_route, ORDERMOE_DEV_WAIT_TIMEOUT, 23);
+      *abort = 1;
+    } else {
+      tc_fence_after();
+      float lg[NE];
+#pragma unroll
+      for (int c = 0; c < NE; c += 32) {
+        uint32_t v[32];
+        tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + c, v);
+        tmem_ld_wait();
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (c + i < NE) lg[c + i] = __uint_as_float(v[i]);
+      }
+      if (t < T && tables_ok) {
+        if (logits_out != nullptr)
+          for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
+        const int M = reinterpret_cast<const int32_t*>(tab)[2];
+        const float qbar = reinterpret_cast<const float*>(tab)[5];
+        const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
+        select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, sm, s_Q, s_Cq, home, loc, qhat,
+                         topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count);
+      }
+      tc_fence_before();
+    }
+    flush_kind_counts(sm, kind_count, counters);
+  }
+
+  __syncthreads();
+  if (s.abort) {
+    volatile int* never = &s.zero;
+    if (warp == 0 && lane == 0)
+      for (int st = 0; st < rt::STAGES; ++st)
+        if ((issued_mask >> st) & 1u) mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, limit_ns, never);
+    if (warp == 1 && lane == 0 && mma_issued) {
+      mma_commit(&s.drain);
+      mbar_wait(&s.drain, 0, limit_ns, never);
+    }
     __syncthreads();
-    if (threadIdx.x < 4 && s_kind[threadIdx.x]) atomicAdd(&counters[threadIdx.x], s_kind[threadIdx.x]);
+  }
+  if (counters != nullptr && tid < 4 && sm.kind[tid]) atomicAdd(&counters[tid], sm.kind[tid]);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -392,42 +501,54 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
     return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: give both loc and qhat, or neither");
   if (logits_in == nullptr) {
     if (!X || !W_r) return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: X/W_r null without logits_in");
-    if (d <= 0 || d % 8 != 0)
-      return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select: d must be a positive multiple of 8");
+    if (d <= 0 || d % 64 != 0)
+      return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select: d must be a positive multiple of 64");
     if (!aligned16(X) || !aligned16(W_r))
       return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: X and W_r must be 16-byte aligned");
   }
-  if (tables_bytes_ < 64) return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: tables too small");
-  if (T == 0) return ORDERMOE_OK;
-  // The table header (E, M) is on the device; E must match. Check the size
-  // against the largest M so that a wrong buffer is caught early.
   if (tables_bytes_ < om::tables_bytes(E, 1))
     return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: tables buffer smaller than E needs");
-  const int threads = 256;
-  const int per_block = threads / 32;
-  int blocks = (T + per_block - 1) / per_block;
-  // Stage W_r in shared memory when it fits in 96 KB; the grid is then a few
-  // persistent blocks per SM so that each block loads it once.
-  const size_t tab_bytes = sizeof(float) * ((2 * E * E + 3) & ~3);
-  const size_t w_bytes = (size_t)E * d * 2;
-  const int stage_w = (logits_in == nullptr && w_bytes <= 96 * 1024) ? 1 : 0;
-  const int cap = num_sms() * (stage_w ? 2 : 8);
-  if (blocks > cap) blocks = cap;
-  const size_t dyn = tab_bytes + (stage_w ? w_bytes : 0);
+  if (T == 0) return ORDERMOE_OK;
   const uint8_t* tb = static_cast<const uint8_t*>(tables);
-#define OM_RS_LAUNCH(EM)                                                                        \
-  do {                                                                                          \
-    cudaFuncSetAttribute(route_select_kernel<EM>, cudaFuncAttributeMaxDynamicSharedMemorySize,  \
-                         (int)dyn);                                                             \
-    route_select_kernel<EM><<<blocks, threads, dyn, stream>>>(                                  \
-        X, W_r, logits_in, T, E, d, k, renorm, tb, home, loc, qhat, logits_out, topk_idx,       \
-        topk_w, chosen_expert, chosen_server, kind, counters, stage_w);                         \
+  const size_t tab_smem = sizeof(float) * 2 * E * E;
+  const int blocks = (T + 127) / 128;
+  if (logits_in != nullptr) {
+#define OM_SEL_LAUNCH(EM)                                                                        \
+  do {                                                                                           \
+    cudaFuncSetAttribute(select_kernel<EM>, cudaFuncAttributeMaxDynamicSharedMemorySize,         \
+                         (int)tab_smem);                                                         \
+    select_kernel<EM><<<blocks, 128, tab_smem, stream>>>(logits_in, T, E, k, renorm, tb, home,   \
+                                                         loc, qhat, logits_out, topk_idx, topk_w, \
+                                                         chosen_expert, chosen_server, kind,      \
+                                                         counters);                               \
   } while (0)
-  if (E <= 8) OM_RS_LAUNCH(8);
-  else if (E <= 16) OM_RS_LAUNCH(16);
-  else if (E <= 32) OM_RS_LAUNCH(32);
-  else OM_RS_LAUNCH(64);
-#undef OM_RS_LAUNCH
-  OM_LAUNCHED("route_select_kernel");
+    if (E <= 8) OM_SEL_LAUNCH(8);
+    else if (E <= 16) OM_SEL_LAUNCH(16);
+    else if (E <= 32) OM_SEL_LAUNCH(32);
+    else OM_SEL_LAUNCH(64);
+#undef OM_SEL_LAUNCH
+    OM_LAUNCHED("select_kernel");
+    return ORDERMOE_OK;
+  }
+  CUtensorMap mX, mW;
+  int rc;
+  const int NE = E <= 16 ? 16 : (E <= 32 ? 32 : 64);
+  if ((rc = make_tmap_bf16(&mX, X, T, d, 128))) return rc;
+  if ((rc = make_tmap_bf16(&mW, W_r, E, d, NE))) return rc;
+  const uint64_t lim = wait_limit_ns();
+#define OM_RT_LAUNCH(N)                                                                          \
+  do {                                                                                           \
+    const size_t dyn = 1024 + rt::STAGES * (rt::A_BYTES + (N) * rt::BK * 2) + 256 + tab_smem;    \
+    cudaFuncSetAttribute(router_select_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,   \
+                         (int)dyn);                                                              \
+    router_select_kernel<N><<<blocks, rt::THREADS, dyn, stream>>>(                               \
+        mX, mW, T, E, d, k, renorm, tb, home, loc, qhat, logits_out, topk_idx, topk_w,           \
+        chosen_expert, chosen_server, kind, counters, lim);                                      \
+  } while (0)
+  if (NE == 16) OM_RT_LAUNCH(16);
+  else if (NE == 32) OM_RT_LAUNCH(32);
+  else OM_RT_LAUNCH(64);
+#undef OM_RT_LAUNCH
+  OM_LAUNCHED("router_select_kernel");
   return ORDERMOE_OK;
 }

@@ -215,25 +215,127 @@ struct PlaceParams {
   double alpha_f, alpha_r, lambda1, lambda2;
 };
 
-__global__ void __launch_bounds__(64) place_kernel(
-    const float* __restrict__ sim, const int32_t* __restrict__ counts, int L, int E, int M,
-    PlaceParams pp, const double* __restrict__ p, const double* __restrict__ C,
-    int32_t* __restrict__ group, int32_t* __restrict__ n_groups, float* __restrict__ theta_out,
-    uint8_t* __restrict__ placement, double* __restrict__ used, int32_t* __restrict__ status) {
-  __shared__ double b[32];
-  __shared__ double Cs[32];
+// Per-layer part of the plan, one block per layer (the layers are
+// independent here): theta_l (Eq. 6), greedy cover (Eqs. 24-26), importance
+// (Eqs. 27-28) and the placement order (p desc, I desc, index asc).
+__global__ void __launch_bounds__(64) group_kernel(
+    const float* __restrict__ sim, const int32_t* __restrict__ counts, int L, int E,
+    PlaceParams pp, const double* __restrict__ p, int32_t* __restrict__ group,
+    int32_t* __restrict__ n_groups, float* __restrict__ theta_out, int32_t* __restrict__ porder) {
   __shared__ double imp[64];
   __shared__ double pls[64];
   __shared__ int order[64];
   __shared__ int dom[64];
   __shared__ int grp[64];
   __shared__ int cnt[64];
-  __shared__ int waiting[64];
-  __shared__ uint8_t xs[32 * 64];   // placement of the current layer, [m][e]
-  __shared__ int eta[32 * 64];      // experts of group g already on server m, [m][g]
-  __shared__ float S[64 * 64];      // Sim of the current layer
-  __shared__ int overflow;
+  __shared__ float S[64 * 64];
   const int t = threadIdx.x;
+  const int l = blockIdx.x;
+  for (int i = t; i < E * E; i += blockDim.x) S[i] = sim[(size_t)l * E * E + i];
+  if (t < E) {
+    cnt[t] = counts[(size_t)l * E + t];
+    pls[t] = p[(size_t)l * E + t];
+  }
+  __syncthreads();
+  // Eq. 6 (layers numbered from 1)
+  float theta;
+  if (L <= 1) {
+    theta = __double2float_rn(pp.theta_single);
+  } else {
+    const double frac = __ddiv_rn(static_cast<double>(L - (l + 1)), static_cast<double>(L - 1));
+    theta = __double2float_rn(
+        __dadd_rn(pp.theta_min, __dmul_rn(__dsub_rn(pp.theta_max, pp.theta_min), frac)));
+  }
+  // visiting order: count desc, index asc
+  if (t < E) {
+    int r = 0;
+    for (int e = 0; e < E; ++e)
+      if (cnt[e] > cnt[t] || (cnt[e] == cnt[t] && e < t)) ++r;
+    order[r] = t;
+  }
+  __syncthreads();
+  // Eqs. 24-26 in the visiting order; warp 0 scans the existing dominants in
+  // parallel (lane g takes dominants g and g + 32; ties to the earlier one).
+  if (t < 32) {
+    int k = 0;
+    for (int pos = 0; pos < E; ++pos) {
+      const int j = order[pos];
+      float bs = -INFINITY;
+      int bg = 1 << 30;
+      for (int g = t; g < k; g += 32) {
+        const float sv = S[j * E + dom[g]];
+        if (bg == (1 << 30) || sv > bs) { bg = g; bs = sv; }
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+        const int og = __shfl_xor_sync(0xffffffffu, bg, o);
+        if (og != (1 << 30) && (bg == (1 << 30) || os > bs || (os == bs && og < bg))) {
+          bs = os;
+          bg = og;
+        }
+      }
+      if (bg == (1 << 30) || bs < theta) {
+        if (t == 0) { dom[k] = j; grp[j] = k; }
+        ++k;
+      } else if (t == 0) {
+        grp[j] = bg;
+      }
+      __syncwarp();
+    }
+    if (t == 0) {
+      n_groups[l] = k;
+      theta_out[l] = theta;
+    }
+  }
+  __syncthreads();
+  // Eqs. 27-28
+  double total = 0.0;
+  for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cnt[e]));
+  if (t < E) {
+    group[(size_t)l * E + t] = grp[t];
+    double sum = 0.0;
+    int size = 0;
+    for (int k2 = 0; k2 < E; ++k2)
+      if (grp[k2] == grp[t]) { sum = __dadd_rn(sum, static_cast<double>(S[t * E + k2])); ++size; }
+    const double rho = __ddiv_rn(sum, static_cast<double>(size));
+    const double f = total > 0.0 ? __ddiv_rn(static_cast<double>(cnt[t]), total) : 0.0;
+    imp[t] = __dadd_rn(__dmul_rn(pp.alpha_f, f), __dmul_rn(pp.alpha_r, rho));
+  }
+  __syncthreads();
+  // placement order: p desc, I desc, index asc
+  if (t < E) {
+    int r = 0;
+    for (int e = 0; e < E; ++e) {
+      bool before;
+      if (pls[e] != pls[t]) before = pls[e] > pls[t];
+      else if (imp[e] != imp[t]) before = imp[e] > imp[t];
+      else before = e < t;
+      if (before) ++r;
+    }
+    porder[(size_t)l * E + r] = t;
+  }
+}
+
+// Mandatory placement, Eqs. 29-31 (Alg. 1 lines 14-24): one warp, layers and
+// experts in order, b_m carried over the layers. Lane m scores server m
+// (lowest score wins, ties to the lower server); eta comes from the
+// per-(server, group) counts of the layer; a waiting-list expert goes to the
+// server with the most room after its layer.
+__global__ void __launch_bounds__(32) place_kernel(
+    const int32_t* __restrict__ group, const int32_t* __restrict__ porder, int L, int E, int M,
+    PlaceParams pp, const double* __restrict__ p, const double* __restrict__ C,
+    uint8_t* __restrict__ placement, double* __restrict__ used, int32_t* __restrict__ status) {
+  __shared__ double b[32];
+  __shared__ double Cs[32];
+  __shared__ int grp[64];
+  __shared__ int ord[64];
+  __shared__ double pls[64];
+  __shared__ int waiting[64];
+  __shared__ uint8_t xs[32 * 64];
+  __shared__ int eta[32 * 64];
+  const int t = threadIdx.x;
+  int overflow = 0;
   if (t < M) {
     b[t] = 0.0;
     Cs[t] = C[t];
@@ -244,147 +346,61 @@ __global__ void __launch_bounds__(64) place_kernel(
     for (int m = 0; m < M; ++m) have = __dadd_rn(have, C[m]);
     overflow = need > have ? 1 : 0;
   }
-  __syncthreads();
+  __syncwarp();
   for (int l = 0; l < L; ++l) {
-    for (int i = t; i < E * E; i += blockDim.x) S[i] = sim[(size_t)l * E * E + i];
-    for (int i = t; i < M * 64; i += blockDim.x) {
+    for (int i = t; i < M * 64; i += 32) {
       xs[i] = 0;
       eta[i] = 0;
     }
-    if (t < E) {
-      cnt[t] = counts[(size_t)l * E + t];
-      pls[t] = p[(size_t)l * E + t];
+    for (int e = t; e < E; e += 32) {
+      grp[e] = group[(size_t)l * E + e];
+      ord[e] = porder[(size_t)l * E + e];
+      pls[e] = p[(size_t)l * E + e];
     }
-    __syncthreads();
-    // Eq. 6 (layers numbered from 1)
-    float theta;
-    if (L <= 1) {
-      theta = __double2float_rn(pp.theta_single);
-    } else {
-      const double frac = __ddiv_rn(static_cast<double>(L - (l + 1)), static_cast<double>(L - 1));
-      theta = __double2float_rn(
-          __dadd_rn(pp.theta_min, __dmul_rn(__dsub_rn(pp.theta_max, pp.theta_min), frac)));
-    }
-    // visiting order: count desc, index asc
-    if (t < E) {
-      int r = 0;
-      for (int e = 0; e < E; ++e)
-        if (cnt[e] > cnt[t] || (cnt[e] == cnt[t] && e < t)) ++r;
-      order[r] = t;
-    }
-    __syncthreads();
-    // Eqs. 24-26 in the visiting order; warp 0 scans the existing dominants
-    // in parallel (lane g takes dominants g and g + 32; argmax ties to the
-    // earlier dominant).
-    if (t < 32) {
-      int k = 0;
-      for (int pos = 0; pos < E; ++pos) {
-        const int j = order[pos];
-        float bs = -INFINITY;
-        int bg = 1 << 30;
-        for (int g = t; g < k; g += 32) {
-          const float sv = S[j * E + dom[g]];
-          if (bg == (1 << 30) || sv > bs) { bg = g; bs = sv; }
-        }
+    __syncwarp();
+    int nw = 0;
+    for (int pos = 0; pos < E; ++pos) {
+      const int j = ord[pos];
+      const int g = grp[j];
+      double sc = 0.0;
+      int m = (t < M && __dadd_rn(b[t], pls[j]) <= Cs[t]) ? t : (1 << 30);
+      if (m != (1 << 30))
+        sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[t], Cs[t])),
+                       __dmul_rn(pp.lambda2, static_cast<double>(eta[t * 64 + g])));
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          const float os = __shfl_xor_sync(0xffffffffu, bs, o);
-          const int og = __shfl_xor_sync(0xffffffffu, bg, o);
-          if (og != (1 << 30) && (bg == (1 << 30) || os > bs || (os == bs && og < bg))) {
-            bs = os;
-            bg = og;
-          }
+      for (int o = 16; o > 0; o >>= 1) {
+        const double osc = __shfl_xor_sync(0xffffffffu, sc, o);
+        const int om_ = __shfl_xor_sync(0xffffffffu, m, o);
+        if (om_ != (1 << 30) && (m == (1 << 30) || osc < sc || (osc == sc && om_ < m))) {
+          sc = osc;
+          m = om_;
         }
-        if (bg == (1 << 30) || bs < theta) {
-          if (t == 0) { dom[k] = j; grp[j] = k; }
-          ++k;
-        } else if (t == 0) {
-          grp[j] = bg;
-        }
-        __syncwarp();
       }
-      if (t == 0) {
-        n_groups[l] = k;
-        theta_out[l] = theta;
+      if (m == (1 << 30)) {
+        if (t == 0) waiting[nw] = j;
+        ++nw;
+      } else if (t == 0) {
+        xs[m * 64 + j] = 1;
+        eta[m * 64 + g] += 1;
+        b[m] = __dadd_rn(b[m], pls[j]);
+      }
+      __syncwarp();
+    }
+    if (t == 0) {
+      for (int w = 0; w < nw; ++w) {
+        const int j = waiting[w];
+        int best = 0;
+        for (int m2 = 1; m2 < M; ++m2)
+          if (__dsub_rn(Cs[m2], b[m2]) > __dsub_rn(Cs[best], b[best])) best = m2;
+        xs[best * 64 + j] = 1;
+        b[best] = __dadd_rn(b[best], pls[j]);
+        if (b[best] > Cs[best]) overflow = 1;
       }
     }
-    __syncthreads();
-    // Eqs. 27-28
-    double total = 0.0;
-    for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cnt[e]));
-    if (t < E) {
-      group[(size_t)l * E + t] = grp[t];
-      double sum = 0.0;
-      int size = 0;
-      for (int k2 = 0; k2 < E; ++k2)
-        if (grp[k2] == grp[t]) { sum = __dadd_rn(sum, static_cast<double>(S[t * E + k2])); ++size; }
-      const double rho = __ddiv_rn(sum, static_cast<double>(size));
-      const double f = total > 0.0 ? __ddiv_rn(static_cast<double>(cnt[t]), total) : 0.0;
-      imp[t] = __dadd_rn(__dmul_rn(pp.alpha_f, f), __dmul_rn(pp.alpha_r, rho));
-    }
-    __syncthreads();
-    // placement order: p desc, I desc, index asc
-    if (t < E) {
-      int r = 0;
-      for (int e = 0; e < E; ++e) {
-        bool before;
-        if (pls[e] != pls[t]) before = pls[e] > pls[t];
-        else if (imp[e] != imp[t]) before = imp[e] > imp[t];
-        else before = e < t;
-        if (before) ++r;
-      }
-      order[r] = t;
-    }
-    __syncthreads();
-    // Eqs. 29-31 in the placement order; warp 0 scores the servers in
-    // parallel (lane m = server m) and takes the lowest score, ties to the
-    // lower server; eta comes from the per-(server, group) counts.
-    if (t < 32) {
-      int nw = 0;
-      for (int pos = 0; pos < E; ++pos) {
-        const int j = order[pos];
-        const int g = grp[j];
-        double sc = 0.0;
-        int m = (t < M && __dadd_rn(b[t], pls[j]) <= Cs[t]) ? t : (1 << 30);
-        if (m != (1 << 30))
-          sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[t], Cs[t])),
-                         __dmul_rn(pp.lambda2, static_cast<double>(eta[t * 64 + g])));
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-          const double osc = __shfl_xor_sync(0xffffffffu, sc, o);
-          const int om_ = __shfl_xor_sync(0xffffffffu, m, o);
-          if (om_ != (1 << 30) && (m == (1 << 30) || osc < sc || (osc == sc && om_ < m))) {
-            sc = osc;
-            m = om_;
-          }
-        }
-        if (m == (1 << 30)) {
-          if (t == 0) waiting[nw] = j;
-          ++nw;
-        } else if (t == 0) {
-          xs[m * 64 + j] = 1;
-          eta[m * 64 + g] += 1;
-          b[m] = __dadd_rn(b[m], pls[j]);
-        }
-        __syncwarp();
-      }
-      if (t == 0) {
-        for (int w = 0; w < nw; ++w) {
-          const int j = waiting[w];
-          int best = 0;
-          for (int m2 = 1; m2 < M; ++m2)
-            if (__dsub_rn(Cs[m2], b[m2]) > __dsub_rn(Cs[best], b[best])) best = m2;
-          xs[best * 64 + j] = 1;
-          eta[best * 64 + grp[j]] += 1;
-          b[best] = __dadd_rn(b[best], pls[j]);
-          if (b[best] > Cs[best]) overflow = 1;
-        }
-      }
-    }
-    __syncthreads();
+    __syncwarp();
     uint8_t* x = placement + (size_t)l * M * E;
-    for (int i = t; i < M * E; i += blockDim.x) x[i] = xs[(i / E) * 64 + (i % E)];
-    __syncthreads();
+    for (int i = t; i < M * E; i += 32) x[i] = xs[(i / E) * 64 + (i % E)];
+    __syncwarp();
   }
   if (t < M) used[t] = b[t];
   if (t == 0) *status = overflow ? ORDERMOE_ERR_CAPACITY : ORDERMOE_OK;
@@ -462,19 +478,28 @@ extern "C" int ordermoe_expert_counts(const float* logits, int64_t N, int E, int
   return ORDERMOE_OK;
 }
 
+extern "C" size_t ordermoe_place_workspace_bytes(int L, int E) {
+  if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS) return 0;
+  return ((size_t)L * E * sizeof(int32_t) + 255) & ~size_t(255);
+}
+
 extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, int E, int M,
                               double theta_min, double theta_max, double theta_single,
                               double alpha_f, double alpha_r, double lambda1, double lambda2,
                               const double* p, const double* C, int32_t* group, int32_t* n_groups,
                               float* theta, uint8_t* placement, double* used, int32_t* status,
-                              ordermoe_stream_t stream) {
+                              void* workspace, size_t workspace_bytes, ordermoe_stream_t stream) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 || M > ORDERMOE_MAX_SERVERS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "place: need L >= 1, 1 <= E <= 64, 1 <= M <= 32");
   if (!sim || !counts || !p || !C || !group || !n_groups || !theta || !placement || !used || !status)
     return fail(ORDERMOE_ERR_INVALID_ARG, "place: null pointer");
+  if (!workspace || workspace_bytes < ordermoe_place_workspace_bytes(L, E))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "place: workspace missing or too small");
+  int32_t* porder_scratch = static_cast<int32_t*>(workspace);
   PlaceParams pp{theta_min, theta_max, theta_single, alpha_f, alpha_r, lambda1, lambda2};
-  place_kernel<<<1, 64, 0, stream>>>(sim, counts, L, E, M, pp, p, C, group, n_groups, theta,
-                                     placement, used, status);
+  group_kernel<<<L, 64, 0, stream>>>(sim, counts, L, E, pp, p, group, n_groups, theta, porder_scratch);
+  OM_LAUNCHED("group_kernel");
+  place_kernel<<<1, 32, 0, stream>>>(group, porder_scratch, L, E, M, pp, p, C, placement, used, status);
   OM_LAUNCHED("place_kernel");
   return ORDERMOE_OK;
 }
