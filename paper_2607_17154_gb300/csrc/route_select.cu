@@ -144,7 +144,6 @@ __device__ __forceinline__ void select_token(
     }
   // top-k by (logit desc, index asc)
   int idx[ORDERMOE_MAX_TOPK];
-  float lsel[ORDERMOE_MAX_TOPK];
   unsigned long long used_targets = 0;
   for (int j = 0; j < k; ++j) {
     int best = -1;
@@ -156,11 +155,13 @@ __device__ __forceinline__ void select_token(
         bv = lg[e];
       }
     idx[j] = best;
-    lsel[j] = bv;
     used_targets |= 1ull << best;
   }
   // softmax over all E in fp32; gate weights of the k slots
-  const float lmax = lsel[0];
+  float lmax = -INFINITY;
+#pragma unroll
+  for (int e = 0; e < EMAX; ++e)
+    if (e < E) lmax = fmaxf(lmax, lg[e]);
   float denom = 0.0f;
 #pragma unroll
   for (int e = 0; e < EMAX; ++e)
@@ -168,7 +169,11 @@ __device__ __forceinline__ void select_token(
   float wsel[ORDERMOE_MAX_TOPK];
   float ssel = 0.0f;
   for (int j = 0; j < k; ++j) {
-    wsel[j] = expf(lsel[j] - lmax) / denom;
+    float v = 0.0f;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e == idx[j]) v = lg[e];
+    wsel[j] = expf(v - lmax) / denom;
     ssel += wsel[j];
   }
   for (int j = 0; j < k; ++j) {
