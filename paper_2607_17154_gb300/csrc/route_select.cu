@@ -292,10 +292,10 @@ __global__ void __launch_bounds__(128) select_kernel(
 // in TMEM; epilogue thread i of warp w (w = 2..5) owns token 32 (w % 4) + i,
 // reads its NE logits from TMEM lane 32 (w % 4) + i and runs select_token.
 // Warp 0 issues the TMA loads (X: 128 x 64 box; W_r: NE x 64 box, rows >= E
-// zero-filled), warp 1 the MMAs; 4-stage mbarrier ring; bounded waits.
+// zero-filled), warp 1 the MMAs; 8-stage mbarrier ring; bounded waits.
 namespace rt {
 constexpr int BK = 64;
-constexpr int STAGES = 4;
+constexpr int STAGES = 8;  // 8 x (16 KB + NE x 128 B) in flight per CTA: X streams at HBM rate
 constexpr int A_BYTES = 128 * BK * 2;
 constexpr int THREADS = 192;
 }  // namespace rt
