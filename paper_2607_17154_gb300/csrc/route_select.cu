@@ -287,23 +287,37 @@ __global__ void __launch_bounds__(128) select_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// Router on tcgen05 + selection. One CTA per 128 tokens: logits = X W_r^T
-// (M = 128 tokens, N = NE >= E padded to a multiple of 16, K = d) accumulate
-// in TMEM; epilogue thread i of warp w (w = 2..5) owns token 32 (w % 4) + i,
-// reads its NE logits from TMEM lane 32 (w % 4) + i and runs select_token.
+// Router on tcgen05 + selection. A cluster of S CTAs (S = 1..8) handles 128
+// tokens: CTA r of the cluster accumulates logits = X W_r^T over its share of
+// the K blocks (M = 128 tokens, N = NE >= E padded to 16/32/64) in TMEM. Its
+// epilogue thread i of warp w (w = 2..5) reads TMEM lane 32 (w % 4) + i (token
+// 32 (w % 4) + i); ranks > 0 store their partial logits into rank 0's shared
+// memory (distributed shared memory), and after a cluster barrier rank 0 adds
+// the partials in rank order (deterministic) and runs select_token. Splitting
+// K lets a few hundred tokens (decode) still stream X over many SMs.
 // Warp 0 issues the TMA loads (X: 128 x 64 box; W_r: NE x 64 box, rows >= E
-// zero-filled), warp 1 the MMAs; 8-stage mbarrier ring; bounded waits.
+// zero-filled), warp 1 the MMAs; mbarrier ring; bounded waits.
 namespace rt {
 constexpr int BK = 64;
-constexpr int STAGES = 8;  // 8 x (16 KB + NE x 128 B) in flight per CTA: X streams at HBM rate
 constexpr int A_BYTES = 128 * BK * 2;
 constexpr int THREADS = 192;
+// stages of (16 KB + NE x 128 B) in flight per CTA, and the largest cluster,
+// sized so the ring, the partial-logit buffer and the tables fit in 227 KB
+template <int NE>
+constexpr int stages() { return NE <= 16 ? 8 : (NE <= 32 ? 6 : 4); }
+template <int NE>
+constexpr int max_split() { return NE <= 16 ? 8 : (NE <= 32 ? 4 : 2); }
+template <int NE>
+constexpr int smem_bytes(int E) {
+  return 1024 + stages<NE>() * (A_BYTES + NE * BK * 2) + 256 + max_split<NE>() * 128 * NE * 4 +
+         8 * E * E;
+}
 }  // namespace rt
 
 template <int NE>
 struct RouterSmem {
-  uint64_t full[rt::STAGES];
-  uint64_t empty[rt::STAGES];
+  uint64_t full[rt::stages<NE>()];
+  uint64_t empty[rt::stages<NE>()];
   uint64_t tfull;
   uint64_t drain;
   uint32_t tmem_base;
@@ -318,23 +332,31 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
     float* __restrict__ logits_out, int32_t* __restrict__ topk_idx, float* __restrict__ topk_w,
     int32_t* __restrict__ chosen_expert, uint8_t* __restrict__ chosen_server,
-    uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters, uint64_t limit_ns) {
+    uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters, uint64_t limit_ns, int split) {
   constexpr int B_BYTES = NE * rt::BK * 2;
   constexpr int STAGE_BYTES = rt::A_BYTES + B_BYTES;
+  constexpr int STAGES = rt::stages<NE>();
   constexpr int TMEM_COLS = NE <= 32 ? 32 : NE;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* tiles = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  RouterSmem<NE>& s = *reinterpret_cast<RouterSmem<NE>*>(tiles + rt::STAGES * STAGE_BYTES);
-  float* s_Q = reinterpret_cast<float*>(tiles + rt::STAGES * STAGE_BYTES + 256);
+  RouterSmem<NE>& s = *reinterpret_cast<RouterSmem<NE>*>(tiles + STAGES * STAGE_BYTES);
+  float* red = reinterpret_cast<float*>(tiles + STAGES * STAGE_BYTES + 256);  // [split][128][NE]
+  float* s_Q = red + rt::max_split<NE>() * 128 * NE;
   float* s_Cq = s_Q + E * E;
   __shared__ SelSmem sm;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * 128;
-  const int kblocks = d / rt::BK;
+  const uint32_t rank = split > 1 ? cluster_ctarank() : 0;
+  const int tile = blockIdx.x / split;
+  const int m0 = tile * 128;
+  const int kblocks_all = d / rt::BK;
+  const int per = (kblocks_all + split - 1) / split;
+  const int kb_begin = static_cast<int>(rank) * per;
+  const int kb_end = min(kblocks_all, kb_begin + per);
+  const int kblocks = kb_end > kb_begin ? kb_end - kb_begin : 0;
 
   if (tid == 0) {
-    for (int i = 0; i < rt::STAGES; ++i) {
+    for (int i = 0; i < STAGES; ++i) {
       mbar_init(&s.full[i], 1);
       mbar_init(&s.empty[i], 1);
     }
@@ -352,7 +374,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     tmem_alloc(&s.tmem_base, TMEM_COLS);
     tmem_relinquish();
   }
-  const bool tables_ok = load_tables(tab, E, sm, s_Q, s_Cq);
+  const bool tables_ok = (rank == 0) ? load_tables(tab, E, sm, s_Q, s_Cq) : true;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -360,18 +382,21 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
   volatile int* abort = &s.abort;
   uint32_t issued_mask = 0, last_phase_bits = 0;
   bool mma_issued = false;
+  float lg[NE];
+  int kind_count[4] = {0, 0, 0, 0};
 
   if (warp == 0) {
     if (lane == 0) {
-      for (int kb = 0; kb < kblocks && !*abort; ++kb) {
-        const int stage = kb % rt::STAGES;
-        const uint32_t phase = (kb / rt::STAGES) & 1;
+      for (int i = 0; i < kblocks && !*abort; ++i) {
+        const int stage = i % STAGES;
+        const uint32_t phase = (i / STAGES) & 1;
         if (!mbar_wait(&s.empty[stage], phase ^ 1u, limit_ns, abort)) {
           if (!*abort) report(&g_err_route, ORDERMOE_DEV_WAIT_TIMEOUT, 21);
           *abort = 1;
           break;
         }
         uint8_t* sa = tiles + stage * STAGE_BYTES;
+        const int kb = kb_begin + i;
         mbar_arrive_expect_tx(&s.full[stage], STAGE_BYTES);
         tma_load_2d(sa, &mapX, &s.full[stage], kb * rt::BK, m0);
         tma_load_2d(sa + rt::A_BYTES, &mapW, &s.full[stage], kb * rt::BK, 0);
@@ -383,9 +408,9 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     if (lane == 0) {
       constexpr uint32_t IDESC = idesc_bf16_f32(128, NE);
       bool ok = true;
-      for (int kb = 0; kb < kblocks && !*abort; ++kb) {
-        const int stage = kb % rt::STAGES;
-        const uint32_t phase = (kb / rt::STAGES) & 1;
+      for (int i = 0; i < kblocks && !*abort; ++i) {
+        const int stage = i % STAGES;
+        const uint32_t phase = (i / STAGES) & 1;
         if (!mbar_wait(&s.full[stage], phase, limit_ns, abort)) {
           if (!*abort) report(&g_err_route, ORDERMOE_DEV_WAIT_TIMEOUT, 22);
           *abort = 1;
@@ -398,23 +423,25 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
 #pragma unroll
         for (int kk = 0; kk < rt::BK / 16; ++kk)
           mma_bf16(tmem_base, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
-                   IDESC, (kb | kk) != 0 ? 1u : 0u);
+                   IDESC, (i | kk) != 0 ? 1u : 0u);
         mma_issued = true;
         mma_commit(&s.empty[stage]);
       }
-      if (ok && !*abort) mma_commit(&s.tfull);
+      if (ok && !*abort) {
+        if (mma_issued) mma_commit(&s.tfull);
+        else mbar_arrive(&s.tfull);  // empty K share: nothing to wait for
+      }
     }
   } else {
+    // epilogue part 1: this CTA's partial logits
     const int q = warp & 3;
-    const int t = m0 + q * 32 + lane;
-    int kind_count[4] = {0, 0, 0, 0};
+    const int row = q * 32 + lane;
     const bool ok = __all_sync(0xffffffffu, mbar_wait(&s.tfull, 0, limit_ns, abort));
     if (!ok) {
       if (lane == 0 && !*abort) report(&g_err_route, ORDERMOE_DEV_WAIT_TIMEOUT, 23);
       *abort = 1;
     } else {
       tc_fence_after();
-      float lg[NE];
 #pragma unroll
       for (int c = 0; c < NE; c += 32) {
         uint32_t v[32];
@@ -422,18 +449,39 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
         tmem_ld_wait();
 #pragma unroll
         for (int i = 0; i < 32; ++i)
-          if (c + i < NE) lg[c + i] = __uint_as_float(v[i]);
-      }
-      if (t < T && tables_ok) {
-        if (logits_out != nullptr)
-          for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
-        const int M = reinterpret_cast<const int32_t*>(tab)[2];
-        const float qbar = reinterpret_cast<const float*>(tab)[5];
-        const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
-        select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, sm, s_Q, s_Cq, home, loc, qhat,
-                         topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count);
+          if (c + i < NE) lg[c + i] = kblocks > 0 ? __uint_as_float(v[i]) : 0.0f;
       }
       tc_fence_before();
+      if (rank > 0) {
+        // partial logits of this rank -> red[rank][row][:] in rank 0's shared memory
+        const uint32_t dst = mapa_shared(smem_u32(red + ((size_t)rank * 128 + row) * NE), 0);
+#pragma unroll
+        for (int c = 0; c < NE; c += 4)
+          asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(dst + c * 4),
+                       "f"(lg[c]), "f"(lg[c + 1]), "f"(lg[c + 2]), "f"(lg[c + 3])
+                       : "memory");
+      }
+    }
+  }
+  if (split > 1) cluster_sync();  // partials visible in rank 0
+  if (warp >= 2 && rank == 0 && !*abort) {
+    // epilogue part 2: full logits (partials in rank order) and the selection
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const int t = m0 + row;
+    for (int r = 1; r < split; ++r) {
+      const float* src = red + ((size_t)r * 128 + row) * NE;
+#pragma unroll
+      for (int c = 0; c < NE; ++c) lg[c] += src[c];
+    }
+    if (t < T && tables_ok) {
+      if (logits_out != nullptr)
+        for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
+      const int M = reinterpret_cast<const int32_t*>(tab)[2];
+      const float qbar = reinterpret_cast<const float*>(tab)[5];
+      const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
+      select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, sm, s_Q, s_Cq, home, loc, qhat, topk_idx,
+                       topk_w, chosen_expert, chosen_server, kind_out, kind_count);
     }
     flush_kind_counts(sm, kind_count, counters);
   }
@@ -442,7 +490,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
   if (s.abort) {
     volatile int* never = &s.zero;
     if (warp == 0 && lane == 0)
-      for (int st = 0; st < rt::STAGES; ++st)
+      for (int st = 0; st < STAGES; ++st)
         if ((issued_mask >> st) & 1u) mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, limit_ns, never);
     if (warp == 1 && lane == 0 && mma_issued) {
       mma_commit(&s.drain);
@@ -450,7 +498,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     }
     __syncthreads();
   }
-  if (counters != nullptr && tid < 4 && sm.kind[tid]) atomicAdd(&counters[tid], sm.kind[tid]);
+  if (rank == 0 && counters != nullptr && tid < 4 && sm.kind[tid]) atomicAdd(&counters[tid], sm.kind[tid]);
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, TMEM_COLS);
@@ -541,19 +589,38 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
   if ((rc = make_tmap_bf16(&mX, X, T, d, 128))) return rc;
   if ((rc = make_tmap_bf16(&mW, W_r, E, d, NE))) return rc;
   const uint64_t lim = wait_limit_ns();
+  // split K over a cluster so that about one CTA per SM streams X
+  const int kblocks = d / rt::BK;
+  const int smax = NE == 16 ? rt::max_split<16>() : (NE == 32 ? rt::max_split<32>() : rt::max_split<64>());
+  int split = 1;
+  while (split * 2 <= smax && (long long)blocks * split * 2 <= num_sms() && split * 2 <= kblocks)
+    split *= 2;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(blocks * split, 1, 1);
+  cfg.blockDim = dim3(rt::THREADS, 1, 1);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = split;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  cudaError_t le;
 #define OM_RT_LAUNCH(N)                                                                          \
   do {                                                                                           \
-    const size_t dyn = 1024 + rt::STAGES * (rt::A_BYTES + (N) * rt::BK * 2) + 256 + tab_smem;    \
+    cfg.dynamicSmemBytes = rt::smem_bytes<N>(E);                                                 \
     cudaFuncSetAttribute(router_select_kernel<N>, cudaFuncAttributeMaxDynamicSharedMemorySize,   \
-                         (int)dyn);                                                              \
-    router_select_kernel<N><<<blocks, rt::THREADS, dyn, stream>>>(                               \
-        mX, mW, T, E, d, k, renorm, tb, home, loc, qhat, logits_out, topk_idx, topk_w,           \
-        chosen_expert, chosen_server, kind, counters, lim);                                      \
+                         (int)cfg.dynamicSmemBytes);                                             \
+    le = cudaLaunchKernelEx(&cfg, router_select_kernel<N>, mX, mW, T, E, d, k, renorm, tb, home, \
+                            loc, qhat, logits_out, topk_idx, topk_w, chosen_expert,              \
+                            chosen_server, kind, counters, lim, split);                          \
   } while (0)
   if (NE == 16) OM_RT_LAUNCH(16);
   else if (NE == 32) OM_RT_LAUNCH(32);
   else OM_RT_LAUNCH(64);
 #undef OM_RT_LAUNCH
+  if (le != cudaSuccess) return cuda_fail(le, "router_select_kernel launch");
   OM_LAUNCHED("router_select_kernel");
   return ORDERMOE_OK;
 }
