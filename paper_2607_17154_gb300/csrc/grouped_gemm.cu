@@ -672,6 +672,12 @@ static int ffn_attrs() {
     if (attr_err == cudaSuccess)
       attr_err = cudaFuncSetAttribute(ffn_gemm_pair_kernel<DOWN>,
                                       cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<GATEUP>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<DOWN>,
+                                      cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
   });
   if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(ffn_gemm_pair_kernel)");
   return ORDERMOE_OK;
@@ -705,6 +711,16 @@ static int max_resident_pairs() {
   return pairs;
 }
 
+// Tile shape: CTA pairs (256-row tiles) when experts average at least 256
+// rows; otherwise single CTAs with 128-row tiles, which compute fewer padding
+// rows for small batches (a decode step: ~32 rows per expert).
+static bool use_pairs(int R, int E) { return (long long)R >= 256LL * E; }
+
+static int single_grid(long long tiles) {
+  const int sms = num_sms();
+  return static_cast<int>(tiles < sms ? tiles : sms);
+}
+
 static int pair_grid(long long tiles) {
   const int pairs_max = max_resident_pairs();
   const long long pairs = tiles < pairs_max ? tiles : pairs_max;
@@ -724,9 +740,15 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
   Args a{};
   a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = d; a.n_tiles = dff / 128; a.b_rows = dff; a.out = H; a.ldo = dff;
-  const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
-  ffn_gemm_pair_kernel<GATEUP><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
-  OM_LAUNCHED("ffn_gemm_pair_kernel<gate_up>");
+  if (use_pairs(R, E)) {
+    const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
+    ffn_gemm_pair_kernel<GATEUP><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
+    OM_LAUNCHED("ffn_gemm_pair_kernel<gate_up>");
+  } else {
+    const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
+    ffn_gemm_kernel<GATEUP><<<single_grid(tiles), THREADS, SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
+    OM_LAUNCHED("ffn_gemm_kernel<gate_up>");
+  }
   return ORDERMOE_OK;
 }
 
@@ -742,9 +764,15 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   Args a{};
   a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = dff; a.n_tiles = d / 256; a.b_rows = d; a.out = Y; a.ldo = d;
-  const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
-  ffn_gemm_pair_kernel<DOWN><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
-  OM_LAUNCHED("ffn_gemm_pair_kernel<down>");
+  if (use_pairs(R, E)) {
+    const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
+    ffn_gemm_pair_kernel<DOWN><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
+    OM_LAUNCHED("ffn_gemm_pair_kernel<down>");
+  } else {
+    const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
+    ffn_gemm_kernel<DOWN><<<single_grid(tiles), THREADS, SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
+    OM_LAUNCHED("ffn_gemm_kernel<down>");
+  }
   return ORDERMOE_OK;
 }
 
