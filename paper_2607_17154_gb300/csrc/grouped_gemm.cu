@@ -172,10 +172,6 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      // the expert weights stream once; the activations are re-read by every N slice
-      // (for the logits GEMM the roles swap: X_cal streams, the router rows stay)
-      const uint64_t pol_a = args.m_major ? l2_policy_evict_first() : l2_policy_evict_last();
-      const uint64_t pol_b = args.m_major ? l2_policy_evict_last() : l2_policy_evict_first();
       for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x) {
         const Tile t = decode(tile, s, args.E, args.n_tiles, args.m_major);
         const int brow = t.e * args.b_rows + t.n * (MODE == GATEUP ? 128 : 256);  // LOGITS: e == 0
@@ -188,13 +184,13 @@ __global__ void __launch_bounds__(THREADS, 1)
           uint8_t* sa = tiles + stage * STAGE_BYTES;
           uint8_t* sb = sa + A_BYTES;
           mbar_arrive_expect_tx(&s.full[stage], STAGE_BYTES);
-          tma_load_2d_hint(sa, &mapA, &s.full[stage], kb * BK, t.m0, pol_a);
+          tma_load_2d(sa, &mapA, &s.full[stage], kb * BK, t.m0);
           if (MODE == GATEUP) {
-            tma_load_2d_hint(sb, &mapB0, &s.full[stage], kb * BK, brow, pol_b);
-            tma_load_2d_hint(sb + BOX_BYTES, &mapB1, &s.full[stage], kb * BK, brow, pol_b);
+            tma_load_2d(sb, &mapB0, &s.full[stage], kb * BK, brow);
+            tma_load_2d(sb + BOX_BYTES, &mapB1, &s.full[stage], kb * BK, brow);
           } else {
-            tma_load_2d_hint(sb, &mapB0, &s.full[stage], kb * BK, brow, pol_b);
-            tma_load_2d_hint(sb + BOX_BYTES, &mapB0, &s.full[stage], kb * BK, brow + 128, pol_b);
+            tma_load_2d(sb, &mapB0, &s.full[stage], kb * BK, brow);
+            tma_load_2d(sb + BOX_BYTES, &mapB0, &s.full[stage], kb * BK, brow + 128);
           }
           issued_mask |= 1u << stage;
           last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
@@ -474,8 +470,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      const uint64_t pol_a = l2_policy_evict_last();   // activations: re-read per N slice
-      const uint64_t pol_b = l2_policy_evict_first();  // expert weights: streamed once
       for (int tile = cluster; tile < total && !*abort; tile += n_clusters) {
         const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
         const int arow = t.m0 + 128 * static_cast<int>(rank);
@@ -492,8 +486,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           uint8_t* sb = sa + BOX_BYTES;
           const uint32_t full_even = mapa_shared(smem_u32(&s.full[stage]), 0);
           if (even) mbar_arrive_expect_tx(&s.full[stage], 2 * P_STAGE_BYTES);
-          tma_load_2d_pair_hint(sa, &mapA, full_even, kb * BK, arow, pol_a);
-          tma_load_2d_pair_hint(sb, mapB, full_even, kb * BK, brow, pol_b);
+          tma_load_2d_pair(sa, &mapA, full_even, kb * BK, arow);
+          tma_load_2d_pair(sb, mapB, full_even, kb * BK, brow);
           issued_mask |= 1u << stage;
           last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
