@@ -29,14 +29,14 @@ UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM bytes (read + write) per launch of the gate/up GEMM at the mixtral_prefill workload, from
-# the ncu capture summarised in profiles/ffn_gemm_gate_up_mixtral_prefill.md, valid only while the
+# the ncu capture summarised in profiles/ffn_gemm_pair_gate_up_mixtral_prefill.md, valid only while the
 # kernel sources hash to the values recorded with it.
 GATE_UP_TRAFFIC = {
-    "bytes": 2173090816,
+    "bytes": 3604226048,
     "sha256": {"paper_2607_17154_gb300/csrc/grouped_gemm.cu":
-               "54bf04f18e3bf96dce70b2c096b0a7dc19eda56fbe66bf983d119f040d63b634",
+               "aa9dd553a0eb5f820c047bd0de26970fc2d53d1861b8f81259815887567e39e9",
                "paper_2607_17154_gb300/csrc/common.cuh":
-               "3df474ac82e60f13f0feed5b9c9d5dc72f79ef090734595e235722b2624e6103"},
+               "171af56f0eacc7d7923d83f259f65b4fcbfa9011a8dd1552a248c1b548e556aa"},
 }
 
 
