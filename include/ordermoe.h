@@ -153,6 +153,28 @@ int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, const float* l
                           uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
                           ordermoe_stream_t stream);
 
+/* Alg. 2 with look-ahead horizon H (Eqs. 41-43): as ordermoe_route_select,
+ * but each candidate (m, k) of this layer costs g_l(m, k) + Phi^(H-1)(m, k),
+ * the expected cheapest cost of the next H - 1 layers from server m:
+ *   Phi^(h)(m, k) = sum_{k'} P_l(k -> k') min over the feasible (m', k'') of
+ *                   target k' at layer l + 1 (from server m, with the loss
+ *                   accumulated so far) of g_{l+1}(m', k'') + Phi^(h-1)(m', k'')
+ * (Eq. 42 read with the bracket closing after the per-step cost; future layers
+ * have a single target and no distinct-expert rule).
+ *   tables      H consecutive layer tables (this layer first), tables_stride
+ *               bytes apart (a multiple of 16, >= ordermoe_tables_bytes(E, M))
+ *   H           1..4 (1 gives exactly ordermoe_route_select's result)
+ *   P           [H-1][E][E] f32: P_l .. P_{l+H-2} (ordermoe_transitions)
+ * Every product and sum of Phi is one rounded fp32 operation, next targets in
+ * ascending order, so decisions are reproducible bit for bit. */
+int ordermoe_route_select_lookahead(const uint16_t* X, const uint16_t* W_r, const float* logits_in,
+                                    int T, int E, int d, int k, int renorm, const void* tables,
+                                    size_t tables_stride, int H, const float* P,
+                                    const uint8_t* home, uint8_t* loc, float* qhat,
+                                    float* logits_out, int32_t* topk_idx, float* topk_w,
+                                    int32_t* chosen_expert, uint8_t* chosen_server, uint8_t* kind,
+                                    int32_t* counters, ordermoe_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * Token permutation: histogram + prefix sum + stable scatter of the T*k
  * (token, slot) entries by executed expert, and the row gather of X into
@@ -273,6 +295,20 @@ size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N);
 int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d, int64_t N,
                         int k_freq, float* sim, int32_t* counts, void* workspace,
                         size_t workspace_bytes, ordermoe_stream_t stream);
+
+/* After ordermoe_similarity returns (and until the workspace is reused), the
+ * first N * L * E * 4 bytes of its workspace hold the calibration logits
+ * H[n][l][e] in fp32, token-major: the input ordermoe_transitions takes. */
+
+/* Expert transition statistics, Eq. 41, from calibration logits
+ * [N][L][E] f32 (token-major, layer-stacked): n_l(k -> k') counts, for every
+ * token, each pair (k in its top-k_freq at layer l, k' in its top-k_freq at
+ * layer l + 1) -- the paper has one target per token; with top-k every routed
+ * pair counts. P_l(k -> k') = n / sum_k'' n(k -> k'') (fp64, rounded once;
+ * a row without transitions is 0).
+ *   counts [L-1][E][E] i32 out, P [L-1][E][E] f32 out. Needs L >= 2. */
+int ordermoe_transitions(const float* logits, int64_t N, int L, int E, int k_freq, int32_t* counts,
+                         float* P, ordermoe_stream_t stream);
 
 /* Activation counts of Eq. 5 from given logits [N][E] f32 (top-k_freq per
  * token, ties to the lower index). counts [E] i32 out (overwritten). */

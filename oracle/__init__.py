@@ -51,6 +51,9 @@ def lib():
             "orc_importance": [_P, _P, _P, _I, _D, _D, _P],
             "orc_place": [_P, _P, _P, _I, _I, _I, _P, _D, _D, _P, _P],
             "orc_coverage": [_P, _P, _I, _I, _I, _P],
+            "orc_transitions": [_P, _I64, _I, _I, _I, _P, _P],
+            "orc_select_lookahead": [_P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P,
+                                     _P, _F, _P, _P, _P, _P, _P, _P],
         }
         for name, args in sigs.items():
             fn = getattr(L, name)
@@ -224,3 +227,38 @@ def coverage(placement_l, group_l, K):
     cov = np.empty((M, K), np.uint8)
     _check(lib().orc_coverage(_ptr(placement_l), _ptr(group_l), E, M, K, _ptr(cov)), "orc_coverage")
     return cov
+
+
+def transitions(logits, kf):
+    """logits [N, L, E] f32 -> (counts [L-1, E, E] i32, P [L-1, E, E] f32), Eq. 41."""
+    logits = _c(logits, np.float32)
+    N, L, E = logits.shape
+    cnt = np.empty((L - 1, E, E), np.int32); P = np.empty((L - 1, E, E), np.float32)
+    _check(lib().orc_transitions(_ptr(logits), N, L, E, kf, _ptr(cnt), _ptr(P)), "orc_transitions")
+    return cnt, P
+
+
+def select_lookahead(idx, tabs, P, home, loc, qhat):
+    """Alg. 2 with horizon H = len(tabs) (Eqs. 42-43); tabs[0] is the current layer's
+    Tables, tabs[1:] the next layers'; P [H-1, E, E] the transition matrices."""
+    idx = _c(idx, np.int32); T, k = idx.shape
+    H = len(tabs); t0 = tabs[0]
+    P = _c(P, np.float32).reshape(-1)
+    if H > 1:
+        assert P.size == (H - 1) * t0.E * t0.E
+    else:
+        P = np.zeros(1, np.float32)
+    arr = lambda name, ct: (ct * max(H - 1, 1))(*[getattr(t, name).ctypes.data_as(ctypes.c_void_p)
+                                                 for t in tabs[1:]] or [None])
+    keep = [t for t in tabs]
+    nQ, nC, nS, nA, nM = (arr(n, ctypes.c_void_p) for n in ("Qtab", "Cq", "subst", "A", "pmask"))
+    home = _c(home, np.uint8); loc = _c(loc, np.uint8).copy(); qhat = _c(qhat, np.float32).copy()
+    chosen = np.empty((T, k), np.int32); server = np.empty((T, k), np.uint8)
+    kind = np.empty((T, k), np.uint8)
+    rc = lib().orc_select_lookahead(_ptr(idx), T, t0.E, k, t0.M, H, _ptr(t0.Qtab), _ptr(t0.Cq),
+                                    _ptr(t0.subst), _ptr(t0.A), _ptr(t0.pmask), nQ, nC, nS, nA, nM,
+                                    _ptr(P), float(t0.qbar), _ptr(home), _ptr(loc), _ptr(qhat),
+                                    _ptr(chosen), _ptr(server), _ptr(kind))
+    del keep
+    _check(rc, "orc_select_lookahead")
+    return chosen, server, kind, loc, qhat

@@ -30,6 +30,7 @@
 //    the used memory b_m accumulates over layers (Alg. 1 initialises it once).
 #include <algorithm>
 #include <cmath>
+#include <limits>
 #include <cstdint>
 #include <cstring>
 #include <vector>
@@ -487,6 +488,163 @@ int orc_place(const int32_t* group, const double* importance, const double* p, i
   }
   for (int m = 0; m < M; ++m) used[m] = b[m];
   return overflow ? ORC_CAPACITY : ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Expert transition statistics, Eq. 41, from calibration logits [N][L][E]:
+// for each token, every pair (k in top-kf of layer l, k' in top-kf of layer
+// l+1) counts one transition k -> k' (the paper has one target per token; with
+// top-k each routed pair counts). P_l(k -> k') = n / sum_k'' n(k -> k''), fp64
+// then rounded to fp32; a row with no transitions is all zero.
+int orc_transitions(const float* logits, int64_t N, int L, int E, int kf, int32_t* count,
+                    float* P) {
+  if (L < 2 || E <= 0 || kf <= 0 || kf > E) return ORC_BAD_ARG;
+  std::memset(count, 0, sizeof(int32_t) * (size_t)(L - 1) * E * E);
+  std::vector<int> cur(kf), nxt(kf), order(E);
+  auto topk = [&](const float* l, std::vector<int>& out) {
+    for (int e = 0; e < E; ++e) order[e] = e;
+    std::sort(order.begin(), order.end(),
+              [&](int a, int b) { return ranks_before(l[a], a, l[b], b); });
+    for (int j = 0; j < kf; ++j) out[j] = order[j];
+  };
+  for (int64_t n = 0; n < N; ++n) {
+    topk(logits + (n * L) * E, cur);
+    for (int l = 0; l + 1 < L; ++l) {
+      topk(logits + (n * L + l + 1) * E, nxt);
+      for (int a : cur)
+        for (int b : nxt) count[((size_t)l * E + a) * E + b]++;
+      cur = nxt;
+    }
+  }
+  for (int l = 0; l + 1 < L; ++l)
+    for (int a = 0; a < E; ++a) {
+      double row = 0.0;
+      for (int b = 0; b < E; ++b) row += count[((size_t)l * E + a) * E + b];
+      for (int b = 0; b < E; ++b)
+        P[((size_t)l * E + a) * E + b] =
+            row > 0.0 ? static_cast<float>(count[((size_t)l * E + a) * E + b] / row) : 0.0f;
+    }
+  return ORC_OK;
+}
+
+// One layer's selection tables as the look-ahead reads them (see orc_tables).
+struct OrcTab {
+  const float* Qtab;
+  const float* Cq;
+  const uint64_t* subst;
+  const float* A;
+  const uint32_t* pmask;
+};
+
+// Look-ahead cost-to-go of Eq. 42 with h future layers (h >= 1): being at
+// server m after executing expert kx at layer l with accumulated loss qacc,
+//   Phi^(h) = sum_{k'} P_l(kx -> k') * min over the feasible pairs (m', k'')
+//             of target k' at layer l+1 (Eq. 40, from server m) of
+//             [ g_{l+1}(m', k'' | s = m) + Phi^(h-1)_{l+1}(m', k'') ],
+// with Phi^(0) = 0. In the future layers a token has the single target k'
+// (no distinct-expert rule) and the same home server a; the loss of a
+// future substitute adds to qacc. fp32 arithmetic: each product and sum is
+// one rounded fp32 operation, k' in ascending order.
+float orc_phi(int h, const OrcTab* tabs, const float* P, int E, int M, int a, int m, int kx,
+              float qacc, float qbar) {
+  if (h <= 0) return 0.0f;
+  const OrcTab& t1 = tabs[1];
+  float acc = 0.0f;
+  for (int kt = 0; kt < E; ++kt) {
+    const float p = P[(size_t)kx * E + kt];
+    if (p == 0.0f) continue;
+    float best = INFINITY;
+    for (int kk = 0; kk < E; ++kk) {
+      const bool exact = (kk == kt);
+      float q2 = qacc;
+      if (!exact) {
+        if (!((t1.subst[kt] >> kk) & 1u)) continue;
+        if (!(qacc + t1.Qtab[kt * E + kk] <= qbar)) continue;
+        q2 = qacc + t1.Qtab[kt * E + kk];
+      }
+      for (int m2 = 0; m2 < M; ++m2) {
+        if (!((t1.pmask[kk] >> m2) & 1u)) continue;
+        float c = t1.A[((int64_t)a * M + m) * M + m2] + (exact ? 0.0f : t1.Cq[kt * E + kk]);
+        if (h > 1) c = c + orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar);
+        if (c < best) best = c;
+      }
+    }
+    const float term = p * best;
+    acc = acc + term;
+  }
+  return acc;
+}
+
+// Alg. 2 with horizon H (Eq. 43): as orc_select, but each candidate (m, k)
+// of layer l costs g_l(m, k) + Phi^(H-1)(m, k) (one fp32 add), the cost-to-go
+// computed with the tables of layers l+1 .. l+H-1 (tabs[1..H-1]) and the
+// transition matrices P_l .. P_{l+H-2} (P, [H-1][E][E]). H = 1 is orc_select.
+int orc_select_lookahead(const int32_t* idx, int T, int E, int k, int M, int H, const float* Qtab,
+                         const float* Cq, const uint64_t* subst, const float* A,
+                         const uint32_t* pmask, const float* const* nQtab, const float* const* nCq,
+                         const uint64_t* const* nsubst, const float* const* nA,
+                         const uint32_t* const* npmask, const float* P, float qbar,
+                         const uint8_t* home, uint8_t* loc, float* qhat, int32_t* chosen,
+                         uint8_t* server, uint8_t* kind) {
+  if (E <= 0 || E > 64 || M <= 0 || M > 32 || k <= 0 || k > E || H < 1 || H > 4) return ORC_BAD_ARG;
+  std::vector<OrcTab> tabs(H);
+  tabs[0] = OrcTab{Qtab, Cq, subst, A, pmask};
+  for (int h = 1; h < H; ++h) tabs[h] = OrcTab{nQtab[h - 1], nCq[h - 1], nsubst[h - 1], nA[h - 1], npmask[h - 1]};
+  for (int t = 0; t < T; ++t) {
+    const int a = home[t];
+    const int s = loc[t];
+    if (a >= M || s >= M) return ORC_BAD_ARG;
+    float q = qhat[t];
+    uint64_t taken = 0;
+    for (int j = 0; j < k; ++j) taken |= (uint64_t)1 << idx[(int64_t)t * k + j];
+    int first_server = -1;
+    for (int j = 0; j < k; ++j) {
+      const int r = idx[(int64_t)t * k + j];
+      if (r < 0 || r >= E) return ORC_BAD_ARG;
+      bool have = false;
+      float best_cost = 0.0f;
+      int best_sub = 0, best_away = 0, best_m = 0, best_k = 0;
+      for (int kk = 0; kk < E; ++kk) {
+        const bool exact = (kk == r);
+        if (!exact) {
+          if (!((subst[r] >> kk) & 1u)) continue;
+          if ((taken >> kk) & 1u) continue;
+          if (!(q + Qtab[r * E + kk] <= qbar)) continue;
+        }
+        const float qn = exact ? q : q + Qtab[r * E + kk];
+        for (int m = 0; m < M; ++m) {
+          if (!((pmask[kk] >> m) & 1u)) continue;
+          float cost = A[((int64_t)a * M + s) * M + m] + (exact ? 0.0f : Cq[r * E + kk]);
+          cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, m, kk, qn, qbar);
+          const int sub = exact ? 0 : 1;
+          const int away = (m != s) ? 1 : 0;
+          bool better;
+          if (!have) better = true;
+          else if (cost != best_cost) better = cost < best_cost;
+          else if (sub != best_sub) better = sub < best_sub;
+          else if (away != best_away) better = away < best_away;
+          else if (m != best_m) better = m < best_m;
+          else better = kk < best_k;
+          if (better) {
+            have = true;
+            best_cost = cost; best_sub = sub; best_away = away; best_m = m; best_k = kk;
+          }
+        }
+      }
+      if (!have) return ORC_BAD_ARG;
+      chosen[(int64_t)t * k + j] = best_k;
+      server[(int64_t)t * k + j] = static_cast<uint8_t>(best_m);
+      kind[(int64_t)t * k + j] = static_cast<uint8_t>(2 * best_away + best_sub);
+      if (best_sub) {
+        taken |= (uint64_t)1 << best_k;
+        q = q + Qtab[r * E + best_k];
+      }
+      if (j == 0) first_server = best_m;
+    }
+    loc[t] = static_cast<uint8_t>(first_server);
+    qhat[t] = q;
+  }
+  return ORC_OK;
 }
 
 // Local group coverage, Eq. 32 (indices read as y_{m,l,g} = 1 when server m

@@ -50,6 +50,9 @@ _SIGNATURES = {
     "ordermoe_layer_scratch_bytes": ([_I, _I, _I, _I, _I], _SZ),
     "ordermoe_layer_forward": ([_P, _I, _P, _P, _P, _P, _P, _P, _I, _P], _I),
     "ordermoe_dispatch_noalloc": ([_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P], _I),
+    "ordermoe_transitions": ([_P, _I64, _I, _I, _I, _P, _P, _P], _I),
+    "ordermoe_route_select_lookahead": ([_P, _P, _P, _I, _I, _I, _I, _I, _P, _SZ, _I, _P, _P, _P,
+                                         _P, _P, _P, _P, _P, _P, _P, _P, _P], _I),
 }
 
 
@@ -310,3 +313,25 @@ def ordermoe_dispatch_noalloc(chosen_expert, X, T, k, E, d, offsets, row_token, 
                                          _ptr(row_token), _ptr(row_of), _ptr(X_perm),
                                          _stream(stream))
     _check("ordermoe_dispatch_noalloc", rc)
+
+
+def ordermoe_transitions(logits, N, L, E, k_freq, counts, P, stream=None):
+    _dt(logits, torch.float32, "logits"); _dt(counts, torch.int32, "counts"); _dt(P, torch.float32, "P")
+    _check("ordermoe_transitions",
+           lib().ordermoe_transitions(_ptr(logits), N, L, E, k_freq, _ptr(counts), _ptr(P),
+                                      _stream(stream)))
+
+
+def ordermoe_route_select_lookahead(X, W_r, logits_in, T, E, d, k, renorm, tables, tables_stride, H,
+                                    P, home, loc, qhat, logits_out, topk_idx, topk_w,
+                                    chosen_expert, chosen_server, kind, counters=None, stream=None):
+    """tables: a uint8 device tensor holding H (or more) consecutive layer tables,
+    tables_stride bytes apart, starting with this layer's."""
+    _dt(X, torch.bfloat16, "X"); _dt(W_r, torch.bfloat16, "W_r"); _dt(logits_in, torch.float32, "logits_in")
+    _dt(P, torch.float32, "P")
+    rc = lib().ordermoe_route_select_lookahead(
+        _ptr(X), _ptr(W_r), _ptr(logits_in), T, E, d, k, int(renorm), _ptr(tables), int(tables_stride),
+        int(H), _ptr(P), _ptr(home), _ptr(loc), _ptr(qhat), _ptr(logits_out), _ptr(topk_idx),
+        _ptr(topk_w), _ptr(chosen_expert), _ptr(chosen_server), _ptr(kind), _ptr(counters),
+        _stream(stream))
+    _check("ordermoe_route_select_lookahead", rc)

@@ -124,6 +124,73 @@ __device__ bool load_tables(const uint8_t* __restrict__ tab, int E, SelSmem& sm,
   return true;
 }
 
+// Look-ahead context (Eqs. 41-43): the tables of the next layers follow the
+// current layer's at a fixed byte stride; P holds P_l .. P_{l+H-2}.
+struct Lookahead {
+  int H;                 // horizon; 1 = myopic (Phi = 0)
+  size_t stride;         // bytes between consecutive layers' tables
+  const float* P;        // [H-1][E][E]
+};
+
+// Cost-to-go of Eq. 42 with D future layers, from server m after executing
+// expert kx with accumulated loss qacc: sum over next targets k' (ascending)
+// of P(kx -> k') times the cheapest feasible (m', k'') of the next layer
+// (Eq. 40 from server m; a single target, no distinct-expert rule), each
+// plus its own cost-to-go. Every product and sum is one rounded fp32
+// operation, so the value is reproducible bit for bit.
+template <int D>
+__device__ float lookahead_phi(const uint8_t* __restrict__ tnext, size_t stride,
+                               const float* __restrict__ P, int E, int M, int a, int m, int kx,
+                               float qacc, float qbar) {
+  const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
+  const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
+  const float* A1 = reinterpret_cast<const float*>(tnext + off_a(E));
+  const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
+  const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
+  float acc = 0.0f;
+  for (int kt = 0; kt < E; ++kt) {
+    const float p = __ldg(P + (size_t)kx * E + kt);
+    if (p == 0.0f) continue;
+    float best = INFINITY;
+    unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);  // substitutes and the target
+    while (cand) {
+      const int kk = __ffsll(static_cast<long long>(cand)) - 1;
+      cand &= cand - 1;
+      const bool exact = (kk == kt);
+      float cq = 0.0f, q2 = qacc;
+      if (!exact) {
+        const float qk = __ldg(Q1 + kt * E + kk);
+        if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
+        q2 = __fadd_rn(qacc, qk);
+        cq = __ldg(C1 + kt * E + kk);
+      }
+      uint32_t pm = __ldg(pm1 + kk);
+      while (pm) {
+        const int m2 = __ffs(pm) - 1;
+        pm &= pm - 1;
+        float c = __fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq);
+        if (D > 1)
+          c = __fadd_rn(c, lookahead_phi<(D > 1 ? D - 1 : 1)>(tnext + stride, stride, P + E * E, E,
+                                                              M, a, m2, kk, q2, qbar));
+        best = fminf(best, c);
+      }
+    }
+    acc = __fadd_rn(acc, __fmul_rn(p, best));
+  }
+  return acc;
+}
+
+__device__ __forceinline__ float lookahead_cost(const Lookahead& la, const uint8_t* tab, int E,
+                                                int M, int a, int m, int kx, float qacc,
+                                                float qbar) {
+  switch (la.H) {
+    case 2: return lookahead_phi<1>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar);
+    case 3: return lookahead_phi<2>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar);
+    case 4: return lookahead_phi<3>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar);
+    default: return 0.0f;
+  }
+}
+
 // One token: softmax over E, top-k, then Alg. 2 (H = 1) per slot in rank
 // order (Eqs. 36-44). The logits are in registers (lg[e], e < E <= EMAX).
 // The argmin of Eq. 43 packs (fp32 cost bits, substitute, away, server,
@@ -132,7 +199,8 @@ __device__ bool load_tables(const uint8_t* __restrict__ tab, int E, SelSmem& sm,
 template <int EMAX>
 __device__ __forceinline__ void select_token(
     int t, const float (&lg)[EMAX], int E, int k, int renorm, int M, float qbar,
-    const float* __restrict__ gA, const SelSmem& sm, const float* s_Q, const float* s_Cq,
+    const float* __restrict__ gA, const uint8_t* __restrict__ tab, const Lookahead& la,
+    const SelSmem& sm, const float* s_Q, const float* s_Cq,
     const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
     int32_t* __restrict__ topk_idx, float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
     uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out, int (&kind_count)[4]) {
@@ -198,17 +266,19 @@ __device__ __forceinline__ void select_token(
     for (int ki = 0; ki <= nsub; ++ki) {
       const int kk = (ki == 0) ? r : sm.sublist[r * 64 + ki - 1];
       const bool sub = (ki != 0);
-      float cq = 0.0f;
+      float cq = 0.0f, qn = q;
       if (sub) {
         if ((taken >> kk) & 1ull) continue;
         if (!(__fadd_rn(q, s_Q[r * E + kk]) <= qbar)) continue;  // Eq. 40 budget
         cq = s_Cq[r * E + kk];
+        qn = __fadd_rn(q, s_Q[r * E + kk]);
       }
       uint32_t pm = sm.pmask[kk];
       while (pm) {
         const int m = __ffs(pm) - 1;
         pm &= pm - 1;
-        const float cost = __fadd_rn(__ldg(Aas + m), cq);
+        float cost = __fadd_rn(__ldg(Aas + m), cq);
+        if (la.H > 1) cost = __fadd_rn(cost, lookahead_cost(la, tab, E, M, a, m, kk, qn, qbar));
         const unsigned long long key =
             (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
             (static_cast<unsigned long long>(sub ? 1u : 0u) << 31) |
@@ -259,7 +329,7 @@ __global__ void __launch_bounds__(128) select_kernel(
     float* __restrict__ qhat, float* __restrict__ logits_out, int32_t* __restrict__ topk_idx,
     float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
     uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
-    int32_t* __restrict__ counters) {
+    int32_t* __restrict__ counters, Lookahead la) {
   __shared__ SelSmem sm;
   extern __shared__ __align__(16) float s_dyn[];
   float* s_Q = s_dyn;
@@ -277,8 +347,8 @@ __global__ void __launch_bounds__(128) select_kernel(
     for (int e = 0; e < EMAX; ++e) lg[e] = (e < E) ? logits_in[(size_t)t * E + e] : 0.0f;
     if (logits_out != nullptr)
       for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
-    select_token<EMAX>(t, lg, E, k, renorm, M, qbar, gA, sm, s_Q, s_Cq, home, loc, qhat, topk_idx,
-                       topk_w, chosen_expert, chosen_server, kind_out, kind_count);
+    select_token<EMAX>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
+                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count);
   }
   flush_kind_counts(sm, kind_count, counters);
   __syncthreads();
@@ -332,7 +402,8 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
     float* __restrict__ logits_out, int32_t* __restrict__ topk_idx, float* __restrict__ topk_w,
     int32_t* __restrict__ chosen_expert, uint8_t* __restrict__ chosen_server,
-    uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters, uint64_t limit_ns, int split) {
+    uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters, uint64_t limit_ns, int split,
+    Lookahead la) {
   constexpr int B_BYTES = NE * rt::BK * 2;
   constexpr int STAGE_BYTES = rt::A_BYTES + B_BYTES;
   constexpr int STAGES = rt::stages<NE>();
@@ -480,8 +551,8 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       const int M = reinterpret_cast<const int32_t*>(tab)[2];
       const float qbar = reinterpret_cast<const float*>(tab)[5];
       const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
-      select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, sm, s_Q, s_Cq, home, loc, qhat, topk_idx,
-                       topk_w, chosen_expert, chosen_server, kind_out, kind_count);
+      select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
+                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count);
     }
     flush_kind_counts(sm, kind_count, counters);
   }
@@ -538,13 +609,12 @@ extern "C" int ordermoe_build_tables(const float* sim, const int32_t* group,
   return ORDERMOE_OK;
 }
 
-extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, const float* logits_in,
-                                     int T, int E, int d, int k, int renorm, const void* tables,
-                                     size_t tables_bytes_, const uint8_t* home, uint8_t* loc,
-                                     float* qhat, float* logits_out, int32_t* topk_idx,
-                                     float* topk_w, int32_t* chosen_expert,
-                                     uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
-                                     ordermoe_stream_t stream) {
+static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float* logits_in, int T,
+                             int E, int d, int k, int renorm, const void* tables,
+                             size_t tables_bytes_, Lookahead la, const uint8_t* home, uint8_t* loc,
+                             float* qhat, float* logits_out, int32_t* topk_idx, float* topk_w,
+                             int32_t* chosen_expert, uint8_t* chosen_server, uint8_t* kind,
+                             int32_t* counters, cudaStream_t stream) {
   if (T < 0) return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: T < 0");
   if (E <= 0 || E > ORDERMOE_MAX_EXPERTS || k <= 0 || k > ORDERMOE_MAX_TOPK || k > E)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select: need 1 <= k <= min(E, 8), E <= 64");
@@ -573,7 +643,7 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
     select_kernel<EM><<<blocks, 128, tab_smem, stream>>>(logits_in, T, E, k, renorm, tb, home,   \
                                                          loc, qhat, logits_out, topk_idx, topk_w, \
                                                          chosen_expert, chosen_server, kind,      \
-                                                         counters);                               \
+                                                         counters, la);                           \
   } while (0)
     if (E <= 8) OM_SEL_LAUNCH(8);
     else if (E <= 16) OM_SEL_LAUNCH(16);
@@ -614,7 +684,7 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
                          (int)cfg.dynamicSmemBytes);                                             \
     le = cudaLaunchKernelEx(&cfg, router_select_kernel<N>, mX, mW, T, E, d, k, renorm, tb, home, \
                             loc, qhat, logits_out, topk_idx, topk_w, chosen_expert,              \
-                            chosen_server, kind, counters, lim, split);                          \
+                            chosen_server, kind, counters, lim, split, la);                      \
   } while (0)
   if (NE == 16) OM_RT_LAUNCH(16);
   else if (NE == 32) OM_RT_LAUNCH(32);
@@ -623,4 +693,35 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
   if (le != cudaSuccess) return cuda_fail(le, "router_select_kernel launch");
   OM_LAUNCHED("router_select_kernel");
   return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, const float* logits_in,
+                                     int T, int E, int d, int k, int renorm, const void* tables,
+                                     size_t tables_bytes_, const uint8_t* home, uint8_t* loc,
+                                     float* qhat, float* logits_out, int32_t* topk_idx,
+                                     float* topk_w, int32_t* chosen_expert,
+                                     uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
+                                     ordermoe_stream_t stream) {
+  Lookahead la{1, 0, nullptr};
+  return route_select_impl(X, W_r, logits_in, T, E, d, k, renorm, tables, tables_bytes_, la, home,
+                           loc, qhat, logits_out, topk_idx, topk_w, chosen_expert, chosen_server,
+                           kind, counters, stream);
+}
+
+extern "C" int ordermoe_route_select_lookahead(
+    const uint16_t* X, const uint16_t* W_r, const float* logits_in, int T, int E, int d, int k,
+    int renorm, const void* tables, size_t tables_stride, int H, const float* P,
+    const uint8_t* home, uint8_t* loc, float* qhat, float* logits_out, int32_t* topk_idx,
+    float* topk_w, int32_t* chosen_expert, uint8_t* chosen_server, uint8_t* kind,
+    int32_t* counters, ordermoe_stream_t stream) {
+  if (H < 1 || H > 4) return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select_lookahead: need 1 <= H <= 4");
+  if (E <= 0 || E > ORDERMOE_MAX_EXPERTS)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select_lookahead: need 1 <= E <= 64");
+  if (H > 1 && (!P || tables_stride < om::tables_bytes(E, 1) || (tables_stride & 15u)))
+    return fail(ORDERMOE_ERR_INVALID_ARG,
+                "route_select_lookahead: need P and a 16-byte multiple table stride for H > 1");
+  Lookahead la{H, tables_stride, P};
+  return route_select_impl(X, W_r, logits_in, T, E, d, k, renorm, tables, tables_stride, la, home,
+                           loc, qhat, logits_out, topk_idx, topk_w, chosen_expert, chosen_server,
+                           kind, counters, stream);
 }

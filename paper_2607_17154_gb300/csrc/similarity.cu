@@ -153,6 +153,71 @@ __global__ void __launch_bounds__(256) counts_kernel(const float* __restrict__ H
   if (threadIdx.x < E && cnt[threadIdx.x]) atomicAdd(&counts[(size_t)l * E + threadIdx.x], cnt[threadIdx.x]);
 }
 
+// Top-kf of one token's E logits (rank order: larger first, lower index on
+// ties) as a bit set.
+template <int EMAX>
+__device__ __forceinline__ unsigned long long topk_set(const float* __restrict__ row, int E, int kf) {
+  float v[EMAX];
+#pragma unroll
+  for (int e = 0; e < EMAX; ++e) v[e] = (e < E) ? row[e] : 0.0f;
+  unsigned long long used = 0;
+  for (int j = 0; j < kf; ++j) {
+    int best = -1;
+    float bv = 0.0f;
+#pragma unroll
+    for (int e = 0; e < EMAX; ++e)
+      if (e < E && !((used >> e) & 1ull) && (best < 0 || v[e] > bv)) {
+        best = e;
+        bv = v[e];
+      }
+    used |= 1ull << best;
+  }
+  return used;
+}
+
+// Transition counts of Eq. 41 for the layer pair (l, l + 1) = blockIdx.y:
+// each token adds one to n_l(k -> k') for every k in its top-kf at layer l
+// and k' in its top-kf at layer l + 1 (integer atomics: order-independent).
+template <int EMAX>
+__global__ void __launch_bounds__(256) transitions_kernel(const float* __restrict__ logits,
+                                                          int64_t N, int L, int E, int kf,
+                                                          int32_t* __restrict__ counts) {
+  __shared__ int h[64 * 64];
+  const int l = blockIdx.y;
+  for (int i = threadIdx.x; i < E * E; i += blockDim.x) h[i] = 0;
+  __syncthreads();
+  for (int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; n < N;
+       n += (int64_t)gridDim.x * blockDim.x) {
+    unsigned long long a = topk_set<EMAX>(logits + ((size_t)n * L + l) * E, E, kf);
+    const unsigned long long b = topk_set<EMAX>(logits + ((size_t)n * L + l + 1) * E, E, kf);
+    while (a) {
+      const int x = __ffsll(static_cast<long long>(a)) - 1;
+      a &= a - 1;
+      unsigned long long bb = b;
+      while (bb) {
+        const int y = __ffsll(static_cast<long long>(bb)) - 1;
+        bb &= bb - 1;
+        atomicAdd(&h[x * E + y], 1);
+      }
+    }
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < E * E; i += blockDim.x)
+    if (h[i]) atomicAdd(&counts[(size_t)l * E * E + i], h[i]);
+}
+
+// P_l(k -> k') = n / sum_k'' n (fp64, rounded once to fp32); 0 for an empty row.
+__global__ void transitions_finish_kernel(const int32_t* __restrict__ counts, int rows, int E,
+                                          float* __restrict__ P) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= rows) return;
+  const int32_t* c = counts + (size_t)r * E;
+  double row = 0.0;
+  for (int b = 0; b < E; ++b) row = __dadd_rn(row, static_cast<double>(c[b]));
+  for (int b = 0; b < E; ++b)
+    P[(size_t)r * E + b] = row > 0.0 ? __double2float_rn(__ddiv_rn(static_cast<double>(c[b]), row)) : 0.0f;
+}
+
 // grid (L, 16), 256 threads: block (l, b) reduces the 256 Gram entries
 // i * 64 + j in [256 b, 256 b + 256) over the chunks, in chunk order (fp64).
 __global__ void __launch_bounds__(256) gram_reduce_kernel(const float* __restrict__ gpart,
@@ -501,5 +566,28 @@ extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, in
   OM_LAUNCHED("group_kernel");
   place_kernel<<<1, 32, 0, stream>>>(group, porder_scratch, L, E, M, pp, p, C, placement, used, status);
   OM_LAUNCHED("place_kernel");
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_transitions(const float* logits, int64_t N, int L, int E, int k_freq,
+                                    int32_t* counts, float* P, ordermoe_stream_t stream) {
+  if (L < 2 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E || N < 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "transitions: need L >= 2, 1 <= k_freq <= E <= 64");
+  if (!counts || !P || (N > 0 && !logits)) return fail(ORDERMOE_ERR_INVALID_ARG, "transitions: null pointer");
+  OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * (size_t)(L - 1) * E * E, stream));
+  if (N > 0) {
+    int64_t blocks = (N + 255) / 256;
+    const int64_t cap = (num_sms() * 4 + L - 2) / (L - 1);
+    if (blocks > cap) blocks = cap;
+    const dim3 grid(static_cast<unsigned>(blocks), L - 1);
+    if (E <= 8) transitions_kernel<8><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
+    else if (E <= 16) transitions_kernel<16><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
+    else if (E <= 32) transitions_kernel<32><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
+    else transitions_kernel<64><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
+    OM_LAUNCHED("transitions_kernel");
+  }
+  const int rows = (L - 1) * E;
+  transitions_finish_kernel<<<(rows + 127) / 128, 128, 0, stream>>>(counts, rows, E, P);
+  OM_LAUNCHED("transitions_finish_kernel");
   return ORDERMOE_OK;
 }

@@ -49,11 +49,13 @@ class MoELayer:
         return y
 
 
-def build_tables(sim, group, placement, theta, qbar, sp, device):
+def build_tables(sim, group, placement, theta, qbar, sp, device, out=None):
     """Device tables for one layer from host arrays (sim, group, placement) and
-    server parameters sp (synth.ServerParams)."""
+    server parameters sp (synth.ServerParams); written into `out` (a uint8
+    device tensor, e.g. one slice of a stack of layers' tables) when given."""
     E = sim.shape[0]; M = placement.shape[0]
-    t = torch.zeros(B.ordermoe_tables_bytes(E, M), dtype=torch.uint8, device=device)
+    t = out if out is not None else torch.zeros(B.ordermoe_tables_bytes(E, M), dtype=torch.uint8,
+                                                device=device)
     f = lambda a, dt: torch.as_tensor(a).to(device=device, dtype=dt).contiguous()
     B.ordermoe_build_tables(f(sim, torch.float32), f(group, torch.int32), f(placement, torch.uint8),
                             theta, qbar, f(sp.F, torch.float64), f(sp.B, torch.float64),

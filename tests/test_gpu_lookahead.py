@@ -1,0 +1,151 @@
+"""GPU parity of the look-ahead selection (Eqs. 41-43): transition statistics
+and the depth-H cost-to-go, against the oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2607_17154_gb300 import binding as B
+from paper_2607_17154_gb300 import synth
+from paper_2607_17154_gb300.layer import build_tables
+
+pytestmark = pytest.mark.gpu
+
+DEV = "cuda:0"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    B.lib()
+    yield
+    code, detail = B.ordermoe_device_error()
+    assert code == 0, (code, detail)
+
+
+@pytest.mark.parametrize("N,L,E,kf", [(5000, 4, 8, 2), (3000, 3, 64, 6), (100, 2, 5, 5)])
+def test_transitions_given_logits_bit_exact(N, L, E, kf):
+    rng = np.random.default_rng(N + E)
+    logits = rng.standard_normal((N, L, E)).astype(np.float32)
+    logits[:7] = 0.25                                   # ties
+    cnt = torch.empty(L - 1, E, E, dtype=torch.int32, device=DEV)
+    P = torch.empty(L - 1, E, E, dtype=torch.float32, device=DEV)
+    B.ordermoe_transitions(torch.as_tensor(logits).to(DEV), N, L, E, kf, cnt, P)
+    rc, rP = oracle.transitions(logits, kf)
+    np.testing.assert_array_equal(cnt.cpu().numpy(), rc)
+    np.testing.assert_array_equal(P.cpu().numpy(), rP)
+
+
+def stack_tables(rng, L, E, M, qbar, cheap_links):
+    """L layers' tables, random groups/placements, as one device buffer plus the
+    oracle's own copies."""
+    stride = B.ordermoe_tables_bytes(E, M)
+    buf = torch.zeros(L * stride, dtype=torch.uint8, device=DEV)
+    otabs = []
+    for l in range(L):
+        Wt = rng.standard_normal((E, 6)); Wt[:, 0] += 3.0 * (np.arange(E) % 3)
+        nrm = np.linalg.norm(Wt, axis=1, keepdims=True)
+        sim = ((Wt / nrm) @ (Wt / nrm).T).astype(np.float32); np.fill_diagonal(sim, 1.0)
+        group = (np.arange(E) % 3).astype(np.int32)
+        x = (rng.random((M, E)) < 0.35).astype(np.uint8)
+        for e in range(E):
+            if not x[:, e].any():
+                x[rng.integers(M), e] = 1
+        sp = synth.server_params(M, 4096, 14336, seed=l)
+        if cheap_links:
+            sp.tau[:] *= 1e-3
+        theta = 0.2
+        build_tables(sim, group, x, theta, qbar, sp, DEV, out=buf[l * stride:(l + 1) * stride])
+        otabs.append(oracle.tables(sim, group, x, theta, qbar, sp.F, sp.B, sp.tau, sp.z, sp.c,
+                                   sp.omega_T, sp.omega_Q))
+    return buf, stride, otabs
+
+
+@pytest.mark.parametrize("E,M,k,H,cheap", [(8, 4, 2, 1, True), (8, 4, 2, 2, True), (8, 4, 2, 3, True),
+                                           (16, 4, 3, 3, False), (6, 3, 2, 4, True), (32, 8, 2, 2, True)])
+def test_route_select_lookahead_given_logits_bit_exact(E, M, k, H, cheap):
+    rng = np.random.default_rng(E * 10 + H)
+    T = 300
+    qbar = 0.2
+    buf, stride, otabs = stack_tables(rng, H, E, M, qbar, cheap)
+    P = rng.random((max(H - 1, 1), E, E)).astype(np.float32)
+    P[P < 0.5] = 0
+    P = (P / np.maximum(P.sum(axis=2, keepdims=True), 1e-9)).astype(np.float32)
+    logits = rng.standard_normal((T, E)).astype(np.float32)
+    home = rng.integers(0, M, T).astype(np.uint8)
+    loc = np.where(rng.random(T) < 0.5, home, rng.integers(0, M, T)).astype(np.uint8)
+    qhat = (rng.random(T) * 0.1).astype(np.float32)
+    g = [torch.empty(T, k, dtype=dt, device=DEV)
+         for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
+    gl = torch.as_tensor(loc).to(DEV); gq = torch.as_tensor(qhat).to(DEV)
+    B.ordermoe_route_select_lookahead(None, None, torch.as_tensor(logits).to(DEV), T, E, 0, k, 1, buf,
+                                      stride, H, torch.as_tensor(P).to(DEV) if H > 1 else None,
+                                      torch.as_tensor(home).to(DEV), gl, gq, None, *g)
+    idx, _ = oracle.topk(logits, k)
+    ref = oracle.select_lookahead(idx, otabs[:H], P[:H - 1], home, loc, qhat)
+    for name, got, want in zip(("chosen", "server", "kind"), (g[2], g[3], g[4]), ref[:3]):
+        np.testing.assert_array_equal(got.cpu().numpy(), want, err_msg=name)
+    np.testing.assert_array_equal(gl.cpu().numpy(), ref[3])
+    np.testing.assert_array_equal(gq.cpu().numpy(), ref[4])
+    if H > 1:
+        myo = oracle.select(idx, otabs[0], home, loc, qhat)
+        print("decisions changed by the look-ahead:", int((myo[0] != ref[0]).sum() + (myo[1] != ref[1]).sum()))
+
+
+def test_lookahead_horizon_one_equals_route_select():
+    rng = np.random.default_rng(5)
+    E, M, k, T = 8, 4, 2, 200
+    buf, stride, otabs = stack_tables(rng, 1, E, M, 0.2, True)
+    logits = torch.as_tensor(rng.standard_normal((T, E)).astype(np.float32)).to(DEV)
+    home = torch.as_tensor(rng.integers(0, M, T).astype(np.uint8)).to(DEV)
+    outs = []
+    for fn in ("plain", "lookahead"):
+        g = [torch.empty(T, k, dtype=dt, device=DEV)
+             for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
+        if fn == "plain":
+            B.ordermoe_route_select(None, None, logits, T, E, 0, k, 1, buf, home, None, None, None, *g)
+        else:
+            B.ordermoe_route_select_lookahead(None, None, logits, T, E, 0, k, 1, buf, stride, 1, None,
+                                              home, None, None, None, *g)
+        outs.append([t.cpu() for t in g])
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
+
+
+def test_decode_stack_with_lookahead_h3_follows_the_oracle():
+    """32 Mixtral-shaped routers, batch 128, H = 3: each layer looks two layers
+    ahead with the transition statistics of the calibration logits. The
+    oracle follows every token through the 32 selections (fed the same fp32
+    logits, so each decision is compared exactly)."""
+    w = synth.workload("decode_stack")
+    L, T, E, k, M = w.L, w.T, w.E, w.k, w.M
+    H = 3
+    rng = np.random.default_rng(21)
+    buf, stride, otabs = stack_tables(rng, L, E, M, w.qbar, cheap_links=True)
+    cal = rng.standard_normal((4096, L, E)).astype(np.float32)
+    _, P = oracle.transitions(cal, k)
+    gP = torch.as_tensor(P).to(DEV)
+    logits = rng.standard_normal((L, T, E)).astype(np.float32)
+    home = rng.integers(0, M, T).astype(np.uint8)
+    gl = torch.as_tensor(home).to(DEV); gq = torch.zeros(T, device=DEV)
+    gh = torch.as_tensor(home).to(DEV)
+    gch = []
+    for l in range(L):
+        Hl = min(H, L - l)
+        g = [torch.empty(T, k, dtype=dt, device=DEV)
+             for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
+        B.ordermoe_route_select_lookahead(None, None, torch.as_tensor(logits[l]).to(DEV), T, E, 0, k, 1,
+                                          buf[l * stride:], stride, Hl,
+                                          gP[l:l + Hl - 1].contiguous() if Hl > 1 else None,
+                                          gh, gl, gq, None, *g)
+        gch.append(g[2].cpu().numpy())
+    loc = home.copy(); q = np.zeros(T, np.float32)
+    for l in range(L):
+        Hl = min(H, L - l)
+        idx, _ = oracle.topk(logits[l], k)
+        ch, sv, kd, loc, q = oracle.select_lookahead(idx, otabs[l:l + Hl], P[l:l + Hl - 1], home, loc, q)
+        np.testing.assert_array_equal(gch[l], ch, err_msg="layer %d" % l)
+    np.testing.assert_array_equal(gl.cpu().numpy(), loc)
+    np.testing.assert_array_equal(gq.cpu().numpy(), q)
+    assert (q <= np.float32(w.qbar)).all()

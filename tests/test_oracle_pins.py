@@ -666,3 +666,152 @@ def test_place_disperses_same_group_experts_even_when_load_alone_would_not(orc):
     x, used, rc = orc.place(group, I, np.ones((1, 4)), np.array([4.0, 4.0]))
     assert rc == 0
     np.testing.assert_array_equal(x[0], [[1, 0, 0, 1], [0, 1, 1, 0]])
+
+
+# --------------------------------------------------------------------------
+# Look-ahead selection (Eqs. 41-43)
+
+def test_transitions_brute_force(orc):
+    rng = np.random.default_rng(30)
+    N, L, E, kf = 40, 4, 6, 2
+    logits = rng.standard_normal((N, L, E)).astype(np.float32)
+    logits[0, 1, :] = 0.5                       # ties
+    cnt, P = orc.transitions(logits, kf)
+    ref = np.zeros((L - 1, E, E), np.int64)
+    for n in range(N):
+        for l in range(L - 1):
+            for a in brute_topk(list(logits[n, l]), kf):
+                for b in brute_topk(list(logits[n, l + 1]), kf):
+                    ref[l, a, b] += 1
+    np.testing.assert_array_equal(cnt, ref)
+    rows = ref.sum(axis=2, keepdims=True)
+    np.testing.assert_allclose(P, np.where(rows > 0, ref / np.maximum(rows, 1), 0), rtol=1e-7)
+    assert cnt.sum() == (L - 1) * N * kf * kf
+
+
+def _rand_tables(orc, rng, E, M, kgroups, tau_scale=1.0):
+    Wt = rng.standard_normal((E, 5)); Wt[:, 0] += 3.0 * (np.arange(E) % kgroups)
+    sim = (1 - cdist(Wt, Wt, "cosine")).astype(np.float32); np.fill_diagonal(sim, 1.0)
+    group = (np.arange(E) % kgroups).astype(np.int32)
+    x = (rng.random((M, E)) < 0.4).astype(np.uint8)
+    for e in range(E):
+        if not x[:, e].any():
+            x[rng.integers(M), e] = 1
+    F, B, tau = _params(rng, M)
+    return orc.tables(sim, group, x, float(rng.choice([0.0, 0.4])), float(rng.choice([0.1, 0.3])),
+                      F, B, tau * tau_scale, 2048.0, 1e9, 0.5, 0.5), sim
+
+
+def test_lookahead_horizon_one_is_the_myopic_selection(orc):
+    rng = np.random.default_rng(31)
+    for _ in range(40):
+        E, M, k, T = int(rng.integers(2, 7)), int(rng.integers(1, 4)), 1, 12
+        k = int(rng.integers(1, min(E, 3) + 1))
+        tab, _ = _rand_tables(orc, rng, E, M, 2, tau_scale=float(rng.choice([1e-4, 1.0])))
+        idx = np.array([rng.permutation(E)[:k] for _ in range(T)], np.int32)
+        home = rng.integers(0, M, T).astype(np.uint8)
+        loc = rng.integers(0, M, T).astype(np.uint8)
+        qhat = (rng.random(T) * 0.05).astype(np.float32)
+        a = orc.select(idx, tab, home, loc, qhat)
+        b = orc.select_lookahead(idx, [tab], None, home, loc, qhat)
+        for u, v in zip(a, b):
+            np.testing.assert_array_equal(u, v)
+
+
+def brute_lookahead_h2(idx, t0, t1, P1, home, loc, qhat):
+    """Eq. 43 with H = 2, Eq. 42 enumerated over every (target k', server m',
+    executed expert k'') triple of the next layer; fp32 as the paper's
+    reading fixes it (each product and sum rounded once)."""
+    f32 = np.float32
+    T, k = idx.shape
+    E, M = t0.E, t0.M
+    out = [np.zeros((T, k), np.int32), np.zeros((T, k), np.uint8), np.zeros((T, k), np.uint8)]
+    loc2 = loc.copy(); q2 = qhat.copy()
+
+    def feasible(t, target, qacc, taken):
+        for m in range(M):
+            for kk in range(E):
+                if not (int(t.pmask[kk]) >> m) & 1:
+                    continue
+                if kk != target:
+                    if not (int(t.subst[target]) >> kk) & 1 or kk in taken:
+                        continue
+                    if not f32(qacc + t.Qtab[target, kk]) <= t.qbar:
+                        continue
+                yield m, kk
+
+    for ti in range(T):
+        a, s, q = int(home[ti]), int(loc[ti]), f32(qhat[ti])
+        taken = set(int(v) for v in idx[ti])
+        for j in range(k):
+            r = int(idx[ti, j])
+            cands = []
+            for m, kk in feasible(t0, r, q, taken):
+                g = f32(t0.A[a, s, m] + (f32(0) if kk == r else t0.Cq[r, kk]))
+                qn = q if kk == r else f32(q + t0.Qtab[r, kk])
+                phi = f32(0)
+                for kt in range(E):
+                    p = P1[kk, kt]
+                    if p == 0:
+                        continue
+                    best = min(f32(t1.A[a, m, m2] + (f32(0) if k2 == kt else t1.Cq[kt, k2]))
+                               for m2, k2 in feasible(t1, kt, qn, set()))
+                    phi = f32(phi + f32(p * best))
+                cands.append((f32(g + phi), kk != r, m != s, m, kk))
+            _, sub, away, m, kk = min(cands)
+            out[0][ti, j] = kk; out[1][ti, j] = m; out[2][ti, j] = 2 * away + sub
+            if sub:
+                taken.add(kk); q = f32(q + t0.Qtab[r, kk])
+            if j == 0:
+                loc2[ti] = m
+        q2[ti] = q
+    return out[0], out[1], out[2], loc2, q2
+
+
+def test_lookahead_h2_matches_brute_force(orc):
+    rng = np.random.default_rng(32)
+    changed = 0
+    for trial in range(60):
+        E, M = int(rng.integers(2, 6)), int(rng.integers(1, 4))
+        k = int(rng.integers(1, min(E, 2) + 1)); T = 8
+        scale = float(rng.choice([1e-4, 1e-2, 1.0]))
+        t0, _ = _rand_tables(orc, rng, E, M, 2, tau_scale=scale)
+        t1, _ = _rand_tables(orc, rng, E, M, 2, tau_scale=scale)
+        t1.qbar = t0.qbar
+        P1 = rng.random((E, E)).astype(np.float32)
+        P1[P1 < 0.3] = 0
+        P1 = (P1 / np.maximum(P1.sum(axis=1, keepdims=True), 1e-9)).astype(np.float32)
+        idx = np.array([rng.permutation(E)[:k] for _ in range(T)], np.int32)
+        home = rng.integers(0, M, T).astype(np.uint8)
+        loc = rng.integers(0, M, T).astype(np.uint8)
+        qhat = (rng.random(T) * 0.05).astype(np.float32)
+        got = orc.select_lookahead(idx, [t0, t1], P1[None], home, loc, qhat)
+        ref = brute_lookahead_h2(idx, t0, t1, P1, home, loc, qhat)
+        for u, v in zip(got, ref):
+            np.testing.assert_array_equal(u, v)
+        myo = orc.select(idx, t0, home, loc, qhat)
+        changed += int((myo[0] != got[0]).sum() + (myo[1] != got[1]).sum())
+    assert changed > 0   # the look-ahead did change some decisions
+
+
+def test_lookahead_moves_the_token_where_the_next_layer_is_cheap(orc):
+    """Hand case (Eqs. 37-43): the target r is only on server 1; its substitute
+    s2 is local on server 0. Myopically the local substitute is cheaper
+    (1 + 0.5 < 5), but every next-layer target lives on server 1 only, so with
+    H = 2 moving now costs 5 + 1 < 1.5 + 5 and the token goes to server 1."""
+    E, M = 3, 2
+    A = np.array([[[1, 5], [5, 1]], [[1, 5], [5, 1]]], np.float32)
+    Q = np.array([[0, .2, .2], [.2, 0, .2], [.2, .2, 0]], np.float32)
+    Cq = np.where(Q > 0, 0.5, 0).astype(np.float32)
+    t0 = orc.Tables(Q, Cq, np.array([0b010, 0b001, 0], np.uint64), A,
+                    np.array([0b10, 0b01, 0b10], np.uint32), 1.0, E, M)
+    t1 = orc.Tables(Q, Cq, np.zeros(E, np.uint64), A, np.array([0b10, 0b10, 0b10], np.uint32), 1.0,
+                    E, M)
+    P = np.zeros((1, E, E), np.float32); P[0, :, 2] = 1.0
+    idx = np.array([[0]], np.int32)
+    home = np.array([0], np.uint8)
+    myo = orc.select(idx, t0, home, home.copy(), np.zeros(1, np.float32))
+    assert myo[0][0, 0] == 1 and myo[1][0, 0] == 0          # local substitute
+    la = orc.select_lookahead(idx, [t0, t1], P, home, home.copy(), np.zeros(1, np.float32))
+    assert la[0][0, 0] == 0 and la[1][0, 0] == 1            # remote exact
+    assert la[3][0] == 1                                     # the token moved (Eq. 44)
