@@ -62,6 +62,8 @@ def parse():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--lookahead", type=int, default=1,
+                   help="selection horizon H (Eqs. 41-43) for the decode stack; 1 = myopic")
     p.add_argument("--cpu-seconds", type=float, default=15.0,
                    help="target CPU seconds of the oracle baseline sample")
     return p.parse_args()
@@ -423,16 +425,22 @@ def run_decode(args, dist, w, device):
                      torch.ones(L, E, dtype=torch.float64, device=device),
                      torch.full((M,), L * E / M, dtype=torch.float64, device=device),
                      group, ng, theta, x, used, st)
+    # transition statistics (Eq. 41) from the calibration logits the similarity
+    # call leaves at the start of its workspace
+    H = max(1, args.lookahead)
+    P = torch.empty(L - 1, E, E, dtype=torch.float32, device=device)
+    tcount = torch.empty(L - 1, E, E, dtype=torch.int32, device=device)
+    B.ordermoe_transitions(ws.view(torch.float32)[: w.n_cal * L * E], w.n_cal, L, E, w.k, tcount, P)
     sp = synth.server_params(M, w.d, w.dff, seed)
     f64 = lambda a: torch.as_tensor(a, dtype=torch.float64).to(device)
     th = theta.cpu().tolist()
-    tabs = []
+    stride = B.ordermoe_tables_bytes(E, M)
+    tabs = torch.zeros(L * stride, dtype=torch.uint8, device=device)
     for l in range(L):
-        t = torch.zeros(B.ordermoe_tables_bytes(E, M), dtype=torch.uint8, device=device)
         B.ordermoe_build_tables(sim[l], group[l], x[l], th[l], w.qbar, f64(sp.F), f64(sp.B),
-                                f64(sp.tau), sp.z, sp.c, sp.omega_T, sp.omega_Q, t)
-        tabs.append(t)
-    stack = LayerStack(layers, tabs, w.k, w.T, device)
+                                f64(sp.tau), sp.z, sp.c, sp.omega_T, sp.omega_Q,
+                                tabs[l * stride:(l + 1) * stride])
+    stack = LayerStack(layers, tabs, w.k, w.T, device, H=H, stride=stride, P=P)
     Xs = [synth.hidden(w.T, w.d, seed + 5000 + l, device=device) for l in range(w.L)]
     ys = [torch.empty(w.T, w.d, dtype=torch.bfloat16, device=device) for _ in range(w.L)]
     loc = home.clone()
@@ -447,6 +455,23 @@ def run_decode(args, dist, w, device):
     code, detail = B.ordermoe_device_error()
     if code:
         raise RuntimeError("device error %d (%d)" % (code, detail))
+    # decision time: the selection alone (router + top-k + Alg. 2) over the 32 layers
+    f = lambda *sh, dt: torch.empty(*sh, dtype=dt, device=device)
+    sel = [f(w.T, w.k, dt=dt) for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    stream = torch.cuda.current_stream(device)
+    ev[0].record(stream)
+    for _ in range(5):
+        loc.copy_(home); qhat.zero_()
+        for l in range(L):
+            Hl = min(H, L - l)
+            B.ordermoe_route_select_lookahead(Xs[l], layers[l]["W_r"], None, w.T, E, w.d, w.k, 1,
+                                              tabs[l * stride:], stride, Hl,
+                                              P[l:l + Hl - 1].contiguous() if Hl > 1 else None,
+                                              home, loc, qhat, None, *sel)
+    ev[1].record(stream)
+    torch.cuda.synchronize(device)
+    select_ms_per_layer = ev[0].elapsed_time(ev[1]) / (5 * L)
     step_s = ms / args.steps / 1e3
     wbytes = 3.0 * w.E * w.d * w.dff * 2 * w.L
     pk, pk_kind = peaks()
@@ -458,14 +483,17 @@ def run_decode(args, dist, w, device):
         "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": w.L, "T": w.T, "d": w.d, "E": w.E, "k": w.k,
-                   "d_ff": w.dff, "M": w.M, "l2": "inputs larger than L2: %.1f GB of expert weights"
-                   % (wbytes / 1e9)},
+                   "d_ff": w.dff, "M": w.M, "lookahead_H": H,
+                   "l2": "inputs larger than L2: %.1f GB of expert weights" % (wbytes / 1e9)},
         "roofline": {"kernel": "whole decode step (expert weight streaming)", "bound": "hbm",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
                      "peak_source": "%s hbm_gbs" % pk_kind, "bytes_per_step": wbytes},
         "gpu_launches": 8 * w.L * args.steps,
         "clocks": clocks,
+        "lookahead_H": H,
+        "selection_ms_per_layer": round(select_ms_per_layer, 4),
+        "selection_us_per_token_layer": round(select_ms_per_layer * 1e3 / w.T, 4),
     }
 
 

@@ -257,6 +257,12 @@ typedef struct {
   size_t tables_bytes;
   void* scratch;
   size_t scratch_bytes;
+  /* look-ahead (Eqs. 41-43); lookahead_H <= 1 selects myopically. With H > 1
+   * `tables` must be followed by the next H - 1 layers' tables at
+   * tables_stride bytes, and P holds [H-1][E][E] transition matrices. */
+  int lookahead_H;
+  size_t tables_stride;
+  const float* P;
 } ordermoe_layer_desc;
 
 size_t ordermoe_layer_scratch_bytes(int T_max, int E, int d, int dff, int k);

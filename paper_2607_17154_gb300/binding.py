@@ -60,7 +60,8 @@ class LayerDesc(ctypes.Structure):
     """Mirror of ordermoe_layer_desc."""
     _fields_ = [("T_max", _I), ("E", _I), ("d", _I), ("dff", _I), ("k", _I), ("renorm", _I),
                 ("W_r", _P), ("W1", _P), ("W3", _P), ("W2", _P), ("tables", _P),
-                ("tables_bytes", _SZ), ("scratch", _P), ("scratch_bytes", _SZ)]
+                ("tables_bytes", _SZ), ("scratch", _P), ("scratch_bytes", _SZ),
+                ("lookahead_H", _I), ("tables_stride", _SZ), ("P", _P)]
 
 
 class OrderMoEError(RuntimeError):
@@ -268,14 +269,19 @@ def ordermoe_layer_scratch_bytes(T_max, E, d, dff, k):
     return int(lib().ordermoe_layer_scratch_bytes(T_max, E, d, dff, k))
 
 
-def make_layer_desc(T_max, W_r, W1, W3, W2, tables, k, scratch, renorm=1):
+def make_layer_desc(T_max, W_r, W1, W3, W2, tables, k, scratch, renorm=1, lookahead_H=1,
+                    tables_stride=0, P=None):
+    """tables: this layer's tables (uint8 device tensor); with lookahead_H > 1 it
+    must continue with the next layers' tables at tables_stride bytes."""
     E, dff, d = W1.shape
     for n, t in (("W_r", W_r), ("W1", W1), ("W3", W3), ("W2", W2)):
         _dt(t, torch.bfloat16, n)
+    _dt(P, torch.float32, "P")
     desc = LayerDesc(T_max, E, d, dff, k, int(renorm), _ptr(W_r), _ptr(W1), _ptr(W3), _ptr(W2),
                      _ptr(tables), tables.numel(), _ptr(scratch),
-                     scratch.numel() * scratch.element_size())
-    desc._keep = (W_r, W1, W3, W2, tables, scratch)
+                     scratch.numel() * scratch.element_size(), int(lookahead_H), int(tables_stride),
+                     _ptr(P))
+    desc._keep = (W_r, W1, W3, W2, tables, scratch, P)
     return desc
 
 

@@ -67,6 +67,12 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
                                      float* topk_w, int32_t* chosen_expert,
                                      uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
                                      ordermoe_stream_t stream);
+extern "C" int ordermoe_route_select_lookahead(
+    const uint16_t* X, const uint16_t* W_r, const float* logits_in, int T, int E, int d, int k,
+    int renorm, const void* tables, size_t tables_stride, int H, const float* P,
+    const uint8_t* home, uint8_t* loc, float* qhat, float* logits_out, int32_t* topk_idx,
+    float* topk_w, int32_t* chosen_expert, uint8_t* chosen_server, uint8_t* kind,
+    int32_t* counters, ordermoe_stream_t stream);
 extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,
                                 const float* topk_w, int T, int k, int d, uint16_t* y,
                                 ordermoe_stream_t stream);
@@ -121,9 +127,16 @@ extern "C" int ordermoe_layer_forward(const ordermoe_layer_desc* L, int T, const
       qd = s.qhat;
     }
   }
-  int rc = ordermoe_route_select(Xd, L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
-                                 L->tables_bytes, homed, locd, qd, nullptr, s.topk_idx, s.topk_w,
-                                 s.chosen, s.server, s.kind, counters, stream);
+  int rc;
+  if (L->lookahead_H > 1)
+    rc = ordermoe_route_select_lookahead(Xd, L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
+                                         L->tables_stride, L->lookahead_H, L->P, homed, locd, qd,
+                                         nullptr, s.topk_idx, s.topk_w, s.chosen, s.server, s.kind,
+                                         counters, stream);
+  else
+    rc = ordermoe_route_select(Xd, L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
+                               L->tables_bytes, homed, locd, qd, nullptr, s.topk_idx, s.topk_w,
+                               s.chosen, s.server, s.kind, counters, stream);
   if (rc) return rc;
   rc = dispatch_launch(s.chosen, Xd, T, k, E, d, s.offsets, s.row_token, s.row_of, s.X_perm,
                        s.hist, st);

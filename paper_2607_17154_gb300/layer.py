@@ -67,13 +67,26 @@ class LayerStack:
     """L MoE layers run through ordermoe_layer_forward with the token state
     (location, accumulated loss; Eqs. 36 and 44) carried from layer to layer."""
 
-    def __init__(self, layers, tables, k, T_max, device):
-        # layers: list of dicts with W_r, W1, W3, W2 (device bf16); tables: list of device buffers
+    def __init__(self, layers, tables, k, T_max, device, H=1, stride=0, P=None):
+        """layers: dicts with W_r, W1, W3, W2 (device bf16). tables: a list of
+        per-layer device buffers, or (for look-ahead, H > 1) one device buffer
+        holding all layers' tables `stride` bytes apart; P [L-1, E, E] the
+        transition matrices. Layer l looks min(H, L - l) - 1 layers ahead."""
         E, dff, d = layers[0]["W1"].shape
+        L = len(layers)
         self.scratch = torch.empty(B.ordermoe_layer_scratch_bytes(T_max, E, d, dff, k),
                                    dtype=torch.uint8, device=device)
-        self.descs = [B.make_layer_desc(T_max, l["W_r"], l["W1"], l["W3"], l["W2"], t, k,
-                                        self.scratch) for l, t in zip(layers, tables)]
+        self.descs = []
+        for l, lay in enumerate(layers):
+            if isinstance(tables, torch.Tensor):
+                t = tables[l * stride:]
+                Hl = min(H, L - l)
+                Pl = P[l:l + Hl - 1].contiguous() if Hl > 1 else None
+            else:
+                t, Hl, Pl = tables[l], 1, None
+            self.descs.append(B.make_layer_desc(T_max, lay["W_r"], lay["W1"], lay["W3"], lay["W2"],
+                                                t, k, self.scratch, lookahead_H=Hl,
+                                                tables_stride=stride, P=Pl))
         self.d, self.T_max = d, T_max
 
     def step(self, X_layers, home, loc, qhat, y_layers, counters=None, stream=None):
