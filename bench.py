@@ -489,7 +489,9 @@ def run_decode(args, dist, w, device):
                      "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
                      "peak_source": "%s hbm_gbs" % pk_kind, "bytes_per_step": wbytes},
-        "gpu_launches": 8 * w.L * args.steps,
+        # 8 kernels a layer, plus the look-ahead selection pass on every layer
+        # that looks ahead (all but the last when H > 1)
+        "gpu_launches": (8 * w.L + sum(min(H, w.L - l) > 1 for l in range(w.L))) * args.steps,
         "clocks": clocks,
         "lookahead_H": H,
         "selection_ms_per_layer": round(select_ms_per_layer, 4),

@@ -203,11 +203,16 @@ __device__ __forceinline__ void select_token(
     const SelSmem& sm, const float* s_Q, const float* s_Cq,
     const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
     int32_t* __restrict__ topk_idx, float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
-    uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out, int (&kind_count)[4]) {
+    uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out, int (&kind_count)[4],
+    bool topk_only = false) {
 #pragma unroll
   for (int e = 0; e < EMAX; ++e)
     if (e < E && isnan(lg[e])) {
       report(&g_err_route, ORDERMOE_DEV_NAN_LOGIT, t);
+      for (int j = 0; j < k; ++j) {  // no targets: a later pass skips this token
+        topk_idx[(size_t)t * k + j] = -1;
+        topk_w[(size_t)t * k + j] = 0.0f;
+      }
       return;
     }
   // top-k by (logit desc, index asc)
@@ -248,6 +253,7 @@ __device__ __forceinline__ void select_token(
     topk_idx[(size_t)t * k + j] = idx[j];
     topk_w[(size_t)t * k + j] = renorm ? wsel[j] / ssel : wsel[j];
   }
+  if (topk_only) return;
   // selection
   const int a = home[t];
   const int s = (loc != nullptr) ? loc[t] : a;  // no state given: first layer (Eq. 36)
@@ -348,7 +354,175 @@ __global__ void __launch_bounds__(128) select_kernel(
     if (logits_out != nullptr)
       for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
     select_token<EMAX>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
-                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count);
+                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count,
+                       la.H > 1);
+  }
+  flush_kind_counts(sm, kind_count, counters);
+  __syncthreads();
+  if (counters != nullptr && threadIdx.x < 4 && sm.kind[threadIdx.x])
+    atomicAdd(&counters[threadIdx.x], sm.kind[threadIdx.x]);
+}
+
+// ---------------------------------------------------------------------------
+// Alg. 2 with horizon H > 1 (Eq. 43), one warp per token, from the targets
+// topk_idx. The candidates of a slot are visited in order by the whole warp;
+// for each, lane i computes the term P(k -> k') * min(...) of Eq. 42 for the
+// next targets k' = i and i + 32 (with the deeper levels of the recursion
+// serial in the lane); the terms are then added in ascending k' by every lane
+// (shuffles), so Phi is the same fp32 value the serial definition gives.
+template <int D>
+__device__ __forceinline__ float phi_term(const uint8_t* __restrict__ tnext, size_t stride,
+                                          const float* __restrict__ P, int E, int M, int a, int m,
+                                          int kx, int kt, float qacc, float qbar) {
+  // the k' = kt term of lookahead_phi<D> (0 when P = 0)
+  const float p = __ldg(P + (size_t)kx * E + kt);
+  if (p == 0.0f) return 0.0f;
+  const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
+  const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
+  const float* A1 = reinterpret_cast<const float*>(tnext + off_a(E));
+  const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
+  const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
+  float best = INFINITY;
+  unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);
+  while (cand) {
+    const int kk = __ffsll(static_cast<long long>(cand)) - 1;
+    cand &= cand - 1;
+    const bool exact = (kk == kt);
+    float cq = 0.0f, q2 = qacc;
+    if (!exact) {
+      const float qk = __ldg(Q1 + kt * E + kk);
+      if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
+      q2 = __fadd_rn(qacc, qk);
+      cq = __ldg(C1 + kt * E + kk);
+    }
+    uint32_t pm = __ldg(pm1 + kk);
+    while (pm) {
+      const int m2 = __ffs(pm) - 1;
+      pm &= pm - 1;
+      float c = __fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq);
+      if (D > 1)
+        c = __fadd_rn(c, lookahead_phi<(D > 1 ? D - 1 : 1)>(tnext + stride, stride, P + E * E, E,
+                                                            M, a, m2, kk, q2, qbar));
+      best = fminf(best, c);
+    }
+  }
+  return __fmul_rn(p, best);
+}
+
+template <int D>
+__device__ __forceinline__ float phi_warp(const uint8_t* tnext, size_t stride, const float* P,
+                                          int E, int M, int a, int m, int kx, float qacc,
+                                          float qbar, int lane) {
+  const float t0 = lane < E ? phi_term<D>(tnext, stride, P, E, M, a, m, kx, lane, qacc, qbar) : 0.0f;
+  const float t1 = lane + 32 < E ? phi_term<D>(tnext, stride, P, E, M, a, m, kx, lane + 32, qacc, qbar) : 0.0f;
+  float acc = 0.0f;
+  for (int kt = 0; kt < E; ++kt) {
+    const float term = __shfl_sync(0xffffffffu, kt < 32 ? t0 : t1, kt & 31);
+    if (__ldg(P + (size_t)kx * E + kt) != 0.0f) acc = __fadd_rn(acc, term);
+  }
+  return acc;
+}
+
+__device__ __forceinline__ float phi_warp_h(const Lookahead& la, const uint8_t* tab, int E, int M,
+                                            int a, int m, int kx, float qacc, float qbar, int lane) {
+  switch (la.H) {
+    case 2: return phi_warp<1>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar, lane);
+    case 3: return phi_warp<2>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar, lane);
+    case 4: return phi_warp<3>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar, lane);
+    default: return 0.0f;
+  }
+}
+
+__global__ void __launch_bounds__(128) lookahead_select_kernel(
+    const int32_t* __restrict__ topk_idx, int T, int E, int k, const uint8_t* __restrict__ tab,
+    Lookahead la, const uint8_t* __restrict__ home, uint8_t* __restrict__ loc,
+    float* __restrict__ qhat, int32_t* __restrict__ chosen_expert,
+    uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
+    int32_t* __restrict__ counters) {
+  __shared__ SelSmem sm;
+  extern __shared__ __align__(16) float s_dyn[];
+  float* s_Q = s_dyn;
+  float* s_Cq = s_dyn + E * E;
+  if (!load_tables(tab, E, sm, s_Q, s_Cq)) return;
+  __syncthreads();
+  const int M = reinterpret_cast<const int32_t*>(tab)[2];
+  const float qbar = reinterpret_cast<const float*>(tab)[5];
+  const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
+  const int lane = threadIdx.x & 31;
+  const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  int kind_count[4] = {0, 0, 0, 0};
+  if (t < T) {
+    const int a = home[t];
+    const int s = (loc != nullptr) ? loc[t] : a;
+    if (a >= M || s >= M) {
+      if (lane == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
+    } else {
+      const float* Aas = gA + ((size_t)a * M + s) * M;
+      float q = (qhat != nullptr) ? qhat[t] : 0.0f;
+      unsigned long long taken = 0;
+      bool ok = true;
+      for (int j = 0; j < k; ++j) {
+        const int r = topk_idx[(size_t)t * k + j];
+        ok = ok && r >= 0 && r < E;  // -1: a token whose logits held a NaN
+        if (ok) taken |= 1ull << r;
+      }
+      int first_server = s;
+      for (int j = 0; j < (ok ? k : 0); ++j) {
+        const int r = topk_idx[(size_t)t * k + j];
+        const int nsub = sm.nsub[r];
+        unsigned long long best = ~0ull;
+        for (int ki = 0; ki <= nsub; ++ki) {
+          const int kk = (ki == 0) ? r : sm.sublist[r * 64 + ki - 1];
+          const bool sub = (ki != 0);
+          float cq = 0.0f, qn = q;
+          if (sub) {
+            if ((taken >> kk) & 1ull) continue;
+            if (!(__fadd_rn(q, s_Q[r * E + kk]) <= qbar)) continue;
+            cq = s_Cq[r * E + kk];
+            qn = __fadd_rn(q, s_Q[r * E + kk]);
+          }
+          uint32_t pm = sm.pmask[kk];
+          while (pm) {
+            const int m = __ffs(pm) - 1;
+            pm &= pm - 1;
+            float cost = __fadd_rn(__ldg(Aas + m), cq);
+            cost = __fadd_rn(cost, phi_warp_h(la, tab, E, M, a, m, kk, qn, qbar, lane));
+            const unsigned long long key =
+                (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
+                (static_cast<unsigned long long>(sub ? 1u : 0u) << 31) |
+                (static_cast<unsigned long long>(m != s ? 1u : 0u) << 30) |
+                (static_cast<unsigned long long>(m) << 8) | static_cast<unsigned long long>(kk);
+            best = key < best ? key : best;
+          }
+        }
+        int kstar, mstar, kd;
+        if (best == ~0ull) {
+          if (lane == 0) report(&g_err_route, ORDERMOE_DEV_NO_CANDIDATE, t);
+          kstar = r; mstar = s; kd = 0;
+        } else {
+          kstar = static_cast<int>(best & 0xFFu);
+          mstar = static_cast<int>((best >> 8) & 0xFFu);
+          const int sub = static_cast<int>((best >> 31) & 1u);
+          const int away = static_cast<int>((best >> 30) & 1u);
+          kd = 2 * away + sub;
+          if (sub) {
+            taken |= 1ull << kstar;
+            q = __fadd_rn(q, s_Q[r * E + kstar]);
+          }
+        }
+        if (j == 0) first_server = mstar;
+        if (lane == 0) {
+          chosen_expert[(size_t)t * k + j] = kstar;
+          chosen_server[(size_t)t * k + j] = static_cast<uint8_t>(mstar);
+          kind_out[(size_t)t * k + j] = static_cast<uint8_t>(kd);
+          kind_count[kd]++;
+        }
+      }
+      if (lane == 0 && ok && loc != nullptr) {
+        loc[t] = static_cast<uint8_t>(first_server);
+        qhat[t] = q;
+      }
+    }
   }
   flush_kind_counts(sm, kind_count, counters);
   __syncthreads();
@@ -552,7 +726,8 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       const float qbar = reinterpret_cast<const float*>(tab)[5];
       const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
       select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
-                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count);
+                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count,
+                       la.H > 1);
     }
     flush_kind_counts(sm, kind_count, counters);
   }
@@ -609,6 +784,20 @@ extern "C" int ordermoe_build_tables(const float* sim, const int32_t* group,
   return ORDERMOE_OK;
 }
 
+static int launch_lookahead_select(const int32_t* topk_idx, int T, int E, int k,
+                                   const uint8_t* tb, Lookahead la, const uint8_t* home,
+                                   uint8_t* loc, float* qhat, int32_t* chosen_expert,
+                                   uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
+                                   size_t tab_smem, cudaStream_t stream) {
+  const int blocks = (T + 3) / 4;  // 4 warps = 4 tokens per block
+  cudaFuncSetAttribute(lookahead_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)tab_smem);
+  lookahead_select_kernel<<<blocks, 128, tab_smem, stream>>>(
+      topk_idx, T, E, k, tb, la, home, loc, qhat, chosen_expert, chosen_server, kind, counters);
+  OM_LAUNCHED("lookahead_select_kernel");
+  return ORDERMOE_OK;
+}
+
 static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float* logits_in, int T,
                              int E, int d, int k, int renorm, const void* tables,
                              size_t tables_bytes_, Lookahead la, const uint8_t* home, uint8_t* loc,
@@ -651,7 +840,10 @@ static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float
     else OM_SEL_LAUNCH(64);
 #undef OM_SEL_LAUNCH
     OM_LAUNCHED("select_kernel");
-    return ORDERMOE_OK;
+    return la.H > 1 ? launch_lookahead_select(topk_idx, T, E, k, tb, la, home, loc, qhat,
+                                              chosen_expert, chosen_server, kind, counters,
+                                              tab_smem, stream)
+                    : ORDERMOE_OK;
   }
   CUtensorMap mX, mW;
   int rc;
@@ -692,6 +884,9 @@ static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float
 #undef OM_RT_LAUNCH
   if (le != cudaSuccess) return cuda_fail(le, "router_select_kernel launch");
   OM_LAUNCHED("router_select_kernel");
+  if (la.H > 1)
+    return launch_lookahead_select(topk_idx, T, E, k, tb, la, home, loc, qhat, chosen_expert,
+                                   chosen_server, kind, counters, tab_smem, stream);
   return ORDERMOE_OK;
 }
 

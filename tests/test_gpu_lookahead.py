@@ -149,3 +149,66 @@ def test_decode_stack_with_lookahead_h3_follows_the_oracle():
     np.testing.assert_array_equal(gl.cpu().numpy(), loc)
     np.testing.assert_array_equal(gq.cpu().numpy(), q)
     assert (q <= np.float32(w.qbar)).all()
+
+
+@pytest.mark.parametrize("E,M,k,H", [(8, 4, 2, 3), (16, 6, 4, 2), (64, 8, 6, 2)])
+def test_router_path_lookahead_bit_exact(E, M, k, H):
+    """Router GEMM on the tensor cores, then the warp-per-token look-ahead
+    pass: the decisions follow the oracle given the logits the router wrote
+    (T spans three 128-row router tiles with a ragged tail)."""
+    rng = np.random.default_rng(E + 100 * H)
+    T, d = 300, 256
+    buf, stride, otabs = stack_tables(rng, H, E, M, 0.25, cheap_links=True)
+    P = rng.random((H - 1, E, E)).astype(np.float32)
+    P[P < 0.6] = 0
+    P = (P / np.maximum(P.sum(axis=2, keepdims=True), 1e-9)).astype(np.float32)
+    X = torch.randn(T, d, device=DEV).to(torch.bfloat16)
+    W_r = (torch.randn(E, d, device=DEV) * 0.2).to(torch.bfloat16)
+    home = rng.integers(0, M, T).astype(np.uint8)
+    loc = np.where(rng.random(T) < 0.5, home, rng.integers(0, M, T)).astype(np.uint8)
+    qhat = (rng.random(T) * 0.1).astype(np.float32)
+    g = [torch.empty(T, k, dtype=dt, device=DEV)
+         for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
+    lg = torch.empty(T, E, device=DEV)
+    cnt = torch.zeros(4, dtype=torch.int32, device=DEV)
+    gl = torch.as_tensor(loc).to(DEV); gq = torch.as_tensor(qhat).to(DEV)
+    B.ordermoe_route_select_lookahead(X, W_r, None, T, E, d, k, 1, buf, stride, H,
+                                      torch.as_tensor(P).to(DEV), torch.as_tensor(home).to(DEV),
+                                      gl, gq, lg, *g, counters=cnt)
+    logits = lg.cpu().numpy()
+    idx, _ = oracle.topk(logits, k)
+    np.testing.assert_array_equal(g[0].cpu().numpy(), idx)
+    ch, sv, kd, rl, rq = oracle.select_lookahead(idx, otabs, P, home, loc, qhat)
+    np.testing.assert_array_equal(g[2].cpu().numpy(), ch)
+    np.testing.assert_array_equal(g[3].cpu().numpy(), sv)
+    np.testing.assert_array_equal(g[4].cpu().numpy(), kd)
+    np.testing.assert_array_equal(gl.cpu().numpy(), rl)
+    np.testing.assert_array_equal(gq.cpu().numpy(), rq)
+    np.testing.assert_array_equal(cnt.cpu().numpy(), np.bincount(kd.ravel(), minlength=4))
+
+
+def test_lookahead_skips_a_nan_token_and_reports_it():
+    rng = np.random.default_rng(9)
+    E, M, k, T, H = 8, 4, 2, 70, 2
+    buf, stride, otabs = stack_tables(rng, H, E, M, 0.2, cheap_links=True)
+    P = np.full((1, E, E), 1.0 / E, np.float32)
+    logits = rng.standard_normal((T, E)).astype(np.float32)
+    bad = logits.copy(); bad[3, 5] = np.nan
+    home = rng.integers(0, M, T).astype(np.uint8)
+    g = [torch.empty(T, k, dtype=dt, device=DEV)
+         for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
+    gl = torch.as_tensor(home).to(DEV); gq = torch.zeros(T, device=DEV)
+    B.ordermoe_route_select_lookahead(None, None, torch.as_tensor(bad).to(DEV), T, E, 0, k, 1, buf,
+                                      stride, H, torch.as_tensor(P).to(DEV),
+                                      torch.as_tensor(home).to(DEV), gl, gq, None, *g)
+    code, detail = B.ordermoe_device_error()
+    assert code == B.DEV_NAN_LOGIT and detail == 3
+    idx, _ = oracle.topk(logits, k)
+    ch, sv, kd, rl, rq = oracle.select_lookahead(idx, otabs, P, home, home.copy(),
+                                                 np.zeros(T, np.float32))
+    keep = np.arange(T) != 3
+    np.testing.assert_array_equal(g[2].cpu().numpy()[keep], ch[keep])
+    np.testing.assert_array_equal(g[3].cpu().numpy()[keep], sv[keep])
+    np.testing.assert_array_equal(gl.cpu().numpy()[keep], rl[keep])
+    assert gl[3].item() == home[3] and gq[3].item() == 0.0       # state of the NaN token kept
+    assert (g[0][3] == -1).all().item()
