@@ -51,6 +51,7 @@ def lib():
             "orc_importance": [_P, _P, _P, _I, _D, _D, _P],
             "orc_place": [_P, _P, _P, _I, _I, _I, _P, _D, _D, _P, _P],
             "orc_coverage": [_P, _P, _I, _I, _I, _P],
+            "orc_replicate": [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P],
             "orc_transitions": [_P, _I64, _I, _I, _I, _P, _P],
             "orc_select_lookahead": [_P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                      _P, _F, _P, _P, _P, _P, _P, _P],
@@ -219,6 +220,22 @@ def place(group, importance, p, C, lambda1=0.5, lambda2=0.5):
     if rc not in (OK, CAPACITY):
         _check(rc, "orc_place")
     return x, used, rc
+
+
+def replicate(group, importance, p, C, pi, placement, used):
+    """Redundant deployment (Eqs. 32-35) after the mandatory placement.
+    group/importance/p: [L,E]; C, pi, used: [M]; placement [L,M,E].
+    Returns (placement, used, replicas [M]) as new arrays."""
+    group = _c(group, np.int32); importance = _c(importance, np.float64)
+    p = _c(p, np.float64); C = _c(C, np.float64); pi = _c(pi, np.float64)
+    x = np.array(placement, dtype=np.uint8, copy=True, order="C")
+    b = np.array(used, dtype=np.float64, copy=True, order="C")
+    L, E = group.shape; M = C.shape[0]
+    assert x.shape == (L, M, E) and b.shape == (M,) and pi.shape == (M,)
+    reps = np.empty(M, np.int32)
+    _check(lib().orc_replicate(_ptr(group), _ptr(importance), _ptr(p), L, E, M, _ptr(C), _ptr(pi),
+                               _ptr(x), _ptr(b), _ptr(reps)), "orc_replicate")
+    return x, b, reps
 
 
 def coverage(placement_l, group_l, K):

@@ -28,6 +28,9 @@
 //  * placement (Eqs. 29-31): the within-layer order is memory demand desc,
 //    then importance desc, then index asc; score ties go to the lower server;
 //    the used memory b_m accumulates over layers (Alg. 1 initialises it once).
+//  * redundancy (Eqs. 32-35): a replica's benefit is pi_m I (1 - y) / p; the
+//    greedy takes the largest fitting benefit (ties: lower layer, server,
+//    expert); pi_m is the share of tokens whose trajectory reaches server m.
 #include <algorithm>
 #include <cmath>
 #include <limits>
@@ -488,6 +491,53 @@ int orc_place(const int32_t* group, const double* importance, const double* p, i
   }
   for (int m = 0; m < M; ++m) used[m] = b[m];
   return overflow ? ORC_CAPACITY : ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Importance-aware redundant deployment, Section IV-C (Eqs. 32-35, Alg. 1
+// lines 25-28), over all layers after the mandatory placement. y[m][l][g]
+// (Eq. 32) is 1 when server m hosts an expert of group g in layer l. A
+// candidate replica of expert j of layer l on server m has the benefit
+// B = pi_m * I_l^j * (1 - y[m][l][g(j)]) / p_l^j (Eq. 33), and fits when
+// b_m + p_l^j <= C_m (Eq. 35). Greedy: each round recomputes every benefit,
+// deploys the largest one that fits (ties: lower layer, then lower server,
+// then lower expert), updates y and b_m, and stops when no fitting candidate
+// has a positive benefit. placement [L][M][E] and used [M] are updated in
+// place; replicas [M] counts the replicas per server. pi [M]: the share of
+// the tokens whose trajectory reaches each server.
+int orc_replicate(const int32_t* group, const double* importance, const double* p, int L, int E,
+                  int M, const double* C, const double* pi, uint8_t* placement, double* used,
+                  int32_t* replicas) {
+  for (int i = 0; i < L * E; ++i)
+    if (!(p[i] > 0.0) || group[i] < 0 || group[i] >= E) return ORC_BAD_ARG;
+  // Eq. 32 from the mandatory placement
+  std::vector<uint8_t> y((size_t)M * L * E, 0);
+  for (int l = 0; l < L; ++l)
+    for (int m = 0; m < M; ++m)
+      for (int j = 0; j < E; ++j)
+        if (placement[((size_t)l * M + m) * E + j])
+          y[((size_t)m * L + l) * E + group[l * E + j]] = 1;
+  for (int m = 0; m < M; ++m) replicas[m] = 0;
+  for (;;) {
+    int bl = -1, bm = -1, bj = -1;
+    double bb = 0.0;
+    for (int l = 0; l < L; ++l)
+      for (int m = 0; m < M; ++m)
+        for (int j = 0; j < E; ++j) {
+          const int g = group[l * E + j];
+          const double cover = 1.0 - static_cast<double>(y[((size_t)m * L + l) * E + g]);
+          const double benefit = pi[m] * importance[l * E + j] * cover / p[l * E + j];
+          if (!(benefit > 0.0)) continue;
+          if (!(used[m] + p[l * E + j] <= C[m])) continue;
+          if (bl < 0 || benefit > bb) { bl = l; bm = m; bj = j; bb = benefit; }
+        }
+    if (bl < 0) break;
+    placement[((size_t)bl * M + bm) * E + bj] = 1;
+    used[bm] += p[bl * E + bj];
+    y[((size_t)bm * L + bl) * E + group[bl * E + bj]] = 1;
+    replicas[bm]++;
+  }
+  return ORC_OK;
 }
 
 // ---------------------------------------------------------------------------

@@ -49,6 +49,17 @@ MUTANTS = [
      "{ s += sim[j * E + k]; ++size; }"),
     ("Eq. 30: dispersion term dropped", "lambda2 * static_cast<double>(eta)", "0.0"),
     ("Eq. 29: capacity ignored", "if (!(b[m] + pl[j] <= C[m])) continue;", ""),
+    ("Eq. 32: coverage not updated after a replica",
+     "y[((size_t)bm * L + bl) * E + group[bl * E + bj]] = 1;", ""),
+    ("Eq. 33: coverage term dropped",
+     "const double cover = 1.0 - static_cast<double>(y[((size_t)m * L + l) * E + g]);",
+     "const double cover = 1.0;"),
+    ("Eq. 33: benefit not per unit memory", "* cover / p[l * E + j];", "* cover;"),
+    ("Eq. 33: pi dropped", "const double benefit = pi[m] * importance", "const double benefit = 1.0 * importance"),
+    ("Eq. 35: capacity ignored", "if (!(used[m] + p[l * E + j] <= C[m])) continue;", ""),
+    ("Eq. 35: used memory not updated", "used[bm] += p[bl * E + bj];", ""),
+    ("redundancy: ties to the later candidate", "if (bl < 0 || benefit > bb) { bl = l;",
+     "if (bl < 0 || benefit >= bb) { bl = l;"),
     ("Eq. 41: transitions of the same layer", "topk(logits + (n * L + l + 1) * E, nxt);",
      "topk(logits + (n * L + l) * E, nxt);"),
     ("Eq. 42: transition from the target, not the executed expert",

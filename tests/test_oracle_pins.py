@@ -644,6 +644,127 @@ def test_coverage(orc):
     np.testing.assert_array_equal(orc.coverage(x, g, 2), [[1, 1], [1, 0]])
 
 
+def test_replicate_hand_example(orc):
+    # Section IV-C on one layer: groups {0,1} x {2,3}; server 0 covers group 0
+    # only, server 1 group 1 only. Benefits (Eq. 33): on server 0, e2 0.15 and
+    # e3 0.075; on server 1, e0 0.1 and e1 0.075. One replica each covers the
+    # missing group, after which the other candidates' benefit is 0.
+    g = np.array([[0, 0, 1, 1]], np.int32)
+    I = np.array([[0.4, 0.3, 0.2, 0.1]]); p = np.ones((1, 4))
+    x = np.zeros((1, 2, 4), np.uint8); x[0, 0, :2] = 1; x[0, 1, 2:] = 1
+    pi = np.array([0.75, 0.25])
+    x1, b1, r1 = orc.replicate(g, I, p, np.array([3.0, 3.0]), pi, x, np.array([2.0, 2.0]))
+    np.testing.assert_array_equal(x1[0], [[1, 1, 1, 0], [1, 0, 1, 1]])
+    np.testing.assert_array_equal(b1, [3, 3]); np.testing.assert_array_equal(r1, [1, 1])
+    # Eq. 35: server 1 is full, so only server 0 gets a replica
+    x2, b2, r2 = orc.replicate(g, I, p, np.array([3.0, 2.0]), pi, x, np.array([2.0, 2.0]))
+    np.testing.assert_array_equal(x2[0], [[1, 1, 1, 0], [0, 0, 1, 1]])
+    np.testing.assert_array_equal(r2, [1, 0])
+    # a server that no token reaches (pi = 0) has no positive benefit
+    x3, _, r3 = orc.replicate(g, I, p, np.array([3.0, 3.0]), np.array([1.0, 0.0]), x,
+                              np.array([2.0, 2.0]))
+    np.testing.assert_array_equal(r3, [1, 0]); assert x3[0, 1].tolist() == [0, 0, 1, 1]
+    # nothing to cover: every server already holds every group
+    xf = np.ones((1, 2, 4), np.uint8)
+    _, _, r4 = orc.replicate(g, I, p, np.array([9.0, 9.0]), pi, xf, np.array([4.0, 4.0]))
+    np.testing.assert_array_equal(r4, [0, 0])
+
+
+def test_replicate_benefit_is_per_unit_memory_and_ties_go_low(orc):
+    # server 0 holds e0 (group 0); group 1 = {e1, e2, e3} with I = .5/.3/.1 and
+    # p = 2/1/1: per unit memory e2 (0.3) beats e1 (0.25).
+    g = np.array([[0, 1, 1, 1]], np.int32)
+    I = np.array([[0.6, 0.5, 0.3, 0.1]]); p = np.array([[1.0, 2.0, 1.0, 1.0]])
+    x = np.zeros((1, 1, 4), np.uint8); x[0, 0, 0] = 1
+    x1, b1, r1 = orc.replicate(g, I, p, np.array([10.0]), np.array([1.0]), x, np.array([1.0]))
+    assert x1[0, 0].tolist() == [1, 0, 1, 0] and b1[0] == 2.0 and r1[0] == 1
+    # equal benefits inside a server: the lower expert wins
+    I2 = np.array([[0.6, 0.3, 0.3, 0.1]]); p2 = np.ones((1, 4))
+    x2, _, _ = orc.replicate(g, I2, p2, np.array([10.0]), np.array([1.0]), x, np.array([1.0]))
+    assert x2[0, 0].tolist() == [1, 1, 0, 0]
+    # room for one replica, equal benefits in two layers: the lower layer wins
+    g3 = np.array([[0, 1], [0, 1]], np.int32)
+    I3 = np.array([[0.5, 0.5], [0.5, 0.5]]); p3 = np.ones((2, 2))
+    x3 = np.zeros((2, 1, 2), np.uint8); x3[:, 0, 0] = 1
+    x4, _, r = orc.replicate(g3, I3, p3, np.array([3.0]), np.array([1.0]), x3, np.array([2.0]))
+    assert x4[0, 0].tolist() == [1, 1] and x4[1, 0].tolist() == [1, 0] and r[0] == 1
+
+
+def per_server_sweep(group, I, p, C, pi, x, used):
+    """The greedy of Eqs. 34-35 decomposes over servers (memory and coverage are
+    per server, benefits only drop to 0): for each server, visit its
+    candidates by benefit desc (ties: layer, expert) and deploy each one whose
+    group is still uncovered there and which still fits."""
+    L, M, E = x.shape
+    x = x.copy(); b = used.astype(np.float64).copy(); reps = np.zeros(M, np.int64)
+    for m in range(M):
+        cov = {(l, group[l, j]) for l in range(L) for j in range(E) if x[l, m, j]}
+        cand = []
+        for l in range(L):
+            for j in range(E):
+                ben = pi[m] * I[l, j] * 1.0 / p[l, j]
+                if ben > 0 and (l, group[l, j]) not in cov:
+                    cand.append((-ben, l, j))
+        for _, l, j in sorted(cand):
+            if (l, group[l, j]) in cov or not (b[m] + p[l, j] <= C[m]):
+                continue
+            x[l, m, j] = 1; b[m] += p[l, j]; cov.add((l, group[l, j])); reps[m] += 1
+    return x, b, reps
+
+
+def test_replicate_invariants_and_per_server_decomposition(orc):
+    rng = np.random.default_rng(33)
+    for it in range(60):
+        L, E, M = int(rng.integers(1, 5)), int(rng.integers(2, 9)), int(rng.integers(1, 6))
+        group = rng.integers(0, min(3, E), (L, E)).astype(np.int32)   # group ids < E
+        I = rng.random((L, E)) - (0.2 if it % 3 == 0 else 0.0)     # some non-positive
+        I[rng.random((L, E)) < 0.2] = 0.5                          # ties
+        p = rng.integers(1, 4, (L, E)).astype(np.float64)
+        C = np.full(M, p.sum() / M) * rng.uniform(1.0, 3.0, M)
+        pi = rng.random(M); pi[rng.random(M) < 0.2] = 0.0
+        x0, used0, rc = orc.place(group, np.abs(I), p, C)
+        if rc != 0:
+            continue
+        x, used, reps = orc.replicate(group, I, p, C, pi, x0, used0)
+        load = np.einsum("lme,le->m", x.astype(np.float64), p)
+        np.testing.assert_allclose(load, used)
+        assert (used <= C).all()                                           # Eq. 35
+        assert ((x >= x0).all() and int((x - x0).sum()) == int(reps.sum()))
+        for l in range(L):
+            K = int(group[l].max()) + 1
+            c0 = orc.coverage(x0[l], group[l], K); c1 = orc.coverage(x[l], group[l], K)
+            new = x[l].astype(int) - x0[l]
+            for m in range(M):
+                for gg in range(K):
+                    nrep = int(new[m][group[l] == gg].sum())
+                    assert nrep <= 1 and (nrep == 0 or c0[m, gg] == 0)     # Eq. 32: one per group
+                    if c1[m, gg] == 0:                                     # greedy stopped for a reason
+                        for j in np.nonzero(group[l] == gg)[0]:
+                            assert pi[m] * I[l, j] <= 0 or used[m] + p[l, j] > C[m]
+        xs, bs, rs = per_server_sweep(group, I, p, C, pi, x0, used0)
+        np.testing.assert_array_equal(x, xs)
+        np.testing.assert_array_equal(used, bs)
+        np.testing.assert_array_equal(reps, rs)
+
+
+def test_replicate_with_ample_memory_covers_every_group_everywhere(orc):
+    rng = np.random.default_rng(4)
+    L, E, M = 3, 8, 4
+    group = rng.integers(0, 4, (L, E)).astype(np.int32)
+    I = rng.random((L, E)) + 0.1; p = np.ones((L, E))
+    x0, used0, rc = orc.place(group, I, p, np.full(M, L * E / M))
+    assert rc == 0
+    x, used, reps = orc.replicate(group, I, p, np.full(M, 1e9), np.full(M, 0.25), x0, used0)
+    uncovered = 0
+    for l in range(L):
+        K = int(group[l].max()) + 1
+        present = np.unique(group[l])
+        c0 = orc.coverage(x0[l], group[l], K); c1 = orc.coverage(x[l], group[l], K)
+        assert (c1[:, present] == 1).all()
+        uncovered += int((c0[:, present] == 0).sum())
+    assert int(reps.sum()) == uncovered
+
+
 def test_group_threshold_is_strict_and_ties_go_to_the_earlier_dominant(orc):
     cnt = np.array([3, 2, 1], np.int32)            # visiting order 0, 1, 2
     # Sim(1, 0) == theta: Eq. 24 needs max Sim < theta for a new dominant, so 1 joins 0
