@@ -196,7 +196,7 @@ def setup_gpu(w, seed, device):
     p = torch.ones(1, w.E, dtype=torch.float64, device=device)
     C = torch.full((w.M,), w.E / w.M, dtype=torch.float64, device=device)
     B.ordermoe_place(sim, counts, 1, w.E, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5, 0.5,
-                     0.5, p, C, group, ngroups, theta, placement, used, status)
+                     0.5, p, C, group, ngroups, theta, None, placement, used, status)
     sp = synth.server_params(w.M, w.d, w.dff, seed)
     f64 = lambda a: torch.as_tensor(a, dtype=torch.float64).to(device)
     tables = torch.zeros(B.ordermoe_tables_bytes(w.E, w.M), dtype=torch.uint8, device=device)
@@ -424,7 +424,7 @@ def run_decode(args, dist, w, device):
     B.ordermoe_place(sim, counts, L, E, M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5, 0.5, 0.5,
                      torch.ones(L, E, dtype=torch.float64, device=device),
                      torch.full((M,), L * E / M, dtype=torch.float64, device=device),
-                     group, ng, theta, x, used, st)
+                     group, ng, theta, None, x, used, st)
     # transition statistics (Eq. 41) from the calibration logits the similarity
     # call leaves at the start of its workspace
     H = max(1, args.lookahead)
@@ -525,7 +525,7 @@ def run_similarity(args, dist, w, device):
     def step():
         B.ordermoe_similarity(Wr, Xcal, L, E, d, N, w.k, sim, counts, ws)
         B.ordermoe_place(sim, counts, L, E, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5,
-                         0.5, 0.5, p, C, group, ng, theta, x, used, st)
+                         0.5, 0.5, p, C, group, ng, theta, None, x, used, st)
 
     ms, clocks = timed_region(args, dist, device, step)
     code, detail = B.ordermoe_device_error()

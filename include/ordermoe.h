@@ -49,7 +49,8 @@ enum {
   ORDERMOE_DEV_NAN_LOGIT = 1,     /* route_select: a logit was NaN             */
   ORDERMOE_DEV_BAD_INDEX = 2,     /* an expert/server index out of range       */
   ORDERMOE_DEV_NO_CANDIDATE = 3,  /* selection: target expert placed nowhere   */
-  ORDERMOE_DEV_WAIT_TIMEOUT = 4   /* a bounded pipeline wait ran out           */
+  ORDERMOE_DEV_WAIT_TIMEOUT = 4,  /* a bounded pipeline wait ran out           */
+  ORDERMOE_DEV_BAD_VALUE = 5      /* redundancy: a memory demand p <= 0 or NaN */
 };
 
 #define ORDERMOE_MAX_EXPERTS 64
@@ -340,6 +341,7 @@ int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq, in
  *   sim [L][E][E] f32, counts [L][E] i32, p [L][E] f64 (memory of each
  *   expert), C [M] f64 (server capacities)
  *   group [L][E] i32 out, n_groups [L] i32 out, theta [L] f32 out,
+ *   importance [L][E] f64 out (nullable; the input of ordermoe_replicate),
  *   placement [L][M][E] u8 out, used [M] f64 out,
  *   status [1] i32 out (device): ORDERMOE_OK, or ORDERMOE_ERR_CAPACITY when
  *   sum C < sum p or a waiting-list expert overflowed its server.
@@ -350,9 +352,44 @@ size_t ordermoe_place_workspace_bytes(int L, int E);
 int ordermoe_place(const float* sim, const int32_t* counts, int L, int E, int M, double theta_min,
                    double theta_max, double theta_single, double alpha_f, double alpha_r,
                    double lambda1, double lambda2, const double* p, const double* C,
-                   int32_t* group, int32_t* n_groups, float* theta, uint8_t* placement,
-                   double* used, int32_t* status, void* workspace, size_t workspace_bytes,
-                   ordermoe_stream_t stream);
+                   int32_t* group, int32_t* n_groups, float* theta, double* importance,
+                   uint8_t* placement, double* used, int32_t* status, void* workspace,
+                   size_t workspace_bytes, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Importance-aware redundant deployment (Section IV-C, Eqs. 32-35; Alg. 1
+ * lines 25-28), after the mandatory placement, over all layers:
+ *   y[m][l][g] = 1 when server m hosts an expert of group g of layer l (Eq. 32);
+ *   benefit of a replica of expert j of layer l on server m:
+ *     B = pi_m * I_l^j * (1 - y[m][l][g(j)]) / p_l^j          (Eq. 33);
+ *   it fits when b_m + p_l^j <= C_m                          (Eq. 35);
+ *   greedy (Eq. 34): deploy the largest fitting positive benefit (ties: lower
+ *   layer, then lower server, then lower expert), update y and b_m, repeat
+ *   until no fitting candidate has a positive benefit.
+ * Memory and coverage are per server and a benefit only ever drops to 0, so
+ * the greedy runs as one independent pass per server (one CTA each): its
+ * candidates sorted by (benefit desc, layer, expert), then swept in order.
+ *   group [L][E] i32 (ids < E), importance [L][E] f64 (ordermoe_place's),
+ *   p [L][E] f64 (> 0), C [M] f64, pi [M] f64 (the share of tokens whose
+ *   trajectory reaches each server; a server with pi_m <= 0 gets no replica);
+ *   placement [L][M][E] u8 in/out, used [M] f64 in/out (b_m),
+ *   replicas [M] i32 out (replicas deployed per server).
+ * Needs L * E <= 16384, L <= 1024, M <= 32. A group id >= E sets
+ * ORDERMOE_DEV_BAD_INDEX, a p <= 0 or NaN ORDERMOE_DEV_BAD_VALUE (the entry is
+ * skipped); both are read with ordermoe_device_error. */
+int ordermoe_replicate(const int32_t* group, const double* importance, const double* p,
+                       const double* C, const double* pi, int L, int E, int M,
+                       uint8_t* placement, double* used, int32_t* replicas,
+                       ordermoe_stream_t stream);
+
+/* Local group coverage (Eq. 32) of a placement: cover[l][m][g] = 1 when server
+ * m hosts an expert of group g in layer l (g < E; entries of groups a layer
+ * does not have stay 0), covered[l] = the number of such (m, g) pairs. The
+ * coverage ratio of Section VI-G is sum covered / (M * sum n_groups).
+ *   group [L][E] i32, placement [L][M][E] u8; cover [L][M][E] u8 out
+ *   (nullable), covered [L] i32 out (nullable). */
+int ordermoe_coverage(const int32_t* group, const uint8_t* placement, int L, int E, int M,
+                      uint8_t* cover, int32_t* covered, ordermoe_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -14,7 +14,7 @@ LIB_PATH = os.path.join(_HERE, "libordermoe.so")
 
 OK = 0
 ERR_INVALID_ARG, ERR_UNSUPPORTED_SHAPE, ERR_CAPACITY, ERR_CUDA, ERR_DEVICE_CHECK = 1, 2, 3, 4, 5
-DEV_OK, DEV_NAN_LOGIT, DEV_BAD_INDEX, DEV_NO_CANDIDATE, DEV_WAIT_TIMEOUT = 0, 1, 2, 3, 4
+DEV_OK, DEV_NAN_LOGIT, DEV_BAD_INDEX, DEV_NO_CANDIDATE, DEV_WAIT_TIMEOUT, DEV_BAD_VALUE = 0, 1, 2, 3, 4, 5
 
 _lib = None
 _P = ctypes.c_void_p
@@ -43,7 +43,9 @@ _SIGNATURES = {
     "ordermoe_similarity": ([_P, _P, _I, _I, _I, _I64, _I, _P, _P, _P, _SZ, _P], _I),
     "ordermoe_expert_counts": ([_P, _I64, _I, _I, _P, _P], _I),
     "ordermoe_place": ([_P, _P, _I, _I, _I, _D, _D, _D, _D, _D, _D, _D, _P, _P, _P, _P, _P, _P,
-                        _P, _P, _P, _SZ, _P], _I),
+                        _P, _P, _P, _P, _SZ, _P], _I),
+    "ordermoe_replicate": ([_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P], _I),
+    "ordermoe_coverage": ([_P, _P, _I, _I, _I, _P, _P, _P], _I),
     "ordermoe_place_workspace_bytes": ([_I, _I], _SZ),
     "ordermoe_expert_gate_up": ([_P, _P, _I, _P, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_expert_down": ([_P, _P, _I, _P, _I, _I, _I, _P, _P], _I),
@@ -226,10 +228,11 @@ def ordermoe_place_workspace_bytes(L, E):
 
 
 def ordermoe_place(sim, counts, L, E, M, theta_min, theta_max, theta_single, alpha_f, alpha_r,
-                   lambda1, lambda2, p, C, group, n_groups, theta, placement, used, status,
-                   workspace=None, stream=None):
-    """workspace: device scratch of ordermoe_place_workspace_bytes(L, E) bytes;
-    allocated here with torch when not given."""
+                   lambda1, lambda2, p, C, group, n_groups, theta, importance, placement, used,
+                   status, workspace=None, stream=None):
+    """importance: [L, E] f64 output or None. workspace: device scratch of
+    ordermoe_place_workspace_bytes(L, E) bytes; allocated here with torch when
+    not given."""
     if workspace is None:
         workspace = torch.empty(ordermoe_place_workspace_bytes(L, E), dtype=torch.uint8,
                                 device=sim.device)
@@ -237,14 +240,33 @@ def ordermoe_place(sim, counts, L, E, M, theta_min, theta_max, theta_single, alp
     _dt(p, torch.float64, "p"); _dt(C, torch.float64, "C"); _dt(group, torch.int32, "group")
     _dt(n_groups, torch.int32, "n_groups"); _dt(theta, torch.float32, "theta")
     _dt(placement, torch.uint8, "placement"); _dt(used, torch.float64, "used")
-    _dt(status, torch.int32, "status")
+    _dt(status, torch.int32, "status"); _dt(importance, torch.float64, "importance")
     rc = lib().ordermoe_place(_ptr(sim), _ptr(counts), L, E, M, float(theta_min), float(theta_max),
                               float(theta_single), float(alpha_f), float(alpha_r), float(lambda1),
                               float(lambda2), _ptr(p), _ptr(C), _ptr(group), _ptr(n_groups),
-                              _ptr(theta), _ptr(placement), _ptr(used), _ptr(status),
+                              _ptr(theta), _ptr(importance), _ptr(placement), _ptr(used), _ptr(status),
                               _ptr(workspace), workspace.numel() * workspace.element_size(),
                               _stream(stream))
     _check("ordermoe_place", rc)
+
+
+def ordermoe_replicate(group, importance, p, C, pi, L, E, M, placement, used, replicas, stream=None):
+    """Redundant deployment (Eqs. 32-35); placement and used are updated in place."""
+    _dt(group, torch.int32, "group"); _dt(importance, torch.float64, "importance")
+    _dt(p, torch.float64, "p"); _dt(C, torch.float64, "C"); _dt(pi, torch.float64, "pi")
+    _dt(placement, torch.uint8, "placement"); _dt(used, torch.float64, "used")
+    _dt(replicas, torch.int32, "replicas")
+    _check("ordermoe_replicate", lib().ordermoe_replicate(
+        _ptr(group), _ptr(importance), _ptr(p), _ptr(C), _ptr(pi), L, E, M, _ptr(placement),
+        _ptr(used), _ptr(replicas), _stream(stream)))
+
+
+def ordermoe_coverage(group, placement, L, E, M, cover=None, covered=None, stream=None):
+    """Local group coverage (Eq. 32): cover [L, M, E] u8 and covered [L] i32 (either may be None)."""
+    _dt(group, torch.int32, "group"); _dt(placement, torch.uint8, "placement")
+    _dt(cover, torch.uint8, "cover"); _dt(covered, torch.int32, "covered")
+    _check("ordermoe_coverage", lib().ordermoe_coverage(_ptr(group), _ptr(placement), L, E, M,
+                                                        _ptr(cover), _ptr(covered), _stream(stream)))
 
 
 def ordermoe_expert_gate_up(X_perm, offsets, R, W1, W3, E, d, dff, H, stream=None):

@@ -3,7 +3,9 @@
 //     Sim = cosine of the rows of H (Eq. 4), activation counts n_j (Eq. 5);
 //   ordermoe_expert_counts: the counts of Eq. 5 from given logits;
 //   ordermoe_place: threshold (Eq. 6), greedy grouping (Eqs. 24-26),
-//     importance (Eqs. 27-28) and mandatory placement (Eqs. 29-31).
+//     importance (Eqs. 27-28) and mandatory placement (Eqs. 29-31);
+//   ordermoe_replicate: redundant deployment (Eqs. 32-35);
+//   ordermoe_coverage: local group coverage (Eq. 32).
 #include "common.cuh"
 
 namespace om {
@@ -286,7 +288,8 @@ struct PlaceParams {
 __global__ void __launch_bounds__(64) group_kernel(
     const float* __restrict__ sim, const int32_t* __restrict__ counts, int L, int E,
     PlaceParams pp, const double* __restrict__ p, int32_t* __restrict__ group,
-    int32_t* __restrict__ n_groups, float* __restrict__ theta_out, int32_t* __restrict__ porder) {
+    int32_t* __restrict__ n_groups, float* __restrict__ theta_out, double* __restrict__ importance,
+    int32_t* __restrict__ porder) {
   __shared__ double imp[64];
   __shared__ double pls[64];
   __shared__ int order[64];
@@ -366,6 +369,7 @@ __global__ void __launch_bounds__(64) group_kernel(
     const double rho = __ddiv_rn(sum, static_cast<double>(size));
     const double f = total > 0.0 ? __ddiv_rn(static_cast<double>(cnt[t]), total) : 0.0;
     imp[t] = __dadd_rn(__dmul_rn(pp.alpha_f, f), __dmul_rn(pp.alpha_r, rho));
+    if (importance != nullptr) importance[(size_t)l * E + t] = imp[t];
   }
   __syncthreads();
   // placement order: p desc, I desc, index asc
@@ -543,6 +547,124 @@ extern "C" int ordermoe_expert_counts(const float* logits, int64_t N, int E, int
   return ORDERMOE_OK;
 }
 
+namespace om {
+
+constexpr int kRepThreads = 512;
+constexpr int kRepMaxCand = 16384;
+constexpr int kRepMaxLayers = 1024;
+
+// Redundant deployment for one server (blockIdx.x = m), Eqs. 32-35. The
+// candidates (l, j) get the key (benefit bits, then candidate id), are sorted
+// by benefit desc and id asc (bitonic sort in shared memory), and one thread
+// deploys them in that order while the group is uncovered and the replica
+// fits. Benefits are positive fp64 values, so their bit patterns order like
+// the values; non-positive and NaN benefits get key 0 and are never taken.
+__global__ void __launch_bounds__(kRepThreads) replicate_kernel(
+    const int32_t* __restrict__ group, const double* __restrict__ importance,
+    const double* __restrict__ p, const double* __restrict__ C, const double* __restrict__ pi,
+    int L, int E, int M, int Np, uint8_t* __restrict__ placement, double* __restrict__ used,
+    int32_t* __restrict__ replicas) {
+  extern __shared__ __align__(16) unsigned char s_rep[];
+  unsigned long long* key = reinterpret_cast<unsigned long long*>(s_rep);
+  unsigned long long* cov = key + Np;  // [L]: bit g = group g covered (Eq. 32)
+  uint32_t* cid = reinterpret_cast<uint32_t*>(cov + L);
+  const int m = blockIdx.x;
+  const int t = threadIdx.x;
+  const int N = L * E;
+  for (int l = t; l < L; l += blockDim.x) {
+    unsigned long long bits = 0;
+    for (int j = 0; j < E; ++j) {
+      const int g = group[(size_t)l * E + j];
+      if (placement[((size_t)l * M + m) * E + j] && g >= 0 && g < E) bits |= 1ull << g;
+    }
+    cov[l] = bits;
+  }
+  const double pim = pi[m];
+  for (int i = t; i < Np; i += blockDim.x) {
+    unsigned long long k = 0;
+    if (i < N) {
+      const int g = group[i];
+      const double pj = p[i];
+      if (g < 0 || g >= E) {
+        if (m == 0) report(&g_err_sim, ORDERMOE_DEV_BAD_INDEX, i);
+      } else if (!(pj > 0.0)) {
+        if (m == 0) report(&g_err_sim, ORDERMOE_DEV_BAD_VALUE, i);
+      } else {
+        const double ben = __ddiv_rn(__dmul_rn(pim, importance[i]), pj);  // Eq. 33, y = 0
+        if (ben > 0.0) k = static_cast<unsigned long long>(__double_as_longlong(ben));
+      }
+    }
+    key[i] = k;
+    cid[i] = i < N ? static_cast<uint32_t>(i) : 0xFFFFFFFFu;
+  }
+  __syncthreads();
+  // bitonic sort into (key desc, cid asc)
+  for (int size = 2; size <= Np; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = t; i < Np; i += blockDim.x) {
+        const int o = i ^ stride;
+        if (o > i) {
+          const unsigned long long ki = key[i], ko = key[o];
+          const uint32_t ci = cid[i], co = cid[o];
+          const bool o_first = ko > ki || (ko == ki && co < ci);
+          const bool i_first = ki > ko || (ki == ko && ci < co);
+          if ((i & size) == 0 ? o_first : i_first) {
+            key[i] = ko; key[o] = ki;
+            cid[i] = co; cid[o] = ci;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+  if (t == 0) {
+    double b = used[m];
+    const double cap = C[m];
+    int count = 0;
+    for (int s = 0; s < N && key[s] != 0; ++s) {
+      const int i = static_cast<int>(cid[s]);
+      const int l = i / E, j = i - l * E;
+      const int g = group[i];
+      if ((cov[l] >> g) & 1ull) continue;  // B = 0 once the group is local
+      const double pj = p[i];
+      if (!(__dadd_rn(b, pj) <= cap)) continue;  // Eq. 35
+      placement[((size_t)l * M + m) * E + j] = 1;
+      b = __dadd_rn(b, pj);
+      cov[l] |= 1ull << g;
+      ++count;
+    }
+    used[m] = b;
+    replicas[m] = count;
+  }
+}
+
+// Eq. 32 for one layer (blockIdx.x = l): thread m ORs its server's groups.
+__global__ void __launch_bounds__(32) coverage_kernel(const int32_t* __restrict__ group,
+                                                      const uint8_t* __restrict__ placement, int L,
+                                                      int E, int M, uint8_t* __restrict__ cover,
+                                                      int32_t* __restrict__ covered) {
+  const int l = blockIdx.x;
+  const int m = threadIdx.x;
+  unsigned long long bits = 0;
+  if (m < M)
+    for (int j = 0; j < E; ++j) {
+      const int g = group[(size_t)l * E + j];
+      if (g < 0 || g >= E) {
+        report(&g_err_sim, ORDERMOE_DEV_BAD_INDEX, l * E + j);
+        continue;
+      }
+      if (placement[((size_t)l * M + m) * E + j]) bits |= 1ull << g;
+    }
+  if (m < M && cover != nullptr)
+    for (int g = 0; g < E; ++g) cover[((size_t)l * M + m) * E + g] = (bits >> g) & 1ull;
+  int n = __popcll(bits);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
+  if (m == 0 && covered != nullptr) covered[l] = n;
+}
+
+}  // namespace om
+
 extern "C" size_t ordermoe_place_workspace_bytes(int L, int E) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS) return 0;
   return ((size_t)L * E * sizeof(int32_t) + 255) & ~size_t(255);
@@ -552,8 +674,9 @@ extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, in
                               double theta_min, double theta_max, double theta_single,
                               double alpha_f, double alpha_r, double lambda1, double lambda2,
                               const double* p, const double* C, int32_t* group, int32_t* n_groups,
-                              float* theta, uint8_t* placement, double* used, int32_t* status,
-                              void* workspace, size_t workspace_bytes, ordermoe_stream_t stream) {
+                              float* theta, double* importance, uint8_t* placement, double* used,
+                              int32_t* status, void* workspace, size_t workspace_bytes,
+                              ordermoe_stream_t stream) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 || M > ORDERMOE_MAX_SERVERS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "place: need L >= 1, 1 <= E <= 64, 1 <= M <= 32");
   if (!sim || !counts || !p || !C || !group || !n_groups || !theta || !placement || !used || !status)
@@ -562,7 +685,8 @@ extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, in
     return fail(ORDERMOE_ERR_INVALID_ARG, "place: workspace missing or too small");
   int32_t* porder_scratch = static_cast<int32_t*>(workspace);
   PlaceParams pp{theta_min, theta_max, theta_single, alpha_f, alpha_r, lambda1, lambda2};
-  group_kernel<<<L, 64, 0, stream>>>(sim, counts, L, E, pp, p, group, n_groups, theta, porder_scratch);
+  group_kernel<<<L, 64, 0, stream>>>(sim, counts, L, E, pp, p, group, n_groups, theta, importance,
+                                     porder_scratch);
   OM_LAUNCHED("group_kernel");
   place_kernel<<<1, 32, 0, stream>>>(group, porder_scratch, L, E, M, pp, p, C, placement, used, status);
   OM_LAUNCHED("place_kernel");
@@ -589,5 +713,38 @@ extern "C" int ordermoe_transitions(const float* logits, int64_t N, int L, int E
   const int rows = (L - 1) * E;
   transitions_finish_kernel<<<(rows + 127) / 128, 128, 0, stream>>>(counts, rows, E, P);
   OM_LAUNCHED("transitions_finish_kernel");
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_replicate(const int32_t* group, const double* importance, const double* p,
+                                  const double* C, const double* pi, int L, int E, int M,
+                                  uint8_t* placement, double* used, int32_t* replicas,
+                                  ordermoe_stream_t stream) {
+  if (L <= 0 || L > kRepMaxLayers || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 ||
+      M > ORDERMOE_MAX_SERVERS || (long long)L * E > kRepMaxCand)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
+                "replicate: need 1 <= L <= 1024, 1 <= E <= 64, L * E <= 16384, 1 <= M <= 32");
+  if (!group || !importance || !p || !C || !pi || !placement || !used || !replicas)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "replicate: null pointer");
+  int Np = 1;
+  while (Np < L * E) Np <<= 1;
+  const size_t smem = (size_t)Np * (sizeof(unsigned long long) + sizeof(uint32_t)) +
+                      (size_t)L * sizeof(unsigned long long);
+  OM_CUDA(cudaFuncSetAttribute(replicate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)smem));
+  replicate_kernel<<<M, kRepThreads, smem, stream>>>(group, importance, p, C, pi, L, E, M, Np,
+                                                     placement, used, replicas);
+  OM_LAUNCHED("replicate_kernel");
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_coverage(const int32_t* group, const uint8_t* placement, int L, int E,
+                                 int M, uint8_t* cover, int32_t* covered,
+                                 ordermoe_stream_t stream) {
+  if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 || M > ORDERMOE_MAX_SERVERS)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "coverage: need L >= 1, 1 <= E <= 64, 1 <= M <= 32");
+  if (!group || !placement) return fail(ORDERMOE_ERR_INVALID_ARG, "coverage: null pointer");
+  coverage_kernel<<<L, 32, 0, stream>>>(group, placement, L, E, M, cover, covered);
+  OM_LAUNCHED("coverage_kernel");
   return ORDERMOE_OK;
 }

@@ -121,6 +121,22 @@ def homes(T, M, seed, dist="uniform"):
     raise ValueError(dist)
 
 
+def capacities(M, total_memory, ratio, seed):
+    """Server memory C_m [M] f64 at a memory budget ratio (total capacity over
+    the memory of one full copy of the experts, Section VI-G): heterogeneous,
+    proportional to U[12, 48] (the testbed's GB range), scaled so that
+    sum C = ratio * total_memory."""
+    rng = np.random.default_rng(seed + 19)
+    raw = rng.uniform(12.0, 48.0, size=M)
+    return raw * (ratio * float(total_memory) / raw.sum())
+
+
+def token_shares(home, M):
+    """pi_m [M] f64: the share of the tokens whose home (user-server
+    association) is server m, the estimate of Eq. 33's pi_m."""
+    return np.bincount(np.asarray(home, dtype=np.int64), minlength=M)[:M] / float(len(home))
+
+
 @dataclass
 class ServerParams:
     F: np.ndarray      # [M] flop/s

@@ -73,7 +73,7 @@ def gpu_place(sim, counts, M, p, C, theta_min=0.5, theta_max=0.9, theta_single=0
     st = torch.empty(1, dtype=torch.int32, device=DEV)
     B.ordermoe_place(t(sim, torch.float32), t(counts, torch.int32), L, E, M, theta_min, theta_max,
                      theta_single, 0.5, 0.5, 0.5, 0.5, t(p, torch.float64), t(C, torch.float64),
-                     group, ng, theta, x, used, st)
+                     group, ng, theta, None, x, used, st)
     torch.cuda.synchronize()
     return (group.cpu().numpy(), ng.cpu().numpy(), theta.cpu().numpy(), x.cpu().numpy(),
             used.cpu().numpy(), int(st.item()))
@@ -127,6 +127,137 @@ def test_place_unequal_sizes_waiting_list_and_capacity():
         ref = oracle_place_all(sim, counts, M, p, C)
         for name, a, b in zip(("group", "n_groups", "theta", "placement", "used", "status"), got, ref):
             np.testing.assert_array_equal(a, b, err_msg="%s scale %g" % (name, scale))
+
+
+def gpu_replicate(group, I, p, C, pi, x, used):
+    L, E = group.shape; M = len(C)
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a)).to(device=DEV, dtype=dt)
+    gx = t(x, torch.uint8); gb = t(used, torch.float64)
+    reps = torch.empty(M, dtype=torch.int32, device=DEV)
+    B.ordermoe_replicate(t(group, torch.int32), t(I, torch.float64), t(p, torch.float64),
+                         t(C, torch.float64), t(pi, torch.float64), L, E, M, gx, gb, reps)
+    torch.cuda.synchronize()
+    return gx.cpu().numpy(), gb.cpu().numpy(), reps.cpu().numpy()
+
+
+def test_place_importance_output_bit_exact():
+    rng = np.random.default_rng(2)
+    L, E, M = 6, 16, 4
+    sim, counts = synthetic_sims(rng, L, E, 4, 0.4)
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a)).to(device=DEV, dtype=dt)
+    group = torch.empty(L, E, dtype=torch.int32, device=DEV)
+    imp = torch.empty(L, E, dtype=torch.float64, device=DEV)
+    x = torch.empty(L, M, E, dtype=torch.uint8, device=DEV)
+    B.ordermoe_place(t(sim, torch.float32), t(counts, torch.int32), L, E, M, 0.5, 0.9, 0.5, 0.5, 0.5,
+                     0.5, 0.5, t(np.ones((L, E)), torch.float64), t(np.full(M, L * E / M), torch.float64),
+                     group, torch.empty(L, dtype=torch.int32, device=DEV),
+                     torch.empty(L, dtype=torch.float32, device=DEV), imp, x,
+                     torch.empty(M, dtype=torch.float64, device=DEV),
+                     torch.empty(1, dtype=torch.int32, device=DEV))
+    g = group.cpu().numpy()
+    for l in range(L):
+        np.testing.assert_array_equal(imp[l].cpu().numpy(), oracle.importance(sim[l], counts[l], g[l]))
+
+
+@pytest.mark.parametrize("L,E,M,ratio,seed", [(1, 4, 2, 1.5, 0), (3, 6, 3, 2.0, 1), (5, 16, 5, 1.3, 2),
+                                              (7, 13, 6, 2.5, 3), (32, 8, 8, 2.0, 4), (24, 64, 8, 2.0, 5),
+                                              (2, 64, 32, 3.0, 6)])
+def test_replicate_bit_exact(L, E, M, ratio, seed):
+    """Redundant deployment after the mandatory placement, unequal memory
+    demands, ties and non-positive importances, servers no token reaches."""
+    rng = np.random.default_rng(seed)
+    K = max(1, E // 4)
+    group = rng.integers(0, K, (L, E)).astype(np.int32)
+    I = rng.random((L, E)); I[rng.random((L, E)) < 0.15] = 0.5; I[rng.random((L, E)) < 0.05] = -0.1
+    p = rng.integers(1, 4, (L, E)).astype(np.float64) if seed % 2 else np.ones((L, E))
+    C = synth.capacities(M, p.sum(), ratio, seed)
+    x0, used0, rc = oracle.place(group, np.abs(I), p, C)
+    assert rc == 0
+    pi = synth.token_shares(synth.homes(4096, M, seed, "zipf1.1"), M)
+    pi[rng.random(M) < 0.2] = 0.0
+    ref = oracle.replicate(group, I, p, C, pi, x0, used0)
+    got = gpu_replicate(group, I, p, C, pi, x0, used0)
+    for name, a, b in zip(("placement", "used", "replicas"), got, ref):
+        np.testing.assert_array_equal(a, b, err_msg=name)
+    if L * E >= 64:
+        assert ref[2].sum() > 0
+
+
+def test_replicate_largest_shape_and_errors():
+    rng = np.random.default_rng(8)
+    L, E, M = 256, 64, 4                          # L * E = 16384, the largest sort
+    group = rng.integers(0, 16, (L, E)).astype(np.int32)
+    I = rng.random((L, E)); p = np.ones((L, E))
+    C = np.full(M, L * E / M * 1.05)
+    x0, used0, rc = oracle.place(group, I, p, C)
+    assert rc == 0
+    pi = np.array([0.4, 0.3, 0.2, 0.1])
+    ref = oracle.replicate(group, I, p, C, pi, x0, used0)
+    got = gpu_replicate(group, I, p, C, pi, x0, used0)
+    for name, a, b in zip(("placement", "used", "replicas"), got, ref):
+        np.testing.assert_array_equal(a, b, err_msg=name)
+    with pytest.raises(B.OrderMoEError) as ei:
+        gpu_replicate(np.zeros((257, 64), np.int32), np.ones((257, 64)), np.ones((257, 64)), C, pi,
+                      np.zeros((257, 4, 64), np.uint8), np.zeros(4))
+    assert ei.value.code == B.ERR_UNSUPPORTED_SHAPE
+    # a non-positive memory demand is reported and skipped
+    p_bad = np.ones((1, 4)); p_bad[0, 2] = 0.0
+    gpu_replicate(np.array([[0, 0, 1, 1]], np.int32), np.ones((1, 4)), p_bad, np.array([9.0, 9.0]),
+                  np.array([0.5, 0.5]), np.zeros((1, 2, 4), np.uint8), np.zeros(2))
+    code, detail = B.ordermoe_device_error()
+    assert code == B.DEV_BAD_VALUE and detail == 2
+
+
+@pytest.mark.parametrize("L,E,M", [(1, 4, 2), (24, 64, 8), (32, 8, 8), (3, 64, 32)])
+def test_coverage_bit_exact(L, E, M):
+    rng = np.random.default_rng(L + E + M)
+    group = rng.integers(0, max(1, E // 3), (L, E)).astype(np.int32)
+    x = (rng.random((L, M, E)) < 0.2).astype(np.uint8)
+    gc = torch.empty(L, M, E, dtype=torch.uint8, device=DEV)
+    gn = torch.empty(L, dtype=torch.int32, device=DEV)
+    B.ordermoe_coverage(torch.as_tensor(group).to(DEV), torch.as_tensor(x).to(DEV), L, E, M, gc, gn)
+    cov = gc.cpu().numpy()
+    for l in range(L):
+        ref = oracle.coverage(x[l], group[l], E)
+        np.testing.assert_array_equal(cov[l], ref)
+        assert gn[l].item() == int(ref.sum())
+
+
+def test_redundant_plan_at_memory_ratio_two_raises_coverage():
+    """The whole of Alg. 1 on the GPU for 32 Mixtral-shaped layers, 8 servers:
+    placement, then redundancy at memory ratio 2.0 with pi from Zipf homes;
+    coverage goes up and matches the oracle's plan."""
+    rng = np.random.default_rng(12)
+    L, E, M = 32, 8, 8
+    sim, counts = synthetic_sims(rng, L, E, 4, 0.3)
+    p = np.ones((L, E)); C = synth.capacities(M, L * E, 2.0, 12)
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a)).to(device=DEV, dtype=dt)
+    group = torch.empty(L, E, dtype=torch.int32, device=DEV)
+    ng = torch.empty(L, dtype=torch.int32, device=DEV)
+    imp = torch.empty(L, E, dtype=torch.float64, device=DEV)
+    x = torch.empty(L, M, E, dtype=torch.uint8, device=DEV)
+    used = torch.empty(M, dtype=torch.float64, device=DEV)
+    st = torch.empty(1, dtype=torch.int32, device=DEV)
+    gp, gC = t(p, torch.float64), t(C, torch.float64)
+    B.ordermoe_place(t(sim, torch.float32), t(counts, torch.int32), L, E, M, 0.5, 0.9, 0.5, 0.5, 0.5,
+                     0.5, 0.5, gp, gC, group, ng, torch.empty(L, dtype=torch.float32, device=DEV), imp,
+                     x, used, st)
+    covered0 = torch.empty(L, dtype=torch.int32, device=DEV)
+    B.ordermoe_coverage(group, x, L, E, M, None, covered0)
+    x0, used0 = x.cpu().numpy(), used.cpu().numpy()
+    pi = synth.token_shares(synth.homes(8192, M, 12, "zipf1.1"), M)
+    reps = torch.empty(M, dtype=torch.int32, device=DEV)
+    B.ordermoe_replicate(group, imp, gp, gC, t(pi, torch.float64), L, E, M, x, used, reps)
+    covered = torch.empty(L, dtype=torch.int32, device=DEV)
+    B.ordermoe_coverage(group, x, L, E, M, None, covered)
+    total = M * int(ng.sum().item())
+    before, after = covered0.sum().item() / total, covered.sum().item() / total
+    print("local group coverage: %.3f -> %.3f with %d replicas" % (before, after, int(reps.sum().item())))
+    assert st.item() == 0 and after > before
+    assert (used.cpu().numpy() <= C).all()
+    ref = oracle.replicate(group.cpu().numpy(), imp.cpu().numpy(), p, C, pi, x0, used0)
+    np.testing.assert_array_equal(x.cpu().numpy(), ref[0])
+    np.testing.assert_array_equal(reps.cpu().numpy(), ref[2])
 
 
 def test_similarity_full_size_sampled():
