@@ -64,6 +64,10 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--lookahead", type=int, default=1,
                    help="selection horizon H (Eqs. 41-43) for the decode stack; 1 = myopic")
+    p.add_argument("--memory-ratio", type=float, default=None,
+                   help="memory budget ratio of the offline plan (Section VI-G): server capacity "
+                        "over one copy of the experts; above 1 the spare memory holds replicas "
+                        "(Eqs. 32-35). Default: 1.0 for the decode stack, 2.0 for the plan")
     p.add_argument("--cpu-seconds", type=float, default=15.0,
                    help="target CPU seconds of the oracle baseline sample")
     return p.parse_args()
@@ -392,6 +396,15 @@ def timed_region(args, dist, device, fn):
     return dist.max(a.elapsed_time(b), device), clocks
 
 
+def plan_coverage(B, group, ng, x, L, E, M, device):
+    """Local group coverage (Eq. 32) of a placement: covered (server, group)
+    pairs over M * sum_l K_l."""
+    import torch
+    covered = torch.empty(L, dtype=torch.int32, device=device)
+    B.ordermoe_coverage(group, x, L, E, M, None, covered)
+    return {"coverage": round(covered.sum().item() / (M * int(ng.sum().item())), 4)}
+
+
 def run_decode(args, dist, w, device):
     """Decode stack: one step = 32 MoE layers over a batch of 128 tokens, with
     the selection state carried across layers; bound by streaming the expert
@@ -421,10 +434,20 @@ def run_decode(args, dist, w, device):
     x = torch.empty(L, M, E, dtype=torch.uint8, device=device)
     used = torch.empty(M, dtype=torch.float64, device=device)
     st = torch.empty(1, dtype=torch.int32, device=device)
+    imp = torch.empty(L, E, dtype=torch.float64, device=device)
+    ratio = 1.0 if args.memory_ratio is None else args.memory_ratio
+    pmem = torch.ones(L, E, dtype=torch.float64, device=device)
+    Cm = (torch.full((M,), L * E / M, dtype=torch.float64, device=device) if ratio == 1.0 else
+          torch.as_tensor(synth.capacities(M, L * E, ratio, seed), dtype=torch.float64).to(device))
     B.ordermoe_place(sim, counts, L, E, M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5, 0.5, 0.5,
-                     torch.ones(L, E, dtype=torch.float64, device=device),
-                     torch.full((M,), L * E / M, dtype=torch.float64, device=device),
-                     group, ng, theta, None, x, used, st)
+                     pmem, Cm, group, ng, theta, imp, x, used, st)
+    plan = plan_coverage(B, group, ng, x, L, E, M, device)
+    if ratio > 1.0:
+        pi = torch.as_tensor(synth.token_shares(home.cpu().numpy(), M), dtype=torch.float64).to(device)
+        reps = torch.empty(M, dtype=torch.int32, device=device)
+        B.ordermoe_replicate(group, imp, pmem, Cm, pi, L, E, M, x, used, reps)
+        plan.update({"replicas": int(reps.sum().item()),
+                     "coverage_after": plan_coverage(B, group, ng, x, L, E, M, device)["coverage"]})
     # transition statistics (Eq. 41) from the calibration logits the similarity
     # call leaves at the start of its workspace
     H = max(1, args.lookahead)
@@ -455,6 +478,12 @@ def run_decode(args, dist, w, device):
     code, detail = B.ordermoe_device_error()
     if code:
         raise RuntimeError("device error %d (%d)" % (code, detail))
+    # execution types of one step's decisions (untimed)
+    kinds = torch.zeros(4, dtype=torch.int32, device=device)
+    loc.copy_(home); qhat.zero_()
+    stack.step(Xs, home, loc, qhat, ys, counters=kinds)
+    exec_types = dict(zip(["local_exact", "local_sub", "remote_exact", "remote_sub"],
+                          kinds.cpu().tolist()))
     # decision time: the selection alone (router + top-k + Alg. 2) over the 32 layers
     f = lambda *sh, dt: torch.empty(*sh, dtype=dt, device=device)
     sel = [f(w.T, w.k, dt=dt) for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
@@ -483,7 +512,7 @@ def run_decode(args, dist, w, device):
         "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": w.L, "T": w.T, "d": w.d, "E": w.E, "k": w.k,
-                   "d_ff": w.dff, "M": w.M, "lookahead_H": H,
+                   "d_ff": w.dff, "M": w.M, "lookahead_H": H, "memory_ratio": ratio,
                    "l2": "inputs larger than L2: %.1f GB of expert weights" % (wbytes / 1e9)},
         "roofline": {"kernel": "whole decode step (expert weight streaming)", "bound": "hbm",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
@@ -494,6 +523,8 @@ def run_decode(args, dist, w, device):
         "gpu_launches": (8 * w.L + sum(min(H, w.L - l) > 1 for l in range(w.L))) * args.steps,
         "clocks": clocks,
         "lookahead_H": H,
+        "plan": plan,
+        "exec_types": exec_types,
         "selection_ms_per_layer": round(select_ms_per_layer, 4),
         "selection_us_per_token_layer": round(select_ms_per_layer * 1e3 / w.T, 4),
     }
@@ -519,13 +550,22 @@ def run_similarity(args, dist, w, device):
     x = torch.empty(L, w.M, E, dtype=torch.uint8, device=device)
     used = torch.empty(w.M, dtype=torch.float64, device=device)
     st = torch.empty(1, dtype=torch.int32, device=device)
+    imp = torch.empty(L, E, dtype=torch.float64, device=device)
+    reps = torch.empty(w.M, dtype=torch.int32, device=device)
+    covered = torch.empty(L, dtype=torch.int32, device=device)
     p = torch.ones(L, E, dtype=torch.float64, device=device)
-    C = torch.full((w.M,), L * E / w.M, dtype=torch.float64, device=device)
+    ratio = 2.0 if args.memory_ratio is None else args.memory_ratio
+    C = torch.as_tensor(synth.capacities(w.M, L * E, ratio, seed), dtype=torch.float64).to(device)
+    # pi_m of Eq. 33 from a non-uniform (Zipf 1.1) user-server association
+    pi = torch.as_tensor(synth.token_shares(synth.homes(65536, w.M, seed, "zipf1.1"), w.M),
+                         dtype=torch.float64).to(device)
 
     def step():
         B.ordermoe_similarity(Wr, Xcal, L, E, d, N, w.k, sim, counts, ws)
         B.ordermoe_place(sim, counts, L, E, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5,
-                         0.5, 0.5, p, C, group, ng, theta, None, x, used, st)
+                         0.5, 0.5, p, C, group, ng, theta, imp, x, used, st)
+        B.ordermoe_replicate(group, imp, p, C, pi, L, E, w.M, x, used, reps)
+        B.ordermoe_coverage(group, x, L, E, w.M, None, covered)
 
     ms, clocks = timed_region(args, dist, device, step)
     code, detail = B.ordermoe_device_error()
@@ -543,13 +583,17 @@ def run_similarity(args, dist, w, device):
         "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": L, "E": E, "d": d, "N": N, "groups": w.n_clusters,
-                   "M": w.M, "k_freq": w.k},
-        "roofline": {"kernel": "ordermoe_similarity + ordermoe_place (whole call)", "bound": "tensor",
+                   "M": w.M, "k_freq": w.k, "memory_ratio": ratio},
+        "roofline": {"kernel": "similarity + place + replicate + coverage (whole plan)", "bound": "tensor",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
                      "peak_source": "%s bf16_tflops (burst)" % pk_kind, "flop_per_step": flop},
-        "gpu_launches": 4 * args.steps,
+        # similarity 5 (logits GEMM, counts, Gram, Gram reduce, finish), place 2,
+        # replicate 1, coverage 1
+        "gpu_launches": 9 * args.steps,
         "n_groups": ng.cpu().tolist()[:3], "place_status": int(st.item()),
+        "replicas": int(reps.sum().item()),
+        "coverage": round(covered.sum().item() / (w.M * int(ng.sum().item())), 4),
         "clocks": clocks,
     }
 

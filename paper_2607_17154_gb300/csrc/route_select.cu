@@ -364,12 +364,13 @@ __global__ void __launch_bounds__(128) select_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// Alg. 2 with horizon H > 1 (Eq. 43), one warp per token, from the targets
-// topk_idx. The candidates of a slot are visited in order by the whole warp;
-// for each, lane i computes the term P(k -> k') * min(...) of Eq. 42 for the
-// next targets k' = i and i + 32 (with the deeper levels of the recursion
-// serial in the lane); the terms are then added in ascending k' by every lane
-// (shuffles), so Phi is the same fp32 value the serial definition gives.
+// Alg. 2 with horizon H > 1 (Eq. 43), one block per token, from the targets
+// topk_idx. For each slot the block lists the slot's candidates (expert,
+// server) in shared memory, then every thread takes (candidate, next target
+// k') items: the term P(k -> k') * min(...) of Eq. 42, with the deeper levels
+// of the recursion serial in the thread. Each candidate's terms are then
+// added in ascending k' (skipping P = 0, as the serial definition does), so
+// Phi is the same fp32 value; the argmin key is reduced with atomicMin.
 template <int D>
 __device__ __forceinline__ float phi_term(const uint8_t* __restrict__ tnext, size_t stride,
                                           const float* __restrict__ P, int E, int M, int a, int m,
@@ -409,125 +410,154 @@ __device__ __forceinline__ float phi_term(const uint8_t* __restrict__ tnext, siz
   return __fmul_rn(p, best);
 }
 
-template <int D>
-__device__ __forceinline__ float phi_warp(const uint8_t* tnext, size_t stride, const float* P,
-                                          int E, int M, int a, int m, int kx, float qacc,
-                                          float qbar, int lane) {
-  const float t0 = lane < E ? phi_term<D>(tnext, stride, P, E, M, a, m, kx, lane, qacc, qbar) : 0.0f;
-  const float t1 = lane + 32 < E ? phi_term<D>(tnext, stride, P, E, M, a, m, kx, lane + 32, qacc, qbar) : 0.0f;
-  float acc = 0.0f;
-  for (int kt = 0; kt < E; ++kt) {
-    const float term = __shfl_sync(0xffffffffu, kt < 32 ? t0 : t1, kt & 31);
-    if (__ldg(P + (size_t)kx * E + kt) != 0.0f) acc = __fadd_rn(acc, term);
-  }
-  return acc;
-}
-
-__device__ __forceinline__ float phi_warp_h(const Lookahead& la, const uint8_t* tab, int E, int M,
-                                            int a, int m, int kx, float qacc, float qbar, int lane) {
+__device__ __forceinline__ float phi_term_h(const Lookahead& la, const uint8_t* tab, int E, int M,
+                                            int a, int m, int kx, int kt, float qacc, float qbar) {
   switch (la.H) {
-    case 2: return phi_warp<1>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar, lane);
-    case 3: return phi_warp<2>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar, lane);
-    case 4: return phi_warp<3>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, qacc, qbar, lane);
+    case 2: return phi_term<1>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, kt, qacc, qbar);
+    case 3: return phi_term<2>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, kt, qacc, qbar);
+    case 4: return phi_term<3>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, kt, qacc, qbar);
     default: return 0.0f;
   }
 }
 
-__global__ void __launch_bounds__(128) lookahead_select_kernel(
+constexpr int kLaThreads = 128;
+constexpr int kLaMaxCand = 65 * 32;  // (target + 64 substitutes) x 32 servers
+constexpr int kLaTerms = 2048;       // (candidate, k') terms per pass
+
+struct LaSmem {
+  uint32_t code[kLaMaxCand];  // expert | server << 8 | substitute << 16
+  float cost0[kLaMaxCand];    // A(a, s, m) + Cq: Eq. 43 without Phi
+  float qn[kLaMaxCand];       // accumulated loss after this candidate (Eq. 44)
+  float terms[kLaTerms];
+  unsigned long long best;
+  int n;
+};
+
+__global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
     const int32_t* __restrict__ topk_idx, int T, int E, int k, const uint8_t* __restrict__ tab,
     Lookahead la, const uint8_t* __restrict__ home, uint8_t* __restrict__ loc,
     float* __restrict__ qhat, int32_t* __restrict__ chosen_expert,
     uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
     int32_t* __restrict__ counters) {
   __shared__ SelSmem sm;
+  __shared__ LaSmem cs;
   extern __shared__ __align__(16) float s_dyn[];
   float* s_Q = s_dyn;
   float* s_Cq = s_dyn + E * E;
+  const int t = blockIdx.x;
+  if (t >= T) return;
   if (!load_tables(tab, E, sm, s_Q, s_Cq)) return;
   __syncthreads();
   const int M = reinterpret_cast<const int32_t*>(tab)[2];
   const float qbar = reinterpret_cast<const float*>(tab)[5];
   const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
-  const int lane = threadIdx.x & 31;
-  const int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  int kind_count[4] = {0, 0, 0, 0};
-  if (t < T) {
-    const int a = home[t];
-    const int s = (loc != nullptr) ? loc[t] : a;
-    if (a >= M || s >= M) {
-      if (lane == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
-    } else {
-      const float* Aas = gA + ((size_t)a * M + s) * M;
-      float q = (qhat != nullptr) ? qhat[t] : 0.0f;
-      unsigned long long taken = 0;
+  const int tid = threadIdx.x;
+  const int a = home[t];
+  const int s = (loc != nullptr) ? loc[t] : a;
+  if (a >= M || s >= M) {
+    if (tid == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
+    return;
+  }
+  unsigned long long taken = 0;
+  for (int j = 0; j < k; ++j) {
+    const int r = topk_idx[(size_t)t * k + j];
+    if (r < 0 || r >= E) return;  // -1: a token whose logits held a NaN (reported)
+    taken |= 1ull << r;
+  }
+  const float* Aas = gA + ((size_t)a * M + s) * M;
+  const int cpp = kLaTerms / E;  // candidates per pass
+  float q = (qhat != nullptr) ? qhat[t] : 0.0f;
+  int first_server = s;
+  for (int j = 0; j < k; ++j) {
+    const int r = topk_idx[(size_t)t * k + j];
+    if (tid == 0) {
+      cs.n = 0;
+      cs.best = ~0ull;
+    }
+    __syncthreads();
+    // candidates: thread i takes the target (i = 0) or substitute i - 1
+    const int nsub = sm.nsub[r];
+    for (int ki = tid; ki <= nsub; ki += blockDim.x) {
+      const int kk = (ki == 0) ? r : sm.sublist[r * 64 + ki - 1];
+      const bool sub = (ki != 0);
+      float cq = 0.0f, qn = q;
       bool ok = true;
-      for (int j = 0; j < k; ++j) {
-        const int r = topk_idx[(size_t)t * k + j];
-        ok = ok && r >= 0 && r < E;  // -1: a token whose logits held a NaN
-        if (ok) taken |= 1ull << r;
-      }
-      int first_server = s;
-      for (int j = 0; j < (ok ? k : 0); ++j) {
-        const int r = topk_idx[(size_t)t * k + j];
-        const int nsub = sm.nsub[r];
-        unsigned long long best = ~0ull;
-        for (int ki = 0; ki <= nsub; ++ki) {
-          const int kk = (ki == 0) ? r : sm.sublist[r * 64 + ki - 1];
-          const bool sub = (ki != 0);
-          float cq = 0.0f, qn = q;
-          if (sub) {
-            if ((taken >> kk) & 1ull) continue;
-            if (!(__fadd_rn(q, s_Q[r * E + kk]) <= qbar)) continue;
-            cq = s_Cq[r * E + kk];
-            qn = __fadd_rn(q, s_Q[r * E + kk]);
-          }
-          uint32_t pm = sm.pmask[kk];
-          while (pm) {
-            const int m = __ffs(pm) - 1;
-            pm &= pm - 1;
-            float cost = __fadd_rn(__ldg(Aas + m), cq);
-            cost = __fadd_rn(cost, phi_warp_h(la, tab, E, M, a, m, kk, qn, qbar, lane));
-            const unsigned long long key =
-                (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
-                (static_cast<unsigned long long>(sub ? 1u : 0u) << 31) |
-                (static_cast<unsigned long long>(m != s ? 1u : 0u) << 30) |
-                (static_cast<unsigned long long>(m) << 8) | static_cast<unsigned long long>(kk);
-            best = key < best ? key : best;
-          }
-        }
-        int kstar, mstar, kd;
-        if (best == ~0ull) {
-          if (lane == 0) report(&g_err_route, ORDERMOE_DEV_NO_CANDIDATE, t);
-          kstar = r; mstar = s; kd = 0;
-        } else {
-          kstar = static_cast<int>(best & 0xFFu);
-          mstar = static_cast<int>((best >> 8) & 0xFFu);
-          const int sub = static_cast<int>((best >> 31) & 1u);
-          const int away = static_cast<int>((best >> 30) & 1u);
-          kd = 2 * away + sub;
-          if (sub) {
-            taken |= 1ull << kstar;
-            q = __fadd_rn(q, s_Q[r * E + kstar]);
-          }
-        }
-        if (j == 0) first_server = mstar;
-        if (lane == 0) {
-          chosen_expert[(size_t)t * k + j] = kstar;
-          chosen_server[(size_t)t * k + j] = static_cast<uint8_t>(mstar);
-          kind_out[(size_t)t * k + j] = static_cast<uint8_t>(kd);
-          kind_count[kd]++;
+      if (sub) {
+        ok = !((taken >> kk) & 1ull) && (__fadd_rn(q, s_Q[r * E + kk]) <= qbar);
+        if (ok) {
+          cq = s_Cq[r * E + kk];
+          qn = __fadd_rn(q, s_Q[r * E + kk]);
         }
       }
-      if (lane == 0 && ok && loc != nullptr) {
-        loc[t] = static_cast<uint8_t>(first_server);
-        qhat[t] = q;
+      uint32_t pm = ok ? sm.pmask[kk] : 0u;
+      int slot = atomicAdd(&cs.n, __popc(pm));
+      while (pm) {
+        const int m = __ffs(pm) - 1;
+        pm &= pm - 1;
+        cs.code[slot] = static_cast<uint32_t>(kk) | (static_cast<uint32_t>(m) << 8) |
+                        (sub ? (1u << 16) : 0u);
+        cs.cost0[slot] = __fadd_rn(__ldg(Aas + m), cq);
+        cs.qn[slot] = qn;
+        ++slot;
       }
     }
+    __syncthreads();
+    const int n = cs.n;
+    for (int base = 0; base < n; base += cpp) {
+      const int nc = min(cpp, n - base);
+      for (int i = tid; i < nc * E; i += blockDim.x) {
+        const int c = base + i / E, kt = i - (i / E) * E;
+        const uint32_t code = cs.code[c];
+        cs.terms[i] = phi_term_h(la, tab, E, M, a, static_cast<int>((code >> 8) & 0xFFu),
+                                 static_cast<int>(code & 0xFFu), kt, cs.qn[c], qbar);
+      }
+      __syncthreads();
+      for (int cl = tid; cl < nc; cl += blockDim.x) {
+        const uint32_t code = cs.code[base + cl];
+        const int kk = static_cast<int>(code & 0xFFu), m = static_cast<int>((code >> 8) & 0xFFu);
+        const unsigned sub = (code >> 16) & 1u;
+        float phi = 0.0f;
+        for (int kt = 0; kt < E; ++kt)
+          if (__ldg(la.P + (size_t)kk * E + kt) != 0.0f) phi = __fadd_rn(phi, cs.terms[cl * E + kt]);
+        const float cost = __fadd_rn(cs.cost0[base + cl], phi);
+        const unsigned long long key =
+            (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
+            (static_cast<unsigned long long>(sub) << 31) |
+            (static_cast<unsigned long long>(m != s ? 1u : 0u) << 30) |
+            (static_cast<unsigned long long>(m) << 8) | static_cast<unsigned long long>(kk);
+        atomicMin(&cs.best, key);
+      }
+      __syncthreads();
+    }
+    const unsigned long long best = cs.best;
+    int kstar, mstar, kd;
+    if (best == ~0ull) {
+      if (tid == 0) report(&g_err_route, ORDERMOE_DEV_NO_CANDIDATE, t);
+      kstar = r; mstar = s; kd = 0;
+    } else {
+      kstar = static_cast<int>(best & 0xFFu);
+      mstar = static_cast<int>((best >> 8) & 0xFFu);
+      const int sub = static_cast<int>((best >> 31) & 1u);
+      const int away = static_cast<int>((best >> 30) & 1u);
+      kd = 2 * away + sub;
+      if (sub) {
+        taken |= 1ull << kstar;
+        q = __fadd_rn(q, s_Q[r * E + kstar]);
+      }
+    }
+    if (j == 0) first_server = mstar;
+    if (tid == 0) {
+      chosen_expert[(size_t)t * k + j] = kstar;
+      chosen_server[(size_t)t * k + j] = static_cast<uint8_t>(mstar);
+      kind_out[(size_t)t * k + j] = static_cast<uint8_t>(kd);
+      if (counters != nullptr) atomicAdd(&counters[kd], 1);
+    }
+    __syncthreads();  // the candidate arrays are rewritten for the next slot
   }
-  flush_kind_counts(sm, kind_count, counters);
-  __syncthreads();
-  if (counters != nullptr && threadIdx.x < 4 && sm.kind[threadIdx.x])
-    atomicAdd(&counters[threadIdx.x], sm.kind[threadIdx.x]);
+  if (tid == 0 && loc != nullptr) {
+    loc[t] = static_cast<uint8_t>(first_server);
+    qhat[t] = q;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -789,10 +819,10 @@ static int launch_lookahead_select(const int32_t* topk_idx, int T, int E, int k,
                                    uint8_t* loc, float* qhat, int32_t* chosen_expert,
                                    uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
                                    size_t tab_smem, cudaStream_t stream) {
-  const int blocks = (T + 3) / 4;  // 4 warps = 4 tokens per block
+  if (T <= 0) return ORDERMOE_OK;
   cudaFuncSetAttribute(lookahead_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)tab_smem);
-  lookahead_select_kernel<<<blocks, 128, tab_smem, stream>>>(
+  lookahead_select_kernel<<<T, kLaThreads, tab_smem, stream>>>(
       topk_idx, T, E, k, tb, la, home, loc, qhat, chosen_expert, chosen_server, kind, counters);
   OM_LAUNCHED("lookahead_select_kernel");
   return ORDERMOE_OK;
