@@ -52,6 +52,9 @@ def lib():
             "orc_place": [_P, _P, _P, _I, _I, _I, _P, _D, _D, _P, _P],
             "orc_coverage": [_P, _P, _I, _I, _I, _P],
             "orc_replicate": [_P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P],
+            "orc_trajectory_cost": [_P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, _P, _D, _D, _P,
+                                    _P, _P, _P],
+            "orc_utility": [_P, _P, _P, _I, _D, _D, _D, _D, _P],
             "orc_transitions": [_P, _I64, _I, _I, _I, _P, _P],
             "orc_select_lookahead": [_P, _I, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P,
                                      _P, _F, _P, _P, _P, _P, _P, _P],
@@ -236,6 +239,31 @@ def replicate(group, importance, p, C, pi, placement, used):
     _check(lib().orc_replicate(_ptr(group), _ptr(importance), _ptr(p), L, E, M, _ptr(C), _ptr(pi),
                                _ptr(x), _ptr(b), _ptr(reps)), "orc_replicate")
     return x, b, reps
+
+
+def trajectory_cost(target, chosen, server, home, F, B, tau, z, c, Qtab):
+    """Edge delay / substitution loss / transfers of L layers' selection records
+    (Eqs. 13-20). target/chosen/server: [L, T, k]; home [T]; Qtab [L, E, E].
+    Returns (delay [T] f64, loss [T] f64, moves [T] i32)."""
+    target = _c(target, np.int32); chosen = _c(chosen, np.int32); server = _c(server, np.uint8)
+    home = _c(home, np.uint8); F = _c(F, np.float64); B = _c(B, np.float64)
+    tau = _c(tau, np.float64); Qtab = _c(Qtab, np.float32)
+    L, T, k = target.shape; E = Qtab.shape[-1]; M = F.shape[0]
+    assert Qtab.shape == (L, E, E)
+    d = np.empty(T, np.float64); q = np.empty(T, np.float64); n = np.empty(T, np.int32)
+    _check(lib().orc_trajectory_cost(_ptr(target), _ptr(chosen), _ptr(server), _ptr(home), L, T, k,
+                                     E, M, _ptr(F), _ptr(B), _ptr(tau), float(z), float(c),
+                                     _ptr(Qtab), _ptr(d), _ptr(q), _ptr(n)), "orc_trajectory_cost")
+    return d, q, n
+
+
+def utility(delay, delay_ref, loss, qmax, omega_T, omega_Q, kappa):
+    """Eq. 23 and Eq. 45: returns (U, Tbar, Qbar, omega_T', omega_Q')."""
+    delay = _c(delay, np.float64); delay_ref = _c(delay_ref, np.float64); loss = _c(loss, np.float64)
+    out = np.empty(5, np.float64)
+    _check(lib().orc_utility(_ptr(delay), _ptr(delay_ref), _ptr(loss), delay.shape[0], float(qmax),
+                             float(omega_T), float(omega_Q), float(kappa), _ptr(out)), "orc_utility")
+    return tuple(float(v) for v in out)
 
 
 def coverage(placement_l, group_l, K):

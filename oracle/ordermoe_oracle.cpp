@@ -541,6 +541,76 @@ int orc_replicate(const int32_t* group, const double* importance, const double* 
 }
 
 // ---------------------------------------------------------------------------
+// Edge cost of the selection records of L layers (Section III-D/E): a token
+// starts at its home server a (Eq. 36); at layer l each slot j executed on
+// server m_j pays the transfer of Eqs. 13-14 from the token's location s_l
+// when m_j != s_l, z / B[s_l][m_j] + tau[s_l][m_j], plus the compute of
+// Eq. 15, c / F[m_j]; the location after the layer is the server of slot 0
+// (Eq. 44). delay[t] = sum over layers and slots (Eqs. 16-17, one token per
+// user), loss[t] = the substitution loss Q_l(r, k) of every substituted slot
+// (Eqs. 18-20; Qtab [L][E][E], the fp32 values the selection uses), moves[t]
+// = the number of transfers. fp64, one running sum per token in (l, j) order.
+int orc_trajectory_cost(const int32_t* target, const int32_t* chosen, const uint8_t* server,
+                        const uint8_t* home, int L, int T, int k, int E, int M, const double* F,
+                        const double* B, const double* tau, double z, double c, const float* Qtab,
+                        double* delay, double* loss, int32_t* moves) {
+  for (int t = 0; t < T; ++t) {
+    int s = home[t];
+    if (s >= M) return ORC_BAD_ARG;
+    double d = 0.0, q = 0.0;
+    int n = 0;
+    for (int l = 0; l < L; ++l) {
+      int next = s;
+      for (int j = 0; j < k; ++j) {
+        const size_t i = ((size_t)l * T + t) * k + j;
+        const int r = target[i], kk = chosen[i], m = server[i];
+        if (r < 0 || r >= E || kk < 0 || kk >= E || m >= M) return ORC_BAD_ARG;
+        double trans = 0.0;
+        if (m != s) {
+          trans = z / B[s * M + m] + tau[s * M + m];
+          ++n;
+        }
+        const double comp = c / F[m];
+        d = d + (trans + comp);
+        if (kk != r) q = q + static_cast<double>(Qtab[((size_t)l * E + r) * E + kk]);
+        if (j == 0) next = m;
+      }
+      s = next;
+    }
+    delay[t] = d;
+    loss[t] = q;
+    moves[t] = n;
+  }
+  return ORC_OK;
+}
+
+// Normalised utility (Eq. 23) and weight adaptation (Eq. 45) over T users
+// (one token each): T~ = delay / delay_ref (delay_ref: the same tokens under
+// pure exact execution on the same deployment), Q~ = loss / qmax;
+// U = omega_T sum T~ + omega_Q sum Q~; Tbar, Qbar the means;
+// omega_Q' = clamp(omega_Q + kappa (Qbar - Tbar), 0, 1), omega_T' = 1 - omega_Q'.
+// out[5] = {U, Tbar, Qbar, omega_T', omega_Q'}.
+int orc_utility(const double* delay, const double* delay_ref, const double* loss, int T,
+                double qmax, double omega_T, double omega_Q, double kappa, double* out) {
+  if (T <= 0 || !(qmax > 0.0)) return ORC_BAD_ARG;
+  double st = 0.0, sq = 0.0;
+  for (int t = 0; t < T; ++t) {
+    if (!(delay_ref[t] > 0.0)) return ORC_BAD_ARG;
+    st += delay[t] / delay_ref[t];
+    sq += loss[t] / qmax;
+  }
+  const double tbar = st / T, qbar = sq / T;
+  double wq = omega_Q + kappa * (qbar - tbar);
+  wq = std::min(1.0, std::max(0.0, wq));
+  out[0] = omega_T * st + omega_Q * sq;
+  out[1] = tbar;
+  out[2] = qbar;
+  out[3] = 1.0 - wq;
+  out[4] = wq;
+  return ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
 // Expert transition statistics, Eq. 41, from calibration logits [N][L][E]:
 // for each token, every pair (k in top-kf of layer l, k' in top-kf of layer
 // l+1) counts one transition k -> k' (the paper has one target per token; with

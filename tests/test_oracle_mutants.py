@@ -60,6 +60,19 @@ MUTANTS = [
     ("Eq. 35: used memory not updated", "used[bm] += p[bl * E + bj];", ""),
     ("redundancy: ties to the later candidate", "if (bl < 0 || benefit > bb) { bl = l;",
      "if (bl < 0 || benefit >= bb) { bl = l;"),
+    ("Eq. 14: simulator transfer from the home server",
+     "trans = z / B[s * M + m] + tau[s * M + m];\n          ++n;",
+     "trans = z / B[home[t] * M + m] + tau[home[t] * M + m];\n          ++n;"),
+    ("Eq. 13: simulator latency dropped", "trans = z / B[s * M + m] + tau[s * M + m];\n          ++n;",
+     "trans = z / B[s * M + m];\n          ++n;"),
+    ("Eq. 15: simulator compute on the source server", "const double comp = c / F[m];",
+     "const double comp = c / F[s];"),
+    ("Eq. 44: simulator location from the last slot", "if (j == 0) next = m;", "next = m;"),
+    ("Eq. 19: loss of the substitute's own row", "Qtab[((size_t)l * E + r) * E + kk]",
+     "Qtab[((size_t)l * E + kk) * E + r]"),
+    ("Eq. 23: weights swapped", "out[0] = omega_T * st + omega_Q * sq;", "out[0] = omega_Q * st + omega_T * sq;"),
+    ("Eq. 45: direction flipped", "omega_Q + kappa * (qbar - tbar)", "omega_Q + kappa * (tbar - qbar)"),
+    ("Eq. 45: no projection", "wq = std::min(1.0, std::max(0.0, wq));", ""),
     ("Eq. 41: transitions of the same layer", "topk(logits + (n * L + l + 1) * E, nxt);",
      "topk(logits + (n * L + l) * E, nxt);"),
     ("Eq. 42: transition from the target, not the executed expert",

@@ -765,6 +765,80 @@ def test_replicate_with_ample_memory_covers_every_group_everywhere(orc):
     assert int(reps.sum()) == uncovered
 
 
+def _sim_params():
+    # dyadic values, so every delay below is exact in fp64; B and tau asymmetric
+    F = np.array([4.0, 2.0, 8.0])
+    B = np.array([[1.0, 2.0, 8.0], [4.0, 1.0, 1.0], [16.0, 2.0, 1.0]])
+    tau = np.array([[0.0, 0.5, 0.25], [0.25, 0.0, 2.0], [0.125, 1.0, 0.0]])
+    return F, B, tau
+
+
+def test_trajectory_cost_hand_example(orc):
+    # Eqs. 13-20 on two layers. Token 0 (home 0): layer 1 slot 0 on server 1
+    # (transfer 8/2 + 0.5, compute 1/2), slot 1 substitutes expert 3 for 2 on
+    # server 0 (compute 1/4); the token is then on server 1 (slot 0). Layer 2:
+    # slot 0 on server 1 (compute 1/2), slot 1 on server 2 (transfer 8/1 + 2,
+    # compute 1/8). Token 1 (home 2) stays on server 2 with exact experts.
+    F, B, tau = _sim_params()
+    E, L, T, k = 4, 2, 2, 2
+    target = np.array([[[1, 2], [0, 1]], [[0, 3], [2, 3]]], np.int32)
+    chosen = np.array([[[1, 3], [0, 1]], [[0, 3], [2, 3]]], np.int32)
+    server = np.array([[[1, 0], [2, 2]], [[1, 2], [2, 2]]], np.uint8)
+    home = np.array([0, 2], np.uint8)
+    Qtab = np.zeros((L, E, E), np.float32); Qtab[0, 2, 3] = 0.125; Qtab[1, 0, 3] = 0.5
+    d, q, n = orc.trajectory_cost(target, chosen, server, home, F, B, tau, 8.0, 1.0, Qtab)
+    assert d[0] == (4.5 + 0.5 + 0.25) + (0.5 + 10.0 + 0.125)
+    assert d[1] == 4 * 0.125
+    assert q.tolist() == [0.125, 0.0] and n.tolist() == [2, 0]
+
+
+def test_trajectory_cost_agrees_with_the_selection_cost_table(orc):
+    # Eq. 37's delay term, built by orc_tables from the same server parameters,
+    # equals omega_T * (Eqs. 13-15 delay) / d_ref(a) for each slot of a
+    # one-layer trajectory that starts at home (up to the tables' fp32 rounding).
+    rng = np.random.default_rng(7)
+    E, M, k, T = 8, 4, 2, 200
+    F = rng.uniform(20e12, 110e12, M)
+    B = rng.uniform(1e8, 1.25e9, (M, M)); tau = rng.uniform(2e-4, 2e-2, (M, M))
+    np.fill_diagonal(tau, 0.0)
+    z, c, wT = 8192.0, 3.5e8, 0.5
+    sim = np.eye(E, dtype=np.float32); group = np.arange(E, dtype=np.int32)
+    x = (rng.random((M, E)) < 0.5).astype(np.uint8); x[0] = 1
+    tab = orc.tables(sim, group, x, 0.5, 0.1, F, B, tau, z, c, wT, 0.5)
+    idx, _ = orc.topk(rng.standard_normal((T, E)).astype(np.float32), k)
+    home = rng.integers(0, M, T).astype(np.uint8)
+    ch, sv, _, _, _ = orc.select(idx, tab, home, home.copy(), np.zeros(T, np.float32))
+    d, q, n = orc.trajectory_cost(idx[None], ch[None], sv[None], home, F, B, tau, z, c,
+                                  tab.Qtab[None])
+    A = tab.A.reshape(M, M, M)
+    for t in range(T):
+        a = home[t]
+        want = sum(float(A[a, a, m]) for m in sv[t])
+        np.testing.assert_allclose(wT * d[t] / (c / F[a]), want, rtol=1e-6)
+        assert n[t] == int((sv[t] != a).sum()) and q[t] == 0.0
+
+
+def test_utility_and_weight_adaptation_closed_forms(orc):
+    T = 8
+    d = np.full(T, 3.0); q = np.full(T, 0.25)
+    # delay equal to the exact-execution reference, half the budget used
+    U, tb, qb, wT, wQ = orc.utility(d, d, q, 0.5, 0.75, 0.25, 0.125)
+    assert (tb, qb) == (1.0, 0.5)
+    assert U == 0.75 * 8 + 0.25 * 4
+    assert wQ == 0.25 + 0.125 * (0.5 - 1.0) and wT == 1.0 - wQ
+    # the projection onto [0, 1]
+    assert orc.utility(d, d, q, 0.5, 0.5, 0.5, 4.0)[4] == 0.0
+    assert orc.utility(d, 2 * d, 4 * q, 0.5, 0.5, 0.5, 4.0)[4] == 1.0
+    # random values against an exactly rounded sum
+    import math
+    rng = np.random.default_rng(3)
+    d = rng.uniform(1, 3, 500); r = rng.uniform(1, 2, 500); q = rng.uniform(0, 0.1, 500)
+    U, tb, qb, wT, wQ = orc.utility(d, r, q, 0.1, 0.6, 0.4, 0.05)
+    st = math.fsum(d / r); sq = math.fsum(q / 0.1)
+    np.testing.assert_allclose([U, tb, qb], [0.6 * st + 0.4 * sq, st / 500, sq / 500], rtol=1e-12)
+    np.testing.assert_allclose(wQ, 0.4 + 0.05 * (sq / 500 - st / 500), rtol=1e-12)
+
+
 def test_group_threshold_is_strict_and_ties_go_to_the_earlier_dominant(orc):
     cnt = np.array([3, 2, 1], np.int32)            # visiting order 0, 1, 2
     # Sim(1, 0) == theta: Eq. 24 needs max Sim < theta for a new dominant, so 1 joins 0
