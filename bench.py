@@ -405,6 +405,87 @@ def plan_coverage(B, group, ng, x, L, E, M, device):
     return {"coverage": round(covered.sum().item() / (M * int(ng.sum().item())), 4)}
 
 
+def edge_cost_windows(args, w, device, layers, Xs, home, tabs, stride, P, H, sim, group, x, theta,
+                      sp, windows=3, kappa=0.1):
+    """Untimed: the edge cost (Eqs. 13-20) of one step's decisions over the
+    layers, the same for the exact-only decisions on the same deployment
+    (substitution off), the utility (Eq. 23), and `windows` rounds of weight
+    adaptation (Eq. 45), each rebuilding the tables with the new weights."""
+    import torch
+    from paper_2607_17154_gb300 import binding as B
+    L, T, E, M, k = w.L, w.T, w.E, w.M, w.k
+    rec = [torch.empty(L, T, k, dtype=dt, device=device) for dt in (torch.int32, torch.int32, torch.uint8)]
+    wtmp = torch.empty(T, k, device=device)
+    ktmp = torch.empty(T, k, dtype=torch.uint8, device=device)
+    loc = torch.empty_like(home)
+    qhat = torch.empty(T, device=device)
+    f64 = lambda a: torch.as_tensor(a, dtype=torch.float64).to(device)
+    gF, gB, gt = f64(sp.F), f64(sp.B), f64(sp.tau)
+    th = theta.cpu().tolist()
+
+    def build(buf, omega_T, omega_Q, exact=False):
+        for l in range(L):
+            B.ordermoe_build_tables(sim[l], group[l], x[l], 2.0 if exact else th[l], w.qbar, gF, gB,
+                                    gt, sp.z, sp.c, omega_T, omega_Q, buf[l * stride:(l + 1) * stride])
+
+    def select_pass(buf):
+        loc.copy_(home); qhat.zero_()
+        for l in range(L):
+            Hl = min(H, L - l)
+            B.ordermoe_route_select_lookahead(Xs[l], layers[l]["W_r"], None, T, E, w.d, k, 1,
+                                              buf[l * stride:], stride, Hl,
+                                              P[l:l + Hl - 1].contiguous() if Hl > 1 else None,
+                                              home, loc, qhat, None, rec[0][l], wtmp, rec[1][l],
+                                              rec[2][l], ktmp)
+
+    def cost(buf):
+        d = torch.empty(T, dtype=torch.float64, device=device)
+        q = torch.empty(T, dtype=torch.float64, device=device)
+        n = torch.empty(T, dtype=torch.int32, device=device)
+        B.ordermoe_trajectory_cost(rec[0], rec[1], rec[2], home, L, T, k, E, buf, stride, M, gF, gB,
+                                   gt, sp.z, sp.c, d, q, n)
+        return d, q, n
+
+    exact_tabs = torch.zeros_like(tabs)
+    build(exact_tabs, sp.omega_T, sp.omega_Q, exact=True)
+    select_pass(exact_tabs)
+    dref, _, nref = cost(exact_tabs)
+    select_pass(tabs)
+    out = torch.empty(5, dtype=torch.float64, device=device)
+    stream = torch.cuda.current_stream(device)
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    ev[0].record(stream)
+    d, q, n = cost(tabs)
+    B.ordermoe_utility(d, dref, q, T, w.qbar, sp.omega_T, sp.omega_Q, kappa, out)
+    ev[1].record(stream)
+    torch.cuda.synchronize(device)
+    first = out.cpu().tolist()
+    res = {
+        "mean_delay_ms": round(d.mean().item() * 1e3, 4),
+        "mean_delay_exact_only_ms": round(dref.mean().item() * 1e3, 4),
+        "mean_loss": round(q.mean().item(), 5), "qbar": w.qbar,
+        "transfers_per_1k_tokens": round(n.sum().item() * 1000.0 / T, 1),
+        "transfers_per_1k_tokens_exact_only": round(nref.sum().item() * 1000.0 / T, 1),
+        "traffic_bytes_per_1k_tokens": round(n.sum().item() * sp.z * 1000.0 / T, 1),
+        "U": round(first[0], 4), "Tbar": round(first[1], 4), "Qbar": round(first[2], 4),
+        "cost_and_utility_us": round(ev[0].elapsed_time(ev[1]) * 1e3, 1),
+    }
+    # adaptation windows: each prices one step under the current weights
+    wT, wQ = first[3], first[4]
+    trace = [[sp.omega_T, round(first[1], 4), round(first[2], 4)]]
+    work = torch.zeros_like(tabs)
+    for _ in range(windows):
+        build(work, wT, wQ)
+        select_pass(work)
+        d, q, n = cost(work)
+        B.ordermoe_utility(d, dref, q, T, w.qbar, wT, wQ, kappa, out)
+        o = out.cpu().tolist()
+        trace.append([round(wT, 4), round(o[1], 4), round(o[2], 4)])
+        wT, wQ = o[3], o[4]
+    res["adaptation"] = {"kappa": kappa, "omega_T_Tbar_Qbar_per_window": trace}
+    return res
+
+
 def run_decode(args, dist, w, device):
     """Decode stack: one step = 32 MoE layers over a batch of 128 tokens, with
     the selection state carried across layers; bound by streaming the expert
@@ -501,6 +582,8 @@ def run_decode(args, dist, w, device):
     ev[1].record(stream)
     torch.cuda.synchronize(device)
     select_ms_per_layer = ev[0].elapsed_time(ev[1]) / (5 * L)
+    edge = edge_cost_windows(args, w, device, layers, Xs, home, tabs, stride, P, H, sim, group, x,
+                             theta, sp)
     step_s = ms / args.steps / 1e3
     wbytes = 3.0 * w.E * w.d * w.dff * 2 * w.L
     pk, pk_kind = peaks()
@@ -525,6 +608,7 @@ def run_decode(args, dist, w, device):
         "lookahead_H": H,
         "plan": plan,
         "exec_types": exec_types,
+        "edge": edge,
         "selection_ms_per_layer": round(select_ms_per_layer, 4),
         "selection_us_per_token_layer": round(select_ms_per_layer * 1e3 / w.T, 4),
     }

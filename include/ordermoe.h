@@ -50,7 +50,7 @@ enum {
   ORDERMOE_DEV_BAD_INDEX = 2,     /* an expert/server index out of range       */
   ORDERMOE_DEV_NO_CANDIDATE = 3,  /* selection: target expert placed nowhere   */
   ORDERMOE_DEV_WAIT_TIMEOUT = 4,  /* a bounded pipeline wait ran out           */
-  ORDERMOE_DEV_BAD_VALUE = 5      /* redundancy: a memory demand p <= 0 or NaN */
+  ORDERMOE_DEV_BAD_VALUE = 5      /* a memory demand p or a reference delay <= 0 */
 };
 
 #define ORDERMOE_MAX_EXPERTS 64
@@ -390,6 +390,44 @@ int ordermoe_replicate(const int32_t* group, const double* importance, const dou
  *   (nullable), covered [L] i32 out (nullable). */
 int ordermoe_coverage(const int32_t* group, const uint8_t* placement, int L, int E, int M,
                       uint8_t* cover, int32_t* covered, ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Edge cost of L layers' selection records (Section III-D/E). Servers are the
+ * logical placement map; the delays are the model's, not this GPU's. Token t
+ * starts at home[t] (Eq. 36); at layer l, slot j executed on server m pays
+ *   the transfer z / B[s][m] + tau[s][m] when m != s, s the token's location
+ *   (Eqs. 13-14), and the compute c / F[m] (Eq. 15);
+ * the location after the layer is the server of slot 0 (Eq. 44). A slot whose
+ * executed expert differs from its target adds Q_l(target, executed), the
+ * fp32 loss table of layer l's tables (Eq. 18), to the loss (Eqs. 19-20).
+ *   target, chosen_expert [L][T][k] i32, chosen_server [L][T][k] u8, home [T] u8;
+ *   tables: L layers' selection tables, tables_stride bytes apart (only Qtab
+ *   is read); F [M] flop/s, B [M][M] bytes/s (row = source), tau [M][M] s,
+ *   z bytes per transfer, c flop per expert execution (all f64, device);
+ *   delay [T] f64 out (s, Eq. 17 with one token per user), loss [T] f64 out,
+ *   moves [T] i32 out (transfers). fp64, one running sum per token in
+ *   (layer, slot) order. An index out of range sets ORDERMOE_DEV_BAD_INDEX
+ *   (detail: the token) and leaves that token's outputs unwritten. */
+int ordermoe_trajectory_cost(const int32_t* target, const int32_t* chosen_expert,
+                             const uint8_t* chosen_server, const uint8_t* home, int L, int T, int k,
+                             int E, const void* tables, size_t tables_stride, int M,
+                             const double* F, const double* B, const double* tau, double z,
+                             double c, double* delay, double* loss, int32_t* moves,
+                             ordermoe_stream_t stream);
+
+/* Normalised utility (Eq. 23) and weight adaptation (Eq. 45) over T users of
+ * one token each: T~ = delay / delay_ref (delay_ref: the same tokens under pure
+ * exact execution on the same deployment), Q~ = loss / qmax;
+ *   U = omega_T sum T~ + omega_Q sum Q~, Tbar = mean T~, Qbar = mean Q~,
+ *   omega_Q' = clamp(omega_Q + kappa (Qbar - Tbar), 0, 1), omega_T' = 1 - omega_Q'.
+ * out [5] f64 device: {U, Tbar, Qbar, omega_T', omega_Q'}. fp64 sums in a fixed
+ * order (strided per thread, then a fixed tree). A delay_ref <= 0 sets
+ * ORDERMOE_DEV_BAD_VALUE and the token is skipped. The caller rebuilds the
+ * selection tables with the new weights (ordermoe_build_tables) once per
+ * observation window. */
+int ordermoe_utility(const double* delay, const double* delay_ref, const double* loss, int T,
+                     double qmax, double omega_T, double omega_Q, double kappa, double* out,
+                     ordermoe_stream_t stream);
 
 #ifdef __cplusplus
 }

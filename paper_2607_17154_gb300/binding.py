@@ -46,6 +46,9 @@ _SIGNATURES = {
                         _P, _P, _P, _P, _SZ, _P], _I),
     "ordermoe_replicate": ([_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P], _I),
     "ordermoe_coverage": ([_P, _P, _I, _I, _I, _P, _P, _P], _I),
+    "ordermoe_trajectory_cost": ([_P, _P, _P, _P, _I, _I, _I, _I, _P, _SZ, _I, _P, _P, _P, _D, _D,
+                                  _P, _P, _P, _P], _I),
+    "ordermoe_utility": ([_P, _P, _P, _I, _D, _D, _D, _D, _P, _P], _I),
     "ordermoe_place_workspace_bytes": ([_I, _I], _SZ),
     "ordermoe_expert_gate_up": ([_P, _P, _I, _P, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_expert_down": ([_P, _P, _I, _P, _I, _I, _I, _P, _P], _I),
@@ -267,6 +270,29 @@ def ordermoe_coverage(group, placement, L, E, M, cover=None, covered=None, strea
     _dt(cover, torch.uint8, "cover"); _dt(covered, torch.int32, "covered")
     _check("ordermoe_coverage", lib().ordermoe_coverage(_ptr(group), _ptr(placement), L, E, M,
                                                         _ptr(cover), _ptr(covered), _stream(stream)))
+
+
+def ordermoe_trajectory_cost(target, chosen_expert, chosen_server, home, L, T, k, E, tables,
+                             tables_stride, M, F, B, tau, z, c, delay, loss, moves, stream=None):
+    """Edge delay, substitution loss and transfers of L layers' records (Eqs. 13-20)."""
+    _dt(target, torch.int32, "target"); _dt(chosen_expert, torch.int32, "chosen_expert")
+    _dt(chosen_server, torch.uint8, "chosen_server"); _dt(home, torch.uint8, "home")
+    for n, v in (("F", F), ("B", B), ("tau", tau), ("delay", delay), ("loss", loss)):
+        _dt(v, torch.float64, n)
+    _dt(moves, torch.int32, "moves")
+    _check("ordermoe_trajectory_cost", lib().ordermoe_trajectory_cost(
+        _ptr(target), _ptr(chosen_expert), _ptr(chosen_server), _ptr(home), L, T, k, E, _ptr(tables),
+        int(tables_stride), M, _ptr(F), _ptr(B), _ptr(tau), float(z), float(c), _ptr(delay),
+        _ptr(loss), _ptr(moves), _stream(stream)))
+
+
+def ordermoe_utility(delay, delay_ref, loss, T, qmax, omega_T, omega_Q, kappa, out, stream=None):
+    """Eq. 23 and Eq. 45 into out [5] f64: U, Tbar, Qbar, omega_T', omega_Q'."""
+    for n, v in (("delay", delay), ("delay_ref", delay_ref), ("loss", loss), ("out", out)):
+        _dt(v, torch.float64, n)
+    _check("ordermoe_utility", lib().ordermoe_utility(
+        _ptr(delay), _ptr(delay_ref), _ptr(loss), T, float(qmax), float(omega_T), float(omega_Q),
+        float(kappa), _ptr(out), _stream(stream)))
 
 
 def ordermoe_expert_gate_up(X_perm, offsets, R, W1, W3, E, d, dff, H, stream=None):
