@@ -668,13 +668,15 @@ def run_similarity(args, dist, w, device):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": L, "E": E, "d": d, "N": N, "groups": w.n_clusters,
                    "M": w.M, "k_freq": w.k, "memory_ratio": ratio},
-        "roofline": {"kernel": "similarity + place + replicate + coverage (whole plan)", "bound": "tensor",
+        "roofline": {"kernel": "similarity (tcgen05 logits + Gram) + place + replicate + coverage (whole plan)",
+                     "bound": "tensor",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
                      "peak_source": "%s bf16_tflops (burst)" % pk_kind, "flop_per_step": flop},
-        # similarity 5 (logits GEMM, counts, Gram, Gram reduce, finish), place 2,
+        # similarity 4 on the tensor-core path (logits with fused counts, Gram,
+        # Gram reduce, finish; E in {8, 16, 32, 64}, L E <= 4096) else 5, place 2,
         # replicate 1, coverage 1
-        "gpu_launches": 9 * args.steps,
+        "gpu_launches": ((4 if E in (8, 16, 32, 64) and L * E <= 4096 else 5) + 4) * args.steps,
         "n_groups": ng.cpu().tolist()[:3], "place_status": int(st.item()),
         "replicas": int(reps.sum().item()),
         "coverage": round(covered.sum().item() / (w.M * int(ng.sum().item())), 4),

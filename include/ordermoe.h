@@ -296,8 +296,9 @@ int ordermoe_layer_forward(const ordermoe_layer_desc* layer, int T, const uint16
  *   sim      [L][E][E] f32 out;  counts [L][E] i32 out
  *   workspace  device scratch of ordermoe_similarity_workspace_bytes(L,E,N)
  *              bytes, 256-byte aligned (holds H in fp32 and partial Grams)
- * Shapes: d % 64 == 0, 1 <= k_freq <= E <= 64. Gram partial sums are reduced
- * in a fixed order: results are deterministic. */
+ * Shapes: d % 64 == 0, 1 <= k_freq <= E <= 64, 1 <= N <= 65535 * 1024, L <=
+ * 65535. Gram partial sums are reduced in a fixed order: results are
+ * deterministic. */
 size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N);
 int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d, int64_t N,
                         int k_freq, float* sim, int32_t* counts, void* workspace,
@@ -334,7 +335,9 @@ int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq, in
  *            dominant's creation order;
  *   importance I = alpha_f f + alpha_r rho (Eqs. 27-28);
  *   placement (Eqs. 29-31): experts by (p desc, I desc, index asc), feasible
- *            servers b_m + p <= C_m, score lambda1 b_m / C_m + lambda2 eta,
+ *            servers b_m + p <= C_m, score lambda1 b_m / C_m + lambda2 eta
+ *            (lambda1, lambda2 >= 0, p >= 0 and C_m > 0 finite; a negative
+ *            or NaN score or a bad C_m sets ORDERMOE_DEV_BAD_VALUE),
  *            lowest score (ties: lower m); experts with no feasible server go,
  *            after the layer, to the server with the most free memory. The
  *            used memory b_m accumulates over the layers.
@@ -355,6 +358,13 @@ int ordermoe_place(const float* sim, const int32_t* counts, int L, int E, int M,
                    int32_t* group, int32_t* n_groups, float* theta, double* importance,
                    uint8_t* placement, double* used, int32_t* status, void* workspace,
                    size_t workspace_bytes, ordermoe_stream_t stream);
+
+/* Self-test of the quotient the placement's scores use (no counterpart in the
+ * paper): out[i] = a[i] / b[i] rounded to nearest, computed as the placement
+ * computes b_m / C_m (a reciprocal and Markstein's correction step).
+ * a, b, out: [n] f64 device. For tests that compare it with IEEE division. */
+int ordermoe_selftest_div_rn(const double* a, const double* b, double* out, int64_t n,
+                             ordermoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
  * Importance-aware redundant deployment (Section IV-C, Eqs. 32-35; Alg. 1

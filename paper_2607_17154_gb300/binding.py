@@ -49,6 +49,7 @@ _SIGNATURES = {
     "ordermoe_trajectory_cost": ([_P, _P, _P, _P, _I, _I, _I, _I, _P, _SZ, _I, _P, _P, _P, _D, _D,
                                   _P, _P, _P, _P], _I),
     "ordermoe_utility": ([_P, _P, _P, _I, _D, _D, _D, _D, _P, _P], _I),
+    "ordermoe_selftest_div_rn": ([_P, _P, _P, _I64, _P], _I),
     "ordermoe_place_workspace_bytes": ([_I, _I], _SZ),
     "ordermoe_expert_gate_up": ([_P, _P, _I, _P, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_expert_down": ([_P, _P, _I, _P, _I, _I, _I, _P, _P], _I),
@@ -293,6 +294,14 @@ def ordermoe_utility(delay, delay_ref, loss, T, qmax, omega_T, omega_Q, kappa, o
     _check("ordermoe_utility", lib().ordermoe_utility(
         _ptr(delay), _ptr(delay_ref), _ptr(loss), T, float(qmax), float(omega_T), float(omega_Q),
         float(kappa), _ptr(out), _stream(stream)))
+
+
+def ordermoe_selftest_div_rn(a, b, out, stream=None):
+    """out = a / b as the placement computes its load ratios (f64 device tensors)."""
+    for n, v in (("a", a), ("b", b), ("out", out)):
+        _dt(v, torch.float64, n)
+    _check("ordermoe_selftest_div_rn", lib().ordermoe_selftest_div_rn(
+        _ptr(a), _ptr(b), _ptr(out), a.numel(), _stream(stream)))
 
 
 def ordermoe_expert_gate_up(X_perm, offsets, R, W1, W3, E, d, dff, H, stream=None):

@@ -12,6 +12,7 @@ int read_clear_err_dispatch(unsigned long long* out);
 int read_clear_err_gemm(unsigned long long* out);
 int read_clear_err_sim(unsigned long long* out);
 int read_clear_err_cost(unsigned long long* out);
+int read_clear_err_simtc(unsigned long long* out);
 int selftest_wait_timeout(uint64_t limit_ns, cudaStream_t stream);
 
 static thread_local char t_msg[512] = "";
@@ -56,13 +57,14 @@ extern "C" int ordermoe_set_wait_limit_ns(uint64_t limit_ns) {
 extern "C" int ordermoe_device_error(int* code, int* detail) {
   if (!code) return fail(ORDERMOE_ERR_INVALID_ARG, "device_error: null code");
   OM_CUDA(cudaDeviceSynchronize());
-  unsigned long long words[5] = {0, 0, 0, 0, 0};
+  unsigned long long words[6] = {0, 0, 0, 0, 0, 0};
   int rc;
   if ((rc = read_clear_err_route(&words[0]))) return rc;
   if ((rc = read_clear_err_dispatch(&words[1]))) return rc;
   if ((rc = read_clear_err_gemm(&words[2]))) return rc;
   if ((rc = read_clear_err_sim(&words[3]))) return rc;
   if ((rc = read_clear_err_cost(&words[4]))) return rc;
+  if ((rc = read_clear_err_simtc(&words[5]))) return rc;
   *code = 0;
   if (detail) *detail = 0;
   for (unsigned long long w : words) {

@@ -1,0 +1,587 @@
+// Offline similarity on the tensor cores (Section III-B, Eqs. 3-5; Alg. 1
+// lines 3-5) for E in {8, 16, 32, 64}:
+//   sim_logits_kernel<E>: H = X_cal W^T for the L routers stacked (W rows =
+//     L * E), one 128-token x 256-logit tile per step of a persistent loop
+//     (TMA ring, tcgen05.mma, two TMEM accumulators, as in the expert FFN).
+//     The epilogue writes H in fp32, token-major (the workspace contract),
+//     writes H^T as two bf16 planes, hi = bf16(h) and lo = bf16(h - hi),
+//     expert-major so that the Gram reads both K-major, and counts each
+//     token's top-k_freq experts of every layer (Eq. 5) in a shared-memory
+//     histogram.
+//   gram_tc_kernel: partial Grams of 128 consecutive rows of H^T (128 / E
+//     layers) over a range of tokens, D = (hi + lo)(hi + lo)^T in fp32 from
+//     four tcgen05 MMAs per K step (hi hi, hi lo, lo hi, lo lo); the epilogue
+//     keeps the diagonal blocks (rows and columns of the same layer: Eq. 4's
+//     inner products). The partials are then reduced in fp64 in a fixed order.
+// Every wait is bounded; a wait that runs out reports ORDERMOE_DEV_WAIT_TIMEOUT,
+// stops the other roles, drains the copies and MMAs in flight and returns.
+#include <mutex>
+
+#include "common.cuh"
+
+namespace om {
+
+namespace gg {
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_fn();
+}  // namespace gg
+
+static __device__ unsigned long long g_err_simtc = 0;
+
+int read_clear_err_simtc(unsigned long long* out) {
+  unsigned long long zero = 0;
+  OM_CUDA(cudaMemcpyFromSymbol(out, g_err_simtc, sizeof(*out)));
+  OM_CUDA(cudaMemcpyToSymbol(g_err_simtc, &zero, sizeof(zero)));
+  return ORDERMOE_OK;
+}
+
+namespace sg {
+
+constexpr int BM = 128;
+constexpr int BN = 256;
+constexpr int BK = 64;  // bf16 elements = one 128-byte swizzled row
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int BOX_BYTES = 128 * BK * 2;
+constexpr int STAGE_BYTES = A_BYTES + 2 * BOX_BYTES;
+constexpr int THREADS = 192;    // Gram: TMA, MMA, 4 epilogue warps
+constexpr int L_EPI_WARPS = 16;  // logits epilogue: four warps per TMEM lane quarter
+constexpr int L_THREADS = 64 + 32 * L_EPI_WARPS;  // + TMA and MMA warps
+constexpr int TMEM_COLS = 512;
+constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
+constexpr int MAX_HIST = 4096;  // L * E counters in shared memory
+
+constexpr int G_STAGES = 6;
+constexpr int G_STAGE_BYTES = 2 * BOX_BYTES;  // hi and lo tiles, 128 rows x 64 tokens
+constexpr int G_TMEM_COLS = 128;
+constexpr uint32_t G_IDESC = idesc_bf16_f32(128, 128);
+
+struct LSmem {
+  uint64_t full[STAGES];
+  uint64_t empty[STAGES];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+  int zero;
+};
+constexpr int L_SMEM_FIXED = STAGES * STAGE_BYTES + 1024 + static_cast<int>(sizeof(LSmem));
+
+struct GSmem {
+  uint64_t full[G_STAGES];
+  uint64_t empty[G_STAGES];
+  uint64_t tfull;
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+  int zero;
+};
+constexpr int G_SMEM_BYTES = G_STAGES * G_STAGE_BYTES + 1024 + static_cast<int>(sizeof(GSmem));
+
+struct LArgs {
+  int N;            // calibration tokens (rows of X)
+  int C;            // L * E logit columns
+  int K;            // d
+  int n_tiles;      // 256-column slices
+  int L;
+  int kf;           // k_freq of Eq. 5
+  float* H;         // [N][C] fp32
+  uint16_t* hi;     // [C][ldT] bf16
+  uint16_t* lo;     // [C][ldT] bf16
+  int ldT;
+  int32_t* counts;  // [C] (added to)
+  uint64_t limit_ns;
+};
+
+struct GArgs {
+  int R;            // L * E rows of H^T
+  int E;
+  int kblocks;      // 64-token steps over all tokens
+  int kb_per_split;
+  int nsplit;
+  float* gpart;     // [L][nsplit][64][64]
+  uint64_t limit_ns;
+};
+
+// larger logit first, equal logits by lower index (the rank order of Eq. 5's
+// top-k): each pass keeps the first unused maximum (strict >, from -inf), so
+// finite logits rank exactly as that order says.
+template <int E>
+__device__ __forceinline__ void count_topk(const float (&x)[E], int kf, int* hist_row) {
+  unsigned long long used = 0;
+  for (int j = 0; j < kf; ++j) {
+    int best = -1;
+    float bv = -INFINITY;
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const bool take = !(used & (1ull << e)) && x[e] > bv;
+      best = take ? e : best;
+      bv = take ? x[e] : bv;
+    }
+    if (best < 0) return;
+    used |= 1ull << best;
+    atomicAdd(&hist_row[best], 1);
+  }
+}
+
+template <int E>
+__global__ void __launch_bounds__(L_THREADS, 1)
+    sim_logits_kernel(const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapW,
+                      LArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* tiles = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  LSmem& s = *reinterpret_cast<LSmem*>(tiles + STAGES * STAGE_BYTES);
+  int* hist = reinterpret_cast<int*>(tiles + STAGES * STAGE_BYTES + sizeof(LSmem));
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+  for (int i = tid; i < args.C; i += blockDim.x) hist[i] = 0;
+  if (tid == 0) {
+    for (int i = 0; i < STAGES; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.empty[i], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&s.tfull[i], 1);
+      mbar_init(&s.tempty[i], 32 * L_EPI_WARPS);
+    }
+    mbar_init(&s.drain, 1);
+    s.abort = 0;
+    s.zero = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&mapX);
+    tma_prefetch_map(&mapW);
+  }
+  if (warp == 1) {
+    tmem_alloc(&s.tmem_base, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = s.tmem_base;
+  const int total = ((args.N + BM - 1) / BM) * args.n_tiles;
+  const int kblocks = args.K / BK;
+  volatile int* abort = &s.abort;
+  uint32_t issued_mask = 0, last_phase_bits = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x) {
+        const int mt = tile / args.n_tiles, n = tile - mt * args.n_tiles;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
+            if (!*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 11);
+            *abort = 1;
+            break;
+          }
+          uint8_t* sa = tiles + stage * STAGE_BYTES;
+          mbar_arrive_expect_tx(&s.full[stage], STAGE_BYTES);
+          tma_load_2d(sa, &mapX, &s.full[stage], kb * BK, mt * BM);
+          tma_load_2d(sa + A_BYTES, &mapW, &s.full[stage], kb * BK, n * BN);
+          tma_load_2d(sa + A_BYTES + BOX_BYTES, &mapW, &s.full[stage], kb * BK, n * BN + 128);
+          issued_mask |= 1u << stage;
+          last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x, ++it) {
+        const int slot = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!mbar_wait(&s.tempty[slot], acc_phase ^ 1u, args.limit_ns, abort)) {
+          if (!*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 12);
+          *abort = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + slot * BN;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(&s.full[stage], phase, args.limit_ns, abort)) {
+            if (!*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 13);
+            *abort = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(tiles + stage * STAGE_BYTES);
+          const uint32_t b0 = a0 + A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_bf16(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
+                     IDESC, (kb | kk) != 0 ? 1u : 0u);
+          mma_issued = true;
+          mma_commit(&s.empty[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+        }
+        if (!ok) break;
+        mma_commit(&s.tfull[slot]);
+      }
+    }
+  } else {
+    // epilogue: warps 2..17; warp w reads TMEM lane quarter w % 4 (thread = one
+    // token) and the 64-column quarter (w - 2) / 4 of the tile
+    const int q = warp & 3;
+    const int part = (warp - 2) >> 2;
+    const int lrow = q * 32 + lane;
+    int it = 0;
+    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+      if (__any_sync(0xffffffffu, *abort != 0)) break;
+      const int slot = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      const bool ok = __all_sync(0xffffffffu, mbar_wait(&s.tfull[slot], acc_phase, args.limit_ns, abort));
+      if (!ok) {
+        if (lane == 0 && !*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 14);
+        *abort = 1;
+        break;
+      }
+      tc_fence_after();
+      const int mt = tile / args.n_tiles, n = tile - mt * args.n_tiles;
+      const int row = mt * BM + lrow;
+      const bool valid = row < args.N;
+      const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
+      float* orow = args.H + (size_t)row * args.C;
+      float prev[32];  // E == 64: the first half of a layer's logits
+#pragma unroll 1
+      for (int c = 2 * part; c < 2 * part + 2; ++c) {
+        const int cb = n * BN + c * 32;
+        if (cb >= args.C) break;  // warp-uniform
+        uint32_t v[32];
+        tmem_ld32(tb + c * 32, v);
+        tmem_ld_wait();
+        const int nv = min(32, args.C - cb);  // C is a multiple of 8
+        if (valid) {
+          float4* dst = reinterpret_cast<float4*>(orow + cb);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            if (4 * i < nv)
+              dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
+                                   __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            if (i >= nv) break;
+            const float h = __uint_as_float(v[i]);
+            const __nv_bfloat16 hb = __float2bfloat16_rn(h);
+            const __nv_bfloat16 lb = __float2bfloat16_rn(h - __bfloat162float(hb));
+            const size_t o = (size_t)(cb + i) * args.ldT + row;
+            args.hi[o] = *reinterpret_cast<const uint16_t*>(&hb);
+            args.lo[o] = *reinterpret_cast<const uint16_t*>(&lb);
+          }
+          if (E == 64) {
+            if ((c & 1) == 0) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) prev[i] = __uint_as_float(v[i]);
+            } else {
+              float x[64];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                x[i] = prev[i];
+                x[32 + i] = __uint_as_float(v[i]);
+              }
+              const int l = (cb - 32) / 64;
+              count_topk<64>(reinterpret_cast<float(&)[64]>(x), args.kf, hist + l * 64);
+            }
+          } else {
+#pragma unroll
+            for (int sub = 0; sub < 32 / E; ++sub) {
+              float x[E];
+#pragma unroll
+              for (int i = 0; i < E; ++i) x[i] = __uint_as_float(v[sub * E + i]);
+              const int l = (cb + sub * E) / E;
+              if (l < args.L) count_topk<E>(x, args.kf, hist + l * E);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&s.tempty[slot]);
+    }
+  }
+
+  __syncthreads();
+  if (s.abort) {
+    volatile int* never = &s.zero;
+    if (warp == 0 && lane == 0) {
+      for (int st = 0; st < STAGES; ++st)
+        if ((issued_mask >> st) & 1u)
+          mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, args.limit_ns, never);
+    }
+    if (warp == 1 && lane == 0 && mma_issued) {
+      mma_commit(&s.drain);
+      mbar_wait(&s.drain, 0, args.limit_ns, never);
+    }
+    __syncthreads();
+  }
+  for (int i = tid; i < args.C; i += blockDim.x)
+    if (hist[i]) atomicAdd(&args.counts[i], hist[i]);
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+// grid (row blocks of 128 rows of H^T, token splits)
+__global__ void __launch_bounds__(THREADS, 1)
+    gram_tc_kernel(const __grid_constant__ CUtensorMap mapHi, const __grid_constant__ CUtensorMap mapLo,
+                   GArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* tiles = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  GSmem& s = *reinterpret_cast<GSmem*>(tiles + G_STAGES * G_STAGE_BYTES);
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5;
+  const int lane = tid & 31;
+  const int rb = blockIdx.x, split = blockIdx.y;
+  const int kb0 = split * args.kb_per_split;
+  const int kb1 = min(kb0 + args.kb_per_split, args.kblocks);
+  const int nkb = kb1 > kb0 ? kb1 - kb0 : 0;
+  if (tid == 0) {
+    for (int i = 0; i < G_STAGES; ++i) {
+      mbar_init(&s.full[i], 1);
+      mbar_init(&s.empty[i], 1);
+    }
+    mbar_init(&s.tfull, 1);
+    mbar_init(&s.drain, 1);
+    s.abort = 0;
+    s.zero = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&mapHi);
+    tma_prefetch_map(&mapLo);
+  }
+  if (warp == 1) {
+    tmem_alloc(&s.tmem_base, G_TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = s.tmem_base;
+  volatile int* abort = &s.abort;
+  uint32_t issued_mask = 0, last_phase_bits = 0;
+  bool mma_issued = false;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int i = 0; i < nkb && !*abort; ++i) {
+        if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
+          if (!*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 21);
+          *abort = 1;
+          break;
+        }
+        uint8_t* st = tiles + stage * G_STAGE_BYTES;
+        mbar_arrive_expect_tx(&s.full[stage], G_STAGE_BYTES);
+        tma_load_2d(st, &mapHi, &s.full[stage], (kb0 + i) * BK, rb * 128);
+        tma_load_2d(st + BOX_BYTES, &mapLo, &s.full[stage], (kb0 + i) * BK, rb * 128);
+        issued_mask |= 1u << stage;
+        last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
+        if (++stage == G_STAGES) { stage = 0; phase ^= 1u; }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && nkb > 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int i = 0; i < nkb; ++i) {
+        if (!mbar_wait(&s.full[stage], phase, args.limit_ns, abort)) {
+          if (!*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 22);
+          *abort = 1;
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t hi = smem_u32(tiles + stage * G_STAGE_BYTES);
+        const uint32_t lo = hi + BOX_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BK / 16; ++kk) {
+          const uint64_t dh = sdesc_kmajor_sw128(hi + kk * 32);
+          const uint64_t dl = sdesc_kmajor_sw128(lo + kk * 32);
+          mma_bf16(tmem_base, dh, dh, G_IDESC, (i | kk) != 0 ? 1u : 0u);
+          mma_bf16(tmem_base, dh, dl, G_IDESC, 1u);
+          mma_bf16(tmem_base, dl, dh, G_IDESC, 1u);
+          mma_bf16(tmem_base, dl, dl, G_IDESC, 1u);
+        }
+        mma_issued = true;
+        mma_commit(&s.empty[stage]);
+        if (++stage == G_STAGES) { stage = 0; phase ^= 1u; }
+      }
+      if (ok) mma_commit(&s.tfull);
+    }
+  } else {
+    // epilogue: warp q reads TMEM lanes 32 q .. 32 q + 31 (rows of the block)
+    const int q = warp & 3;
+    const int r = q * 32 + lane;
+    const int gr = rb * 128 + r;
+    const int E = args.E;
+    bool ok = true;
+    if (nkb > 0) {
+      ok = __all_sync(0xffffffffu, mbar_wait(&s.tfull, 0, args.limit_ns, abort));
+      if (!ok && lane == 0 && !*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 23);
+      if (!ok) *abort = 1;
+    }
+    if (ok && !__any_sync(0xffffffffu, *abort != 0)) {
+      tc_fence_after();
+      // the columns of this row's layer: E <= 32 -> inside chunk q; E == 64 ->
+      // chunks 2 (q / 2) and 2 (q / 2) + 1 (warp-uniform either way)
+      const int nch = E == 64 ? 2 : 1;
+      const int ch0 = E == 64 ? 2 * (q >> 1) : q;
+      const int l = gr / E, i = gr - l * E;
+      float* dst = args.gpart + (((size_t)l * args.nsplit + split) * 64 + i) * 64;
+      for (int cc = 0; cc < nch; ++cc) {
+        const int ch = ch0 + cc;
+        uint32_t v[32];
+        if (nkb > 0) {
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ch * 32, v);
+          tmem_ld_wait();
+        } else {
+#pragma unroll
+          for (int x = 0; x < 32; ++x) v[x] = 0u;
+        }
+        if (gr < args.R) {
+#pragma unroll
+          for (int x = 0; x < 32; ++x) {
+            const int col = rb * 128 + ch * 32 + x;
+            if (col / E == l) dst[col - l * E] = __uint_as_float(v[x]);
+          }
+        }
+      }
+    }
+  }
+
+  __syncthreads();
+  if (s.abort) {
+    volatile int* never = &s.zero;
+    if (warp == 0 && lane == 0) {
+      for (int st = 0; st < G_STAGES; ++st)
+        if ((issued_mask >> st) & 1u)
+          mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, args.limit_ns, never);
+    }
+    if (warp == 1 && lane == 0 && mma_issued) {
+      mma_commit(&s.drain);
+      mbar_wait(&s.drain, 0, args.limit_ns, never);
+    }
+    __syncthreads();
+  }
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, G_TMEM_COLS);
+  }
+}
+
+// 2-D bf16 map over [rows][cols] with row pitch ld elements (ld * 2 a multiple
+// of 16 bytes), a 64-column x 128-row box and the 128-byte swizzle; reads past
+// cols or rows return zeros.
+int make_map_ld(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld) {
+  gg::EncodeTiledFn enc = gg::encode_fn();
+  if (!enc) return fail(ORDERMOE_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {BK, 128};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(ORDERMOE_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)r);
+  return ORDERMOE_OK;
+}
+
+}  // namespace sg
+
+bool sim_tc_supported(int L, int E) {
+  return (E == 8 || E == 16 || E == 32 || E == 64) && (long long)L * E <= sg::MAX_HIST;
+}
+
+int sim_tc_nsplit(int L, int E, int64_t N) {
+  const int n_rb = (L * E + 127) / 128;
+  const int kblocks = static_cast<int>((N + sg::BK - 1) / sg::BK);
+  int ns = num_sms() / n_rb;
+  if (ns < 1) ns = 1;
+  if (ns > kblocks) ns = kblocks;
+  return ns;
+}
+
+// H [N][L E] fp32, the hi/lo planes [L E][ldT], counts (zeroed by the caller),
+// and the partial Grams gpart [L][nsplit][64][64].
+int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int d, int kf,
+                  float* H, uint16_t* hi, uint16_t* lo, int ldT, int32_t* counts, float* gpart,
+                  int nsplit, cudaStream_t stream) {
+  using namespace sg;
+  const int C = L * E;
+  const size_t lsmem = L_SMEM_FIXED + sizeof(int) * (size_t)C;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    const int lmax = L_SMEM_FIXED + static_cast<int>(sizeof(int)) * MAX_HIST;
+    attr_err = cudaFuncSetAttribute(sim_logits_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(sim_logits_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(sim_logits_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(sim_logits_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, G_SMEM_BYTES);
+  });
+  if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(similarity)");
+  CUtensorMap mX, mW, mHi, mLo;
+  int rc;
+  if ((rc = make_tmap_bf16(&mX, X, N, d, 128))) return rc;
+  if ((rc = make_tmap_bf16(&mW, W, C, d, 128))) return rc;
+  if ((rc = make_map_ld(&mHi, hi, C, N, ldT))) return rc;
+  if ((rc = make_map_ld(&mLo, lo, C, N, ldT))) return rc;
+  LArgs la{};
+  la.N = N;
+  la.C = C;
+  la.K = d;
+  la.n_tiles = (C + BN - 1) / BN;
+  la.L = L;
+  la.kf = kf;
+  la.H = H;
+  la.hi = hi;
+  la.lo = lo;
+  la.ldT = ldT;
+  la.counts = counts;
+  la.limit_ns = wait_limit_ns();
+  const long long tiles = (long long)((N + BM - 1) / BM) * la.n_tiles;
+  const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
+  switch (E) {
+    case 8: sim_logits_kernel<8><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    case 16: sim_logits_kernel<16><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    case 32: sim_logits_kernel<32><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    default: sim_logits_kernel<64><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+  }
+  OM_LAUNCHED("sim_logits_kernel");
+  GArgs ga{};
+  ga.R = C;
+  ga.E = E;
+  ga.kblocks = (N + BK - 1) / BK;
+  ga.kb_per_split = (ga.kblocks + nsplit - 1) / nsplit;
+  ga.nsplit = nsplit;
+  ga.gpart = gpart;
+  ga.limit_ns = la.limit_ns;
+  gram_tc_kernel<<<dim3((C + 127) / 128, nsplit), THREADS, G_SMEM_BYTES, stream>>>(mHi, mLo, ga);
+  OM_LAUNCHED("gram_tc_kernel");
+  return ORDERMOE_OK;
+}
+
+}  // namespace om

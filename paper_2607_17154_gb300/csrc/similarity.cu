@@ -47,8 +47,10 @@ __device__ __forceinline__ void add_topk_counts(const float* l, int E, int kf, i
 __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ H, int64_t N, int L,
                                                    int E, float* __restrict__ gpart) {
   __shared__ __align__(16) float sh[kSub][64];
-  const int chunk = blockIdx.x, l = blockIdx.y;
-  const int nchunks = gridDim.x;
+  // the layers of one chunk are neighbouring blocks, so each token's record
+  // of L * E logits is read from DRAM once and shared through L2
+  const int l = blockIdx.x, chunk = blockIdx.y;
+  const int nchunks = gridDim.y;
   const int tid = threadIdx.x;
   const int ti = tid >> 4, tj = tid & 15;
   const int LE = L * E;
@@ -114,13 +116,13 @@ template <int EMAX>
 __global__ void __launch_bounds__(256) counts_kernel(const float* __restrict__ H, int64_t N, int L,
                                                      int E, int kf, int32_t* __restrict__ counts) {
   __shared__ int cnt[64];
-  const int l = blockIdx.y;
+  const int l = blockIdx.x;  // layers of the same tokens run side by side (L2 reuse)
   if (threadIdx.x < 64) cnt[threadIdx.x] = 0;
   __syncthreads();
   const int LE = L * E;
   const bool vec = (E & 3) == 0 && (LE & 3) == 0;
-  for (int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; n < N;
-       n += (int64_t)gridDim.x * blockDim.x) {
+  for (int64_t n = (int64_t)blockIdx.y * blockDim.x + threadIdx.x; n < N;
+       n += (int64_t)gridDim.y * blockDim.x) {
     const float* row = H + n * LE + (int64_t)l * E;
     float v[EMAX];
     if (vec) {
@@ -386,29 +388,55 @@ __global__ void __launch_bounds__(64) group_kernel(
   }
 }
 
+// b / C rounded to nearest by Markstein's correction step (P. Markstein, IBM J.
+// Res. Dev. 34(1), 1990): with y = 1/C rounded to nearest and q = RN(b y)
+// within one ulp of b / C, the residual r = b - C q is exact in one fma, and
+// RN(q + r y) is the correctly rounded quotient (no underflow or overflow).
+// Three dependent fp64 operations instead of a full division.
+__device__ __forceinline__ double div_rn_markstein(double b, double C, double y) {
+  const double q = __dmul_rn(b, y);
+  const double r = __fma_rn(-q, C, b);
+  return __fma_rn(r, y, q);
+}
+
+__global__ void div_selftest_kernel(const double* __restrict__ a, const double* __restrict__ b,
+                                    double* __restrict__ out, int64_t n) {
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x)
+    out[i] = div_rn_markstein(a[i], b[i], __drcp_rn(b[i]));
+}
+
 // Mandatory placement, Eqs. 29-31 (Alg. 1 lines 14-24): one warp, layers and
-// experts in order, b_m carried over the layers. Lane m scores server m
-// (lowest score wins, ties to the lower server); eta comes from the
-// per-(server, group) counts of the layer; a waiting-list expert goes to the
-// server with the most room after its layer.
+// experts in order, b_m carried over the layers. Lane m keeps server m's
+// state in registers: b_m, C_m and lambda1 * (b_m / C_m); lambda2 * eta for
+// every count is a table. Per expert, lane m forms its score (one fp64 add of
+// the two terms, as Eq. 30 states them) and, speculatively, the ratio term it
+// would have after taking the expert; the argmin runs on integer keys
+// (scores are non-negative, so their bit patterns order like the values; ties
+// to the lower server), and the winner keeps its speculative term. A
+// waiting-list expert goes to the server with the most room after its layer.
 __global__ void __launch_bounds__(32) place_kernel(
     const int32_t* __restrict__ group, const int32_t* __restrict__ porder, int L, int E, int M,
     PlaceParams pp, const double* __restrict__ p, const double* __restrict__ C,
     uint8_t* __restrict__ placement, double* __restrict__ used, int32_t* __restrict__ status) {
-  __shared__ double b[32];
-  __shared__ double Cs[32];
   __shared__ int grp[64];
   __shared__ int ord[64];
   __shared__ double pls[64];
   __shared__ int waiting[64];
   __shared__ uint8_t xs[32 * 64];
   __shared__ int eta[32 * 64];
+  __shared__ double l2eta[65];  // lambda2 * eta for eta = 0 .. 64
   const int t = threadIdx.x;
   int overflow = 0;
-  if (t < M) {
-    b[t] = 0.0;
-    Cs[t] = C[t];
-  }
+  const bool srv = t < M;
+  double b = 0.0;
+  const double cap = srv ? C[t] : 1.0;
+  const double rcap = __drcp_rn(cap);
+  // non-negative finite values compare like their bit patterns
+  const long long cap_bits = __double_as_longlong(cap);
+  double a1 = srv ? __dmul_rn(pp.lambda1, div_rn_markstein(b, cap, rcap)) : 0.0;
+  bool bad_score = srv && !(cap > 0.0 && cap <= 1.7976931348623157e308);
+  for (int i = t; i <= 64; i += 32) l2eta[i] = __dmul_rn(pp.lambda2, static_cast<double>(i));
   if (t == 0) {
     double need = 0.0, have = 0.0;
     for (int i = 0; i < L * E; ++i) need = __dadd_rn(need, p[i]);
@@ -417,7 +445,7 @@ __global__ void __launch_bounds__(32) place_kernel(
   }
   __syncwarp();
   for (int l = 0; l < L; ++l) {
-    for (int i = t; i < M * 64; i += 32) {
+    for (int i = t; i < 32 * 64; i += 32) {
       xs[i] = 0;
       eta[i] = 0;
     }
@@ -428,50 +456,78 @@ __global__ void __launch_bounds__(32) place_kernel(
     }
     __syncwarp();
     int nw = 0;
+    int jn = ord[0];
+    int gn = grp[jn];
+    double pn = pls[jn];
     for (int pos = 0; pos < E; ++pos) {
-      const int j = ord[pos];
-      const int g = grp[j];
-      double sc = 0.0;
-      int m = (t < M && __dadd_rn(b[t], pls[j]) <= Cs[t]) ? t : (1 << 30);
-      if (m != (1 << 30))
-        sc = __dadd_rn(__dmul_rn(pp.lambda1, __ddiv_rn(b[t], Cs[t])),
-                       __dmul_rn(pp.lambda2, static_cast<double>(eta[t * 64 + g])));
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const double osc = __shfl_xor_sync(0xffffffffu, sc, o);
-        const int om_ = __shfl_xor_sync(0xffffffffu, m, o);
-        if (om_ != (1 << 30) && (m == (1 << 30) || osc < sc || (osc == sc && om_ < m))) {
-          sc = osc;
-          m = om_;
-        }
+      const int j = jn, g = gn;
+      const double pj = pn;
+      if (pos + 1 < E) {  // the next expert does not depend on this one's outcome
+        jn = ord[pos + 1];
+        gn = grp[jn];
+        pn = pls[jn];
       }
-      if (m == (1 << 30)) {
+      const double bn = __dadd_rn(b, pj);
+      const bool feas = srv && __double_as_longlong(bn) <= cap_bits;  // bn <= C_m, bn >= 0
+      // eta of this lane's server (lanes past M are no server: 0); at most E <= 64
+      const int et = srv ? min(eta[t * 64 + g], 64) : 0;
+      const double sc = __dadd_rn(a1, l2eta[et]);
+      double a1n = 0.0;
+      if (feas) a1n = __dmul_rn(pp.lambda1, div_rn_markstein(bn, cap, rcap));  // kept if this lane wins
+      bad_score |= feas && !(sc >= 0.0);
+      unsigned long long key = static_cast<unsigned long long>(__double_as_longlong(sc));
+      if (key == 0x8000000000000000ull) key = 0;  // -0 orders like +0
+      if (!feas) key = ~0ull;
+      // argmin of the 64-bit keys, ties to the lower server: minimum of the high
+      // words, then of the low words among those lanes, then the lowest lane
+      const unsigned khi = static_cast<unsigned>(key >> 32), klo = static_cast<unsigned>(key);
+      const unsigned mhi = __reduce_min_sync(0xffffffffu, khi);
+      const unsigned mlo = __reduce_min_sync(0xffffffffu, khi == mhi ? klo : 0xffffffffu);
+      const unsigned win = __ballot_sync(0xffffffffu, khi == mhi && klo == mlo);
+      int m = __ffs(win) - 1;
+      if (mhi == 0xffffffffu && mlo == 0xffffffffu) m = 64;  // no feasible server
+      if (m == 64) {
         if (t == 0) waiting[nw] = j;
         ++nw;
-      } else if (t == 0) {
+      } else if (t == m) {
         xs[m * 64 + j] = 1;
         eta[m * 64 + g] += 1;
-        b[m] = __dadd_rn(b[m], pls[j]);
+        b = bn;
+        a1 = a1n;
       }
       __syncwarp();
     }
-    if (t == 0) {
-      for (int w = 0; w < nw; ++w) {
-        const int j = waiting[w];
-        int best = 0;
-        for (int m2 = 1; m2 < M; ++m2)
-          if (__dsub_rn(Cs[m2], b[m2]) > __dsub_rn(Cs[best], b[best])) best = m2;
-        xs[best * 64 + j] = 1;
-        b[best] = __dadd_rn(b[best], pls[j]);
-        if (b[best] > Cs[best]) overflow = 1;
+    // waiting list: the server with the largest C_m - b_m (ties: lower m)
+    for (int w = 0; w < nw; ++w) {
+      const int j = waiting[w];
+      const double room = srv ? __dsub_rn(cap, b) : -INFINITY;
+      double br = room;
+      int bm = srv ? t : 64;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const double orr = __shfl_xor_sync(0xffffffffu, br, o);
+        const int om_ = __shfl_xor_sync(0xffffffffu, bm, o);
+        if (orr > br || (orr == br && om_ < bm)) {
+          br = orr;
+          bm = om_;
+        }
       }
+      if (t == bm) {
+        xs[bm * 64 + j] = 1;
+        b = __dadd_rn(b, pls[j]);
+        a1 = __dmul_rn(pp.lambda1, div_rn_markstein(b, cap, rcap));
+        if (b > cap) overflow = 1;
+      }
+      __syncwarp();
     }
-    __syncwarp();
     uint8_t* x = placement + (size_t)l * M * E;
     for (int i = t; i < M * E; i += 32) x[i] = xs[(i / E) * 64 + (i % E)];
     __syncwarp();
   }
-  if (t < M) used[t] = b[t];
+  if (srv) used[t] = b;
+  overflow = __any_sync(0xffffffffu, overflow != 0);
+  if (__any_sync(0xffffffffu, bad_score) && t == 0)
+    report(&g_err_sim, ORDERMOE_DEV_BAD_VALUE, 0);
   if (t == 0) *status = overflow ? ORDERMOE_ERR_CAPACITY : ORDERMOE_OK;
 }
 
@@ -479,14 +535,33 @@ __global__ void __launch_bounds__(32) place_kernel(
 
 using namespace om;
 
+namespace om {
+bool sim_tc_supported(int L, int E);
+int sim_tc_nsplit(int L, int E, int64_t N);
+int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int d, int kf,
+                  float* H, uint16_t* hi, uint16_t* lo, int ldT, int32_t* counts, float* gpart,
+                  int nsplit, cudaStream_t stream);
+}  // namespace om
+
+// Workspace: H [N][L E] fp32 | the hi/lo bf16 planes of H^T [L E][ldT] (tensor-core
+// path) | partial Grams [L][parts][64][64] fp32 | G [L][64][64] fp64.
+static int64_t sim_ldT(int64_t N) { return (N + 7) / 8 * 8; }
+
 extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || N <= 0) return 0;
   const int64_t nchunks = (N + kSimChunk - 1) / kSimChunk;
-  const size_t h = (size_t)N * L * E * sizeof(float);
-  const size_t g = (size_t)L * nchunks * 64 * 64 * sizeof(float);
-  const size_t gd = (size_t)L * 64 * 64 * sizeof(double);
   auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
-  return up(h) + up(g) + up(gd);
+  const size_t h = (size_t)N * L * E * sizeof(float);
+  const size_t planes = sim_tc_supported(L, E) ? 2 * up((size_t)L * E * sim_ldT(N) * 2) : 0;
+  int64_t parts = nchunks;
+  if (sim_tc_supported(L, E)) {
+    // the split count depends on the device; bound it by the number of 64-token steps
+    const int64_t kb = (N + 63) / 64;
+    if (kb > parts) parts = kb;
+  }
+  const size_t g = (size_t)L * parts * 64 * 64 * sizeof(float);
+  const size_t gd = (size_t)L * 64 * 64 * sizeof(double);
+  return up(h) + planes + up(g) + up(gd);
 }
 
 extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
@@ -497,8 +572,8 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: need L >= 1, 1 <= k_freq <= E <= 64");
   if (d <= 0 || d % 64 != 0)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: d must be a positive multiple of 64");
-  if (N <= 0 || N > INT32_MAX || (int64_t)L * E > INT32_MAX)
-    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: bad N");
+  if (N <= 0 || N > 65535LL * kSimChunk || (int64_t)L * E > INT32_MAX || L > 65535)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: need 1 <= N <= 65535 * 1024");
   if (!W_r || !X_cal || !sim || !counts || !workspace)
     return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: null pointer");
   if (!aligned16(W_r) || !aligned16(X_cal) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
@@ -509,22 +584,41 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
   auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
   uint8_t* ws = static_cast<uint8_t*>(workspace);
   float* H = reinterpret_cast<float*>(ws);
-  float* gpart = reinterpret_cast<float*>(ws + up((size_t)N * L * E * sizeof(float)));
+  const bool tc = sim_tc_supported(L, E);
+  const int64_t ldT = sim_ldT(N);
+  const size_t plane = up((size_t)L * E * ldT * 2);
+  uint16_t* hi = reinterpret_cast<uint16_t*>(ws + up((size_t)N * L * E * sizeof(float)));
+  uint16_t* lo = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(hi) + plane);
+  float* gpart = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(hi) + (tc ? 2 * plane : 0));
+  int64_t parts = nchunks;
+  if (tc && (N + 63) / 64 > parts) parts = (N + 63) / 64;
   double* G = reinterpret_cast<double*>(reinterpret_cast<uint8_t*>(gpart) +
-                                        up((size_t)L * nchunks * 64 * 64 * sizeof(float)));
+                                        up((size_t)L * parts * 64 * 64 * sizeof(float)));
+  OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, stream));
+  if (tc) {
+    // tensor-core path: logits with fused counts and hi/lo planes, then the Gram
+    const int nsplit = sim_tc_nsplit(L, E, N);
+    int rc = sim_tc_launch(X_cal, static_cast<int>(N), W_r, L, E, d, k_freq, H, hi, lo,
+                           static_cast<int>(ldT), counts, gpart, nsplit, stream);
+    if (rc) return rc;
+    gram_reduce_kernel<<<dim3(L, 16), 256, 0, stream>>>(gpart, nsplit, G);
+    OM_LAUNCHED("gram_reduce_kernel");
+    sim_finish_kernel<<<L, 256, 0, stream>>>(G, E, sim);
+    OM_LAUNCHED("sim_finish_kernel");
+    return ORDERMOE_OK;
+  }
   int rc = logits_gemm_launch(X_cal, static_cast<int>(N), W_r, L * E, d, H, stream);
   if (rc) return rc;
-  OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, stream));
   int64_t cblocks = (N + 255) / 256;
   const int64_t ccap = (num_sms() * 8 + L - 1) / L;
   if (cblocks > ccap) cblocks = ccap;
-  const dim3 cgrid(static_cast<unsigned>(cblocks), L);
+  const dim3 cgrid(L, static_cast<unsigned>(cblocks));
   if (E <= 8) counts_kernel<8><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
   else if (E <= 16) counts_kernel<16><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
   else if (E <= 32) counts_kernel<32><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
   else counts_kernel<64><<<cgrid, 256, 0, stream>>>(H, N, L, E, k_freq, counts);
   OM_LAUNCHED("counts_kernel");
-  gram_kernel<<<dim3(nchunks, L), 256, 0, stream>>>(H, N, L, E, gpart);
+  gram_kernel<<<dim3(L, nchunks), 256, 0, stream>>>(H, N, L, E, gpart);
   OM_LAUNCHED("gram_kernel");
   gram_reduce_kernel<<<dim3(L, 16), 256, 0, stream>>>(gpart, nchunks, G);
   OM_LAUNCHED("gram_reduce_kernel");
@@ -746,5 +840,17 @@ extern "C" int ordermoe_coverage(const int32_t* group, const uint8_t* placement,
   if (!group || !placement) return fail(ORDERMOE_ERR_INVALID_ARG, "coverage: null pointer");
   coverage_kernel<<<L, 32, 0, stream>>>(group, placement, L, E, M, cover, covered);
   OM_LAUNCHED("coverage_kernel");
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_selftest_div_rn(const double* a, const double* b, double* out, int64_t n,
+                                        ordermoe_stream_t stream) {
+  if (n < 0) return fail(ORDERMOE_ERR_INVALID_ARG, "selftest_div_rn: n < 0");
+  if (n == 0) return ORDERMOE_OK;
+  if (!a || !b || !out) return fail(ORDERMOE_ERR_INVALID_ARG, "selftest_div_rn: null pointer");
+  int64_t blocks = (n + 255) / 256;
+  if (blocks > num_sms() * 8) blocks = num_sms() * 8;
+  div_selftest_kernel<<<static_cast<int>(blocks), 256, 0, stream>>>(a, b, out, n);
+  OM_LAUNCHED("div_selftest_kernel");
   return ORDERMOE_OK;
 }

@@ -116,6 +116,41 @@ def test_place_bit_exact(L, E, M, K, noise):
         np.testing.assert_array_equal(a, b, err_msg=name)
 
 
+def test_placement_quotient_is_correctly_rounded():
+    """The placement's load ratio b_m / C_m (reciprocal + Markstein's correction)
+    equals IEEE division (numpy) bit for bit on random and edge operands."""
+    rng = np.random.default_rng(17)
+    n = 1 << 22
+    a = np.concatenate([rng.random(n // 4) * 1e3, np.floor(rng.random(n // 4) * 4096),
+                        2.0 ** rng.uniform(-300, 300, n // 4) * rng.uniform(1, 2, n // 4),
+                        rng.integers(0, 1 << 40, n // 4).astype(np.float64)])
+    b = np.concatenate([rng.random(n // 4) * 1e3 + 1e-3, np.floor(rng.random(n // 4) * 512) + 1,
+                        2.0 ** rng.uniform(-300, 300, n // 4) * rng.uniform(1, 2, n // 4),
+                        rng.integers(1, 1 << 30, n // 4).astype(np.float64)])
+    b[:64] = 1.0; a[64:128] = 0.0; b[128:192] = 3.0; a[128:192] = np.arange(64)   # exact and repeating
+    bits = rng.integers(0, 1 << 52, 2 * 4096, dtype=np.int64)
+    a[192:4288] = (bits[:4096] | (1023 << 52)).view(np.float64)                    # [1, 2) all mantissas
+    b[192:4288] = (bits[4096:] | (1023 << 52)).view(np.float64)
+    out = torch.empty(n, dtype=torch.float64, device=DEV)
+    B.ordermoe_selftest_div_rn(torch.as_tensor(a).to(DEV), torch.as_tensor(b).to(DEV), out)
+    got = out.cpu().numpy()
+    want = a / b
+    bad = np.nonzero(got.view(np.int64) != want.view(np.int64))[0]
+    assert bad.size == 0, (bad[:5], a[bad[:5]], b[bad[:5]], got[bad[:5]], want[bad[:5]])
+
+
+def test_place_fractional_sizes_and_capacities_bit_exact():
+    rng = np.random.default_rng(23)
+    for L, E, M in [(40, 64, 32), (7, 13, 5), (64, 8, 3)]:
+        sim, counts = synthetic_sims(rng, L, E, 4, 0.4)
+        p = rng.uniform(0.5, 2.5, (L, E))
+        C = p.sum() / M * rng.uniform(1.05, 1.6, M)
+        got = gpu_place(sim, counts, M, p, C)
+        ref = oracle_place_all(sim, counts, M, p, C)
+        for name, a, b in zip(("group", "n_groups", "theta", "placement", "used", "status"), got, ref):
+            np.testing.assert_array_equal(a, b, err_msg="%s L=%d E=%d M=%d" % (name, L, E, M))
+
+
 def test_place_unequal_sizes_waiting_list_and_capacity():
     rng = np.random.default_rng(9)
     L, E, M = 3, 6, 3
