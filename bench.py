@@ -68,6 +68,9 @@ def parse():
                    help="memory budget ratio of the offline plan (Section VI-G): server capacity "
                         "over one copy of the experts; above 1 the spare memory holds replicas "
                         "(Eqs. 32-35). Default: 1.0 for the decode stack, 2.0 for the plan")
+    p.add_argument("--n-cal", type=int, default=None,
+                   help="calibration tokens of the offline plan (default: the workload's; a "
+                        "smaller count makes a short profiling case of the same kernels)")
     p.add_argument("--cpu-seconds", type=float, default=15.0,
                    help="target CPU seconds of the oracle baseline sample")
     return p.parse_args()
@@ -223,7 +226,7 @@ def run_ours(args, dist):
     device = torch.device("cuda", dist.local_rank)
     torch.cuda.set_device(device)
     B.lib()
-    w = synth.workload(args.workload)
+    w = synth.workload(args.workload, **({"n_cal": args.n_cal} if args.n_cal else {}))
     if w.name == "decode_stack":
         return run_decode(args, dist, w, device)
     if w.name == "similarity":

@@ -37,7 +37,8 @@ def gpu_similarity(Wr_stack, Xcal, kf):
 
 
 @pytest.mark.parametrize("L,E,d,N,kf,K", [(1, 8, 256, 4096, 2, 2), (3, 64, 512, 3000, 6, 8),
-                                          (2, 16, 128, 700, 3, 4)])
+                                          (2, 16, 128, 700, 3, 4), (5, 32, 256, 1029, 4, 4),
+                                          (2, 12, 128, 1000, 3, 3), (3, 48, 256, 2100, 6, 6)])
 def test_similarity_matches_oracle(L, E, d, N, kf, K):
     Wr = torch.stack([synth.router_weights(E, d, K, seed=10 + l) for l in range(L)])
     Xcal = synth.calibration(N, d, seed=L * 100 + E)
