@@ -410,6 +410,52 @@ __device__ __forceinline__ float phi_term(const uint8_t* __restrict__ tnext, siz
   return __fmul_rn(p, best);
 }
 
+// H = 3: the term of Eq. 42 with the deepest cost-to-go Phi^(1)(m2, k2, q2)
+// read from a per-token table U[m2][k2] whenever no budget check of that level
+// can fail: U was evaluated with q2 = 0, and with Qmax[k2] the largest loss of
+// a substitute that level can consider (targets k' with P(k2 -> k') != 0),
+// fadd(q2, Qmax[k2]) <= Qbar means every check passes for q2 as for 0 (fadd
+// is monotone and q2 >= 0), so the value is the same; otherwise it is
+// evaluated directly.
+__device__ __forceinline__ float phi_term2_memo(const uint8_t* __restrict__ tnext, size_t stride,
+                                                const float* __restrict__ P, int E, int M, int a,
+                                                int m, int kx, int kt, float qacc, float qbar,
+                                                const float* U, const float* qmax1) {
+  const float p = __ldg(P + (size_t)kx * E + kt);
+  if (p == 0.0f) return 0.0f;
+  const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
+  const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
+  const float* A1 = reinterpret_cast<const float*>(tnext + off_a(E));
+  const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
+  const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
+  float best = INFINITY;
+  unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);
+  while (cand) {
+    const int kk = __ffsll(static_cast<long long>(cand)) - 1;
+    cand &= cand - 1;
+    const bool exact = (kk == kt);
+    float cq = 0.0f, q2 = qacc;
+    if (!exact) {
+      const float qk = __ldg(Q1 + kt * E + kk);
+      if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
+      q2 = __fadd_rn(qacc, qk);
+      cq = __ldg(C1 + kt * E + kk);
+    }
+    const bool free = __fadd_rn(q2, qmax1[kk]) <= qbar;
+    uint32_t pm = __ldg(pm1 + kk);
+    while (pm) {
+      const int m2 = __ffs(pm) - 1;
+      pm &= pm - 1;
+      const float phi1 = free ? U[m2 * E + kk]
+                              : lookahead_phi<1>(tnext + stride, stride, P + E * E, E, M, a, m2, kk,
+                                                 q2, qbar);
+      const float c = __fadd_rn(__fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq), phi1);
+      best = fminf(best, c);
+    }
+  }
+  return __fmul_rn(p, best);
+}
+
 __device__ __forceinline__ float phi_term_h(const Lookahead& la, const uint8_t* tab, int E, int M,
                                             int a, int m, int kx, int kt, float qacc, float qbar) {
   switch (la.H) {
@@ -429,6 +475,8 @@ struct LaSmem {
   float cost0[kLaMaxCand];    // A(a, s, m) + Cq: Eq. 43 without Phi
   float qn[kLaMaxCand];       // accumulated loss after this candidate (Eq. 44)
   float terms[kLaTerms];
+  float U[32 * 64];           // H = 3: Phi^(1)(m2, k2) with every budget check passing
+  float qmax1[64];            // H = 3: largest substitute loss Phi^(1)(., k2) can consider
   unsigned long long best;
   int n;
 };
@@ -467,6 +515,32 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
   const float* Aas = gA + ((size_t)a * M + s) * M;
   const int cpp = kLaTerms / E;  // candidates per pass
   float q = (qhat != nullptr) ? qhat[t] : 0.0f;
+  const bool memo = (la.H == 3) && !(q < 0.0f);  // accumulated losses are never negative
+  if (memo) {
+    // the deepest level's tables (layer l + 2) and transitions (l + 1 -> l + 2)
+    const uint8_t* t2 = tab + 2 * la.stride;
+    const float* P2 = la.P + (size_t)E * E;
+    const float* Q2 = reinterpret_cast<const float*>(t2 + kOffQtab);
+    const unsigned long long* sb2 = reinterpret_cast<const unsigned long long*>(t2 + kOffSubst);
+    for (int k2 = tid; k2 < E; k2 += blockDim.x) {
+      float mx = -INFINITY;
+      for (int kt = 0; kt < E; ++kt) {
+        if (__ldg(P2 + (size_t)k2 * E + kt) == 0.0f) continue;
+        unsigned long long sb = __ldg(sb2 + kt);
+        while (sb) {
+          const int k3 = __ffsll(static_cast<long long>(sb)) - 1;
+          sb &= sb - 1;
+          mx = fmaxf(mx, __ldg(Q2 + kt * E + k3));
+        }
+      }
+      cs.qmax1[k2] = mx;
+    }
+    for (int i = tid; i < M * E; i += blockDim.x) {
+      const int m2 = i / E, k2 = i - (i / E) * E;
+      cs.U[i] = lookahead_phi<1>(tab + 2 * la.stride, la.stride, P2, E, M, a, m2, k2, 0.0f, qbar);
+    }
+    __syncthreads();
+  }
   int first_server = s;
   for (int j = 0; j < k; ++j) {
     const int r = topk_idx[(size_t)t * k + j];
@@ -508,8 +582,10 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
       for (int i = tid; i < nc * E; i += blockDim.x) {
         const int c = base + i / E, kt = i - (i / E) * E;
         const uint32_t code = cs.code[c];
-        cs.terms[i] = phi_term_h(la, tab, E, M, a, static_cast<int>((code >> 8) & 0xFFu),
-                                 static_cast<int>(code & 0xFFu), kt, cs.qn[c], qbar);
+        const int cm = static_cast<int>((code >> 8) & 0xFFu), ck = static_cast<int>(code & 0xFFu);
+        cs.terms[i] = memo ? phi_term2_memo(tab + la.stride, la.stride, la.P, E, M, a, cm, ck, kt,
+                                            cs.qn[c], qbar, cs.U, cs.qmax1)
+                           : phi_term_h(la, tab, E, M, a, cm, ck, kt, cs.qn[c], qbar);
       }
       __syncthreads();
       for (int cl = tid; cl < nc; cl += blockDim.x) {
