@@ -212,3 +212,48 @@ def test_lookahead_skips_a_nan_token_and_reports_it():
     np.testing.assert_array_equal(gl.cpu().numpy()[keep], rl[keep])
     assert gl[3].item() == home[3] and gq[3].item() == 0.0       # state of the NaN token kept
     assert (g[0][3] == -1).all().item()
+
+
+def test_layer_stack_lookahead_through_layer_forward():
+    """Six small layers through ordermoe_layer_forward with H = 3 (router on the
+    tensor cores, tables of all layers in one stack, transition matrices
+    between them): the carried location and loss follow the oracle's
+    look-ahead selection on the oracle's own router logits, for every token
+    whose top-k has no near tie at any layer."""
+    from paper_2607_17154_gb300.layer import LayerStack
+    rng = np.random.default_rng(44)
+    L, T, E, k, M, d, dff, H = 6, 300, 8, 2, 4, 256, 512, 3
+    buf, stride, otabs = stack_tables(rng, L, E, M, 0.3, cheap_links=True)
+    P = rng.random((L - 1, E, E)).astype(np.float32)
+    P[P < 0.5] = 0
+    P = (P / np.maximum(P.sum(axis=2, keepdims=True), 1e-9)).astype(np.float32)
+    layers, Wrb = [], []
+    for l in range(L):
+        Wr = synth.router_weights(E, d, 2, seed=70 + l, device=DEV)
+        W1, W3, W2 = synth.ffn_weights(E, d, dff, seed=80 + l, device=DEV)
+        layers.append({"W_r": Wr, "W1": W1, "W3": W3, "W2": W2})
+        Wrb.append(synth.bits(Wr))
+    stack = LayerStack(layers, buf, k, T, DEV, H=H, stride=stride, P=torch.as_tensor(P).to(DEV))
+    Xs = [synth.hidden(T, d, 90 + l, device=DEV) for l in range(L)]
+    ys = [torch.empty(T, d, dtype=torch.bfloat16, device=DEV) for _ in range(L)]
+    home_np = rng.integers(0, M, T).astype(np.uint8)
+    home = torch.as_tensor(home_np).to(DEV)
+    loc, qhat = home.clone(), torch.zeros(T, device=DEV)
+    counters = torch.zeros(4, dtype=torch.int32, device=DEV)
+    stack.step(Xs, home, loc, qhat, ys, counters)
+    torch.cuda.synchronize()
+    assert counters.sum().item() == L * T * k
+    o_loc, o_q = home_np.copy(), np.zeros(T, np.float32)
+    clear = np.ones(T, bool)
+    for l in range(L):
+        logits = oracle.router_logits(synth.bits(Xs[l]), Wrb[l])
+        srt = -np.sort(-logits.astype(np.float64), axis=1)
+        clear &= np.abs(np.diff(srt[:, :k + 1], axis=1)).min(axis=1) > 1e-3
+        idx, _ = oracle.topk(logits, k)
+        Hl = min(H, L - l)
+        _, _, _, o_loc, o_q = oracle.select_lookahead(idx, otabs[l:l + Hl], P[l:l + Hl - 1], home_np,
+                                                      o_loc, o_q)
+    assert clear.mean() > 0.6
+    np.testing.assert_array_equal(loc.cpu().numpy()[clear], o_loc[clear])
+    np.testing.assert_array_equal(qhat.cpu().numpy()[clear], o_q[clear])
+    assert torch.isfinite(ys[-1].float()).all()
