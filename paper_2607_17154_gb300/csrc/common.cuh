@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "../../include/ordermoe.h"
 
 namespace om {
@@ -21,6 +23,26 @@ int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
                    uint32_t box_rows);
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// A value computed once per device (the current device at the call) and then
+// cached: kernel attributes and occupancy are properties of a device, so a
+// process that drives several GPUs sets them on each. Devices 0..63.
+struct PerDevice {
+  std::mutex mu;
+  int value[64];
+  bool done[64];
+};
+template <class F>
+int per_device(PerDevice& c, F init) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return init();
+  std::lock_guard<std::mutex> g(c.mu);
+  if (!c.done[dev]) {
+    c.value[dev] = init();
+    c.done[dev] = true;
+  }
+  return c.value[dev];
+}
 
 #define OM_CUDA(call)                                   \
   do {                                                  \

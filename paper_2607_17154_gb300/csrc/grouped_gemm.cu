@@ -664,21 +664,21 @@ int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
 
 static int ffn_attrs() {
   using namespace gg;
-  static std::once_flag attr_once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(attr_once, [] {
-    attr_err = cudaFuncSetAttribute(ffn_gemm_pair_kernel<GATEUP>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(ffn_gemm_pair_kernel<DOWN>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<GATEUP>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<DOWN>,
-                                      cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-  });
+  static PerDevice cache;
+  const cudaError_t attr_err = static_cast<cudaError_t>(per_device(cache, [] {
+    cudaError_t e = cudaFuncSetAttribute(ffn_gemm_pair_kernel<GATEUP>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(ffn_gemm_pair_kernel<DOWN>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(ffn_gemm_kernel<GATEUP>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(ffn_gemm_kernel<DOWN>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    return static_cast<int>(e);
+  }));
   if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(ffn_gemm_pair_kernel)");
   return ORDERMOE_OK;
 }
@@ -687,9 +687,8 @@ static int ffn_attrs() {
 // its GPC); the persistent grid never exceeds it, so no pair waits for another.
 static int max_resident_pairs() {
   using namespace gg;
-  static std::once_flag once;
-  static int pairs = 0;
-  std::call_once(once, [] {
+  static PerDevice cache;
+  return per_device(cache, [] {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * (num_sms() / 2), 1, 1);
     cfg.blockDim = dim3(THREADS, 1, 1);
@@ -706,9 +705,8 @@ static int max_resident_pairs() {
       cudaGetLastError();
       n = num_sms() / 2;
     }
-    pairs = n < num_sms() / 2 ? n : num_sms() / 2;
+    return n < num_sms() / 2 ? n : num_sms() / 2;
   });
-  return pairs;
 }
 
 // Tile shape: CTA pairs (256-row tiles) when experts average at least 256
@@ -789,12 +787,12 @@ int ffn_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const uint
 int logits_gemm_launch(const uint16_t* X, int N, const uint16_t* W, int C, int d, float* H,
                        cudaStream_t stream) {
   using namespace gg;
-  static std::once_flag attr_once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(attr_once, [] {
-    attr_err = cudaFuncSetAttribute(ffn_gemm_kernel<LOGITS>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-  });
+  static PerDevice cache;
+  const cudaError_t attr_err = static_cast<cudaError_t>(per_device(cache, [] {
+    return static_cast<int>(cudaFuncSetAttribute(ffn_gemm_kernel<LOGITS>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 SMEM_BYTES));
+  }));
   if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(logits)");
   CUtensorMap mX, mW;
   int rc;

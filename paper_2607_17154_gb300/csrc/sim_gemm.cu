@@ -528,20 +528,20 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
   using namespace sg;
   const int C = L * E;
   const size_t lsmem = L_SMEM_FIXED + sizeof(int) * (size_t)C;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
+  static PerDevice cache;
+  const cudaError_t attr_err = static_cast<cudaError_t>(per_device(cache, [] {
     const int lmax = L_SMEM_FIXED + static_cast<int>(sizeof(int)) * MAX_HIST;
-    attr_err = cudaFuncSetAttribute(sim_logits_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(sim_logits_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(sim_logits_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(sim_logits_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, G_SMEM_BYTES);
-  });
+    cudaError_t e = cudaFuncSetAttribute(sim_logits_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(sim_logits_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(sim_logits_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(sim_logits_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, G_SMEM_BYTES);
+    return static_cast<int>(e);
+  }));
   if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(similarity)");
   CUtensorMap mX, mW, mHi, mLo;
   int rc;
