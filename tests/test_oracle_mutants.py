@@ -93,18 +93,19 @@ import pytest
 @pytest.fixture(scope="session")
 def orc():
     import oracle
-    assert "mutant" in oracle.__file__, oracle.__file__
+    if "mutant" not in oracle.__file__:  # rc 3, never the rc 1 of a caught mistake
+        pytest.exit("the real oracle was imported: " + oracle.__file__, returncode=3)
     oracle.lib()
     return oracle
 """
 
 
-@pytest.mark.parametrize("name,orig,bad", MUTANTS, ids=[m[0] for m in MUTANTS])
-def test_pins_catch_planted_mistake(name, orig, bad, tmp_path):
+def run_mutant(orig, bad, base):
+    """Builds the oracle with one planted mistake under `base` and runs the pins
+    against it; returns the pytest process result."""
     src = open(SRC).read()
     # an anchor that occurs more than once is mutated at its first occurrence
     assert src.count(orig) >= 1, "mutation anchor not found: %r" % orig
-    base = tmp_path / "mutant"
     pkg = base / "oracle"
     pkg.mkdir(parents=True)
     for f in ("__init__.py", "build.py"):
@@ -115,10 +116,26 @@ def test_pins_catch_planted_mistake(name, orig, bad, tmp_path):
     tdir.mkdir()
     shutil.copy(os.path.join(ROOT, "tests", "test_oracle_pins.py"), tdir / "test_oracle_pins.py")
     (tdir / "conftest.py").write_text(CONFTEST)
-    env = dict(os.environ, PYTHONPATH=str(base) + os.pathsep + ROOT)
-    r = subprocess.run([sys.executable, "-m", "pytest", str(tdir), "-q", "-x", "-p", "no:cacheprovider",
-                        "--rootdir", str(base)],
-                       capture_output=True, text=True, env=env, cwd=str(base))
-    assert "mutant" not in r.stdout or "AssertionError: /" not in r.stdout
+    env = dict(os.environ, PYTHONPATH=str(base) + os.pathsep + ROOT, OMP_NUM_THREADS="1")
+    return subprocess.run([sys.executable, "-m", "pytest", str(tdir), "-q", "-x", "-p", "no:cacheprovider",
+                           "--rootdir", str(base)],
+                          capture_output=True, text=True, env=env, cwd=str(base))
+
+
+@pytest.fixture(scope="session")
+def mutant_results(tmp_path_factory):
+    """Every mutant built and checked once, side by side on the host cores."""
+    from concurrent.futures import ThreadPoolExecutor
+    root = tmp_path_factory.mktemp("mutants")
+    workers = max(1, min(len(MUTANTS), os.cpu_count() or 1))
+    with ThreadPoolExecutor(max_workers=workers) as ex:
+        futs = {name: ex.submit(run_mutant, orig, bad, root / ("m%02d" % i))
+                for i, (name, orig, bad) in enumerate(MUTANTS)}
+        return {name: f.result() for name, f in futs.items()}
+
+
+@pytest.mark.parametrize("name,orig,bad", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_planted_mistake(name, orig, bad, mutant_results):
+    r = mutant_results[name]
     assert r.returncode == 1, "no pin caught the planted mistake %r (rc %d):\n%s" % (
         name, r.returncode, r.stdout[-2000:])
