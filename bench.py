@@ -604,9 +604,11 @@ def run_decode(args, dist, w, device):
                      "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
                      "peak_source": "%s hbm_gbs" % pk_kind, "bytes_per_step": wbytes},
-        # 8 kernels a layer, plus the look-ahead selection pass on every layer
-        # that looks ahead (all but the last when H > 1)
-        "gpu_launches": (8 * w.L + sum(min(H, w.L - l) > 1 for l in range(w.L))) * args.steps,
+        # route_select 1, dispatch 2 (one block ranks up to 4096 entries) or 4,
+        # gate/up 1, down 1, combine 1 a layer, plus the look-ahead selection
+        # pass on every layer that looks ahead (all but the last when H > 1)
+        "gpu_launches": ((4 + (2 if w.T * w.k <= 4096 else 4)) * w.L
+                         + sum(min(H, w.L - l) > 1 for l in range(w.L))) * args.steps,
         "clocks": clocks,
         "lookahead_H": H,
         "plan": plan,

@@ -1,8 +1,10 @@
 // Token permutation (histogram, prefix sum, stable scatter + row gather) and
 // the weighted combine.
 //
-// The (token, slot) entries i = t*k + j are cut into chunks of kChunk = 256
-// consecutive entries, one block each:
+// Up to 4096 entries (a decode step) one block computes the histogram, the
+// offsets and the stable ranks (dispatch_small_kernel). Otherwise the (token,
+// slot) entries i = t*k + j are cut into chunks of kChunk = 256 consecutive
+// entries, one block each:
 //   1. chunk_hist: per-chunk expert histogram -> hist[chunk][E]
 //   2. chunk_scan: one block; for every expert the exclusive prefix of its
 //      count over chunks, plus the expert offsets (exclusive prefix over
@@ -146,15 +148,24 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const uint16_t* __rest
   }
 }
 
-// One warp per token; lane l handles the 16-byte vectors l, l + 32, ...
+// One warp per (token, part of 1024 columns): lane l handles the 16-byte
+// vectors part * 128 + l + 32 u, u = 0..3, the loads of a slot in flight
+// together; small batches (a decode step) still spread over many warps.
+constexpr int kCombVec = 128;  // 16-byte vectors per warp item
+
 __global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict__ Yp,
                                                       const int32_t* __restrict__ row_of,
                                                       const float* __restrict__ w, int T, int k,
                                                       int d, uint16_t* __restrict__ y) {
   const int lane = threadIdx.x & 31;
-  const int warps_total = gridDim.x * (blockDim.x >> 5);
+  const int64_t warps_total = (int64_t)gridDim.x * (blockDim.x >> 5);
   const int nvec = d >> 3;
-  for (int t = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); t < T; t += warps_total) {
+  const int parts = (nvec + kCombVec - 1) / kCombVec;
+  const int64_t items = (int64_t)T * parts;
+  for (int64_t it = (int64_t)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); it < items;
+       it += warps_total) {
+    const int t = static_cast<int>(it / parts);
+    const int part = static_cast<int>(it - (int64_t)t * parts);
     int rows[ORDERMOE_MAX_TOPK];
     float ws[ORDERMOE_MAX_TOPK];
     bool ok = true;
@@ -164,23 +175,96 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict
       if (rows[j] < 0 || (int64_t)rows[j] >= (int64_t)T * k) ok = false;
     }
     if (!ok) {  // a row index outside Y_perm: report, leave y[t] untouched
-      if (lane == 0) report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, t);
+      if (lane == 0 && part == 0) report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, t);
       continue;
     }
-    for (int v = lane; v < nvec; v += 32) {
-      float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-      for (int j = 0; j < k; ++j) {
-        const uint4 yv = __ldg(reinterpret_cast<const uint4*>(Yp + (size_t)rows[j] * d) + v);
-        const float wj = ws[j];
-        acc[0] = fmaf(wj, bf16_lo(yv.x), acc[0]); acc[1] = fmaf(wj, bf16_hi(yv.x), acc[1]);
-        acc[2] = fmaf(wj, bf16_lo(yv.y), acc[2]); acc[3] = fmaf(wj, bf16_hi(yv.y), acc[3]);
-        acc[4] = fmaf(wj, bf16_lo(yv.z), acc[4]); acc[5] = fmaf(wj, bf16_hi(yv.z), acc[5]);
-        acc[6] = fmaf(wj, bf16_lo(yv.w), acc[6]); acc[7] = fmaf(wj, bf16_hi(yv.w), acc[7]);
+    float acc[4][8];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int x = 0; x < 8; ++x) acc[u][x] = 0.0f;
+    const int v0 = part * kCombVec + lane;
+    for (int j = 0; j < k; ++j) {
+      const uint4* src = reinterpret_cast<const uint4*>(Yp + (size_t)rows[j] * d);
+      uint4 yv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (v0 + 32 * u < nvec) yv[u] = __ldg(src + v0 + 32 * u);
+      const float wj = ws[j];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (v0 + 32 * u >= nvec) continue;
+        acc[u][0] = fmaf(wj, bf16_lo(yv[u].x), acc[u][0]); acc[u][1] = fmaf(wj, bf16_hi(yv[u].x), acc[u][1]);
+        acc[u][2] = fmaf(wj, bf16_lo(yv[u].y), acc[u][2]); acc[u][3] = fmaf(wj, bf16_hi(yv[u].y), acc[u][3]);
+        acc[u][4] = fmaf(wj, bf16_lo(yv[u].z), acc[u][4]); acc[u][5] = fmaf(wj, bf16_hi(yv[u].z), acc[u][5]);
+        acc[u][6] = fmaf(wj, bf16_lo(yv[u].w), acc[u][6]); acc[u][7] = fmaf(wj, bf16_hi(yv[u].w), acc[u][7]);
       }
+    }
+    uint4* dst = reinterpret_cast<uint4*>(y + (size_t)t * d);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (v0 + 32 * u >= nvec) continue;
       uint4 o;
-      o.x = pack_bf16x2(acc[0], acc[1]); o.y = pack_bf16x2(acc[2], acc[3]);
-      o.z = pack_bf16x2(acc[4], acc[5]); o.w = pack_bf16x2(acc[6], acc[7]);
-      reinterpret_cast<uint4*>(y + (size_t)t * d)[v] = o;
+      o.x = pack_bf16x2(acc[u][0], acc[u][1]); o.y = pack_bf16x2(acc[u][2], acc[u][3]);
+      o.z = pack_bf16x2(acc[u][4], acc[u][5]); o.w = pack_bf16x2(acc[u][6], acc[u][7]);
+      dst[v0 + 32 * u] = o;
+    }
+  }
+}
+
+// Small batches (n <= kSmallN entries, e.g. a decode step): histogram, offsets
+// and the stable rank in one block of 1024 threads. Pass 1 counts every
+// expert; pass 2 walks the entries in rounds of 1024 in index order, ranks
+// each round like rank_kernel and advances the experts' running starts, so
+// the permutation equals the chunked path's.
+constexpr int kSmallN = 4096;
+
+__global__ void __launch_bounds__(1024) dispatch_small_kernel(
+    const int32_t* __restrict__ chosen, int n, int k, int E, int32_t* __restrict__ offsets,
+    int32_t* __restrict__ row_token, int32_t* __restrict__ row_of) {
+  __shared__ int total[64];
+  __shared__ int start[64];
+  __shared__ int wc[32][64];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  if (tid < 64) total[tid] = 0;
+  __syncthreads();
+  for (int i = tid; i < n; i += blockDim.x) {
+    const int e = chosen[i];
+    if (e >= 0 && e < E) atomicAdd(&total[e], 1);
+    else report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, i);
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int acc = 0;
+    for (int x = 0; x < E; ++x) {
+      start[x] = acc;
+      offsets[x] = acc;
+      acc += total[x];
+    }
+    offsets[E] = acc;
+  }
+  for (int r0 = 0; r0 < n; r0 += blockDim.x) {
+    for (int x = tid; x < 32 * 64; x += blockDim.x) (&wc[0][0])[x] = 0;
+    __syncthreads();
+    const int i = r0 + tid;
+    int e = i < n ? chosen[i] : -1;
+    if (e >= E || e < -1) e = -1;  // reported in pass 1
+    const unsigned peers = __match_any_sync(0xffffffffu, e);
+    const int rank_in_warp = __popc(peers & ((1u << lane) - 1u));
+    if (e >= 0 && rank_in_warp == 0) wc[warp][e] = __popc(peers);
+    __syncthreads();
+    if (e >= 0) {
+      int before = 0;
+      for (int w = 0; w < warp; ++w) before += wc[w][e];
+      const int row = start[e] + before + rank_in_warp;
+      row_of[i] = row;
+      row_token[row] = i / k;
+    }
+    __syncthreads();
+    if (tid < E) {
+      int c = 0;
+      for (int w = 0; w < 32; ++w) c += wc[w][tid];
+      start[tid] += c;
     }
   }
 }
@@ -199,12 +283,18 @@ int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int 
     OM_CUDA(cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), stream));
     return ORDERMOE_OK;
   }
-  chunk_hist_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, E, hist);
-  OM_LAUNCHED("chunk_hist_kernel");
-  chunk_scan_kernel<<<1, 1024, 0, stream>>>(hist, nchunks, E, offsets);
-  OM_LAUNCHED("chunk_scan_kernel");
-  rank_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, hist, row_token, row_of);
-  OM_LAUNCHED("rank_kernel");
+  if (n <= kSmallN) {
+    dispatch_small_kernel<<<1, 1024, 0, stream>>>(chosen, static_cast<int>(n), k, E, offsets,
+                                                  row_token, row_of);
+    OM_LAUNCHED("dispatch_small_kernel");
+  } else {
+    chunk_hist_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, E, hist);
+    OM_LAUNCHED("chunk_hist_kernel");
+    chunk_scan_kernel<<<1, 1024, 0, stream>>>(hist, nchunks, E, offsets);
+    OM_LAUNCHED("chunk_scan_kernel");
+    rank_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, hist, row_token, row_of);
+    OM_LAUNCHED("rank_kernel");
+  }
   int64_t blocks = (n + 7) / 8;
   const int cap = num_sms() * 8;
   if (blocks > cap) blocks = cap;
@@ -254,10 +344,11 @@ extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,
   if (!Y_perm || !row_of || !topk_w || !y) return fail(ORDERMOE_ERR_INVALID_ARG, "combine: null pointer");
   if (!aligned16(Y_perm) || !aligned16(y))
     return fail(ORDERMOE_ERR_INVALID_ARG, "combine: Y_perm and y must be 16-byte aligned");
-  int blocks = (T + 7) / 8;
+  const int64_t items = (int64_t)T * (((d >> 3) + kCombVec - 1) / kCombVec);
+  int64_t blocks = (items + 7) / 8;  // 8 warps per block
   const int cap = num_sms() * 8;
   if (blocks > cap) blocks = cap;
-  combine_kernel<<<blocks, 256, 0, stream>>>(Y_perm, row_of, topk_w, T, k, d, y);
+  combine_kernel<<<static_cast<int>(blocks), 256, 0, stream>>>(Y_perm, row_of, topk_w, T, k, d, y);
   OM_LAUNCHED("combine_kernel");
   return ORDERMOE_OK;
 }
