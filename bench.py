@@ -68,6 +68,9 @@ def parse():
                    help="memory budget ratio of the offline plan (Section VI-G): server capacity "
                         "over one copy of the experts; above 1 the spare memory holds replicas "
                         "(Eqs. 32-35). Default: 1.0 for the decode stack, 2.0 for the plan")
+    p.add_argument("--eager", action="store_true",
+                   help="decode stack: launch every kernel from the host instead of replaying "
+                        "each step as one CUDA graph")
     p.add_argument("--n-cal", type=int, default=None,
                    help="calibration tokens of the offline plan (default: the workload's; a "
                         "smaller count makes a short profiling case of the same kernels)")
@@ -553,10 +556,17 @@ def run_decode(args, dist, w, device):
     loc = home.clone()
     qhat = torch.zeros(w.T, device=device)
 
-    def step():
+    def reset():
         loc.copy_(home)
         qhat.zero_()
-        stack.step(Xs, home, loc, qhat, ys)
+
+    if not args.eager:
+        graph = stack.capture(Xs, home, loc, qhat, ys, prologue=reset)
+        step = graph.replay
+    else:
+        def step():
+            reset()
+            stack.step(Xs, home, loc, qhat, ys)
 
     ms, clocks = timed_region(args, dist, device, step)
     code, detail = B.ordermoe_device_error()
@@ -599,6 +609,7 @@ def run_decode(args, dist, w, device):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": w.L, "T": w.T, "d": w.d, "E": w.E, "k": w.k,
                    "d_ff": w.dff, "M": w.M, "lookahead_H": H, "memory_ratio": ratio,
+                   "cuda_graph": not args.eager,
                    "l2": "inputs larger than L2: %.1f GB of expert weights" % (wbytes / 1e9)},
         "roofline": {"kernel": "whole decode step (expert weight streaming)", "bound": "hbm",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",

@@ -95,3 +95,23 @@ class LayerStack:
         T = X_layers[0].shape[0]
         for desc, X, y in zip(self.descs, X_layers, y_layers):
             B.ordermoe_layer_forward(desc, T, X, home, loc, qhat, y, counters, 0, stream)
+
+    def capture(self, X_layers, home, loc, qhat, y_layers, counters=None, prologue=None):
+        """Records one step (every layer's kernels, after the optional prologue,
+        e.g. resetting loc and qhat) as a CUDA graph over these buffers, so a
+        step is one graph launch. Returns the torch.cuda.CUDAGraph; replay()
+        runs the step on the buffers' current contents."""
+        s = torch.cuda.Stream(device=self.scratch.device)
+        s.wait_stream(torch.cuda.current_stream(self.scratch.device))
+        with torch.cuda.stream(s):  # one eager step first: per-device set-up outside the capture
+            if prologue is not None:
+                prologue()
+            self.step(X_layers, home, loc, qhat, y_layers, counters, stream=s)
+        torch.cuda.current_stream(self.scratch.device).wait_stream(s)
+        torch.cuda.synchronize(self.scratch.device)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            if prologue is not None:
+                prologue()
+            self.step(X_layers, home, loc, qhat, y_layers, counters, stream=s)
+        return g

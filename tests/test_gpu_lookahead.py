@@ -257,3 +257,43 @@ def test_layer_stack_lookahead_through_layer_forward():
     np.testing.assert_array_equal(loc.cpu().numpy()[clear], o_loc[clear])
     np.testing.assert_array_equal(qhat.cpu().numpy()[clear], o_q[clear])
     assert torch.isfinite(ys[-1].float()).all()
+
+
+def test_layer_stack_graph_replay_equals_eager_step():
+    """A step captured as one CUDA graph and replayed gives the eager step's
+    outputs bit for bit (location, loss, every layer's y), with look-ahead."""
+    from paper_2607_17154_gb300.layer import LayerStack
+    rng = np.random.default_rng(45)
+    L, T, E, k, M, d, dff, H = 4, 128, 8, 2, 4, 256, 512, 3
+    buf, stride, _ = stack_tables(rng, L, E, M, 0.3, cheap_links=True)
+    P = rng.random((L - 1, E, E)).astype(np.float32)
+    P = (P / P.sum(axis=2, keepdims=True)).astype(np.float32)
+    layers = []
+    for l in range(L):
+        W1, W3, W2 = synth.ffn_weights(E, d, dff, seed=180 + l, device=DEV)
+        layers.append({"W_r": synth.router_weights(E, d, 2, seed=170 + l, device=DEV),
+                       "W1": W1, "W3": W3, "W2": W2})
+    stack = LayerStack(layers, buf, k, T, DEV, H=H, stride=stride, P=torch.as_tensor(P).to(DEV))
+    Xs = [synth.hidden(T, d, 190 + l, device=DEV) for l in range(L)]
+    home = torch.as_tensor(rng.integers(0, M, T).astype(np.uint8)).to(DEV)
+    outs = []
+    for mode in ("eager", "graph"):
+        ys = [torch.zeros(T, d, dtype=torch.bfloat16, device=DEV) for _ in range(L)]
+        loc, qhat = home.clone(), torch.zeros(T, device=DEV)
+
+        def reset():
+            loc.copy_(home)
+            qhat.zero_()
+        if mode == "eager":
+            reset()
+            stack.step(Xs, home, loc, qhat, ys)
+        else:
+            g = stack.capture(Xs, home, loc, qhat, ys, prologue=reset)
+            for y in ys:
+                y.zero_()
+            loc.fill_(0)
+            g.replay()
+        torch.cuda.synchronize()
+        outs.append([loc.clone(), qhat.clone()] + [y.clone() for y in ys])
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
