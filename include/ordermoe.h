@@ -146,7 +146,10 @@ int ordermoe_build_tables(const float* sim, const int32_t* group, const uint8_t*
  * substitute already given to it; the token's new location is the server of
  * slot 0; ties in Eq. 43 go to lower cost, exact, current server, lower
  * server, lower expert. Shapes: 1 <= E <= 64, 1 <= k <= min(E, 8),
- * d % 8 == 0 (X and W_r 16-byte aligned) unless logits_in is given. */
+ * d % 64 == 0 (X and W_r 16-byte aligned) unless logits_in is given.
+ * A token with a NaN logit sets ORDERMOE_DEV_NAN_LOGIT (detail: the token);
+ * its topk_idx row is -1 and its topk_w row 0; its chosen_expert,
+ * chosen_server, kind, loc and qhat are not written. */
 int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, const float* logits_in, int T,
                           int E, int d, int k, int renorm, const void* tables, size_t tables_bytes,
                           const uint8_t* home, uint8_t* loc, float* qhat, float* logits_out,
