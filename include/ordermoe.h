@@ -286,6 +286,25 @@ int ordermoe_layer_forward(const ordermoe_layer_desc* layer, int T, const uint16
                            const uint8_t* home, uint8_t* loc, float* qhat, uint16_t* y,
                            int32_t* counters, int host_io, ordermoe_stream_t stream);
 
+/* nbatch independent batches of T tokens through one layer, from and to
+ * pinned HOST memory, each batch as ordermoe_layer_forward with host_io = 1
+ * and the tokens at their home servers (a first layer: no loc / qhat), with
+ * the copies overlapped with the compute: batch b's inputs are copied in
+ * while batch b - 1 computes, and its output is copied out while batch b + 1
+ * computes (two staging slots, two copy streams owned by the library, one per
+ * device). Serves a queue of requests; has no counterpart in the paper.
+ *   X [nbatch][T][d] bf16, home [nbatch][T] u8, y [nbatch][T][d] bf16 out
+ *   (host); counters as ordermoe_layer_forward.
+ *   layer->scratch: ordermoe_layer_batches_scratch_bytes(T_max, E, d, dff, k)
+ *   bytes (the layer scratch plus a second staging slot).
+ * The call enqueues everything; `stream` is ordered after every copy, so the
+ * caller synchronises it before reading y. Calls on the same device from
+ * several host threads at once must be serialised by the caller. */
+size_t ordermoe_layer_batches_scratch_bytes(int T_max, int E, int d, int dff, int k);
+int ordermoe_layer_forward_batches(const ordermoe_layer_desc* layer, int nbatch, int T,
+                                   const uint16_t* X, const uint8_t* home, uint16_t* y,
+                                   int32_t* counters, ordermoe_stream_t stream);
+
 /* ------------------------------------------------------------------------
  * Offline expert similarity (Section III-B, Eqs. 3-5; Alg. 1 lines 3-5).
  * For each layer l: H_l = W_r^l X_cal^T (router logits over the calibration

@@ -50,6 +50,8 @@ _SIGNATURES = {
                                   _P, _P, _P, _P], _I),
     "ordermoe_utility": ([_P, _P, _P, _I, _D, _D, _D, _D, _P, _P], _I),
     "ordermoe_selftest_div_rn": ([_P, _P, _P, _I64, _P], _I),
+    "ordermoe_layer_batches_scratch_bytes": ([_I, _I, _I, _I, _I], _SZ),
+    "ordermoe_layer_forward_batches": ([_P, _I, _I, _P, _P, _P, _P, _P], _I),
     "ordermoe_place_workspace_bytes": ([_I, _I], _SZ),
     "ordermoe_expert_gate_up": ([_P, _P, _I, _P, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_expert_down": ([_P, _P, _I, _P, _I, _I, _I, _P, _P], _I),
@@ -363,6 +365,22 @@ def ordermoe_layer_forward(desc, T, X, home, loc, qhat, y, counters=None, host_i
                                       _host_or_dev_ptr(qhat, h), _host_or_dev_ptr(y, h),
                                       _ptr(counters), int(host_io), _stream(stream))
     _check("ordermoe_layer_forward", rc)
+
+
+def ordermoe_layer_batches_scratch_bytes(T_max, E, d, dff, k):
+    return int(lib().ordermoe_layer_batches_scratch_bytes(T_max, E, d, dff, k))
+
+
+def ordermoe_layer_forward_batches(desc, nbatch, T, X, home, y, counters=None, stream=None):
+    """X [nbatch, T, d] bf16, home [nbatch, T] u8, y [nbatch, T, d] bf16: pinned host tensors."""
+    _dt(X, torch.bfloat16, "X"); _dt(y, torch.bfloat16, "y"); _dt(home, torch.uint8, "home")
+    for n, t in (("X", X), ("home", home), ("y", y)):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError("%s must be a contiguous host tensor" % n)
+    rc = lib().ordermoe_layer_forward_batches(ctypes.byref(desc), int(nbatch), int(T),
+                                              _host_or_dev_ptr(X, True), _host_or_dev_ptr(home, True),
+                                              _host_or_dev_ptr(y, True), _ptr(counters), _stream(stream))
+    _check("ordermoe_layer_forward_batches", rc)
 
 
 def ordermoe_dispatch_noalloc(chosen_expert, X, T, k, E, d, offsets, row_token, row_of, X_perm,

@@ -2,6 +2,8 @@
 // expert gate/up -> expert down -> combine, with its scratch carved from one
 // caller-provided buffer. With host_io the inputs are copied host -> device
 // and the output device -> host on the same stream.
+#include <mutex>
+
 #include "common.cuh"
 
 namespace om {
@@ -76,6 +78,42 @@ extern "C" int ordermoe_route_select_lookahead(
 extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,
                                 const float* topk_w, int T, int k, int d, uint16_t* y,
                                 ordermoe_stream_t stream);
+
+// Second staging set (X, home, y) of the batched entry point.
+static size_t batch_extra_bytes(int T_max, int d) {
+  return up256((size_t)T_max * d * 2) * 2 + up256((size_t)T_max);
+}
+
+// Copy streams and events of the batched entry point, one set per device.
+struct BatchStreams {
+  cudaStream_t h2d = nullptr, d2h = nullptr;
+  cudaEvent_t start, end, in_ready[2], x_free[2], y_ready[2], y_free[2];
+  bool ok = false;
+};
+
+static BatchStreams* batch_streams() {
+  static std::mutex mu;
+  static BatchStreams per_dev[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> g(mu);
+  BatchStreams& b = per_dev[dev];
+  if (!b.ok) {
+    const unsigned fl = cudaEventDisableTiming;
+    bool good = cudaStreamCreateWithFlags(&b.h2d, cudaStreamNonBlocking) == cudaSuccess &&
+                cudaStreamCreateWithFlags(&b.d2h, cudaStreamNonBlocking) == cudaSuccess &&
+                cudaEventCreateWithFlags(&b.start, fl) == cudaSuccess &&
+                cudaEventCreateWithFlags(&b.end, fl) == cudaSuccess;
+    for (int i = 0; i < 2 && good; ++i)
+      good = cudaEventCreateWithFlags(&b.in_ready[i], fl) == cudaSuccess &&
+             cudaEventCreateWithFlags(&b.x_free[i], fl) == cudaSuccess &&
+             cudaEventCreateWithFlags(&b.y_ready[i], fl) == cudaSuccess &&
+             cudaEventCreateWithFlags(&b.y_free[i], fl) == cudaSuccess;
+    if (!good) return nullptr;
+    b.ok = true;
+  }
+  return &b;
+}
 
 extern "C" size_t ordermoe_layer_scratch_bytes(int T_max, int E, int d, int dff, int k) {
   if (T_max <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || d <= 0 || dff <= 0 || k <= 0 ||
@@ -154,5 +192,86 @@ extern "C" int ordermoe_layer_forward(const ordermoe_layer_desc* L, int T, const
       OM_CUDA(cudaMemcpyAsync(qhat, s.qhat, (size_t)T * 4, cudaMemcpyDeviceToHost, st));
     }
   }
+  return ORDERMOE_OK;
+}
+
+extern "C" size_t ordermoe_layer_batches_scratch_bytes(int T_max, int E, int d, int dff, int k) {
+  const size_t base = ordermoe_layer_scratch_bytes(T_max, E, d, dff, k);
+  return base ? base + batch_extra_bytes(T_max, d) : 0;
+}
+
+extern "C" int ordermoe_layer_forward_batches(const ordermoe_layer_desc* L, int nbatch, int T,
+                                              const uint16_t* X, const uint8_t* home, uint16_t* y,
+                                              int32_t* counters, ordermoe_stream_t stream) {
+  if (!L) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: null layer");
+  if (nbatch < 0 || T < 0 || T > L->T_max)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: need nbatch >= 0, 0 <= T <= T_max");
+  if (!L->W_r || !L->W1 || !L->W3 || !L->W2 || !L->tables || !L->scratch)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: null pointer in the layer");
+  if ((reinterpret_cast<uintptr_t>(L->scratch) & 255u) != 0)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: scratch must be 256-byte aligned");
+  const size_t need = ordermoe_layer_batches_scratch_bytes(L->T_max, L->E, L->d, L->dff, L->k);
+  if (need == 0 || L->scratch_bytes < need)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: scratch too small or bad shape");
+  if (L->d % 256 != 0 || L->dff % 128 != 0 || L->k > L->E)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "layer_forward_batches: need d %% 256 == 0, dff %% 128 == 0, k <= E");
+  if (!aligned16(L->W_r) || !aligned16(L->W1) || !aligned16(L->W3) || !aligned16(L->W2))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: weights must be 16-byte aligned");
+  if (T == 0 || nbatch == 0) return ORDERMOE_OK;
+  if (!X || !home || !y) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: null X/home/y");
+  BatchStreams* bs = batch_streams();
+  if (!bs) return fail(ORDERMOE_ERR_CUDA, "layer_forward_batches: could not create its copy streams");
+  const int E = L->E, d = L->d, dff = L->dff, k = L->k, R = T * k;
+  LayerScratch s = carve(static_cast<uint8_t*>(L->scratch), L->T_max, E, d, dff, k);
+  // staging slot 0 is the layer scratch's X / home / y, slot 1 follows the layer scratch
+  uint8_t* extra = static_cast<uint8_t*>(L->scratch) + s.bytes;
+  uint16_t* Xs[2] = {s.X, reinterpret_cast<uint16_t*>(extra)};
+  uint16_t* ys[2] = {s.y, reinterpret_cast<uint16_t*>(extra + up256((size_t)L->T_max * d * 2))};
+  uint8_t* hs[2] = {s.home, extra + 2 * up256((size_t)L->T_max * d * 2)};
+  cudaStream_t st = stream;
+  const size_t xb = (size_t)T * d * 2;
+  // the copy streams start after everything already on the caller's stream
+  OM_CUDA(cudaEventRecord(bs->start, st));
+  OM_CUDA(cudaStreamWaitEvent(bs->h2d, bs->start, 0));
+  OM_CUDA(cudaStreamWaitEvent(bs->d2h, bs->start, 0));
+  for (int b = 0; b < nbatch; ++b) {
+    const int sl = b & 1;
+    // batch b's inputs: after batch b - 2 has finished reading this slot
+    if (b >= 2) OM_CUDA(cudaStreamWaitEvent(bs->h2d, bs->x_free[sl], 0));
+    OM_CUDA(cudaMemcpyAsync(Xs[sl], X + (size_t)b * T * d, xb, cudaMemcpyHostToDevice, bs->h2d));
+    OM_CUDA(cudaMemcpyAsync(hs[sl], home + (size_t)b * T, (size_t)T, cudaMemcpyHostToDevice, bs->h2d));
+    OM_CUDA(cudaEventRecord(bs->in_ready[sl], bs->h2d));
+    OM_CUDA(cudaStreamWaitEvent(st, bs->in_ready[sl], 0));
+    int rc;
+    if (L->lookahead_H > 1)
+      rc = ordermoe_route_select_lookahead(Xs[sl], L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
+                                           L->tables_stride, L->lookahead_H, L->P, hs[sl], nullptr,
+                                           nullptr, nullptr, s.topk_idx, s.topk_w, s.chosen,
+                                           s.server, s.kind, counters, st);
+    else
+      rc = ordermoe_route_select(Xs[sl], L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
+                                 L->tables_bytes, hs[sl], nullptr, nullptr, nullptr, s.topk_idx,
+                                 s.topk_w, s.chosen, s.server, s.kind, counters, st);
+    if (rc) return rc;
+    rc = dispatch_launch(s.chosen, Xs[sl], T, k, E, d, s.offsets, s.row_token, s.row_of, s.X_perm,
+                         s.hist, st);
+    if (rc) return rc;
+    OM_CUDA(cudaEventRecord(bs->x_free[sl], st));  // X and home of this slot are read
+    rc = gate_up_launch(s.X_perm, s.offsets, R, L->W1, L->W3, E, d, dff, s.H, st);
+    if (rc) return rc;
+    rc = down_launch(s.H, s.offsets, R, L->W2, E, d, dff, s.Y_perm, st);
+    if (rc) return rc;
+    // the output slot: after batch b - 2's copy out has read it
+    if (b >= 2) OM_CUDA(cudaStreamWaitEvent(st, bs->y_free[sl], 0));
+    rc = ordermoe_combine(s.Y_perm, s.row_of, s.topk_w, T, k, d, ys[sl], st);
+    if (rc) return rc;
+    OM_CUDA(cudaEventRecord(bs->y_ready[sl], st));
+    OM_CUDA(cudaStreamWaitEvent(bs->d2h, bs->y_ready[sl], 0));
+    OM_CUDA(cudaMemcpyAsync(y + (size_t)b * T * d, ys[sl], xb, cudaMemcpyDeviceToHost, bs->d2h));
+    OM_CUDA(cudaEventRecord(bs->y_free[sl], bs->d2h));
+  }
+  // the caller's stream is ordered after every copy of this call
+  OM_CUDA(cudaEventRecord(bs->end, bs->d2h));
+  OM_CUDA(cudaStreamWaitEvent(st, bs->end, 0));
   return ORDERMOE_OK;
 }

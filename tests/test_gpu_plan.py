@@ -9,6 +9,7 @@ from paper_2607_17154_gb300 import binding as B
 from paper_2607_17154_gb300 import synth
 from paper_2607_17154_gb300.layer import build_tables
 from tests.helpers import assert_close_bf16
+from tests.test_gpu_path import random_tables_case
 
 pytestmark = pytest.mark.gpu
 
@@ -367,3 +368,31 @@ def test_layer_forward_device_and_host_io_match_the_stepwise_path():
     B.ordermoe_layer_forward(desc, w.T, g["X"], home, None, None, y2)
     torch.cuda.synchronize()
     assert torch.equal(y2, y_dev)
+
+
+def test_layer_forward_batches_matches_single_calls():
+    """Five batches through the overlapped host-I/O entry point (both staging
+    slots reused) give each batch's single-call output bit for bit, and the
+    execution-type counters add up."""
+    w = synth.workload("tiny")
+    E, d, dff, k, M = w.E, w.d, w.dff, w.k, w.M
+    T, nb = 200, 5
+    inp = synth.layer_inputs(w, seed=3, device=DEV)
+    rng = np.random.default_rng(3)
+    sim, group, x = random_tables_case(rng, E, M, 2)
+    tab = build_tables(sim, group, x, 0.5, w.qbar, synth.server_params(M, d, dff, 0), DEV)
+    scratch = torch.empty(B.ordermoe_layer_batches_scratch_bytes(T, E, d, dff, k), dtype=torch.uint8,
+                          device=DEV)
+    desc = B.make_layer_desc(T, inp["Wr"], inp["W1"], inp["W3"], inp["W2"], tab, k, scratch)
+    X = torch.stack([synth.hidden(T, d, 40 + b) for b in range(nb)]).pin_memory()
+    home = torch.as_tensor(rng.integers(0, M, (nb, T)).astype(np.uint8)).pin_memory()
+    y = torch.zeros(nb, T, d, dtype=torch.bfloat16).pin_memory()
+    cnt = torch.zeros(4, dtype=torch.int32, device=DEV)
+    B.ordermoe_layer_forward_batches(desc, nb, T, X, home, y, cnt)
+    torch.cuda.synchronize()
+    assert cnt.sum().item() == nb * T * k
+    for b in range(nb):
+        y1 = torch.zeros(T, d, dtype=torch.bfloat16).pin_memory()
+        B.ordermoe_layer_forward(desc, T, X[b], home[b], None, None, y1, host_io=1)
+        torch.cuda.synchronize()
+        assert torch.equal(y[b], y1), b
