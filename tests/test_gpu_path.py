@@ -119,8 +119,13 @@ def test_route_select_given_logits_bit_exact(T, E, M, k):
         np.testing.assert_array_equal(g["cnt"].cpu().numpy(), np.bincount(okd.ravel(), minlength=4))
 
 
-def test_router_logits_match_oracle():
-    w = synth.workload("tiny", T=300, d=1024)
+@pytest.mark.parametrize("T,d,E", [(300, 1024, 8), (600, 1024, 8), (100, 2048, 16), (700, 512, 16),
+                                   (200, 256, 64), (512, 4096, 8), (513, 4096, 8)])
+def test_router_logits_match_oracle(T, d, E):
+    """The tcgen05 router (one to five 128-row tiles, split-K clusters, E up to
+    64) against the oracle's logits, and the decisions taken from the GPU's
+    own logits."""
+    w = synth.workload("tiny", T=T, d=d, E=E, n_clusters=2)
     inp = synth.layer_inputs(w, seed=3, with_ffn=False)
     Xb, Wb = gbits(inp["X"]), gbits(inp["Wr"])
     ref = oracle.router_logits(Xb, Wb)
@@ -135,9 +140,17 @@ def test_router_logits_match_oracle():
                             home.clone(), torch.zeros(T, device=DEV), logits, *outs)
     got = logits.cpu().numpy()
     np.testing.assert_allclose(got, ref, rtol=1e-3, atol=2e-3)
-    # top-k from the GPU's own logits equals the oracle's top-k of the same logits
+    # top-k and selection from the GPU's own logits equal the oracle's on the same logits
     o_idx, _ = oracle.topk(got, k, 1)
     np.testing.assert_array_equal(outs[0].cpu().numpy(), o_idx)
+    sp = synth.server_params(M, w.d, w.dff, 0)
+    otab = oracle.tables(sim, group, x, 0.5, 0.05, sp.F, sp.B, sp.tau, sp.z, sp.c, sp.omega_T,
+                         sp.omega_Q)
+    h = inp["home"]
+    ch, sv, kd, _, _ = oracle.select(o_idx, otab, h, h.copy(), np.zeros(T, np.float32))
+    np.testing.assert_array_equal(outs[2].cpu().numpy(), ch)
+    np.testing.assert_array_equal(outs[3].cpu().numpy(), sv)
+    np.testing.assert_array_equal(outs[4].cpu().numpy(), kd)
 
 
 # ------------------------------------------------------------------ permutation
