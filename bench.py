@@ -32,11 +32,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # the ncu capture summarised in profiles/ffn_gemm_pair_gate_up_mixtral_prefill.md, valid only while the
 # kernel sources hash to the values recorded with it.
 GATE_UP_TRAFFIC = {
-    "bytes": 2542504704 + 230374144,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
+    "bytes": 2588649728 + 230168064,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
     "sha256": {"paper_2607_17154_gb300/csrc/grouped_gemm.cu":
-               "83270e19b01a7afb5e020b7d6069fc300d330595c354da999ba6bf3bac0c14db",
+               "811b142f57239313369f8f6b9c7c1eb9a4afc8d44d99ba3e2e183fabcbd266d7",
                "paper_2607_17154_gb300/csrc/common.cuh":
-               "73d4c1a58ecdac5707b43b988bf4992cada3bac61861ebfed28e8e69800cd673"},
+               "05db1330c6012b7861955d139033ee2abc5373149a3289af6cdb1771f30fd2cd"},
 }
 
 
@@ -461,6 +461,12 @@ def edge_cost_windows(args, w, device, layers, Xs, home, tabs, stride, P, H, sim
     select_pass(exact_tabs)
     dref, _, nref = cost(exact_tabs)
     select_pass(tabs)
+    # per-server load (slot executions per server over the step) and the
+    # distribution of the accumulated loss q^ against the budget after the last layer
+    load = torch.bincount(rec[2].reshape(-1).to(torch.int64), minlength=M).cpu().tolist()
+    qh = qhat.float().cpu()
+    edges = [round(w.qbar * i / 10, 4) for i in range(11)]
+    qhist = torch.histc(qh, bins=10, min=0.0, max=float(w.qbar)).to(torch.int64).tolist()
     out = torch.empty(5, dtype=torch.float64, device=device)
     stream = torch.cuda.current_stream(device)
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
@@ -479,6 +485,8 @@ def edge_cost_windows(args, w, device, layers, Xs, home, tabs, stride, P, H, sim
         "traffic_bytes_per_1k_tokens": round(n.sum().item() * sp.z * 1000.0 / T, 1),
         "U": round(first[0], 4), "Tbar": round(first[1], 4), "Qbar": round(first[2], 4),
         "cost_and_utility_us": round(ev[0].elapsed_time(ev[1]) * 1e3, 1),
+        "server_load": load,
+        "qhat_hist": {"edges": edges, "counts": qhist},
     }
     # adaptation windows: each prices one step under the current weights
     wT, wQ = first[3], first[4]

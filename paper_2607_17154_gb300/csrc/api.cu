@@ -55,6 +55,7 @@ extern "C" int ordermoe_set_wait_limit_ns(uint64_t limit_ns) {
 }
 
 extern "C" int ordermoe_device_error(int* code, int* detail) {
+  OM_TRACE();
   if (!code) return fail(ORDERMOE_ERR_INVALID_ARG, "device_error: null code");
   OM_CUDA(cudaDeviceSynchronize());
   unsigned long long words[6] = {0, 0, 0, 0, 0, 0};
@@ -79,6 +80,7 @@ extern "C" int ordermoe_device_error(int* code, int* detail) {
 }
 
 extern "C" int ordermoe_selftest_wait_timeout(uint64_t limit_ns, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (limit_ns == 0 || limit_ns > 10000000000ull)
     return fail(ORDERMOE_ERR_INVALID_ARG, "selftest_wait_timeout: need 0 < limit <= 10 s");
   return selftest_wait_timeout(limit_ns, stream);

@@ -8,6 +8,8 @@
 
 #include <mutex>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/ordermoe.h"
 
 namespace om {
@@ -23,6 +25,16 @@ int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
                    uint32_t box_rows);
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// An NVTX range over one C-ABI call, named after it: visible to the Nsight
+// tools, a no-op when none is attached.
+struct TraceRange {
+  explicit TraceRange(const char* name) { nvtxRangePushA(name); }
+  ~TraceRange() { nvtxRangePop(); }
+  TraceRange(const TraceRange&) = delete;
+  TraceRange& operator=(const TraceRange&) = delete;
+};
+#define OM_TRACE() ::om::TraceRange om_trace_range_(__func__)
 
 // A value computed once per device (the current device at the call) and then
 // cached: kernel attributes and occupancy are properties of a device, so a

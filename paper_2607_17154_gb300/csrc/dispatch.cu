@@ -317,6 +317,7 @@ extern "C" int ordermoe_dispatch(const int32_t* chosen_expert, const uint16_t* X
                                  int E, int d, int32_t* offsets, int32_t* row_token,
                                  int32_t* row_of, uint16_t* X_perm, void* workspace,
                                  size_t workspace_bytes, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (T < 0 || k <= 0 || k > ORDERMOE_MAX_TOPK || E <= 0 || E > ORDERMOE_MAX_EXPERTS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "dispatch: need T >= 0, 1 <= k <= 8, 1 <= E <= 64");
   if (d <= 0 || d % 8 != 0)
@@ -336,6 +337,7 @@ extern "C" int ordermoe_dispatch(const int32_t* chosen_expert, const uint16_t* X
 extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,
                                 const float* topk_w, int T, int k, int d, uint16_t* y,
                                 ordermoe_stream_t stream) {
+  OM_TRACE();
   if (T < 0 || k <= 0 || k > ORDERMOE_MAX_TOPK)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "combine: need T >= 0, 1 <= k <= 8");
   if (d <= 0 || d % 8 != 0)

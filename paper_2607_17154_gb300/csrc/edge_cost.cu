@@ -125,6 +125,7 @@ extern "C" int ordermoe_trajectory_cost(const int32_t* target, const int32_t* ch
                                         const double* B, const double* tau, double z, double c,
                                         double* delay, double* loss, int32_t* moves,
                                         ordermoe_stream_t stream) {
+  OM_TRACE();
   if (L <= 0 || T < 0 || k <= 0 || k > ORDERMOE_MAX_TOPK || E <= 0 || E > ORDERMOE_MAX_EXPERTS ||
       M <= 0 || M > ORDERMOE_MAX_SERVERS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
@@ -145,6 +146,7 @@ extern "C" int ordermoe_trajectory_cost(const int32_t* target, const int32_t* ch
 extern "C" int ordermoe_utility(const double* delay, const double* delay_ref, const double* loss,
                                 int T, double qmax, double omega_T, double omega_Q, double kappa,
                                 double* out, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (T <= 0) return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "utility: need T >= 1");
   if (!(qmax > 0.0)) return fail(ORDERMOE_ERR_INVALID_ARG, "utility: need qmax > 0");
   if (!delay || !delay_ref || !loss || !out) return fail(ORDERMOE_ERR_INVALID_ARG, "utility: null pointer");

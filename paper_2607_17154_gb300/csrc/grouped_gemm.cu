@@ -864,6 +864,7 @@ extern "C" int ordermoe_expert_ffn(const uint16_t* X_perm, const int32_t* offset
                                    const uint16_t* W1, const uint16_t* W3, const uint16_t* W2,
                                    int E, int d, int dff, uint16_t* H, uint16_t* Y_perm,
                                    ordermoe_stream_t stream) {
+  OM_TRACE();
   int rc = ffn_check("expert_ffn", R, E, d, dff);
   if (rc || R == 0) return rc;
   if (!offsets || !all_aligned({X_perm, W1, W3, W2, H, Y_perm}))
@@ -874,6 +875,7 @@ extern "C" int ordermoe_expert_ffn(const uint16_t* X_perm, const int32_t* offset
 extern "C" int ordermoe_expert_gate_up(const uint16_t* X_perm, const int32_t* offsets, int R,
                                        const uint16_t* W1, const uint16_t* W3, int E, int d, int dff,
                                        uint16_t* H, ordermoe_stream_t stream) {
+  OM_TRACE();
   int rc = ffn_check("expert_gate_up", R, E, d, dff);
   if (rc || R == 0) return rc;
   if (!offsets || !all_aligned({X_perm, W1, W3, H}))
@@ -884,6 +886,7 @@ extern "C" int ordermoe_expert_gate_up(const uint16_t* X_perm, const int32_t* of
 extern "C" int ordermoe_expert_down(const uint16_t* H, const int32_t* offsets, int R,
                                     const uint16_t* W2, int E, int d, int dff, uint16_t* Y_perm,
                                     ordermoe_stream_t stream) {
+  OM_TRACE();
   int rc = ffn_check("expert_down", R, E, d, dff);
   if (rc || R == 0) return rc;
   if (!offsets || !all_aligned({H, W2, Y_perm}))

@@ -125,6 +125,7 @@ extern "C" size_t ordermoe_layer_scratch_bytes(int T_max, int E, int d, int dff,
 extern "C" int ordermoe_layer_forward(const ordermoe_layer_desc* L, int T, const uint16_t* X,
                                       const uint8_t* home, uint8_t* loc, float* qhat, uint16_t* y,
                                       int32_t* counters, int host_io, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (!L) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: null layer");
   if (T < 0 || T > L->T_max) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: need 0 <= T <= T_max");
   if (!L->W_r || !L->W1 || !L->W3 || !L->W2 || !L->tables || !L->scratch)
@@ -203,6 +204,7 @@ extern "C" size_t ordermoe_layer_batches_scratch_bytes(int T_max, int E, int d, 
 extern "C" int ordermoe_layer_forward_batches(const ordermoe_layer_desc* L, int nbatch, int T,
                                               const uint16_t* X, const uint8_t* home, uint16_t* y,
                                               int32_t* counters, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (!L) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: null layer");
   if (nbatch < 0 || T < 0 || T > L->T_max)
     return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_batches: need nbatch >= 0, 0 <= T <= T_max");

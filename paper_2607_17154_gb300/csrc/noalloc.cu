@@ -63,6 +63,7 @@ extern "C" int ordermoe_dispatch_noalloc(const int32_t* chosen_expert, const uin
                                          int k, int E, int d, int32_t* offsets, int32_t* row_token,
                                          int32_t* row_of, uint16_t* X_perm,
                                          ordermoe_stream_t stream) {
+  OM_TRACE();
   if (T < 0 || k <= 0 || k > ORDERMOE_MAX_TOPK || E <= 0 || E > ORDERMOE_MAX_EXPERTS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
                 "dispatch_noalloc: need T >= 0, 1 <= k <= 8, 1 <= E <= 64");

@@ -872,6 +872,7 @@ extern "C" int ordermoe_build_tables(const float* sim, const int32_t* group,
                                      const double* tau, double z, double c, double omega_T,
                                      double omega_Q, void* tables, size_t tables_bytes_,
                                      ordermoe_stream_t stream) {
+  OM_TRACE();
   if (!sim || !group || !placement || !F || !B || !tau || !tables)
     return fail(ORDERMOE_ERR_INVALID_ARG, "build_tables: null pointer");
   if (E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 || M > ORDERMOE_MAX_SERVERS)
@@ -1003,6 +1004,7 @@ extern "C" int ordermoe_route_select(const uint16_t* X, const uint16_t* W_r, con
                                      float* topk_w, int32_t* chosen_expert,
                                      uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
                                      ordermoe_stream_t stream) {
+  OM_TRACE();
   Lookahead la{1, 0, nullptr};
   return route_select_impl(X, W_r, logits_in, T, E, d, k, renorm, tables, tables_bytes_, la, home,
                            loc, qhat, logits_out, topk_idx, topk_w, chosen_expert, chosen_server,
@@ -1015,6 +1017,7 @@ extern "C" int ordermoe_route_select_lookahead(
     const uint8_t* home, uint8_t* loc, float* qhat, float* logits_out, int32_t* topk_idx,
     float* topk_w, int32_t* chosen_expert, uint8_t* chosen_server, uint8_t* kind,
     int32_t* counters, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (H < 1 || H > 4) return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select_lookahead: need 1 <= H <= 4");
   if (E <= 0 || E > ORDERMOE_MAX_EXPERTS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "route_select_lookahead: need 1 <= E <= 64");

@@ -568,6 +568,7 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
                                    int64_t N, int k_freq, float* sim, int32_t* counts,
                                    void* workspace, size_t workspace_bytes,
                                    ordermoe_stream_t stream) {
+  OM_TRACE();
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: need L >= 1, 1 <= k_freq <= E <= 64");
   if (d <= 0 || d % 64 != 0)
@@ -629,6 +630,7 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
 
 extern "C" int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq,
                                       int32_t* counts, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E || N < 0)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "expert_counts: need 1 <= k_freq <= E <= 64");
   if (!counts || (N > 0 && !logits)) return fail(ORDERMOE_ERR_INVALID_ARG, "expert_counts: null pointer");
@@ -771,6 +773,7 @@ extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, in
                               float* theta, double* importance, uint8_t* placement, double* used,
                               int32_t* status, void* workspace, size_t workspace_bytes,
                               ordermoe_stream_t stream) {
+  OM_TRACE();
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 || M > ORDERMOE_MAX_SERVERS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "place: need L >= 1, 1 <= E <= 64, 1 <= M <= 32");
   if (!sim || !counts || !p || !C || !group || !n_groups || !theta || !placement || !used || !status)
@@ -789,6 +792,7 @@ extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, in
 
 extern "C" int ordermoe_transitions(const float* logits, int64_t N, int L, int E, int k_freq,
                                     int32_t* counts, float* P, ordermoe_stream_t stream) {
+  OM_TRACE();
   if (L < 2 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E || N < 0)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "transitions: need L >= 2, 1 <= k_freq <= E <= 64");
   if (!counts || !P || (N > 0 && !logits)) return fail(ORDERMOE_ERR_INVALID_ARG, "transitions: null pointer");
@@ -814,6 +818,7 @@ extern "C" int ordermoe_replicate(const int32_t* group, const double* importance
                                   const double* C, const double* pi, int L, int E, int M,
                                   uint8_t* placement, double* used, int32_t* replicas,
                                   ordermoe_stream_t stream) {
+  OM_TRACE();
   if (L <= 0 || L > kRepMaxLayers || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 ||
       M > ORDERMOE_MAX_SERVERS || (long long)L * E > kRepMaxCand)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
@@ -835,6 +840,7 @@ extern "C" int ordermoe_replicate(const int32_t* group, const double* importance
 extern "C" int ordermoe_coverage(const int32_t* group, const uint8_t* placement, int L, int E,
                                  int M, uint8_t* cover, int32_t* covered,
                                  ordermoe_stream_t stream) {
+  OM_TRACE();
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || M <= 0 || M > ORDERMOE_MAX_SERVERS)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "coverage: need L >= 1, 1 <= E <= 64, 1 <= M <= 32");
   if (!group || !placement) return fail(ORDERMOE_ERR_INVALID_ARG, "coverage: null pointer");
@@ -845,6 +851,7 @@ extern "C" int ordermoe_coverage(const int32_t* group, const uint8_t* placement,
 
 extern "C" int ordermoe_selftest_div_rn(const double* a, const double* b, double* out, int64_t n,
                                         ordermoe_stream_t stream) {
+  OM_TRACE();
   if (n < 0) return fail(ORDERMOE_ERR_INVALID_ARG, "selftest_div_rn: n < 0");
   if (n == 0) return ORDERMOE_OK;
   if (!a || !b || !out) return fail(ORDERMOE_ERR_INVALID_ARG, "selftest_div_rn: null pointer");
