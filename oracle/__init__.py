@@ -241,6 +241,26 @@ def replicate(group, importance, p, C, pi, placement, used):
     return x, b, reps
 
 
+class _OrcTab(ctypes.Structure):
+    _fields_ = [("Qtab", ctypes.c_void_p), ("Cq", ctypes.c_void_p), ("subst", ctypes.c_void_p),
+                ("A", ctypes.c_void_p), ("pmask", ctypes.c_void_p)]
+
+
+def phi(h, tabs, P, a, m, kx, qacc):
+    """Eq. 42's cost-to-go Phi^(h) of orc_phi: tabs[0] is the current layer's
+    Tables (not read), tabs[1..h] the next layers'; P [h, E, E] the transition
+    matrices from the current layer on. Returns the fp32 value as a float."""
+    t0 = tabs[0]
+    arr = (_OrcTab * len(tabs))(*[_OrcTab(t.Qtab.ctypes.data, t.Cq.ctypes.data, t.subst.ctypes.data,
+                                          t.A.ctypes.data, t.pmask.ctypes.data) for t in tabs])
+    P = _c(P, np.float32)
+    fn = lib().orc_phi
+    fn.restype = ctypes.c_float
+    fn.argtypes = [_I, ctypes.c_void_p, _P, _I, _I, _I, _I, _I, ctypes.c_float, ctypes.c_float]
+    return float(fn(int(h), ctypes.cast(arr, ctypes.c_void_p), _ptr(P), t0.E, t0.M, int(a), int(m),
+                    int(kx), ctypes.c_float(qacc), ctypes.c_float(t0.qbar)))
+
+
 def trajectory_cost(target, chosen, server, home, F, B, tau, z, c, Qtab):
     """Edge delay / substitution loss / transfers of L layers' selection records
     (Eqs. 13-20). target/chosen/server: [L, T, k]; home [T]; Qtab [L, E, E].

@@ -81,6 +81,12 @@ MUTANTS = [
     ("Eq. 42: next move measured from the home server",
      "float c = t1.A[((int64_t)a * M + m) * M + m2]", "float c = t1.A[((int64_t)a * M + a) * M + m2]"),
     ("Eq. 42: probabilities dropped", "const float term = p * best;", "const float term = best;"),
+    ("Eq. 42: deeper levels reuse the first transition matrix",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar)",
+     "orc_phi(h - 1, tabs + 1, P, E, M, a, m2, kk, q2, qbar)"),
+    ("Eq. 42: deeper levels reuse the next layer's tables",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar)",
+     "orc_phi(h - 1, tabs, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar)"),
     ("Eq. 43: cost-to-go ignored",
      "cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, m, kk, qn, qbar);", ""),
 ]

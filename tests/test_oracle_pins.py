@@ -989,6 +989,151 @@ def test_lookahead_h2_matches_brute_force(orc):
     assert changed > 0   # the look-ahead did change some decisions
 
 
+def _feasible(t, target, qacc, taken):
+    """Eq. 40 from its definition: (server, executed expert) pairs where the
+    expert is placed, is the target or an unused within-budget substitute."""
+    f32 = np.float32
+    for m in range(t.M):
+        for kk in range(t.E):
+            if not (int(t.pmask[kk]) >> m) & 1:
+                continue
+            if kk != target:
+                if not (int(t.subst[target]) >> kk) & 1 or kk in taken:
+                    continue
+                if not f32(qacc + t.Qtab[target, kk]) <= t.qbar:
+                    continue
+            yield m, kk
+
+
+def brute_phi(h, tabs, Ps, a, m, kx, qacc):
+    """Eq. 42's Phi^(h) by recursive enumeration (tabs[len - h] is the next
+    layer, Ps[len - 1 - h] the transition into it), fp32."""
+    f32 = np.float32
+    if h == 0:
+        return f32(0)
+    t1, P = tabs[len(tabs) - h], Ps[len(tabs) - 1 - h]
+    acc = f32(0)
+    for kt in range(t1.E):
+        p = P[kx, kt]
+        if p == 0:
+            continue
+        best = f32(np.inf)
+        for m2, k2 in _feasible(t1, kt, qacc, set()):
+            c = f32(t1.A[a, m, m2] + (f32(0) if k2 == kt else t1.Cq[kt, k2]))
+            if h > 1:
+                qn = qacc if k2 == kt else f32(qacc + t1.Qtab[kt, k2])
+                c = f32(c + brute_phi(h - 1, tabs, Ps, a, m2, k2, qn))
+            best = min(best, c)
+        acc = f32(acc + f32(p * best))
+    return acc
+
+
+def brute_lookahead(idx, tabs, Ps, home, loc, qhat):
+    """Eq. 43 with any horizon H = len(tabs): Eq. 42's cost-to-go enumerated
+    recursively over every (target k', server m', executed expert k'') path of
+    the future layers, straight from the feasibility rule of Eq. 40 (no
+    substitute bitmask or placement-mask shortcut), fp32 as the reading fixes it."""
+    f32 = np.float32
+    T, k = idx.shape
+    t0 = tabs[0]
+    E, M = t0.E, t0.M
+    out = [np.zeros((T, k), np.int32), np.zeros((T, k), np.uint8), np.zeros((T, k), np.uint8)]
+    loc2 = loc.copy(); q2 = qhat.copy()
+
+    def feasible(t, target, qacc, taken):
+        for m in range(M):
+            for kk in range(E):
+                if not (int(t.pmask[kk]) >> m) & 1:
+                    continue
+                if kk != target:
+                    if not (int(t.subst[target]) >> kk) & 1 or kk in taken:
+                        continue
+                    if not f32(qacc + t.Qtab[target, kk]) <= t.qbar:
+                        continue
+                yield m, kk
+
+    def phi(h, a, m, kx, qacc):
+        return brute_phi(h, tabs, Ps, a, m, kx, qacc)
+
+    H = len(tabs)
+    for ti in range(T):
+        a, s, q = int(home[ti]), int(loc[ti]), f32(qhat[ti])
+        taken = set(int(v) for v in idx[ti])
+        for j in range(k):
+            r = int(idx[ti, j])
+            cands = []
+            for m, kk in feasible(t0, r, q, taken):
+                g = f32(t0.A[a, s, m] + (f32(0) if kk == r else t0.Cq[r, kk]))
+                qn = q if kk == r else f32(q + t0.Qtab[r, kk])
+                cost = f32(g + phi(H - 1, a, m, kk, qn)) if H > 1 else g
+                cands.append((cost, kk != r, m != s, m, kk))
+            _, sub, away, m, kk = min(cands)
+            out[0][ti, j] = kk; out[1][ti, j] = m; out[2][ti, j] = 2 * away + sub
+            if sub:
+                taken.add(kk); q = f32(q + t0.Qtab[r, kk])
+            if j == 0:
+                loc2[ti] = m
+        q2[ti] = q
+    return out[0], out[1], out[2], loc2, q2
+
+
+@pytest.mark.parametrize("H,trials", [(3, 30), (4, 8)])
+def test_lookahead_deep_horizons_match_brute_force(orc, H, trials):
+    """The paper's default horizon H = 3 (and H = 4) against the recursive
+    enumeration, with budgets tight enough that future substitutes become
+    infeasible along some paths."""
+    rng = np.random.default_rng(40 + H)
+    for trial in range(trials):
+        E, M = int(rng.integers(2, 5)), int(rng.integers(1, 4))
+        k = int(rng.integers(1, min(E, 2) + 1)); T = 6
+        scale = float(rng.choice([1e-4, 1e-2, 1.0]))
+        tabs = [_rand_tables(orc, rng, E, M, 2, tau_scale=scale)[0] for _ in range(H)]
+        for t in tabs[1:]:
+            t.qbar = tabs[0].qbar
+        Ps = []
+        for _ in range(H - 1):
+            P = rng.random((E, E)).astype(np.float32)
+            P[P < 0.3] = 0
+            Ps.append((P / np.maximum(P.sum(axis=1, keepdims=True), 1e-9)).astype(np.float32))
+        idx = np.array([rng.permutation(E)[:k] for _ in range(T)], np.int32)
+        home = rng.integers(0, M, T).astype(np.uint8)
+        loc = rng.integers(0, M, T).astype(np.uint8)
+        qhat = (rng.random(T) * float(rng.choice([0.05, 0.25]))).astype(np.float32)
+        got = orc.select_lookahead(idx, tabs, np.stack(Ps), home, loc, qhat)
+        ref = brute_lookahead(idx, tabs, Ps, home, loc, qhat)
+        for u, v in zip(got, ref):
+            np.testing.assert_array_equal(u, v)
+
+
+def test_cost_to_go_values_match_brute_force(orc):
+    """Phi^(h), h = 1..3, value for value (the same fp32 operations), so that a
+    deeper level reading the wrong layer or transition matrix shows even where
+    it would not change a decision."""
+    rng = np.random.default_rng(47)
+    n = 0
+    for trial in range(12):
+        E, M = int(rng.integers(2, 5)), int(rng.integers(1, 4))
+        H = 4
+        scale = float(rng.choice([1e-3, 1.0]))
+        tabs = [_rand_tables(orc, rng, E, M, 2, tau_scale=scale)[0] for _ in range(H)]
+        for t in tabs[1:]:
+            t.qbar = tabs[0].qbar
+        Ps = []
+        for _ in range(H - 1):
+            P = rng.random((E, E)).astype(np.float32)
+            P[P < 0.3] = 0
+            Ps.append((P / np.maximum(P.sum(axis=1, keepdims=True), 1e-9)).astype(np.float32))
+        for h in (1, 2, 3):
+            for _ in range(6):
+                a, m, kx = int(rng.integers(M)), int(rng.integers(M)), int(rng.integers(E))
+                q = float(np.float32(rng.random() * 0.2))
+                want = brute_phi(h, tabs[:h + 1], Ps[:h], a, m, kx, np.float32(q))
+                got = orc.phi(h, tabs[:h + 1], np.stack(Ps[:h]), a, m, kx, q)
+                assert np.float32(got) == want or (np.isinf(got) and np.isinf(want)), (h, got, want)
+                n += 1
+    assert n == 12 * 3 * 6
+
+
 def test_lookahead_moves_the_token_where_the_next_layer_is_cheap(orc):
     """Hand case (Eqs. 37-43): the target r is only on server 1; its substitute
     s2 is local on server 0. Myopically the local substitute is cheaper
