@@ -73,6 +73,19 @@ MUTANTS = [
     ("Eq. 23: weights swapped", "out[0] = omega_T * st + omega_Q * sq;", "out[0] = omega_Q * st + omega_T * sq;"),
     ("Eq. 45: direction flipped", "omega_Q + kappa * (qbar - tbar)", "omega_Q + kappa * (tbar - qbar)"),
     ("Eq. 45: no projection", "wq = std::min(1.0, std::max(0.0, wq));", ""),
+    ("Eq. 6: threshold runs the wrong way over the layers",
+     "double frac = static_cast<double>(N - l) / static_cast<double>(N - 1);",
+     "double frac = static_cast<double>(l - 1) / static_cast<double>(N - 1);"),
+    ("placement order: importance ascending", "if (I[a] != I[c]) return I[a] > I[c];",
+     "if (I[a] != I[c]) return I[a] < I[c];"),
+    ("waiting list to the fullest server", "if (C[m] - b[m] > C[best] - b[best]) best = m;",
+     "if (C[m] - b[m] < C[best] - b[best]) best = m;"),
+    ("Eq. 34: ties to the later layer", "if (bl < 0 || benefit > bb) { bl = l; bm = m; bj = j; bb = benefit; }",
+     "if (bl < 0 || benefit >= bb) { if (benefit == bb && l == bl) continue; bl = l; bm = m; bj = j; bb = benefit; }"),
+    ("Eq. 45: sums instead of means", "const double tbar = st / T, qbar = sq / T;",
+     "const double tbar = st, qbar = sq;"),
+    ("Eq. 42: future substitutes ignore the budget",
+     "if (!(qacc + t1.Qtab[kt * E + kk] <= qbar)) continue;", ""),
     ("Eq. 41: transitions of the same layer", "topk(logits + (n * L + l + 1) * E, nxt);",
      "topk(logits + (n * L + l) * E, nxt);"),
     ("Eq. 42: transition from the target, not the executed expert",

@@ -619,6 +619,12 @@ def test_place_waiting_list_and_capacity(orc):
     x2, used2, rc2 = orc.place(group, I, p2, C2)
     assert x2[0].sum(axis=0).tolist() == [1, 1, 1]          # c.2 still met
     assert rc2 == orc.CAPACITY                               # sum C < sum p
+    # unequal room: 2 (p 3) -> server 0, 0 -> server 1, 1 fits nowhere and
+    # waits, then goes to the server with the most room left (1: 1.5 > 0)
+    x3, used3, rc3 = orc.place(group, I, np.array([[2.0, 2.0, 3.0]]), np.array([3.0, 3.5]))
+    np.testing.assert_array_equal(x3[0], [[0, 0, 1], [1, 1, 0]])
+    np.testing.assert_array_equal(used3, [3.0, 4.0])
+    assert rc3 == orc.CAPACITY
 
 
 def test_place_invariants_over_layers(orc):
