@@ -86,6 +86,19 @@ MUTANTS = [
      "const double tbar = st, qbar = sq;"),
     ("Eq. 42: future substitutes ignore the budget",
      "if (!(qacc + t1.Qtab[kt * E + kk] <= qbar)) continue;", ""),
+    ("Eq. 37: selection transfer measured from the home server",
+     "const float cost = A[((int64_t)a * M + s) * M + m] + (exact ? 0.0f : Cq[r * E + kk]);",
+     "const float cost = A[((int64_t)a * M + a) * M + m] + (exact ? 0.0f : Cq[r * E + kk]);"),
+    ("Eq. 38: delay weight dropped", "double num = omega_T * dl;", "double num = dl;"),
+    ("Eq. 5: counts from the top-1 only", "for (int j = 0; j < kf; ++j) count[order[j]]++;",
+     "count[order[0]]++;"),
+    ("Eq. 41: normalised over the wrong index",
+     "for (int b = 0; b < E; ++b) row += count[((size_t)l * E + a) * E + b];",
+     "for (int b = 0; b < E; ++b) row += count[((size_t)l * E + b) * E + a];"),
+    ("Eq. 32: coverage of experts instead of groups", "cover[m * K + group_l[e]] = 1;",
+     "cover[m * K + (e % K)] = 1;"),
+    ("Eq. 28: weights swapped", "importance[j] = alpha_f * f + alpha_r * rho;",
+     "importance[j] = alpha_r * f + alpha_f * rho;"),
     ("Eq. 41: transitions of the same layer", "topk(logits + (n * L + l + 1) * E, nxt);",
      "topk(logits + (n * L + l) * E, nxt);"),
     ("Eq. 42: transition from the target, not the executed expert",

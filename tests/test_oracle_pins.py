@@ -591,6 +591,10 @@ def test_importance_closed_forms(orc):
     I = orc.importance(sim, cnt, group, 0.5, 0.5)
     np.testing.assert_allclose(I, [0.5 * 0.5 + 0.5 * 0.8, 0.5 * 0.25 + 0.5 * 0.8, 0.5 * 0.25 + 0.5],
                                rtol=1e-7)
+    # unequal weights (Eq. 28: alpha_f on the frequency, alpha_r on the representativeness)
+    I2 = orc.importance(sim, cnt, group, 0.75, 0.25)
+    np.testing.assert_allclose(I2, [0.75 * 0.5 + 0.25 * 0.8, 0.75 * 0.25 + 0.25 * 0.8,
+                                    0.75 * 0.25 + 0.25 * 1.0], rtol=1e-7)
 
 
 def test_place_hand_example_disperses_groups(orc):
