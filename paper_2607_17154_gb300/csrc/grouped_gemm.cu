@@ -354,23 +354,39 @@ __global__ void __launch_bounds__(THREADS, 1)
 
 // ------------------------------------------------- CTA-pair variant (gate/up, down)
 //
-// A cluster of 2 CTAs on 2 SMs computes a 256-row x 256-column tile with
-// tcgen05.mma.cta_group::2 issued by the even CTA: each CTA holds 128 rows
-// of A and 128 of the 256 B rows in its own shared memory (the same offsets in
-// both), and receives its 128 accumulator rows in its own TMEM. Per SM this
-// halves the B bytes loaded from L2 and written to shared memory per flop
-// compared with a one-CTA 128 x 256 tile. gate/up: B rows 0..127 (even CTA)
-// are W1_e rows, 128..255 (odd CTA) the same rows of W3_e, so accumulator
-// columns 0..127 are the gate and 128..255 the up projection.
+// A cluster of 2 CTAs on 2 SMs computes, with tcgen05.mma.cta_group::2 issued
+// by the even CTA, a tile of 256 weight rows (the MMA's M side; 128 in each
+// CTA's shared memory and TMEM lanes) by up to 256 permuted rows of one expert
+// (the N side, split evenly between the two CTAs' shared memory). The weight
+// side is always full; an expert's last row tile is cut to the next multiple of
+// 16 rows (the N granularity of the instruction), so at most 15 padding rows
+// are computed per expert instead of up to 255 for a 256-row M tile. Each CTA
+// loads its rows as one 128-row TMA box (of which the MMA reads the first N/2):
+// a stage of 5-6 smaller boxes starved the tensor pipe.
+//   gate/up: CTA r holds W1_e rows f..f+63 (TMEM lanes 0..63) and the same
+//            rows of W3_e (lanes 64..127), f = 128 n + 64 r; the epilogue
+//            warps of the gate and up lanes exchange half of their values
+//            through shared memory and each forms SwiGLU for half the rows.
+//   down:    CTA r holds W2_e rows 256 n + 128 r + 0..127 (all 128 lanes).
+// The accumulator is transposed (lane = output column, TMEM column = row);
+// the epilogue writes it row-major through a shared-memory tile with 16-byte
+// coalesced stores, skipping rows beyond the expert's range.
 // Barriers: full[s] (even CTA, one arrive with the pair's bytes; both CTAs'
 // TMA loads complete on it), empty[s] and tfull[b] (both CTAs, arrived by the
 // even CTA's MMA commits multicast to the pair), tempty[b] (even CTA, one
-// arrive per epilogue warp of either CTA).
-constexpr int P_BM = 256;            // rows per CTA pair
+// arrive per epilogue warp of either CTA). Named barrier 1 (the 128 epilogue
+// threads of a CTA) orders the shared-memory exchange; the decision to stop
+// is taken with a barrier reduction so the four epilogue warps always leave
+// together.
+constexpr int P_BM = 256;            // permuted rows (N side) per tile
 constexpr int P_STAGES = 6;
-constexpr int P_STAGE_BYTES = 2 * BOX_BYTES;  // 128 A rows + 128 B rows per CTA
-constexpr uint32_t P_IDESC = idesc_bf16_f32(256, 256);
-constexpr int P_SMEM_BYTES = P_STAGES * P_STAGE_BYTES + 1024 + static_cast<int>(sizeof(Smem));
+constexpr int P_W_BYTES = 128 * BK * 2;   // 128 weight rows per CTA and K block
+constexpr int P_T_BYTES = 128 * BK * 2;   // one box of 128 permuted rows per CTA
+constexpr int P_STAGE_BYTES = P_W_BYTES + P_T_BYTES;
+constexpr int P_X_PITCH = 17;             // floats per exchange row (odd: no bank conflicts)
+constexpr int P_XBUF_FLOATS = 128 * P_X_PITCH;
+constexpr int P_EPI_BYTES = 2 * (P_XBUF_FLOATS * 4 + 32 * 64 * 2);  // gate/up; down needs 2 x 32 x 128 x 2
+static_assert(P_EPI_BYTES >= 2 * 32 * 128 * 2, "down staging fits");
 
 struct PSmem {
   uint64_t full[P_STAGES];
@@ -384,7 +400,9 @@ struct PSmem {
   int mt_start[ORDERMOE_MAX_EXPERTS + 1];
   int offs[ORDERMOE_MAX_EXPERTS + 1];
 };
-static_assert(sizeof(PSmem) <= sizeof(Smem) + 8 * 8, "PSmem size");
+constexpr int P_SMEM_BYTES =
+    P_STAGES * P_STAGE_BYTES + P_EPI_BYTES + 1024 + static_cast<int>(sizeof(PSmem));
+static_assert(P_SMEM_BYTES <= 227 * 1024, "pair kernel shared memory");
 
 __device__ __forceinline__ Tile decode_pair(int tile, const PSmem& s, int E, int n_tiles) {
   int e = 0;
@@ -399,15 +417,37 @@ __device__ __forceinline__ Tile decode_pair(int tile, const PSmem& s, int E, int
   return t;
 }
 
+// rows of the tile rounded up to the MMA's N granularity (16)
+__device__ __forceinline__ int tile_n(const Tile& t) {
+  const int rows = min(P_BM, t.m_end - t.m0);
+  return (rows + 15) & ~15;
+}
+
+// the 128 epilogue threads of this CTA
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+__device__ __forceinline__ bool epi_all(bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.and.pred po, 1, 128, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(p))
+      : "memory");
+  return r != 0;
+}
+
 template <int MODE>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
-    ffn_gemm_pair_kernel(const __grid_constant__ CUtensorMap mapA,
-                         const __grid_constant__ CUtensorMap mapB0,
-                         const __grid_constant__ CUtensorMap mapB1, Args args) {
+    ffn_gemm_pair_kernel(const __grid_constant__ CUtensorMap mapW0,
+                         const __grid_constant__ CUtensorMap mapW1,
+                         const __grid_constant__ CUtensorMap mapT, Args args) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* tiles = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  PSmem& s = *reinterpret_cast<PSmem*>(tiles + P_STAGES * P_STAGE_BYTES);
+  uint8_t* epi = tiles + P_STAGES * P_STAGE_BYTES;
+  PSmem& s = *reinterpret_cast<PSmem*>(epi + P_EPI_BYTES);
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
@@ -448,9 +488,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_map(&mapA);
-    tma_prefetch_map(&mapB0);
-    if (MODE == GATEUP) tma_prefetch_map(&mapB1);
+    tma_prefetch_map(&mapW0);
+    if (MODE == GATEUP) tma_prefetch_map(&mapW1);
+    tma_prefetch_map(&mapT);
   }
   if (warp == 1) {
     tmem_alloc_pair(&s.tmem_base, TMEM_COLS);
@@ -472,22 +512,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       uint32_t phase = 0;
       for (int tile = cluster; tile < total && !*abort; tile += n_clusters) {
         const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
-        const int arow = t.m0 + 128 * static_cast<int>(rank);
-        const int brow = (MODE == GATEUP) ? t.e * args.b_rows + t.n * 128
-                                          : t.e * args.b_rows + t.n * 256 + 128 * static_cast<int>(rank);
-        const CUtensorMap* mapB = (MODE == GATEUP && !even) ? &mapB1 : &mapB0;
+        const int trow = t.m0 + static_cast<int>(rank) * (tile_n(t) >> 1);  // N/2 rows per CTA
+        const int wrow = (MODE == GATEUP)
+                             ? t.e * args.b_rows + t.n * 128 + 64 * static_cast<int>(rank)
+                             : t.e * args.b_rows + t.n * 256 + 128 * static_cast<int>(rank);
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
             if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 11);
             *abort = 1;
             break;
           }
-          uint8_t* sa = tiles + stage * P_STAGE_BYTES;
-          uint8_t* sb = sa + BOX_BYTES;
+          uint8_t* sw = tiles + stage * P_STAGE_BYTES;
+          uint8_t* st = sw + P_W_BYTES;
           const uint32_t full_even = mapa_shared(smem_u32(&s.full[stage]), 0);
           if (even) mbar_arrive_expect_tx(&s.full[stage], 2 * P_STAGE_BYTES);
-          tma_load_2d_pair(sa, &mapA, full_even, kb * BK, arow);
-          tma_load_2d_pair(sb, mapB, full_even, kb * BK, brow);
+          if (MODE == GATEUP) {
+            tma_load_2d_pair(sw, &mapW0, full_even, kb * BK, wrow);             // W1: lanes 0..63
+            tma_load_2d_pair(sw + P_W_BYTES / 2, &mapW1, full_even, kb * BK, wrow);  // W3: 64..127
+          } else {
+            tma_load_2d_pair(sw, &mapW0, full_even, kb * BK, wrow);
+          }
+          tma_load_2d_pair(st, &mapT, full_even, kb * BK, trow);
           issued_mask |= 1u << stage;
           last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
@@ -508,6 +553,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           break;
         }
         tc_fence_after();
+        const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
+        const uint32_t idesc = idesc_bf16_f32(256, tile_n(t));
         const uint32_t d_tmem = tmem_base + slot * BN;
         bool ok = true;
         for (int kb = 0; kb < kblocks; ++kb) {
@@ -519,11 +566,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           }
           tc_fence_after();
           const uint32_t a0 = smem_u32(tiles + stage * P_STAGE_BYTES);
-          const uint32_t b0 = a0 + BOX_BYTES;
+          const uint32_t b0 = a0 + P_W_BYTES;
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
             mma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32),
-                          sdesc_kmajor_sw128(b0 + kk * 32), P_IDESC, (kb | kk) != 0 ? 1u : 0u);
+                          sdesc_kmajor_sw128(b0 + kk * 32), idesc, (kb | kk) != 0 ? 1u : 0u);
           mma_issued = true;
           mma_commit_pair(&s.empty[stage], 0x3);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
@@ -533,65 +580,89 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       }
     }
   } else {
+    // epilogue: warps 2..5, TMEM lane quarter q = warp % 4
     const int q = warp & 3;
-    const int lrow = q * 32 + lane;
+    const int et = tid - 64;  // 0..127
+    float* xbuf = reinterpret_cast<float*>(epi);                          // [2][128][P_X_PITCH]
+    uint16_t* obuf = reinterpret_cast<uint16_t*>(epi + 2 * P_XBUF_FLOATS * 4);  // gate/up [2][32][64]
+    uint16_t* ybuf = reinterpret_cast<uint16_t*>(epi);                    // down [2][32][128]
     int it = 0;
     for (int tile = cluster; tile < total; tile += n_clusters, ++it) {
-      if (__any_sync(0xffffffffu, *abort != 0)) break;
       const int slot = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
-      const bool ok =
-          __all_sync(0xffffffffu, mbar_wait(&s.tfull[slot], acc_phase, args.limit_ns, abort));
-      if (!ok) {
-        if (lane == 0 && !*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 14);
+      const bool waited = (*abort == 0) && mbar_wait(&s.tfull[slot], acc_phase, args.limit_ns, abort);
+      if (!epi_all(waited)) {  // the same decision in all four warps
+        if (!waited && lane == 0 && !*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 14);
         *abort = 1;
         break;
       }
       tc_fence_after();
       const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
-      const int row = t.m0 + 128 * static_cast<int>(rank) + lrow;
-      const bool valid = row < t.m_end;
+      const int rows = min(P_BM, t.m_end - t.m0);
+      const int nchunks = (rows + 31) >> 5;
       const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
-      if (MODE == GATEUP) {
-        uint16_t* orow = args.out + (size_t)row * args.ldo + t.n * 128;
 #pragma unroll 1
-        for (int c = 0; c < 4; ++c) {
-          uint32_t g[32], u[32];
-          tmem_ld32(tb + c * 32, g);
-          tmem_ld32(tb + 128 + c * 32, u);
-          tmem_ld_wait();
-          if (valid) {
-            uint32_t pk[16];
+      for (int c = 0; c < nchunks; ++c) {
+        const int buf = c & 1;
+        uint32_t v[32];
+        tmem_ld32(tb + c * 32, v);  // TMEM column = row c*32 + i of the tile
+        tmem_ld_wait();
+        if (MODE == GATEUP) {
+          // gate lanes (q 0, 1) keep rows 0..15 of the chunk and hand 16..31
+          // to the up lanes (q 2, 3) of the same columns, which hand back 0..15
+          const bool gate = q < 2;
+          const int keep = gate ? 0 : 16;
+          float* xb = xbuf + buf * P_XBUF_FLOATS;
+          float* mine = xb + (q * 32 + lane) * P_X_PITCH;
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const float g0 = __uint_as_float(g[2 * i]), g1 = __uint_as_float(g[2 * i + 1]);
-              const float u0 = __uint_as_float(u[2 * i]), u1 = __uint_as_float(u[2 * i + 1]);
-              const float h0 = g0 / (1.0f + __expf(-g0)) * u0;
-              const float h1 = g1 / (1.0f + __expf(-g1)) * u1;
-              pk[i] = pack_bf16x2(h0, h1);
+          for (int i = 0; i < 16; ++i) mine[i] = __uint_as_float(gate ? v[16 + i] : v[i]);
+          epi_sync();
+          const float* other = xb + ((q ^ 2) * 32 + lane) * P_X_PITCH;
+          uint16_t* ob = obuf + buf * (32 * 64);
+          const int col = (q & 1) * 32 + lane;
+#pragma unroll
+          for (int i = 0; i < 16; i += 2) {
+            float h[2];
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+              const float own = __uint_as_float(gate ? v[i + j] : v[16 + i + j]);
+              const float oth = other[i + j];
+              const float g = gate ? own : oth;
+              const float u = gate ? oth : own;
+              h[j] = g / (1.0f + __expf(-g)) * u;
             }
-            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
-#pragma unroll
-            for (int i = 0; i < 4; ++i)
-              dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+            const uint32_t pk = pack_bf16x2(h[0], h[1]);
+            ob[(keep + i) * 64 + col] = static_cast<uint16_t>(pk & 0xFFFFu);
+            ob[(keep + i + 1) * 64 + col] = static_cast<uint16_t>(pk >> 16);
           }
-        }
-      } else {
-        uint16_t* orow = args.out + (size_t)row * args.ldo + t.n * 256;
-#pragma unroll 1
-        for (int c = 0; c < 8; ++c) {
-          uint32_t v[32];
-          tmem_ld32(tb + c * 32, v);
-          tmem_ld_wait();
-          if (valid) {
-            uint32_t pk[16];
+          epi_sync();
+          uint16_t* gcol = args.out + t.n * 128 + 64 * static_cast<int>(rank) + (et & 7) * 8;
 #pragma unroll
-            for (int i = 0; i < 16; ++i)
-              pk[i] = pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+          for (int p = 0; p < 2; ++p) {
+            const int r = p * 16 + (et >> 3);
+            const int row = c * 32 + r;
+            if (row < rows)
+              *reinterpret_cast<uint4*>(gcol + (size_t)(t.m0 + row) * args.ldo) =
+                  *reinterpret_cast<const uint4*>(ob + r * 64 + (et & 7) * 8);
+          }
+        } else {
+          uint16_t* yb = ybuf + buf * (32 * 128);
+          const int col = q * 32 + lane;
 #pragma unroll
-            for (int i = 0; i < 4; ++i)
-              dst[i] = make_uint4(pk[4 * i], pk[4 * i + 1], pk[4 * i + 2], pk[4 * i + 3]);
+          for (int i = 0; i < 32; i += 2) {
+            const uint32_t pk = pack_bf16x2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+            yb[i * 128 + col] = static_cast<uint16_t>(pk & 0xFFFFu);
+            yb[(i + 1) * 128 + col] = static_cast<uint16_t>(pk >> 16);
+          }
+          epi_sync();
+          uint16_t* gcol = args.out + t.n * 256 + 128 * static_cast<int>(rank) + (et & 15) * 8;
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const int r = p * 8 + (et >> 4);
+            const int row = c * 32 + r;
+            if (row < rows)
+              *reinterpret_cast<uint4*>(gcol + (size_t)(t.m0 + row) * args.ldo) =
+                  *reinterpret_cast<const uint4*>(yb + r * 128 + (et & 15) * 8);
           }
         }
       }
@@ -731,18 +802,21 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
   using namespace gg;
   int rc;
   if ((rc = ffn_attrs())) return rc;
-  CUtensorMap mX, mW1, mW3;
-  if ((rc = make_map(&mX, X_perm, R, d))) return rc;
-  if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
-  if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
   Args a{};
   a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = d; a.n_tiles = dff / 128; a.b_rows = dff; a.out = H; a.ldo = dff;
+  CUtensorMap mX, mW1, mW3;
+  if ((rc = make_map(&mX, X_perm, R, d))) return rc;
   if (use_pairs(R, E)) {
+    // weights on the MMA's M side in 64-row boxes of W1 and W3
+    if ((rc = make_tmap_bf16(&mW1, W1, (uint64_t)E * dff, d, 64))) return rc;
+    if ((rc = make_tmap_bf16(&mW3, W3, (uint64_t)E * dff, d, 64))) return rc;
     const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
-    ffn_gemm_pair_kernel<GATEUP><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
+    ffn_gemm_pair_kernel<GATEUP><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mW1, mW3, mX, a);
     OM_LAUNCHED("ffn_gemm_pair_kernel<gate_up>");
   } else {
+    if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
+    if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
     const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
     ffn_gemm_kernel<GATEUP><<<single_grid(tiles), THREADS, SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
     OM_LAUNCHED("ffn_gemm_kernel<gate_up>");
@@ -756,15 +830,15 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   using namespace gg;
   int rc;
   if ((rc = ffn_attrs())) return rc;
-  CUtensorMap mH, mW2;
-  if ((rc = make_map(&mH, H, R, dff))) return rc;
-  if ((rc = make_map(&mW2, W2, (uint64_t)E * d, dff))) return rc;
   Args a{};
   a.offsets = offsets; a.rows = R; a.E = E; a.limit_ns = wait_limit_ns();
   a.K = dff; a.n_tiles = d / 256; a.b_rows = d; a.out = Y; a.ldo = d;
+  CUtensorMap mH, mW2;
+  if ((rc = make_map(&mW2, W2, (uint64_t)E * d, dff))) return rc;
+  if ((rc = make_map(&mH, H, R, dff))) return rc;
   if (use_pairs(R, E)) {
     const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
-    ffn_gemm_pair_kernel<DOWN><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
+    ffn_gemm_pair_kernel<DOWN><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mW2, mW2, mH, a);
     OM_LAUNCHED("ffn_gemm_pair_kernel<down>");
   } else {
     const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;

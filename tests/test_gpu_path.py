@@ -212,8 +212,9 @@ def run_gpu_ffn(E, R, off, Xp, W1, W3, W2, d, dff):
     ([300, 0, 1, 128, 129, 77], 512, 384),                # ragged tails, empty and 1-row experts
     ([37], 256, 128),                                     # one partial tile
     ([256, 256], 1024, 1024),                             # several full tiles and K blocks
-    # CTA pairs (at least 256 rows per expert on average): tails of 1, 128, 88,
-    # 44 and 1 rows run as half-height (M = 128) tiles, 129 and 255 as full ones
+    # CTA pairs (at least 256 rows per expert on average): last row tiles of
+    # 1, 128, 88, 44, 1, 129 and 255 rows, cut to N = 16, 128, 96, 48, 16, 144
+    # and 256 columns of the transposed accumulator
     ([257, 384, 600, 300, 512, 1], 256, 512),
     ([129, 255, 256, 384], 512, 384),
 ])
