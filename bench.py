@@ -32,9 +32,9 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # the ncu capture summarised in profiles/ffn_gemm_pair_gate_up_mixtral_prefill.md, valid only while the
 # kernel sources hash to the values recorded with it.
 GATE_UP_TRAFFIC = {
-    "bytes": 1967000576 + 228295680,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
+    "bytes": 1968486656 + 228585216,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
     "sha256": {"paper_2607_17154_gb300/csrc/grouped_gemm.cu":
-               "3271952fc1ede18f0ea1e8bfb935bc509fae75ecbef0dfdd231d03ffffaf10c5",
+               "87a4eff77262b927f72bd4af01b34d96d18720058974c363af9a53970794de33",
                "paper_2607_17154_gb300/csrc/common.cuh":
                "05db1330c6012b7861955d139033ee2abc5373149a3289af6cdb1771f30fd2cd"},
 }
@@ -348,7 +348,7 @@ def run_ours(args, dist):
                    "home": w.home, "seed": args.seed, "parallelism": "replicas",
                    "l2": "inputs larger than L2: %.2f GB of expert weights read every step"
                          % (3 * E * d * dff * 2 / 1e9)},
-        "roofline": {"kernel": "ffn_gemm_pair_kernel<gate_up> (tcgen05, CTA pair)", "bound": "tensor",
+        "roofline": {"kernel": "ffn_gemm_pair_kernel<gate_up, 4> (tcgen05 CTA pairs, clusters of 4)", "bound": "tensor",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(achieved / peak, 4), "traffic": gate_up_traffic(w.name),
                      "peak_source": "%s bf16_tflops_sustained" % pk_kind,

@@ -354,7 +354,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
 // ------------------------------------------------- CTA-pair variant (gate/up, down)
 //
-// A cluster of 2 CTAs on 2 SMs computes, with tcgen05.mma.cta_group::2 issued
+// A pair of CTAs on 2 SMs computes, with tcgen05.mma.cta_group::2 issued
 // by the even CTA, a tile of 256 weight rows (the MMA's M side; 128 in each
 // CTA's shared memory and TMEM lanes) by up to 256 permuted rows of one expert
 // (the N side, split evenly between the two CTAs' shared memory). The weight
@@ -371,9 +371,16 @@ __global__ void __launch_bounds__(THREADS, 1)
 // The accumulator is transposed (lane = output column, TMEM column = row);
 // the epilogue writes it row-major through a shared-memory tile with 16-byte
 // coalesced stores, skipping rows beyond the expert's range.
+// Clusters of 4 CTAs (two pairs) halve the L2 reads of the permuted rows: the
+// two pairs take neighbouring column slices of the same row tile, and each
+// CTA loads half of its 128-row box of rows and multicasts it to the CTA of
+// the same rank in the other pair (TMA reads from L2 per CTA and K step drop
+// from 32 KB to 24 KB); used when the slice count is even. A stage then holds
+// data from both pairs, so each pair's MMA commit releases it in all four CTAs.
 // Barriers: full[s] (even CTA, one arrive with the pair's bytes; both CTAs'
-// TMA loads complete on it), empty[s] and tfull[b] (both CTAs, arrived by the
-// even CTA's MMA commits multicast to the pair), tempty[b] (even CTA, one
+// TMA loads, and the other pair's multicast, complete on it), empty[s] and tfull[b] (both CTAs, arrived by the
+// even CTA's MMA commits multicast to the pair, or to all four CTAs for
+// empty[s] in a cluster of 4), tempty[b] (even CTA, one
 // arrive per epilogue warp of either CTA). Named barrier 1 (the 128 epilogue
 // threads of a CTA) orders the shared-memory exchange; the decision to stop
 // is taken with a barrier reduction so the four epilogue warps always leave
@@ -417,6 +424,19 @@ __device__ __forceinline__ Tile decode_pair(int tile, const PSmem& s, int E, int
   return t;
 }
 
+// Multicast TMA load of a CTA pair: the box lands at the same offset in every
+// CTA of cta_mask, and its bytes complete on the mbarrier at bar's offset in
+// the even CTA of each destination's pair (bar is an even CTA's barrier).
+__device__ __forceinline__ void tma_load_2d_pair_mc(void* smem_dst, const CUtensorMap* map,
+                                                    uint32_t bar_cluster_addr, int c0, int c1,
+                                                    uint16_t cta_mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      ".multicast::cluster.cta_group::2 [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(smem_dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster_addr), "r"(c0), "r"(c1), "h"(cta_mask)
+      : "memory");
+}
+
 // rows of the tile rounded up to the MMA's N granularity (16)
 __device__ __forceinline__ int tile_n(const Tile& t) {
   const int rows = min(P_BM, t.m_end - t.m0);
@@ -438,8 +458,9 @@ __device__ __forceinline__ bool epi_all(bool p) {
   return r != 0;
 }
 
-template <int MODE>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+// CL = CTAs per cluster (2: one pair; 4: two pairs sharing the row tile).
+template <int MODE, int CL>
+__global__ void __launch_bounds__(THREADS, 1)
     ffn_gemm_pair_kernel(const __grid_constant__ CUtensorMap mapW0,
                          const __grid_constant__ CUtensorMap mapW1,
                          const __grid_constant__ CUtensorMap mapT, Args args) {
@@ -452,14 +473,18 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   const int warp = tid >> 5;
   const int lane = tid & 31;
   const uint32_t rank = cluster_ctarank();
-  const bool even = (rank == 0);
-  const int cluster = blockIdx.x >> 1;
-  const int n_clusters = gridDim.x >> 1;
+  const uint32_t rp = rank & 1u;     // rank within the pair
+  const uint32_t pr = rank >> 1;     // pair within the cluster (0 when CL == 2)
+  const uint32_t lead = rank & ~1u;  // the pair's even CTA (MMA issuer)
+  const bool even = (rp == 0);
+  const int cluster = blockIdx.x / CL;
+  const int n_clusters = gridDim.x / CL;
+  const int n_q = CL == 4 ? args.n_tiles / 2 : args.n_tiles;  // slice units per cluster tile
 
   if (tid == 0) {
     for (int i = 0; i < P_STAGES; ++i) {
       mbar_init(&s.full[i], 1);
-      mbar_init(&s.empty[i], 1);
+      mbar_init(&s.empty[i], CL / 2);  // one MMA commit per pair
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s.tfull[i], 1);
@@ -500,22 +525,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
   cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
   tc_fence_after();
   const uint32_t tmem_base = s.tmem_base;
-  const int total = s.mt_start[args.E] * args.n_tiles;
+  const int total = s.mt_start[args.E] * n_q;
   const int kblocks = args.K / BK;
   volatile int* abort = &s.abort;
   uint32_t issued_mask = 0, last_phase_bits = 0;
   bool mma_issued = false;
+  // tile -> (expert, this pair's column slice, row range)
+  auto tile_of = [&](int tile) {
+    Tile t = decode_pair(tile, s, args.E, n_q);
+    if (CL == 4) t.n = 2 * t.n + static_cast<int>(pr);
+    return t;
+  };
 
   if (warp == 0) {
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       for (int tile = cluster; tile < total && !*abort; tile += n_clusters) {
-        const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
-        const int trow = t.m0 + static_cast<int>(rank) * (tile_n(t) >> 1);  // N/2 rows per CTA
+        const Tile t = tile_of(tile);
+        const int trow = t.m0 + static_cast<int>(rp) * (tile_n(t) >> 1);  // N/2 rows per CTA
         const int wrow = (MODE == GATEUP)
-                             ? t.e * args.b_rows + t.n * 128 + 64 * static_cast<int>(rank)
-                             : t.e * args.b_rows + t.n * 256 + 128 * static_cast<int>(rank);
+                             ? t.e * args.b_rows + t.n * 128 + 64 * static_cast<int>(rp)
+                             : t.e * args.b_rows + t.n * 256 + 128 * static_cast<int>(rp);
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
             if (!*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 11);
@@ -524,7 +555,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           }
           uint8_t* sw = tiles + stage * P_STAGE_BYTES;
           uint8_t* st = sw + P_W_BYTES;
-          const uint32_t full_even = mapa_shared(smem_u32(&s.full[stage]), 0);
+          const uint32_t full_even = mapa_shared(smem_u32(&s.full[stage]), lead);
           if (even) mbar_arrive_expect_tx(&s.full[stage], 2 * P_STAGE_BYTES);
           if (MODE == GATEUP) {
             tma_load_2d_pair(sw, &mapW0, full_even, kb * BK, wrow);             // W1: lanes 0..63
@@ -532,7 +563,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           } else {
             tma_load_2d_pair(sw, &mapW0, full_even, kb * BK, wrow);
           }
-          tma_load_2d_pair(st, &mapT, full_even, kb * BK, trow);
+          if (CL == 4)  // rows 64 pr .. 64 pr + 63 of the box, to this CTA and its counterpart
+            tma_load_2d_pair_mc(st + pr * (P_T_BYTES / 2), &mapT, full_even, kb * BK,
+                                trow + 64 * static_cast<int>(pr),
+                                static_cast<uint16_t>((1u << rank) | (1u << (rank ^ 2u))));
+          else
+            tma_load_2d_pair(st, &mapT, full_even, kb * BK, trow);
           issued_mask |= 1u << stage;
           last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
@@ -553,7 +589,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           break;
         }
         tc_fence_after();
-        const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
+        const Tile t = tile_of(tile);
         const uint32_t idesc = idesc_bf16_f32(256, tile_n(t));
         const uint32_t d_tmem = tmem_base + slot * BN;
         bool ok = true;
@@ -572,11 +608,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             mma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32),
                           sdesc_kmajor_sw128(b0 + kk * 32), idesc, (kb | kk) != 0 ? 1u : 0u);
           mma_issued = true;
-          mma_commit_pair(&s.empty[stage], 0x3);
+          mma_commit_pair(&s.empty[stage], CL == 4 ? 0xF : 0x3);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        mma_commit_pair(&s.tfull[slot], 0x3);
+        mma_commit_pair(&s.tfull[slot], static_cast<uint16_t>(0x3u << (2 * pr)));
       }
     }
   } else {
@@ -597,7 +633,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
         break;
       }
       tc_fence_after();
-      const Tile t = decode_pair(tile, s, args.E, args.n_tiles);
+      const Tile t = tile_of(tile);
       const int rows = min(P_BM, t.m_end - t.m0);
       const int nchunks = (rows + 31) >> 5;
       const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
@@ -636,7 +672,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             ob[(keep + i + 1) * 64 + col] = static_cast<uint16_t>(pk >> 16);
           }
           epi_sync();
-          uint16_t* gcol = args.out + t.n * 128 + 64 * static_cast<int>(rank) + (et & 7) * 8;
+          uint16_t* gcol = args.out + t.n * 128 + 64 * static_cast<int>(rp) + (et & 7) * 8;
 #pragma unroll
           for (int p = 0; p < 2; ++p) {
             const int r = p * 16 + (et >> 3);
@@ -655,7 +691,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
             yb[(i + 1) * 128 + col] = static_cast<uint16_t>(pk >> 16);
           }
           epi_sync();
-          uint16_t* gcol = args.out + t.n * 256 + 128 * static_cast<int>(rank) + (et & 15) * 8;
+          uint16_t* gcol = args.out + t.n * 256 + 128 * static_cast<int>(rp) + (et & 15) * 8;
 #pragma unroll
           for (int p = 0; p < 4; ++p) {
             const int r = p * 8 + (et >> 4);
@@ -668,7 +704,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&s.tempty[slot]), 0));
+      if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&s.tempty[slot]), lead));
     }
   }
 
@@ -681,12 +717,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
           mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, args.limit_ns, never);
     }
     if (warp == 1 && lane == 0 && even && mma_issued) {
-      mma_commit_pair(&s.drain, 0x1);
+      mma_commit_pair(&s.drain, static_cast<uint16_t>(1u << rank));
       mbar_wait(&s.drain, 0, args.limit_ns, never);
     }
   }
   tc_fence_before();
-  cluster_sync();  // both CTAs finished: no more arrivals or copies into either
+  cluster_sync();  // every CTA finished: no more arrivals or copies into any
   tc_fence_after();
   if (warp == 1) tmem_dealloc_pair(tmem_base, TMEM_COLS);
 }
@@ -733,15 +769,20 @@ int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
   return ORDERMOE_OK;
 }
 
+template <int MODE, int CL>
+static cudaError_t pair_attr() {
+  return cudaFuncSetAttribute(gg::ffn_gemm_pair_kernel<MODE, CL>,
+                              cudaFuncAttributeMaxDynamicSharedMemorySize, gg::P_SMEM_BYTES);
+}
+
 static int ffn_attrs() {
   using namespace gg;
   static PerDevice cache;
   const cudaError_t attr_err = static_cast<cudaError_t>(per_device(cache, [] {
-    cudaError_t e = cudaFuncSetAttribute(ffn_gemm_pair_kernel<GATEUP>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(ffn_gemm_pair_kernel<DOWN>,
-                               cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_BYTES);
+    cudaError_t e = pair_attr<GATEUP, 2>();
+    if (e == cudaSuccess) e = pair_attr<DOWN, 2>();
+    if (e == cudaSuccess) e = pair_attr<GATEUP, 4>();
+    if (e == cudaSuccess) e = pair_attr<DOWN, 4>();
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(ffn_gemm_kernel<GATEUP>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
@@ -754,30 +795,55 @@ static int ffn_attrs() {
   return ORDERMOE_OK;
 }
 
-// CTA pairs that can be resident at once (not every SM may find a partner in
-// its GPC); the persistent grid never exceeds it, so no pair waits for another.
-static int max_resident_pairs() {
-  using namespace gg;
+static cudaLaunchConfig_t pair_config(int grid, int cl, cudaStream_t stream,
+                                      cudaLaunchAttribute* attr) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(gg::THREADS, 1, 1);
+  cfg.dynamicSmemBytes = gg::P_SMEM_BYTES;
+  cfg.stream = stream;
+  attr->id = cudaLaunchAttributeClusterDimension;
+  attr->val.clusterDim.x = cl;
+  attr->val.clusterDim.y = 1;
+  attr->val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cfg;
+}
+
+// Clusters of `cl` CTAs that can be resident at once (not every SM finds
+// partners in its GPC: on GB300, 76 clusters of 2 and 36 of 4); the persistent
+// grid never exceeds it, so no cluster waits for another. 0: none fit.
+template <int CL>
+static int max_resident_clusters() {
   static PerDevice cache;
   return per_device(cache, [] {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2 * (num_sms() / 2), 1, 1);
-    cfg.blockDim = dim3(THREADS, 1, 1);
-    cfg.dynamicSmemBytes = P_SMEM_BYTES;
     cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = 2;
-    attr.val.clusterDim.y = 1;
-    attr.val.clusterDim.z = 1;
-    cfg.attrs = &attr;
-    cfg.numAttrs = 1;
+    cudaLaunchConfig_t cfg = pair_config(CL * (num_sms() / CL), CL, nullptr, &attr);
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, ffn_gemm_pair_kernel<GATEUP>, &cfg) != cudaSuccess || n <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, gg::ffn_gemm_pair_kernel<gg::GATEUP, CL>, &cfg) !=
+            cudaSuccess ||
+        n < 0) {
       cudaGetLastError();
-      n = num_sms() / 2;
+      n = CL == 2 ? num_sms() / 2 : 0;
     }
-    return n < num_sms() / 2 ? n : num_sms() / 2;
+    return n < num_sms() / CL ? n : num_sms() / CL;
   });
+}
+
+// One launch of the CTA-pair kernel over `tiles` cluster tiles.
+template <int MODE, int CL>
+static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const CUtensorMap& t,
+                       const gg::Args& a, long long tiles, cudaStream_t stream, const char* what) {
+  const long long cmax = max_resident_clusters<CL>();
+  const long long clusters = tiles < cmax ? tiles : cmax;
+  cudaLaunchAttribute attr;
+  cudaLaunchConfig_t cfg =
+      pair_config(static_cast<int>(CL * (clusters > 0 ? clusters : 1)), CL, stream, &attr);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, gg::ffn_gemm_pair_kernel<MODE, CL>, w0, w1, t, a);
+  if (e != cudaSuccess) return cuda_fail(e, what);
+  OM_LAUNCHED(what);
+  return ORDERMOE_OK;
 }
 
 // Tile shape: CTA pairs (256-row tiles) when experts average at least 256
@@ -788,12 +854,6 @@ static bool use_pairs(int R, int E) { return (long long)R >= 256LL * E; }
 static int single_grid(long long tiles) {
   const int sms = num_sms();
   return static_cast<int>(tiles < sms ? tiles : sms);
-}
-
-static int pair_grid(long long tiles) {
-  const int pairs_max = max_resident_pairs();
-  const long long pairs = tiles < pairs_max ? tiles : pairs_max;
-  return static_cast<int>(2 * (pairs > 0 ? pairs : 1));
 }
 
 // H = SwiGLU(X_perm W1^T, X_perm W3^T) over the expert row ranges.
@@ -811,9 +871,14 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
     // weights on the MMA's M side in 64-row boxes of W1 and W3
     if ((rc = make_tmap_bf16(&mW1, W1, (uint64_t)E * dff, d, 64))) return rc;
     if ((rc = make_tmap_bf16(&mW3, W3, (uint64_t)E * dff, d, 64))) return rc;
-    const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
-    ffn_gemm_pair_kernel<GATEUP><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mW1, mW3, mX, a);
-    OM_LAUNCHED("ffn_gemm_pair_kernel<gate_up>");
+    const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
+    if (a.n_tiles % 2 == 0 && max_resident_clusters<4>() > 0) {
+      if ((rc = make_tmap_bf16(&mX, X_perm, R, d, 64))) return rc;  // half boxes, multicast
+      return launch_pair<GATEUP, 4>(mW1, mW3, mX, a, row_tiles * (a.n_tiles / 2), stream,
+                                    "ffn_gemm_pair_kernel<gate_up, 4>");
+    }
+    return launch_pair<GATEUP, 2>(mW1, mW3, mX, a, row_tiles * a.n_tiles, stream,
+                                  "ffn_gemm_pair_kernel<gate_up, 2>");
   } else {
     if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
     if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
@@ -837,9 +902,15 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   if ((rc = make_map(&mW2, W2, (uint64_t)E * d, dff))) return rc;
   if ((rc = make_map(&mH, H, R, dff))) return rc;
   if (use_pairs(R, E)) {
-    const long long tiles = ((long long)(R + P_BM - 1) / P_BM + E) * a.n_tiles;
-    ffn_gemm_pair_kernel<DOWN><<<pair_grid(tiles), THREADS, P_SMEM_BYTES, stream>>>(mW2, mW2, mH, a);
-    OM_LAUNCHED("ffn_gemm_pair_kernel<down>");
+    const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
+    if (a.n_tiles % 2 == 0 && max_resident_clusters<4>() > 0) {
+      CUtensorMap mHh;
+      if ((rc = make_tmap_bf16(&mHh, H, R, dff, 64))) return rc;  // half boxes, multicast
+      return launch_pair<DOWN, 4>(mW2, mW2, mHh, a, row_tiles * (a.n_tiles / 2), stream,
+                                  "ffn_gemm_pair_kernel<down, 4>");
+    }
+    return launch_pair<DOWN, 2>(mW2, mW2, mH, a, row_tiles * a.n_tiles, stream,
+                                "ffn_gemm_pair_kernel<down, 2>");
   } else {
     const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
     ffn_gemm_kernel<DOWN><<<single_grid(tiles), THREADS, SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
