@@ -52,6 +52,14 @@ def gate_up_traffic(workload):
     return GATE_UP_TRAFFIC["bytes"]
 
 
+def gate_up_kernel_name(R, E, dff):
+    """The gate/up kernel the library picks for R permuted rows (grouped_gemm.cu)."""
+    if R < 256 * E:
+        return "ffn_gemm_kernel<gate_up> (tcgen05, one CTA, 128-row tiles)"
+    cl = 4 if (dff // 128) % 2 == 0 else 2
+    return "ffn_gemm_pair_kernel<gate_up, %d> (tcgen05 CTA pairs, clusters of %d)" % (cl, cl)
+
+
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
@@ -59,6 +67,8 @@ def parse():
     p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="mixtral_prefill")
+    p.add_argument("--theta", type=float, default=None,
+                   help="similarity threshold theta of the grouping (default: the workload's)")
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
@@ -229,7 +239,12 @@ def run_ours(args, dist):
     device = torch.device("cuda", dist.local_rank)
     torch.cuda.set_device(device)
     B.lib()
-    w = synth.workload(args.workload, **({"n_cal": args.n_cal} if args.n_cal else {}))
+    over = {}
+    if args.n_cal:
+        over["n_cal"] = args.n_cal
+    if args.theta is not None:
+        over["theta"] = args.theta
+    w = synth.workload(args.workload, **over)
     if w.name == "decode_stack":
         return run_decode(args, dist, w, device)
     if w.name == "similarity":
@@ -348,7 +363,7 @@ def run_ours(args, dist):
                    "home": w.home, "seed": args.seed, "parallelism": "replicas",
                    "l2": "inputs larger than L2: %.2f GB of expert weights read every step"
                          % (3 * E * d * dff * 2 / 1e9)},
-        "roofline": {"kernel": "ffn_gemm_pair_kernel<gate_up, 4> (tcgen05 CTA pairs, clusters of 4)", "bound": "tensor",
+        "roofline": {"kernel": gate_up_kernel_name(T * k, E, dff), "bound": "tensor",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(achieved / peak, 4), "traffic": gate_up_traffic(w.name),
                      "peak_source": "%s bf16_tflops_sustained" % pk_kind,

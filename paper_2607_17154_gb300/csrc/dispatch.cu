@@ -48,40 +48,74 @@ __global__ void __launch_bounds__(kChunk) chunk_hist_kernel(const int32_t* __res
 
 // One block of 1024 threads. Warp w scans the chunk counts of experts w and
 // w + 32 with warp shuffles (32 chunks at a time, carrying the running sum),
-// then the expert totals are scanned into offsets and added back.
+// then warp 0 scans the expert totals into offsets and they are added back.
+// With `staged` the histogram is first copied into shared memory with
+// coalesced loads, transposed to [E][P] with an odd pitch P (a warp's 32
+// consecutive chunks of one expert then fall in 32 banks), and written back
+// coalesced; otherwise each warp reads its expert's column, E words apart.
+constexpr int kScanStageBytes = 96 * 1024;
+
 __global__ void __launch_bounds__(1024) chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks,
-                                                          int E, int32_t* __restrict__ offsets) {
+                                                          int E, int32_t* __restrict__ offsets,
+                                                          int staged) {
+  extern __shared__ int hs[];  // staged: [E][P]
   __shared__ int total[64];
   __shared__ int start[65];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int P = nchunks | 1;
+  if (staged) {
+    for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) {
+      const int b = i / E;
+      hs[(i - b * E) * P + b] = hist[i];
+    }
+    __syncthreads();
+  }
   for (int e = warp; e < E; e += 32) {
     int carry = 0;
     for (int b0 = 0; b0 < nchunks; b0 += 32) {
       const int b = b0 + lane;
-      const int v = (b < nchunks) ? hist[(size_t)b * E + e] : 0;
+      const int v = (b < nchunks) ? (staged ? hs[e * P + b] : hist[(size_t)b * E + e]) : 0;
       int incl = v;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int u = __shfl_up_sync(0xffffffffu, incl, o);
         if (lane >= o) incl += u;
       }
-      if (b < nchunks) hist[(size_t)b * E + e] = carry + incl - v;
+      if (b < nchunks) {
+        if (staged)
+          hs[e * P + b] = carry + incl - v;
+        else
+          hist[(size_t)b * E + e] = carry + incl - v;
+      }
       carry += __shfl_sync(0xffffffffu, incl, 31);
     }
     if (lane == 0) total[e] = carry;
   }
   __syncthreads();
-  if (threadIdx.x == 0) {
-    int acc = 0;
-    for (int x = 0; x < E; ++x) {
-      start[x] = acc;
-      acc += total[x];
+  if (warp == 0) {  // exclusive scan of the E <= 64 totals, two per lane
+    const int t0 = (2 * lane < E) ? total[2 * lane] : 0;
+    const int t1 = (2 * lane + 1 < E) ? total[2 * lane + 1] : 0;
+    int incl = t0 + t1;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int u = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += u;
     }
-    start[E] = acc;
+    const int excl = incl - t0 - t1;
+    if (2 * lane < E) start[2 * lane] = excl;
+    if (2 * lane + 1 < E) start[2 * lane + 1] = excl + t0;
+    if (lane == 31) start[E] = incl;
   }
   __syncthreads();
   if (threadIdx.x <= E) offsets[threadIdx.x] = start[threadIdx.x];
-  for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) hist[i] += start[i % E];
+  if (staged) {
+    for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) {
+      const int b = i / E, e = i - b * E;
+      hist[i] = hs[e * P + b] + start[e];
+    }
+  } else {
+    for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) hist[i] += start[i % E];
+  }
 }
 
 __global__ void __launch_bounds__(kChunk) rank_kernel(
@@ -290,7 +324,16 @@ int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int 
   } else {
     chunk_hist_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, E, hist);
     OM_LAUNCHED("chunk_hist_kernel");
-    chunk_scan_kernel<<<1, 1024, 0, stream>>>(hist, nchunks, E, offsets);
+    static PerDevice scan_attr;
+    const int attr_ok = per_device(scan_attr, [] {
+      return static_cast<int>(cudaFuncSetAttribute(
+          chunk_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kScanStageBytes));
+    });
+    if (attr_ok != static_cast<int>(cudaSuccess)) cudaGetLastError();
+    const size_t stage_bytes = (size_t)(nchunks | 1) * E * sizeof(int32_t);
+    const int staged = attr_ok == static_cast<int>(cudaSuccess) && stage_bytes <= kScanStageBytes;
+    chunk_scan_kernel<<<1, 1024, staged ? stage_bytes : 0, stream>>>(hist, nchunks, E, offsets,
+                                                                     staged);
     OM_LAUNCHED("chunk_scan_kernel");
     rank_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, hist, row_token, row_of);
     OM_LAUNCHED("rank_kernel");

@@ -215,8 +215,10 @@ __device__ __forceinline__ void select_token(
       }
       return;
     }
-  // top-k by (logit desc, index asc)
+  // top-k by (logit desc, index asc); vtop keeps each chosen logit, so no
+  // lookup lg[idx[j]] (a run-time index would put lg[] in local memory)
   int idx[ORDERMOE_MAX_TOPK];
+  float vtop[ORDERMOE_MAX_TOPK];
   unsigned long long used_targets = 0;
   for (int j = 0; j < k; ++j) {
     int best = -1;
@@ -228,6 +230,7 @@ __device__ __forceinline__ void select_token(
         bv = lg[e];
       }
     idx[j] = best;
+    vtop[j] = bv;
     used_targets |= 1ull << best;
   }
   // softmax over all E in fp32; gate weights of the k slots
@@ -242,11 +245,7 @@ __device__ __forceinline__ void select_token(
   float wsel[ORDERMOE_MAX_TOPK];
   float ssel = 0.0f;
   for (int j = 0; j < k; ++j) {
-    float v = 0.0f;
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e == idx[j]) v = lg[e];
-    wsel[j] = expf(v - lmax) / denom;
+    wsel[j] = expf(vtop[j] - lmax) / denom;
     ssel += wsel[j];
   }
   for (int j = 0; j < k; ++j) {
@@ -312,7 +311,10 @@ __device__ __forceinline__ void select_token(
     chosen_expert[(size_t)t * k + j] = kstar;
     chosen_server[(size_t)t * k + j] = static_cast<uint8_t>(mstar);
     kind_out[(size_t)t * k + j] = static_cast<uint8_t>(kd);
-    kind_count[kd]++;
+    if (kd == 0) ++kind_count[0];  // constant indices: kind_count[] stays in registers
+    else if (kd == 1) ++kind_count[1];
+    else if (kd == 2) ++kind_count[2];
+    else ++kind_count[3];
   }
   if (loc != nullptr) {
     loc[t] = static_cast<uint8_t>(first_server);
@@ -351,8 +353,11 @@ __global__ void __launch_bounds__(128) select_kernel(
     float lg[EMAX];
 #pragma unroll
     for (int e = 0; e < EMAX; ++e) lg[e] = (e < E) ? logits_in[(size_t)t * E + e] : 0.0f;
-    if (logits_out != nullptr)
-      for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
+    if (logits_out != nullptr) {
+#pragma unroll
+      for (int e = 0; e < EMAX; ++e)  // constant indices keep lg[] in registers
+        if (e < E) logits_out[(size_t)t * E + e] = lg[e];
+    }
     select_token<EMAX>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
                        topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count,
                        la.H > 1);
@@ -826,8 +831,11 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       for (int c = 0; c < NE; ++c) lg[c] += src[c];
     }
     if (t < T && tables_ok) {
-      if (logits_out != nullptr)
-        for (int e = 0; e < E; ++e) logits_out[(size_t)t * E + e] = lg[e];
+      if (logits_out != nullptr) {
+#pragma unroll
+        for (int e = 0; e < NE; ++e)  // constant indices keep lg[] in registers
+          if (e < E) logits_out[(size_t)t * E + e] = lg[e];
+      }
       const int M = reinterpret_cast<const int32_t*>(tab)[2];
       const float qbar = reinterpret_cast<const float*>(tab)[5];
       const float* gA = reinterpret_cast<const float*>(tab + off_a(E));

@@ -156,7 +156,9 @@ def test_router_logits_match_oracle(T, d, E):
 # ------------------------------------------------------------------ permutation
 
 @pytest.mark.parametrize("T,k,E,d", [(64, 2, 8, 256), (1000, 6, 64, 64), (1, 1, 1, 8), (333, 3, 7, 40),
-                                     (4096, 2, 8, 4096)])
+                                     (4096, 2, 8, 4096),
+                                     (8192, 6, 64, 64),     # 192 chunks: histogram staged in shared memory
+                                     (20000, 6, 64, 64)])   # 469 chunks x 64: too large to stage
 def test_dispatch_bit_exact(T, k, E, d):
     rng = np.random.default_rng(T * k + E)
     chosen = rng.integers(0, E, (T, k)).astype(np.int32)
