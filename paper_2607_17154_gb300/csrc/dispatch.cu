@@ -200,13 +200,20 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict
        it += warps_total) {
     const int t = static_cast<int>(it / parts);
     const int part = static_cast<int>(it - (int64_t)t * parts);
+    // slot loops unrolled to the largest k with a j < k guard: constant indices keep
+    // rows[] and ws[] in registers and let the loads of later slots issue early
     int rows[ORDERMOE_MAX_TOPK];
     float ws[ORDERMOE_MAX_TOPK];
     bool ok = true;
-    for (int j = 0; j < k; ++j) {
-      rows[j] = row_of[(size_t)t * k + j];
-      ws[j] = w[(size_t)t * k + j];
-      if (rows[j] < 0 || (int64_t)rows[j] >= (int64_t)T * k) ok = false;
+#pragma unroll
+    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
+      rows[j] = 0;
+      ws[j] = 0.0f;
+      if (j < k) {
+        rows[j] = row_of[(size_t)t * k + j];
+        ws[j] = w[(size_t)t * k + j];
+        if (rows[j] < 0 || (int64_t)rows[j] >= (int64_t)T * k) ok = false;
+      }
     }
     if (!ok) {  // a row index outside Y_perm: report, leave y[t] untouched
       if (lane == 0 && part == 0) report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, t);
@@ -218,7 +225,9 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict
 #pragma unroll
       for (int x = 0; x < 8; ++x) acc[u][x] = 0.0f;
     const int v0 = part * kCombVec + lane;
-    for (int j = 0; j < k; ++j) {
+#pragma unroll
+    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
+      if (j >= k) break;
       const uint4* src = reinterpret_cast<const uint4*>(Yp + (size_t)rows[j] * d);
       uint4 yv[4];
 #pragma unroll
