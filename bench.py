@@ -687,8 +687,8 @@ def run_similarity(args, dist, w, device):
     pi = torch.as_tensor(synth.token_shares(synth.homes(65536, w.M, seed, "zipf1.1"), w.M),
                          dtype=torch.float64).to(device)
 
-    def step():
-        B.ordermoe_similarity(Wr, Xcal, L, E, d, N, w.k, sim, counts, ws)
+    def step():  # no look-ahead transitions follow: the calibration logits are not kept
+        B.ordermoe_similarity_no_logits(Wr, Xcal, L, E, d, N, w.k, sim, counts, ws)
         B.ordermoe_place(sim, counts, L, E, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5,
                          0.5, 0.5, p, C, group, ng, theta, imp, x, used, st)
         B.ordermoe_replicate(group, imp, p, C, pi, L, E, w.M, x, used, reps)

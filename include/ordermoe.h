@@ -330,6 +330,17 @@ int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E
  * first N * L * E * 4 bytes of its workspace hold the calibration logits
  * H[n][l][e] in fp32, token-major: the input ordermoe_transitions takes. */
 
+/* ordermoe_similarity without the calibration logits: the same arguments,
+ * workspace size and results (sim and counts bit for bit), but the first
+ * N * L * E * 4 bytes of the workspace are left undefined, which saves
+ * writing them (1.6 GB for 24 layers x 64 experts x 262144 tokens) when no
+ * ordermoe_transitions call follows. Where the tensor-core path does not apply
+ * (E not in {8, 16, 32, 64}) the logits are computed and kept anyway. */
+int ordermoe_similarity_no_logits(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
+                                  int64_t N, int k_freq, float* sim, int32_t* counts,
+                                  void* workspace, size_t workspace_bytes,
+                                  ordermoe_stream_t stream);
+
 /* Expert transition statistics, Eq. 41, from calibration logits
  * [N][L][E] f32 (token-major, layer-stacked): n_l(k -> k') counts, for every
  * token, each pair (k in its top-k_freq at layer l, k' in its top-k_freq at

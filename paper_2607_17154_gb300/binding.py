@@ -41,6 +41,7 @@ _SIGNATURES = {
     "ordermoe_combine": ([_P, _P, _P, _I, _I, _I, _P, _P], _I),
     "ordermoe_similarity_workspace_bytes": ([_I, _I, _I64], _SZ),
     "ordermoe_similarity": ([_P, _P, _I, _I, _I, _I64, _I, _P, _P, _P, _SZ, _P], _I),
+    "ordermoe_similarity_no_logits": ([_P, _P, _I, _I, _I, _I64, _I, _P, _P, _P, _SZ, _P], _I),
     "ordermoe_expert_counts": ([_P, _I64, _I, _I, _P, _P], _I),
     "ordermoe_place": ([_P, _P, _I, _I, _I, _D, _D, _D, _D, _D, _D, _D, _P, _P, _P, _P, _P, _P,
                         _P, _P, _P, _P, _SZ, _P], _I),
@@ -221,6 +222,17 @@ def ordermoe_similarity(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, 
                                    _ptr(counts), _ptr(workspace),
                                    workspace.numel() * workspace.element_size(), _stream(stream))
     _check("ordermoe_similarity", rc)
+
+
+def ordermoe_similarity_no_logits(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace,
+                                  stream=None):
+    _dt(W_r, torch.bfloat16, "W_r"); _dt(X_cal, torch.bfloat16, "X_cal")
+    _dt(sim, torch.float32, "sim"); _dt(counts, torch.int32, "counts")
+    rc = lib().ordermoe_similarity_no_logits(_ptr(W_r), _ptr(X_cal), L, E, d, N, k_freq,
+                                             _ptr(sim), _ptr(counts), _ptr(workspace),
+                                             workspace.numel() * workspace.element_size(),
+                                             _stream(stream))
+    _check("ordermoe_similarity_no_logits", rc)
 
 
 def ordermoe_expert_counts(logits, N, E, k_freq, counts, stream=None):

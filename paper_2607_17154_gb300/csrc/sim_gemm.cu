@@ -89,7 +89,7 @@ struct LArgs {
   int n_tiles;      // 256-column slices
   int L;
   int kf;           // k_freq of Eq. 5
-  float* H;         // [N][C] fp32
+  float* H;         // [N][C] fp32, or null: not written
   uint16_t* hi;     // [C][ldT] bf16
   uint16_t* lo;     // [C][ldT] bf16
   int ldT;
@@ -270,7 +270,7 @@ __global__ void __launch_bounds__(L_THREADS, 1)
           float4* dst = reinterpret_cast<float4*>(orow + cb);
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            if (4 * i < nv)
+            if (args.H != nullptr && 4 * i < nv)  // logits kept only when asked for
               dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
                                    __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
 #pragma unroll

@@ -564,11 +564,11 @@ extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
   return up(h) + planes + up(g) + up(gd);
 }
 
-extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
-                                   int64_t N, int k_freq, float* sim, int32_t* counts,
-                                   void* workspace, size_t workspace_bytes,
-                                   ordermoe_stream_t stream) {
-  OM_TRACE();
+// keep_logits: leave the fp32 calibration logits H in the workspace (the
+// input of ordermoe_transitions); the tensor-core path can skip writing them.
+static int similarity_impl(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
+                           int64_t N, int k_freq, float* sim, int32_t* counts, void* workspace,
+                           size_t workspace_bytes, bool keep_logits, cudaStream_t stream) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: need L >= 1, 1 <= k_freq <= E <= 64");
   if (d <= 0 || d % 64 != 0)
@@ -599,8 +599,9 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
   if (tc) {
     // tensor-core path: logits with fused counts and hi/lo planes, then the Gram
     const int nsplit = sim_tc_nsplit(L, E, N);
-    int rc = sim_tc_launch(X_cal, static_cast<int>(N), W_r, L, E, d, k_freq, H, hi, lo,
-                           static_cast<int>(ldT), counts, gpart, nsplit, stream);
+    int rc = sim_tc_launch(X_cal, static_cast<int>(N), W_r, L, E, d, k_freq,
+                           keep_logits ? H : nullptr, hi, lo, static_cast<int>(ldT), counts, gpart,
+                           nsplit, stream);
     if (rc) return rc;
     gram_reduce_kernel<<<dim3(L, 16), 256, 0, stream>>>(gpart, nsplit, G);
     OM_LAUNCHED("gram_reduce_kernel");
@@ -626,6 +627,24 @@ extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, i
   sim_finish_kernel<<<L, 256, 0, stream>>>(G, E, sim);
   OM_LAUNCHED("sim_finish_kernel");
   return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_similarity(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
+                                   int64_t N, int k_freq, float* sim, int32_t* counts,
+                                   void* workspace, size_t workspace_bytes,
+                                   ordermoe_stream_t stream) {
+  OM_TRACE();
+  return similarity_impl(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, workspace_bytes,
+                         true, stream);
+}
+
+extern "C" int ordermoe_similarity_no_logits(const uint16_t* W_r, const uint16_t* X_cal, int L,
+                                             int E, int d, int64_t N, int k_freq, float* sim,
+                                             int32_t* counts, void* workspace,
+                                             size_t workspace_bytes, ordermoe_stream_t stream) {
+  OM_TRACE();
+  return similarity_impl(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, workspace_bytes,
+                         false, stream);
 }
 
 extern "C" int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq,

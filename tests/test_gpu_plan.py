@@ -54,6 +54,30 @@ def test_similarity_matches_oracle(L, E, d, N, kf, K):
         assert np.abs(counts[l] - ref_counts).sum() <= max(2, N // 500), (counts[l], ref_counts)
 
 
+@pytest.mark.parametrize("L,E,d,N,kf", [(3, 64, 512, 3000, 6), (2, 16, 128, 700, 3), (2, 12, 128, 1000, 3)])
+def test_similarity_no_logits_same_results(L, E, d, N, kf):
+    # the entry point that skips the fp32 logits gives the same sim and counts bit for bit
+    Wr = torch.stack([synth.router_weights(E, d, 4, seed=20 + l) for l in range(L)]).to(DEV).contiguous()
+    Xcal = synth.calibration(N, d, seed=7 * L + E).to(DEV)
+    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+    sim_a = torch.empty(L, E, E, dtype=torch.float32, device=DEV)
+    cnt_a = torch.empty(L, E, dtype=torch.int32, device=DEV)
+    B.ordermoe_similarity(Wr, Xcal, L, E, d, N, kf, sim_a, cnt_a, ws)
+    logits = ws[: N * L * E * 4].view(torch.float32).view(N, L * E).clone()
+    ws.fill_(0xFF)  # the logits region is not rewritten by the second call
+    sim_b = torch.empty_like(sim_a)
+    cnt_b = torch.empty_like(cnt_a)
+    B.ordermoe_similarity_no_logits(Wr, Xcal, L, E, d, N, kf, sim_b, cnt_b, ws)
+    torch.cuda.synchronize()
+    assert torch.equal(sim_a, sim_b) and torch.equal(cnt_a, cnt_b)
+    assert torch.isfinite(logits).all()
+    region = ws[: N * L * E * 4]
+    if E in (8, 16, 32, 64):  # tensor-core path: the logits are skipped
+        assert (region == 0xFF).all()
+    else:  # the CUDA-core path needs them and keeps them
+        assert torch.equal(region.view(torch.float32).view(N, L * E), logits)
+
+
 def test_expert_counts_given_logits_bit_exact():
     rng = np.random.default_rng(3)
     for N, E, kf in [(5000, 64, 6), (100, 8, 2), (33, 5, 5)]:
