@@ -1,7 +1,10 @@
 // Grouped SwiGLU expert FFN on sm_103a tensor cores (tcgen05 + TMEM + TMA).
 //
-// Two persistent warp-specialised kernels over the expert-contiguous rows of
-// ordermoe_dispatch, with the per-expert row ranges read on the device:
+// Persistent warp-specialised kernels over the expert-contiguous rows of
+// ordermoe_dispatch, with the per-expert row ranges read on the device: a
+// one-CTA kernel for small batches (described here) and a CTA-pair kernel
+// with the weights on the MMA's M side for large ones (its own section below).
+// One-CTA kernel:
 //   gate/up: H[rows of e, n0:n0+128] = bf16(silu(X W1_e^T) * (X W3_e^T)) for a
 //            128-column slice n0 of d_ff. One tcgen05.mma of N = 256 computes
 //            the gate (TMEM columns 0..127) and up (128..255) projections from
@@ -846,9 +849,11 @@ static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const CUten
   return ORDERMOE_OK;
 }
 
-// Tile shape: CTA pairs (256-row tiles) when experts average at least 256
-// rows; otherwise single CTAs with 128-row tiles, which compute fewer padding
-// rows for small batches (a decode step: ~32 rows per expert).
+// Tile shape: CTA pairs (256 weight rows x up to 256 permuted rows, in
+// clusters of 2 or 4) when experts average at least 256 rows; otherwise single
+// CTAs with 128-row tiles and the rows on the M side (a decode step: ~32 rows
+// per expert, where the weights are streamed once and the MMA shape hardly
+// matters).
 static bool use_pairs(int R, int E) { return (long long)R >= 256LL * E; }
 
 static int single_grid(long long tiles) {
