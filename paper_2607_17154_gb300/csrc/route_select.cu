@@ -461,6 +461,69 @@ __device__ __forceinline__ float phi_term2_memo(const uint8_t* __restrict__ tnex
   return __fmul_rn(p, best);
 }
 
+// lookahead_phi<2> with its deepest level read from U / qmax1 as in
+// phi_term2_memo (the same fp32 operations in the same order).
+__device__ float lookahead_phi2_memo(const uint8_t* __restrict__ tnext, size_t stride,
+                                     const float* __restrict__ P, int E, int M, int a, int m,
+                                     int kx, float qacc, float qbar, const float* U,
+                                     const float* qmax1) {
+  float acc = 0.0f;
+  for (int kt = 0; kt < E; ++kt) {
+    if (__ldg(P + (size_t)kx * E + kt) == 0.0f) continue;
+    acc = __fadd_rn(acc, phi_term2_memo(tnext, stride, P, E, M, a, m, kx, kt, qacc, qbar, U, qmax1));
+  }
+  return acc;
+}
+
+// H = 4: the term of Eq. 42 with Phi^(2)(m2, k2, q2) read from a per-token
+// table U2[m2][k2] (evaluated with q2 = 0) whenever no budget check inside it
+// can fail: every loss it adds at its own level is at most qmax2[k2] and every
+// loss one level deeper at most qmaxL1 (losses are not negative; -inf: none),
+// so fadd(q2, qmax2[k2]) <= Qbar and fadd(that, qmaxL1) <= Qbar mean every
+// check passes for q2 as for 0 (fadd is monotone) and the value is the same.
+// Otherwise Phi^(2) is evaluated, its deepest level again from U1 when free.
+__device__ __forceinline__ float phi_term3_memo(const uint8_t* __restrict__ tnext, size_t stride,
+                                                const float* __restrict__ P, int E, int M, int a,
+                                                int m, int kx, int kt, float qacc, float qbar,
+                                                const float* U2, const float* qmax2, float qmaxL1,
+                                                const float* U1, const float* qmax1) {
+  const float p = __ldg(P + (size_t)kx * E + kt);
+  if (p == 0.0f) return 0.0f;
+  const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
+  const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
+  const float* A1 = reinterpret_cast<const float*>(tnext + off_a(E));
+  const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
+  const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
+  float best = INFINITY;
+  unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);
+  while (cand) {
+    const int kk = __ffsll(static_cast<long long>(cand)) - 1;
+    cand &= cand - 1;
+    const bool exact = (kk == kt);
+    float cq = 0.0f, q2 = qacc;
+    if (!exact) {
+      const float qk = __ldg(Q1 + kt * E + kk);
+      if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
+      q2 = __fadd_rn(qacc, qk);
+      cq = __ldg(C1 + kt * E + kk);
+    }
+    const float qa = __fadd_rn(q2, qmax2[kk]);
+    const float q3max = (qmax2[kk] == -INFINITY) ? q2 : qa;  // largest loss entering level 1
+    const bool free = qa <= qbar && __fadd_rn(q3max, qmaxL1) <= qbar;
+    uint32_t pm = __ldg(pm1 + kk);
+    while (pm) {
+      const int m2 = __ffs(pm) - 1;
+      pm &= pm - 1;
+      const float phi2 = free ? U2[m2 * E + kk]
+                              : lookahead_phi2_memo(tnext + stride, stride, P + E * E, E, M, a, m2,
+                                                    kk, q2, qbar, U1, qmax1);
+      const float c = __fadd_rn(__fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq), phi2);
+      best = fminf(best, c);
+    }
+  }
+  return __fmul_rn(p, best);
+}
+
 __device__ __forceinline__ float phi_term_h(const Lookahead& la, const uint8_t* tab, int E, int M,
                                             int a, int m, int kx, int kt, float qacc, float qbar) {
   switch (la.H) {
@@ -480,8 +543,8 @@ struct LaSmem {
   float cost0[kLaMaxCand];    // A(a, s, m) + Cq: Eq. 43 without Phi
   float qn[kLaMaxCand];       // accumulated loss after this candidate (Eq. 44)
   float terms[kLaTerms];
-  float U[32 * 64];           // H = 3: Phi^(1)(m2, k2) with every budget check passing
-  float qmax1[64];            // H = 3: largest substitute loss Phi^(1)(., k2) can consider
+  float U[32 * 64];           // H = 3, 4: Phi^(1)(m2, k2) with every budget check passing
+  float qmax1[64];            // H = 3, 4: largest substitute loss Phi^(1)(., k2) can consider
   unsigned long long best;
   int n;
 };
@@ -521,29 +584,49 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
   const int cpp = kLaTerms / E;  // candidates per pass
   float q = (qhat != nullptr) ? qhat[t] : 0.0f;
   const bool memo = (la.H == 3) && !(q < 0.0f);  // accumulated losses are never negative
-  if (memo) {
-    // the deepest level's tables (layer l + 2) and transitions (l + 1 -> l + 2)
-    const uint8_t* t2 = tab + 2 * la.stride;
-    const float* P2 = la.P + (size_t)E * E;
-    const float* Q2 = reinterpret_cast<const float*>(t2 + kOffQtab);
-    const unsigned long long* sb2 = reinterpret_cast<const unsigned long long*>(t2 + kOffSubst);
-    for (int k2 = tid; k2 < E; k2 += blockDim.x) {
-      float mx = -INFINITY;
-      for (int kt = 0; kt < E; ++kt) {
-        if (__ldg(P2 + (size_t)k2 * E + kt) == 0.0f) continue;
-        unsigned long long sb = __ldg(sb2 + kt);
-        while (sb) {
-          const int k3 = __ffsll(static_cast<long long>(sb)) - 1;
-          sb &= sb - 1;
-          mx = fmaxf(mx, __ldg(Q2 + kt * E + k3));
-        }
+  const bool memo4 = (la.H == 4) && !(q < 0.0f);
+  float* U2 = s_dyn + 2 * E * E;  // H = 4: Phi^(2)(m2, k2) with every check passing, [32][E]
+  float* qmax2 = U2 + 32 * E;     // H = 4: largest loss Phi^(2)(., k2) adds at its level
+  float qmaxL1 = -INFINITY;       // H = 4: largest such loss one level deeper
+  // the largest substitute loss lookahead_phi<1> on tables tl and transitions Pl
+  // can add for expert kx (targets with P(kx -> k') != 0; -inf: none)
+  auto qmax_of = [&](const uint8_t* tl, const float* Pl, int kx) {
+    const float* Ql = reinterpret_cast<const float*>(tl + kOffQtab);
+    const unsigned long long* sbl = reinterpret_cast<const unsigned long long*>(tl + kOffSubst);
+    float mx = -INFINITY;
+    for (int kt = 0; kt < E; ++kt) {
+      if (__ldg(Pl + (size_t)kx * E + kt) == 0.0f) continue;
+      unsigned long long sb = __ldg(sbl + kt);
+      while (sb) {
+        const int k3 = __ffsll(static_cast<long long>(sb)) - 1;
+        sb &= sb - 1;
+        mx = fmaxf(mx, __ldg(Ql + kt * E + k3));
       }
-      cs.qmax1[k2] = mx;
     }
+    return mx;
+  };
+  if (memo || memo4) {
+    // the deepest level's tables (layer l + H - 1) and transitions into it
+    const int dl = la.H - 1;
+    const uint8_t* td = tab + dl * la.stride;
+    const float* Pd = la.P + (size_t)(dl - 1) * E * E;
+    for (int k2 = tid; k2 < E; k2 += blockDim.x) cs.qmax1[k2] = qmax_of(td, Pd, k2);
     for (int i = tid; i < M * E; i += blockDim.x) {
       const int m2 = i / E, k2 = i - (i / E) * E;
-      cs.U[i] = lookahead_phi<1>(tab + 2 * la.stride, la.stride, P2, E, M, a, m2, k2, 0.0f, qbar);
+      cs.U[i] = lookahead_phi<1>(td, la.stride, Pd, E, M, a, m2, k2, 0.0f, qbar);
     }
+    __syncthreads();
+  }
+  if (memo4) {
+    // one level up (layer l + 2): Phi^(2) at q = 0, through the U table above
+    const uint8_t* t2 = tab + 2 * la.stride;
+    const float* P2 = la.P + (size_t)E * E;
+    for (int k2 = tid; k2 < E; k2 += blockDim.x) qmax2[k2] = qmax_of(t2, P2, k2);
+    for (int i = tid; i < M * E; i += blockDim.x) {
+      const int m2 = i / E, k2 = i - (i / E) * E;
+      U2[i] = lookahead_phi2_memo(t2, la.stride, P2, E, M, a, m2, k2, 0.0f, qbar, cs.U, cs.qmax1);
+    }
+    for (int k3 = 0; k3 < E; ++k3) qmaxL1 = fmaxf(qmaxL1, cs.qmax1[k3]);
     __syncthreads();
   }
   int first_server = s;
@@ -588,9 +671,12 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
         const int c = base + i / E, kt = i - (i / E) * E;
         const uint32_t code = cs.code[c];
         const int cm = static_cast<int>((code >> 8) & 0xFFu), ck = static_cast<int>(code & 0xFFu);
-        cs.terms[i] = memo ? phi_term2_memo(tab + la.stride, la.stride, la.P, E, M, a, cm, ck, kt,
-                                            cs.qn[c], qbar, cs.U, cs.qmax1)
-                           : phi_term_h(la, tab, E, M, a, cm, ck, kt, cs.qn[c], qbar);
+        cs.terms[i] = memo    ? phi_term2_memo(tab + la.stride, la.stride, la.P, E, M, a, cm, ck,
+                                               kt, cs.qn[c], qbar, cs.U, cs.qmax1)
+                      : memo4 ? phi_term3_memo(tab + la.stride, la.stride, la.P, E, M, a, cm, ck,
+                                               kt, cs.qn[c], qbar, U2, qmax2, qmaxL1, cs.U,
+                                               cs.qmax1)
+                              : phi_term_h(la, tab, E, M, a, cm, ck, kt, cs.qn[c], qbar);
       }
       __syncthreads();
       for (int cl = tid; cl < nc; cl += blockDim.x) {
@@ -905,6 +991,7 @@ static int launch_lookahead_select(const int32_t* topk_idx, int T, int E, int k,
                                    uint8_t* chosen_server, uint8_t* kind, int32_t* counters,
                                    size_t tab_smem, cudaStream_t stream) {
   if (T <= 0) return ORDERMOE_OK;
+  if (la.H == 4) tab_smem += sizeof(float) * (32 * E + E);  // the Phi^(2) table and its bounds
   cudaFuncSetAttribute(lookahead_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)tab_smem);
   lookahead_select_kernel<<<T, kLaThreads, tab_smem, stream>>>(

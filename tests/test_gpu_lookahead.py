@@ -63,7 +63,10 @@ def stack_tables(rng, L, E, M, qbar, cheap_links):
 
 
 @pytest.mark.parametrize("E,M,k,H,cheap", [(8, 4, 2, 1, True), (8, 4, 2, 2, True), (8, 4, 2, 3, True),
-                                           (16, 4, 3, 3, False), (6, 3, 2, 4, True), (32, 8, 2, 2, True)])
+                                           (16, 4, 3, 3, False), (6, 3, 2, 4, True), (32, 8, 2, 2, True),
+                                           # H = 4: the Phi^(2) table used (cheap substitutes) and
+                                           # bypassed when budget checks can fail (dear ones)
+                                           (8, 4, 2, 4, False), (16, 4, 3, 4, True), (12, 5, 2, 4, False)])
 def test_route_select_lookahead_given_logits_bit_exact(E, M, k, H, cheap):
     rng = np.random.default_rng(E * 10 + H)
     T = 300
