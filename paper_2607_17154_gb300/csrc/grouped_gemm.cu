@@ -384,23 +384,26 @@ __global__ void __launch_bounds__(THREADS, 1)
 // TMA loads, and the other pair's multicast, complete on it), empty[s] and tfull[b] (both CTAs, arrived by the
 // even CTA's MMA commits multicast to the pair, or to all four CTAs for
 // empty[s] in a cluster of 4), tempty[b] (even CTA, one
-// arrive per epilogue warp of either CTA). Named barrier 1 (the 128 epilogue
-// threads of a CTA) orders the shared-memory exchange; the decision to stop
-// is taken with a barrier reduction so the four epilogue warps always leave
-// together.
+// arrive per epilogue warp of either CTA). The gate/up epilogue runs on two
+// groups of four warps that take alternate 32-row chunks, so two chunks are
+// in flight (short-K tiles are otherwise epilogue-bound); down runs one group.
+// Named barriers 1 and 2 (the 128 threads of a group) order each group's
+// shared-memory exchange, and the decision to stop is a barrier reduction over
+// all epilogue warps (barrier 3), so they always leave together.
 constexpr int P_BM = 256;            // permuted rows (N side) per tile
-constexpr int P_STAGES = 6;
+constexpr int P_MAX_STAGES = 6;
 constexpr int P_W_BYTES = 128 * BK * 2;   // 128 weight rows per CTA and K block
 constexpr int P_T_BYTES = 128 * BK * 2;   // one box of 128 permuted rows per CTA
 constexpr int P_STAGE_BYTES = P_W_BYTES + P_T_BYTES;
 constexpr int P_X_PITCH = 17;             // floats per exchange row (odd: no bank conflicts)
 constexpr int P_XBUF_FLOATS = 128 * P_X_PITCH;
-constexpr int P_EPI_BYTES = 2 * (P_XBUF_FLOATS * 4 + 32 * 64 * 2);  // gate/up; down needs 2 x 32 x 128 x 2
-static_assert(P_EPI_BYTES >= 2 * 32 * 128 * 2, "down staging fits");
+constexpr int P_EPI_GROUP_BYTES = 2 * (P_XBUF_FLOATS * 4 + 32 * 64 * 2);  // gate/up, double-buffered
+static_assert(P_EPI_GROUP_BYTES >= 2 * 32 * 128 * 2, "down staging fits");
+
 
 struct PSmem {
-  uint64_t full[P_STAGES];
-  uint64_t empty[P_STAGES];
+  uint64_t full[P_MAX_STAGES];
+  uint64_t empty[P_MAX_STAGES];
   uint64_t tfull[2];
   uint64_t tempty[2];
   uint64_t drain;
@@ -410,9 +413,22 @@ struct PSmem {
   int mt_start[ORDERMOE_MAX_EXPERTS + 1];
   int offs[ORDERMOE_MAX_EXPERTS + 1];
 };
-constexpr int P_SMEM_BYTES =
-    P_STAGES * P_STAGE_BYTES + P_EPI_BYTES + 1024 + static_cast<int>(sizeof(PSmem));
-static_assert(P_SMEM_BYTES <= 227 * 1024, "pair kernel shared memory");
+// Per projection: gate/up (SwiGLU exchange in the epilogue) runs two epilogue
+// groups of four warps and five stages; down (a plain conversion) one group
+// and six stages. Five stages time the same as six for gate/up, and a second
+// group made down slower.
+template <int MODE>
+struct PCfg {
+  static constexpr int GROUPS = MODE == GATEUP ? 2 : 1;
+  static constexpr int EPI_WARPS = 4 * GROUPS;
+  static constexpr int THREADS = 64 + 32 * EPI_WARPS;
+  static constexpr int STAGES = MODE == GATEUP ? 5 : 6;
+  static constexpr int EPI_BYTES = GROUPS * P_EPI_GROUP_BYTES;
+  static constexpr int SMEM_BYTES =
+      STAGES * P_STAGE_BYTES + EPI_BYTES + 1024 + static_cast<int>(sizeof(PSmem));
+  static_assert(STAGES <= P_MAX_STAGES, "stage barriers");
+  static_assert(SMEM_BYTES <= 227 * 1024, "pair kernel shared memory");
+};
 
 __device__ __forceinline__ Tile decode_pair(int tile, const PSmem& s, int E, int n_tiles) {
   int e = 0;
@@ -446,32 +462,37 @@ __device__ __forceinline__ int tile_n(const Tile& t) {
   return (rows + 15) & ~15;
 }
 
-// the 128 epilogue threads of this CTA
-__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+// the 128 threads of epilogue group grp (named barriers 1 and 2)
+__device__ __forceinline__ void epi_sync(int grp) {
+  asm volatile("bar.sync %0, 128;" ::"r"(1 + grp) : "memory");
+}
+// true in every epilogue thread iff p holds in all N of them (named barrier 3)
+template <int N>
 __device__ __forceinline__ bool epi_all(bool p) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred pi, po;\n\t"
       "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.and.pred po, 1, 128, pi;\n\t"
+      "bar.red.and.pred po, 3, %2, pi;\n\t"
       "selp.u32 %0, 1, 0, po;\n\t}"
       : "=r"(r)
-      : "r"(static_cast<uint32_t>(p))
+      : "r"(static_cast<uint32_t>(p)), "n"(N)
       : "memory");
   return r != 0;
 }
 
 // CL = CTAs per cluster (2: one pair; 4: two pairs sharing the row tile).
 template <int MODE, int CL>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
     ffn_gemm_pair_kernel(const __grid_constant__ CUtensorMap mapW0,
                          const __grid_constant__ CUtensorMap mapW1,
                          const __grid_constant__ CUtensorMap mapT, Args args) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* tiles = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  constexpr int P_STAGES = PCfg<MODE>::STAGES;
   uint8_t* epi = tiles + P_STAGES * P_STAGE_BYTES;
-  PSmem& s = *reinterpret_cast<PSmem*>(epi + P_EPI_BYTES);
+  PSmem& s = *reinterpret_cast<PSmem*>(epi + PCfg<MODE>::EPI_BYTES);
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
@@ -491,7 +512,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s.tfull[i], 1);
-      mbar_init(&s.tempty[i], 8);
+      mbar_init(&s.tempty[i], 2 * PCfg<MODE>::EPI_WARPS);  // every epilogue warp of both CTAs
     }
     mbar_init(&s.drain, 1);
     s.abort = 0;
@@ -619,18 +640,21 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
     }
   } else {
-    // epilogue: warps 2..5, TMEM lane quarter q = warp % 4
+    // epilogue: warps 2..9 in two groups of four; TMEM lane quarter q = warp % 4;
+    // group grp takes the 32-row chunks grp, grp + 2, ... of every tile
     const int q = warp & 3;
-    const int et = tid - 64;  // 0..127
-    float* xbuf = reinterpret_cast<float*>(epi);                          // [2][128][P_X_PITCH]
-    uint16_t* obuf = reinterpret_cast<uint16_t*>(epi + 2 * P_XBUF_FLOATS * 4);  // gate/up [2][32][64]
-    uint16_t* ybuf = reinterpret_cast<uint16_t*>(epi);                    // down [2][32][128]
+    const int grp = (warp - 2) >> 2;  // 0 .. GROUPS - 1
+    const int et = tid - 64 - 128 * grp;  // 0..127 within the group
+    uint8_t* ge = epi + grp * P_EPI_GROUP_BYTES;
+    float* xbuf = reinterpret_cast<float*>(ge);                          // [2][128][P_X_PITCH]
+    uint16_t* obuf = reinterpret_cast<uint16_t*>(ge + 2 * P_XBUF_FLOATS * 4);  // gate/up [2][32][64]
+    uint16_t* ybuf = reinterpret_cast<uint16_t*>(ge);                    // down [2][32][128]
     int it = 0;
     for (int tile = cluster; tile < total; tile += n_clusters, ++it) {
       const int slot = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       const bool waited = (*abort == 0) && mbar_wait(&s.tfull[slot], acc_phase, args.limit_ns, abort);
-      if (!epi_all(waited)) {  // the same decision in all four warps
+      if (!epi_all<PCfg<MODE>::EPI_WARPS * 32>(waited)) {  // the same decision in every epilogue warp
         if (!waited && lane == 0 && !*abort) report(&g_err_gemm, ORDERMOE_DEV_WAIT_TIMEOUT, 14);
         *abort = 1;
         break;
@@ -641,8 +665,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       const int nchunks = (rows + 31) >> 5;
       const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
 #pragma unroll 1
-      for (int c = 0; c < nchunks; ++c) {
-        const int buf = c & 1;
+      for (int c = grp; c < nchunks; c += PCfg<MODE>::GROUPS) {
+        const int buf = (c / PCfg<MODE>::GROUPS) & 1;
         uint32_t v[32];
         tmem_ld32(tb + c * 32, v);  // TMEM column = row c*32 + i of the tile
         tmem_ld_wait();
@@ -655,7 +679,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           float* mine = xb + (q * 32 + lane) * P_X_PITCH;
 #pragma unroll
           for (int i = 0; i < 16; ++i) mine[i] = __uint_as_float(gate ? v[16 + i] : v[i]);
-          epi_sync();
+          epi_sync(grp);
           const float* other = xb + ((q ^ 2) * 32 + lane) * P_X_PITCH;
           uint16_t* ob = obuf + buf * (32 * 64);
           const int col = (q & 1) * 32 + lane;
@@ -674,7 +698,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             ob[(keep + i) * 64 + col] = static_cast<uint16_t>(pk & 0xFFFFu);
             ob[(keep + i + 1) * 64 + col] = static_cast<uint16_t>(pk >> 16);
           }
-          epi_sync();
+          epi_sync(grp);
           uint16_t* gcol = args.out + t.n * 128 + 64 * static_cast<int>(rp) + (et & 7) * 8;
 #pragma unroll
           for (int p = 0; p < 2; ++p) {
@@ -693,7 +717,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             yb[i * 128 + col] = static_cast<uint16_t>(pk & 0xFFFFu);
             yb[(i + 1) * 128 + col] = static_cast<uint16_t>(pk >> 16);
           }
-          epi_sync();
+          epi_sync(grp);
           uint16_t* gcol = args.out + t.n * 256 + 128 * static_cast<int>(rp) + (et & 15) * 8;
 #pragma unroll
           for (int p = 0; p < 4; ++p) {
@@ -775,7 +799,8 @@ int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
 template <int MODE, int CL>
 static cudaError_t pair_attr() {
   return cudaFuncSetAttribute(gg::ffn_gemm_pair_kernel<MODE, CL>,
-                              cudaFuncAttributeMaxDynamicSharedMemorySize, gg::P_SMEM_BYTES);
+                              cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              gg::PCfg<MODE>::SMEM_BYTES);
 }
 
 static int ffn_attrs() {
@@ -798,12 +823,13 @@ static int ffn_attrs() {
   return ORDERMOE_OK;
 }
 
+template <int MODE>
 static cudaLaunchConfig_t pair_config(int grid, int cl, cudaStream_t stream,
                                       cudaLaunchAttribute* attr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid, 1, 1);
-  cfg.blockDim = dim3(gg::THREADS, 1, 1);
-  cfg.dynamicSmemBytes = gg::P_SMEM_BYTES;
+  cfg.blockDim = dim3(gg::PCfg<MODE>::THREADS, 1, 1);
+  cfg.dynamicSmemBytes = gg::PCfg<MODE>::SMEM_BYTES;
   cfg.stream = stream;
   attr->id = cudaLaunchAttributeClusterDimension;
   attr->val.clusterDim.x = cl;
@@ -817,14 +843,14 @@ static cudaLaunchConfig_t pair_config(int grid, int cl, cudaStream_t stream,
 // Clusters of `cl` CTAs that can be resident at once (not every SM finds
 // partners in its GPC: on GB300, 76 clusters of 2 and 36 of 4); the persistent
 // grid never exceeds it, so no cluster waits for another. 0: none fit.
-template <int CL>
+template <int MODE, int CL>
 static int max_resident_clusters() {
   static PerDevice cache;
   return per_device(cache, [] {
     cudaLaunchAttribute attr;
-    cudaLaunchConfig_t cfg = pair_config(CL * (num_sms() / CL), CL, nullptr, &attr);
+    cudaLaunchConfig_t cfg = pair_config<MODE>(CL * (num_sms() / CL), CL, nullptr, &attr);
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gg::ffn_gemm_pair_kernel<gg::GATEUP, CL>, &cfg) !=
+    if (cudaOccupancyMaxActiveClusters(&n, gg::ffn_gemm_pair_kernel<MODE, CL>, &cfg) !=
             cudaSuccess ||
         n < 0) {
       cudaGetLastError();
@@ -838,11 +864,11 @@ static int max_resident_clusters() {
 template <int MODE, int CL>
 static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const CUtensorMap& t,
                        const gg::Args& a, long long tiles, cudaStream_t stream, const char* what) {
-  const long long cmax = max_resident_clusters<CL>();
+  const long long cmax = max_resident_clusters<MODE, CL>();
   const long long clusters = tiles < cmax ? tiles : cmax;
   cudaLaunchAttribute attr;
   cudaLaunchConfig_t cfg =
-      pair_config(static_cast<int>(CL * (clusters > 0 ? clusters : 1)), CL, stream, &attr);
+      pair_config<MODE>(static_cast<int>(CL * (clusters > 0 ? clusters : 1)), CL, stream, &attr);
   const cudaError_t e = cudaLaunchKernelEx(&cfg, gg::ffn_gemm_pair_kernel<MODE, CL>, w0, w1, t, a);
   if (e != cudaSuccess) return cuda_fail(e, what);
   OM_LAUNCHED(what);
@@ -877,7 +903,7 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
     if ((rc = make_tmap_bf16(&mW1, W1, (uint64_t)E * dff, d, 64))) return rc;
     if ((rc = make_tmap_bf16(&mW3, W3, (uint64_t)E * dff, d, 64))) return rc;
     const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
-    if (a.n_tiles % 2 == 0 && max_resident_clusters<4>() > 0) {
+    if (a.n_tiles % 2 == 0 && max_resident_clusters<GATEUP, 4>() > 0) {
       if ((rc = make_tmap_bf16(&mX, X_perm, R, d, 64))) return rc;  // half boxes, multicast
       return launch_pair<GATEUP, 4>(mW1, mW3, mX, a, row_tiles * (a.n_tiles / 2), stream,
                                     "ffn_gemm_pair_kernel<gate_up, 4>");
@@ -908,7 +934,7 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   if ((rc = make_map(&mH, H, R, dff))) return rc;
   if (use_pairs(R, E)) {
     const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
-    if (a.n_tiles % 2 == 0 && max_resident_clusters<4>() > 0) {
+    if (a.n_tiles % 2 == 0 && max_resident_clusters<DOWN, 4>() > 0) {
       CUtensorMap mHh;
       if ((rc = make_tmap_bf16(&mHh, H, R, dff, 64))) return rc;  // half boxes, multicast
       return launch_pair<DOWN, 4>(mW2, mW2, mHh, a, row_tiles * (a.n_tiles / 2), stream,
