@@ -94,18 +94,19 @@ struct SelSmem {
   uint8_t sublist[64 * 64];
 };
 
-// Loads the layer's tables into shared memory (whole block). Returns false
-// if the header does not match E (reported once).
-__device__ bool load_tables(const uint8_t* __restrict__ tab, int E, SelSmem& sm, float* s_Q,
-                            float* s_Cq) {
+// Threads t0, t0 + nt, ... of the block load the layer's tables into shared
+// memory. The E x E tables are copied with 16-byte loads, four in flight per
+// thread, where sizes and addresses allow.
+__device__ bool load_tables_range(const uint8_t* __restrict__ tab, int E, SelSmem& sm, float* s_Q,
+                                  float* s_Cq, int t0, int nt) {
   const int M = reinterpret_cast<const int32_t*>(tab)[2];
   if (reinterpret_cast<const int32_t*>(tab)[1] != E || M <= 0 || M > 32) {
-    if (blockIdx.x == 0 && threadIdx.x == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, -1);
+    if (blockIdx.x == 0 && t0 == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, -1);
     return false;
   }
   const float* gQ = reinterpret_cast<const float*>(tab + kOffQtab);
   const float* gCq = reinterpret_cast<const float*>(tab + off_cq(E));
-  for (int i = threadIdx.x; i < 64; i += blockDim.x) {
+  for (int i = t0; i < 64; i += nt) {
     sm.pmask[i] = reinterpret_cast<const uint32_t*>(tab + kOffPmask)[i];
     unsigned long long sb = reinterpret_cast<const unsigned long long*>(tab + kOffSubst)[i];
     int n = 0;
@@ -116,12 +117,35 @@ __device__ bool load_tables(const uint8_t* __restrict__ tab, int E, SelSmem& sm,
     }
     sm.nsub[i] = n;
   }
-  for (int i = threadIdx.x; i < E * E; i += blockDim.x) {
-    s_Q[i] = gQ[i];
-    s_Cq[i] = gCq[i];
+  const int n = E * E;
+  const bool vec = (n & 3) == 0 && ((reinterpret_cast<uintptr_t>(gQ) | reinterpret_cast<uintptr_t>(gCq) |
+                                     reinterpret_cast<uintptr_t>(s_Q) | reinterpret_cast<uintptr_t>(s_Cq)) &
+                                    15u) == 0;
+  if (vec) {
+    const float4* q4 = reinterpret_cast<const float4*>(gQ);
+    const float4* c4 = reinterpret_cast<const float4*>(gCq);
+#pragma unroll 4
+    for (int i = t0; i < n / 4; i += nt) {
+      const float4 x = __ldg(q4 + i), y = __ldg(c4 + i);
+      reinterpret_cast<float4*>(s_Q)[i] = x;
+      reinterpret_cast<float4*>(s_Cq)[i] = y;
+    }
+  } else {
+#pragma unroll 4
+    for (int i = t0; i < n; i += nt) {
+      s_Q[i] = gQ[i];
+      s_Cq[i] = gCq[i];
+    }
   }
-  if (threadIdx.x < 4) sm.kind[threadIdx.x] = 0;
+  for (int i = t0; i < 4; i += nt) sm.kind[i] = 0;
   return true;
+}
+
+// Loads the layer's tables into shared memory (whole block). Returns false
+// if the header does not match E (reported once).
+__device__ bool load_tables(const uint8_t* __restrict__ tab, int E, SelSmem& sm, float* s_Q,
+                            float* s_Cq) {
+  return load_tables_range(tab, E, sm, s_Q, s_Cq, threadIdx.x, blockDim.x);
 }
 
 // Look-ahead context (Eqs. 41-43): the tables of the next layers follow the
@@ -816,7 +840,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     tmem_alloc(&s.tmem_base, TMEM_COLS);
     tmem_relinquish();
   }
-  const bool tables_ok = (rank == 0) ? load_tables(tab, E, sm, s_Q, s_Cq) : true;
+  bool tables_ok = true;  // rank 0's epilogue warps load the tables during the main loop
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -875,6 +899,10 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       }
     }
   } else {
+    // the selection tables, while the TMA and MMA warps run (named barrier 1:
+    // the 128 epilogue threads)
+    if (rank == 0) tables_ok = load_tables_range(tab, E, sm, s_Q, s_Cq, tid - 64, 128);
+    asm volatile("bar.sync 1, 128;" ::: "memory");
     // epilogue part 1: this CTA's partial logits
     const int q = warp & 3;
     const int row = q * 32 + lane;
