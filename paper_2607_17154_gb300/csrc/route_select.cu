@@ -154,7 +154,15 @@ struct Lookahead {
   int H;                 // horizon; 1 = myopic (Phi = 0)
   size_t stride;         // bytes between consecutive layers' tables
   const float* P;        // [H-1][E][E]
+  int staged;            // lookahead_select_kernel copies layers l+1.. and P to shared memory
 };
+
+// A plain (generic) load: the look-ahead reads the next layers' tables either
+// from global memory or from the kernel's shared-memory copy of them.
+template <class T>
+__device__ __forceinline__ T ldt(const T* p) {
+  return *p;
+}
 
 // Cost-to-go of Eq. 42 with D future layers, from server m after executing
 // expert kx with accumulated loss qacc: sum over next targets k' (ascending)
@@ -173,26 +181,26 @@ __device__ float lookahead_phi(const uint8_t* __restrict__ tnext, size_t stride,
   const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
   float acc = 0.0f;
   for (int kt = 0; kt < E; ++kt) {
-    const float p = __ldg(P + (size_t)kx * E + kt);
+    const float p = ldt(P + (size_t)kx * E + kt);
     if (p == 0.0f) continue;
     float best = INFINITY;
-    unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);  // substitutes and the target
+    unsigned long long cand = ldt(sb1 + kt) | (1ull << kt);  // substitutes and the target
     while (cand) {
       const int kk = __ffsll(static_cast<long long>(cand)) - 1;
       cand &= cand - 1;
       const bool exact = (kk == kt);
       float cq = 0.0f, q2 = qacc;
       if (!exact) {
-        const float qk = __ldg(Q1 + kt * E + kk);
+        const float qk = ldt(Q1 + kt * E + kk);
         if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
         q2 = __fadd_rn(qacc, qk);
-        cq = __ldg(C1 + kt * E + kk);
+        cq = ldt(C1 + kt * E + kk);
       }
-      uint32_t pm = __ldg(pm1 + kk);
+      uint32_t pm = ldt(pm1 + kk);
       while (pm) {
         const int m2 = __ffs(pm) - 1;
         pm &= pm - 1;
-        float c = __fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq);
+        float c = __fadd_rn(ldt(A1 + ((size_t)a * M + m) * M + m2), cq);
         if (D > 1)
           c = __fadd_rn(c, lookahead_phi<(D > 1 ? D - 1 : 1)>(tnext + stride, stride, P + E * E, E,
                                                               M, a, m2, kk, q2, qbar));
@@ -405,7 +413,7 @@ __device__ __forceinline__ float phi_term(const uint8_t* __restrict__ tnext, siz
                                           const float* __restrict__ P, int E, int M, int a, int m,
                                           int kx, int kt, float qacc, float qbar) {
   // the k' = kt term of lookahead_phi<D> (0 when P = 0)
-  const float p = __ldg(P + (size_t)kx * E + kt);
+  const float p = ldt(P + (size_t)kx * E + kt);
   if (p == 0.0f) return 0.0f;
   const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
   const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
@@ -413,23 +421,23 @@ __device__ __forceinline__ float phi_term(const uint8_t* __restrict__ tnext, siz
   const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
   const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
   float best = INFINITY;
-  unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);
+  unsigned long long cand = ldt(sb1 + kt) | (1ull << kt);
   while (cand) {
     const int kk = __ffsll(static_cast<long long>(cand)) - 1;
     cand &= cand - 1;
     const bool exact = (kk == kt);
     float cq = 0.0f, q2 = qacc;
     if (!exact) {
-      const float qk = __ldg(Q1 + kt * E + kk);
+      const float qk = ldt(Q1 + kt * E + kk);
       if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
       q2 = __fadd_rn(qacc, qk);
-      cq = __ldg(C1 + kt * E + kk);
+      cq = ldt(C1 + kt * E + kk);
     }
-    uint32_t pm = __ldg(pm1 + kk);
+    uint32_t pm = ldt(pm1 + kk);
     while (pm) {
       const int m2 = __ffs(pm) - 1;
       pm &= pm - 1;
-      float c = __fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq);
+      float c = __fadd_rn(ldt(A1 + ((size_t)a * M + m) * M + m2), cq);
       if (D > 1)
         c = __fadd_rn(c, lookahead_phi<(D > 1 ? D - 1 : 1)>(tnext + stride, stride, P + E * E, E,
                                                             M, a, m2, kk, q2, qbar));
@@ -450,7 +458,7 @@ __device__ __forceinline__ float phi_term2_memo(const uint8_t* __restrict__ tnex
                                                 const float* __restrict__ P, int E, int M, int a,
                                                 int m, int kx, int kt, float qacc, float qbar,
                                                 const float* U, const float* qmax1) {
-  const float p = __ldg(P + (size_t)kx * E + kt);
+  const float p = ldt(P + (size_t)kx * E + kt);
   if (p == 0.0f) return 0.0f;
   const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
   const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
@@ -458,27 +466,27 @@ __device__ __forceinline__ float phi_term2_memo(const uint8_t* __restrict__ tnex
   const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
   const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
   float best = INFINITY;
-  unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);
+  unsigned long long cand = ldt(sb1 + kt) | (1ull << kt);
   while (cand) {
     const int kk = __ffsll(static_cast<long long>(cand)) - 1;
     cand &= cand - 1;
     const bool exact = (kk == kt);
     float cq = 0.0f, q2 = qacc;
     if (!exact) {
-      const float qk = __ldg(Q1 + kt * E + kk);
+      const float qk = ldt(Q1 + kt * E + kk);
       if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
       q2 = __fadd_rn(qacc, qk);
-      cq = __ldg(C1 + kt * E + kk);
+      cq = ldt(C1 + kt * E + kk);
     }
     const bool free = __fadd_rn(q2, qmax1[kk]) <= qbar;
-    uint32_t pm = __ldg(pm1 + kk);
+    uint32_t pm = ldt(pm1 + kk);
     while (pm) {
       const int m2 = __ffs(pm) - 1;
       pm &= pm - 1;
       const float phi1 = free ? U[m2 * E + kk]
                               : lookahead_phi<1>(tnext + stride, stride, P + E * E, E, M, a, m2, kk,
                                                  q2, qbar);
-      const float c = __fadd_rn(__fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq), phi1);
+      const float c = __fadd_rn(__fadd_rn(ldt(A1 + ((size_t)a * M + m) * M + m2), cq), phi1);
       best = fminf(best, c);
     }
   }
@@ -493,7 +501,7 @@ __device__ float lookahead_phi2_memo(const uint8_t* __restrict__ tnext, size_t s
                                      const float* qmax1) {
   float acc = 0.0f;
   for (int kt = 0; kt < E; ++kt) {
-    if (__ldg(P + (size_t)kx * E + kt) == 0.0f) continue;
+    if (ldt(P + (size_t)kx * E + kt) == 0.0f) continue;
     acc = __fadd_rn(acc, phi_term2_memo(tnext, stride, P, E, M, a, m, kx, kt, qacc, qbar, U, qmax1));
   }
   return acc;
@@ -511,7 +519,7 @@ __device__ __forceinline__ float phi_term3_memo(const uint8_t* __restrict__ tnex
                                                 int m, int kx, int kt, float qacc, float qbar,
                                                 const float* U2, const float* qmax2, float qmaxL1,
                                                 const float* U1, const float* qmax1) {
-  const float p = __ldg(P + (size_t)kx * E + kt);
+  const float p = ldt(P + (size_t)kx * E + kt);
   if (p == 0.0f) return 0.0f;
   const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
   const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
@@ -519,43 +527,56 @@ __device__ __forceinline__ float phi_term3_memo(const uint8_t* __restrict__ tnex
   const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
   const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
   float best = INFINITY;
-  unsigned long long cand = __ldg(sb1 + kt) | (1ull << kt);
+  unsigned long long cand = ldt(sb1 + kt) | (1ull << kt);
   while (cand) {
     const int kk = __ffsll(static_cast<long long>(cand)) - 1;
     cand &= cand - 1;
     const bool exact = (kk == kt);
     float cq = 0.0f, q2 = qacc;
     if (!exact) {
-      const float qk = __ldg(Q1 + kt * E + kk);
+      const float qk = ldt(Q1 + kt * E + kk);
       if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
       q2 = __fadd_rn(qacc, qk);
-      cq = __ldg(C1 + kt * E + kk);
+      cq = ldt(C1 + kt * E + kk);
     }
     const float qa = __fadd_rn(q2, qmax2[kk]);
     const float q3max = (qmax2[kk] == -INFINITY) ? q2 : qa;  // largest loss entering level 1
     const bool free = qa <= qbar && __fadd_rn(q3max, qmaxL1) <= qbar;
-    uint32_t pm = __ldg(pm1 + kk);
+    uint32_t pm = ldt(pm1 + kk);
     while (pm) {
       const int m2 = __ffs(pm) - 1;
       pm &= pm - 1;
       const float phi2 = free ? U2[m2 * E + kk]
                               : lookahead_phi2_memo(tnext + stride, stride, P + E * E, E, M, a, m2,
                                                     kk, q2, qbar, U1, qmax1);
-      const float c = __fadd_rn(__fadd_rn(__ldg(A1 + ((size_t)a * M + m) * M + m2), cq), phi2);
+      const float c = __fadd_rn(__fadd_rn(ldt(A1 + ((size_t)a * M + m) * M + m2), cq), phi2);
       best = fminf(best, c);
     }
   }
   return __fmul_rn(p, best);
 }
 
-__device__ __forceinline__ float phi_term_h(const Lookahead& la, const uint8_t* tab, int E, int M,
-                                            int a, int m, int kx, int kt, float qacc, float qbar) {
-  switch (la.H) {
-    case 2: return phi_term<1>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, kt, qacc, qbar);
-    case 3: return phi_term<2>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, kt, qacc, qbar);
-    case 4: return phi_term<3>(tab + la.stride, la.stride, la.P, E, M, a, m, kx, kt, qacc, qbar);
+// tn: the tables of layer l + 1 (the deeper layers follow, stride bytes
+// apart), Pn: the transitions l -> l + 1 (the deeper ones follow).
+__device__ __forceinline__ float phi_term_h(int H, const uint8_t* tn, size_t stride,
+                                            const float* Pn, int E, int M, int a, int m, int kx,
+                                            int kt, float qacc, float qbar) {
+  switch (H) {
+    case 2: return phi_term<1>(tn, stride, Pn, E, M, a, m, kx, kt, qacc, qbar);
+    case 3: return phi_term<2>(tn, stride, Pn, E, M, a, m, kx, kt, qacc, qbar);
+    case 4: return phi_term<3>(tn, stride, Pn, E, M, a, m, kx, kt, qacc, qbar);
     default: return 0.0f;
   }
+}
+
+// Shared-memory copy of the next layers' tables and transitions for the
+// look-ahead (bytes after the E x E tables and the H = 4 extras).
+__host__ __device__ inline size_t la_stage_offset(int E, int H) {
+  const size_t f = 2 * (size_t)E * E + (H == 4 ? 33 * (size_t)E : 0);
+  return (f * sizeof(float) + 15) & ~size_t(15);
+}
+__host__ __device__ inline size_t la_stage_bytes(int E, int H, size_t stride) {
+  return (size_t)(H - 1) * stride + (size_t)(H - 1) * E * E * sizeof(float);
 }
 
 constexpr int kLaThreads = 128;
@@ -587,6 +608,29 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
   const int t = blockIdx.x;
   if (t >= T) return;
   if (!load_tables(tab, E, sm, s_Q, s_Cq)) return;
+  // the next H - 1 layers' tables and transitions: read in place, or from a
+  // shared-memory copy (every Phi term reads them along serial chains)
+  const uint8_t* tn = tab + la.stride;
+  const float* Pn = la.P;
+  if (la.staged && la.H > 1) {
+    uint8_t* st_tab = reinterpret_cast<uint8_t*>(s_dyn) + la_stage_offset(E, la.H);
+    float* st_P = reinterpret_cast<float*>(st_tab + (size_t)(la.H - 1) * la.stride);
+    const size_t tb = (size_t)(la.H - 1) * la.stride;  // a multiple of 16
+    const size_t pn = (size_t)(la.H - 1) * E * E;
+    if (((reinterpret_cast<uintptr_t>(tn) | reinterpret_cast<uintptr_t>(la.P)) & 15u) == 0) {
+      const uint4* src = reinterpret_cast<const uint4*>(tn);
+#pragma unroll 4
+      for (size_t i = threadIdx.x; i < tb / 16; i += blockDim.x)
+        reinterpret_cast<uint4*>(st_tab)[i] = __ldg(src + i);
+    } else {
+      const uint32_t* src = reinterpret_cast<const uint32_t*>(tn);
+      for (size_t i = threadIdx.x; i < tb / 4; i += blockDim.x)
+        reinterpret_cast<uint32_t*>(st_tab)[i] = src[i];
+    }
+    for (size_t i = threadIdx.x; i < pn; i += blockDim.x) st_P[i] = la.P[i];
+    tn = st_tab;
+    Pn = st_P;
+  }
   __syncthreads();
   const int M = reinterpret_cast<const int32_t*>(tab)[2];
   const float qbar = reinterpret_cast<const float*>(tab)[5];
@@ -619,12 +663,12 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
     const unsigned long long* sbl = reinterpret_cast<const unsigned long long*>(tl + kOffSubst);
     float mx = -INFINITY;
     for (int kt = 0; kt < E; ++kt) {
-      if (__ldg(Pl + (size_t)kx * E + kt) == 0.0f) continue;
-      unsigned long long sb = __ldg(sbl + kt);
+      if (ldt(Pl + (size_t)kx * E + kt) == 0.0f) continue;
+      unsigned long long sb = ldt(sbl + kt);
       while (sb) {
         const int k3 = __ffsll(static_cast<long long>(sb)) - 1;
         sb &= sb - 1;
-        mx = fmaxf(mx, __ldg(Ql + kt * E + k3));
+        mx = fmaxf(mx, ldt(Ql + kt * E + k3));
       }
     }
     return mx;
@@ -632,8 +676,8 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
   if (memo || memo4) {
     // the deepest level's tables (layer l + H - 1) and transitions into it
     const int dl = la.H - 1;
-    const uint8_t* td = tab + dl * la.stride;
-    const float* Pd = la.P + (size_t)(dl - 1) * E * E;
+    const uint8_t* td = tn + (dl - 1) * la.stride;
+    const float* Pd = Pn + (size_t)(dl - 1) * E * E;
     for (int k2 = tid; k2 < E; k2 += blockDim.x) cs.qmax1[k2] = qmax_of(td, Pd, k2);
     for (int i = tid; i < M * E; i += blockDim.x) {
       const int m2 = i / E, k2 = i - (i / E) * E;
@@ -643,8 +687,8 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
   }
   if (memo4) {
     // one level up (layer l + 2): Phi^(2) at q = 0, through the U table above
-    const uint8_t* t2 = tab + 2 * la.stride;
-    const float* P2 = la.P + (size_t)E * E;
+    const uint8_t* t2 = tn + la.stride;
+    const float* P2 = Pn + (size_t)E * E;
     for (int k2 = tid; k2 < E; k2 += blockDim.x) qmax2[k2] = qmax_of(t2, P2, k2);
     for (int i = tid; i < M * E; i += blockDim.x) {
       const int m2 = i / E, k2 = i - (i / E) * E;
@@ -682,7 +726,7 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
         pm &= pm - 1;
         cs.code[slot] = static_cast<uint32_t>(kk) | (static_cast<uint32_t>(m) << 8) |
                         (sub ? (1u << 16) : 0u);
-        cs.cost0[slot] = __fadd_rn(__ldg(Aas + m), cq);
+        cs.cost0[slot] = __fadd_rn(ldt(Aas + m), cq);
         cs.qn[slot] = qn;
         ++slot;
       }
@@ -695,12 +739,12 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
         const int c = base + i / E, kt = i - (i / E) * E;
         const uint32_t code = cs.code[c];
         const int cm = static_cast<int>((code >> 8) & 0xFFu), ck = static_cast<int>(code & 0xFFu);
-        cs.terms[i] = memo    ? phi_term2_memo(tab + la.stride, la.stride, la.P, E, M, a, cm, ck,
-                                               kt, cs.qn[c], qbar, cs.U, cs.qmax1)
-                      : memo4 ? phi_term3_memo(tab + la.stride, la.stride, la.P, E, M, a, cm, ck,
-                                               kt, cs.qn[c], qbar, U2, qmax2, qmaxL1, cs.U,
-                                               cs.qmax1)
-                              : phi_term_h(la, tab, E, M, a, cm, ck, kt, cs.qn[c], qbar);
+        cs.terms[i] = memo    ? phi_term2_memo(tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c],
+                                               qbar, cs.U, cs.qmax1)
+                      : memo4 ? phi_term3_memo(tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c],
+                                               qbar, U2, qmax2, qmaxL1, cs.U, cs.qmax1)
+                              : phi_term_h(la.H, tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c],
+                                           qbar);
       }
       __syncthreads();
       for (int cl = tid; cl < nc; cl += blockDim.x) {
@@ -709,7 +753,7 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
         const unsigned sub = (code >> 16) & 1u;
         float phi = 0.0f;
         for (int kt = 0; kt < E; ++kt)
-          if (__ldg(la.P + (size_t)kk * E + kt) != 0.0f) phi = __fadd_rn(phi, cs.terms[cl * E + kt]);
+          if (ldt(Pn + (size_t)kk * E + kt) != 0.0f) phi = __fadd_rn(phi, cs.terms[cl * E + kt]);
         const float cost = __fadd_rn(cs.cost0[base + cl], phi);
         const unsigned long long key =
             (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
@@ -1020,6 +1064,15 @@ static int launch_lookahead_select(const int32_t* topk_idx, int T, int E, int k,
                                    size_t tab_smem, cudaStream_t stream) {
   if (T <= 0) return ORDERMOE_OK;
   if (la.H == 4) tab_smem += sizeof(float) * (32 * E + E);  // the Phi^(2) table and its bounds
+  // the next layers' tables and transitions in shared memory when they fit
+  la.staged = 0;
+  if (la.H > 1) {
+    const size_t staged = la_stage_offset(E, la.H) + la_stage_bytes(E, la.H, la.stride);
+    if (staged <= 160 * 1024) {
+      tab_smem = staged;
+      la.staged = 1;
+    }
+  }
   cudaFuncSetAttribute(lookahead_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)tab_smem);
   lookahead_select_kernel<<<T, kLaThreads, tab_smem, stream>>>(
