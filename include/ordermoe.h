@@ -306,7 +306,7 @@ int ordermoe_layer_forward_batches(const ordermoe_layer_desc* layer, int nbatch,
                                    int32_t* counters, ordermoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
- * Offline expert similarity (Section III-B, Eqs. 3-5; Alg. 1 lines 3-5).
+ * Offline expert similarity (Section III-B, Eqs. 3-5; Alg. 1).
  * For each layer l: H_l = W_r^l X_cal^T (router logits over the calibration
  * tokens, fp32 accumulation on tcgen05 tensor cores),
  * Sim_l(i,j) = <H_l,i, H_l,j> / (|H_l,i| |H_l,j|) (Eq. 4; diagonal exactly 1,
@@ -357,7 +357,7 @@ int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq, in
                            ordermoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
- * Grouping and mandatory placement (Section IV-A/B; Alg. 1 lines 1-24), all
+ * Grouping and mandatory placement (Section IV-A/B; Alg. 1), all
  * layers in order:
  *   theta_l = theta_min + (theta_max - theta_min)(L - l)/(L - 1), l = 1..L
  *            (Eq. 6; L == 1 uses theta_single);
@@ -400,8 +400,8 @@ int ordermoe_selftest_div_rn(const double* a, const double* b, double* out, int6
                              ordermoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
- * Importance-aware redundant deployment (Section IV-C, Eqs. 32-35; Alg. 1
- * lines 25-28), after the mandatory placement, over all layers:
+ * Importance-aware redundant deployment (Section IV-C, Eqs. 32-35; Alg. 1),
+ * after the mandatory placement, over all layers:
  *   y[m][l][g] = 1 when server m hosts an expert of group g of layer l (Eq. 32);
  *   benefit of a replica of expert j of layer l on server m:
  *     B = pi_m * I_l^j * (1 - y[m][l][g(j)]) / p_l^j          (Eq. 33);

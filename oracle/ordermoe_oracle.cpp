@@ -494,8 +494,8 @@ int orc_place(const int32_t* group, const double* importance, const double* p, i
 }
 
 // ---------------------------------------------------------------------------
-// Importance-aware redundant deployment, Section IV-C (Eqs. 32-35, Alg. 1
-// lines 25-28), over all layers after the mandatory placement. y[m][l][g]
+// Importance-aware redundant deployment, Section IV-C (Eqs. 32-35, Alg. 1),
+// over all layers after the mandatory placement. y[m][l][g]
 // (Eq. 32) is 1 when server m hosts an expert of group g in layer l. A
 // candidate replica of expert j of layer l on server m has the benefit
 // B = pi_m * I_l^j * (1 - y[m][l][g(j)]) / p_l^j (Eq. 33), and fits when

@@ -1,5 +1,5 @@
-// Offline similarity on the tensor cores (Section III-B, Eqs. 3-5; Alg. 1
-// lines 3-5) for E in {8, 16, 32, 64}:
+// Offline similarity on the tensor cores (Section III-B, Eqs. 3-5; Alg. 1)
+// for E in {8, 16, 32, 64}:
 //   sim_logits_kernel<E>: H = X_cal W^T for the L routers stacked (W rows =
 //     L * E), one 128-token x 256-logit tile per step of a persistent loop
 //     (TMA ring, tcgen05.mma, two TMEM accumulators, as in the expert FFN).

@@ -406,7 +406,7 @@ __global__ void div_selftest_kernel(const double* __restrict__ a, const double* 
     out[i] = div_rn_markstein(a[i], b[i], __drcp_rn(b[i]));
 }
 
-// Mandatory placement, Eqs. 29-31 (Alg. 1 lines 14-24): one warp, layers and
+// Mandatory placement, Eqs. 29-31 (Alg. 1): one warp, layers and
 // experts in order, b_m carried over the layers. Lane m keeps server m's
 // state in registers: b_m, C_m and lambda1 * (b_m / C_m); lambda2 * eta for
 // every count is a table. Per expert, lane m forms its score (one fp64 add of
@@ -474,8 +474,10 @@ __global__ void __launch_bounds__(32) place_kernel(
       const double sc = __dadd_rn(a1, l2eta[et]);
       double a1n = 0.0;
       if (feas) a1n = __dmul_rn(pp.lambda1, div_rn_markstein(bn, cap, rcap));  // kept if this lane wins
-      bad_score |= feas && !(sc >= 0.0);
       unsigned long long key = static_cast<unsigned long long>(__double_as_longlong(sc));
+      // !(sc >= 0) on the bits: a NaN, or a negative value other than -0
+      const unsigned long long mag = key & 0x7FFFFFFFFFFFFFFFull;
+      bad_score |= feas && (mag > 0x7FF0000000000000ull || (key != mag && mag != 0));
       if (key == 0x8000000000000000ull) key = 0;  // -0 orders like +0
       if (!feas) key = ~0ull;
       // argmin of the 64-bit keys, ties to the lower server: minimum of the high
@@ -670,10 +672,14 @@ constexpr int kRepMaxLayers = 1024;
 
 // Redundant deployment for one server (blockIdx.x = m), Eqs. 32-35. The
 // candidates (l, j) get the key (benefit bits, then candidate id), are sorted
-// by benefit desc and id asc (bitonic sort in shared memory), and one thread
-// deploys them in that order while the group is uncovered and the replica
-// fits. Benefits are positive fp64 values, so their bit patterns order like
-// the values; non-positive and NaN benefits get key 0 and are never taken.
+// by benefit desc and id asc (bitonic sort in shared memory), and are deployed
+// in that order while the group is uncovered and the replica fits. Benefits
+// are positive fp64 values, so their bit patterns order like the values;
+// non-positive and NaN benefits get key 0 and are never taken. A server's
+// state (b_m and its covered groups) changes only when it takes a candidate,
+// so one warp tests 32 sorted candidates at a time against the current state
+// and takes the first that passes: every candidate it passes over failed
+// under the same state it would have met one at a time.
 __global__ void __launch_bounds__(kRepThreads) replicate_kernel(
     const int32_t* __restrict__ group, const double* __restrict__ importance,
     const double* __restrict__ p, const double* __restrict__ C, const double* __restrict__ pi,
@@ -732,24 +738,61 @@ __global__ void __launch_bounds__(kRepThreads) replicate_kernel(
       __syncthreads();
     }
   }
-  if (t == 0) {
+  // the candidates (key != 0) are a prefix of the sorted order; each sorted
+  // slot is repacked in place as (l, g, j) and the bits of p_{l,j}
+  __shared__ int n_cand;
+  if (t == 0) n_cand = 0;
+  __syncthreads();
+  int mine = 0;
+  for (int s = t; s < N; s += blockDim.x) {
+    if (key[s] == 0) continue;
+    ++mine;
+    const int i = static_cast<int>(cid[s]);
+    const int l = i / E, j = i - l * E;
+    cid[s] = (static_cast<uint32_t>(l) << 12) | (static_cast<uint32_t>(group[i]) << 6) |
+             static_cast<uint32_t>(j);
+    key[s] = static_cast<unsigned long long>(__double_as_longlong(p[i]));
+  }
+  if (mine) atomicAdd(&n_cand, mine);
+  __syncthreads();
+  if (t < 32) {
+    const unsigned full = 0xffffffffu;
+    const int nc = n_cand;
     double b = used[m];
     const double cap = C[m];
     int count = 0;
-    for (int s = 0; s < N && key[s] != 0; ++s) {
-      const int i = static_cast<int>(cid[s]);
-      const int l = i / E, j = i - l * E;
-      const int g = group[i];
-      if ((cov[l] >> g) & 1ull) continue;  // B = 0 once the group is local
-      const double pj = p[i];
-      if (!(__dadd_rn(b, pj) <= cap)) continue;  // Eq. 35
-      placement[((size_t)l * M + m) * E + j] = 1;
-      b = __dadd_rn(b, pj);
-      cov[l] |= 1ull << g;
+    for (int base = 0; base < nc;) {
+      const int s = base + t;
+      uint32_t rec = 0;
+      double pj = 0.0;
+      bool take = false;
+      if (s < nc) {
+        rec = cid[s];
+        pj = __longlong_as_double(static_cast<long long>(key[s]));
+        const int l = static_cast<int>(rec >> 12), g = static_cast<int>((rec >> 6) & 63u);
+        take = !((cov[l] >> g) & 1ull) &&        // B = 0 once the group is local
+               __dadd_rn(b, pj) <= cap;          // Eq. 35
+      }
+      const unsigned bal = __ballot_sync(full, take);
+      if (bal == 0) {
+        base += 32;
+        continue;
+      }
+      const int w = __ffs(bal) - 1;
+      if (t == w) {
+        const int l = static_cast<int>(rec >> 12), g = static_cast<int>((rec >> 6) & 63u);
+        placement[((size_t)l * M + m) * E + static_cast<int>(rec & 63u)] = 1;
+        cov[l] |= 1ull << g;
+      }
+      b = __dadd_rn(b, __shfl_sync(full, pj, w));
       ++count;
+      base += w + 1;
+      __syncwarp();
     }
-    used[m] = b;
-    replicas[m] = count;
+    if (t == 0) {
+      used[m] = b;
+      replicas[m] = count;
+    }
   }
 }
 

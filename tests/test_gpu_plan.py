@@ -142,6 +142,27 @@ def test_place_bit_exact(L, E, M, K, noise):
         np.testing.assert_array_equal(a, b, err_msg=name)
 
 
+@pytest.mark.parametrize("L,E,M,scale,frac", [(4, 1, 2, 1.0, False), (5, 2, 3, 1.2, True),
+                                                (6, 3, 2, 0.9, False), (9, 64, 16, 1.1, False),
+                                                (9, 64, 17, 1.1, True), (12, 37, 16, 0.95, True),
+                                                (3, 40, 1, 1.0, False), (20, 24, 7, 0.97, False)])
+def test_place_ties_waiting_lists_and_server_counts(L, E, M, scale, frac):
+    """Integer sizes and equal capacities give exact score ties (to the lower
+    server); capacities below the demand send experts to the waiting list and
+    report the overflow; one to 17 servers, one to 64 experts a layer."""
+    rng = np.random.default_rng(L * 1000 + E * 10 + M)
+    sim, counts = synthetic_sims(rng, L, E, max(1, min(4, E)), 0.4)
+    if frac:
+        p = rng.uniform(0.5, 2.5, (L, E)); C = p.sum() / M * scale * rng.uniform(0.9, 1.1, M)
+    else:
+        p = rng.integers(1, 4, (L, E)).astype(np.float64); C = np.full(M, np.ceil(p.sum() / M * scale))
+    got = gpu_place(sim, counts, M, p, C)
+    ref = oracle_place_all(sim, counts, M, p, C)
+    for name, a, b in zip(("group", "n_groups", "theta", "placement", "used", "status"), got, ref):
+        np.testing.assert_array_equal(a, b, err_msg="%s L=%d E=%d M=%d" % (name, L, E, M))
+    assert (got[3].sum(axis=1) == 1).all()  # every expert on exactly one server
+
+
 def test_placement_quotient_is_correctly_rounded():
     """The placement's load ratio b_m / C_m (reciprocal + Markstein's correction)
     equals IEEE division (numpy) bit for bit on random and edge operands."""
@@ -257,6 +278,19 @@ def test_replicate_largest_shape_and_errors():
     got = gpu_replicate(group, I, p, C, pi, x0, used0)
     for name, a, b in zip(("placement", "used", "replicas"), got, ref):
         np.testing.assert_array_equal(a, b, err_msg=name)
+    # the most layers (1024), unequal memory demands
+    L2, E2, M2 = 1024, 16, 3
+    group2 = rng.integers(0, 4, (L2, E2)).astype(np.int32)
+    I2 = rng.random((L2, E2)); p2 = rng.integers(1, 4, (L2, E2)).astype(np.float64)
+    C2 = np.full(M2, p2.sum() / M2 * 1.1)
+    x2, used2, rc = oracle.place(group2, I2, p2, C2)
+    assert rc == 0
+    pi2 = np.array([0.5, 0.3, 0.2])
+    ref = oracle.replicate(group2, I2, p2, C2, pi2, x2, used2)
+    got = gpu_replicate(group2, I2, p2, C2, pi2, x2, used2)
+    for name, a, b in zip(("placement", "used", "replicas"), got, ref):
+        np.testing.assert_array_equal(a, b, err_msg="L 1024 " + name)
+    assert ref[2].min() > 0
     with pytest.raises(B.OrderMoEError) as ei:
         gpu_replicate(np.zeros((257, 64), np.int32), np.ones((257, 64)), np.ones((257, 64)), C, pi,
                       np.zeros((257, 4, 64), np.uint8), np.zeros(4))
