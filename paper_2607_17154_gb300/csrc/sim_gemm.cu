@@ -128,6 +128,49 @@ __device__ __forceinline__ void count_topk(const float (&x)[E], int kf, int* his
   }
 }
 
+// The same counts for k_freq <= K with fewer compare/select operations: a
+// descending min/max insertion network keeps the K largest logits with
+// multiplicity, T = the k_freq-th of them, and every logit >= T is counted;
+// when more than k_freq logits reach T (equal logits at the boundary), the
+// surplus logits equal to T are taken back from the highest index down, which
+// leaves the lowest indices, as the rank order says. Inserting c into the
+// descending v keeps min(v[i-1], max(v[i], c)) in slot i, which leaves v as it
+// was for a NaN c (min/max return the other operand), and -inf logits are
+// never counted, as in the passes above.
+template <int E, int K>
+__device__ __forceinline__ void count_topk_net(const float (&x)[E], int kf, int* hist_row) {
+  float v[K];
+#pragma unroll
+  for (int i = 0; i < K; ++i) v[i] = -INFINITY;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const float c = x[e];
+#pragma unroll
+    for (int i = K - 1; i > 0; --i) v[i] = fminf(v[i - 1], fmaxf(v[i], c));
+    v[0] = fmaxf(v[0], c);
+  }
+  float T = v[0];
+#pragma unroll
+  for (int i = 1; i < K; ++i) T = (i == kf - 1) ? v[i] : T;
+  const float Tc = fmaxf(T, -3.402823466e38f);  // below every finite logit, above -inf
+  int n = 0;
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const bool take = x[e] >= Tc;
+    n += take ? 1 : 0;
+    if (take) atomicAdd(&hist_row[e], 1);
+  }
+  if (n > kf) {
+    int extra = n - kf;
+#pragma unroll
+    for (int e = E - 1; e >= 0; --e) {
+      const bool back = extra > 0 && x[e] == T;
+      extra -= back ? 1 : 0;
+      if (back) atomicSub(&hist_row[e], 1);
+    }
+  }
+}
+
 template <int E>
 __global__ void __launch_bounds__(L_THREADS, 1)
     sim_logits_kernel(const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapW,
@@ -265,7 +308,36 @@ __global__ void __launch_bounds__(L_THREADS, 1)
         uint32_t v[32];
         tmem_ld32(tb + c * 32, v);
         tmem_ld_wait();
-        const int nv = min(32, args.C - cb);  // C is a multiple of 8
+        const int nv = min(32, args.C - cb);  // C is a multiple of 8, so nv is even
+        // hi/lo planes: each lane converts two adjacent logits at a time, and
+        // the lanes of a pair (tokens 2k, 2k + 1) swap halves so that the even
+        // lane holds expert i and the odd lane expert i + 1 of both tokens:
+        // one 4-byte store per plane and expert pair (ldT and the even row
+        // keep it aligned; row 2k + 1 < ldT whenever row 2k < N)
+        {
+          const int odd = lane & 1;
+          const uint32_t psel = odd ? 0x3276u : 0x5410u;
+          const size_t orow_pair = static_cast<size_t>(row & ~1) + (size_t)(cb + odd) * args.ldT;
+          const bool pair_valid = (row & ~1) < args.N;
+#pragma unroll
+          for (int i = 0; i < 32; i += 2) {
+            if (i >= nv) break;  // warp-uniform
+            const float2 x2 = make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1]));
+            const __nv_bfloat162 h2 = __float22bfloat162_rn(x2);
+            // x - hi, exact: one packed fma with -1
+            const float2 r2 = __ffma2_rn(__bfloat1622float2(h2), make_float2(-1.0f, -1.0f), x2);
+            const __nv_bfloat162 l2 = __float22bfloat162_rn(r2);
+            const uint32_t hw = *reinterpret_cast<const uint32_t*>(&h2);
+            const uint32_t lw = *reinterpret_cast<const uint32_t*>(&l2);
+            const uint32_t hp = __shfl_xor_sync(0xffffffffu, hw, 1);
+            const uint32_t lp = __shfl_xor_sync(0xffffffffu, lw, 1);
+            if (pair_valid) {
+              const size_t o = orow_pair + (size_t)i * args.ldT;
+              *reinterpret_cast<uint32_t*>(args.hi + o) = __byte_perm(hw, hp, psel);
+              *reinterpret_cast<uint32_t*>(args.lo + o) = __byte_perm(lw, lp, psel);
+            }
+          }
+        }
         if (valid) {
           float4* dst = reinterpret_cast<float4*>(orow + cb);
 #pragma unroll
@@ -273,16 +345,6 @@ __global__ void __launch_bounds__(L_THREADS, 1)
             if (args.H != nullptr && 4 * i < nv)  // logits kept only when asked for
               dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
                                    __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            if (i >= nv) break;
-            const float h = __uint_as_float(v[i]);
-            const __nv_bfloat16 hb = __float2bfloat16_rn(h);
-            const __nv_bfloat16 lb = __float2bfloat16_rn(h - __bfloat162float(hb));
-            const size_t o = (size_t)(cb + i) * args.ldT + row;
-            args.hi[o] = *reinterpret_cast<const uint16_t*>(&hb);
-            args.lo[o] = *reinterpret_cast<const uint16_t*>(&lb);
-          }
           if (E == 64) {
             if ((c & 1) == 0) {
 #pragma unroll
@@ -295,7 +357,10 @@ __global__ void __launch_bounds__(L_THREADS, 1)
                 x[32 + i] = __uint_as_float(v[i]);
               }
               const int l = (cb - 32) / 64;
-              count_topk<64>(reinterpret_cast<float(&)[64]>(x), args.kf, hist + l * 64);
+              float(&xr)[64] = reinterpret_cast<float(&)[64]>(x);
+              if (args.kf <= 6) count_topk_net<64, 6>(xr, args.kf, hist + l * 64);
+              else if (args.kf <= 8) count_topk_net<64, 8>(xr, args.kf, hist + l * 64);
+              else count_topk<64>(xr, args.kf, hist + l * 64);
             }
           } else {
 #pragma unroll

@@ -78,6 +78,33 @@ def test_similarity_no_logits_same_results(L, E, d, N, kf):
         assert torch.equal(region.view(torch.float32).view(N, L * E), logits)
 
 
+@pytest.mark.parametrize("kf", [1, 6, 8, 9])
+def test_similarity_counts_exact_with_tied_logits(kf):
+    """The counts of Eq. 5 equal the oracle's on the kernel's own fp32 logits,
+    bit for bit, with exact ties: duplicated router rows give equal logits for
+    every token, so equal logits straddle the top-k boundary (the lower index
+    wins). k_freq <= 8 runs the min/max network, 9 the selection passes."""
+    L, E, d, N = 2, 64, 128, 2000
+    Wr = torch.stack([synth.router_weights(E, d, 8, seed=40 + l) for l in range(L)])
+    Wr[:, 10:14] = Wr[:, 9:10]          # five equal rows
+    Wr[:, 40] = Wr[:, 20]
+    Wr[:, 63] = Wr[:, 0]
+    Wr = Wr.to(DEV).contiguous()
+    Xcal = synth.calibration(N, d, seed=kf).to(DEV)
+    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+    sim = torch.empty(L, E, E, dtype=torch.float32, device=DEV)
+    cnt = torch.empty(L, E, dtype=torch.int32, device=DEV)
+    B.ordermoe_similarity(Wr, Xcal, L, E, d, N, kf, sim, cnt, ws)
+    torch.cuda.synchronize()
+    logits = ws[: N * L * E * 4].view(torch.float32).view(N, L * E).cpu().numpy()
+    got = cnt.cpu().numpy()
+    for l in range(L):
+        lg = np.ascontiguousarray(logits[:, l * E:(l + 1) * E])
+        assert (lg[:, 10] == lg[:, 9]).all() and (lg[:, 40] == lg[:, 20]).all()
+        np.testing.assert_array_equal(got[l], oracle.expert_counts(lg, kf), err_msg="layer %d" % l)
+        assert got[l].sum() == N * kf
+
+
 def test_expert_counts_given_logits_bit_exact():
     rng = np.random.default_rng(3)
     for N, E, kf in [(5000, 64, 6), (100, 8, 2), (33, 5, 5)]:
