@@ -657,6 +657,18 @@ def run_decode(args, dist, w, device):
     }
 
 
+def plan_launches(L, E):
+    """Kernels of one ordermoe_plan call: on the tensor-core path (E in {8,
+    16, 32, 64}, L E <= 4096) each block of 512 logit columns launches the
+    logits GEMM, the Gram, its reduction, the similarities, the grouping and
+    the placement; otherwise the similarity takes 5 and the placement 2.
+    Replication and coverage add 1 each."""
+    if E in (8, 16, 32, 64) and L * E <= 4096:
+        part = max(1, 512 // E)
+        return 6 * ((L + part - 1) // part) + 2
+    return 5 + 2 + 2
+
+
 def run_similarity(args, dist, w, device):
     """Offline similarity of 24 layers x 64 experts over 262144 calibration
     tokens (Eqs. 3-5), then grouping and placement (Eqs. 6, 24-31)."""
@@ -670,7 +682,7 @@ def run_similarity(args, dist, w, device):
     Xcal = synth.calibration(N, d, seed, device=device)
     sim = torch.empty(L, E, E, dtype=torch.float32, device=device)
     counts = torch.empty(L, E, dtype=torch.int32, device=device)
-    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, N), dtype=torch.uint8, device=device)
+    ws = torch.empty(B.ordermoe_plan_workspace_bytes(L, E, N), dtype=torch.uint8, device=device)
     group = torch.empty(L, E, dtype=torch.int32, device=device)
     ng = torch.empty(L, dtype=torch.int32, device=device)
     theta = torch.empty(L, dtype=torch.float32, device=device)
@@ -687,12 +699,10 @@ def run_similarity(args, dist, w, device):
     pi = torch.as_tensor(synth.token_shares(synth.homes(65536, w.M, seed, "zipf1.1"), w.M),
                          dtype=torch.float64).to(device)
 
-    def step():  # no look-ahead transitions follow: the calibration logits are not kept
-        B.ordermoe_similarity_no_logits(Wr, Xcal, L, E, d, N, w.k, sim, counts, ws)
-        B.ordermoe_place(sim, counts, L, E, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5,
-                         0.5, 0.5, p, C, group, ng, theta, imp, x, used, st)
-        B.ordermoe_replicate(group, imp, p, C, pi, L, E, w.M, x, used, reps)
-        B.ordermoe_coverage(group, x, L, E, w.M, None, covered)
+    def step():  # one call: similarity (no logits kept), grouping, placement, redundancy, coverage
+        B.ordermoe_plan(Wr, Xcal, L, E, d, N, w.k, w.M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5,
+                        0.5, 0.5, p, C, pi, sim, counts, group, ng, theta, imp, x, used, st, reps,
+                        None, covered, ws)
 
     ms, clocks = timed_region(args, dist, device, step)
     code, detail = B.ordermoe_device_error()
@@ -711,15 +721,12 @@ def run_similarity(args, dist, w, device):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": L, "E": E, "d": d, "N": N, "groups": w.n_clusters,
                    "M": w.M, "k_freq": w.k, "memory_ratio": ratio},
-        "roofline": {"kernel": "similarity (tcgen05 logits + Gram) + place + replicate + coverage (whole plan)",
+        "roofline": {"kernel": "ordermoe_plan: similarity (tcgen05 logits + Gram) + group + place + replicate + coverage (whole plan)",
                      "bound": "tensor",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
                      "peak_source": "%s bf16_tflops (burst)" % pk_kind, "flop_per_step": flop},
-        # similarity 4 on the tensor-core path (logits with fused counts, Gram,
-        # Gram reduce, finish; E in {8, 16, 32, 64}, L E <= 4096) else 5, place 2,
-        # replicate 1, coverage 1
-        "gpu_launches": ((4 if E in (8, 16, 32, 64) and L * E <= 4096 else 5) + 4) * args.steps,
+        "gpu_launches": plan_launches(L, E) * args.steps,
         "n_groups": ng.cpu().tolist()[:3], "place_status": int(st.item()),
         "replicas": int(reps.sum().item()),
         "coverage": round(covered.sum().item() / (w.M * int(ng.sum().item())), 4),

@@ -435,6 +435,39 @@ int ordermoe_coverage(const int32_t* group, const uint8_t* placement, int L, int
                       uint8_t* cover, int32_t* covered, ordermoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * The whole offline plan of Alg. 1 in one call: similarity and counts
+ * (Section III-B, Eqs. 3-5), thresholds, grouping and importance (Eqs. 6,
+ * 24-28), mandatory placement (Eqs. 29-31), redundant deployment (Eqs. 32-35)
+ * and coverage (Eq. 32). Every output equals, bit for bit, what
+ * ordermoe_similarity_no_logits, ordermoe_place, ordermoe_replicate and
+ * ordermoe_coverage write when called in that order with the same arguments.
+ * For E in {8, 16, 32, 64} the layers go in blocks of 512 logit columns
+ * (8 layers of 64 experts): the caller's stream computes a block's logits,
+ * Gram and similarities while a side stream of the library, ordered behind it
+ * by events, groups and places the block before; the call joins the side
+ * stream back into the caller's before replication, so work queued on the
+ * caller's stream afterwards sees every output (CUDA graph capture included).
+ * Other E run the steps one after the other on the caller's stream.
+ *   Arguments as in those four calls: W_r [L][E][d] bf16, X_cal [N][d] bf16;
+ *   p [L][E] f64, C [M] f64, pi [M] f64; sim [L][E][E] f32, counts [L][E] i32,
+ *   group [L][E] i32, n_groups [L] i32, theta [L] f32, importance [L][E] f64
+ *   (not nullable here), placement [L][M][E] u8, used [M] f64, status [1] i32
+ *   (ORDERMOE_OK or ORDERMOE_ERR_CAPACITY, as ordermoe_place), replicas [M] i32,
+ *   cover [L][M][E] u8 (nullable), covered [L] i32 (nullable).
+ *   workspace: ordermoe_plan_workspace_bytes(L, E, N) bytes, 256-byte aligned.
+ * Needs the limits of the four calls together (L * E <= 16384, L <= 1024,
+ * M <= 32, d a multiple of 64). */
+size_t ordermoe_plan_workspace_bytes(int L, int E, int64_t N);
+int ordermoe_plan(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d, int64_t N,
+                  int k_freq, int M, double theta_min, double theta_max, double theta_single,
+                  double alpha_f, double alpha_r, double lambda1, double lambda2, const double* p,
+                  const double* C, const double* pi, float* sim, int32_t* counts, int32_t* group,
+                  int32_t* n_groups, float* theta, double* importance, uint8_t* placement,
+                  double* used, int32_t* status, int32_t* replicas, uint8_t* cover,
+                  int32_t* covered, void* workspace, size_t workspace_bytes,
+                  ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * Edge cost of L layers' selection records (Section III-D/E). Servers are the
  * logical placement map; the delays are the model's, not this GPU's. Token t
  * starts at home[t] (Eq. 36); at layer l, slot j executed on server m pays

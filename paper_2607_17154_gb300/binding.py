@@ -60,6 +60,9 @@ _SIGNATURES = {
     "ordermoe_layer_forward": ([_P, _I, _P, _P, _P, _P, _P, _P, _I, _P], _I),
     "ordermoe_dispatch_noalloc": ([_P, _P, _I, _I, _I, _I, _P, _P, _P, _P, _P], _I),
     "ordermoe_transitions": ([_P, _I64, _I, _I, _I, _P, _P, _P], _I),
+    "ordermoe_plan_workspace_bytes": ([_I, _I, _I64], _SZ),
+    "ordermoe_plan": ([_P, _P, _I, _I, _I, _I64, _I, _I, _D, _D, _D, _D, _D, _D, _D, _P, _P, _P,
+                       _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ordermoe_route_select_lookahead": ([_P, _P, _P, _I, _I, _I, _I, _I, _P, _SZ, _I, _P, _P, _P,
                                          _P, _P, _P, _P, _P, _P, _P, _P, _P], _I),
 }
@@ -285,6 +288,32 @@ def ordermoe_coverage(group, placement, L, E, M, cover=None, covered=None, strea
     _dt(cover, torch.uint8, "cover"); _dt(covered, torch.int32, "covered")
     _check("ordermoe_coverage", lib().ordermoe_coverage(_ptr(group), _ptr(placement), L, E, M,
                                                         _ptr(cover), _ptr(covered), _stream(stream)))
+
+
+def ordermoe_plan_workspace_bytes(L, E, N):
+    return int(lib().ordermoe_plan_workspace_bytes(L, E, N))
+
+
+def ordermoe_plan(W_r, X_cal, L, E, d, N, k_freq, M, theta_min, theta_max, theta_single, alpha_f,
+                  alpha_r, lambda1, lambda2, p, C, pi, sim, counts, group, n_groups, theta,
+                  importance, placement, used, status, replicas, cover, covered, workspace,
+                  stream=None):
+    """The whole offline plan (similarity, grouping, placement, redundancy,
+    coverage) in one call; workspace: ordermoe_plan_workspace_bytes(L, E, N) bytes."""
+    _dt(W_r, torch.bfloat16, "W_r"); _dt(X_cal, torch.bfloat16, "X_cal")
+    for n, v in (("p", p), ("C", C), ("pi", pi), ("importance", importance), ("used", used)):
+        _dt(v, torch.float64, n)
+    _dt(sim, torch.float32, "sim"); _dt(counts, torch.int32, "counts"); _dt(group, torch.int32, "group")
+    _dt(n_groups, torch.int32, "n_groups"); _dt(theta, torch.float32, "theta")
+    _dt(placement, torch.uint8, "placement"); _dt(status, torch.int32, "status")
+    _dt(replicas, torch.int32, "replicas"); _dt(cover, torch.uint8, "cover")
+    _dt(covered, torch.int32, "covered"); _dt(workspace, torch.uint8, "workspace")
+    _check("ordermoe_plan", lib().ordermoe_plan(
+        _ptr(W_r), _ptr(X_cal), L, E, d, N, k_freq, M, float(theta_min), float(theta_max),
+        float(theta_single), float(alpha_f), float(alpha_r), float(lambda1), float(lambda2), _ptr(p),
+        _ptr(C), _ptr(pi), _ptr(sim), _ptr(counts), _ptr(group), _ptr(n_groups), _ptr(theta),
+        _ptr(importance), _ptr(placement), _ptr(used), _ptr(status), _ptr(replicas), _ptr(cover),
+        _ptr(covered), _ptr(workspace), workspace.numel(), _stream(stream)))
 
 
 def ordermoe_trajectory_cost(target, chosen_expert, chosen_server, home, L, T, k, E, tables,

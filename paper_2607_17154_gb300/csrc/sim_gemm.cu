@@ -576,26 +576,55 @@ bool sim_tc_supported(int L, int E) {
   return (E == 8 || E == 16 || E == 32 || E == 64) && (long long)L * E <= sg::MAX_HIST;
 }
 
+// Layers per block of the pipelined plan: 512 logit columns (four 128-row
+// blocks of H^T for the Gram). Every block streams all of X_cal once; with
+// 512 columns a block's GEMM stays compute-bound (about 410 flops per byte).
+int sim_tc_part_layers(int E) { return E >= 512 ? 1 : 512 / E; }
+
+// Token splits of the Gram. They depend on E and N only (the row blocks of
+// one part of the pipelined plan fill the GPU), so the partial sums, and the
+// similarities, are the same whether the layers are done in one call or part
+// by part.
 int sim_tc_nsplit(int L, int E, int64_t N) {
-  const int n_rb = (L * E + 127) / 128;
+  const int part = sim_tc_part_layers(E);
+  const int n_rb = ((L < part ? L : part) * E + 127) / 128;
   const int kblocks = static_cast<int>((N + sg::BK - 1) / sg::BK);
-  int ns = num_sms() / n_rb;
+  const int sms = num_sms() > 1 ? num_sms() - 1 : 1;  // the pipelined plan keeps one SM free
+  int ns = sms / n_rb;
   if (ns < 1) ns = 1;
   if (ns > kblocks) ns = kblocks;
   return ns;
 }
 
+// Largest dynamic shared memory a block may ask for: asking for it keeps any
+// other kernel's block off that SM.
+static int whole_sm_smem() {
+  int dev = 0, v = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+    return 0;
+  return v;
+}
+
 // H [N][L E] fp32, the hi/lo planes [L E][ldT], counts (zeroed by the caller),
-// and the partial Grams gpart [L][nsplit][64][64].
+// and the partial Grams gpart [L][nsplit][64][64]. reserve_sm: run on all SMs
+// but one and take each SM's whole shared memory, so that the one left over
+// takes the kernels of another stream (the pipelined plan's grouping and
+// placement) without slowing a block of these persistent grids.
 int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int d, int kf,
                   float* H, uint16_t* hi, uint16_t* lo, int ldT, int32_t* counts, float* gpart,
-                  int nsplit, cudaStream_t stream) {
+                  int nsplit, bool reserve_sm, cudaStream_t stream) {
   using namespace sg;
   const int C = L * E;
-  const size_t lsmem = L_SMEM_FIXED + sizeof(int) * (size_t)C;
+  size_t lsmem = L_SMEM_FIXED + sizeof(int) * (size_t)C;
+  size_t gsmem = G_SMEM_BYTES;
   static PerDevice cache;
   const cudaError_t attr_err = static_cast<cudaError_t>(per_device(cache, [] {
-    const int lmax = L_SMEM_FIXED + static_cast<int>(sizeof(int)) * MAX_HIST;
+    int lmax = L_SMEM_FIXED + static_cast<int>(sizeof(int)) * MAX_HIST;
+    int gmax = G_SMEM_BYTES;
+    const int whole = whole_sm_smem();
+    if (whole > lmax) lmax = whole;
+    if (whole > gmax) gmax = whole;
     cudaError_t e = cudaFuncSetAttribute(sim_logits_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(sim_logits_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
@@ -604,7 +633,7 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(sim_logits_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, G_SMEM_BYTES);
+      e = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, gmax);
     return static_cast<int>(e);
   }));
   if (attr_err != cudaSuccess) return cuda_fail(attr_err, "cudaFuncSetAttribute(similarity)");
@@ -628,7 +657,14 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
   la.counts = counts;
   la.limit_ns = wait_limit_ns();
   const long long tiles = (long long)((N + BM - 1) / BM) * la.n_tiles;
-  const int grid = static_cast<int>(tiles < num_sms() ? tiles : num_sms());
+  int sms = num_sms();
+  if (reserve_sm && sms > 1) {
+    --sms;
+    const size_t whole = static_cast<size_t>(whole_sm_smem());
+    if (whole > lsmem) lsmem = whole;
+    if (whole > gsmem) gsmem = whole;
+  }
+  const int grid = static_cast<int>(tiles < sms ? tiles : sms);
   switch (E) {
     case 8: sim_logits_kernel<8><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
     case 16: sim_logits_kernel<16><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
@@ -644,7 +680,7 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
   ga.nsplit = nsplit;
   ga.gpart = gpart;
   ga.limit_ns = la.limit_ns;
-  gram_tc_kernel<<<dim3((C + 127) / 128, nsplit), THREADS, G_SMEM_BYTES, stream>>>(mHi, mLo, ga);
+  gram_tc_kernel<<<dim3((C + 127) / 128, nsplit), THREADS, gsmem, stream>>>(mHi, mLo, ga);
   OM_LAUNCHED("gram_tc_kernel");
   return ORDERMOE_OK;
 }

@@ -242,22 +242,27 @@ __global__ void __launch_bounds__(256) gram_reduce_kernel(const float* __restric
   G[(size_t)l * 4096 + x] = s;
 }
 
-// grid L: Sim(i,j) = G_ij / (sqrt(G_ii) sqrt(G_jj)) (Eq. 4), diagonal 1, zero-norm 0.
+// grid (L, 16): Sim(i,j) = G_ij / (sqrt(G_ii) sqrt(G_jj)) (Eq. 4), diagonal 1,
+// zero-norm 0; block y takes entries 256 y .. 256 y + 255 of layer l (the fp64
+// square roots and divides of a layer spread over 16 SMs).
 __global__ void __launch_bounds__(256) sim_finish_kernel(const double* __restrict__ Gall, int E,
                                                          float* __restrict__ sim) {
+  __shared__ double norm[64];
   const int l = blockIdx.x;
   const double* G = Gall + (size_t)l * 4096;
-  for (int x = threadIdx.x; x < E * E; x += blockDim.x) {
-    const int i = x / E, j = x % E;
-    float v;
-    if (i == j) {
-      v = 1.0f;
-    } else {
-      const double ni = sqrt(G[i * 64 + i]), nj = sqrt(G[j * 64 + j]);
-      v = (ni == 0.0 || nj == 0.0) ? 0.0f : __double2float_rn(G[i * 64 + j] / (ni * nj));
-    }
-    sim[(size_t)l * E * E + x] = v;
+  if (threadIdx.x < E) norm[threadIdx.x] = sqrt(G[threadIdx.x * 64 + threadIdx.x]);
+  __syncthreads();
+  const int x = blockIdx.y * 256 + threadIdx.x;
+  if (x >= E * E) return;
+  const int i = x / E, j = x % E;
+  float v;
+  if (i == j) {
+    v = 1.0f;
+  } else {
+    const double ni = norm[i], nj = norm[j];
+    v = (ni == 0.0 || nj == 0.0) ? 0.0f : __double2float_rn(G[i * 64 + j] / (ni * nj));
   }
+  sim[(size_t)l * E * E + x] = v;
 }
 
 __global__ void counts_from_logits_kernel(const float* __restrict__ logits, int64_t N, int E,
@@ -284,27 +289,40 @@ struct PlaceParams {
   double alpha_f, alpha_r, lambda1, lambda2;
 };
 
-// Per-layer part of the plan, one block per layer (the layers are
-// independent here): theta_l (Eq. 6), greedy cover (Eqs. 24-26), importance
-// (Eqs. 27-28) and the placement order (p desc, I desc, index asc).
-__global__ void __launch_bounds__(64) group_kernel(
-    const float* __restrict__ sim, const int32_t* __restrict__ counts, int L, int E,
-    PlaceParams pp, const double* __restrict__ p, int32_t* __restrict__ group,
-    int32_t* __restrict__ n_groups, float* __restrict__ theta_out, double* __restrict__ importance,
-    int32_t* __restrict__ porder) {
-  __shared__ double imp[64];
-  __shared__ double pls[64];
-  __shared__ int order[64];
-  __shared__ int dom[64];
-  __shared__ int grp[64];
-  __shared__ int cnt[64];
-  __shared__ float S[64 * 64];
-  const int t = threadIdx.x;
-  const int l = blockIdx.x;
-  for (int i = t; i < E * E; i += blockDim.x) S[i] = sim[(size_t)l * E * E + i];
-  if (t < E) {
-    cnt[t] = counts[(size_t)l * E + t];
-    pls[t] = p[(size_t)l * E + t];
+// One layer's scratch of the grouping.
+struct GroupSmem {
+  double imp[64];
+  double pls[64];
+  int order[64];
+  int dom[64];
+  int grp[64];
+  int cnt[64];
+  float S[64 * 64];
+};
+
+// Per-layer part of the plan for layer l, on 64 threads t = 0..63 of a block
+// (the layers are independent here): theta_l (Eq. 6), greedy cover
+// (Eqs. 24-26), importance (Eqs. 27-28) and the placement order (p desc,
+// I desc, index asc). A slice with live == false has no layer this round but
+// meets every barrier of the block.
+__device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float* __restrict__ sim,
+                            const int32_t* __restrict__ counts, int L, int E, PlaceParams pp,
+                            const double* __restrict__ p, int32_t* __restrict__ group,
+                            int32_t* __restrict__ n_groups, float* __restrict__ theta_out,
+                            double* __restrict__ importance, int32_t* __restrict__ porder) {
+  double* imp = sm.imp;
+  double* pls = sm.pls;
+  int* order = sm.order;
+  int* dom = sm.dom;
+  int* grp = sm.grp;
+  int* cnt = sm.cnt;
+  float* S = sm.S;
+  if (live) {
+    for (int i = t; i < E * E; i += 64) S[i] = sim[(size_t)l * E * E + i];
+    if (t < E) {
+      cnt[t] = counts[(size_t)l * E + t];
+      pls[t] = p[(size_t)l * E + t];
+    }
   }
   __syncthreads();
   // Eq. 6 (layers numbered from 1)
@@ -317,7 +335,7 @@ __global__ void __launch_bounds__(64) group_kernel(
         __dadd_rn(pp.theta_min, __dmul_rn(__dsub_rn(pp.theta_max, pp.theta_min), frac)));
   }
   // visiting order: count desc, index asc
-  if (t < E) {
+  if (live && t < E) {
     int r = 0;
     for (int e = 0; e < E; ++e)
       if (cnt[e] > cnt[t] || (cnt[e] == cnt[t] && e < t)) ++r;
@@ -326,7 +344,7 @@ __global__ void __launch_bounds__(64) group_kernel(
   __syncthreads();
   // Eqs. 24-26 in the visiting order; warp 0 scans the existing dominants in
   // parallel (lane g takes dominants g and g + 32; ties to the earlier one).
-  if (t < 32) {
+  if (live && t < 32) {
     int k = 0;
     for (int pos = 0; pos < E; ++pos) {
       const int j = order[pos];
@@ -361,8 +379,9 @@ __global__ void __launch_bounds__(64) group_kernel(
   __syncthreads();
   // Eqs. 27-28
   double total = 0.0;
-  for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cnt[e]));
-  if (t < E) {
+  if (live)
+    for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cnt[e]));
+  if (live && t < E) {
     group[(size_t)l * E + t] = grp[t];
     double sum = 0.0;
     int size = 0;
@@ -375,7 +394,7 @@ __global__ void __launch_bounds__(64) group_kernel(
   }
   __syncthreads();
   // placement order: p desc, I desc, index asc
-  if (t < E) {
+  if (live && t < E) {
     int r = 0;
     for (int e = 0; e < E; ++e) {
       bool before;
@@ -386,6 +405,17 @@ __global__ void __launch_bounds__(64) group_kernel(
     }
     porder[(size_t)l * E + r] = t;
   }
+}
+
+// One block per layer l = l0 + blockIdx.x, 64 threads.
+__global__ void __launch_bounds__(64) group_kernel(
+    const float* __restrict__ sim, const int32_t* __restrict__ counts, int L, int E, int l0,
+    PlaceParams pp, const double* __restrict__ p, int32_t* __restrict__ group,
+    int32_t* __restrict__ n_groups, float* __restrict__ theta_out, double* __restrict__ importance,
+    int32_t* __restrict__ porder) {
+  __shared__ GroupSmem sm;
+  group_layer(sm, true, threadIdx.x, l0 + blockIdx.x, sim, counts, L, E, pp, p, group, n_groups,
+              theta_out, importance, porder);
 }
 
 // b / C rounded to nearest by Markstein's correction step (P. Markstein, IBM J.
@@ -415,21 +445,38 @@ __global__ void div_selftest_kernel(const double* __restrict__ a, const double* 
 // (scores are non-negative, so their bit patterns order like the values; ties
 // to the lower server), and the winner keeps its speculative term. A
 // waiting-list expert goes to the server with the most room after its layer.
-__global__ void __launch_bounds__(32) place_kernel(
-    const int32_t* __restrict__ group, const int32_t* __restrict__ porder, int L, int E, int M,
-    PlaceParams pp, const double* __restrict__ p, const double* __restrict__ C,
-    uint8_t* __restrict__ placement, double* __restrict__ used, int32_t* __restrict__ status) {
-  __shared__ int grp[64];
-  __shared__ int ord[64];
-  __shared__ double pls[64];
-  __shared__ int waiting[64];
-  __shared__ uint8_t xs[32 * 64];
-  __shared__ int eta[32 * 64];
-  __shared__ double l2eta[65];  // lambda2 * eta for eta = 0 .. 64
+// Layers l0 .. l1 - 1: the first range starts from b_m = 0 and sets the
+// status, a later range continues from b_m in used (lambda1 * (b_m / C_m) is
+// recomputed from it, the same function the loop applies) and only raises the
+// capacity status.
+struct PlaceSmem {
+  int grp[64];
+  int ord[64];
+  double pls[64];
+  int waiting[64];
+  uint8_t xs[32 * 64];
+  int eta[32 * 64];
+  double l2eta[65];  // lambda2 * eta for eta = 0 .. 64
+};
+
+// The placement on warp 0 of a block (threadIdx.x < 32); returns 1 when a
+// waiting-list expert overfilled its server.
+__device__ int place_layers(PlaceSmem& sm, const int32_t* __restrict__ group,
+                             const int32_t* __restrict__ porder, int L, int E, int M, int l0,
+                             int l1, int first, PlaceParams pp, const double* __restrict__ p,
+                             const double* __restrict__ C, uint8_t* __restrict__ placement,
+                             double* __restrict__ used, int32_t* __restrict__ status) {
+  int* grp = sm.grp;
+  int* ord = sm.ord;
+  double* pls = sm.pls;
+  int* waiting = sm.waiting;
+  uint8_t* xs = sm.xs;
+  int* eta = sm.eta;
+  double* l2eta = sm.l2eta;
   const int t = threadIdx.x;
   int overflow = 0;
   const bool srv = t < M;
-  double b = 0.0;
+  double b = (srv && !first) ? used[t] : 0.0;
   const double cap = srv ? C[t] : 1.0;
   const double rcap = __drcp_rn(cap);
   // non-negative finite values compare like their bit patterns
@@ -437,14 +484,8 @@ __global__ void __launch_bounds__(32) place_kernel(
   double a1 = srv ? __dmul_rn(pp.lambda1, div_rn_markstein(b, cap, rcap)) : 0.0;
   bool bad_score = srv && !(cap > 0.0 && cap <= 1.7976931348623157e308);
   for (int i = t; i <= 64; i += 32) l2eta[i] = __dmul_rn(pp.lambda2, static_cast<double>(i));
-  if (t == 0) {
-    double need = 0.0, have = 0.0;
-    for (int i = 0; i < L * E; ++i) need = __dadd_rn(need, p[i]);
-    for (int m = 0; m < M; ++m) have = __dadd_rn(have, C[m]);
-    overflow = need > have ? 1 : 0;
-  }
   __syncwarp();
-  for (int l = 0; l < L; ++l) {
+  for (int l = l0; l < l1; ++l) {
     for (int i = t; i < 32 * 64; i += 32) {
       xs[i] = 0;
       eta[i] = 0;
@@ -530,7 +571,72 @@ __global__ void __launch_bounds__(32) place_kernel(
   overflow = __any_sync(0xffffffffu, overflow != 0);
   if (__any_sync(0xffffffffu, bad_score) && t == 0)
     report(&g_err_sim, ORDERMOE_DEV_BAD_VALUE, 0);
-  if (t == 0) *status = overflow ? ORDERMOE_ERR_CAPACITY : ORDERMOE_OK;
+  return overflow;
+}
+
+// Eq. 29's memory over all layers against the servers' total (the capacity
+// status of the first range), summed in order by one thread.
+__device__ int demand_exceeds(const double* __restrict__ p, int n, const double* __restrict__ C,
+                              int M) {
+  double need = 0.0, have = 0.0;
+  for (int i = 0; i < n; ++i) need = __dadd_rn(need, p[i]);
+  for (int m = 0; m < M; ++m) have = __dadd_rn(have, C[m]);
+  return need > have ? 1 : 0;
+}
+
+// Status of a placed range: the first range sets it, a later one only raises
+// the capacity error.
+__device__ void place_status(int first, int overflow, int32_t* __restrict__ status) {
+  if (first || overflow) *status = overflow ? ORDERMOE_ERR_CAPACITY : ORDERMOE_OK;
+}
+
+__global__ void __launch_bounds__(64) place_kernel(
+    const int32_t* __restrict__ group, const int32_t* __restrict__ porder, int L, int E, int M,
+    int l0, int l1, int first, PlaceParams pp, const double* __restrict__ p,
+    const double* __restrict__ C, uint8_t* __restrict__ placement, double* __restrict__ used,
+    int32_t* __restrict__ status) {
+  __shared__ PlaceSmem sm;
+  __shared__ int s_over;
+  int over = 0;
+  if (threadIdx.x < 32)
+    over = place_layers(sm, group, porder, L, E, M, l0, l1, first, pp, p, C, placement, used, status);
+  else if (threadIdx.x == 32 && first)  // beside the placement, on the second warp
+    s_over = demand_exceeds(p, L * E, C, M);
+  __syncthreads();
+  if (threadIdx.x == 0) place_status(first, over | (first ? s_over : 0), status);
+}
+
+// Grouping and placement of layers l0 .. l1 - 1 in one block: 64 threads per
+// layer group kGroupSlices layers at a time, then warp 0 places them (one
+// block, so the pipelined plan's side stream holds one SM).
+constexpr int kGroupSlices = 4;
+constexpr size_t kGroupPlaceSmem = kGroupSlices * sizeof(GroupSmem) + sizeof(PlaceSmem);
+
+__global__ void __launch_bounds__(64 * kGroupSlices) group_place_kernel(
+    const float* __restrict__ sim, const int32_t* __restrict__ counts, int L, int E, int M, int l0,
+    int l1, int first, PlaceParams pp, const double* __restrict__ p, const double* __restrict__ C,
+    int32_t* __restrict__ group, int32_t* __restrict__ n_groups, float* __restrict__ theta_out,
+    double* __restrict__ importance, int32_t* __restrict__ porder, uint8_t* __restrict__ placement,
+    double* __restrict__ used, int32_t* __restrict__ status) {
+  extern __shared__ __align__(16) unsigned char s_gp[];
+  GroupSmem* gs = reinterpret_cast<GroupSmem*>(s_gp);
+  PlaceSmem& ps = *reinterpret_cast<PlaceSmem*>(s_gp + kGroupSlices * sizeof(GroupSmem));
+  const int slice = threadIdx.x / 64;
+  for (int lb = l0; lb < l1; lb += kGroupSlices) {
+    const int l = lb + slice;
+    group_layer(gs[slice], l < l1, threadIdx.x % 64, l, sim, counts, L, E, pp, p, group, n_groups,
+                theta_out, importance, porder);
+    __syncthreads();  // the slices' scratch is reused by the next round
+  }
+  // group and porder written above are visible to the block after the barrier
+  __shared__ int s_over;
+  int over = 0;
+  if (threadIdx.x < 32)
+    over = place_layers(ps, group, porder, L, E, M, l0, l1, first, pp, p, C, placement, used, status);
+  else if (threadIdx.x == 32 && first)
+    s_over = demand_exceeds(p, L * E, C, M);
+  __syncthreads();
+  if (threadIdx.x == 0) place_status(first, over | (first ? s_over : 0), status);
 }
 
 }  // namespace om
@@ -542,7 +648,7 @@ bool sim_tc_supported(int L, int E);
 int sim_tc_nsplit(int L, int E, int64_t N);
 int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int d, int kf,
                   float* H, uint16_t* hi, uint16_t* lo, int ldT, int32_t* counts, float* gpart,
-                  int nsplit, cudaStream_t stream);
+                  int nsplit, bool reserve_sm, cudaStream_t stream);
 }  // namespace om
 
 // Workspace: H [N][L E] fp32 | the hi/lo bf16 planes of H^T [L E][ldT] (tensor-core
@@ -566,11 +672,10 @@ extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
   return up(h) + planes + up(g) + up(gd);
 }
 
-// keep_logits: leave the fp32 calibration logits H in the workspace (the
-// input of ordermoe_transitions); the tensor-core path can skip writing them.
-static int similarity_impl(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
-                           int64_t N, int k_freq, float* sim, int32_t* counts, void* workspace,
-                           size_t workspace_bytes, bool keep_logits, cudaStream_t stream) {
+// The similarity arguments a call needs (Eqs. 3-5), checked.
+static int similarity_check(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
+                            int64_t N, int k_freq, const float* sim, const int32_t* counts,
+                            const void* workspace, size_t workspace_bytes) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: need L >= 1, 1 <= k_freq <= E <= 64");
   if (d <= 0 || d % 64 != 0)
@@ -583,31 +688,67 @@ static int similarity_impl(const uint16_t* W_r, const uint16_t* X_cal, int L, in
     return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: W_r/X_cal 16-byte and workspace 256-byte aligned");
   if (workspace_bytes < ordermoe_similarity_workspace_bytes(L, E, N))
     return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: workspace too small");
-  const int nchunks = static_cast<int>((N + kSimChunk - 1) / kSimChunk);
+  return ORDERMOE_OK;
+}
+
+// Where the similarity's scratch lives in its workspace.
+struct SimLayout {
+  float* H;
+  uint16_t* hi;
+  uint16_t* lo;
+  float* gpart;
+  double* G;
+  int64_t ldT;
+  int nchunks;
+  bool tc;
+};
+
+static SimLayout similarity_layout(void* workspace, int L, int E, int64_t N) {
   auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
+  SimLayout w;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  float* H = reinterpret_cast<float*>(ws);
-  const bool tc = sim_tc_supported(L, E);
-  const int64_t ldT = sim_ldT(N);
-  const size_t plane = up((size_t)L * E * ldT * 2);
-  uint16_t* hi = reinterpret_cast<uint16_t*>(ws + up((size_t)N * L * E * sizeof(float)));
-  uint16_t* lo = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(hi) + plane);
-  float* gpart = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(hi) + (tc ? 2 * plane : 0));
-  int64_t parts = nchunks;
-  if (tc && (N + 63) / 64 > parts) parts = (N + 63) / 64;
-  double* G = reinterpret_cast<double*>(reinterpret_cast<uint8_t*>(gpart) +
-                                        up((size_t)L * parts * 64 * 64 * sizeof(float)));
+  w.H = reinterpret_cast<float*>(ws);
+  w.tc = sim_tc_supported(L, E);
+  w.nchunks = static_cast<int>((N + kSimChunk - 1) / kSimChunk);
+  w.ldT = sim_ldT(N);
+  const size_t plane = up((size_t)L * E * w.ldT * 2);
+  w.hi = reinterpret_cast<uint16_t*>(ws + up((size_t)N * L * E * sizeof(float)));
+  w.lo = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(w.hi) + plane);
+  w.gpart = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(w.hi) + (w.tc ? 2 * plane : 0));
+  int64_t parts = w.nchunks;
+  if (w.tc && (N + 63) / 64 > parts) parts = (N + 63) / 64;
+  w.G = reinterpret_cast<double*>(reinterpret_cast<uint8_t*>(w.gpart) +
+                                  up((size_t)L * parts * 64 * 64 * sizeof(float)));
+  return w;
+}
+
+// keep_logits: leave the fp32 calibration logits H in the workspace (the
+// input of ordermoe_transitions); the tensor-core path can skip writing them.
+static int similarity_impl(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
+                           int64_t N, int k_freq, float* sim, int32_t* counts, void* workspace,
+                           size_t workspace_bytes, bool keep_logits, cudaStream_t stream) {
+  int rc0 = similarity_check(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, workspace_bytes);
+  if (rc0) return rc0;
+  const SimLayout w = similarity_layout(workspace, L, E, N);
+  float* H = w.H;
+  uint16_t* hi = w.hi;
+  uint16_t* lo = w.lo;
+  float* gpart = w.gpart;
+  double* G = w.G;
+  const bool tc = w.tc;
+  const int64_t ldT = w.ldT;
+  const int nchunks = w.nchunks;
   OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, stream));
   if (tc) {
     // tensor-core path: logits with fused counts and hi/lo planes, then the Gram
     const int nsplit = sim_tc_nsplit(L, E, N);
     int rc = sim_tc_launch(X_cal, static_cast<int>(N), W_r, L, E, d, k_freq,
                            keep_logits ? H : nullptr, hi, lo, static_cast<int>(ldT), counts, gpart,
-                           nsplit, stream);
+                           nsplit, false, stream);
     if (rc) return rc;
     gram_reduce_kernel<<<dim3(L, 16), 256, 0, stream>>>(gpart, nsplit, G);
     OM_LAUNCHED("gram_reduce_kernel");
-    sim_finish_kernel<<<L, 256, 0, stream>>>(G, E, sim);
+    sim_finish_kernel<<<dim3(L, 16), 256, 0, stream>>>(G, E, sim);
     OM_LAUNCHED("sim_finish_kernel");
     return ORDERMOE_OK;
   }
@@ -626,7 +767,7 @@ static int similarity_impl(const uint16_t* W_r, const uint16_t* X_cal, int L, in
   OM_LAUNCHED("gram_kernel");
   gram_reduce_kernel<<<dim3(L, 16), 256, 0, stream>>>(gpart, nchunks, G);
   OM_LAUNCHED("gram_reduce_kernel");
-  sim_finish_kernel<<<L, 256, 0, stream>>>(G, E, sim);
+  sim_finish_kernel<<<dim3(L, 16), 256, 0, stream>>>(G, E, sim);
   OM_LAUNCHED("sim_finish_kernel");
   return ORDERMOE_OK;
 }
@@ -844,10 +985,11 @@ extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, in
     return fail(ORDERMOE_ERR_INVALID_ARG, "place: workspace missing or too small");
   int32_t* porder_scratch = static_cast<int32_t*>(workspace);
   PlaceParams pp{theta_min, theta_max, theta_single, alpha_f, alpha_r, lambda1, lambda2};
-  group_kernel<<<L, 64, 0, stream>>>(sim, counts, L, E, pp, p, group, n_groups, theta, importance,
+  group_kernel<<<L, 64, 0, stream>>>(sim, counts, L, E, 0, pp, p, group, n_groups, theta, importance,
                                      porder_scratch);
   OM_LAUNCHED("group_kernel");
-  place_kernel<<<1, 32, 0, stream>>>(group, porder_scratch, L, E, M, pp, p, C, placement, used, status);
+  place_kernel<<<1, 64, 0, stream>>>(group, porder_scratch, L, E, M, 0, L, 1, pp, p, C, placement,
+                                     used, status);
   OM_LAUNCHED("place_kernel");
   return ORDERMOE_OK;
 }
@@ -891,8 +1033,16 @@ extern "C" int ordermoe_replicate(const int32_t* group, const double* importance
   while (Np < L * E) Np <<= 1;
   const size_t smem = (size_t)Np * (sizeof(unsigned long long) + sizeof(uint32_t)) +
                       (size_t)L * sizeof(unsigned long long);
-  OM_CUDA(cudaFuncSetAttribute(replicate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)smem));
+  // once per device, for the largest sort (no attribute call per launch, so
+  // the call can be captured into a CUDA graph)
+  static PerDevice attr;
+  const cudaError_t ae = static_cast<cudaError_t>(per_device(attr, [] {
+    const size_t most = (size_t)kRepMaxCand * (sizeof(unsigned long long) + sizeof(uint32_t)) +
+                        (size_t)kRepMaxLayers * sizeof(unsigned long long);
+    return static_cast<int>(cudaFuncSetAttribute(
+        replicate_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)most));
+  }));
+  if (ae != cudaSuccess) return cuda_fail(ae, "cudaFuncSetAttribute(replicate_kernel)");
   replicate_kernel<<<M, kRepThreads, smem, stream>>>(group, importance, p, C, pi, L, E, M, Np,
                                                      placement, used, replicas);
   OM_LAUNCHED("replicate_kernel");
@@ -922,4 +1072,133 @@ extern "C" int ordermoe_selftest_div_rn(const double* a, const double* b, double
   div_selftest_kernel<<<static_cast<int>(blocks), 256, 0, stream>>>(a, b, out, n);
   OM_LAUNCHED("div_selftest_kernel");
   return ORDERMOE_OK;
+}
+
+// ----------------------------------------------------------------------------
+// The whole offline plan in one call (Alg. 1): similarity (Eqs. 3-5), grouping
+// (Eqs. 6, 24-28), mandatory placement (Eqs. 29-31), redundant deployment
+// (Eqs. 32-35) and coverage (Eq. 32). On the tensor-core path the layers go in
+// blocks of 512 logit columns: the caller's stream runs a block's logits GEMM,
+// Gram and similarities, and a side stream, behind an event, runs that
+// block's grouping and placement while the next block's GEMM runs. The
+// placement carries b_m from block to block in `used`; its layers stay in
+// order because the side stream runs the blocks in order. The results are
+// those of ordermoe_similarity_no_logits, ordermoe_place, ordermoe_replicate
+// and ordermoe_coverage called one after the other.
+namespace om {
+
+int sim_tc_part_layers(int E);
+
+struct PlanSync {
+  cudaStream_t side;
+  cudaEvent_t ev[4];
+};
+static PlanSync g_plan_sync[64];
+static PerDevice g_plan_sync_once;
+
+static int plan_sync(PlanSync** out) {
+  int dev = 0;
+  OM_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 64) return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "plan: device index above 63");
+  const int e = per_device(g_plan_sync_once, [dev] {
+    PlanSync& ps = g_plan_sync[dev];
+    cudaError_t err = cudaFuncSetAttribute(group_place_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           static_cast<int>(kGroupPlaceSmem));
+    if (err == cudaSuccess) err = cudaStreamCreateWithFlags(&ps.side, cudaStreamNonBlocking);
+    for (int i = 0; i < 4 && err == cudaSuccess; ++i)
+      err = cudaEventCreateWithFlags(&ps.ev[i], cudaEventDisableTiming);
+    return static_cast<int>(err);
+  });
+  if (e != cudaSuccess) return cuda_fail(static_cast<cudaError_t>(e), "plan: side stream and events");
+  *out = &g_plan_sync[dev];
+  return ORDERMOE_OK;
+}
+
+static int launched(const char* what) {
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? ORDERMOE_OK : cuda_fail(e, what);
+}
+
+}  // namespace om
+
+extern "C" size_t ordermoe_plan_workspace_bytes(int L, int E, int64_t N) {
+  const size_t a = ordermoe_similarity_workspace_bytes(L, E, N);  // a multiple of 256
+  const size_t b = ordermoe_place_workspace_bytes(L, E);
+  return (a == 0 || b == 0) ? 0 : a + b;
+}
+
+extern "C" int ordermoe_plan(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
+                             int64_t N, int k_freq, int M, double theta_min, double theta_max,
+                             double theta_single, double alpha_f, double alpha_r, double lambda1,
+                             double lambda2, const double* p, const double* C, const double* pi,
+                             float* sim, int32_t* counts, int32_t* group, int32_t* n_groups,
+                             float* theta, double* importance, uint8_t* placement, double* used,
+                             int32_t* status, int32_t* replicas, uint8_t* cover, int32_t* covered,
+                             void* workspace, size_t workspace_bytes, ordermoe_stream_t stream) {
+  OM_TRACE();
+  const size_t sim_ws = ordermoe_similarity_workspace_bytes(L, E, N);
+  int rc = similarity_check(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, sim_ws);
+  if (rc) return rc;
+  if (M <= 0 || M > ORDERMOE_MAX_SERVERS || L > kRepMaxLayers || (long long)L * E > kRepMaxCand)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
+                "plan: need 1 <= M <= 32, L <= 1024 and L * E <= 16384");
+  if (!p || !C || !pi || !group || !n_groups || !theta || !importance || !placement || !used ||
+      !status || !replicas)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "plan: null pointer");
+  if (workspace_bytes < ordermoe_plan_workspace_bytes(L, E, N))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "plan: workspace too small");
+  int32_t* porder = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + sim_ws);
+  const size_t porder_bytes = workspace_bytes - sim_ws;
+  cudaStream_t S = static_cast<cudaStream_t>(stream);
+  const SimLayout w = similarity_layout(workspace, L, E, N);
+  if (!w.tc) {  // the CUDA-core similarity needs every layer's logits at once
+    rc = similarity_impl(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, sim_ws, false, S);
+    if (!rc)
+      rc = ordermoe_place(sim, counts, L, E, M, theta_min, theta_max, theta_single, alpha_f, alpha_r,
+                          lambda1, lambda2, p, C, group, n_groups, theta, importance, placement,
+                          used, status, porder, porder_bytes, stream);
+  } else {
+    PlanSync* ps = nullptr;
+    if ((rc = plan_sync(&ps))) return rc;
+    OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, S));
+    OM_CUDA(cudaEventRecord(ps->ev[0], S));
+    OM_CUDA(cudaStreamWaitEvent(ps->side, ps->ev[0], 0));
+    const PlaceParams pp{theta_min, theta_max, theta_single, alpha_f, alpha_r, lambda1, lambda2};
+    const int part = sim_tc_part_layers(E);
+    const int nsplit = sim_tc_nsplit(L, E, N);
+    for (int l0 = 0, k = 0; l0 < L && !rc; l0 += part, ++k) {
+      const int lp = L - l0 < part ? L - l0 : part;
+      const size_t rows = (size_t)l0 * E;
+      float* gpart = w.gpart + (size_t)l0 * nsplit * 4096;
+      double* G = w.G + (size_t)l0 * 4096;
+      rc = sim_tc_launch(X_cal, static_cast<int>(N), W_r + rows * d, lp, E, d, k_freq, nullptr,
+                         w.hi + rows * w.ldT, w.lo + rows * w.ldT, static_cast<int>(w.ldT),
+                         counts + rows, gpart, nsplit, true, S);
+      if (rc) break;
+      gram_reduce_kernel<<<dim3(lp, 16), 256, 0, S>>>(gpart, nsplit, G);
+      if ((rc = launched("gram_reduce_kernel"))) break;
+      sim_finish_kernel<<<dim3(lp, 16), 256, 0, S>>>(G, E, sim + rows * E);
+      if ((rc = launched("sim_finish_kernel"))) break;
+      cudaEvent_t ev = ps->ev[1 + (k & 1)];
+      cudaError_t e = cudaEventRecord(ev, S);
+      if (e == cudaSuccess) e = cudaStreamWaitEvent(ps->side, ev, 0);
+      if (e != cudaSuccess) {
+        rc = cuda_fail(e, "plan: block event");
+        break;
+      }
+      group_place_kernel<<<1, 64 * kGroupSlices, kGroupPlaceSmem, ps->side>>>(
+          sim, counts, L, E, M, l0, l0 + lp, l0 == 0 ? 1 : 0, pp, p, C, group, n_groups, theta,
+          importance, porder, placement, used, status);
+      if ((rc = launched("group_place_kernel"))) break;
+    }
+    // every exit after the fork joins the side stream back into the caller's
+    cudaError_t e = cudaEventRecord(ps->ev[3], ps->side);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(S, ps->ev[3], 0);
+    if (!rc && e != cudaSuccess) rc = cuda_fail(e, "plan: join");
+  }
+  if (!rc)
+    rc = ordermoe_replicate(group, importance, p, C, pi, L, E, M, placement, used, replicas, stream);
+  if (!rc) rc = ordermoe_coverage(group, placement, L, E, M, cover, covered, stream);
+  return rc;
 }

@@ -481,3 +481,103 @@ def test_layer_forward_batches_matches_single_calls():
         B.ordermoe_layer_forward(desc, T, X[b], home[b], None, None, y1, host_io=1)
         torch.cuda.synchronize()
         assert torch.equal(y[b], y1), b
+
+
+def _plan_inputs(L, E, d, N, M, seed, unequal):
+    Wr = torch.stack([synth.router_weights(E, d, 4, seed=seed + 70 + l) for l in range(L)]).to(DEV).contiguous()
+    Xcal = synth.calibration(N, d, seed=seed + 3).to(DEV)
+    rng = np.random.default_rng(seed)
+    p = rng.integers(1, 4, (L, E)).astype(np.float64) if unequal else np.ones((L, E))
+    C = synth.capacities(M, p.sum(), 1.6, seed)
+    pi = synth.token_shares(synth.homes(4096, M, seed, "zipf1.1"), M)
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a)).to(device=DEV, dtype=dt)
+    return Wr, Xcal, t(p, torch.float64), t(C, torch.float64), t(pi, torch.float64)
+
+
+def _plan_outputs(L, E, M):
+    f = lambda *s, dt: torch.full(s, 7, dtype=dt, device=DEV)
+    return dict(sim=f(L, E, E, dt=torch.float32), counts=f(L, E, dt=torch.int32),
+                group=f(L, E, dt=torch.int32), n_groups=f(L, dt=torch.int32),
+                theta=f(L, dt=torch.float32), importance=f(L, E, dt=torch.float64),
+                placement=f(L, M, E, dt=torch.uint8), used=f(M, dt=torch.float64),
+                status=f(1, dt=torch.int32), replicas=f(M, dt=torch.int32),
+                cover=f(L, M, E, dt=torch.uint8), covered=f(L, dt=torch.int32))
+
+
+TH = (0.5, 0.9, 0.6, 0.5, 0.5, 0.5, 0.5)  # theta_min, theta_max, theta_single, alpha_f, alpha_r, lambda1, lambda2
+
+
+def _serial_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi):
+    o = _plan_outputs(L, E, M)
+    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+    B.ordermoe_similarity_no_logits(Wr, Xcal, L, E, d, N, kf, o["sim"], o["counts"], ws)
+    B.ordermoe_place(o["sim"], o["counts"], L, E, M, *TH, p, C, o["group"], o["n_groups"], o["theta"],
+                     o["importance"], o["placement"], o["used"], o["status"])
+    B.ordermoe_replicate(o["group"], o["importance"], p, C, pi, L, E, M, o["placement"], o["used"],
+                         o["replicas"])
+    B.ordermoe_coverage(o["group"], o["placement"], L, E, M, o["cover"], o["covered"])
+    return o
+
+
+def _one_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi, ws, stream=None):
+    o = _plan_outputs(L, E, M)
+    B.ordermoe_plan(Wr, Xcal, L, E, d, N, kf, M, *TH, p, C, pi, o["sim"], o["counts"], o["group"],
+                    o["n_groups"], o["theta"], o["importance"], o["placement"], o["used"], o["status"],
+                    o["replicas"], o["cover"], o["covered"], ws, stream=stream)
+    return o
+
+
+def _same(a, b, what):
+    for k in a:
+        assert torch.equal(a[k], b[k]), "%s: %s differs" % (what, k)
+
+
+@pytest.mark.parametrize("L,E,N,M,kf,unequal", [(24, 64, 4096, 8, 6, False), (13, 64, 3000, 4, 6, True),
+                                                 (1, 64, 1000, 3, 2, False), (20, 32, 2100, 5, 4, True),
+                                                 (40, 16, 1500, 16, 3, False), (80, 8, 1200, 6, 2, True),
+                                                 (3, 12, 900, 3, 3, False)])
+def test_plan_equals_the_four_calls(L, E, N, M, kf, unequal):
+    """ordermoe_plan (blocks of 512 logit columns; grouping and placement of a
+    block on a side stream while the next block's GEMM runs) writes what the
+    four calls write one after the other, bit for bit: ragged last blocks,
+    b_m carried across blocks, E = 12 on the one-stream path."""
+    d = 128
+    Wr, Xcal, p, C, pi = _plan_inputs(L, E, d, N, M, L * 7 + E, unequal)
+    ref = _serial_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi)
+    ws = torch.empty(B.ordermoe_plan_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+    got = _one_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi, ws)
+    torch.cuda.synchronize()
+    _same(got, ref, "plan")
+    assert int(ref["status"].item()) in (B.OK, B.ERR_CAPACITY)
+    assert (got["placement"].sum(dim=1) >= 1).all()  # every expert somewhere
+
+
+def test_plan_back_to_back_and_in_a_cuda_graph():
+    """Calls queued back to back on one stream (the library's events reused)
+    and a captured-and-replayed call give the single call's results; work
+    queued after the call on the caller's stream sees its outputs."""
+    L, E, d, N, M, kf = 13, 64, 128, 2000, 6, 6
+    Wr, Xcal, p, C, pi = _plan_inputs(L, E, d, N, M, 5, True)
+    ws = torch.empty(B.ordermoe_plan_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+    ref = _one_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi, ws)
+    torch.cuda.synchronize()
+    runs = [_one_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi, ws) for _ in range(3)]
+    after = [r["placement"].to(torch.int32).sum() for r in runs]  # queued behind each call
+    torch.cuda.synchronize()
+    for r, a in zip(runs, after):
+        _same(r, ref, "back to back")
+        assert int(a.item()) == int(ref["placement"].to(torch.int32).sum().item())
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(s):
+        o = _plan_outputs(L, E, M)
+        with torch.cuda.graph(g, stream=s):
+            B.ordermoe_plan(Wr, Xcal, L, E, d, N, kf, M, *TH, p, C, pi, o["sim"], o["counts"], o["group"],
+                            o["n_groups"], o["theta"], o["importance"], o["placement"], o["used"],
+                            o["status"], o["replicas"], o["cover"], o["covered"], ws)
+    for v in o.values():
+        v.fill_(7)
+    g.replay()
+    torch.cuda.synchronize()
+    _same(o, ref, "graph replay")
