@@ -659,13 +659,17 @@ def run_decode(args, dist, w, device):
 
 def plan_launches(L, E):
     """Kernels of one ordermoe_plan call: on the tensor-core path (E in {8,
-    16, 32, 64}, L E <= 4096) each block of 512 logit columns launches the
-    logits GEMM, the Gram, its reduction, the similarities, the grouping and
-    the placement; otherwise the similarity takes 5 and the placement 2.
-    Replication and coverage add 1 each."""
+    16, 32, 64}, L E <= 4096) the layers go in blocks of 512 logit columns,
+    the last block in two halves when there is more than one, and each block
+    launches the logits GEMM, the Gram, its reduction, the similarities and
+    one grouping + placement kernel (5); otherwise the similarity takes 5 and
+    the placement 2. Replication and coverage add 1 each."""
     if E in (8, 16, 32, 64) and L * E <= 4096:
         part = max(1, 512 // E)
-        return 6 * ((L + part - 1) // part) + 2
+        nfull = (L + part - 1) // part
+        last_n = L - (nfull - 1) * part
+        blocks = nfull + (1 if nfull > 1 and last_n >= 2 else 0)
+        return 5 * blocks + 2
     return 5 + 2 + 2
 
 

@@ -441,13 +441,15 @@ int ordermoe_coverage(const int32_t* group, const uint8_t* placement, int L, int
  * and coverage (Eq. 32). Every output equals, bit for bit, what
  * ordermoe_similarity_no_logits, ordermoe_place, ordermoe_replicate and
  * ordermoe_coverage write when called in that order with the same arguments.
- * For E in {8, 16, 32, 64} the layers go in blocks of 512 logit columns
- * (8 layers of 64 experts): the caller's stream computes a block's logits,
+ * For E in {8, 16, 32, 64} and L * E <= 4096 the layers go in blocks of 512 logit columns
+ * (8 layers of 64 experts; the last block in two halves when there are
+ * several, so that less grouping and placement is left after the last GEMM):
+ * the caller's stream computes a block's logits,
  * Gram and similarities while a side stream of the library, ordered behind it
  * by events, groups and places the block before; the call joins the side
  * stream back into the caller's before replication, so work queued on the
  * caller's stream afterwards sees every output (CUDA graph capture included).
- * Other E run the steps one after the other on the caller's stream.
+ * Otherwise the steps run one after the other on the caller's stream.
  *   Arguments as in those four calls: W_r [L][E][d] bf16, X_cal [N][d] bf16;
  *   p [L][E] f64, C [M] f64, pi [M] f64; sim [L][E][E] f32, counts [L][E] i32,
  *   group [L][E] i32, n_groups [L] i32, theta [L] f32, importance [L][E] f64

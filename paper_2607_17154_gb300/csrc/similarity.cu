@@ -1078,7 +1078,8 @@ extern "C" int ordermoe_selftest_div_rn(const double* a, const double* b, double
 // The whole offline plan in one call (Alg. 1): similarity (Eqs. 3-5), grouping
 // (Eqs. 6, 24-28), mandatory placement (Eqs. 29-31), redundant deployment
 // (Eqs. 32-35) and coverage (Eq. 32). On the tensor-core path the layers go in
-// blocks of 512 logit columns: the caller's stream runs a block's logits GEMM,
+// blocks of 512 logit columns (the last block in two halves when there are
+// several): the caller's stream runs a block's logits GEMM,
 // Gram and similarities, and a side stream, behind an event, runs that
 // block's grouping and placement while the next block's GEMM runs. The
 // placement carries b_m from block to block in `used`; its layers stay in
@@ -1167,8 +1168,13 @@ extern "C" int ordermoe_plan(const uint16_t* W_r, const uint16_t* X_cal, int L, 
     const PlaceParams pp{theta_min, theta_max, theta_single, alpha_f, alpha_r, lambda1, lambda2};
     const int part = sim_tc_part_layers(E);
     const int nsplit = sim_tc_nsplit(L, E, N);
-    for (int l0 = 0, k = 0; l0 < L && !rc; l0 += part, ++k) {
-      const int lp = L - l0 < part ? L - l0 : part;
+    // the last block's grouping and placement are not hidden behind a GEMM:
+    // when there is more than one block, the last one goes in two halves
+    const int nfull = (L + part - 1) / part;
+    const int last0 = (nfull - 1) * part, last_n = L - last0;
+    for (int l0 = 0, k = 0; l0 < L && !rc; ++k) {
+      int lp = L - l0 < part ? L - l0 : part;
+      if (nfull > 1 && l0 >= last0 && last_n >= 2) lp = l0 == last0 ? (last_n + 1) / 2 : L - l0;
       const size_t rows = (size_t)l0 * E;
       float* gpart = w.gpart + (size_t)l0 * nsplit * 4096;
       double* G = w.G + (size_t)l0 * 4096;
@@ -1191,6 +1197,7 @@ extern "C" int ordermoe_plan(const uint16_t* W_r, const uint16_t* X_cal, int L, 
           sim, counts, L, E, M, l0, l0 + lp, l0 == 0 ? 1 : 0, pp, p, C, group, n_groups, theta,
           importance, porder, placement, used, status);
       if ((rc = launched("group_place_kernel"))) break;
+      l0 += lp;
     }
     // every exit after the fork joins the side stream back into the caller's
     cudaError_t e = cudaEventRecord(ps->ev[3], ps->side);
