@@ -581,3 +581,36 @@ def test_plan_back_to_back_and_in_a_cuda_graph():
     g.replay()
     torch.cuda.synchronize()
     _same(o, ref, "graph replay")
+
+
+def test_plan_argument_errors_and_nullable_coverage():
+    """Argument errors come back before anything is enqueued; cover and
+    covered may be omitted."""
+    L, E, d, N, M, kf = 3, 64, 128, 700, 4, 6
+    Wr, Xcal, p, C, pi = _plan_inputs(L, E, d, N, M, 9, False)
+    ws = torch.empty(B.ordermoe_plan_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+    o = _plan_outputs(L, E, M)
+    args = lambda **kw: dict(dict(sim=o["sim"], counts=o["counts"], group=o["group"], n_groups=o["n_groups"],
+                                  theta=o["theta"], importance=o["importance"], placement=o["placement"],
+                                  used=o["used"], status=o["status"], replicas=o["replicas"],
+                                  cover=None, covered=None, workspace=ws), **kw)
+
+    def call(L_=L, E_=E, M_=M, kf_=kf, **kw):
+        a = args(**kw)
+        B.ordermoe_plan(Wr, Xcal, L_, E_, d, N, kf_, M_, *TH, p, C, pi, a["sim"], a["counts"], a["group"],
+                        a["n_groups"], a["theta"], a["importance"], a["placement"], a["used"], a["status"],
+                        a["replicas"], a["cover"], a["covered"], a["workspace"])
+
+    call()  # cover and covered omitted
+    torch.cuda.synchronize()
+    ref = _one_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi, ws)
+    torch.cuda.synchronize()
+    for k in ("sim", "group", "placement", "used", "replicas"):
+        assert torch.equal(o[k], ref[k]), k
+    for kw, code in [(dict(importance=None), B.ERR_INVALID_ARG), (dict(workspace=ws[:1024]), B.ERR_INVALID_ARG),
+                     (dict(M_=33), B.ERR_UNSUPPORTED_SHAPE), (dict(kf_=65), B.ERR_UNSUPPORTED_SHAPE),
+                     (dict(E_=65), B.ERR_UNSUPPORTED_SHAPE)]:
+        with pytest.raises(B.OrderMoEError) as ei:
+            call(**kw)
+        assert ei.value.code == code, kw
+    torch.cuda.synchronize()
