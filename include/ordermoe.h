@@ -449,7 +449,10 @@ int ordermoe_coverage(const int32_t* group, const uint8_t* placement, int L, int
  * by events, groups and places the block before; the call joins the side
  * stream back into the caller's before replication, so work queued on the
  * caller's stream afterwards sees every output (CUDA graph capture included).
- * Otherwise the steps run one after the other on the caller's stream.
+ * The side stream is the device's, shared by all calls: calls from several
+ * host threads are enqueued one at a time, and their side-stream work runs in
+ * that order. Otherwise the steps run one after the other on the caller's
+ * stream.
  *   Arguments as in those four calls: W_r [L][E][d] bf16, X_cal [N][d] bf16;
  *   p [L][E] f64, C [M] f64, pi [M] f64; sim [L][E][E] f32, counts [L][E] i32,
  *   group [L][E] i32, n_groups [L] i32, theta [L] f32, importance [L][E] f64

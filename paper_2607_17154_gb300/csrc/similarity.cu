@@ -1090,7 +1090,12 @@ namespace om {
 
 int sim_tc_part_layers(int E);
 
+// One side stream and its events per device, shared by every call: a call
+// holds `mu` while it enqueues, so calls from several host threads cannot
+// interleave their event records (a stream wait takes the event as it was
+// when the wait was enqueued).
 struct PlanSync {
+  std::mutex mu;
   cudaStream_t side;
   cudaEvent_t ev[4];
 };
@@ -1162,6 +1167,7 @@ extern "C" int ordermoe_plan(const uint16_t* W_r, const uint16_t* X_cal, int L, 
   } else {
     PlanSync* ps = nullptr;
     if ((rc = plan_sync(&ps))) return rc;
+    std::lock_guard<std::mutex> hold(ps->mu);
     OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * L * E, S));
     OM_CUDA(cudaEventRecord(ps->ev[0], S));
     OM_CUDA(cudaStreamWaitEvent(ps->side, ps->ev[0], 0));

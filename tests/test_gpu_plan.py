@@ -614,3 +614,45 @@ def test_plan_argument_errors_and_nullable_coverage():
             call(**kw)
         assert ei.value.code == code, kw
     torch.cuda.synchronize()
+
+
+def test_plan_from_two_host_threads():
+    """Two host threads, each on its own stream, call the plan at the same
+    time with different inputs (the device's side stream and events are
+    shared): every call writes its own single-call results."""
+    import threading
+    cases = [(13, 64, 128, 1500, 5, 6, 21), (9, 32, 128, 1200, 3, 4, 22)]
+    prepared = []
+    for L, E, d, N, M, kf, seed in cases:
+        Wr, Xcal, p, C, pi = _plan_inputs(L, E, d, N, M, seed, True)
+        ws = torch.empty(B.ordermoe_plan_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+        ref = _one_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi, ws)
+        prepared.append(((Wr, Xcal, L, E, d, N, kf, M, p, C, pi), ref))
+    torch.cuda.synchronize()
+    results = [[], []]
+    errors = []
+
+    def run(i):
+        try:
+            a, _ = prepared[i]
+            s = torch.cuda.Stream()
+            ws = torch.empty(B.ordermoe_plan_workspace_bytes(a[2], a[3], a[5]), dtype=torch.uint8,
+                             device=DEV)
+            with torch.cuda.stream(s):
+                for _ in range(4):
+                    results[i].append(_one_plan(*a, ws))
+            s.synchronize()
+        except Exception as e:  # reported below, in the test's thread
+            errors.append(e)
+
+    threads = [threading.Thread(target=run, args=(i,)) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    torch.cuda.synchronize()
+    assert not errors, errors
+    for i in range(2):
+        assert len(results[i]) == 4
+        for r in results[i]:
+            _same(r, prepared[i][1], "thread %d" % i)
