@@ -84,8 +84,11 @@ static size_t batch_extra_bytes(int T_max, int d) {
   return up256((size_t)T_max * d * 2) * 2 + up256((size_t)T_max);
 }
 
-// Copy streams and events of the batched entry point, one set per device.
+// Copy streams and events of the batched entry point, one set per device,
+// shared by every call: a call holds `enq` while it enqueues, so calls from
+// several host threads cannot interleave their event records.
 struct BatchStreams {
+  std::mutex enq;
   cudaStream_t h2d = nullptr, d2h = nullptr;
   cudaEvent_t start, end, in_ready[2], x_free[2], y_ready[2], y_free[2];
   bool ok = false;
@@ -232,19 +235,25 @@ extern "C" int ordermoe_layer_forward_batches(const ordermoe_layer_desc* L, int 
   uint8_t* hs[2] = {s.home, extra + 2 * up256((size_t)L->T_max * d * 2)};
   cudaStream_t st = stream;
   const size_t xb = (size_t)T * d * 2;
+  std::lock_guard<std::mutex> hold(bs->enq);
   // the copy streams start after everything already on the caller's stream
   OM_CUDA(cudaEventRecord(bs->start, st));
   OM_CUDA(cudaStreamWaitEvent(bs->h2d, bs->start, 0));
   OM_CUDA(cudaStreamWaitEvent(bs->d2h, bs->start, 0));
-  for (int b = 0; b < nbatch; ++b) {
+  auto ck = [](cudaError_t e, const char* what) { return e == cudaSuccess ? 0 : cuda_fail(e, what); };
+  int rc = 0;
+  for (int b = 0; b < nbatch && !rc; ++b) {
     const int sl = b & 1;
     // batch b's inputs: after batch b - 2 has finished reading this slot
-    if (b >= 2) OM_CUDA(cudaStreamWaitEvent(bs->h2d, bs->x_free[sl], 0));
-    OM_CUDA(cudaMemcpyAsync(Xs[sl], X + (size_t)b * T * d, xb, cudaMemcpyHostToDevice, bs->h2d));
-    OM_CUDA(cudaMemcpyAsync(hs[sl], home + (size_t)b * T, (size_t)T, cudaMemcpyHostToDevice, bs->h2d));
-    OM_CUDA(cudaEventRecord(bs->in_ready[sl], bs->h2d));
-    OM_CUDA(cudaStreamWaitEvent(st, bs->in_ready[sl], 0));
-    int rc;
+    if (b >= 2 && (rc = ck(cudaStreamWaitEvent(bs->h2d, bs->x_free[sl], 0), "wait x_free"))) break;
+    if ((rc = ck(cudaMemcpyAsync(Xs[sl], X + (size_t)b * T * d, xb, cudaMemcpyHostToDevice, bs->h2d),
+                 "copy X")))
+      break;
+    if ((rc = ck(cudaMemcpyAsync(hs[sl], home + (size_t)b * T, (size_t)T, cudaMemcpyHostToDevice,
+                                 bs->h2d), "copy home")))
+      break;
+    if ((rc = ck(cudaEventRecord(bs->in_ready[sl], bs->h2d), "record in_ready"))) break;
+    if ((rc = ck(cudaStreamWaitEvent(st, bs->in_ready[sl], 0), "wait in_ready"))) break;
     if (L->lookahead_H > 1)
       rc = ordermoe_route_select_lookahead(Xs[sl], L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
                                            L->tables_stride, L->lookahead_H, L->P, hs[sl], nullptr,
@@ -254,26 +263,33 @@ extern "C" int ordermoe_layer_forward_batches(const ordermoe_layer_desc* L, int 
       rc = ordermoe_route_select(Xs[sl], L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
                                  L->tables_bytes, hs[sl], nullptr, nullptr, nullptr, s.topk_idx,
                                  s.topk_w, s.chosen, s.server, s.kind, counters, st);
-    if (rc) return rc;
+    if (rc) break;
     rc = dispatch_launch(s.chosen, Xs[sl], T, k, E, d, s.offsets, s.row_token, s.row_of, s.X_perm,
                          s.hist, st);
-    if (rc) return rc;
-    OM_CUDA(cudaEventRecord(bs->x_free[sl], st));  // X and home of this slot are read
+    if (rc) break;
+    if ((rc = ck(cudaEventRecord(bs->x_free[sl], st), "record x_free"))) break;  // slot's X, home read
     rc = gate_up_launch(s.X_perm, s.offsets, R, L->W1, L->W3, E, d, dff, s.H, st);
-    if (rc) return rc;
+    if (rc) break;
     rc = down_launch(s.H, s.offsets, R, L->W2, E, d, dff, s.Y_perm, st);
-    if (rc) return rc;
+    if (rc) break;
     // the output slot: after batch b - 2's copy out has read it
-    if (b >= 2) OM_CUDA(cudaStreamWaitEvent(st, bs->y_free[sl], 0));
+    if (b >= 2 && (rc = ck(cudaStreamWaitEvent(st, bs->y_free[sl], 0), "wait y_free"))) break;
     rc = ordermoe_combine(s.Y_perm, s.row_of, s.topk_w, T, k, d, ys[sl], st);
-    if (rc) return rc;
-    OM_CUDA(cudaEventRecord(bs->y_ready[sl], st));
-    OM_CUDA(cudaStreamWaitEvent(bs->d2h, bs->y_ready[sl], 0));
-    OM_CUDA(cudaMemcpyAsync(y + (size_t)b * T * d, ys[sl], xb, cudaMemcpyDeviceToHost, bs->d2h));
-    OM_CUDA(cudaEventRecord(bs->y_free[sl], bs->d2h));
+    if (rc) break;
+    if ((rc = ck(cudaEventRecord(bs->y_ready[sl], st), "record y_ready"))) break;
+    if ((rc = ck(cudaStreamWaitEvent(bs->d2h, bs->y_ready[sl], 0), "wait y_ready"))) break;
+    if ((rc = ck(cudaMemcpyAsync(y + (size_t)b * T * d, ys[sl], xb, cudaMemcpyDeviceToHost, bs->d2h),
+                 "copy y")))
+      break;
+    if ((rc = ck(cudaEventRecord(bs->y_free[sl], bs->d2h), "record y_free"))) break;
   }
-  // the caller's stream is ordered after every copy of this call
-  OM_CUDA(cudaEventRecord(bs->end, bs->d2h));
-  OM_CUDA(cudaStreamWaitEvent(st, bs->end, 0));
-  return ORDERMOE_OK;
+  // the caller's stream is ordered after every copy of this call, on every
+  // exit once the copy streams have been forked (the error of a failed step
+  // stays the one returned)
+  cudaError_t e = cudaEventRecord(bs->end, bs->h2d);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(st, bs->end, 0);
+  if (e == cudaSuccess) e = cudaEventRecord(bs->end, bs->d2h);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent(st, bs->end, 0);
+  if (!rc && e != cudaSuccess) rc = cuda_fail(e, "layer_forward_batches: join");
+  return rc;
 }

@@ -483,6 +483,62 @@ def test_layer_forward_batches_matches_single_calls():
         assert torch.equal(y[b], y1), b
 
 
+def test_layer_forward_batches_from_two_host_threads():
+    """Two host threads, each with its own layer scratch and stream, run the
+    batched host-I/O entry point at the same time (the device's copy streams
+    and events are shared): each gets its single-call outputs."""
+    import threading
+    w = synth.workload("tiny")
+    E, d, dff, k, M = w.E, w.d, w.dff, w.k, w.M
+    T, nb = 128, 4
+    inp = synth.layer_inputs(w, seed=5, device=DEV)
+    rng = np.random.default_rng(5)
+    sim, group, x = random_tables_case(rng, E, M, 2)
+    tab = build_tables(sim, group, x, 0.5, w.qbar, synth.server_params(M, d, dff, 0), DEV)
+    jobs = []
+    for i in range(2):
+        scratch = torch.empty(B.ordermoe_layer_batches_scratch_bytes(T, E, d, dff, k), dtype=torch.uint8,
+                              device=DEV)
+        desc = B.make_layer_desc(T, inp["Wr"], inp["W1"], inp["W3"], inp["W2"], tab, k, scratch)
+        X = torch.stack([synth.hidden(T, d, 80 + 10 * i + b) for b in range(nb)]).pin_memory()
+        home = torch.as_tensor(rng.integers(0, M, (nb, T)).astype(np.uint8)).pin_memory()
+        ref = []
+        for b in range(nb):
+            y1 = torch.zeros(T, d, dtype=torch.bfloat16).pin_memory()
+            B.ordermoe_layer_forward(desc, T, X[b], home[b], None, None, y1, host_io=1)
+            ref.append(y1)
+        jobs.append((desc, scratch, X, home, ref))
+    torch.cuda.synchronize()
+    outs = [[], []]
+    errors = []
+
+    def run(i):
+        try:
+            desc, _, X, home, _ = jobs[i]
+            s = torch.cuda.Stream()
+            with torch.cuda.stream(s):
+                for _ in range(3):
+                    y = torch.zeros(nb, T, d, dtype=torch.bfloat16).pin_memory()
+                    B.ordermoe_layer_forward_batches(desc, nb, T, X, home, y, None)
+                    outs[i].append(y)
+            s.synchronize()
+        except Exception as e:  # reported below, in the test's thread
+            errors.append(e)
+
+    threads = [threading.Thread(target=run, args=(i,)) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    torch.cuda.synchronize()
+    assert not errors, errors
+    for i in range(2):
+        assert len(outs[i]) == 3
+        for y in outs[i]:
+            for b in range(nb):
+                assert torch.equal(y[b], jobs[i][4][b]), (i, b)
+
+
 def _plan_inputs(L, E, d, N, M, seed, unequal):
     Wr = torch.stack([synth.router_weights(E, d, 4, seed=seed + 70 + l) for l in range(L)]).to(DEV).contiguous()
     Xcal = synth.calibration(N, d, seed=seed + 3).to(DEV)
