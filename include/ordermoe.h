@@ -297,9 +297,11 @@ int ordermoe_layer_forward(const ordermoe_layer_desc* layer, int T, const uint16
  *   (host); counters as ordermoe_layer_forward.
  *   layer->scratch: ordermoe_layer_batches_scratch_bytes(T_max, E, d, dff, k)
  *   bytes (the layer scratch plus a second staging slot).
- * The call enqueues everything; `stream` is ordered after every copy, so the
- * caller synchronises it before reading y. Calls on the same device from
- * several host threads at once must be serialised by the caller. */
+ * The call enqueues everything; `stream` is ordered after every copy (also
+ * when it returns an error after enqueueing some), so the caller synchronises
+ * it before reading y. Calls on the same device from several host threads are
+ * enqueued one at a time (the copy streams are the device's); each needs its
+ * own layer->scratch. */
 size_t ordermoe_layer_batches_scratch_bytes(int T_max, int E, int d, int dff, int k);
 int ordermoe_layer_forward_batches(const ordermoe_layer_desc* layer, int nbatch, int T,
                                    const uint16_t* X, const uint8_t* home, uint16_t* y,
