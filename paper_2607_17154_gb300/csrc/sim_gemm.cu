@@ -581,6 +581,9 @@ bool sim_tc_supported(int L, int E) {
 // 512 columns a block's GEMM stays compute-bound (about 410 flops per byte).
 int sim_tc_part_layers(int E) { return E >= 512 ? 1 : 512 / E; }
 
+// Most token splits of the Gram (the workspace holds this many partials).
+int sim_tc_max_splits() { return 256; }
+
 // Token splits of the Gram. They depend on E and N only (the row blocks of
 // one part of the pipelined plan fill the GPU), so the partial sums, and the
 // similarities, are the same whether the layers are done in one call or part
@@ -593,6 +596,7 @@ int sim_tc_nsplit(int L, int E, int64_t N) {
   int ns = sms / n_rb;
   if (ns < 1) ns = 1;
   if (ns > kblocks) ns = kblocks;
+  if (ns > sim_tc_max_splits()) ns = sim_tc_max_splits();
   return ns;
 }
 

@@ -646,6 +646,7 @@ using namespace om;
 namespace om {
 bool sim_tc_supported(int L, int E);
 int sim_tc_nsplit(int L, int E, int64_t N);
+int sim_tc_max_splits();
 int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int d, int kf,
                   float* H, uint16_t* hi, uint16_t* lo, int ldT, int32_t* counts, float* gpart,
                   int nsplit, bool reserve_sm, cudaStream_t stream);
@@ -655,27 +656,36 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
 // path) | partial Grams [L][parts][64][64] fp32 | G [L][64][64] fp64.
 static int64_t sim_ldT(int64_t N) { return (N + 7) / 8 * 8; }
 
-extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
+// Partial Grams per layer the workspace holds: one per 1024-token chunk on
+// the CUDA-core path, one per token split (at most sim_tc_max_splits, and at
+// most one per 64-token step) on the tensor-core path.
+static int64_t sim_parts(int L, int E, int64_t N) {
+  if (!sim_tc_supported(L, E)) return (N + kSimChunk - 1) / kSimChunk;
+  const int64_t kb = (N + 63) / 64;
+  return kb < sim_tc_max_splits() ? kb : sim_tc_max_splits();
+}
+
+// Workspace of the similarity: H [N][L E] fp32 (with_H; the CUDA-core path
+// and the logits-keeping call need it), the hi/lo planes (tensor-core path),
+// the partial Grams and G.
+static size_t sim_ws_bytes(int L, int E, int64_t N, bool with_H) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || N <= 0) return 0;
-  const int64_t nchunks = (N + kSimChunk - 1) / kSimChunk;
   auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
-  const size_t h = (size_t)N * L * E * sizeof(float);
+  const size_t h = with_H ? up((size_t)N * L * E * sizeof(float)) : 0;
   const size_t planes = sim_tc_supported(L, E) ? 2 * up((size_t)L * E * sim_ldT(N) * 2) : 0;
-  int64_t parts = nchunks;
-  if (sim_tc_supported(L, E)) {
-    // the split count depends on the device; bound it by the number of 64-token steps
-    const int64_t kb = (N + 63) / 64;
-    if (kb > parts) parts = kb;
-  }
-  const size_t g = (size_t)L * parts * 64 * 64 * sizeof(float);
+  const size_t g = (size_t)L * sim_parts(L, E, N) * 64 * 64 * sizeof(float);
   const size_t gd = (size_t)L * 64 * 64 * sizeof(double);
-  return up(h) + planes + up(g) + up(gd);
+  return h + planes + up(g) + up(gd);
+}
+
+extern "C" size_t ordermoe_similarity_workspace_bytes(int L, int E, int64_t N) {
+  return sim_ws_bytes(L, E, N, true);
 }
 
 // The similarity arguments a call needs (Eqs. 3-5), checked.
 static int similarity_check(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
                             int64_t N, int k_freq, const float* sim, const int32_t* counts,
-                            const void* workspace, size_t workspace_bytes) {
+                            const void* workspace, size_t workspace_bytes, size_t need_bytes) {
   if (L <= 0 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "similarity: need L >= 1, 1 <= k_freq <= E <= 64");
   if (d <= 0 || d % 64 != 0)
@@ -686,7 +696,7 @@ static int similarity_check(const uint16_t* W_r, const uint16_t* X_cal, int L, i
     return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: null pointer");
   if (!aligned16(W_r) || !aligned16(X_cal) || (reinterpret_cast<uintptr_t>(workspace) & 255u))
     return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: W_r/X_cal 16-byte and workspace 256-byte aligned");
-  if (workspace_bytes < ordermoe_similarity_workspace_bytes(L, E, N))
+  if (workspace_bytes < need_bytes)
     return fail(ORDERMOE_ERR_INVALID_ARG, "similarity: workspace too small");
   return ORDERMOE_OK;
 }
@@ -703,22 +713,20 @@ struct SimLayout {
   bool tc;
 };
 
-static SimLayout similarity_layout(void* workspace, int L, int E, int64_t N) {
+static SimLayout similarity_layout(void* workspace, int L, int E, int64_t N, bool with_H) {
   auto up = [](size_t v) { return (v + 255) & ~size_t(255); };
   SimLayout w;
   uint8_t* ws = static_cast<uint8_t*>(workspace);
-  w.H = reinterpret_cast<float*>(ws);
+  w.H = with_H ? reinterpret_cast<float*>(ws) : nullptr;
   w.tc = sim_tc_supported(L, E);
   w.nchunks = static_cast<int>((N + kSimChunk - 1) / kSimChunk);
   w.ldT = sim_ldT(N);
   const size_t plane = up((size_t)L * E * w.ldT * 2);
-  w.hi = reinterpret_cast<uint16_t*>(ws + up((size_t)N * L * E * sizeof(float)));
+  w.hi = reinterpret_cast<uint16_t*>(ws + (with_H ? up((size_t)N * L * E * sizeof(float)) : 0));
   w.lo = reinterpret_cast<uint16_t*>(reinterpret_cast<uint8_t*>(w.hi) + plane);
   w.gpart = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(w.hi) + (w.tc ? 2 * plane : 0));
-  int64_t parts = w.nchunks;
-  if (w.tc && (N + 63) / 64 > parts) parts = (N + 63) / 64;
   w.G = reinterpret_cast<double*>(reinterpret_cast<uint8_t*>(w.gpart) +
-                                  up((size_t)L * parts * 64 * 64 * sizeof(float)));
+                                  up((size_t)L * sim_parts(L, E, N) * 64 * 64 * sizeof(float)));
   return w;
 }
 
@@ -727,9 +735,10 @@ static SimLayout similarity_layout(void* workspace, int L, int E, int64_t N) {
 static int similarity_impl(const uint16_t* W_r, const uint16_t* X_cal, int L, int E, int d,
                            int64_t N, int k_freq, float* sim, int32_t* counts, void* workspace,
                            size_t workspace_bytes, bool keep_logits, cudaStream_t stream) {
-  int rc0 = similarity_check(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, workspace_bytes);
+  int rc0 = similarity_check(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, workspace_bytes,
+                             ordermoe_similarity_workspace_bytes(L, E, N));
   if (rc0) return rc0;
-  const SimLayout w = similarity_layout(workspace, L, E, N);
+  const SimLayout w = similarity_layout(workspace, L, E, N, true);
   float* H = w.H;
   uint16_t* hi = w.hi;
   uint16_t* lo = w.lo;
@@ -1128,8 +1137,14 @@ static int launched(const char* what) {
 
 }  // namespace om
 
+// The similarity part of the plan's workspace: without H on the tensor-core
+// path (the plan keeps no logits), the whole similarity workspace otherwise.
+static size_t plan_sim_bytes(int L, int E, int64_t N) {
+  return sim_ws_bytes(L, E, N, !sim_tc_supported(L, E));
+}
+
 extern "C" size_t ordermoe_plan_workspace_bytes(int L, int E, int64_t N) {
-  const size_t a = ordermoe_similarity_workspace_bytes(L, E, N);  // a multiple of 256
+  const size_t a = plan_sim_bytes(L, E, N);  // a multiple of 256
   const size_t b = ordermoe_place_workspace_bytes(L, E);
   return (a == 0 || b == 0) ? 0 : a + b;
 }
@@ -1143,8 +1158,8 @@ extern "C" int ordermoe_plan(const uint16_t* W_r, const uint16_t* X_cal, int L, 
                              int32_t* status, int32_t* replicas, uint8_t* cover, int32_t* covered,
                              void* workspace, size_t workspace_bytes, ordermoe_stream_t stream) {
   OM_TRACE();
-  const size_t sim_ws = ordermoe_similarity_workspace_bytes(L, E, N);
-  int rc = similarity_check(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, sim_ws);
+  const size_t sim_ws = plan_sim_bytes(L, E, N);
+  int rc = similarity_check(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, sim_ws, sim_ws);
   if (rc) return rc;
   if (M <= 0 || M > ORDERMOE_MAX_SERVERS || L > kRepMaxLayers || (long long)L * E > kRepMaxCand)
     return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
@@ -1157,7 +1172,7 @@ extern "C" int ordermoe_plan(const uint16_t* W_r, const uint16_t* X_cal, int L, 
   int32_t* porder = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(workspace) + sim_ws);
   const size_t porder_bytes = workspace_bytes - sim_ws;
   cudaStream_t S = static_cast<cudaStream_t>(stream);
-  const SimLayout w = similarity_layout(workspace, L, E, N);
+  const SimLayout w = similarity_layout(workspace, L, E, N, !sim_tc_supported(L, E));
   if (!w.tc) {  // the CUDA-core similarity needs every layer's logits at once
     rc = similarity_impl(W_r, X_cal, L, E, d, N, k_freq, sim, counts, workspace, sim_ws, false, S);
     if (!rc)
