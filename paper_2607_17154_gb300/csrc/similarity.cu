@@ -465,7 +465,7 @@ __device__ int place_layers(PlaceSmem& sm, const int32_t* __restrict__ group,
                              const int32_t* __restrict__ porder, int L, int E, int M, int l0,
                              int l1, int first, PlaceParams pp, const double* __restrict__ p,
                              const double* __restrict__ C, uint8_t* __restrict__ placement,
-                             double* __restrict__ used, int32_t* __restrict__ status) {
+                             double* __restrict__ used) {
   int* grp = sm.grp;
   int* ord = sm.ord;
   double* pls = sm.pls;
@@ -599,15 +599,16 @@ __global__ void __launch_bounds__(64) place_kernel(
   __shared__ int s_over;
   int over = 0;
   if (threadIdx.x < 32)
-    over = place_layers(sm, group, porder, L, E, M, l0, l1, first, pp, p, C, placement, used, status);
+    over = place_layers(sm, group, porder, L, E, M, l0, l1, first, pp, p, C, placement, used);
   else if (threadIdx.x == 32 && first)  // beside the placement, on the second warp
     s_over = demand_exceeds(p, L * E, C, M);
   __syncthreads();
   if (threadIdx.x == 0) place_status(first, over | (first ? s_over : 0), status);
 }
 
-// Grouping and placement of layers l0 .. l1 - 1 in one block: 64 threads per
-// layer group kGroupSlices layers at a time, then warp 0 places them (one
+// Grouping and placement of layers l0 .. l1 - 1 in one block: the grouping
+// runs kGroupSlices layers at a time, 64 threads a layer; then warp 0 places
+// the layers in order while the second warp sums the capacity check (one
 // block, so the pipelined plan's side stream holds one SM).
 constexpr int kGroupSlices = 4;
 constexpr size_t kGroupPlaceSmem = kGroupSlices * sizeof(GroupSmem) + sizeof(PlaceSmem);
@@ -632,7 +633,7 @@ __global__ void __launch_bounds__(64 * kGroupSlices) group_place_kernel(
   __shared__ int s_over;
   int over = 0;
   if (threadIdx.x < 32)
-    over = place_layers(ps, group, porder, L, E, M, l0, l1, first, pp, p, C, placement, used, status);
+    over = place_layers(ps, group, porder, L, E, M, l0, l1, first, pp, p, C, placement, used);
   else if (threadIdx.x == 32 && first)
     s_over = demand_exceeds(p, L * E, C, M);
   __syncthreads();
