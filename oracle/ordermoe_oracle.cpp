@@ -459,9 +459,15 @@ int orc_place(const int32_t* group, const double* importance, const double* p, i
     uint8_t* x = placement + (int64_t)l * M * E;
     std::vector<int> order(E);
     for (int e = 0; e < E; ++e) order[e] = e;
+    // p desc, I desc, index asc; a NaN (the importance of NaN similarities)
+    // comes after every number, so the comparison is a strict weak order
+    auto same = [](double x, double y) { return x == y || (std::isnan(x) && std::isnan(y)); };
+    auto above = [](double x, double y) {
+      return std::isnan(y) ? !std::isnan(x) : (!std::isnan(x) && x > y);
+    };
     std::sort(order.begin(), order.end(), [&](int a, int c) {
-      if (pl[a] != pl[c]) return pl[a] > pl[c];
-      if (I[a] != I[c]) return I[a] > I[c];
+      if (!same(pl[a], pl[c])) return above(pl[a], pl[c]);
+      if (!same(I[a], I[c])) return above(I[a], I[c]);
       return a < c;
     });
     std::vector<int> waiting;

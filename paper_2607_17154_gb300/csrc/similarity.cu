@@ -289,8 +289,19 @@ struct PlaceParams {
   double alpha_f, alpha_r, lambda1, lambda2;
 };
 
+// Integer key of an fp64 value for a descending order with NaN after every
+// number: larger values get larger keys (the bits, sign-flipped for
+// negatives, with -0 taken as +0), and every NaN gets 0, below them all.
+__device__ __forceinline__ unsigned long long rank_key(double x) {
+  if (x != x) return 0ull;
+  unsigned long long b = static_cast<unsigned long long>(__double_as_longlong(x == 0.0 ? 0.0 : x));
+  return (b >> 63) ? ~b : (b | 0x8000000000000000ull);
+}
+
 // One layer's scratch of the grouping.
 struct GroupSmem {
+  unsigned long long kp[64];  // rank_key of p and of I, for the placement order
+  unsigned long long ki[64];
   double imp[64];
   double pls[64];
   int order[64];
@@ -344,6 +355,11 @@ __device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float*
   __syncthreads();
   // Eqs. 24-26 in the visiting order; warp 0 scans the existing dominants in
   // parallel (lane g takes dominants g and g + 32; ties to the earlier one).
+  // The choice is the scan's in dominant order: the first dominant unless a
+  // later one is strictly more similar. With NaN similarities that is the
+  // first dominant when its similarity is NaN, else the first maximum with
+  // NaN counted as -inf: a total order, so every lane of the reduction ends
+  // with the same group.
   if (live && t < 32) {
     int k = 0;
     for (int pos = 0; pos < E; ++pos) {
@@ -352,7 +368,8 @@ __device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float*
       int bg = 1 << 30;
       for (int g = t; g < k; g += 32) {
         const float sv = S[j * E + dom[g]];
-        if (bg == (1 << 30) || sv > bs) { bg = g; bs = sv; }
+        const float v = sv != sv ? -INFINITY : sv;
+        if (bg == (1 << 30) || v > bs) { bg = g; bs = v; }
       }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
@@ -361,6 +378,13 @@ __device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float*
         if (og != (1 << 30) && (bg == (1 << 30) || os > bs || (os == bs && og < bg))) {
           bs = os;
           bg = og;
+        }
+      }
+      if (k > 0) {
+        const float s0 = S[j * E + dom[0]];
+        if (s0 != s0) {  // NaN first: the scan keeps dominant 0 (and NaN < theta is false)
+          bg = 0;
+          bs = s0;
         }
       }
       if (bg == (1 << 30) || bs < theta) {
@@ -393,15 +417,20 @@ __device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float*
     if (importance != nullptr) importance[(size_t)l * E + t] = imp[t];
   }
   __syncthreads();
-  // placement order: p desc, I desc, index asc
+  // placement order: p desc, I desc, index asc, with NaN after every number
+  // (a total order, so the ranks are a permutation whatever the values),
+  // compared on integer keys
   if (live && t < E) {
+    sm.kp[t] = rank_key(pls[t]);
+    sm.ki[t] = rank_key(imp[t]);
+  }
+  __syncthreads();
+  if (live && t < E) {
+    const unsigned long long kpt = sm.kp[t], kit = sm.ki[t];
     int r = 0;
     for (int e = 0; e < E; ++e) {
-      bool before;
-      if (pls[e] != pls[t]) before = pls[e] > pls[t];
-      else if (imp[e] != imp[t]) before = imp[e] > imp[t];
-      else before = e < t;
-      if (before) ++r;
+      const unsigned long long kpe = sm.kp[e], kie = sm.ki[e];
+      r += (kpe > kpt || (kpe == kpt && (kie > kit || (kie == kit && e < t)))) ? 1 : 0;
     }
     porder[(size_t)l * E + r] = t;
   }

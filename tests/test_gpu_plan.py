@@ -190,6 +190,44 @@ def test_place_ties_waiting_lists_and_server_counts(L, E, M, scale, frac):
     assert (got[3].sum(axis=1) == 1).all()  # every expert on exactly one server
 
 
+def test_place_with_nan_similarities_matches_oracle():
+    """NaN similarities (bad inputs) give the oracle's groups, importances
+    (NaN where a group mean meets one), placement order and placement: the
+    grouping follows the scan's rule, and NaN importances go after every
+    number."""
+    rng = np.random.default_rng(31)
+    L, E, M = 6, 16, 4
+    sim, counts = synthetic_sims(rng, L, E, 4, 0.4)
+    for l in range(L):
+        for _ in range(3):  # symmetric NaN pairs off the diagonal
+            i, j = rng.choice(E, 2, replace=False)
+            sim[l, i, j] = sim[l, j, i] = np.nan
+    # a NaN to the first dominant (the expert with the most activations)
+    first = int(np.argmax(counts[0])); other = (first + 1) % E
+    sim[0, first, other] = sim[0, other, first] = np.nan
+    p = np.ones((L, E)); C = np.full(M, L * E / M * 1.2)
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a)).to(device=DEV, dtype=dt)
+    group = torch.empty(L, E, dtype=torch.int32, device=DEV)
+    ng = torch.empty(L, dtype=torch.int32, device=DEV)
+    theta = torch.empty(L, dtype=torch.float32, device=DEV)
+    imp = torch.empty(L, E, dtype=torch.float64, device=DEV)
+    x = torch.empty(L, M, E, dtype=torch.uint8, device=DEV)
+    used = torch.empty(M, dtype=torch.float64, device=DEV)
+    st = torch.empty(1, dtype=torch.int32, device=DEV)
+    B.ordermoe_place(t(sim, torch.float32), t(counts, torch.int32), L, E, M, 0.5, 0.9, 0.5, 0.5, 0.5,
+                     0.5, 0.5, t(p, torch.float64), t(C, torch.float64), group, ng, theta, imp, x, used, st)
+    torch.cuda.synchronize()
+    ref = oracle_place_all(sim, counts, M, p, C)
+    got = (group.cpu().numpy(), ng.cpu().numpy(), theta.cpu().numpy(), x.cpu().numpy(),
+           used.cpu().numpy(), int(st.item()))
+    for name, a, b in zip(("group", "n_groups", "theta", "placement", "used", "status"), got, ref):
+        np.testing.assert_array_equal(a, b, err_msg=name)
+    ref_imp = np.stack([oracle.importance(sim[l], counts[l], ref[0][l]) for l in range(L)])
+    np.testing.assert_array_equal(imp.cpu().numpy(), ref_imp)
+    assert np.isnan(ref_imp).any()
+    assert (got[3].sum(axis=1) == 1).all()
+
+
 def test_placement_quotient_is_correctly_rounded():
     """The placement's load ratio b_m / C_m (reciprocal + Markstein's correction)
     equals IEEE division (numpy) bit for bit on random and edge operands."""

@@ -76,8 +76,8 @@ MUTANTS = [
     ("Eq. 6: threshold runs the wrong way over the layers",
      "double frac = static_cast<double>(N - l) / static_cast<double>(N - 1);",
      "double frac = static_cast<double>(l - 1) / static_cast<double>(N - 1);"),
-    ("placement order: importance ascending", "if (I[a] != I[c]) return I[a] > I[c];",
-     "if (I[a] != I[c]) return I[a] < I[c];"),
+    ("placement order: importance ascending", "if (!same(I[a], I[c])) return above(I[a], I[c]);",
+     "if (!same(I[a], I[c])) return above(I[c], I[a]);"),
     ("waiting list to the fullest server", "if (C[m] - b[m] > C[best] - b[best]) best = m;",
      "if (C[m] - b[m] < C[best] - b[best]) best = m;"),
     ("Eq. 34: ties to the later layer", "if (bl < 0 || benefit > bb) { bl = l; bm = m; bj = j; bb = benefit; }",

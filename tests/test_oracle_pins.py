@@ -1165,3 +1165,39 @@ def test_lookahead_moves_the_token_where_the_next_layer_is_cheap(orc):
     la = orc.select_lookahead(idx, [t0, t1], P, home, home.copy(), np.zeros(1, np.float32))
     assert la[0][0, 0] == 0 and la[1][0, 0] == 1            # remote exact
     assert la[3][0] == 1                                     # the token moved (Eq. 44)
+
+
+def test_group_and_place_with_nan_similarities(orc):
+    """NaN similarities (bad inputs) follow the scan's own rule: an expert joins
+    the first dominant when its similarity to it is NaN (NaN < theta is
+    false, and nothing strictly exceeds NaN), and otherwise a NaN never wins.
+    The importance of such experts is NaN; the placement order puts NaN after
+    every number (a total order), so the placement stays a permutation."""
+    # counts order: 0, 1, 2, 3; dominant 0 first
+    sim = np.array([[1, .9, .2, np.nan],
+                    [.9, 1, .1, .3],
+                    [.2, .1, 1, .8],
+                    [np.nan, .3, .8, 1]], np.float32)
+    cnt = np.array([9, 7, 5, 3], np.int32)
+    g, K, dom = orc.group(sim, cnt, 0.5)
+    # 0 -> group 0; 1 joins 0 (.9); 2: .2 < .5 -> group 1 (dominant 2);
+    # 3: NaN to dominant 0 first -> joins group 0 although .8 to dominant 2 is larger
+    assert K == 2 and list(dom[:2]) == [0, 2] and list(g) == [0, 0, 1, 0]
+    sim2 = sim.copy(); sim2[3, 0] = sim2[0, 3] = 0.1; sim2[3, 2] = sim2[2, 3] = np.nan
+    g2, K2, _ = orc.group(sim2, cnt, 0.5)
+    # 3: .1 to dominant 0, NaN to dominant 2 (never wins) -> best .1 < .5 -> new group 2
+    assert K2 == 3 and list(g2) == [0, 0, 1, 2]
+    imp = orc.importance(sim, cnt, g)
+    # rho of 0 and 3 averages the NaN pair Sim(0,3); expert 1's group mean does not include it
+    assert np.isnan(imp[[0, 3]]).all() and np.isfinite(imp[[1, 2]]).all()
+    assert imp[2] == pytest.approx(0.5 * 5 / 24 + 0.5) and imp[1] == pytest.approx(0.5 * 7 / 24 + 0.5 * 2.2 / 3)
+    # placement order: 2 (I .604), 1 (.5125), then the NaN importances 0, 3 by index.
+    # 2 -> server 0 (both empty, ties to the lower m); 1 -> server 1 (0.25 against 0);
+    # 0 (group 0) -> server 0 (0.25 + 0 against 0.25 + 0.5 for expert 1's group on 1);
+    # 3 -> server 1 (server 0 is full)
+    L, E, M = 1, 4, 2
+    x, used, rc = orc.place(g[None], imp[None], np.ones((1, E)), np.full(M, 2.0))
+    assert rc == 0 and list(used) == [2.0, 2.0]
+    assert x[0].tolist() == [[1, 0, 1, 0], [0, 1, 0, 1]]
+    x2, _, _ = orc.place(g[None], imp[None], np.ones((1, E)), np.full(M, 2.0))
+    assert (x2 == x).all()                                          # deterministic
