@@ -372,7 +372,8 @@ int ordermoe_expert_counts(const float* logits, int64_t N, int E, int k_freq, in
  *   placement (Eqs. 29-31): experts by (p desc, I desc, index asc), feasible
  *            servers b_m + p <= C_m, score lambda1 b_m / C_m + lambda2 eta
  *            (lambda1, lambda2 >= 0, p >= 0 and C_m > 0 finite; a negative
- *            or NaN score or a bad C_m sets ORDERMOE_DEV_BAD_VALUE),
+ *            or NaN p (detail = l * E + j), a negative or NaN score or a bad
+ *            C_m sets ORDERMOE_DEV_BAD_VALUE),
  *            lowest score (ties: lower m); experts with no feasible server go,
  *            after the layer, to the server with the most free memory. The
  *            used memory b_m accumulates over the layers.

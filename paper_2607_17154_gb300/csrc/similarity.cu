@@ -333,6 +333,7 @@ __device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float*
     if (t < E) {
       cnt[t] = counts[(size_t)l * E + t];
       pls[t] = p[(size_t)l * E + t];
+      if (!(pls[t] >= 0.0)) report(&g_err_sim, ORDERMOE_DEV_BAD_VALUE, l * E + t);  // Eq. 29's p
     }
   }
   __syncthreads();

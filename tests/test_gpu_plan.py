@@ -228,6 +228,21 @@ def test_place_with_nan_similarities_matches_oracle():
     assert (got[3].sum(axis=1) == 1).all()
 
 
+def test_place_reports_a_bad_memory_demand():
+    """A negative or NaN memory demand p is reported (ORDERMOE_DEV_BAD_VALUE,
+    detail = l * E + j) and the call still completes."""
+    rng = np.random.default_rng(41)
+    L, E, M = 3, 8, 2
+    sim, counts = synthetic_sims(rng, L, E, 2, 0.4)
+    for bad, where in ((np.nan, (1, 5)), (-1.0, (2, 0))):
+        p = np.ones((L, E)); p[where] = bad
+        gpu_place(sim, counts, M, p, np.full(M, L * E))
+        code, detail = B.ordermoe_device_error()
+        assert code == B.DEV_BAD_VALUE and detail == where[0] * E + where[1], (bad, code, detail)
+    gpu_place(sim, counts, M, np.ones((L, E)), np.full(M, L * E))
+    assert B.ordermoe_device_error()[0] == 0
+
+
 def test_placement_quotient_is_correctly_rounded():
     """The placement's load ratio b_m / C_m (reciprocal + Markstein's correction)
     equals IEEE division (numpy) bit for bit on random and edge operands."""
