@@ -644,12 +644,14 @@ def _same(a, b, what):
 @pytest.mark.parametrize("L,E,N,M,kf,unequal", [(24, 64, 4096, 8, 6, False), (13, 64, 3000, 4, 6, True),
                                                  (1, 64, 1000, 3, 2, False), (20, 32, 2100, 5, 4, True),
                                                  (40, 16, 1500, 16, 3, False), (80, 8, 1200, 6, 2, True),
-                                                 (3, 12, 900, 3, 3, False)])
+                                                 (3, 12, 900, 3, 3, False), (64, 64, 700, 8, 6, True),
+                                                 (65, 64, 700, 8, 6, False)])
 def test_plan_equals_the_four_calls(L, E, N, M, kf, unequal):
     """ordermoe_plan (blocks of 512 logit columns; grouping and placement of a
     block on a side stream while the next block's GEMM runs) writes what the
     four calls write one after the other, bit for bit: ragged last blocks,
-    b_m carried across blocks, E = 12 on the one-stream path."""
+    b_m carried across blocks, the tensor-core limit L E = 4096 (8 blocks),
+    and the one-stream path for E = 12 and for L E = 4160."""
     d = 128
     Wr, Xcal, p, C, pi = _plan_inputs(L, E, d, N, M, L * 7 + E, unequal)
     ref = _serial_plan(Wr, Xcal, L, E, d, N, kf, M, p, C, pi)
