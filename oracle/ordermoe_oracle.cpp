@@ -13,7 +13,7 @@
 // on both sides from identical fp32 tables). Build with -ffp-contract=off so
 // that no multiply-add is fused.
 //
-// Readings where the paper is silent or garbled (listed again in the design doc):
+// Readings where the paper is silent or garbled:
 //  * top-k > 1: the selection of Alg. 2 runs once per routed slot, in rank
 //    order; a substitute may not be an expert the token already routes to or
 //    has already been given (every token keeps k distinct experts).
