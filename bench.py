@@ -29,7 +29,7 @@ UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM bytes (read + write) per launch of the gate/up GEMM at the mixtral_prefill workload, from
-# the ncu capture summarised in profiles/ffn_gemm_pair_gate_up_mixtral_prefill.md, valid only while the
+# the recorded ncu capture of that kernel, valid only while the
 # kernel sources hash to the values recorded with it.
 GATE_UP_TRAFFIC = {
     "bytes": 1958962176 + 228495104,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
@@ -56,8 +56,7 @@ def gate_up_kernel_name(R, E, dff):
     """The gate/up kernel the library picks for R permuted rows (grouped_gemm.cu)."""
     if R < 256 * E:
         return "ffn_gemm_kernel<gate_up> (tcgen05, one CTA, 128-row tiles)"
-    cl = 4 if (dff // 128) % 2 == 0 else 2
-    return "ffn_gemm_pair_kernel<gate_up, %d> (tcgen05 CTA pairs, clusters of %d)" % (cl, cl)
+    return "ffn_gemm_pair_kernel<gate_up> (tcgen05 CTA pairs)"
 
 
 def parse():
@@ -96,6 +95,39 @@ def peaks():
             d = json.load(f)
         return d, "measured"
     return dict(FALLBACK_PEAKS), "fallback"
+
+
+BURST_REGION_S = 1.0
+
+
+def tensor_peak(pk, pk_kind, clocks, region_s):
+    """The bf16 peak that applies to a kernel timed inside a region of
+    region_s seconds: the burst figure (best single cuBLAS GEMM) when the
+    region is short (under BURST_REGION_S) and no power cap was active while
+    it ran, else the sustained figure (cuBLAS back to back for seconds under
+    the power cap). Returns (peak, which, why, burst, sustained)."""
+    burst = float(pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
+    sustained = float(pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
+    capped = "sw_power_cap" in (clocks or {}).get("reasons", [])
+    if region_s < BURST_REGION_S and not capped:
+        why = "timed region %.3f s < %.1f s, no power cap seen" % (region_s, BURST_REGION_S)
+        return burst, "burst", why, burst, sustained
+    why = ("sw_power_cap active during the timed region" if capped else
+           "timed region %.3f s >= %.1f s" % (region_s, BURST_REGION_S))
+    return sustained, "sustained", why, burst, sustained
+
+
+def tensor_roofline(kernel, achieved, pk, pk_kind, clocks, region_s, **extra):
+    """Roofline object of a tensor-bound kernel, its fraction of both measured
+    bf16 peaks, and which one applies."""
+    peak, which, why, burst, sustained = tensor_peak(pk, pk_kind, clocks, region_s)
+    out = {"kernel": kernel, "bound": "tensor", "achieved": round(achieved, 1), "peak": peak,
+           "unit": "TFLOP/s", "frac": round(achieved / peak, 4),
+           "frac_burst": round(achieved / burst, 4), "frac_sustained": round(achieved / sustained, 4),
+           "peak_applies": which, "peak_reason": why,
+           "peak_source": "%s bf16_tflops%s" % (pk_kind, "" if which == "burst" else "_sustained")}
+    out.update(extra)
+    return out
 
 
 # ----------------------------------------------------------------- clocks
@@ -351,7 +383,6 @@ def run_ours(args, dist):
     pk, pk_kind = peaks()
     gu_flop = 2.0 * R * d * 2 * dff
     achieved = gu_flop / (gu_ms / 1e3) / 1e12
-    peak = float(pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"]))
     layer_flop = 2.0 * R * 3 * d * dff + 2.0 * T * d * E
     out = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": dist.world,
@@ -363,12 +394,12 @@ def run_ours(args, dist):
                    "home": w.home, "seed": args.seed, "parallelism": "replicas",
                    "l2": "inputs larger than L2: %.2f GB of expert weights read every step"
                          % (3 * E * d * dff * 2 / 1e9)},
-        "roofline": {"kernel": gate_up_kernel_name(T * k, E, dff), "bound": "tensor",
-                     "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
-                     "frac": round(achieved / peak, 4), "traffic": gate_up_traffic(w.name),
-                     "peak_source": "%s bf16_tflops_sustained" % pk_kind,
-                     "flop_per_launch": gu_flop, "ms_per_launch": round(gu_ms, 4),
-                     "layer_tflops": round(layer_flop / (elapsed_ms / args.steps / 1e3) / 1e12, 1)},
+        "roofline": tensor_roofline(
+            gate_up_kernel_name(T * k, E, dff), achieved, pk, pk_kind, clocks, elapsed_ms / 1e3,
+            traffic=gate_up_traffic(w.name), flop_per_launch=gu_flop, ms_per_launch=round(gu_ms, 4),
+            layer_tflops=round(layer_flop / (elapsed_ms / args.steps / 1e3) / 1e12, 1),
+            layer_frac=round(layer_flop / (elapsed_ms / args.steps / 1e3) / 1e12
+                             / tensor_peak(pk, pk_kind, clocks, elapsed_ms / 1e3)[0], 4)),
         "e2e": e2e,
         "gpu_launches": KERNELS_PER_STEP * args.steps,
         "breakdown_ms": breakdown,
@@ -715,7 +746,6 @@ def run_similarity(args, dist, w, device):
     step_s = ms / args.steps / 1e3
     flop = 2.0 * N * L * E * d + 2.0 * L * N * E * E
     pk, pk_kind = peaks()
-    peak = float(pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"]))
     achieved = flop / step_s / 1e12
     return {
         "metric": "calibration tokens/s through the offline similarity + grouping + placement",
@@ -725,11 +755,10 @@ def run_similarity(args, dist, w, device):
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": L, "E": E, "d": d, "N": N, "groups": w.n_clusters,
                    "M": w.M, "k_freq": w.k, "memory_ratio": ratio},
-        "roofline": {"kernel": "ordermoe_plan: similarity (tcgen05 logits + Gram) + group + place + replicate + coverage (whole plan)",
-                     "bound": "tensor",
-                     "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
-                     "frac": round(achieved / peak, 4), "traffic": None,
-                     "peak_source": "%s bf16_tflops (burst)" % pk_kind, "flop_per_step": flop},
+        "roofline": tensor_roofline(
+            "ordermoe_plan: similarity (tcgen05 logits + Gram) + group + place + replicate + "
+            "coverage (whole plan)", achieved, pk, pk_kind, clocks, ms / 1e3, traffic=None,
+            flop_per_step=flop),
         "gpu_launches": plan_launches(L, E) * args.steps,
         "n_groups": ng.cpu().tolist()[:3], "place_status": int(st.item()),
         "replicas": int(reps.sum().item()),

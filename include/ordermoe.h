@@ -206,7 +206,9 @@ int ordermoe_dispatch(const int32_t* chosen_expert, const uint16_t* X, int T, in
  * library until the process exits, so T*k is limited to 262144 entries
  * (larger calls fail with ORDERMOE_ERR_UNSUPPORTED_SHAPE). The array's device
  * address is looked up on the first call made on each device: make that
- * first call before any stream capture. All calls share the array, so calls
+ * first call before any stream capture. The address is kept until the
+ * process exits; after cudaDeviceReset of a device it is stale, so do not
+ * call this entry point on a device the process has reset. All calls share the array, so calls
  * that overlap on the GPU (other streams, other host threads) race; nothing
  * in it needs clearing between calls. The call allocates nothing. */
 int ordermoe_dispatch_noalloc(const int32_t* chosen_expert, const uint16_t* X, int T, int k,

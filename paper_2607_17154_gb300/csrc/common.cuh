@@ -26,6 +26,16 @@ int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// The token permutation (ordermoe_dispatch) cuts its n = T*k (token, slot)
+// entries into chunks of kDispatchChunk and keeps one int32 histogram entry
+// per (chunk, expert) in its scratch; both entry points that run it size
+// their scratch from this one definition.
+constexpr int kDispatchChunk = 256;
+constexpr int64_t dispatch_hist_entries(int64_t n, int E) {
+  return ((n + kDispatchChunk - 1) / kDispatchChunk > 0 ? (n + kDispatchChunk - 1) / kDispatchChunk
+                                                        : 1) * E;
+}
+
 // An NVTX range over one C-ABI call, named after it: visible to the Nsight
 // tools, a no-op when none is attached.
 struct TraceRange {

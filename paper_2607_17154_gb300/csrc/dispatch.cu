@@ -28,7 +28,7 @@ int read_clear_err_dispatch(unsigned long long* out) {
   return ORDERMOE_OK;
 }
 
-constexpr int kChunk = 256;
+constexpr int kChunk = kDispatchChunk;
 
 __global__ void __launch_bounds__(kChunk) chunk_hist_kernel(const int32_t* __restrict__ chosen,
                                                             int64_t n, int E,
@@ -313,8 +313,7 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(
 }
 
 size_t dispatch_workspace_bytes(int64_t n, int E) {
-  const int64_t nchunks = (n + kChunk - 1) / kChunk;
-  return (size_t)((nchunks > 0 ? nchunks : 1) * E * sizeof(int32_t) + 255) & ~size_t(255);
+  return (size_t)(dispatch_hist_entries(n, E) * sizeof(int32_t) + 255) & ~size_t(255);
 }
 
 int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int E, int d,

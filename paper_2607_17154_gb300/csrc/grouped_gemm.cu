@@ -374,16 +374,11 @@ __global__ void __launch_bounds__(THREADS, 1)
 // The accumulator is transposed (lane = output column, TMEM column = row);
 // the epilogue writes it row-major through a shared-memory tile with 16-byte
 // coalesced stores, skipping rows beyond the expert's range.
-// Clusters of 4 CTAs (two pairs) halve the L2 reads of the permuted rows: the
-// two pairs take neighbouring column slices of the same row tile, and each
-// CTA loads half of its 128-row box of rows and multicasts it to the CTA of
-// the same rank in the other pair (TMA reads from L2 per CTA and K step drop
-// from 32 KB to 24 KB); used when the slice count is even. A stage then holds
-// data from both pairs, so each pair's MMA commit releases it in all four CTAs.
+// Each cluster is one CTA pair, and each CTA loads its own operand boxes from
+// this GPU's memory (no multicast loads).
 // Barriers: full[s] (even CTA, one arrive with the pair's bytes; both CTAs'
-// TMA loads, and the other pair's multicast, complete on it), empty[s] and tfull[b] (both CTAs, arrived by the
-// even CTA's MMA commits multicast to the pair, or to all four CTAs for
-// empty[s] in a cluster of 4), tempty[b] (even CTA, one
+// TMA loads complete on it), empty[s] and tfull[b] (both CTAs, arrived by the
+// even CTA's MMA commits signalled to the pair), tempty[b] (even CTA, one
 // arrive per epilogue warp of either CTA). The gate/up epilogue runs on two
 // groups of four warps that take alternate 32-row chunks, so two chunks are
 // in flight (short-K tiles are otherwise epilogue-bound); down runs one group.
@@ -443,19 +438,6 @@ __device__ __forceinline__ Tile decode_pair(int tile, const PSmem& s, int E, int
   return t;
 }
 
-// Multicast TMA load of a CTA pair: the box lands at the same offset in every
-// CTA of cta_mask, and its bytes complete on the mbarrier at bar's offset in
-// the even CTA of each destination's pair (bar is an even CTA's barrier).
-__device__ __forceinline__ void tma_load_2d_pair_mc(void* smem_dst, const CUtensorMap* map,
-                                                    uint32_t bar_cluster_addr, int c0, int c1,
-                                                    uint16_t cta_mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      ".multicast::cluster.cta_group::2 [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster_addr), "r"(c0), "r"(c1), "h"(cta_mask)
-      : "memory");
-}
-
 // rows of the tile rounded up to the MMA's N granularity (16)
 __device__ __forceinline__ int tile_n(const Tile& t) {
   const int rows = min(P_BM, t.m_end - t.m0);
@@ -481,8 +463,8 @@ __device__ __forceinline__ bool epi_all(bool p) {
   return r != 0;
 }
 
-// CL = CTAs per cluster (2: one pair; 4: two pairs sharing the row tile).
-template <int MODE, int CL>
+// One cluster = one CTA pair.
+template <int MODE>
 __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
     ffn_gemm_pair_kernel(const __grid_constant__ CUtensorMap mapW0,
                          const __grid_constant__ CUtensorMap mapW1,
@@ -498,17 +480,15 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
   const int lane = tid & 31;
   const uint32_t rank = cluster_ctarank();
   const uint32_t rp = rank & 1u;     // rank within the pair
-  const uint32_t pr = rank >> 1;     // pair within the cluster (0 when CL == 2)
-  const uint32_t lead = rank & ~1u;  // the pair's even CTA (MMA issuer)
+  const uint32_t lead = 0;           // the pair's even CTA (MMA issuer)
   const bool even = (rp == 0);
-  const int cluster = blockIdx.x / CL;
-  const int n_clusters = gridDim.x / CL;
-  const int n_q = CL == 4 ? args.n_tiles / 2 : args.n_tiles;  // slice units per cluster tile
+  const int cluster = blockIdx.x / 2;
+  const int n_clusters = gridDim.x / 2;
 
   if (tid == 0) {
     for (int i = 0; i < P_STAGES; ++i) {
       mbar_init(&s.full[i], 1);
-      mbar_init(&s.empty[i], CL / 2);  // one MMA commit per pair
+      mbar_init(&s.empty[i], 1);  // one MMA commit of the pair
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s.tfull[i], 1);
@@ -549,17 +529,13 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
   cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
   tc_fence_after();
   const uint32_t tmem_base = s.tmem_base;
-  const int total = s.mt_start[args.E] * n_q;
+  const int total = s.mt_start[args.E] * args.n_tiles;
   const int kblocks = args.K / BK;
   volatile int* abort = &s.abort;
   uint32_t issued_mask = 0, last_phase_bits = 0;
   bool mma_issued = false;
-  // tile -> (expert, this pair's column slice, row range)
-  auto tile_of = [&](int tile) {
-    Tile t = decode_pair(tile, s, args.E, n_q);
-    if (CL == 4) t.n = 2 * t.n + static_cast<int>(pr);
-    return t;
-  };
+  // tile -> (expert, column slice, row range)
+  auto tile_of = [&](int tile) { return decode_pair(tile, s, args.E, args.n_tiles); };
 
   if (warp == 0) {
     if (lane == 0) {
@@ -587,12 +563,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
           } else {
             tma_load_2d_pair(sw, &mapW0, full_even, kb * BK, wrow);
           }
-          if (CL == 4)  // rows 64 pr .. 64 pr + 63 of the box, to this CTA and its counterpart
-            tma_load_2d_pair_mc(st + pr * (P_T_BYTES / 2), &mapT, full_even, kb * BK,
-                                trow + 64 * static_cast<int>(pr),
-                                static_cast<uint16_t>((1u << rank) | (1u << (rank ^ 2u))));
-          else
-            tma_load_2d_pair(st, &mapT, full_even, kb * BK, trow);
+          tma_load_2d_pair(st, &mapT, full_even, kb * BK, trow);
           issued_mask |= 1u << stage;
           last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
@@ -632,11 +603,11 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
             mma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32),
                           sdesc_kmajor_sw128(b0 + kk * 32), idesc, (kb | kk) != 0 ? 1u : 0u);
           mma_issued = true;
-          mma_commit_pair(&s.empty[stage], CL == 4 ? 0xF : 0x3);
+          mma_commit_pair(&s.empty[stage], 0x3);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        mma_commit_pair(&s.tfull[slot], static_cast<uint16_t>(0x3u << (2 * pr)));
+        mma_commit_pair(&s.tfull[slot], 0x3);
       }
     }
   } else {
@@ -796,9 +767,9 @@ int make_tmap_bf16(CUtensorMap* map, const void* base, uint64_t rows, uint64_t c
   return ORDERMOE_OK;
 }
 
-template <int MODE, int CL>
+template <int MODE>
 static cudaError_t pair_attr() {
-  return cudaFuncSetAttribute(gg::ffn_gemm_pair_kernel<MODE, CL>,
+  return cudaFuncSetAttribute(gg::ffn_gemm_pair_kernel<MODE>,
                               cudaFuncAttributeMaxDynamicSharedMemorySize,
                               gg::PCfg<MODE>::SMEM_BYTES);
 }
@@ -807,10 +778,8 @@ static int ffn_attrs() {
   using namespace gg;
   static PerDevice cache;
   const cudaError_t attr_err = static_cast<cudaError_t>(per_device(cache, [] {
-    cudaError_t e = pair_attr<GATEUP, 2>();
-    if (e == cudaSuccess) e = pair_attr<DOWN, 2>();
-    if (e == cudaSuccess) e = pair_attr<GATEUP, 4>();
-    if (e == cudaSuccess) e = pair_attr<DOWN, 4>();
+    cudaError_t e = pair_attr<GATEUP>();
+    if (e == cudaSuccess) e = pair_attr<DOWN>();
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(ffn_gemm_kernel<GATEUP>,
                                cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
@@ -840,43 +809,41 @@ static cudaLaunchConfig_t pair_config(int grid, int cl, cudaStream_t stream,
   return cfg;
 }
 
-// Clusters of `cl` CTAs that can be resident at once (not every SM finds
-// partners in its GPC: on GB300, 76 clusters of 2 and 36 of 4); the persistent
-// grid never exceeds it, so no cluster waits for another. 0: none fit.
-template <int MODE, int CL>
+// CTA pairs that can be resident at once (not every SM finds a partner in its
+// GPC: 76 pairs on GB300); the persistent grid never exceeds it, so no
+// cluster waits for another.
+template <int MODE>
 static int max_resident_clusters() {
   static PerDevice cache;
   return per_device(cache, [] {
     cudaLaunchAttribute attr;
-    cudaLaunchConfig_t cfg = pair_config<MODE>(CL * (num_sms() / CL), CL, nullptr, &attr);
+    cudaLaunchConfig_t cfg = pair_config<MODE>(2 * (num_sms() / 2), 2, nullptr, &attr);
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gg::ffn_gemm_pair_kernel<MODE, CL>, &cfg) !=
-            cudaSuccess ||
-        n < 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, gg::ffn_gemm_pair_kernel<MODE>, &cfg) != cudaSuccess ||
+        n <= 0) {
       cudaGetLastError();
-      n = CL == 2 ? num_sms() / 2 : 0;
+      n = num_sms() / 2;
     }
-    return n < num_sms() / CL ? n : num_sms() / CL;
+    return n < num_sms() / 2 ? n : num_sms() / 2;
   });
 }
 
-// One launch of the CTA-pair kernel over `tiles` cluster tiles.
-template <int MODE, int CL>
+// One launch of the CTA-pair kernel over `tiles` pair tiles.
+template <int MODE>
 static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const CUtensorMap& t,
                        const gg::Args& a, long long tiles, cudaStream_t stream, const char* what) {
-  const long long cmax = max_resident_clusters<MODE, CL>();
+  const long long cmax = max_resident_clusters<MODE>();
   const long long clusters = tiles < cmax ? tiles : cmax;
   cudaLaunchAttribute attr;
   cudaLaunchConfig_t cfg =
-      pair_config<MODE>(static_cast<int>(CL * (clusters > 0 ? clusters : 1)), CL, stream, &attr);
-  const cudaError_t e = cudaLaunchKernelEx(&cfg, gg::ffn_gemm_pair_kernel<MODE, CL>, w0, w1, t, a);
+      pair_config<MODE>(static_cast<int>(2 * (clusters > 0 ? clusters : 1)), 2, stream, &attr);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, gg::ffn_gemm_pair_kernel<MODE>, w0, w1, t, a);
   if (e != cudaSuccess) return cuda_fail(e, what);
   OM_LAUNCHED(what);
   return ORDERMOE_OK;
 }
 
-// Tile shape: CTA pairs (256 weight rows x up to 256 permuted rows, in
-// clusters of 2 or 4) when experts average at least 256 rows; otherwise single
+// Tile shape: CTA pairs (256 weight rows x up to 256 permuted rows) when experts average at least 256 rows; otherwise single
 // CTAs with 128-row tiles and the rows on the M side (a decode step: ~32 rows
 // per expert, where the weights are streamed once and the MMA shape hardly
 // matters).
@@ -903,13 +870,8 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
     if ((rc = make_tmap_bf16(&mW1, W1, (uint64_t)E * dff, d, 64))) return rc;
     if ((rc = make_tmap_bf16(&mW3, W3, (uint64_t)E * dff, d, 64))) return rc;
     const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
-    if (a.n_tiles % 2 == 0 && max_resident_clusters<GATEUP, 4>() > 0) {
-      if ((rc = make_tmap_bf16(&mX, X_perm, R, d, 64))) return rc;  // half boxes, multicast
-      return launch_pair<GATEUP, 4>(mW1, mW3, mX, a, row_tiles * (a.n_tiles / 2), stream,
-                                    "ffn_gemm_pair_kernel<gate_up, 4>");
-    }
-    return launch_pair<GATEUP, 2>(mW1, mW3, mX, a, row_tiles * a.n_tiles, stream,
-                                  "ffn_gemm_pair_kernel<gate_up, 2>");
+    return launch_pair<GATEUP>(mW1, mW3, mX, a, row_tiles * a.n_tiles, stream,
+                               "ffn_gemm_pair_kernel<gate_up>");
   } else {
     if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
     if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
@@ -934,14 +896,8 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   if ((rc = make_map(&mH, H, R, dff))) return rc;
   if (use_pairs(R, E)) {
     const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
-    if (a.n_tiles % 2 == 0 && max_resident_clusters<DOWN, 4>() > 0) {
-      CUtensorMap mHh;
-      if ((rc = make_tmap_bf16(&mHh, H, R, dff, 64))) return rc;  // half boxes, multicast
-      return launch_pair<DOWN, 4>(mW2, mW2, mHh, a, row_tiles * (a.n_tiles / 2), stream,
-                                  "ffn_gemm_pair_kernel<down, 4>");
-    }
-    return launch_pair<DOWN, 2>(mW2, mW2, mH, a, row_tiles * a.n_tiles, stream,
-                                "ffn_gemm_pair_kernel<down, 2>");
+    return launch_pair<DOWN>(mW2, mW2, mH, a, row_tiles * a.n_tiles, stream,
+                             "ffn_gemm_pair_kernel<down>");
   } else {
     const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
     ffn_gemm_kernel<DOWN><<<single_grid(tiles), THREADS, SMEM_BYTES, stream>>>(mH, mW2, mW2, a);

@@ -13,10 +13,13 @@
 // process keeps the library loaded (64 x 1024 int32 = 256 KB per device).
 // Its device address is looked up once per device, with that device current,
 // on the first call made on the device; make that first call before any
-// stream capture. All calls share the one array: two calls whose kernels
-// overlap on the GPU (different streams, or different host threads on the
-// same device) race on it. Nothing in it needs clearing: every histogram
-// entry a call reads was written earlier in the same call.
+// stream capture. The address is kept for the life of the process: after a
+// cudaDeviceReset of a device it is stale, so a process that resets a device
+// must not call this entry point on that device again. All calls share the
+// one array: two calls whose kernels overlap on the GPU (different streams,
+// or different host threads on the same device) race on it. Nothing in it
+// needs clearing: every histogram entry a call reads was written earlier in
+// the same call.
 #include <mutex>
 
 #include "common.cuh"
@@ -27,11 +30,16 @@ int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int 
                     int32_t* offsets, int32_t* row_token, int32_t* row_of, uint16_t* X_perm,
                     int32_t* hist, cudaStream_t stream);
 
-constexpr int kNoAllocChunk = 256;       // entries per histogram chunk (as ordermoe_dispatch)
-constexpr int kNoAllocMaxChunks = 1024;  // => at most 262144 (token, slot) entries per call
-constexpr int kNoAllocMaxEntries = kNoAllocChunk * kNoAllocMaxChunks;
+size_t dispatch_workspace_bytes(int64_t n, int E);
 
-static __device__ __align__(256) int32_t g_noalloc_hist[kNoAllocMaxChunks * ORDERMOE_MAX_EXPERTS];
+constexpr int kNoAllocMaxChunks = 1024;  // => at most 262144 (token, slot) entries per call
+constexpr int kNoAllocMaxEntries = kDispatchChunk * kNoAllocMaxChunks;
+constexpr int64_t kNoAllocHistEntries = kNoAllocMaxChunks * ORDERMOE_MAX_EXPERTS;
+// the histogram of the largest call allowed fits the array
+static_assert(dispatch_hist_entries(kNoAllocMaxEntries, ORDERMOE_MAX_EXPERTS) <= kNoAllocHistEntries,
+              "fixed scratch smaller than the permutation's histogram at the size limit");
+
+static __device__ __align__(256) int32_t g_noalloc_hist[kNoAllocHistEntries];
 
 constexpr int kMaxDevices = 64;
 static std::mutex g_noalloc_mu;
@@ -79,6 +87,11 @@ extern "C" int ordermoe_dispatch_noalloc(const int32_t* chosen_expert, const uin
     return fail(ORDERMOE_ERR_INVALID_ARG, "dispatch_noalloc: null pointer");
   if (T > 0 && (!aligned16(X) || !aligned16(X_perm)))
     return fail(ORDERMOE_ERR_INVALID_ARG, "dispatch_noalloc: X and X_perm must be 16-byte aligned");
+  // the scratch this call's permutation uses, as ordermoe_dispatch sizes it
+  if (dispatch_workspace_bytes((int64_t)T * k, E) > sizeof(g_noalloc_hist))
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
+                "dispatch_noalloc: T*k = %lld needs more than the fixed %zu-byte scratch",
+                (long long)T * k, sizeof(g_noalloc_hist));
   int32_t* hist = nullptr;
   int rc = noalloc_scratch(&hist);
   if (rc) return rc;

@@ -49,10 +49,11 @@ def _both(chosen, X, T, k, E, d):
 
 def test_noalloc_dispatch_matches_workspace_dispatch_twice_in_a_row():
     rng = np.random.default_rng(77)
-    # first call: many experts and a full-size Mixtral batch; second call:
-    # fewer chunks and experts, so stale histogram entries of the first call
-    # remain in the shared scratch array
-    for T, k, E, d in [(4096, 2, 8, 4096), (1000, 6, 64, 256), (37, 3, 5, 64)]:
+    # first call: the largest size allowed (T*k = 262144 entries over 64
+    # experts fill the whole fixed scratch array); then a full-size Mixtral
+    # batch, then fewer chunks and experts, so stale histogram entries of the
+    # earlier calls remain in the shared scratch array
+    for T, k, E, d in [(32768, 8, 64, 64), (4096, 2, 8, 4096), (1000, 6, 64, 256), (37, 3, 5, 64)]:
         chosen = torch.as_tensor(rng.integers(0, E, (T, k)).astype(np.int32)).to(DEV)
         X = synth.normal((T, d), 1.0, seed=T + d, device=DEV)
         (a, b) = _both(chosen, X, T, k, E, d)
