@@ -32,11 +32,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # the recorded ncu capture of that kernel, valid only while the
 # kernel sources hash to the values recorded with it.
 GATE_UP_TRAFFIC = {
-    "bytes": 1958962176 + 228495104,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
+    "bytes": 2036953088 + 229376256,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
     "sha256": {"paper_2607_17154_gb300/csrc/grouped_gemm.cu":
-               "f49dcc230bf648405856ba4df19b215bd6b2da0df11ed4da96f2602ce903bc25",
+               "64119f0e07702e7a84e9a87cae2b3fe3fd64e15e1565fbc24e11e52530c58ed9",
                "paper_2607_17154_gb300/csrc/common.cuh":
-               "05db1330c6012b7861955d139033ee2abc5373149a3289af6cdb1771f30fd2cd"},
+               "5f0611cf723907b96ee41883667bfb1045d2e7d81cef1f06cf17694b13751bfb"},
 }
 
 
@@ -71,6 +71,8 @@ def parse():
     p.add_argument("--seed", type=int, default=0)
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-extras", action="store_true",
+                   help="mixtral_prefill: skip timing the other workloads after the main line")
     p.add_argument("--lookahead", type=int, default=1,
                    help="selection horizon H (Eqs. 41-43) for the decode stack; 1 = myopic")
     p.add_argument("--memory-ratio", type=float, default=None,
@@ -411,6 +413,78 @@ def run_ours(args, dist):
     }
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(w, inp, args.seed, args.cpu_seconds)
+    if w.name == "mixtral_prefill" and not args.no_extras:
+        torch.cuda.empty_cache()
+        out["other_workloads"] = other_workloads(args, dist, device)
+    return out
+
+
+EXTRA_STEPS = 50
+
+
+def other_workloads(args, dist, device):
+    """The other full-size workloads, each timed in this run like the main
+    one (CUDA events around K steps after W warm-up steps, clocks sampled
+    during the region), reported compactly: the fine-grained layer, the
+    decode stack (myopic and with the paper's default horizon H = 3) and the
+    offline plan."""
+    import copy
+
+    import torch
+    from paper_2607_17154_gb300 import synth
+    sub = copy.copy(args)
+    sub.steps = min(args.steps, EXTRA_STEPS)
+    sub.warmup = max(3, min(args.warmup, 5))
+    sub.no_cpu_baseline = True
+    sub.no_e2e = True
+    sub.no_extras = True
+    sub.theta = None
+    sub.n_cal = None
+    out = {}
+    # fine-grained layer: E = 64, top-6, Zipf homes
+    sub.workload = "fine_grained"
+    fg = run_ours(sub, dist)
+    r = fg["roofline"]
+    out["fine_grained"] = {
+        "value": fg["value"], "unit": UNIT, "steps": sub.steps, "ms_per_step": fg["ms_per_step"],
+        "gate_up": {k: r[k] for k in ("kernel", "achieved", "frac", "frac_burst", "frac_sustained",
+                                      "peak_applies", "ms_per_launch")},
+        "layer_tflops": r["layer_tflops"], "layer_frac": r["layer_frac"],
+        "breakdown_ms": fg["breakdown_ms"], "clocks": fg["clocks"],
+        "gpu_launches": fg["gpu_launches"]}
+    del fg
+    torch.cuda.empty_cache()
+    # decode stack on the residual map, H = 1 and H = 3
+    w = synth.workload("decode_stack")
+    sub.workload = "decode_stack"
+    sub.memory_ratio = None
+    S = decode_setup(sub, dist, w, device, 1)
+    dec = {}
+    for H in (1, 3):
+        ms, clocks, stack, *_ = decode_timed(sub, dist, w, device, S, H)
+        line = decode_line(sub, dist, w, ms, clocks, H, S)
+        dec["H%d" % H] = {"value": line["value"], "unit": UNIT, "steps": sub.steps,
+                          "ms_per_step": line["ms_per_step"],
+                          "hbm": {k: line["roofline"][k] for k in ("achieved", "peak", "frac", "unit",
+                                                                   "peak_source")},
+                          "clocks": clocks, "gpu_launches": line["gpu_launches"]}
+        del stack
+    dec["config"] = line["config"]
+    out["decode_stack"] = dec
+    del S
+    torch.cuda.empty_cache()
+    # offline plan: similarity + grouping + placement + redundancy + coverage
+    w = synth.workload("similarity")
+    sub.workload = "similarity"
+    pl = run_similarity(sub, dist, w, device)
+    out["similarity_plan"] = {
+        "value": pl["value"], "unit": pl["unit"], "metric": pl["metric"], "steps": sub.steps,
+        "ms_per_step": pl["ms_per_step"],
+        "tensor": {k: pl["roofline"][k] for k in ("achieved", "frac", "frac_burst", "frac_sustained",
+                                                  "peak_applies")},
+        "clocks": pl["clocks"], "gpu_launches": pl["gpu_launches"]}
+    del pl
+    torch.cuda.empty_cache()
     return out
 
 
@@ -550,14 +624,15 @@ def edge_cost_windows(args, w, device, layers, Xs, home, tabs, stride, P, H, sim
     return res
 
 
-def run_decode(args, dist, w, device):
-    """Decode stack: one step = 32 MoE layers over a batch of 128 tokens, with
-    the selection state carried across layers; bound by streaming the expert
-    weights from HBM."""
+def decode_setup(args, dist, w, device, H):
+    """The decode stack on the residual map: weights of every layer, the
+    calibration pass through the unmodified stack (similarity, counts and
+    transitions of each layer on the inputs it sees), the placement with b_m
+    carried over the layers (Alg. 1), optional replicas, and the tables."""
     import torch
     from paper_2607_17154_gb300 import binding as B
     from paper_2607_17154_gb300 import synth
-    from paper_2607_17154_gb300.layer import LayerStack
+    from paper_2607_17154_gb300.layer import calibrate_stack
     seed = args.seed + 1000 * dist.rank
     L, E, M = w.L, w.E, w.M
     layers = []
@@ -565,14 +640,9 @@ def run_decode(args, dist, w, device):
         inp = synth.layer_inputs(w, seed=seed, layer=l, device=device)
         layers.append({"W_r": inp["Wr"], "W1": inp["W1"], "W3": inp["W3"], "W2": inp["W2"]})
     home = torch.as_tensor(synth.layer_inputs(w, seed=seed, with_ffn=False)["home"]).to(device)
-    # offline plan of all layers at once: theta_l of Eq. 6, b_m carried over the layers
-    Xcal = synth.calibration(w.n_cal, w.d, seed, device=device)
-    Wr = torch.stack([l["W_r"] for l in layers])
-    sim = torch.empty(L, E, E, dtype=torch.float32, device=device)
-    counts = torch.empty(L, E, dtype=torch.int32, device=device)
-    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, w.n_cal), dtype=torch.uint8,
-                     device=device)
-    B.ordermoe_similarity(Wr, Xcal, L, E, w.d, w.n_cal, w.k, sim, counts, ws)
+    cal = calibrate_stack(layers, synth.calibration(w.n_cal, w.d, seed, device=device), w.k, M)
+    sim, counts, P = cal["sim"], cal["counts"], cal["P"]
+    del cal
     group = torch.empty(L, E, dtype=torch.int32, device=device)
     ng = torch.empty(L, dtype=torch.int32, device=device)
     theta = torch.empty(L, dtype=torch.float32, device=device)
@@ -593,12 +663,6 @@ def run_decode(args, dist, w, device):
         B.ordermoe_replicate(group, imp, pmem, Cm, pi, L, E, M, x, used, reps)
         plan.update({"replicas": int(reps.sum().item()),
                      "coverage_after": plan_coverage(B, group, ng, x, L, E, M, device)["coverage"]})
-    # transition statistics (Eq. 41) from the calibration logits the similarity
-    # call leaves at the start of its workspace
-    H = max(1, args.lookahead)
-    P = torch.empty(L - 1, E, E, dtype=torch.float32, device=device)
-    tcount = torch.empty(L - 1, E, E, dtype=torch.int32, device=device)
-    B.ordermoe_transitions(ws.view(torch.float32)[: w.n_cal * L * E], w.n_cal, L, E, w.k, tcount, P)
     sp = synth.server_params(M, w.d, w.dff, seed)
     f64 = lambda a: torch.as_tensor(a, dtype=torch.float64).to(device)
     th = theta.cpu().tolist()
@@ -608,9 +672,22 @@ def run_decode(args, dist, w, device):
         B.ordermoe_build_tables(sim[l], group[l], x[l], th[l], w.qbar, f64(sp.F), f64(sp.B),
                                 f64(sp.tau), sp.z, sp.c, sp.omega_T, sp.omega_Q,
                                 tabs[l * stride:(l + 1) * stride])
-    stack = LayerStack(layers, tabs, w.k, w.T, device, H=H, stride=stride, P=P)
-    Xs = [synth.hidden(w.T, w.d, seed + 5000 + l, device=device) for l in range(w.L)]
-    ys = [torch.empty(w.T, w.d, dtype=torch.bfloat16, device=device) for _ in range(w.L)]
+    h0 = synth.hidden(w.T, w.d, seed + 5000, device=device)
+    return {"layers": layers, "home": home, "sim": sim, "group": group, "x": x, "theta": theta,
+            "P": P, "tabs": tabs, "stride": stride, "sp": sp, "plan": plan, "ratio": ratio,
+            "h0": h0}
+
+
+def decode_timed(args, dist, w, device, S, H):
+    """Times graph-replayed (or eager) decode steps of the stack S with
+    horizon H; returns (ms, clocks, stack, hs, xs, loc, qhat)."""
+    import torch
+    from paper_2607_17154_gb300.layer import LayerStack
+    L = w.L
+    stack = LayerStack(S["layers"], S["tabs"], w.k, w.T, device, H=H, stride=S["stride"], P=S["P"])
+    home = S["home"]
+    hs = [S["h0"]] + [torch.empty_like(S["h0"]) for _ in range(L)]
+    xs = [torch.empty_like(S["h0"]) for _ in range(L + 1)]
     loc = home.clone()
     qhat = torch.zeros(w.T, device=device)
 
@@ -619,24 +696,46 @@ def run_decode(args, dist, w, device):
         qhat.zero_()
 
     if not args.eager:
-        graph = stack.capture(Xs, home, loc, qhat, ys, prologue=reset)
+        graph = stack.capture_residual(hs, xs, home, loc, qhat, prologue=reset)
         step = graph.replay
     else:
         def step():
             reset()
-            stack.step(Xs, home, loc, qhat, ys)
-
+            stack.step_residual(hs, xs, home, loc, qhat)
     ms, clocks = timed_region(args, dist, device, step)
+    return ms, clocks, stack, hs, xs, loc, qhat
+
+
+def decode_launches(w, H):
+    """Kernels of one decode step: the first layer's RMSNorm, then per layer
+    route_select 1, dispatch 2 (one block ranks up to 4096 entries) or 4,
+    gate/up 1, down 1 and the residual combine 1."""
+    return 1 + (4 + (2 if w.T * w.k <= 4096 else 4)) * w.L
+
+
+def run_decode(args, dist, w, device):
+    """Decode stack: one step = 32 MoE layers over a batch of 128 tokens on the
+    residual map (h_{l+1} = h_l + y_l, each layer reading RMSNorm(h_l)), with
+    the selection state carried across layers; bound by streaming the expert
+    weights from HBM."""
+    import torch
+    from paper_2607_17154_gb300 import binding as B
+    H = max(1, args.lookahead)
+    S = decode_setup(args, dist, w, device, H)
+    L, E = w.L, w.E
+    ms, clocks, stack, hs, xs, loc, qhat = decode_timed(args, dist, w, device, S, H)
     code, detail = B.ordermoe_device_error()
     if code:
         raise RuntimeError("device error %d (%d)" % (code, detail))
+    home, tabs, stride, P, layers = S["home"], S["tabs"], S["stride"], S["P"], S["layers"]
     # execution types of one step's decisions (untimed)
     kinds = torch.zeros(4, dtype=torch.int32, device=device)
     loc.copy_(home); qhat.zero_()
-    stack.step(Xs, home, loc, qhat, ys, counters=kinds)
+    stack.step_residual(hs, xs, home, loc, qhat, counters=kinds)
     exec_types = dict(zip(["local_exact", "local_sub", "remote_exact", "remote_sub"],
                           kinds.cpu().tolist()))
-    # decision time: the selection alone (router + top-k + Alg. 2) over the 32 layers
+    # decision time: the selection alone (router + top-k + Alg. 2) over the 32 layers, on the
+    # layer inputs of that step
     f = lambda *sh, dt: torch.empty(*sh, dtype=dt, device=device)
     sel = [f(w.T, w.k, dt=dt) for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
@@ -646,15 +745,23 @@ def run_decode(args, dist, w, device):
         loc.copy_(home); qhat.zero_()
         for l in range(L):
             Hl = min(H, L - l)
-            B.ordermoe_route_select_lookahead(Xs[l], layers[l]["W_r"], None, w.T, E, w.d, w.k, 1,
+            B.ordermoe_route_select_lookahead(xs[l], layers[l]["W_r"], None, w.T, E, w.d, w.k, 1,
                                               tabs[l * stride:], stride, Hl,
                                               P[l:l + Hl - 1].contiguous() if Hl > 1 else None,
                                               home, loc, qhat, None, *sel)
     ev[1].record(stream)
     torch.cuda.synchronize(device)
     select_ms_per_layer = ev[0].elapsed_time(ev[1]) / (5 * L)
-    edge = edge_cost_windows(args, w, device, layers, Xs, home, tabs, stride, P, H, sim, group, x,
-                             theta, sp)
+    edge = edge_cost_windows(args, w, device, layers, xs[:L], home, tabs, stride, P, H, S["sim"],
+                             S["group"], S["x"], S["theta"], S["sp"])
+    out = decode_line(args, dist, w, ms, clocks, H, S)
+    out.update({"plan": S["plan"], "exec_types": exec_types, "edge": edge,
+                "selection_ms_per_layer": round(select_ms_per_layer, 4),
+                "selection_us_per_token_layer": round(select_ms_per_layer * 1e3 / w.T, 4)})
+    return out
+
+
+def decode_line(args, dist, w, ms, clocks, H, S):
     step_s = ms / args.steps / 1e3
     wbytes = 3.0 * w.E * w.d * w.dff * 2 * w.L
     pk, pk_kind = peaks()
@@ -666,25 +773,20 @@ def run_decode(args, dist, w, device):
         "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": {"workload": w.name, "layers": w.L, "T": w.T, "d": w.d, "E": w.E, "k": w.k,
-                   "d_ff": w.dff, "M": w.M, "lookahead_H": H, "memory_ratio": ratio,
+                   "d_ff": w.dff, "M": w.M, "lookahead_H": H, "memory_ratio": S["ratio"],
+                   "inter_layer": "h_{l+1} = h_l + y_l, layer input RMSNorm(h_l)",
                    "cuda_graph": not args.eager,
                    "l2": "inputs larger than L2: %.1f GB of expert weights" % (wbytes / 1e9)},
         "roofline": {"kernel": "whole decode step (expert weight streaming)", "bound": "hbm",
                      "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": None,
                      "peak_source": "%s hbm_gbs" % pk_kind, "bytes_per_step": wbytes},
-        # route_select 1, dispatch 2 (one block ranks up to 4096 entries) or 4,
-        # gate/up 1, down 1, combine 1 a layer, plus the look-ahead selection
-        # pass on every layer that looks ahead (all but the last when H > 1)
-        "gpu_launches": ((4 + (2 if w.T * w.k <= 4096 else 4)) * w.L
+        # plus the look-ahead selection pass on every layer that looks ahead
+        # (all but the last when H > 1)
+        "gpu_launches": (decode_launches(w, H)
                          + sum(min(H, w.L - l) > 1 for l in range(w.L))) * args.steps,
         "clocks": clocks,
         "lookahead_H": H,
-        "plan": plan,
-        "exec_types": exec_types,
-        "edge": edge,
-        "selection_ms_per_layer": round(select_ms_per_layer, 4),
-        "selection_us_per_token_layer": round(select_ms_per_layer * 1e3 / w.T, 4),
     }
 
 
@@ -813,8 +915,57 @@ def cpu_cores():
         return os.cpu_count() or 1
 
 
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() in ("Model name", "Model"):
+                name = line.split(":", 1)[1].strip()
+                if name and not name.isdigit():
+                    return name
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu part")):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return "unknown"
+
+
+def tiny_oracle_rate(seed, threads):
+    """Tokens/s of the whole oracle path on the tiny layer (T 64, d 256, E 8,
+    top-2, d_ff 512) with the given OpenMP thread count."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_17154_gb300 import synth
+    w = synth.workload("tiny")
+    inp = synth.layer_inputs(w, seed=seed)
+    host, home, tab = oracle_setup(w, inp, seed)
+    prev = oracle.threads()
+    oracle.set_threads(threads)
+    try:
+        toks = np.arange(w.T)
+        oracle_tokens(w, host, home, tab, toks)
+        reps, t0 = 0, time.perf_counter()
+        while reps < 3 or time.perf_counter() - t0 < 1.0:
+            oracle_tokens(w, host, home, tab, toks)
+            reps += 1
+        dt = time.perf_counter() - t0
+    finally:
+        oracle.set_threads(prev)
+    return {"value": round(w.T * reps / dt, 1), "unit": UNIT, "threads": threads,
+            "sample": "all %d tokens of the tiny layer, %d passes, %.2f s" % (w.T, reps, dt)}
+
+
 def cpu_baseline(w, inp, seed, target_s):
     import numpy as np
+
+    import oracle
     host, home, tab = oracle_setup(w, inp, seed)
     rng = np.random.default_rng(seed)
     t0 = time.perf_counter()
@@ -825,16 +976,21 @@ def cpu_baseline(w, inp, seed, target_s):
     t0 = time.perf_counter()
     oracle_tokens(w, host, home, tab, toks)
     dt = time.perf_counter() - t0
-    return {"value": round(n / dt, 3), "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+    return {"value": round(n / dt, 3), "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
             "sample": "%d of the %d tokens of one %s layer through the whole oracle path "
                       "(router, top-k, selection, permutation, SwiGLU FFN, combine), %.1f s"
-                      % (n, w.T, w.name, dt)}
+                      % (n, w.T, w.name, dt),
+            "cpu_model": cpu_model(), "host_cpus": cpu_cores(), "omp_threads": oracle.threads(),
+            "tiny_1_thread": tiny_oracle_rate(seed, 1),
+            "tiny_all_threads": tiny_oracle_rate(seed, oracle.threads())}
 
 
 def run_reference(args, dist):
     """The CPU oracle as it stands, each step a bounded sample of the workload."""
     import numpy as np
     import torch
+
+    import oracle
     from paper_2607_17154_gb300 import synth
     w = synth.workload(args.workload)
     device = "cuda" if torch.cuda.is_available() else "cpu"
@@ -862,8 +1018,9 @@ def run_reference(args, dist):
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": w.name, "T": w.T, "d": w.d, "E": w.E, "k": w.k, "d_ff": w.dff,
                    "M": w.M, "tokens_per_step": n},
-        "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cpu_cores(),
-                         "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": oracle.threads(),
+                         "kind": "oracle", "sample": sample, "cpu_model": cpu_model(),
+                         "host_cpus": cpu_cores(), "omp_threads": oracle.threads()},
         "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }

@@ -247,6 +247,34 @@ int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of, const float*
                      int k, int d, uint16_t* y, ordermoe_stream_t stream);
 
 /* ------------------------------------------------------------------------
+ * Residual map between stacked MoE layers (a decoder block without its
+ * attention half; the paper's Mixtral-8x7B model, Section VI-A, stacks 32
+ * such layers). The residual stream h (bf16) carries the layer outputs and
+ * each layer reads its RMS-normalised copy x (pre-norm, unit gain):
+ *   x_0 = RMSNorm(h_0),  h_{l+1} = h_l + y_l,  x_{l+1} = RMSNorm(h_{l+1}),
+ *   RMSNorm(v)[c] = bf16( v[c] / sqrt(mean_c(v[c]^2) + eps) ).
+ * Without the normalisation the outputs of random-weight SwiGLU experts grow
+ * quadratically with their input and overflow within a few layers.
+ *
+ * ordermoe_rmsnorm: x = RMSNorm(h) for T rows of d.
+ *   h, x [T][d] bf16 (16-byte aligned), eps > 0; x may not overlap h.
+ * ordermoe_combine_residual_norm: the weighted combine added to the residual
+ * stream, and the next layer's input, in one pass:
+ *   h_out[t] = bf16( h[t] + sum_{j<k} topk_w[t][j] Y_perm[row_of[t][j]] )
+ *   (fp32, slot order), x_out[t] = RMSNorm(h_out[t]) (sum of squares of the
+ *   bf16 values of h_out in fp32, fixed reduction order).
+ *   Y_perm [T*k][d], h, h_out, x_out [T][d] bf16 (16-byte aligned, h, h_out
+ *   and x_out mutually disjoint); row_of, topk_w as ordermoe_combine; d % 8 == 0.
+ *   A row_of entry outside [0, T*k) sets ORDERMOE_DEV_BAD_INDEX (detail: the
+ *   token) and leaves that token's h_out and x_out unwritten. */
+int ordermoe_rmsnorm(const uint16_t* h, int T, int d, float eps, uint16_t* x,
+                     ordermoe_stream_t stream);
+int ordermoe_combine_residual_norm(const uint16_t* Y_perm, const int32_t* row_of,
+                                   const float* topk_w, const uint16_t* h, int T, int k, int d,
+                                   float eps, uint16_t* h_out, uint16_t* x_out,
+                                   ordermoe_stream_t stream);
+
+/* ------------------------------------------------------------------------
  * One whole MoE layer: route_select, dispatch, expert_gate_up, expert_down and
  * combine in order on `stream`, with all intermediates in `scratch`.
  * The descriptor (host memory) holds device pointers owned by the caller:
@@ -287,6 +315,20 @@ size_t ordermoe_layer_scratch_bytes(int T_max, int E, int d, int dff, int k);
 int ordermoe_layer_forward(const ordermoe_layer_desc* layer, int T, const uint16_t* X,
                            const uint8_t* home, uint8_t* loc, float* qhat, uint16_t* y,
                            int32_t* counters, int host_io, ordermoe_stream_t stream);
+
+/* One layer of a stack on the residual map above (device pointers only):
+ * the layer routes and runs x (= RMSNorm(h)), then
+ * ordermoe_combine_residual_norm writes h_out = h + y and x_out =
+ * RMSNorm(h_out), the next layer's h and x. loc / qhat, counters and the
+ * look-ahead fields of the descriptor as ordermoe_layer_forward; logits_out
+ * [T][E] f32 (nullable) receives the router logits of x (the calibration
+ * pass of a stack records them for ordermoe_transitions_strided).
+ *   x, h, h_out, x_out [T][d] bf16, 16-byte aligned, h / h_out / x_out
+ *   mutually disjoint; eps > 0. */
+int ordermoe_layer_forward_residual(const ordermoe_layer_desc* layer, int T, const uint16_t* x,
+                                    const uint16_t* h, const uint8_t* home, uint8_t* loc,
+                                    float* qhat, float eps, uint16_t* h_out, uint16_t* x_out,
+                                    float* logits_out, int32_t* counters, ordermoe_stream_t stream);
 
 /* nbatch independent batches of T tokens through one layer, from and to
  * pinned HOST memory, each batch as ordermoe_layer_forward with host_io = 1
@@ -354,6 +396,16 @@ int ordermoe_similarity_no_logits(const uint16_t* W_r, const uint16_t* X_cal, in
  *   counts [L-1][E][E] i32 out, P [L-1][E][E] f32 out. Needs L >= 2. */
 int ordermoe_transitions(const float* logits, int64_t N, int L, int E, int k_freq, int32_t* counts,
                          float* P, ordermoe_stream_t stream);
+
+/* ordermoe_transitions over logits in any layout: the E logits of token n at
+ * layer l start at logits + n * token_stride + l * layer_stride (floats; both
+ * strides >= E). Layer-major logits [L][N][E], as a stack's calibration pass
+ * records them one layer at a time, have token_stride = E and
+ * layer_stride = N * E; ordermoe_transitions is token_stride = L * E,
+ * layer_stride = E. Same results and rules. */
+int ordermoe_transitions_strided(const float* logits, int64_t N, int L, int E, int k_freq,
+                                 int64_t token_stride, int64_t layer_stride, int32_t* counts,
+                                 float* P, ordermoe_stream_t stream);
 
 /* Activation counts of Eq. 5 from given logits [N][E] f32 (top-k_freq per
  * token, ties to the lower index). counts [E] i32 out (overwritten). */

@@ -45,6 +45,8 @@ def lib():
             "orc_gather_rows": [_P, _P, _I64, _I, _P],
             "orc_ffn_rows": [_P, _P, _I64, _P, _P, _P, _I, _I, _I, _P, _P],
             "orc_combine": [_P, _P, _P, _I, _I, _I, _P],
+            "orc_rmsnorm": [_P, _I, _I, _D, _P],
+            "orc_combine_residual": [_P, _P, _P, _P, _I, _I, _I, _P],
             "orc_similarity": [_P, _P, _I, _I, _I64, _P, _P],
             "orc_expert_counts": [_P, _I64, _I, _I, _P],
             "orc_group": [_P, _P, _I, _F, _P, _P, _P],
@@ -63,6 +65,10 @@ def lib():
             fn = getattr(L, name)
             fn.argtypes = args
             fn.restype = _I
+        L.orc_threads.argtypes = []
+        L.orc_threads.restype = _I
+        L.orc_set_threads.argtypes = [_I]
+        L.orc_set_threads.restype = _I
         L.orc_theta.argtypes = [_I, _I, _D, _D, _D]
         L.orc_theta.restype = _F
         _lib = L
@@ -171,6 +177,34 @@ def combine(Yp, row_of, w):
     y = np.empty((T, d), np.uint16)
     _check(lib().orc_combine(_ptr(Yp), _ptr(row_of), _ptr(w), T, k, d, _ptr(y)), "orc_combine")
     return y
+
+
+def threads():
+    """OpenMP threads the oracle's parallel loops use."""
+    return int(lib().orc_threads())
+
+
+def set_threads(n):
+    _check(lib().orc_set_threads(int(n)), "orc_set_threads")
+
+
+def rmsnorm(h, eps=1e-6):
+    """x = RMSNorm(h) of the residual map between stacked layers (bf16 bits, fp64 math)."""
+    h = _c(h, np.uint16); T, d = h.shape
+    x = np.empty((T, d), np.uint16)
+    _check(lib().orc_rmsnorm(_ptr(h), T, d, float(eps), _ptr(x)), "orc_rmsnorm")
+    return x
+
+
+def combine_residual(Yp, row_of, w, h):
+    """h_out = bf16(h + sum_j w_j Y[row_of[t][j]]) (bf16 bits, fp64 math)."""
+    Yp = _c(Yp, np.uint16); row_of = _c(row_of, np.int32); w = _c(w, np.float32)
+    h = _c(h, np.uint16)
+    T, k = row_of.shape; d = h.shape[1]
+    out = np.empty((T, d), np.uint16)
+    _check(lib().orc_combine_residual(_ptr(Yp), _ptr(row_of), _ptr(w), _ptr(h), T, k, d,
+                                      _ptr(out)), "orc_combine_residual")
+    return out
 
 
 def similarity(W, Xc, return_H=False):

@@ -38,6 +38,8 @@
 #include <cstring>
 #include <vector>
 
+#include <omp.h>
+
 namespace {
 
 float bf16_bits_to_float(uint16_t h) {
@@ -326,6 +328,41 @@ int orc_combine(const uint16_t* Yp, const int32_t* row_of, const float* w, int T
         acc += static_cast<double>(w[(int64_t)t * k + j]) * bf(Yp, row * d + c);
       }
       y[(int64_t)t * d + c] = float_to_bf16_bits(static_cast<float>(acc));
+    }
+  return ORC_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Residual map between stacked MoE layers. The paper serves Mixtral-8x7B
+// (Section VI-A), a stack of pre-norm decoder blocks; without the attention
+// half, block l maps the residual stream h_l to h_{l+1} = h_l + y_l, where
+// y_l is the MoE layer's output for the input x_l = RMSNorm(h_l) (unit gain):
+//   RMSNorm(v)[c] = bf16( v[c] / sqrt( (1/d) sum_c v[c]^2 + eps ) )    (fp64)
+//   h_out[t][c]   = bf16( h[t][c] + sum_j w[t][j] Y[row_of[t][j]][c] )  (fp64, slot order)
+int orc_rmsnorm(const uint16_t* h, int T, int d, double eps, uint16_t* x) {
+  if (T < 0 || d <= 0 || !(eps > 0.0)) return ORC_BAD_ARG;
+  for (int t = 0; t < T; ++t) {
+    const uint16_t* row = h + (int64_t)t * d;
+    double ss = 0.0;
+    for (int c = 0; c < d; ++c) ss += bf(row, c) * bf(row, c);
+    const double rms = std::sqrt(ss / d + eps);
+    for (int c = 0; c < d; ++c)
+      x[(int64_t)t * d + c] = float_to_bf16_bits(static_cast<float>(bf(row, c) / rms));
+  }
+  return ORC_OK;
+}
+
+int orc_combine_residual(const uint16_t* Yp, const int32_t* row_of, const float* w,
+                         const uint16_t* h, int T, int k, int d, uint16_t* h_out) {
+  if (T < 0 || k <= 0 || d <= 0) return ORC_BAD_ARG;
+  for (int t = 0; t < T; ++t)
+    for (int c = 0; c < d; ++c) {
+      double acc = bf(h, (int64_t)t * d + c);
+      for (int j = 0; j < k; ++j) {
+        const int64_t row = row_of[(int64_t)t * k + j];
+        acc += static_cast<double>(w[(int64_t)t * k + j]) * bf(Yp, row * d + c);
+      }
+      h_out[(int64_t)t * d + c] = float_to_bf16_bits(static_cast<float>(acc));
     }
   return ORC_OK;
 }
@@ -781,6 +818,16 @@ int orc_coverage(const uint8_t* placement_l, const int32_t* group_l, int E, int 
   for (int m = 0; m < M; ++m)
     for (int e = 0; e < E; ++e)
       if (placement_l[m * E + e]) cover[m * K + group_l[e]] = 1;
+  return ORC_OK;
+}
+
+// Threads of the oracle's OpenMP loops (only over independent tokens and
+// rows, so the results do not depend on it): the count the next parallel
+// region uses, and a setter (n >= 1) for timing the oracle on fewer cores.
+int orc_threads(void) { return omp_get_max_threads(); }
+int orc_set_threads(int n) {
+  if (n < 1) return ORC_BAD_ARG;
+  omp_set_num_threads(n);
   return ORC_OK;
 }
 

@@ -65,7 +65,14 @@ _SIGNATURES = {
                        _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _SZ, _P], _I),
     "ordermoe_route_select_lookahead": ([_P, _P, _P, _I, _I, _I, _I, _I, _P, _SZ, _I, _P, _P, _P,
                                          _P, _P, _P, _P, _P, _P, _P, _P, _P], _I),
+    "ordermoe_rmsnorm": ([_P, _I, _I, _F, _P, _P], _I),
+    "ordermoe_combine_residual_norm": ([_P, _P, _P, _P, _I, _I, _I, _F, _P, _P, _P], _I),
+    "ordermoe_layer_forward_residual": ([_P, _I, _P, _P, _P, _P, _P, _F, _P, _P, _P, _P, _P], _I),
+    "ordermoe_transitions_strided": ([_P, _I64, _I, _I, _I, _I64, _I64, _P, _P, _P], _I),
 }
+
+# RMSNorm epsilon of the residual map between stacked layers
+NORM_EPS = 1e-6
 
 
 class LayerDesc(ctypes.Structure):
@@ -408,6 +415,37 @@ def ordermoe_layer_forward(desc, T, X, home, loc, qhat, y, counters=None, host_i
     _check("ordermoe_layer_forward", rc)
 
 
+def ordermoe_rmsnorm(h, T, d, eps, x, stream=None):
+    _dt(h, torch.bfloat16, "h"); _dt(x, torch.bfloat16, "x")
+    _check("ordermoe_rmsnorm", lib().ordermoe_rmsnorm(_ptr(h), T, d, float(eps), _ptr(x),
+                                                      _stream(stream)))
+
+
+def ordermoe_combine_residual_norm(Y_perm, row_of, topk_w, h, T, k, d, eps, h_out, x_out,
+                                   stream=None):
+    _dt(Y_perm, torch.bfloat16, "Y_perm"); _dt(row_of, torch.int32, "row_of")
+    _dt(topk_w, torch.float32, "topk_w")
+    for n, t in (("h", h), ("h_out", h_out), ("x_out", x_out)):
+        _dt(t, torch.bfloat16, n)
+    rc = lib().ordermoe_combine_residual_norm(_ptr(Y_perm), _ptr(row_of), _ptr(topk_w), _ptr(h), T,
+                                              k, d, float(eps), _ptr(h_out), _ptr(x_out),
+                                              _stream(stream))
+    _check("ordermoe_combine_residual_norm", rc)
+
+
+def ordermoe_layer_forward_residual(desc, T, x, h, home, loc, qhat, eps, h_out, x_out,
+                                    logits_out=None, counters=None, stream=None):
+    for n, t in (("x", x), ("h", h), ("h_out", h_out), ("x_out", x_out)):
+        _dt(t, torch.bfloat16, n)
+    _dt(home, torch.uint8, "home"); _dt(loc, torch.uint8, "loc"); _dt(qhat, torch.float32, "qhat")
+    _dt(logits_out, torch.float32, "logits_out")
+    rc = lib().ordermoe_layer_forward_residual(ctypes.byref(desc), T, _ptr(x), _ptr(h), _ptr(home),
+                                               _ptr(loc), _ptr(qhat), float(eps), _ptr(h_out),
+                                               _ptr(x_out), _ptr(logits_out), _ptr(counters),
+                                               _stream(stream))
+    _check("ordermoe_layer_forward_residual", rc)
+
+
 def ordermoe_layer_batches_scratch_bytes(T_max, E, d, dff, k):
     return int(lib().ordermoe_layer_batches_scratch_bytes(T_max, E, d, dff, k))
 
@@ -442,6 +480,15 @@ def ordermoe_transitions(logits, N, L, E, k_freq, counts, P, stream=None):
     _check("ordermoe_transitions",
            lib().ordermoe_transitions(_ptr(logits), N, L, E, k_freq, _ptr(counts), _ptr(P),
                                       _stream(stream)))
+
+
+def ordermoe_transitions_strided(logits, N, L, E, k_freq, token_stride, layer_stride, counts, P,
+                                 stream=None):
+    _dt(logits, torch.float32, "logits"); _dt(counts, torch.int32, "counts"); _dt(P, torch.float32, "P")
+    _check("ordermoe_transitions_strided",
+           lib().ordermoe_transitions_strided(_ptr(logits), N, L, E, k_freq, int(token_stride),
+                                              int(layer_stride), _ptr(counts), _ptr(P),
+                                              _stream(stream)))
 
 
 def ordermoe_route_select_lookahead(X, W_r, logits_in, T, E, d, k, renorm, tables, tables_stride, H,

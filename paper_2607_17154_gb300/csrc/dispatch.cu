@@ -255,6 +255,104 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict
   }
 }
 
+// Pre-norm residual map between MoE layers (a decoder block without its
+// attention half): h' = h + sum_j w_j Y_perm[row_of[t][j]] (the layer output
+// added to the residual stream), x' = RMSNorm(h') = h' / sqrt(mean(h'^2) + eps)
+// (the next layer's input, unit gain). One block of kNormThreads per token;
+// thread i handles the 16-byte vectors i, i + kNormThreads, ...; the sum of
+// squares is taken over the bf16 values written to h', reduced in a fixed
+// order (warp butterflies, then the warps in order), so the result is
+// deterministic. WITH_Y = false is RMSNorm alone (x = RMSNorm(h)).
+constexpr int kNormThreads = 128;
+
+template <bool WITH_Y>
+__global__ void __launch_bounds__(kNormThreads) residual_norm_kernel(
+    const uint16_t* __restrict__ Yp, const int32_t* __restrict__ row_of,
+    const float* __restrict__ w, const uint16_t* __restrict__ h, int T, int k, int d, float eps,
+    uint16_t* __restrict__ h_out, uint16_t* __restrict__ x_out) {
+  __shared__ float wsum[kNormThreads / 32];
+  __shared__ int bad;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nvec = d >> 3;
+  for (int t = blockIdx.x; t < T; t += gridDim.x) {
+    int rows[ORDERMOE_MAX_TOPK];
+    float ws[ORDERMOE_MAX_TOPK];
+    if (tid == 0) bad = 0;
+    __syncthreads();
+#pragma unroll
+    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
+      rows[j] = 0;
+      ws[j] = 0.0f;
+      if (WITH_Y && j < k) {
+        rows[j] = row_of[(size_t)t * k + j];
+        ws[j] = w[(size_t)t * k + j];
+        if (rows[j] < 0 || (int64_t)rows[j] >= (int64_t)T * k) bad = 1;
+      }
+    }
+    __syncthreads();
+    if (bad) {  // a row index outside Y_perm: report, leave token t untouched
+      if (tid == 0) report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, t);
+      __syncthreads();
+      continue;
+    }
+    const uint4* hrow = reinterpret_cast<const uint4*>(h + (size_t)t * d);
+    uint4* hw = reinterpret_cast<uint4*>(h_out + (size_t)t * d);
+    float ss = 0.0f;
+    for (int v = tid; v < nvec; v += kNormThreads) {
+      const uint4 hv = __ldg(hrow + v);
+      float a[8] = {bf16_lo(hv.x), bf16_hi(hv.x), bf16_lo(hv.y), bf16_hi(hv.y),
+                    bf16_lo(hv.z), bf16_hi(hv.z), bf16_lo(hv.w), bf16_hi(hv.w)};
+      if (WITH_Y) {
+        uint4 yv[ORDERMOE_MAX_TOPK];
+#pragma unroll
+        for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j)
+          if (j < k) yv[j] = __ldg(reinterpret_cast<const uint4*>(Yp + (size_t)rows[j] * d) + v);
+#pragma unroll
+        for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
+          if (j >= k) break;
+          const float wj = ws[j];
+          a[0] = fmaf(wj, bf16_lo(yv[j].x), a[0]); a[1] = fmaf(wj, bf16_hi(yv[j].x), a[1]);
+          a[2] = fmaf(wj, bf16_lo(yv[j].y), a[2]); a[3] = fmaf(wj, bf16_hi(yv[j].y), a[3]);
+          a[4] = fmaf(wj, bf16_lo(yv[j].z), a[4]); a[5] = fmaf(wj, bf16_hi(yv[j].z), a[5]);
+          a[6] = fmaf(wj, bf16_lo(yv[j].w), a[6]); a[7] = fmaf(wj, bf16_hi(yv[j].w), a[7]);
+        }
+        uint4 o;
+        o.x = pack_bf16x2(a[0], a[1]); o.y = pack_bf16x2(a[2], a[3]);
+        o.z = pack_bf16x2(a[4], a[5]); o.w = pack_bf16x2(a[6], a[7]);
+        hw[v] = o;
+        const float r[8] = {bf16_lo(o.x), bf16_hi(o.x), bf16_lo(o.y), bf16_hi(o.y),
+                            bf16_lo(o.z), bf16_hi(o.z), bf16_lo(o.w), bf16_hi(o.w)};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ss = fmaf(r[i], r[i], ss);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) ss = fmaf(a[i], a[i], ss);
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    if (lane == 0) wsum[warp] = ss;
+    __syncthreads();
+    float tot = 0.0f;
+#pragma unroll
+    for (int i = 0; i < kNormThreads / 32; ++i) tot += wsum[i];
+    const float inv = __frsqrt_rn(__fadd_rn(__fdiv_rn(tot, static_cast<float>(d)), eps));
+    // the residual values this thread wrote above (its own stores), or h
+    const uint4* src = WITH_Y ? reinterpret_cast<const uint4*>(h_out + (size_t)t * d) : hrow;
+    uint4* xw = reinterpret_cast<uint4*>(x_out + (size_t)t * d);
+    for (int v = tid; v < nvec; v += kNormThreads) {
+      const uint4 hv = src[v];
+      uint4 o;
+      o.x = pack_bf16x2(__fmul_rn(bf16_lo(hv.x), inv), __fmul_rn(bf16_hi(hv.x), inv));
+      o.y = pack_bf16x2(__fmul_rn(bf16_lo(hv.y), inv), __fmul_rn(bf16_hi(hv.y), inv));
+      o.z = pack_bf16x2(__fmul_rn(bf16_lo(hv.z), inv), __fmul_rn(bf16_hi(hv.z), inv));
+      o.w = pack_bf16x2(__fmul_rn(bf16_lo(hv.w), inv), __fmul_rn(bf16_hi(hv.w), inv));
+      xw[v] = o;
+    }
+    __syncthreads();  // wsum and bad are reused by the next token
+  }
+}
+
 // Small batches (n <= kSmallN entries, e.g. a decode step): histogram, offsets
 // and the stable rank in one block of 1024 threads. Pass 1 counts every
 // expert; pass 2 walks the entries in rounds of 1024 in index order, ranks
@@ -383,6 +481,54 @@ extern "C" int ordermoe_dispatch(const int32_t* chosen_expert, const uint16_t* X
     return fail(ORDERMOE_ERR_INVALID_ARG, "dispatch: workspace too small");
   return dispatch_launch(chosen_expert, X, T, k, E, d, offsets, row_token, row_of, X_perm,
                          static_cast<int32_t*>(workspace), stream);
+}
+
+static bool overlaps(const void* a, const void* b, size_t bytes) {
+  const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+  return x < y + bytes && y < x + bytes;
+}
+
+extern "C" int ordermoe_rmsnorm(const uint16_t* h, int T, int d, float eps, uint16_t* x,
+                                ordermoe_stream_t stream) {
+  OM_TRACE();
+  if (T < 0 || d <= 0 || d % 8 != 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "rmsnorm: need T >= 0 and d a positive multiple of 8");
+  if (!(eps > 0.0f)) return fail(ORDERMOE_ERR_INVALID_ARG, "rmsnorm: eps must be > 0");
+  if (T == 0) return ORDERMOE_OK;
+  if (!h || !x || !aligned16(h) || !aligned16(x))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "rmsnorm: null or not 16-byte aligned pointer");
+  const int grid = T < num_sms() * 16 ? T : num_sms() * 16;
+  residual_norm_kernel<false><<<grid, kNormThreads, 0, stream>>>(nullptr, nullptr, nullptr, h, T, 1,
+                                                                  d, eps, nullptr, x);
+  OM_LAUNCHED("residual_norm_kernel<rmsnorm>");
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_combine_residual_norm(const uint16_t* Y_perm, const int32_t* row_of,
+                                              const float* topk_w, const uint16_t* h, int T, int k,
+                                              int d, float eps, uint16_t* h_out, uint16_t* x_out,
+                                              ordermoe_stream_t stream) {
+  OM_TRACE();
+  if (T < 0 || k <= 0 || k > ORDERMOE_MAX_TOPK)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "combine_residual_norm: need T >= 0, 1 <= k <= 8");
+  if (d <= 0 || d % 8 != 0)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE,
+                "combine_residual_norm: d must be a positive multiple of 8");
+  if (!(eps > 0.0f)) return fail(ORDERMOE_ERR_INVALID_ARG, "combine_residual_norm: eps must be > 0");
+  if (T == 0) return ORDERMOE_OK;
+  if (!Y_perm || !row_of || !topk_w || !h || !h_out || !x_out)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "combine_residual_norm: null pointer");
+  if (!aligned16(Y_perm) || !aligned16(h) || !aligned16(h_out) || !aligned16(x_out))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "combine_residual_norm: bf16 arrays must be 16-byte aligned");
+  const size_t row_bytes = (size_t)T * d * 2;
+  if (overlaps(h, h_out, row_bytes) || overlaps(h, x_out, row_bytes) ||
+      overlaps(h_out, x_out, row_bytes))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "combine_residual_norm: h, h_out and x_out must not overlap");
+  const int grid = T < num_sms() * 16 ? T : num_sms() * 16;
+  residual_norm_kernel<true><<<grid, kNormThreads, 0, stream>>>(Y_perm, row_of, topk_w, h, T, k, d,
+                                                                 eps, h_out, x_out);
+  OM_LAUNCHED("residual_norm_kernel<combine>");
+  return ORDERMOE_OK;
 }
 
 extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,

@@ -125,23 +125,73 @@ extern "C" size_t ordermoe_layer_scratch_bytes(int T_max, int E, int d, int dff,
   return carve(nullptr, T_max, E, d, dff, k).bytes;
 }
 
+// Checks of the layer descriptor shared by the single-call entry points.
+static int check_layer(const ordermoe_layer_desc* L, int T, const char* who) {
+  if (!L) return fail(ORDERMOE_ERR_INVALID_ARG, "%s: null layer", who);
+  if (T < 0 || T > L->T_max) return fail(ORDERMOE_ERR_INVALID_ARG, "%s: need 0 <= T <= T_max", who);
+  if (!L->W_r || !L->W1 || !L->W3 || !L->W2 || !L->tables || !L->scratch)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "%s: null pointer in the layer", who);
+  if ((reinterpret_cast<uintptr_t>(L->scratch) & 255u) != 0)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "%s: scratch must be 256-byte aligned", who);
+  const size_t need = ordermoe_layer_scratch_bytes(L->T_max, L->E, L->d, L->dff, L->k);
+  if (need == 0 || L->scratch_bytes < need)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "%s: scratch too small or bad shape", who);
+  if (L->d % 256 != 0 || L->dff % 128 != 0 || L->k > L->E)
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "%s: need d %% 256 == 0, dff %% 128 == 0, k <= E", who);
+  if (!aligned16(L->W_r) || !aligned16(L->W1) || !aligned16(L->W3) || !aligned16(L->W2))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "%s: weights must be 16-byte aligned", who);
+  return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_combine_residual_norm(const uint16_t* Y_perm, const int32_t* row_of,
+                                              const float* topk_w, const uint16_t* h, int T, int k,
+                                              int d, float eps, uint16_t* h_out, uint16_t* x_out,
+                                              ordermoe_stream_t stream);
+
+extern "C" int ordermoe_layer_forward_residual(const ordermoe_layer_desc* L, int T,
+                                               const uint16_t* x, const uint16_t* h,
+                                               const uint8_t* home, uint8_t* loc, float* qhat,
+                                               float eps, uint16_t* h_out, uint16_t* x_out,
+                                               float* logits_out, int32_t* counters,
+                                               ordermoe_stream_t stream) {
+  OM_TRACE();
+  int rc = check_layer(L, T, "layer_forward_residual");
+  if (rc || T == 0) return rc;
+  if (!x || !h || !home || !h_out || !x_out)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_residual: null x/h/home/h_out/x_out");
+  if (!aligned16(x) || !aligned16(h) || !aligned16(h_out) || !aligned16(x_out))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_residual: x, h, h_out, x_out must be 16-byte aligned");
+  if ((loc == nullptr) != (qhat == nullptr))
+    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward_residual: give both loc and qhat, or neither");
+  const int E = L->E, d = L->d, dff = L->dff, k = L->k, R = T * k;
+  LayerScratch s = carve(static_cast<uint8_t*>(L->scratch), L->T_max, E, d, dff, k);
+  if (L->lookahead_H > 1)
+    rc = ordermoe_route_select_lookahead(x, L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
+                                         L->tables_stride, L->lookahead_H, L->P, home, loc, qhat,
+                                         logits_out, s.topk_idx, s.topk_w, s.chosen, s.server,
+                                         s.kind, counters, stream);
+  else
+    rc = ordermoe_route_select(x, L->W_r, nullptr, T, E, d, k, L->renorm, L->tables,
+                               L->tables_bytes, home, loc, qhat, logits_out, s.topk_idx, s.topk_w,
+                               s.chosen, s.server, s.kind, counters, stream);
+  if (rc) return rc;
+  rc = dispatch_launch(s.chosen, x, T, k, E, d, s.offsets, s.row_token, s.row_of, s.X_perm, s.hist,
+                       stream);
+  if (rc) return rc;
+  rc = gate_up_launch(s.X_perm, s.offsets, R, L->W1, L->W3, E, d, dff, s.H, stream);
+  if (rc) return rc;
+  rc = down_launch(s.H, s.offsets, R, L->W2, E, d, dff, s.Y_perm, stream);
+  if (rc) return rc;
+  return ordermoe_combine_residual_norm(s.Y_perm, s.row_of, s.topk_w, h, T, k, d, eps, h_out,
+                                        x_out, stream);
+}
+
 extern "C" int ordermoe_layer_forward(const ordermoe_layer_desc* L, int T, const uint16_t* X,
                                       const uint8_t* home, uint8_t* loc, float* qhat, uint16_t* y,
                                       int32_t* counters, int host_io, ordermoe_stream_t stream) {
   OM_TRACE();
-  if (!L) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: null layer");
-  if (T < 0 || T > L->T_max) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: need 0 <= T <= T_max");
-  if (!L->W_r || !L->W1 || !L->W3 || !L->W2 || !L->tables || !L->scratch)
-    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: null pointer in the layer");
-  if ((reinterpret_cast<uintptr_t>(L->scratch) & 255u) != 0)
-    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: scratch must be 256-byte aligned");
-  const size_t need = ordermoe_layer_scratch_bytes(L->T_max, L->E, L->d, L->dff, L->k);
-  if (need == 0 || L->scratch_bytes < need)
-    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: scratch too small or bad shape");
-  if (L->d % 256 != 0 || L->dff % 128 != 0 || L->k > L->E)
-    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "layer_forward: need d %% 256 == 0, dff %% 128 == 0, k <= E");
-  if (!aligned16(L->W_r) || !aligned16(L->W1) || !aligned16(L->W3) || !aligned16(L->W2))
-    return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: weights must be 16-byte aligned");
+  int rc0 = check_layer(L, T, "layer_forward");
+  if (rc0) return rc0;
   if (T == 0) return ORDERMOE_OK;
   if (!X || !home || !y) return fail(ORDERMOE_ERR_INVALID_ARG, "layer_forward: null X/home/y");
   if ((loc == nullptr) != (qhat == nullptr))

@@ -183,8 +183,10 @@ __device__ __forceinline__ unsigned long long topk_set(const float* __restrict__
 // each token adds one to n_l(k -> k') for every k in its top-kf at layer l
 // and k' in its top-kf at layer l + 1 (integer atomics: order-independent).
 template <int EMAX>
+// logits of token n at layer l start at n * sn + l * sl (floats).
 __global__ void __launch_bounds__(256) transitions_kernel(const float* __restrict__ logits,
                                                           int64_t N, int L, int E, int kf,
+                                                          int64_t sn, int64_t sl,
                                                           int32_t* __restrict__ counts) {
   __shared__ int h[64 * 64];
   const int l = blockIdx.y;
@@ -192,8 +194,8 @@ __global__ void __launch_bounds__(256) transitions_kernel(const float* __restric
   __syncthreads();
   for (int64_t n = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; n < N;
        n += (int64_t)gridDim.x * blockDim.x) {
-    unsigned long long a = topk_set<EMAX>(logits + ((size_t)n * L + l) * E, E, kf);
-    const unsigned long long b = topk_set<EMAX>(logits + ((size_t)n * L + l + 1) * E, E, kf);
+    unsigned long long a = topk_set<EMAX>(logits + n * sn + l * sl, E, kf);
+    const unsigned long long b = topk_set<EMAX>(logits + n * sn + (l + 1) * sl, E, kf);
     while (a) {
       const int x = __ffsll(static_cast<long long>(a)) - 1;
       a &= a - 1;
@@ -1034,28 +1036,45 @@ extern "C" int ordermoe_place(const float* sim, const int32_t* counts, int L, in
   return ORDERMOE_OK;
 }
 
-extern "C" int ordermoe_transitions(const float* logits, int64_t N, int L, int E, int k_freq,
-                                    int32_t* counts, float* P, ordermoe_stream_t stream) {
-  OM_TRACE();
+static int transitions_launch(const char* who, const float* logits, int64_t N, int L, int E,
+                              int k_freq, int64_t sn, int64_t sl, int32_t* counts, float* P,
+                              cudaStream_t stream) {
   if (L < 2 || E <= 0 || E > ORDERMOE_MAX_EXPERTS || k_freq <= 0 || k_freq > E || N < 0)
-    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "transitions: need L >= 2, 1 <= k_freq <= E <= 64");
-  if (!counts || !P || (N > 0 && !logits)) return fail(ORDERMOE_ERR_INVALID_ARG, "transitions: null pointer");
+    return fail(ORDERMOE_ERR_UNSUPPORTED_SHAPE, "%s: need L >= 2, 1 <= k_freq <= E <= 64", who);
+  if (!counts || !P || (N > 0 && !logits)) return fail(ORDERMOE_ERR_INVALID_ARG, "%s: null pointer", who);
   OM_CUDA(cudaMemsetAsync(counts, 0, sizeof(int32_t) * (size_t)(L - 1) * E * E, stream));
   if (N > 0) {
     int64_t blocks = (N + 255) / 256;
     const int64_t cap = (num_sms() * 4 + L - 2) / (L - 1);
     if (blocks > cap) blocks = cap;
     const dim3 grid(static_cast<unsigned>(blocks), L - 1);
-    if (E <= 8) transitions_kernel<8><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
-    else if (E <= 16) transitions_kernel<16><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
-    else if (E <= 32) transitions_kernel<32><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
-    else transitions_kernel<64><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, counts);
+    if (E <= 8) transitions_kernel<8><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, sn, sl, counts);
+    else if (E <= 16) transitions_kernel<16><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, sn, sl, counts);
+    else if (E <= 32) transitions_kernel<32><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, sn, sl, counts);
+    else transitions_kernel<64><<<grid, 256, 0, stream>>>(logits, N, L, E, k_freq, sn, sl, counts);
     OM_LAUNCHED("transitions_kernel");
   }
   const int rows = (L - 1) * E;
   transitions_finish_kernel<<<(rows + 127) / 128, 128, 0, stream>>>(counts, rows, E, P);
   OM_LAUNCHED("transitions_finish_kernel");
   return ORDERMOE_OK;
+}
+
+extern "C" int ordermoe_transitions(const float* logits, int64_t N, int L, int E, int k_freq,
+                                    int32_t* counts, float* P, ordermoe_stream_t stream) {
+  OM_TRACE();
+  return transitions_launch("transitions", logits, N, L, E, k_freq, (int64_t)L * E, E, counts, P,
+                            stream);
+}
+
+extern "C" int ordermoe_transitions_strided(const float* logits, int64_t N, int L, int E,
+                                            int k_freq, int64_t token_stride, int64_t layer_stride,
+                                            int32_t* counts, float* P, ordermoe_stream_t stream) {
+  OM_TRACE();
+  if (token_stride < E || layer_stride < E)
+    return fail(ORDERMOE_ERR_INVALID_ARG, "transitions_strided: strides must be >= E");
+  return transitions_launch("transitions_strided", logits, N, L, E, k_freq, token_stride,
+                            layer_stride, counts, P, stream);
 }
 
 extern "C" int ordermoe_replicate(const int32_t* group, const double* importance, const double* p,

@@ -71,3 +71,36 @@ def assert_close_combined(got_bits, ref_bits, w, Yref_bits, rtol=2e-2, atol=1e-2
         raise AssertionError("%s: %d / %d elements outside the combine bound; first %s: got %s ref %s"
                              % (what, bad.sum(), bad.size, i.tolist(), g[tuple(i.T)].tolist(),
                                 r[tuple(i.T)].tolist()))
+
+
+def check_layer_integers_full(logits, gpu, o_tab, home, loc_in, qhat_in, k, E, X_bits=None,
+                              renorm=1, what=""):
+    """Bit-exact parity of every integer decision of one layer over ALL its
+    tokens, near ties included: the oracle's top-k (Alg. 2's target), the
+    selection of Eqs. 40, 43, 44 and the permutation are run on the GPU's own
+    fp32 router logits, so both sides decide from the same numbers.
+
+    gpu: dict of host arrays from the GPU (idx, w, chosen, server, kind, loc,
+    qhat, and optionally offsets, row_token, row_of, X_perm bits).
+    Returns the oracle's (idx, w, chosen) for reuse."""
+    logits = np.ascontiguousarray(logits, np.float32)
+    idx, w = oracle.topk(logits, k, renorm)
+    np.testing.assert_array_equal(gpu["idx"], idx, err_msg=what + " top-k idx")
+    np.testing.assert_allclose(gpu["w"], w, rtol=1e-5, atol=1e-7, err_msg=what + " gate weights")
+    chosen, server, kind, loc2, q2 = oracle.select(idx, o_tab, np.asarray(home, np.uint8),
+                                                   np.array(loc_in, np.uint8, copy=True),
+                                                   np.array(qhat_in, np.float32, copy=True))
+    for name, ref in (("chosen", chosen), ("server", server), ("kind", kind), ("loc", loc2)):
+        np.testing.assert_array_equal(gpu[name], ref, err_msg="%s %s" % (what, name))
+    # the accumulated loss compared as bits (Eq. 44's fp32 adds in slot order)
+    np.testing.assert_array_equal(np.asarray(gpu["qhat"], np.float32).view(np.uint32),
+                                  q2.view(np.uint32), err_msg=what + " qhat")
+    if "offsets" in gpu:
+        off, rt, row_of = oracle.dispatch(chosen.astype(np.int32), E)
+        np.testing.assert_array_equal(gpu["offsets"], off, err_msg=what + " offsets")
+        np.testing.assert_array_equal(gpu["row_token"], rt, err_msg=what + " row_token")
+        np.testing.assert_array_equal(gpu["row_of"], row_of, err_msg=what + " row_of")
+        if X_bits is not None and "X_perm" in gpu:
+            np.testing.assert_array_equal(gpu["X_perm"], oracle.gather_rows(X_bits, rt),
+                                          err_msg=what + " X_perm")
+    return idx, w, chosen

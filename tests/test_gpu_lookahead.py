@@ -300,3 +300,68 @@ def test_layer_stack_graph_replay_equals_eager_step():
         outs.append([loc.clone(), qhat.clone()] + [y.clone() for y in ys])
     for a, b in zip(*outs):
         assert torch.equal(a, b)
+
+
+def test_residual_stack_lookahead_teacher_forced():
+    """Six small layers on the residual map (each layer reads RMSNorm of the
+    residual stream) through ordermoe_layer_forward_residual with H = 3: with
+    the oracle fed each layer's recorded router logits (teacher forcing), the
+    look-ahead selection carries the same location and accumulated loss for
+    every token, bit for bit, near ties included; the recorded logits match
+    the oracle's on the GPU's layer inputs; a CUDA-graph replay of the step
+    gives the eager step's results bit for bit."""
+    from paper_2607_17154_gb300.layer import LayerStack
+    rng = np.random.default_rng(46)
+    L, T, E, k, M, d, dff, H = 6, 300, 8, 2, 4, 256, 512, 3
+    buf, stride, otabs = stack_tables(rng, L, E, M, 0.3, cheap_links=True)
+    P = rng.random((L - 1, E, E)).astype(np.float32)
+    P[P < 0.5] = 0
+    P = (P / np.maximum(P.sum(axis=2, keepdims=True), 1e-9)).astype(np.float32)
+    layers, Wrb = [], []
+    for l in range(L):
+        Wr = synth.router_weights(E, d, 2, seed=270 + l, device=DEV)
+        W1, W3, W2 = synth.ffn_weights(E, d, dff, seed=280 + l, device=DEV)
+        layers.append({"W_r": Wr, "W1": W1, "W3": W3, "W2": W2})
+        Wrb.append(synth.bits(Wr))
+    stack = LayerStack(layers, buf, k, T, DEV, H=H, stride=stride, P=torch.as_tensor(P).to(DEV))
+    home_np = rng.integers(0, M, T).astype(np.uint8)
+    home = torch.as_tensor(home_np).to(DEV)
+    h0 = synth.hidden(T, d, 290, device=DEV)
+    outs = []
+    for mode in ("eager", "graph"):
+        hs = [h0] + [torch.zeros_like(h0) for _ in range(L)]
+        xs = [torch.zeros_like(h0) for _ in range(L + 1)]
+        loc, qhat = home.clone(), torch.zeros(T, device=DEV)
+        logits = torch.zeros(L, T, E, device=DEV)
+
+        def reset():
+            loc.copy_(home)
+            qhat.zero_()
+        if mode == "eager":
+            counters = torch.zeros(4, dtype=torch.int32, device=DEV)
+            reset()
+            stack.step_residual(hs, xs, home, loc, qhat, counters=counters, logits=logits)
+            torch.cuda.synchronize()
+            assert counters.sum().item() == L * T * k
+            lg = logits.cpu().numpy()
+            o_loc, o_q = home_np.copy(), np.zeros(T, np.float32)
+            for l in range(L):
+                np.testing.assert_allclose(lg[l], oracle.router_logits(synth.bits(xs[l]), Wrb[l]),
+                                           rtol=1e-3, atol=2e-3)
+                idx, _ = oracle.topk(lg[l], k)
+                Hl = min(H, L - l)
+                _, _, _, o_loc, o_q = oracle.select_lookahead(idx, otabs[l:l + Hl], P[l:l + Hl - 1],
+                                                              home_np, o_loc, o_q)
+            np.testing.assert_array_equal(loc.cpu().numpy(), o_loc)
+            np.testing.assert_array_equal(qhat.cpu().numpy().view(np.uint32), o_q.view(np.uint32))
+            assert torch.isfinite(hs[-1].float()).all()
+        else:
+            g = stack.capture_residual(hs, xs, home, loc, qhat, prologue=reset)
+            for t in hs[1:] + xs:
+                t.zero_()
+            loc.fill_(0)
+            g.replay()
+            torch.cuda.synchronize()
+        outs.append([loc.clone(), qhat.clone()] + [t.clone() for t in hs[1:] + xs])
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)

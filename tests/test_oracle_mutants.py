@@ -42,6 +42,12 @@ MUTANTS = [
     ("FFN: W2 transposed", "W2 + ((int64_t)e * d + o) * dff", "W2 + (int64_t)e * d * dff + o"),
     ("combine: weights dropped", "acc += static_cast<double>(w[(int64_t)t * k + j]) * bf(Yp, row * d + c);",
      "acc += bf(Yp, row * d + c);"),
+    ("RMSNorm: sum of squares not divided by d", "std::sqrt(ss / d + eps)", "std::sqrt(ss + eps)"),
+    ("RMSNorm: square root dropped", "std::sqrt(ss / d + eps)", "(ss / d + eps)"),
+    ("residual combine: residual dropped", "double acc = bf(h, (int64_t)t * d + c);", "double acc = 0.0;"),
+    ("residual combine: weights dropped",
+     "acc += static_cast<double>(w[(int64_t)t * k + j]) * bf(Yp, row * d + c);\n      }\n      h_out",
+     "acc += bf(Yp, row * d + c);\n      }\n      h_out"),
     ("Eq. 4: not normalised", "dot / (norm[i] * norm[j])", "dot"),
     ("Eq. 24: threshold inclusive", "best_s < theta", "best_s <= theta"),
     ("Eq. 25: argmax ties to the later dominant", "if (best_g < 0 || s > best_s)", "if (best_g < 0 || s >= best_s)"),

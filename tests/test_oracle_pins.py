@@ -457,6 +457,59 @@ def test_combine_special_cases(orc):
 
 
 # --------------------------------------------------------------------------
+# Residual map between stacked layers: RMSNorm and the residual add
+
+def test_rmsnorm_closed_forms(orc):
+    d = 16
+    h = np.zeros((4, d), np.float32)
+    h[0] = 1.0                           # mean square 1: x = 1/sqrt(1 + eps) -> 1.0 in bf16
+    h[1] = -3.0                          # mean square 9: -3/3 = -1
+    h[2, :8] = 2.0                       # mean square 2: 2/sqrt(2) = sqrt(2)
+    h[3, 0] = 4.0                        # one non-zero: 4/sqrt(16/16) = 4, rest 0
+    x = bits_to_f(orc.rmsnorm(bf16_bits(h), eps=1e-6))
+    np.testing.assert_array_equal(x[0], np.ones(d, np.float32))
+    np.testing.assert_array_equal(x[1], -np.ones(d, np.float32))
+    np.testing.assert_array_equal(x[2], np.r_[np.full(8, bits_to_f(bf16_bits([np.sqrt(2.0)]))[0]),
+                                              np.zeros(8)].astype(np.float32))
+    np.testing.assert_array_equal(x[3], np.r_[[4.0], np.zeros(d - 1)].astype(np.float32))
+
+
+def test_rmsnorm_scale_invariant_and_unit_rms(orc):
+    rng = np.random.default_rng(41)
+    h = rnd_bf16(rng, (7, 40), std=3.0)
+    x = orc.rmsnorm(h, eps=1e-30)
+    # a power-of-two scaling of h changes nothing (exact in binary, eps negligible)
+    np.testing.assert_array_equal(orc.rmsnorm(bf16_bits(bits_to_f(h) * 8.0), eps=1e-30), x)
+    np.testing.assert_array_equal(orc.rmsnorm(bf16_bits(bits_to_f(h) * -0.25), eps=1e-30),
+                                  bf16_bits(-bits_to_f(x)))
+    # every row has unit root mean square up to the bf16 rounding of x
+    ms = (bits_to_f(x).astype(np.float64) ** 2).mean(axis=1)
+    np.testing.assert_allclose(ms, 1.0, rtol=2 * 2.0 ** -8)
+
+
+def test_combine_residual_special_cases(orc):
+    rng = np.random.default_rng(42)
+    T, k, d = 5, 3, 12
+    Y = rnd_bf16(rng, (T * k, d))
+    rof = rng.permutation(T * k).astype(np.int32).reshape(T, k)
+    w = rng.random((T, k)).astype(np.float32)
+    h = rnd_bf16(rng, (T, d))
+    # zero weights: the residual stream passes through unchanged
+    np.testing.assert_array_equal(orc.combine_residual(Y, rof, np.zeros((T, k), np.float32), h), h)
+    # a zero residual stream: the plain weighted combine
+    np.testing.assert_array_equal(orc.combine_residual(Y, rof, w, np.zeros_like(h)),
+                                  orc.combine(Y, rof, w))
+    # small integers and dyadic weights: every sum is exact
+    Yi = bf16_bits(rng.integers(-8, 8, (T * k, d)).astype(np.float32))
+    hi = bf16_bits(rng.integers(-16, 16, (T, d)).astype(np.float32))
+    wd = np.tile(np.array([0.5, 0.25, 0.125], np.float32), (T, 1))
+    got = bits_to_f(orc.combine_residual(Yi, rof, wd, hi))
+    Yf = bits_to_f(Yi)
+    ref = bits_to_f(hi) + sum(wd[:, j:j + 1] * Yf[rof[:, j]] for j in range(k))
+    np.testing.assert_array_equal(got, ref)
+
+
+# --------------------------------------------------------------------------
 # Similarity (Eqs. 3-4) and activation counts (Eq. 5)
 
 def test_similarity_identity_calibration_is_cosine_of_router_rows(orc):
