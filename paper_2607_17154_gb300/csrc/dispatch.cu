@@ -407,6 +407,7 @@ __global__ void __launch_bounds__(1024) dispatch_small_kernel(
       for (int w = 0; w < 32; ++w) c += wc[w][tid];
       start[tid] += c;
     }
+    __syncthreads();  // wc is read above before the next round clears it
   }
 }
 

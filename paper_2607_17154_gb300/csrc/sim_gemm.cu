@@ -171,6 +171,81 @@ __device__ __forceinline__ void count_topk_net(const float (&x)[E], int kf, int*
   }
 }
 
+// The top-k_freq set of 64 logits as a bit mask (experts 0-31 in lo, 32-63
+// in hi), by the rules of count_topk_net (k_freq <= K) or count_topk.
+template <int K>
+__device__ __forceinline__ void topk_mask64_net(const float (&x)[64], int kf, uint32_t& lo,
+                                                uint32_t& hi) {
+  float v[K];
+#pragma unroll
+  for (int i = 0; i < K; ++i) v[i] = -INFINITY;
+#pragma unroll
+  for (int e = 0; e < 64; ++e) {
+    const float c = x[e];
+#pragma unroll
+    for (int i = K - 1; i > 0; --i) v[i] = fminf(v[i - 1], fmaxf(v[i], c));
+    v[0] = fmaxf(v[0], c);
+  }
+  float T = v[0];
+#pragma unroll
+  for (int i = 1; i < K; ++i) T = (i == kf - 1) ? v[i] : T;
+  const float Tc = fmaxf(T, -3.402823466e38f);
+  lo = 0u;
+  hi = 0u;
+  int n = 0;
+#pragma unroll
+  for (int e = 0; e < 64; ++e) {
+    const bool take = x[e] >= Tc;
+    n += take ? 1 : 0;
+    if (e < 32) lo |= take ? (1u << e) : 0u;
+    else hi |= take ? (1u << (e - 32)) : 0u;
+  }
+  if (n > kf) {
+    int extra = n - kf;
+#pragma unroll
+    for (int e = 63; e >= 0; --e) {
+      const bool back = extra > 0 && x[e] == T;
+      extra -= back ? 1 : 0;
+      if (e < 32) lo &= back ? ~(1u << e) : ~0u;
+      else hi &= back ? ~(1u << (e - 32)) : ~0u;
+    }
+  }
+}
+
+__device__ __forceinline__ void topk_mask64_passes(const float (&x)[64], int kf, uint32_t& lo,
+                                                   uint32_t& hi) {
+  unsigned long long used = 0;
+  for (int j = 0; j < kf; ++j) {
+    int best = -1;
+    float bv = -INFINITY;
+#pragma unroll
+    for (int e = 0; e < 64; ++e) {
+      const bool take = !(used & (1ull << e)) && x[e] > bv;
+      best = take ? e : best;
+      bv = take ? x[e] : bv;
+    }
+    if (best < 0) break;
+    used |= 1ull << best;
+  }
+  lo = static_cast<uint32_t>(used);
+  hi = static_cast<uint32_t>(used >> 32);
+}
+
+// 32 x 32 bit transpose across a warp: lane r holds row r (bit c = entry
+// (r, c)); afterwards lane c holds column c (bit r = entry (r, c)). Each step
+// swaps the off-diagonal s x s blocks of every 2s x 2s block between lanes r
+// and r ^ s.
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, int lane) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) {
+    const uint32_t keep = s == 16 ? 0x0000FFFFu : s == 8 ? 0x00FF00FFu : s == 4 ? 0x0F0F0F0Fu
+                          : s == 2 ? 0x33333333u : 0x55555555u;  // columns with bit s clear
+    const uint32_t y = __shfl_xor_sync(0xffffffffu, x, s);
+    x = (lane & s) ? ((x & ~keep) | ((y & ~keep) >> s)) : ((x & keep) | ((y & keep) << s));
+  }
+  return x;
+}
+
 template <int E>
 __global__ void __launch_bounds__(L_THREADS, 1)
     sim_logits_kernel(const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapW,
@@ -338,39 +413,49 @@ __global__ void __launch_bounds__(L_THREADS, 1)
             }
           }
         }
-        if (valid) {
+        if (valid && args.H != nullptr) {  // logits kept only when asked for
           float4* dst = reinterpret_cast<float4*>(orow + cb);
 #pragma unroll
           for (int i = 0; i < 8; ++i)
-            if (args.H != nullptr && 4 * i < nv)  // logits kept only when asked for
+            if (4 * i < nv)
               dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
                                    __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
-          if (E == 64) {
-            if ((c & 1) == 0) {
+        }
+        if (E == 64) {
+          // Eq. 5 for one layer and the warp's 32 tokens: each lane's top-k
+          // set as a 64-bit mask, the masks transposed across the warp, and
+          // lane j adds the number of tokens that select expert j (and
+          // j + 32): two conflict-free shared-memory adds per lane
+          if ((c & 1) == 0) {
 #pragma unroll
-              for (int i = 0; i < 32; ++i) prev[i] = __uint_as_float(v[i]);
-            } else {
+            for (int i = 0; i < 32; ++i) prev[i] = __uint_as_float(v[i]);
+          } else {
+            uint32_t mlo = 0u, mhi = 0u;
+            if (valid) {
               float x[64];
 #pragma unroll
               for (int i = 0; i < 32; ++i) {
                 x[i] = prev[i];
                 x[32 + i] = __uint_as_float(v[i]);
               }
-              const int l = (cb - 32) / 64;
-              float(&xr)[64] = reinterpret_cast<float(&)[64]>(x);
-              if (args.kf <= 6) count_topk_net<64, 6>(xr, args.kf, hist + l * 64);
-              else if (args.kf <= 8) count_topk_net<64, 8>(xr, args.kf, hist + l * 64);
-              else count_topk<64>(xr, args.kf, hist + l * 64);
+              if (args.kf <= 6) topk_mask64_net<6>(x, args.kf, mlo, mhi);
+              else if (args.kf <= 8) topk_mask64_net<8>(x, args.kf, mlo, mhi);
+              else topk_mask64_passes(x, args.kf, mlo, mhi);
             }
-          } else {
+            const int l = (cb - 32) / 64;
+            const int nlo = __popc(warp_transpose32(mlo, lane));
+            const int nhi = __popc(warp_transpose32(mhi, lane));
+            if (nlo) atomicAdd(&hist[l * 64 + lane], nlo);
+            if (nhi) atomicAdd(&hist[l * 64 + 32 + lane], nhi);
+          }
+        } else if (valid) {
 #pragma unroll
-            for (int sub = 0; sub < 32 / E; ++sub) {
-              float x[E];
+          for (int sub = 0; sub < 32 / E; ++sub) {
+            float x[E];
 #pragma unroll
-              for (int i = 0; i < E; ++i) x[i] = __uint_as_float(v[sub * E + i]);
-              const int l = (cb + sub * E) / E;
-              if (l < args.L) count_topk<E>(x, args.kf, hist + l * E);
-            }
+            for (int i = 0; i < E; ++i) x[i] = __uint_as_float(v[sub * E + i]);
+            const int l = (cb + sub * E) / E;
+            if (l < args.L) count_topk<E>(x, args.kf, hist + l * E);
           }
         }
       }

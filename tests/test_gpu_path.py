@@ -156,6 +156,9 @@ def test_router_logits_match_oracle(T, d, E):
 # ------------------------------------------------------------------ permutation
 
 @pytest.mark.parametrize("T,k,E,d", [(64, 2, 8, 256), (1000, 6, 64, 64), (1, 1, 1, 8), (333, 3, 7, 40),
+                                     # one block ranking several rounds of 1024 entries, up to
+                                     # its limit of 4096, and the first size past it
+                                     (1500, 2, 8, 64), (2048, 2, 8, 16), (683, 6, 64, 8),
                                      (4096, 2, 8, 4096),
                                      (8192, 6, 64, 64),     # 192 chunks: histogram staged in shared memory
                                      (20000, 6, 64, 64)])   # 469 chunks x 64: too large to stage
