@@ -128,90 +128,8 @@ __device__ __forceinline__ void count_topk(const float (&x)[E], int kf, int* his
   }
 }
 
-// The same counts for k_freq <= K with fewer compare/select operations: a
-// descending min/max insertion network keeps the K largest logits with
-// multiplicity, T = the k_freq-th of them, and every logit >= T is counted;
-// when more than k_freq logits reach T (equal logits at the boundary), the
-// surplus logits equal to T are taken back from the highest index down, which
-// leaves the lowest indices, as the rank order says. Inserting c into the
-// descending v keeps min(v[i-1], max(v[i], c)) in slot i, which leaves v as it
-// was for a NaN c (min/max return the other operand), and -inf logits are
-// never counted, as in the passes above.
-template <int E, int K>
-__device__ __forceinline__ void count_topk_net(const float (&x)[E], int kf, int* hist_row) {
-  float v[K];
-#pragma unroll
-  for (int i = 0; i < K; ++i) v[i] = -INFINITY;
-#pragma unroll
-  for (int e = 0; e < E; ++e) {
-    const float c = x[e];
-#pragma unroll
-    for (int i = K - 1; i > 0; --i) v[i] = fminf(v[i - 1], fmaxf(v[i], c));
-    v[0] = fmaxf(v[0], c);
-  }
-  float T = v[0];
-#pragma unroll
-  for (int i = 1; i < K; ++i) T = (i == kf - 1) ? v[i] : T;
-  const float Tc = fmaxf(T, -3.402823466e38f);  // below every finite logit, above -inf
-  int n = 0;
-#pragma unroll
-  for (int e = 0; e < E; ++e) {
-    const bool take = x[e] >= Tc;
-    n += take ? 1 : 0;
-    if (take) atomicAdd(&hist_row[e], 1);
-  }
-  if (n > kf) {
-    int extra = n - kf;
-#pragma unroll
-    for (int e = E - 1; e >= 0; --e) {
-      const bool back = extra > 0 && x[e] == T;
-      extra -= back ? 1 : 0;
-      if (back) atomicSub(&hist_row[e], 1);
-    }
-  }
-}
-
 // The top-k_freq set of 64 logits as a bit mask (experts 0-31 in lo, 32-63
-// in hi), by the rules of count_topk_net (k_freq <= K) or count_topk.
-template <int K>
-__device__ __forceinline__ void topk_mask64_net(const float (&x)[64], int kf, uint32_t& lo,
-                                                uint32_t& hi) {
-  float v[K];
-#pragma unroll
-  for (int i = 0; i < K; ++i) v[i] = -INFINITY;
-#pragma unroll
-  for (int e = 0; e < 64; ++e) {
-    const float c = x[e];
-#pragma unroll
-    for (int i = K - 1; i > 0; --i) v[i] = fminf(v[i - 1], fmaxf(v[i], c));
-    v[0] = fmaxf(v[0], c);
-  }
-  float T = v[0];
-#pragma unroll
-  for (int i = 1; i < K; ++i) T = (i == kf - 1) ? v[i] : T;
-  const float Tc = fmaxf(T, -3.402823466e38f);
-  lo = 0u;
-  hi = 0u;
-  int n = 0;
-#pragma unroll
-  for (int e = 0; e < 64; ++e) {
-    const bool take = x[e] >= Tc;
-    n += take ? 1 : 0;
-    if (e < 32) lo |= take ? (1u << e) : 0u;
-    else hi |= take ? (1u << (e - 32)) : 0u;
-  }
-  if (n > kf) {
-    int extra = n - kf;
-#pragma unroll
-    for (int e = 63; e >= 0; --e) {
-      const bool back = extra > 0 && x[e] == T;
-      extra -= back ? 1 : 0;
-      if (e < 32) lo &= back ? ~(1u << e) : ~0u;
-      else hi &= back ? ~(1u << (e - 32)) : ~0u;
-    }
-  }
-}
-
+// in hi), by the rules of count_topk.
 __device__ __forceinline__ void topk_mask64_passes(const float (&x)[64], int kf, uint32_t& lo,
                                                    uint32_t& hi) {
   unsigned long long used = 0;
@@ -246,7 +164,10 @@ __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, int lane) {
   return x;
 }
 
-template <int E>
+// NK: 6 or 8 = Eq. 5's counts of 64-expert layers with a network keeping the
+// NK largest logits (k_freq <= NK), streamed over the two 32-logit halves of
+// a layer; 0 = the selection passes over all 64 (k_freq > 8) or E < 64.
+template <int E, int NK>
 __global__ void __launch_bounds__(L_THREADS, 1)
     sim_logits_kernel(const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapW,
                       LArgs args) {
@@ -375,9 +296,11 @@ __global__ void __launch_bounds__(L_THREADS, 1)
       const bool valid = row < args.N;
       const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
       float* orow = args.H + (size_t)row * args.C;
-      float prev[32];  // E == 64: the first half of a layer's logits
-#pragma unroll 1
-      for (int c = 2 * part; c < 2 * part + 2; ++c) {
+      float prev[32];  // E == 64, NK == 0: the first half of a layer's logits
+      float net[NK > 0 ? NK : 1];  // E == 64, NK > 0: the NK largest logits so far, descending
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {  // the two 32-column chunks of the warp's part
+        const int c = 2 * part + half;
         const int cb = n * BN + c * 32;
         if (cb >= args.C) break;  // warp-uniform
         uint32_t v[32];
@@ -421,11 +344,68 @@ __global__ void __launch_bounds__(L_THREADS, 1)
               dst[i] = make_float4(__uint_as_float(v[4 * i]), __uint_as_float(v[4 * i + 1]),
                                    __uint_as_float(v[4 * i + 2]), __uint_as_float(v[4 * i + 3]));
         }
-        if (E == 64) {
-          // Eq. 5 for one layer and the warp's 32 tokens: each lane's top-k
-          // set as a 64-bit mask, the masks transposed across the warp, and
-          // lane j adds the number of tokens that select expert j (and
-          // j + 32): two conflict-free shared-memory adds per lane
+        if (E == 64 && NK > 0) {
+          // Eq. 5 for one layer and the warp's 32 tokens with fewer
+          // compare/select operations than the passes: a descending min/max
+          // insertion network keeps the NK largest logits with multiplicity
+          // (min(v[j-1], max(v[j], x)) in slot j leaves v as it was for a NaN
+          // x), T = the k_freq-th of them, and every logit >= T is selected;
+          // when more than k_freq logits reach T (equal logits at the
+          // boundary), the surplus equal to T is taken back from the highest
+          // index down, which leaves the lowest indices, as the rank order
+          // says; -inf logits are never selected, as in the passes. The
+          // network takes the layer's first 32 logits (each lane's token),
+          // then the next 32; with T known the first half is read from TMEM
+          // again for its mask. Each lane's top-k set becomes a 64-bit mask,
+          // the masks are transposed across the warp, and lane j adds the
+          // number of tokens that select expert j (and j + 32): two
+          // conflict-free shared-memory adds per lane.
+          if (half == 0) {
+#pragma unroll
+            for (int i = 0; i < NK; ++i) net[i] = -INFINITY;
+          }
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float x = __uint_as_float(v[i]);
+#pragma unroll
+            for (int j = NK - 1; j > 0; --j) net[j] = fminf(net[j - 1], fmaxf(net[j], x));
+            net[0] = fmaxf(net[0], x);
+          }
+          if (half == 1) {
+            // T = net[kf - 1], the smallest of the first kf (net is descending),
+            // written as a running minimum so that net stays in registers
+            float T = net[0];
+#pragma unroll
+            for (int j = 1; j < NK; ++j) T = j < args.kf ? fminf(T, net[j]) : T;
+            const float Tc = fmaxf(T, -3.402823466e38f);  // below every finite logit, above -inf
+            uint32_t mhi = 0u, ehi = 0u, mlo = 0u, elo = 0u;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float x = __uint_as_float(v[i]);
+              mhi |= x >= Tc ? (1u << i) : 0u;
+              ehi |= x == T ? (1u << i) : 0u;
+            }
+            tmem_ld32(tb + (c - 1) * 32, v);  // the first half again
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float x = __uint_as_float(v[i]);
+              mlo |= x >= Tc ? (1u << i) : 0u;
+              elo |= x == T ? (1u << i) : 0u;
+            }
+            unsigned long long sel = valid ? ((static_cast<unsigned long long>(mhi) << 32) | mlo) : 0ull;
+            const unsigned long long eq = (static_cast<unsigned long long>(ehi) << 32) | elo;
+            // equal logits straddling the boundary: take back the surplus from the highest index
+            for (int extra = __popcll(sel) - args.kf; extra > 0 && (sel & eq) != 0ull; --extra)
+              sel &= ~(1ull << (63 - __clzll(sel & eq)));
+            const int l = (cb - 32) / 64;
+            const int nlo = __popc(warp_transpose32(static_cast<uint32_t>(sel), lane));
+            const int nhi = __popc(warp_transpose32(static_cast<uint32_t>(sel >> 32), lane));
+            if (nlo) atomicAdd(&hist[l * 64 + lane], nlo);
+            if (nhi) atomicAdd(&hist[l * 64 + 32 + lane], nhi);
+          }
+        } else if (E == 64) {
+          // k_freq > 8: the selection passes over the layer's 64 logits
           if ((c & 1) == 0) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) prev[i] = __uint_as_float(v[i]);
@@ -438,9 +418,7 @@ __global__ void __launch_bounds__(L_THREADS, 1)
                 x[i] = prev[i];
                 x[32 + i] = __uint_as_float(v[i]);
               }
-              if (args.kf <= 6) topk_mask64_net<6>(x, args.kf, mlo, mhi);
-              else if (args.kf <= 8) topk_mask64_net<8>(x, args.kf, mlo, mhi);
-              else topk_mask64_passes(x, args.kf, mlo, mhi);
+              topk_mask64_passes(x, args.kf, mlo, mhi);
             }
             const int l = (cb - 32) / 64;
             const int nlo = __popc(warp_transpose32(mlo, lane));
@@ -714,13 +692,17 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
     const int whole = whole_sm_smem();
     if (whole > lmax) lmax = whole;
     if (whole > gmax) gmax = whole;
-    cudaError_t e = cudaFuncSetAttribute(sim_logits_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    cudaError_t e = cudaFuncSetAttribute(sim_logits_kernel<8, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<16>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<16, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<32, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<64, 6>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(sim_logits_kernel<64, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(sim_logits_kernel<64, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, gmax);
     return static_cast<int>(e);
@@ -755,10 +737,14 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
   }
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);
   switch (E) {
-    case 8: sim_logits_kernel<8><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
-    case 16: sim_logits_kernel<16><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
-    case 32: sim_logits_kernel<32><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
-    default: sim_logits_kernel<64><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    case 8: sim_logits_kernel<8, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    case 16: sim_logits_kernel<16, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    case 32: sim_logits_kernel<32, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    default:
+      if (kf <= 6) sim_logits_kernel<64, 6><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la);
+      else if (kf <= 8) sim_logits_kernel<64, 8><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la);
+      else sim_logits_kernel<64, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la);
+      break;
   }
   OM_LAUNCHED("sim_logits_kernel");
   GArgs ga{};
