@@ -59,9 +59,19 @@ constexpr int G_STAGE_BYTES = 2 * BOX_BYTES;  // hi and lo tiles, 128 rows x 64 
 constexpr int G_TMEM_COLS = 128;
 constexpr uint32_t G_IDESC = idesc_bf16_f32(128, 128);
 
+// CTA-pair variant of the logits kernel: a pair computes 256 tokens x 256
+// columns with one cta_group::2 MMA (M = 256 across the pair, each CTA's
+// TMEM holding its 128 tokens); each CTA loads its 128 tokens and half of the
+// 256 weight rows per K step (32 KB instead of 48 KB: a third less L2 -> shared
+// memory traffic per flop), six stages deep.
+constexpr int P_STAGES = 6;
+constexpr int P_STAGE_BYTES = A_BYTES + BOX_BYTES;
+constexpr int L_MAX_STAGES = P_STAGES > STAGES ? P_STAGES : STAGES;
+static_assert(P_STAGES * P_STAGE_BYTES <= STAGES * STAGE_BYTES, "pair ring fits the 1-CTA ring's space");
+
 struct LSmem {
-  uint64_t full[STAGES];
-  uint64_t empty[STAGES];
+  uint64_t full[L_MAX_STAGES];
+  uint64_t empty[L_MAX_STAGES];
   uint64_t tfull[2];
   uint64_t tempty[2];
   uint64_t drain;
@@ -167,10 +177,14 @@ __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, int lane) {
 // NK: 6 or 8 = Eq. 5's counts of 64-expert layers with a network keeping the
 // NK largest logits (k_freq <= NK), streamed over the two 32-logit halves of
 // a layer; 0 = the selection passes over all 64 (k_freq > 8) or E < 64.
-template <int E, int NK>
+// PAIR: clusters of two CTAs with cta_group::2 MMAs (see P_STAGES).
+template <int E, int NK, bool PAIR>
 __global__ void __launch_bounds__(L_THREADS, 1)
     sim_logits_kernel(const __grid_constant__ CUtensorMap mapX, const __grid_constant__ CUtensorMap mapW,
                       LArgs args) {
+  constexpr int KSTAGES = PAIR ? P_STAGES : STAGES;
+  constexpr int KSTAGE_BYTES = PAIR ? P_STAGE_BYTES : STAGE_BYTES;
+  constexpr int TBM = PAIR ? 2 * BM : BM;  // tokens per tile
   extern __shared__ uint8_t smem_raw[];
   uint8_t* tiles = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -179,15 +193,19 @@ __global__ void __launch_bounds__(L_THREADS, 1)
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
+  const uint32_t rp = PAIR ? (cluster_ctarank() & 1u) : 0u;  // rank within the pair
+  const int cid = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+  const int ncl = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
   for (int i = tid; i < args.C; i += blockDim.x) hist[i] = 0;
   if (tid == 0) {
-    for (int i = 0; i < STAGES; ++i) {
+    for (int i = 0; i < KSTAGES; ++i) {
       mbar_init(&s.full[i], 1);
       mbar_init(&s.empty[i], 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&s.tfull[i], 1);
-      mbar_init(&s.tempty[i], 32 * L_EPI_WARPS);
+      // pair: one arrive per epilogue warp of either CTA, on the even CTA's barrier
+      mbar_init(&s.tempty[i], PAIR ? 2 * L_EPI_WARPS : 32 * L_EPI_WARPS);
     }
     mbar_init(&s.drain, 1);
     s.abort = 0;
@@ -199,14 +217,20 @@ __global__ void __launch_bounds__(L_THREADS, 1)
     tma_prefetch_map(&mapW);
   }
   if (warp == 1) {
-    tmem_alloc(&s.tmem_base, TMEM_COLS);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(&s.tmem_base, TMEM_COLS);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(&s.tmem_base, TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
-  __syncthreads();
+  if (PAIR) cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
+  else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = s.tmem_base;
-  const int total = ((args.N + BM - 1) / BM) * args.n_tiles;
+  const int total = ((args.N + TBM - 1) / TBM) * args.n_tiles;
   const int kblocks = args.K / BK;
   volatile int* abort = &s.abort;
   uint32_t issued_mask = 0, last_phase_bits = 0;
@@ -216,7 +240,7 @@ __global__ void __launch_bounds__(L_THREADS, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x) {
+      for (int tile = cid; tile < total && !*abort; tile += ncl) {
         const int mt = tile / args.n_tiles, n = tile - mt * args.n_tiles;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(&s.empty[stage], phase ^ 1u, args.limit_ns, abort)) {
@@ -224,23 +248,32 @@ __global__ void __launch_bounds__(L_THREADS, 1)
             *abort = 1;
             break;
           }
-          uint8_t* sa = tiles + stage * STAGE_BYTES;
-          mbar_arrive_expect_tx(&s.full[stage], STAGE_BYTES);
-          tma_load_2d(sa, &mapX, &s.full[stage], kb * BK, mt * BM);
-          tma_load_2d(sa + A_BYTES, &mapW, &s.full[stage], kb * BK, n * BN);
-          tma_load_2d(sa + A_BYTES + BOX_BYTES, &mapW, &s.full[stage], kb * BK, n * BN + 128);
+          uint8_t* sa = tiles + stage * KSTAGE_BYTES;
+          if (PAIR) {
+            // this CTA's 128 tokens and 128 of the tile's 256 weight rows; both
+            // CTAs' bytes complete on the even CTA's barrier
+            const uint32_t full_even = mapa_shared(smem_u32(&s.full[stage]), 0);
+            if (rp == 0) mbar_arrive_expect_tx(&s.full[stage], 2 * P_STAGE_BYTES);
+            tma_load_2d_pair(sa, &mapX, full_even, kb * BK, mt * TBM + static_cast<int>(rp) * BM);
+            tma_load_2d_pair(sa + A_BYTES, &mapW, full_even, kb * BK, n * BN + static_cast<int>(rp) * 128);
+          } else {
+            mbar_arrive_expect_tx(&s.full[stage], STAGE_BYTES);
+            tma_load_2d(sa, &mapX, &s.full[stage], kb * BK, mt * BM);
+            tma_load_2d(sa + A_BYTES, &mapW, &s.full[stage], kb * BK, n * BN);
+            tma_load_2d(sa + A_BYTES + BOX_BYTES, &mapW, &s.full[stage], kb * BK, n * BN + 128);
+          }
           issued_mask |= 1u << stage;
           last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
-          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+          if (++stage == KSTAGES) { stage = 0; phase ^= 1u; }
         }
       }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && rp == 0) {  // pair: the even CTA issues the pair's MMAs
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
-      for (int tile = blockIdx.x; tile < total && !*abort; tile += gridDim.x, ++it) {
+      for (int tile = cid; tile < total && !*abort; tile += ncl, ++it) {
         const int slot = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
         if (!mbar_wait(&s.tempty[slot], acc_phase ^ 1u, args.limit_ns, abort)) {
@@ -259,18 +292,29 @@ __global__ void __launch_bounds__(L_THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(tiles + stage * STAGE_BYTES);
+          const uint32_t a0 = smem_u32(tiles + stage * KSTAGE_BYTES);
           const uint32_t b0 = a0 + A_BYTES;
+          if (PAIR) {
+            constexpr uint32_t PIDESC = idesc_bf16_f32(256, BN);
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)
-            mma_bf16(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
-                     IDESC, (kb | kk) != 0 ? 1u : 0u);
-          mma_issued = true;
-          mma_commit(&s.empty[stage]);
-          if (++stage == STAGES) { stage = 0; phase ^= 1u; }
+            for (int kk = 0; kk < BK / 16; ++kk)
+              mma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32),
+                            sdesc_kmajor_sw128(b0 + kk * 32), PIDESC, (kb | kk) != 0 ? 1u : 0u);
+            mma_issued = true;
+            mma_commit_pair(&s.empty[stage], 0x3);
+          } else {
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              mma_bf16(d_tmem, sdesc_kmajor_sw128(a0 + kk * 32), sdesc_kmajor_sw128(b0 + kk * 32),
+                       IDESC, (kb | kk) != 0 ? 1u : 0u);
+            mma_issued = true;
+            mma_commit(&s.empty[stage]);
+          }
+          if (++stage == KSTAGES) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
-        mma_commit(&s.tfull[slot]);
+        if (PAIR) mma_commit_pair(&s.tfull[slot], 0x3);
+        else mma_commit(&s.tfull[slot]);
       }
     }
   } else {
@@ -280,7 +324,7 @@ __global__ void __launch_bounds__(L_THREADS, 1)
     const int part = (warp - 2) >> 2;
     const int lrow = q * 32 + lane;
     int it = 0;
-    for (int tile = blockIdx.x; tile < total; tile += gridDim.x, ++it) {
+    for (int tile = cid; tile < total; tile += ncl, ++it) {
       if (__any_sync(0xffffffffu, *abort != 0)) break;
       const int slot = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
@@ -292,7 +336,7 @@ __global__ void __launch_bounds__(L_THREADS, 1)
       }
       tc_fence_after();
       const int mt = tile / args.n_tiles, n = tile - mt * args.n_tiles;
-      const int row = mt * BM + lrow;
+      const int row = mt * TBM + static_cast<int>(rp) * BM + lrow;
       const bool valid = row < args.N;
       const uint32_t tb = tmem_base + slot * BN + (static_cast<uint32_t>(q * 32) << 16);
       float* orow = args.H + (size_t)row * args.C;
@@ -438,29 +482,43 @@ __global__ void __launch_bounds__(L_THREADS, 1)
         }
       }
       tc_fence_before();
-      mbar_arrive(&s.tempty[slot]);
+      if (PAIR) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&s.tempty[slot]), 0));
+      } else {
+        mbar_arrive(&s.tempty[slot]);
+      }
     }
   }
 
   __syncthreads();
   if (s.abort) {
+    // drain the copies (pair: all complete on the even CTA's barriers) and
+    // the MMAs in flight, both bounded
     volatile int* never = &s.zero;
-    if (warp == 0 && lane == 0) {
-      for (int st = 0; st < STAGES; ++st)
+    if (warp == 0 && lane == 0 && rp == 0) {
+      for (int st = 0; st < KSTAGES; ++st)
         if ((issued_mask >> st) & 1u)
           mbar_wait(&s.full[st], (last_phase_bits >> st) & 1u, args.limit_ns, never);
     }
-    if (warp == 1 && lane == 0 && mma_issued) {
-      mma_commit(&s.drain);
+    if (warp == 1 && lane == 0 && rp == 0 && mma_issued) {
+      if (PAIR) mma_commit_pair(&s.drain, 0x1);
+      else mma_commit(&s.drain);
       mbar_wait(&s.drain, 0, args.limit_ns, never);
     }
     __syncthreads();
+  }
+  if (PAIR) {
+    tc_fence_before();
+    cluster_sync();  // both CTAs done: no more arrivals or copies into either
+    tc_fence_after();
   }
   for (int i = tid; i < args.C; i += blockDim.x)
     if (hist[i]) atomicAdd(&args.counts[i], hist[i]);
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    if (PAIR) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -692,17 +750,17 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
     const int whole = whole_sm_smem();
     if (whole > lmax) lmax = whole;
     if (whole > gmax) gmax = whole;
-    cudaError_t e = cudaFuncSetAttribute(sim_logits_kernel<8, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+    cudaError_t e = cudaFuncSetAttribute(sim_logits_kernel<8, 0, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<16, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<16, 0, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<32, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<32, 0, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<64, 6>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<64, 6, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<64, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<64, 8, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(sim_logits_kernel<64, 0>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
+      e = cudaFuncSetAttribute(sim_logits_kernel<64, 0, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, lmax);
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(gram_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, gmax);
     return static_cast<int>(e);
@@ -736,15 +794,32 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
     if (whole > gsmem) gsmem = whole;
   }
   const int grid = static_cast<int>(tiles < sms ? tiles : sms);
-  switch (E) {
-    case 8: sim_logits_kernel<8, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
-    case 16: sim_logits_kernel<16, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
-    case 32: sim_logits_kernel<32, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
-    default:
-      if (kf <= 6) sim_logits_kernel<64, 6><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la);
-      else if (kf <= 8) sim_logits_kernel<64, 8><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la);
-      else sim_logits_kernel<64, 0><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la);
-      break;
+  if (E == 64 && kf <= 8) {
+    // CTA pairs over 256-token tiles, at most one pair per two SMs
+    const long long ptiles = (long long)((N + 2 * BM - 1) / (2 * BM)) * la.n_tiles;
+    const int pairs = static_cast<int>(ptiles < sms / 2 ? ptiles : sms / 2);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    cfg.gridDim = dim3(2 * (pairs > 0 ? pairs : 1), 1, 1);
+    cfg.blockDim = dim3(L_THREADS, 1, 1);
+    cfg.dynamicSmemBytes = lsmem;
+    cfg.stream = stream;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = 2;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = kf <= 6 ? cudaLaunchKernelEx(&cfg, sim_logits_kernel<64, 6, true>, mX, mW, la)
+                                  : cudaLaunchKernelEx(&cfg, sim_logits_kernel<64, 8, true>, mX, mW, la);
+    if (e != cudaSuccess) return cuda_fail(e, "sim_logits_kernel (CTA pairs)");
+  } else {
+    switch (E) {
+      case 8: sim_logits_kernel<8, 0, false><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+      case 16: sim_logits_kernel<16, 0, false><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+      case 32: sim_logits_kernel<32, 0, false><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+      default: sim_logits_kernel<64, 0, false><<<grid, L_THREADS, lsmem, stream>>>(mX, mW, la); break;
+    }
   }
   OM_LAUNCHED("sim_logits_kernel");
   GArgs ga{};
