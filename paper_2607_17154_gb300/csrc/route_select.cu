@@ -155,6 +155,8 @@ struct Lookahead {
   size_t stride;         // bytes between consecutive layers' tables
   const float* P;        // [H-1][E][E]
   int staged;            // lookahead_select_kernel copies layers l+1.. and P to shared memory
+  int topk_only;         // H = 1 with many experts: the router writes the targets and weights,
+                         // select_lanes_kernel selects
 };
 
 // A plain (generic) load: the look-ahead reads the next layers' tables either
@@ -393,6 +395,134 @@ __global__ void __launch_bounds__(128) select_kernel(
     select_token<EMAX>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
                        topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count,
                        la.H > 1);
+  }
+  flush_kind_counts(sm, kind_count, counters);
+  __syncthreads();
+  if (counters != nullptr && threadIdx.x < 4 && sm.kind[threadIdx.x])
+    atomicAdd(&counters[threadIdx.x], sm.kind[threadIdx.x]);
+}
+
+// ---------------------------------------------------------------------------
+// Alg. 2 with H = 1 from the targets topk_idx, eight lanes per token: for
+// each slot the lanes split the target and its substitutes (lane j takes
+// candidates j, j + 8, ... of the list), each keeps the smallest 64-bit key
+// of select_token (cost bits, substitute, away, server, expert: a total
+// order, so the minimum over any split is the same), and three butterfly
+// steps over the eight lanes give the slot's argmin to all of them; they
+// then update the taken set and the loss identically. Used for many experts,
+// where one thread per token walks a long serial chain of candidates.
+constexpr int kLaneTokens = 4;   // tokens per warp (eight lanes each)
+constexpr int kLaneThreads = 256;
+
+__global__ void __launch_bounds__(kLaneThreads) select_lanes_kernel(
+    const int32_t* __restrict__ topk_idx, int T, int E, int k, const uint8_t* __restrict__ tab,
+    const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
+    int32_t* __restrict__ chosen_expert, uint8_t* __restrict__ chosen_server,
+    uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters) {
+  __shared__ SelSmem sm;
+  extern __shared__ __align__(16) float s_dyn[];
+  float* s_Q = s_dyn;
+  float* s_Cq = s_dyn + E * E;
+  if (!load_tables(tab, E, sm, s_Q, s_Cq)) return;
+  __syncthreads();
+  const int M = reinterpret_cast<const int32_t*>(tab)[2];
+  const float qbar = reinterpret_cast<const float*>(tab)[5];
+  const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
+  const int lane = threadIdx.x & 31;
+  const int sub = lane & 7;       // lane within the token's group of eight
+  const int grp = lane >> 3;
+  const int warps_total = gridDim.x * (kLaneThreads / 32);
+  int kind_count[4] = {0, 0, 0, 0};
+  for (int base = (blockIdx.x * (kLaneThreads / 32) + (threadIdx.x >> 5)) * kLaneTokens; base < T;
+       base += warps_total * kLaneTokens) {
+    const int t = base + grp;
+    // every lane runs every slot (the butterflies need the whole warp);
+    // inactive tokens (past T, a NaN token's -1 targets, bad servers) write nothing
+    bool active = t < T;
+    int idx[ORDERMOE_MAX_TOPK];
+    unsigned long long taken = 0;
+#pragma unroll
+    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
+      idx[j] = 0;
+      if (j < k && active) {
+        const int r = topk_idx[(size_t)t * k + j];
+        if (r < 0 || r >= E) active = false;
+        else { idx[j] = r; taken |= 1ull << r; }
+      }
+    }
+    const int a = active ? home[t] : 0;
+    const int s = active ? ((loc != nullptr) ? loc[t] : a) : 0;
+    if (active && (a >= M || s >= M)) {
+      if (sub == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
+      active = false;
+    }
+    const float* Aas = gA + ((size_t)a * M + s) * M;
+    float q = (active && qhat != nullptr) ? qhat[t] : 0.0f;
+    int first_server = s;
+#pragma unroll
+    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
+      if (j >= k) break;  // k is the same for every lane
+      const int r = idx[j];
+      const int nsub = active ? sm.nsub[r] : -1;
+      unsigned long long best = ~0ull;
+      for (int ki = sub; ki <= nsub; ki += 8) {
+        const int kk = (ki == 0) ? r : sm.sublist[r * 64 + ki - 1];
+        const bool issub = (ki != 0);
+        float cq = 0.0f;
+        if (issub) {
+          if ((taken >> kk) & 1ull) continue;
+          if (!(__fadd_rn(q, s_Q[r * E + kk]) <= qbar)) continue;  // Eq. 40 budget
+          cq = s_Cq[r * E + kk];
+        }
+        uint32_t pm = sm.pmask[kk];
+        while (pm) {
+          const int m = __ffs(pm) - 1;
+          pm &= pm - 1;
+          const float cost = __fadd_rn(__ldg(Aas + m), cq);
+          const unsigned long long key =
+              (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
+              (static_cast<unsigned long long>(issub ? 1u : 0u) << 31) |
+              (static_cast<unsigned long long>(m != s ? 1u : 0u) << 30) |
+              (static_cast<unsigned long long>(m) << 8) | static_cast<unsigned long long>(kk);
+          best = key < best ? key : best;
+        }
+      }
+#pragma unroll
+      for (int o = 4; o > 0; o >>= 1) {
+        const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+        best = other < best ? other : best;
+      }
+      if (!active) continue;
+      int kstar, mstar, kd;
+      if (best == ~0ull) {
+        if (sub == 0) report(&g_err_route, ORDERMOE_DEV_NO_CANDIDATE, t);
+        kstar = r; mstar = s; kd = 0;
+      } else {
+        kstar = static_cast<int>(best & 0xFFu);
+        mstar = static_cast<int>((best >> 8) & 0xFFu);
+        const int bsub = static_cast<int>((best >> 31) & 1u);
+        const int away = static_cast<int>((best >> 30) & 1u);
+        kd = 2 * away + bsub;
+        if (bsub) {
+          taken |= 1ull << kstar;
+          q = __fadd_rn(q, s_Q[r * E + kstar]);
+        }
+      }
+      if (j == 0) first_server = mstar;
+      if (sub == 0) {
+        chosen_expert[(size_t)t * k + j] = kstar;
+        chosen_server[(size_t)t * k + j] = static_cast<uint8_t>(mstar);
+        kind_out[(size_t)t * k + j] = static_cast<uint8_t>(kd);
+        if (kd == 0) ++kind_count[0];  // constant indices: kind_count[] stays in registers
+        else if (kd == 1) ++kind_count[1];
+        else if (kd == 2) ++kind_count[2];
+        else ++kind_count[3];
+      }
+    }
+    if (active && sub == 0 && loc != nullptr) {
+      loc[t] = static_cast<uint8_t>(first_server);
+      qhat[t] = q;
+    }
   }
   flush_kind_counts(sm, kind_count, counters);
   __syncthreads();
@@ -999,7 +1129,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
       select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
                        topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count,
-                       la.H > 1);
+                       la.H > 1 || la.topk_only);
     }
     flush_kind_counts(sm, kind_count, counters);
   }
@@ -1081,6 +1211,23 @@ static int launch_lookahead_select(const int32_t* topk_idx, int T, int E, int k,
   return ORDERMOE_OK;
 }
 
+static int launch_select_lanes(const int32_t* topk_idx, int T, int E, int k, const uint8_t* tb,
+                               const uint8_t* home, uint8_t* loc, float* qhat,
+                               int32_t* chosen_expert, uint8_t* chosen_server, uint8_t* kind,
+                               int32_t* counters, size_t tab_smem, cudaStream_t stream) {
+  if (T <= 0) return ORDERMOE_OK;
+  const int per_block = (kLaneThreads / 32) * kLaneTokens;
+  long long blocks = (T + per_block - 1) / per_block;
+  const long long cap = 4LL * num_sms();
+  if (blocks > cap) blocks = cap;
+  cudaFuncSetAttribute(select_lanes_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                       (int)tab_smem);
+  select_lanes_kernel<<<static_cast<int>(blocks), kLaneThreads, tab_smem, stream>>>(
+      topk_idx, T, E, k, tb, home, loc, qhat, chosen_expert, chosen_server, kind, counters);
+  OM_LAUNCHED("select_lanes_kernel");
+  return ORDERMOE_OK;
+}
+
 static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float* logits_in, int T,
                              int E, int d, int k, int renorm, const void* tables,
                              size_t tables_bytes_, Lookahead la, const uint8_t* home, uint8_t* loc,
@@ -1128,6 +1275,10 @@ static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float
                                               tab_smem, stream)
                     : ORDERMOE_OK;
   }
+  // many experts (long candidate lists per slot): the router writes the
+  // targets and select_lanes_kernel selects with eight lanes per token
+  const bool lanes = la.H == 1 && E > 16;
+  if (lanes) la.topk_only = 1;
   CUtensorMap mX, mW;
   int rc;
   const int NE = E <= 16 ? 16 : (E <= 32 ? 32 : 64);
@@ -1170,6 +1321,9 @@ static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float
   if (la.H > 1)
     return launch_lookahead_select(topk_idx, T, E, k, tb, la, home, loc, qhat, chosen_expert,
                                    chosen_server, kind, counters, tab_smem, stream);
+  if (lanes)
+    return launch_select_lanes(topk_idx, T, E, k, tb, home, loc, qhat, chosen_expert,
+                               chosen_server, kind, counters, tab_smem, stream);
   return ORDERMOE_OK;
 }
 
