@@ -982,7 +982,59 @@ def cpu_baseline(w, inp, seed, target_s):
                       % (n, w.T, w.name, dt),
             "cpu_model": cpu_model(), "host_cpus": cpu_cores(), "omp_threads": oracle.threads(),
             "tiny_1_thread": tiny_oracle_rate(seed, 1),
-            "tiny_all_threads": tiny_oracle_rate(seed, oracle.threads())}
+            "tiny_all_threads": tiny_oracle_rate(seed, oracle.threads()),
+            "other_workloads": cpu_other_workloads(seed, inp["X"].device)}
+
+
+def cpu_other_workloads(seed, device, budget_s=3.0):
+    """The oracle on bounded samples of the other workloads, each scaled to
+    that workload's unit and labelled with its sample: tokens of the
+    fine-grained layer; tokens of one decode layer, scaled to the 32-layer
+    step; calibration tokens of one similarity layer, scaled to 24 layers."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_17154_gb300 import synth
+    out = {}
+    rng = np.random.default_rng(seed)
+
+    def sample_rate(w, inp, layers):
+        host, home, tab = oracle_setup(w, inp, seed)
+        t0 = time.perf_counter()
+        oracle_tokens(w, host, home, tab, np.arange(2))
+        per_tok = max((time.perf_counter() - t0) / 2, 1e-6)
+        n = int(min(w.T, max(2, budget_s / per_tok)))
+        toks = np.sort(rng.choice(w.T, n, replace=False))
+        t0 = time.perf_counter()
+        oracle_tokens(w, host, home, tab, toks)
+        dt = time.perf_counter() - t0
+        return n, dt, n / dt / layers
+
+    w = synth.workload("fine_grained")
+    n, dt, v = sample_rate(w, synth.layer_inputs(w, seed=seed, device=device), 1)
+    out["fine_grained"] = {"value": round(v, 3), "unit": UNIT,
+                           "sample": "%d of the %d tokens of the layer, whole oracle path, %.1f s"
+                                     % (n, w.T, dt)}
+    w = synth.workload("decode_stack")
+    n, dt, v = sample_rate(w, synth.layer_inputs(w, seed=seed, device=device), w.L)
+    out["decode_stack"] = {"value": round(v, 3), "unit": UNIT,
+                           "sample": "%d of the %d tokens of one of the %d layers, whole oracle path, "
+                                     "%.1f s; the step rate extrapolated as one layer's rate / %d"
+                                     % (n, w.T, w.L, dt, w.L)}
+    w = synth.workload("similarity")
+    Wr = synth.bits(synth.router_weights(w.E, w.d, w.n_clusters, seed=seed + 500, device=device))
+    n = 4096
+    Xs = synth.bits(synth.calibration(n, w.d, seed, device=device))
+    t0 = time.perf_counter()
+    sim, H = oracle.similarity(Wr, Xs, return_H=True)
+    oracle.expert_counts(np.ascontiguousarray(H.T), w.k)
+    dt = time.perf_counter() - t0
+    out["similarity"] = {"value": round(n / dt / w.L, 1), "unit": "tokens/s",
+                         "sample": "%d calibration tokens through one of the %d layers (logits, "
+                                   "cosine similarity, counts), %.1f s; the plan rate extrapolated "
+                                   "as one layer's rate / %d; grouping and placement not timed"
+                                   % (n, w.L, dt, w.L)}
+    return out
 
 
 def run_reference(args, dist):
