@@ -463,12 +463,20 @@ __device__ __forceinline__ bool epi_all(bool p) {
   return r != 0;
 }
 
+// Tensor maps of the permuted rows with boxes of 16, 32, ..., 128 rows: a
+// tile cut to N rows loads N/2 rows per CTA (rounded up to 16) instead of a
+// full 128-row box, since it is the row boxes, not the MMAs, that bound a
+// cut tile (an expert's last one).
+struct RowMaps {
+  CUtensorMap m[8];  // m[i]: box of 16 (i + 1) rows
+};
+
 // One cluster = one CTA pair.
 template <int MODE>
 __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
     ffn_gemm_pair_kernel(const __grid_constant__ CUtensorMap mapW0,
                          const __grid_constant__ CUtensorMap mapW1,
-                         const __grid_constant__ CUtensorMap mapT, Args args) {
+                         const __grid_constant__ RowMaps mapT, Args args) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* tiles = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -519,7 +527,8 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_map(&mapW0);
     if (MODE == GATEUP) tma_prefetch_map(&mapW1);
-    tma_prefetch_map(&mapT);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) tma_prefetch_map(&mapT.m[i]);
   }
   if (warp == 1) {
     tmem_alloc_pair(&s.tmem_base, TMEM_COLS);
@@ -544,6 +553,9 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
       for (int tile = cluster; tile < total && !*abort; tile += n_clusters) {
         const Tile t = tile_of(tile);
         const int trow = t.m0 + static_cast<int>(rp) * (tile_n(t) >> 1);  // N/2 rows per CTA
+        const int hb = ((tile_n(t) >> 1) + 15) & ~15;  // rows per CTA's box (16 .. 128)
+        const CUtensorMap* mrow = &mapT.m[(hb >> 4) - 1];
+        const uint32_t stage_tx = 2u * static_cast<uint32_t>(P_W_BYTES + hb * BK * 2);
         const int wrow = (MODE == GATEUP)
                              ? t.e * args.b_rows + t.n * 128 + 64 * static_cast<int>(rp)
                              : t.e * args.b_rows + t.n * 256 + 128 * static_cast<int>(rp);
@@ -556,14 +568,14 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
           uint8_t* sw = tiles + stage * P_STAGE_BYTES;
           uint8_t* st = sw + P_W_BYTES;
           const uint32_t full_even = mapa_shared(smem_u32(&s.full[stage]), lead);
-          if (even) mbar_arrive_expect_tx(&s.full[stage], 2 * P_STAGE_BYTES);
+          if (even) mbar_arrive_expect_tx(&s.full[stage], stage_tx);
           if (MODE == GATEUP) {
             tma_load_2d_pair(sw, &mapW0, full_even, kb * BK, wrow);             // W1: lanes 0..63
             tma_load_2d_pair(sw + P_W_BYTES / 2, &mapW1, full_even, kb * BK, wrow);  // W3: 64..127
           } else {
             tma_load_2d_pair(sw, &mapW0, full_even, kb * BK, wrow);
           }
-          tma_load_2d_pair(st, &mapT, full_even, kb * BK, trow);
+          tma_load_2d_pair(st, mrow, full_even, kb * BK, trow);
           issued_mask |= 1u << stage;
           last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1u; }
@@ -830,7 +842,7 @@ static int max_resident_clusters() {
 
 // One launch of the CTA-pair kernel over `tiles` pair tiles.
 template <int MODE>
-static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const CUtensorMap& t,
+static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const gg::RowMaps& t,
                        const gg::Args& a, long long tiles, cudaStream_t stream, const char* what) {
   const long long cmax = max_resident_clusters<MODE>();
   const long long clusters = tiles < cmax ? tiles : cmax;
@@ -840,6 +852,15 @@ static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const CUten
   const cudaError_t e = cudaLaunchKernelEx(&cfg, gg::ffn_gemm_pair_kernel<MODE>, w0, w1, t, a);
   if (e != cudaSuccess) return cuda_fail(e, what);
   OM_LAUNCHED(what);
+  return ORDERMOE_OK;
+}
+
+// The row maps of a [rows][cols] bf16 tensor, boxes of 16 .. 128 rows.
+static int make_row_maps(gg::RowMaps* rm, const void* base, uint64_t rows, uint64_t cols) {
+  for (int i = 0; i < 8; ++i) {
+    const int rc = make_tmap_bf16(&rm->m[i], base, rows, cols, static_cast<uint32_t>(16 * (i + 1)));
+    if (rc) return rc;
+  }
   return ORDERMOE_OK;
 }
 
@@ -870,7 +891,9 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
     if ((rc = make_tmap_bf16(&mW1, W1, (uint64_t)E * dff, d, 64))) return rc;
     if ((rc = make_tmap_bf16(&mW3, W3, (uint64_t)E * dff, d, 64))) return rc;
     const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
-    return launch_pair<GATEUP>(mW1, mW3, mX, a, row_tiles * a.n_tiles, stream,
+    gg::RowMaps rX;
+    if ((rc = make_row_maps(&rX, X_perm, R, d))) return rc;
+    return launch_pair<GATEUP>(mW1, mW3, rX, a, row_tiles * a.n_tiles, stream,
                                "ffn_gemm_pair_kernel<gate_up>");
   } else {
     if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
@@ -896,7 +919,9 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
   if ((rc = make_map(&mH, H, R, dff))) return rc;
   if (use_pairs(R, E)) {
     const long long row_tiles = (long long)(R + P_BM - 1) / P_BM + E;
-    return launch_pair<DOWN>(mW2, mW2, mH, a, row_tiles * a.n_tiles, stream,
+    gg::RowMaps rH;
+    if ((rc = make_row_maps(&rH, H, R, dff))) return rc;
+    return launch_pair<DOWN>(mW2, mW2, rH, a, row_tiles * a.n_tiles, stream,
                              "ffn_gemm_pair_kernel<down>");
   } else {
     const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
