@@ -70,3 +70,22 @@ def test_reference_arm_prints_the_contract_line():
     assert line["higher_is_better"] is True
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["d2h_bytes_per_step"] == 0
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+
+
+def test_tensor_peak_follows_the_run():
+    """The bf16 peak a tensor-bound fraction divides by: the burst figure for
+    a short region with no power cap seen, the sustained one otherwise; both
+    fractions are printed and the one that applies is named."""
+    sys.path.insert(0, ROOT)
+    import bench
+    pk = {"bf16_tflops": 1918.0, "bf16_tflops_sustained": 1723.6}
+    quiet = {"reasons": []}
+    capped = {"reasons": ["sw_power_cap"]}
+    assert bench.tensor_peak(pk, "measured", quiet, 0.036)[:2] == (1918.0, "burst")
+    assert bench.tensor_peak(pk, "measured", capped, 0.036)[:2] == (1723.6, "sustained")
+    assert bench.tensor_peak(pk, "measured", quiet, 2.0)[:2] == (1723.6, "sustained")
+    r = bench.tensor_roofline("k", 1700.0, pk, "measured", quiet, 0.036, traffic=None)
+    assert r["peak_applies"] == "burst" and r["frac"] == round(1700.0 / 1918.0, 4)
+    assert r["frac_burst"] == round(1700.0 / 1918.0, 4)
+    assert r["frac_sustained"] == round(1700.0 / 1723.6, 4)
+    assert r["peak_source"] == "measured bf16_tflops" and r["traffic"] is None
