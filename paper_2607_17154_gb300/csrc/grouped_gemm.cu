@@ -88,8 +88,14 @@ struct Tile {
 };
 
 __device__ __forceinline__ Tile decode(int tile, const Smem& s, int E, int n_tiles, int m_major) {
-  int e = 0;
-  while (e < E - 1 && s.mt_start[e + 1] * n_tiles <= tile) ++e;
+  // the last expert whose first tile is <= tile (binary search: the row-tile
+  // starts never decrease; empty experts share their successor's start)
+  int e = 0, hi = E - 1;
+  while (e < hi) {
+    const int mid = (e + hi + 1) >> 1;
+    if (s.mt_start[mid] * n_tiles <= tile) e = mid;
+    else hi = mid - 1;
+  }
   const int local = tile - s.mt_start[e] * n_tiles;
   const int n_mt = s.mt_start[e + 1] - s.mt_start[e];
   Tile t;
@@ -426,8 +432,14 @@ struct PCfg {
 };
 
 __device__ __forceinline__ Tile decode_pair(int tile, const PSmem& s, int E, int n_tiles) {
-  int e = 0;
-  while (e < E - 1 && s.mt_start[e + 1] * n_tiles <= tile) ++e;
+  // the last expert whose first tile is <= tile (binary search: the row-tile
+  // starts never decrease; empty experts share their successor's start)
+  int e = 0, hi = E - 1;
+  while (e < hi) {
+    const int mid = (e + hi + 1) >> 1;
+    if (s.mt_start[mid] * n_tiles <= tile) e = mid;
+    else hi = mid - 1;
+  }
   const int local = tile - s.mt_start[e] * n_tiles;
   const int n_mt = s.mt_start[e + 1] - s.mt_start[e];
   Tile t;
