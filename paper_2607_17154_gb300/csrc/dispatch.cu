@@ -5,10 +5,10 @@
 // offsets and the stable ranks (dispatch_small_kernel). Otherwise the (token,
 // slot) entries i = t*k + j are cut into chunks of kChunk = 256 consecutive
 // entries, one block each:
-//   1. chunk_hist: per-chunk expert histogram -> hist[chunk][E]
+//   1. chunk_hist: per-chunk expert histogram -> hist[E][chunk]
 //   2. chunk_scan: one block; for every expert the exclusive prefix of its
 //      count over chunks, plus the expert offsets (exclusive prefix over
-//      experts) -> base[chunk][e] = offsets[e] + entries of e in earlier chunks
+//      experts) -> base[e][chunk] = offsets[e] + entries of e in earlier chunks
 //   3. rank: stable rank inside the chunk (per-warp match + per-warp
 //      counts), row = base + rank;
 //   4. gather_rows: one warp per permuted row copies X[row_token[row]] into
@@ -43,50 +43,32 @@ __global__ void __launch_bounds__(kChunk) chunk_hist_kernel(const int32_t* __res
     else report(&g_err_dispatch, ORDERMOE_DEV_BAD_INDEX, static_cast<int>(i));
   }
   __syncthreads();
-  if (threadIdx.x < E) hist[(size_t)blockIdx.x * E + threadIdx.x] = h[threadIdx.x];
+  if (threadIdx.x < E) hist[(size_t)threadIdx.x * gridDim.x + blockIdx.x] = h[threadIdx.x];
 }
 
-// One block of 1024 threads. Warp w scans the chunk counts of experts w and
-// w + 32 with warp shuffles (32 chunks at a time, carrying the running sum),
-// then warp 0 scans the expert totals into offsets and they are added back.
-// With `staged` the histogram is first copied into shared memory with
-// coalesced loads, transposed to [E][P] with an odd pitch P (a warp's 32
-// consecutive chunks of one expert then fall in 32 banks), and written back
-// coalesced; otherwise each warp reads its expert's column, E words apart.
-constexpr int kScanStageBytes = 96 * 1024;
-
+// One block of 1024 threads over hist[E][nchunks] (expert-major, as
+// chunk_hist_kernel writes it): warp w scans the chunk counts of experts w
+// and w + 32 with warp shuffles (32 chunks at a time, coalesced, carrying the
+// running sum), then warp 0 scans the expert totals into offsets and they are
+// added back: base[e][chunk] = offsets[e] + entries of e in earlier chunks.
 __global__ void __launch_bounds__(1024) chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks,
-                                                          int E, int32_t* __restrict__ offsets,
-                                                          int staged) {
-  extern __shared__ int hs[];  // staged: [E][P]
+                                                          int E, int32_t* __restrict__ offsets) {
   __shared__ int total[64];
   __shared__ int start[65];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int P = nchunks | 1;
-  if (staged) {
-    for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) {
-      const int b = i / E;
-      hs[(i - b * E) * P + b] = hist[i];
-    }
-    __syncthreads();
-  }
   for (int e = warp; e < E; e += 32) {
+    int32_t* row = hist + (size_t)e * nchunks;
     int carry = 0;
     for (int b0 = 0; b0 < nchunks; b0 += 32) {
       const int b = b0 + lane;
-      const int v = (b < nchunks) ? (staged ? hs[e * P + b] : hist[(size_t)b * E + e]) : 0;
+      const int v = (b < nchunks) ? row[b] : 0;
       int incl = v;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int u = __shfl_up_sync(0xffffffffu, incl, o);
         if (lane >= o) incl += u;
       }
-      if (b < nchunks) {
-        if (staged)
-          hs[e * P + b] = carry + incl - v;
-        else
-          hist[(size_t)b * E + e] = carry + incl - v;
-      }
+      if (b < nchunks) row[b] = carry + incl - v;
       carry += __shfl_sync(0xffffffffu, incl, 31);
     }
     if (lane == 0) total[e] = carry;
@@ -108,13 +90,10 @@ __global__ void __launch_bounds__(1024) chunk_scan_kernel(int32_t* __restrict__ 
   }
   __syncthreads();
   if (threadIdx.x <= E) offsets[threadIdx.x] = start[threadIdx.x];
-  if (staged) {
-    for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) {
-      const int b = i / E, e = i - b * E;
-      hist[i] = hs[e * P + b] + start[e];
-    }
-  } else {
-    for (int i = threadIdx.x; i < nchunks * E; i += blockDim.x) hist[i] += start[i % E];
+  for (int e = warp; e < E; e += 32) {
+    int32_t* row = hist + (size_t)e * nchunks;
+    const int add = start[e];
+    for (int b = lane; b < nchunks; b += 32) row[b] += add;
   }
 }
 
@@ -137,7 +116,7 @@ __global__ void __launch_bounds__(kChunk) rank_kernel(
   if (e >= 0) {
     int before = 0;
     for (int w = 0; w < warp; ++w) before += cnt[w][e];
-    const int row = base[(size_t)blockIdx.x * E + e] + before + rank_in_warp;
+    const int row = base[(size_t)e * gridDim.x + blockIdx.x] + before + rank_in_warp;
     row_of[i] = row;
     row_token[row] = static_cast<int32_t>(i / k);
   }
@@ -431,16 +410,7 @@ int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int 
   } else {
     chunk_hist_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, E, hist);
     OM_LAUNCHED("chunk_hist_kernel");
-    static PerDevice scan_attr;
-    const int attr_ok = per_device(scan_attr, [] {
-      return static_cast<int>(cudaFuncSetAttribute(
-          chunk_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kScanStageBytes));
-    });
-    if (attr_ok != static_cast<int>(cudaSuccess)) cudaGetLastError();
-    const size_t stage_bytes = (size_t)(nchunks | 1) * E * sizeof(int32_t);
-    const int staged = attr_ok == static_cast<int>(cudaSuccess) && stage_bytes <= kScanStageBytes;
-    chunk_scan_kernel<<<1, 1024, staged ? stage_bytes : 0, stream>>>(hist, nchunks, E, offsets,
-                                                                     staged);
+    chunk_scan_kernel<<<1, 1024, 0, stream>>>(hist, nchunks, E, offsets);
     OM_LAUNCHED("chunk_scan_kernel");
     rank_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, hist, row_token, row_of);
     OM_LAUNCHED("rank_kernel");
