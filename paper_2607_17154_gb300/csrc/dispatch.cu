@@ -48,14 +48,82 @@ __global__ void __launch_bounds__(kChunk) chunk_hist_kernel(const int32_t* __res
 
 // One block of 1024 threads over hist[E][nchunks] (expert-major, as
 // chunk_hist_kernel writes it): warp w scans the chunk counts of experts w
-// and w + 32 with warp shuffles (32 chunks at a time, coalesced, carrying the
-// running sum), then warp 0 scans the expert totals into offsets and they are
+// and w + 32, then warp 0 scans the expert totals into offsets and they are
 // added back: base[e][chunk] = offsets[e] + entries of e in earlier chunks.
-__global__ void __launch_bounds__(1024) chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks,
+// Up to kScanRegs * 32 chunks (T*k up to 65536 entries) both rows are loaded
+// at once (coalesced: lane j holds chunks j, j + 32, ...) and scanned in
+// registers, 32 chunks at a time with the running sum carried, and each base
+// is written once. Longer rows go 32 chunks at a time from memory.
+constexpr int kScanRegs = 8;
+
+__device__ __forceinline__ int warp_excl_scan(int v, int lane, int* total) {
+  int incl = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int u = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += u;
+  }
+  *total = __shfl_sync(0xffffffffu, incl, 31);
+  return incl - v;
+}
+
+__global__ void __launch_bounds__(1024, 1) chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks,
                                                           int E, int32_t* __restrict__ offsets) {
   __shared__ int total[64];
   __shared__ int start[65];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (nchunks <= 32 * kScanRegs) {
+    int v[2][kScanRegs];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int e = warp + 32 * r;
+#pragma unroll
+      for (int i = 0; i < kScanRegs; ++i) {
+        const int b = i * 32 + lane;
+        v[r][i] = (e < E && b < nchunks) ? hist[(size_t)e * nchunks + b] : 0;
+      }
+    }
+    int carry[2] = {0, 0};
+#pragma unroll
+    for (int i = 0; i < kScanRegs; ++i) {
+      if (i * 32 < nchunks) {  // the same for the whole warp
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {  // v becomes the row's exclusive prefix
+          int sum;
+          const int excl = warp_excl_scan(v[r][i], lane, &sum);
+          v[r][i] = carry[r] + excl;
+          carry[r] += sum;
+        }
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r)
+      if (lane == 0 && warp + 32 * r < E) total[warp + 32 * r] = carry[r];
+    __syncthreads();
+    if (warp == 0) {  // exclusive scan of the E <= 64 totals, two per lane
+      const int t0 = (2 * lane < E) ? total[2 * lane] : 0;
+      const int t1 = (2 * lane + 1 < E) ? total[2 * lane + 1] : 0;
+      int all;
+      const int excl = warp_excl_scan(t0 + t1, lane, &all);
+      if (2 * lane < E) start[2 * lane] = excl;
+      if (2 * lane + 1 < E) start[2 * lane + 1] = excl + t0;
+      if (lane == 31) start[E] = all;
+    }
+    __syncthreads();
+    if (threadIdx.x <= E) offsets[threadIdx.x] = start[threadIdx.x];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const int e = warp + 32 * r;
+      if (e >= E) continue;
+      const int add = start[e];
+#pragma unroll
+      for (int i = 0; i < kScanRegs; ++i) {
+        const int b = i * 32 + lane;
+        if (b < nchunks) hist[(size_t)e * nchunks + b] = add + v[r][i];
+      }
+    }
+    return;
+  }
   for (int e = warp; e < E; e += 32) {
     int32_t* row = hist + (size_t)e * nchunks;
     int carry = 0;

@@ -1075,7 +1075,13 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
   } else {
     // the selection tables, while the TMA and MMA warps run (named barrier 1:
     // the 128 epilogue threads)
-    if (rank == 0) tables_ok = load_tables_range(tab, E, sm, s_Q, s_Cq, tid - 64, 128);
+    if (rank == 0) {
+      if (la.H > 1 || la.topk_only) {  // targets only: a selection kernel reads the tables
+        if (tid - 64 < 4) sm.kind[tid - 64] = 0;
+      } else {
+        tables_ok = load_tables_range(tab, E, sm, s_Q, s_Cq, tid - 64, 128);
+      }
+    }
     asm volatile("bar.sync 1, 128;" ::: "memory");
     // epilogue part 1: this CTA's partial logits
     const int q = warp & 3;
