@@ -32,9 +32,9 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # the recorded ncu capture of that kernel, valid only while the
 # kernel sources hash to the values recorded with it.
 GATE_UP_TRAFFIC = {
-    "bytes": 1959263232 + 228937984,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
+    "bytes": 2129134336 + 230202880,  # dram__bytes_read.sum + dram__bytes_write.sum, one launch
     "sha256": {"paper_2607_17154_gb300/csrc/grouped_gemm.cu":
-               "eef110b728fad2a5b2db6094392f637633e269fd4774b4f62a5a8ade69e70b4f",
+               "4927e63493fe44ece0df5c13e0ce64762ebb2b4cfc2beb1056afd2fe774f8cb2",
                "paper_2607_17154_gb300/csrc/common.cuh":
                "5f0611cf723907b96ee41883667bfb1045d2e7d81cef1f06cf17694b13751bfb"},
 }
@@ -321,7 +321,9 @@ def run_ours(args, dist):
             ("combine", lambda: B.ordermoe_combine(Yp, row_of, wts, T, k, d, y)),
         ]
 
-    KERNELS_PER_STEP = 8   # route_select 1, dispatch 4, gate/up 1, down 1, combine 1
+    # route_select 1 (2 for more than 16 experts: the lane selection kernel),
+    # dispatch 4, gate/up 1, down 1, combine 1
+    KERNELS_PER_STEP = 8 + (1 if E > 16 else 0)
     step(cnt=counters)     # one counted pass for the execution-type breakdown
     for _ in range(max(args.warmup, 3)):
         step()
@@ -708,9 +710,11 @@ def decode_timed(args, dist, w, device, S, H):
 
 def decode_launches(w, H):
     """Kernels of one decode step: the first layer's RMSNorm, then per layer
-    route_select 1, dispatch 2 (one block ranks up to 4096 entries) or 4,
-    gate/up 1, down 1 and the residual combine 1."""
-    return 1 + (4 + (2 if w.T * w.k <= 4096 else 4)) * w.L
+    route_select 1 (2 with a look-ahead horizon H > 1 or more than 16
+    experts: a separate selection kernel), dispatch 2 (one block ranks up to
+    4096 entries) or 4, gate/up 1, down 1 and the residual combine 1."""
+    route = 1 if (H == 1 and w.E <= 16) else 2
+    return 1 + (route + 3 + (2 if w.T * w.k <= 4096 else 4)) * w.L
 
 
 def run_decode(args, dist, w, device):
