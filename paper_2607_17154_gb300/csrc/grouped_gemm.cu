@@ -728,7 +728,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&s.tempty[slot]), lead));
+      if (lane == 0) mbar_arrive_remote(mapa_shared(smem_u32(&s.tempty[slot]), lead));
     }
   }
 

@@ -484,7 +484,7 @@ __global__ void __launch_bounds__(L_THREADS, 1)
       tc_fence_before();
       if (PAIR) {
         __syncwarp();
-        if (lane == 0) mbar_arrive_cluster(mapa_shared(smem_u32(&s.tempty[slot]), 0));
+        if (lane == 0) mbar_arrive_remote(mapa_shared(smem_u32(&s.tempty[slot]), 0));
       } else {
         mbar_arrive(&s.tempty[slot]);
       }
