@@ -160,8 +160,10 @@ def test_router_logits_match_oracle(T, d, E):
                                      # its limit of 4096, and the first size past it
                                      (1500, 2, 8, 64), (2048, 2, 8, 16), (683, 6, 64, 8),
                                      (4096, 2, 8, 4096),
-                                     (8192, 6, 64, 64),     # 192 chunks: histogram staged in shared memory
-                                     (20000, 6, 64, 64)])   # 469 chunks x 64: too large to stage
+                                     (8192, 6, 64, 64),     # 192 chunks: the scan holds them in registers
+                                     (16384, 4, 64, 64),    # 256 chunks: the most it holds in registers
+                                     (16385, 4, 33, 64),    # 257 chunks: 32 at a time from memory
+                                     (20000, 6, 64, 64)])   # 469 chunks x 64
 def test_dispatch_bit_exact(T, k, E, d):
     rng = np.random.default_rng(T * k + E)
     chosen = rng.integers(0, E, (T, k)).astype(np.int32)
