@@ -78,6 +78,48 @@ int per_device(PerDevice& c, F init) {
     if (e_ != cudaSuccess) return om::cuda_fail(e_, what); \
   } while (0)
 
+// Programmatic dependent launch. The hot path's per-step kernels are launched
+// with launch_pdl: a kernel's blocks may start (and set up shared memory,
+// barriers, TMEM and tensor-map prefetches) while the previous kernel on the
+// stream finishes. Every kernel launched this way calls pdl_wait() before its
+// first access to global memory: it returns once the previous kernel has
+// completed and its writes are visible (at once when there is no such kernel).
+// pdl_trigger() lets the next kernel's blocks be scheduled as soon as every
+// block of this one has started.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Whether launches on the stream use programmatic dependent launch: not while
+// it is being captured into a graph.
+inline bool pdl_on(cudaStream_t stream) {
+  cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+  return cudaStreamIsCapturing(stream, &st) == cudaSuccess && st == cudaStreamCaptureStatusNone;
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_on(stream) ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+#define OM_LAUNCH_PDL(what, ...)                           \
+  do {                                                     \
+    cudaError_t e_ = om::launch_pdl(__VA_ARGS__);          \
+    if (e_ != cudaSuccess) return om::cuda_fail(e_, what); \
+  } while (0)
+
 // Device error word: one per translation unit (no relocatable device code).
 // Low 32 bits: ORDERMOE_DEV_* code of the first error; high 32 bits: detail.
 struct DevErr {

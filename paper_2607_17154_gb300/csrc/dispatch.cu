@@ -33,6 +33,8 @@ constexpr int kChunk = kDispatchChunk;
 __global__ void __launch_bounds__(kChunk) chunk_hist_kernel(const int32_t* __restrict__ chosen,
                                                             int64_t n, int E,
                                                             int32_t* __restrict__ hist) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   __shared__ int h[64];
   if (threadIdx.x < 64) h[threadIdx.x] = 0;
   __syncthreads();
@@ -69,6 +71,8 @@ __device__ __forceinline__ int warp_excl_scan(int v, int lane, int* total) {
 
 __global__ void __launch_bounds__(1024, 1) chunk_scan_kernel(int32_t* __restrict__ hist, int nchunks,
                                                           int E, int32_t* __restrict__ offsets) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   __shared__ int total[64];
   __shared__ int start[65];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -168,6 +172,8 @@ __global__ void __launch_bounds__(1024, 1) chunk_scan_kernel(int32_t* __restrict
 __global__ void __launch_bounds__(kChunk) rank_kernel(
     const int32_t* __restrict__ chosen, int64_t n, int k, int E, const int32_t* __restrict__ base,
     int32_t* __restrict__ row_token, int32_t* __restrict__ row_of) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   constexpr int kWarps = kChunk / 32;
   __shared__ int cnt[kWarps][64];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -199,6 +205,8 @@ __global__ void __launch_bounds__(256) gather_rows_kernel(const uint16_t* __rest
                                                           const int32_t* __restrict__ offsets,
                                                           int E, int T, int d,
                                                           uint16_t* __restrict__ X_perm) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   constexpr int kUnroll = 8;
   const int lane = threadIdx.x & 31;
   const int nvec = d >> 3;
@@ -238,6 +246,8 @@ __global__ void __launch_bounds__(256) combine_kernel(const uint16_t* __restrict
                                                       const int32_t* __restrict__ row_of,
                                                       const float* __restrict__ w, int T, int k,
                                                       int d, uint16_t* __restrict__ y) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int64_t warps_total = (int64_t)gridDim.x * (blockDim.x >> 5);
   const int nvec = d >> 3;
@@ -317,6 +327,8 @@ __global__ void __launch_bounds__(kNormThreads) residual_norm_kernel(
     const uint16_t* __restrict__ Yp, const int32_t* __restrict__ row_of,
     const float* __restrict__ w, const uint16_t* __restrict__ h, int T, int k, int d, float eps,
     uint16_t* __restrict__ h_out, uint16_t* __restrict__ x_out) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   __shared__ float wsum[kNormThreads / 32];
   __shared__ int bad;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -410,6 +422,8 @@ constexpr int kSmallN = 4096;
 __global__ void __launch_bounds__(1024) dispatch_small_kernel(
     const int32_t* __restrict__ chosen, int n, int k, int E, int32_t* __restrict__ offsets,
     int32_t* __restrict__ row_token, int32_t* __restrict__ row_of) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   __shared__ int total[64];
   __shared__ int start[64];
   __shared__ int wc[32][64];
@@ -472,23 +486,21 @@ int dispatch_launch(const int32_t* chosen, const uint16_t* X, int T, int k, int 
     return ORDERMOE_OK;
   }
   if (n <= kSmallN) {
-    dispatch_small_kernel<<<1, 1024, 0, stream>>>(chosen, static_cast<int>(n), k, E, offsets,
-                                                  row_token, row_of);
-    OM_LAUNCHED("dispatch_small_kernel");
+    OM_LAUNCH_PDL("dispatch_small_kernel", dispatch_small_kernel, dim3(1), dim3(1024), 0, stream,
+                  chosen, static_cast<int>(n), k, E, offsets, row_token, row_of);
   } else {
-    chunk_hist_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, E, hist);
-    OM_LAUNCHED("chunk_hist_kernel");
-    chunk_scan_kernel<<<1, 1024, 0, stream>>>(hist, nchunks, E, offsets);
-    OM_LAUNCHED("chunk_scan_kernel");
-    rank_kernel<<<nchunks, kChunk, 0, stream>>>(chosen, n, k, E, hist, row_token, row_of);
-    OM_LAUNCHED("rank_kernel");
+    OM_LAUNCH_PDL("chunk_hist_kernel", chunk_hist_kernel, dim3(nchunks), dim3(kChunk), 0, stream,
+                  chosen, n, E, hist);
+    OM_LAUNCH_PDL("chunk_scan_kernel", chunk_scan_kernel, dim3(1), dim3(1024), 0, stream,
+                  hist, nchunks, E, offsets);
+    OM_LAUNCH_PDL("rank_kernel", rank_kernel, dim3(nchunks), dim3(kChunk), 0, stream,
+                  chosen, n, k, E, hist, row_token, row_of);
   }
   int64_t blocks = (n + 7) / 8;
   const int cap = num_sms() * 8;
   if (blocks > cap) blocks = cap;
-  gather_rows_kernel<<<static_cast<int>(blocks), 256, 0, stream>>>(X, row_token, offsets, E, T, d,
-                                                                    X_perm);
-  OM_LAUNCHED("gather_rows_kernel");
+  OM_LAUNCH_PDL("gather_rows_kernel", gather_rows_kernel, dim3(static_cast<int>(blocks)), dim3(256),
+                0, stream, X, row_token, offsets, E, T, d, X_perm);
   return ORDERMOE_OK;
 }
 
@@ -537,9 +549,9 @@ extern "C" int ordermoe_rmsnorm(const uint16_t* h, int T, int d, float eps, uint
   if (!h || !x || !aligned16(h) || !aligned16(x))
     return fail(ORDERMOE_ERR_INVALID_ARG, "rmsnorm: null or not 16-byte aligned pointer");
   const int grid = T < num_sms() * 16 ? T : num_sms() * 16;
-  residual_norm_kernel<false><<<grid, kNormThreads, 0, stream>>>(nullptr, nullptr, nullptr, h, T, 1,
-                                                                  d, eps, nullptr, x);
-  OM_LAUNCHED("residual_norm_kernel<rmsnorm>");
+  OM_LAUNCH_PDL("residual_norm_kernel<rmsnorm>", residual_norm_kernel<false>, dim3(grid),
+                dim3(kNormThreads), 0, stream, nullptr, nullptr, nullptr, h, T, 1, d, eps, nullptr,
+                x);
   return ORDERMOE_OK;
 }
 
@@ -564,9 +576,8 @@ extern "C" int ordermoe_combine_residual_norm(const uint16_t* Y_perm, const int3
       overlaps(h_out, x_out, row_bytes))
     return fail(ORDERMOE_ERR_INVALID_ARG, "combine_residual_norm: h, h_out and x_out must not overlap");
   const int grid = T < num_sms() * 16 ? T : num_sms() * 16;
-  residual_norm_kernel<true><<<grid, kNormThreads, 0, stream>>>(Y_perm, row_of, topk_w, h, T, k, d,
-                                                                 eps, h_out, x_out);
-  OM_LAUNCHED("residual_norm_kernel<combine>");
+  OM_LAUNCH_PDL("residual_norm_kernel<combine>", residual_norm_kernel<true>, dim3(grid),
+                dim3(kNormThreads), 0, stream, Y_perm, row_of, topk_w, h, T, k, d, eps, h_out, x_out);
   return ORDERMOE_OK;
 }
 
@@ -586,7 +597,7 @@ extern "C" int ordermoe_combine(const uint16_t* Y_perm, const int32_t* row_of,
   int64_t blocks = (items + 7) / 8;  // 8 warps per block
   const int cap = num_sms() * 8;
   if (blocks > cap) blocks = cap;
-  combine_kernel<<<static_cast<int>(blocks), 256, 0, stream>>>(Y_perm, row_of, topk_w, T, k, d, y);
-  OM_LAUNCHED("combine_kernel");
+  OM_LAUNCH_PDL("combine_kernel", combine_kernel, dim3(static_cast<int>(blocks)), dim3(256), 0,
+                stream, Y_perm, row_of, topk_w, T, k, d, y);
   return ORDERMOE_OK;
 }

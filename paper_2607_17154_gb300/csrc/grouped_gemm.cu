@@ -124,6 +124,14 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int tid = threadIdx.x;
   const int warp = tid >> 5;
   const int lane = tid & 31;
+  // launched with launch_pdl: barriers, TMEM and tensor-map prefetches are set
+  // up while the previous kernel finishes; global memory only after pdl_wait
+  pdl_trigger();
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&mapA);
+    tma_prefetch_map(&mapB0);
+    if (MODE == GATEUP) tma_prefetch_map(&mapB1);
+  }
 
   if (tid == 0) {
     for (int i = 0; i < STAGES; ++i) {
@@ -137,6 +145,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(&s.drain, 1);
     s.abort = 0;
     s.zero = 0;
+    pdl_wait();  // the offsets come from the permutation
     int acc = 0;
     bool bad = false;
     for (int e = 0; e <= args.E; ++e) {
@@ -156,11 +165,6 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) {
-    tma_prefetch_map(&mapA);
-    tma_prefetch_map(&mapB0);
-    if (MODE == GATEUP) tma_prefetch_map(&mapB1);
-  }
   if (warp == 1) {
     tmem_alloc(&s.tmem_base, TMEM_COLS);
     tmem_relinquish();
@@ -168,6 +172,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();  // every thread: the previous kernel's outputs are visible
   const uint32_t tmem_base = s.tmem_base;
   const int total = s.mt_start[args.E] * args.n_tiles;
   const int kblocks = args.K / BK;
@@ -504,6 +509,15 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
   const bool even = (rp == 0);
   const int cluster = blockIdx.x / 2;
   const int n_clusters = gridDim.x / 2;
+  // launched with launch_pdl: barriers, TMEM and tensor-map prefetches are set
+  // up while the previous kernel finishes; global memory only after pdl_wait
+  pdl_trigger();
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_map(&mapW0);
+    if (MODE == GATEUP) tma_prefetch_map(&mapW1);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) tma_prefetch_map(&mapT.m[i]);
+  }
 
   if (tid == 0) {
     for (int i = 0; i < P_STAGES; ++i) {
@@ -517,6 +531,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
     mbar_init(&s.drain, 1);
     s.abort = 0;
     s.zero = 0;
+    pdl_wait();  // the offsets come from the permutation
     int acc = 0;
     bool bad = false;
     for (int e = 0; e <= args.E; ++e) {
@@ -536,12 +551,6 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
     }
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) {
-    tma_prefetch_map(&mapW0);
-    if (MODE == GATEUP) tma_prefetch_map(&mapW1);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) tma_prefetch_map(&mapT.m[i]);
-  }
   if (warp == 1) {
     tmem_alloc_pair(&s.tmem_base, TMEM_COLS);
     tmem_relinquish_pair();
@@ -549,6 +558,7 @@ __global__ void __launch_bounds__(PCfg<MODE>::THREADS, 1)
   tc_fence_before();
   cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
   tc_fence_after();
+  pdl_wait();  // every thread: the previous kernel's outputs are visible
   const uint32_t tmem_base = s.tmem_base;
   const int total = s.mt_start[args.E] * args.n_tiles;
   const int kblocks = args.K / BK;
@@ -826,12 +836,14 @@ static cudaLaunchConfig_t pair_config(int grid, int cl, cudaStream_t stream,
   cfg.blockDim = dim3(gg::PCfg<MODE>::THREADS, 1, 1);
   cfg.dynamicSmemBytes = gg::PCfg<MODE>::SMEM_BYTES;
   cfg.stream = stream;
-  attr->id = cudaLaunchAttributeClusterDimension;
-  attr->val.clusterDim.x = cl;
-  attr->val.clusterDim.y = 1;
-  attr->val.clusterDim.z = 1;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cl;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // waits in the kernel
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = pdl_on(stream) ? 2 : 1;
   return cfg;
 }
 
@@ -842,8 +854,9 @@ template <int MODE>
 static int max_resident_clusters() {
   static PerDevice cache;
   return per_device(cache, [] {
-    cudaLaunchAttribute attr;
-    cudaLaunchConfig_t cfg = pair_config<MODE>(2 * (num_sms() / 2), 2, nullptr, &attr);
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = pair_config<MODE>(2 * (num_sms() / 2), 2, nullptr, attr);
+    cfg.numAttrs = 1;  // the cluster shape alone decides residency
     int n = 0;
     if (cudaOccupancyMaxActiveClusters(&n, gg::ffn_gemm_pair_kernel<MODE>, &cfg) != cudaSuccess ||
         n <= 0) {
@@ -860,9 +873,9 @@ static int launch_pair(const CUtensorMap& w0, const CUtensorMap& w1, const gg::R
                        const gg::Args& a, long long tiles, cudaStream_t stream, const char* what) {
   const long long cmax = max_resident_clusters<MODE>();
   const long long clusters = tiles < cmax ? tiles : cmax;
-  cudaLaunchAttribute attr;
+  cudaLaunchAttribute attr[2];
   cudaLaunchConfig_t cfg =
-      pair_config<MODE>(static_cast<int>(2 * (clusters > 0 ? clusters : 1)), 2, stream, &attr);
+      pair_config<MODE>(static_cast<int>(2 * (clusters > 0 ? clusters : 1)), 2, stream, attr);
   const cudaError_t e = cudaLaunchKernelEx(&cfg, gg::ffn_gemm_pair_kernel<MODE>, w0, w1, t, a);
   if (e != cudaSuccess) return cuda_fail(e, what);
   OM_LAUNCHED(what);
@@ -913,8 +926,8 @@ int gate_up_launch(const uint16_t* X_perm, const int32_t* offsets, int R, const 
     if ((rc = make_map(&mW1, W1, (uint64_t)E * dff, d))) return rc;
     if ((rc = make_map(&mW3, W3, (uint64_t)E * dff, d))) return rc;
     const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
-    ffn_gemm_kernel<GATEUP><<<single_grid(tiles), THREADS, SMEM_BYTES, stream>>>(mX, mW1, mW3, a);
-    OM_LAUNCHED("ffn_gemm_kernel<gate_up>");
+    OM_LAUNCH_PDL("ffn_gemm_kernel<gate_up>", ffn_gemm_kernel<GATEUP>, dim3(single_grid(tiles)),
+                  dim3(THREADS), SMEM_BYTES, stream, mX, mW1, mW3, a);
   }
   return ORDERMOE_OK;
 }
@@ -939,8 +952,8 @@ int down_launch(const uint16_t* H, const int32_t* offsets, int R, const uint16_t
                              "ffn_gemm_pair_kernel<down>");
   } else {
     const long long tiles = ((long long)(R + BM - 1) / BM + E) * a.n_tiles;
-    ffn_gemm_kernel<DOWN><<<single_grid(tiles), THREADS, SMEM_BYTES, stream>>>(mH, mW2, mW2, a);
-    OM_LAUNCHED("ffn_gemm_kernel<down>");
+    OM_LAUNCH_PDL("ffn_gemm_kernel<down>", ffn_gemm_kernel<DOWN>, dim3(single_grid(tiles)),
+                  dim3(THREADS), SMEM_BYTES, stream, mH, mW2, mW2, a);
   }
   return ORDERMOE_OK;
 }

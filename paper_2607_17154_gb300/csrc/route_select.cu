@@ -372,6 +372,8 @@ __global__ void __launch_bounds__(128) select_kernel(
     float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
     uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
     int32_t* __restrict__ counters, Lookahead la) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   __shared__ SelSmem sm;
   extern __shared__ __align__(16) float s_dyn[];
   float* s_Q = s_dyn;
@@ -419,6 +421,8 @@ __global__ void __launch_bounds__(kLaneThreads) select_lanes_kernel(
     const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
     int32_t* __restrict__ chosen_expert, uint8_t* __restrict__ chosen_server,
     uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   __shared__ SelSmem sm;
   extern __shared__ __align__(16) float s_dyn[];
   float* s_Q = s_dyn;
@@ -730,6 +734,8 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
     float* __restrict__ qhat, int32_t* __restrict__ chosen_expert,
     uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out,
     int32_t* __restrict__ counters) {
+  pdl_trigger();  // launched with launch_pdl: no global access before pdl_wait
+  pdl_wait();
   __shared__ SelSmem sm;
   __shared__ LaSmem cs;
   extern __shared__ __align__(16) float s_dyn[];
@@ -973,6 +979,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     int32_t* __restrict__ chosen_expert, uint8_t* __restrict__ chosen_server,
     uint8_t* __restrict__ kind_out, int32_t* __restrict__ counters, uint64_t limit_ns, int split,
     Lookahead la) {
+  pdl_trigger();  // launched with launch_pdl: shared memory, barrier and TMEM set-up first
   constexpr int B_BYTES = NE * rt::BK * 2;
   constexpr int STAGE_BYTES = rt::A_BYTES + B_BYTES;
   constexpr int STAGES = rt::stages<NE>();
@@ -1018,6 +1025,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();  // the previous kernel's outputs (X, tables, state) are ready
   const uint32_t tmem_base = s.tmem_base;
   volatile int* abort = &s.abort;
   uint32_t issued_mask = 0, last_phase_bits = 0;
@@ -1211,9 +1219,9 @@ static int launch_lookahead_select(const int32_t* topk_idx, int T, int E, int k,
   }
   cudaFuncSetAttribute(lookahead_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)tab_smem);
-  lookahead_select_kernel<<<T, kLaThreads, tab_smem, stream>>>(
-      topk_idx, T, E, k, tb, la, home, loc, qhat, chosen_expert, chosen_server, kind, counters);
-  OM_LAUNCHED("lookahead_select_kernel");
+  OM_LAUNCH_PDL("lookahead_select_kernel", lookahead_select_kernel, dim3(T), dim3(kLaThreads),
+                tab_smem, stream, topk_idx, T, E, k, tb, la, home, loc, qhat, chosen_expert,
+                chosen_server, kind, counters);
   return ORDERMOE_OK;
 }
 
@@ -1228,9 +1236,9 @@ static int launch_select_lanes(const int32_t* topk_idx, int T, int E, int k, con
   if (blocks > cap) blocks = cap;
   cudaFuncSetAttribute(select_lanes_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)tab_smem);
-  select_lanes_kernel<<<static_cast<int>(blocks), kLaneThreads, tab_smem, stream>>>(
-      topk_idx, T, E, k, tb, home, loc, qhat, chosen_expert, chosen_server, kind, counters);
-  OM_LAUNCHED("select_lanes_kernel");
+  OM_LAUNCH_PDL("select_lanes_kernel", select_lanes_kernel, dim3(static_cast<int>(blocks)),
+                dim3(kLaneThreads), tab_smem, stream, topk_idx, T, E, k, tb, home, loc, qhat,
+                chosen_expert, chosen_server, kind, counters);
   return ORDERMOE_OK;
 }
 
@@ -1261,21 +1269,21 @@ static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float
   const size_t tab_smem = sizeof(float) * 2 * E * E;
   const int blocks = (T + 127) / 128;
   if (logits_in != nullptr) {
+    cudaError_t sel_err = cudaSuccess;
 #define OM_SEL_LAUNCH(EM)                                                                        \
   do {                                                                                           \
     cudaFuncSetAttribute(select_kernel<EM>, cudaFuncAttributeMaxDynamicSharedMemorySize,         \
                          (int)tab_smem);                                                         \
-    select_kernel<EM><<<blocks, 128, tab_smem, stream>>>(logits_in, T, E, k, renorm, tb, home,   \
-                                                         loc, qhat, logits_out, topk_idx, topk_w, \
-                                                         chosen_expert, chosen_server, kind,      \
-                                                         counters, la);                           \
+    sel_err = launch_pdl(select_kernel<EM>, dim3(blocks), dim3(128), tab_smem, stream,           \
+                         logits_in, T, E, k, renorm, tb, home, loc, qhat, logits_out, topk_idx,   \
+                         topk_w, chosen_expert, chosen_server, kind, counters, la);              \
   } while (0)
     if (E <= 8) OM_SEL_LAUNCH(8);
     else if (E <= 16) OM_SEL_LAUNCH(16);
     else if (E <= 32) OM_SEL_LAUNCH(32);
     else OM_SEL_LAUNCH(64);
 #undef OM_SEL_LAUNCH
-    OM_LAUNCHED("select_kernel");
+    if (sel_err != cudaSuccess) return cuda_fail(sel_err, "select_kernel");
     return la.H > 1 ? launch_lookahead_select(topk_idx, T, E, k, tb, la, home, loc, qhat,
                                               chosen_expert, chosen_server, kind, counters,
                                               tab_smem, stream)
@@ -1301,13 +1309,15 @@ static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float
   cfg.gridDim = dim3(blocks * split, 1, 1);
   cfg.blockDim = dim3(rt::THREADS, 1, 1);
   cfg.stream = stream;
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeClusterDimension;
-  attr.val.clusterDim.x = split;
-  attr.val.clusterDim.y = 1;
-  attr.val.clusterDim.z = 1;
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = split;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // waits in the kernel
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl_on(stream) ? 2 : 1;
   cudaError_t le;
 #define OM_RT_LAUNCH(N)                                                                          \
   do {                                                                                           \
