@@ -94,38 +94,68 @@ struct SelSmem {
   uint8_t sublist[64 * 64];
 };
 
-// Threads t0, t0 + nt, ... of the block load the layer's tables into shared
-// memory. The E x E tables are copied with 16-byte loads, four in flight per
-// thread, where sizes and addresses allow.
+// Threads t0, t0 + nt (nt >= 64) ... of the block load the layer's tables
+// into shared memory. The header, masks and the first E x E entries are
+// loaded before any of them is used, so that their latencies overlap; the
+// E x E tables are copied with 16-byte loads where sizes and addresses
+// allow.
 __device__ bool load_tables_range(const uint8_t* __restrict__ tab, int E, SelSmem& sm, float* s_Q,
                                   float* s_Cq, int t0, int nt) {
-  const int M = reinterpret_cast<const int32_t*>(tab)[2];
-  if (reinterpret_cast<const int32_t*>(tab)[1] != E || M <= 0 || M > 32) {
-    if (blockIdx.x == 0 && t0 == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, -1);
-    return false;
-  }
   const float* gQ = reinterpret_cast<const float*>(tab + kOffQtab);
   const float* gCq = reinterpret_cast<const float*>(tab + off_cq(E));
-  for (int i = t0; i < 64; i += nt) {
-    sm.pmask[i] = reinterpret_cast<const uint32_t*>(tab + kOffPmask)[i];
-    unsigned long long sb = reinterpret_cast<const unsigned long long*>(tab + kOffSubst)[i];
-    int n = 0;
-    while (sb) {
-      const int b = __ffsll(static_cast<long long>(sb)) - 1;
-      sm.sublist[i * 64 + n++] = static_cast<uint8_t>(b);
-      sb &= sb - 1;
-    }
-    sm.nsub[i] = n;
-  }
   const int n = E * E;
   const bool vec = (n & 3) == 0 && ((reinterpret_cast<uintptr_t>(gQ) | reinterpret_cast<uintptr_t>(gCq) |
                                      reinterpret_cast<uintptr_t>(s_Q) | reinterpret_cast<uintptr_t>(s_Cq)) &
                                     15u) == 0;
+  const int Eh = reinterpret_cast<const int32_t*>(tab)[1];
+  const int M = reinterpret_cast<const int32_t*>(tab)[2];
+  uint32_t pm = 0;
+  unsigned long long sb = 0;
+  if (t0 < 64) {
+    pm = reinterpret_cast<const uint32_t*>(tab + kOffPmask)[t0];
+    sb = reinterpret_cast<const unsigned long long*>(tab + kOffSubst)[t0];
+  }
+  constexpr int kFirst = 4;  // 16-byte chunks of each table a thread loads up front
+  float4 q_first[kFirst], c_first[kFirst];
   if (vec) {
     const float4* q4 = reinterpret_cast<const float4*>(gQ);
     const float4* c4 = reinterpret_cast<const float4*>(gCq);
+#pragma unroll
+    for (int u = 0; u < kFirst; ++u) {
+      const int i = t0 + u * nt;
+      if (i < n / 4) {
+        q_first[u] = __ldg(q4 + i);
+        c_first[u] = __ldg(c4 + i);
+      }
+    }
+  }
+  if (Eh != E || M <= 0 || M > 32) {
+    if (blockIdx.x == 0 && t0 == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, -1);
+    return false;
+  }
+  if (t0 < 64) {
+    sm.pmask[t0] = pm;
+    int cnt = 0;
+    while (sb) {
+      const int b = __ffsll(static_cast<long long>(sb)) - 1;
+      sm.sublist[t0 * 64 + cnt++] = static_cast<uint8_t>(b);
+      sb &= sb - 1;
+    }
+    sm.nsub[t0] = cnt;
+  }
+  if (vec) {
+    const float4* q4 = reinterpret_cast<const float4*>(gQ);
+    const float4* c4 = reinterpret_cast<const float4*>(gCq);
+#pragma unroll
+    for (int u = 0; u < kFirst; ++u) {
+      const int i = t0 + u * nt;
+      if (i < n / 4) {
+        reinterpret_cast<float4*>(s_Q)[i] = q_first[u];
+        reinterpret_cast<float4*>(s_Cq)[i] = c_first[u];
+      }
+    }
 #pragma unroll 4
-    for (int i = t0; i < n / 4; i += nt) {
+    for (int i = t0 + kFirst * nt; i < n / 4; i += nt) {
       const float4 x = __ldg(q4 + i), y = __ldg(c4 + i);
       reinterpret_cast<float4*>(s_Q)[i] = x;
       reinterpret_cast<float4*>(s_Cq)[i] = y;
@@ -145,7 +175,23 @@ __device__ bool load_tables_range(const uint8_t* __restrict__ tab, int E, SelSme
 // if the header does not match E (reported once).
 __device__ bool load_tables(const uint8_t* __restrict__ tab, int E, SelSmem& sm, float* s_Q,
                             float* s_Cq) {
-  return load_tables_range(tab, E, sm, s_Q, s_Cq, threadIdx.x, blockDim.x);
+  return load_tables_range(tab, E, sm, s_Q, s_Cq, threadIdx.x, blockDim.x);  // blockDim.x >= 64
+}
+
+// The delay table A[a][s][m] of Eq. 38 (M^3 floats) is read once per
+// candidate (expert, server) of every slot, so the selection keeps it in
+// shared memory when it has at most kDelayStage entries (M <= 16);
+// larger tables stay in global memory. Threads t0, t0 + nt, ... copy it;
+// every thread gets the same pointer back, the one the selection reads.
+constexpr int kDelayStage = 4096;
+__device__ const float* load_delay_range(const uint8_t* __restrict__ tab, int E, float* s_A,
+                                         int t0, int nt) {
+  const int M = reinterpret_cast<const int32_t*>(tab)[2];
+  const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
+  if (M <= 0 || M > 16) return gA;
+  const int n = M * M * M;
+  for (int i = t0; i < n; i += nt) s_A[i] = gA[i];
+  return s_A;
 }
 
 // Look-ahead context (Eqs. 41-43): the tables of the next layers follow the
@@ -225,77 +271,135 @@ __device__ __forceinline__ float lookahead_cost(const Lookahead& la, const uint8
   }
 }
 
+// A token's logits in shared memory as 16-byte chunks: chunk c holds
+// logits 4c .. 4c + 3 (-inf past E), at p[128 c] (one thread's column of a
+// [chunk][128 tokens] array, so the 32 tokens of a warp read consecutive
+// chunks: no bank conflicts).
+struct ColLogits {
+  const float4* p;
+  __device__ __forceinline__ float4 chunk(int c) const { return p[c * 128]; }
+};
+
+// The KN largest of the token's nc chunks of logits by (logit desc, index
+// asc) into v[0..KN), ix[0..KN), as a sorted list built by inserting the
+// logits in index order: logit e goes to the first position whose value it
+// exceeds, so an equal value stays behind the earlier index, and the entries
+// from that position on move down one. The positions it exceeds form a
+// suffix of the list (g[p] implies g[p+1]), which makes every position one
+// select of its own value, the new logit or its predecessor; positions
+// p >= e are still empty when logit e arrives. The list stays in registers
+// (compile-time positions), nothing branches inside a chunk, and the loop
+// over chunks keeps the code short (a long unrolled form stalled on
+// instruction fetch). The -inf logits past E go behind every real one, so
+// the first k <= E entries are real. Returns whether a logit was NaN.
+template <int KN, class Src>
+__device__ __forceinline__ bool topk_list(const Src& src, int nc, float (&v)[ORDERMOE_MAX_TOPK],
+                                          int (&ix)[ORDERMOE_MAX_TOPK]) {
+#pragma unroll
+  for (int p = 0; p < ORDERMOE_MAX_TOPK; ++p) {
+    v[p] = -INFINITY;
+    ix[p] = -1;
+  }
+  bool nan = false;
+#pragma unroll 1
+  for (int c4 = 0; c4 < nc; ++c4) {
+    const float4 x4 = src.chunk(c4);
+    const float xs[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float c = xs[u];
+      const int e = 4 * c4 + u;
+      nan |= isnan(c);
+      bool g[KN];
+#pragma unroll
+      for (int p = 0; p < KN; ++p) g[p] = (p >= e) | (c > v[p]);
+#pragma unroll
+      for (int p = KN - 1; p >= 1; --p) {
+        const float tv = g[p] ? c : v[p];
+        const int ti = g[p] ? e : ix[p];
+        v[p] = g[p - 1] ? v[p - 1] : tv;
+        ix[p] = g[p - 1] ? ix[p - 1] : ti;
+      }
+      v[0] = g[0] ? c : v[0];
+      ix[0] = g[0] ? e : ix[0];
+    }
+  }
+  return nan;
+}
+
 // One token: softmax over E, top-k, then Alg. 2 (H = 1) per slot in rank
-// order (Eqs. 36-44). The logits are in registers (lg[e], e < E <= EMAX).
-// The argmin of Eq. 43 packs (fp32 cost bits, substitute, away, server,
-// expert) into a 64-bit key and keeps the smallest; costs are never
-// negative, so the bit pattern orders them like the values.
-template <int EMAX>
+// order (Eqs. 36-44). src gives the logits in 16-byte chunks (ColLogits).
+// The caller loads the token's home a, location s (Eq. 36: a on the first
+// layer) and accumulated loss q. Atab is the delay table of Eq. 38, in
+// shared or global memory. The argmin of Eq. 43 packs (fp32 cost bits,
+// substitute, away, server, expert) into a 64-bit key and keeps the
+// smallest; costs are never negative, so the bit pattern orders them like
+// the values.
+template <class Src>
 __device__ __forceinline__ void select_token(
-    int t, const float (&lg)[EMAX], int E, int k, int renorm, int M, float qbar,
-    const float* __restrict__ gA, const uint8_t* __restrict__ tab, const Lookahead& la,
-    const SelSmem& sm, const float* s_Q, const float* s_Cq,
-    const uint8_t* __restrict__ home, uint8_t* __restrict__ loc, float* __restrict__ qhat,
+    int t, const Src& src, int E, int k, int renorm, int M, float qbar,
+    const float* Atab, const uint8_t* __restrict__ tab, const Lookahead& la,
+    const SelSmem& sm, const float* s_Q, const float* s_Cq, int a, int s, float q,
+    uint8_t* __restrict__ loc, float* __restrict__ qhat,
     int32_t* __restrict__ topk_idx, float* __restrict__ topk_w, int32_t* __restrict__ chosen_expert,
     uint8_t* __restrict__ chosen_server, uint8_t* __restrict__ kind_out, int (&kind_count)[4],
     bool topk_only = false) {
-#pragma unroll
-  for (int e = 0; e < EMAX; ++e)
-    if (e < E && isnan(lg[e])) {
-      report(&g_err_route, ORDERMOE_DEV_NAN_LOGIT, t);
-      for (int j = 0; j < k; ++j) {  // no targets: a later pass skips this token
-        topk_idx[(size_t)t * k + j] = -1;
-        topk_w[(size_t)t * k + j] = 0.0f;
-      }
-      return;
-    }
-  // top-k by (logit desc, index asc); vtop keeps each chosen logit, so no
-  // lookup lg[idx[j]] (a run-time index would put lg[] in local memory)
-  int idx[ORDERMOE_MAX_TOPK];
+  // top-k by (logit desc, index asc): a sorted list of 2, 4, 6 or 8 >= k
   float vtop[ORDERMOE_MAX_TOPK];
-  unsigned long long used_targets = 0;
-  for (int j = 0; j < k; ++j) {
-    int best = -1;
-    float bv = 0.0f;
-#pragma unroll
-    for (int e = 0; e < EMAX; ++e)
-      if (e < E && !((used_targets >> e) & 1ull) && (best < 0 || lg[e] > bv)) {
-        best = e;
-        bv = lg[e];
-      }
-    idx[j] = best;
-    vtop[j] = bv;
-    used_targets |= 1ull << best;
+  int itop[ORDERMOE_MAX_TOPK];
+  const int nc = (E + 3) / 4;
+  bool nan;
+  if (k <= 2) nan = topk_list<2>(src, nc, vtop, itop);
+  else if (k <= 4) nan = topk_list<4>(src, nc, vtop, itop);
+  else if (k <= 6) nan = topk_list<6>(src, nc, vtop, itop);
+  else nan = topk_list<8>(src, nc, vtop, itop);
+  if (nan) {
+    report(&g_err_route, ORDERMOE_DEV_NAN_LOGIT, t);
+    for (int j = 0; j < k; ++j) {  // no targets: a later pass skips this token
+      topk_idx[(size_t)t * k + j] = -1;
+      topk_w[(size_t)t * k + j] = 0.0f;
+    }
+    return;
   }
-  // softmax over all E in fp32; gate weights of the k slots
-  float lmax = -INFINITY;
-#pragma unroll
-  for (int e = 0; e < EMAX; ++e)
-    if (e < E) lmax = fmaxf(lmax, lg[e]);
+  // softmax over all E in fp32, summed in index order (the maximum is the
+  // list's head; the -inf logits past E add exact zeros after the real
+  // terms); gate weights of the k slots
+  const float lmax = vtop[0];
   float denom = 0.0f;
-#pragma unroll
-  for (int e = 0; e < EMAX; ++e)
-    if (e < E) denom += expf(lg[e] - lmax);
+#pragma unroll 1
+  for (int c4 = 0; c4 < nc; ++c4) {
+    const float4 x4 = src.chunk(c4);
+    denom += expf(x4.x - lmax);
+    denom += expf(x4.y - lmax);
+    denom += expf(x4.z - lmax);
+    denom += expf(x4.w - lmax);
+  }
   float wsel[ORDERMOE_MAX_TOPK];
   float ssel = 0.0f;
-  for (int j = 0; j < k; ++j) {
-    wsel[j] = expf(vtop[j] - lmax) / denom;
-    ssel += wsel[j];
-  }
-  for (int j = 0; j < k; ++j) {
-    topk_idx[(size_t)t * k + j] = idx[j];
-    topk_w[(size_t)t * k + j] = renorm ? wsel[j] / ssel : wsel[j];
+#pragma unroll
+  for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j)
+    if (j < k) {
+      wsel[j] = expf(vtop[j] - lmax) / denom;
+      ssel += wsel[j];
+    }
+  int idx[ORDERMOE_MAX_TOPK];
+  unsigned long long used_targets = 0;
+#pragma unroll
+  for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
+    idx[j] = itop[j];
+    if (j < k) {
+      topk_idx[(size_t)t * k + j] = itop[j];
+      topk_w[(size_t)t * k + j] = renorm ? wsel[j] / ssel : wsel[j];
+      used_targets |= 1ull << itop[j];
+    }
   }
   if (topk_only) return;
   // selection
-  const int a = home[t];
-  const int s = (loc != nullptr) ? loc[t] : a;  // no state given: first layer (Eq. 36)
   if (a >= M || s >= M) {
     report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
     return;
   }
-  const float* Aas = gA + ((size_t)a * M + s) * M;
-  float q = (qhat != nullptr) ? qhat[t] : 0.0f;
+  const float* Aas = Atab + (a * M + s) * M;
   unsigned long long taken = used_targets;
   int first_server = s;
   for (int j = 0; j < k; ++j) {
@@ -316,7 +420,7 @@ __device__ __forceinline__ void select_token(
       while (pm) {
         const int m = __ffs(pm) - 1;
         pm &= pm - 1;
-        float cost = __fadd_rn(__ldg(Aas + m), cq);
+        float cost = __fadd_rn(Aas[m], cq);
         if (la.H > 1) cost = __fadd_rn(cost, lookahead_cost(la, tab, E, M, a, m, kk, qn, qbar));
         const unsigned long long key =
             (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
@@ -376,27 +480,39 @@ __global__ void __launch_bounds__(128) select_kernel(
   pdl_wait();
   __shared__ SelSmem sm;
   extern __shared__ __align__(16) float s_dyn[];
-  float* s_Q = s_dyn;
-  float* s_Cq = s_dyn + E * E;
+  float4* s_lg = reinterpret_cast<float4*>(s_dyn);  // [EMAX / 4][128] chunks of logits
+  float* s_Q = s_dyn + EMAX * 128;
+  float* s_Cq = s_Q + E * E;
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  // the token's state first: its loads overlap the tables'
+  int a = 0, sl = 0;
+  float q0 = 0.0f;
+  if (t < T && la.H == 1) {
+    a = home[t];
+    sl = (loc != nullptr) ? loc[t] : a;  // no state given: first layer (Eq. 36)
+    q0 = (qhat != nullptr) ? qhat[t] : 0.0f;
+  }
   if (!load_tables(tab, E, sm, s_Q, s_Cq)) return;
+  const float* Atab = load_delay_range(tab, E, s_Cq + E * E, threadIdx.x, blockDim.x);
   __syncthreads();
   const int M = reinterpret_cast<const int32_t*>(tab)[2];
   const float qbar = reinterpret_cast<const float*>(tab)[5];
-  const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
   int kind_count[4] = {0, 0, 0, 0};
-  const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t < T) {
     float lg[EMAX];
 #pragma unroll
-    for (int e = 0; e < EMAX; ++e) lg[e] = (e < E) ? logits_in[(size_t)t * E + e] : 0.0f;
+    for (int e = 0; e < EMAX; ++e) lg[e] = (e < E) ? logits_in[(size_t)t * E + e] : -INFINITY;
     if (logits_out != nullptr) {
 #pragma unroll
       for (int e = 0; e < EMAX; ++e)  // constant indices keep lg[] in registers
         if (e < E) logits_out[(size_t)t * E + e] = lg[e];
     }
-    select_token<EMAX>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
-                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count,
-                       la.H > 1);
+#pragma unroll
+    for (int c = 0; c < EMAX; c += 4)
+      s_lg[(c / 4) * 128 + threadIdx.x] = make_float4(lg[c], lg[c + 1], lg[c + 2], lg[c + 3]);
+    select_token(t, ColLogits{s_lg + threadIdx.x}, E, k, renorm, M, qbar, Atab, tab, la, sm, s_Q,
+                 s_Cq, a, sl, q0, loc, qhat, topk_idx, topk_w, chosen_expert, chosen_server,
+                 kind_out, kind_count, la.H > 1);
   }
   flush_kind_counts(sm, kind_count, counters);
   __syncthreads();
@@ -428,10 +544,12 @@ __global__ void __launch_bounds__(kLaneThreads) select_lanes_kernel(
   float* s_Q = s_dyn;
   float* s_Cq = s_dyn + E * E;
   if (!load_tables(tab, E, sm, s_Q, s_Cq)) return;
+  // the delay table stays in global memory here: staging it took longer
+  // than the reads it saves (one per candidate, eight lanes at a time)
+  const float* Atab = reinterpret_cast<const float*>(tab + off_a(E));
   __syncthreads();
   const int M = reinterpret_cast<const int32_t*>(tab)[2];
   const float qbar = reinterpret_cast<const float*>(tab)[5];
-  const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
   const int lane = threadIdx.x & 31;
   const int sub = lane & 7;       // lane within the token's group of eight
   const int grp = lane >> 3;
@@ -443,25 +561,29 @@ __global__ void __launch_bounds__(kLaneThreads) select_lanes_kernel(
     // every lane runs every slot (the butterflies need the whole warp);
     // inactive tokens (past T, a NaN token's -1 targets, bad servers) write nothing
     bool active = t < T;
+    // the token's state and targets, loaded together
+    int a = 0, s = 0;
+    float q = 0.0f;
+    if (active) {
+      a = home[t];
+      s = (loc != nullptr) ? loc[t] : a;
+      q = (qhat != nullptr) ? qhat[t] : 0.0f;
+    }
     int idx[ORDERMOE_MAX_TOPK];
     unsigned long long taken = 0;
 #pragma unroll
-    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
-      idx[j] = 0;
+    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) idx[j] = (j < k && active) ? topk_idx[(size_t)t * k + j] : 0;
+#pragma unroll
+    for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j)
       if (j < k && active) {
-        const int r = topk_idx[(size_t)t * k + j];
-        if (r < 0 || r >= E) active = false;
-        else { idx[j] = r; taken |= 1ull << r; }
+        if (idx[j] < 0 || idx[j] >= E) active = false;
+        else taken |= 1ull << idx[j];
       }
-    }
-    const int a = active ? home[t] : 0;
-    const int s = active ? ((loc != nullptr) ? loc[t] : a) : 0;
     if (active && (a >= M || s >= M)) {
       if (sub == 0) report(&g_err_route, ORDERMOE_DEV_BAD_INDEX, t);
       active = false;
     }
-    const float* Aas = gA + ((size_t)a * M + s) * M;
-    float q = (active && qhat != nullptr) ? qhat[t] : 0.0f;
+    const float* Aas = Atab + (active ? (a * M + s) * M : 0);
     int first_server = s;
 #pragma unroll
     for (int j = 0; j < ORDERMOE_MAX_TOPK; ++j) {
@@ -482,7 +604,7 @@ __global__ void __launch_bounds__(kLaneThreads) select_lanes_kernel(
         while (pm) {
           const int m = __ffs(pm) - 1;
           pm &= pm - 1;
-          const float cost = __fadd_rn(__ldg(Aas + m), cq);
+          const float cost = __fadd_rn(Aas[m], cq);
           const unsigned long long key =
               (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
               (static_cast<unsigned long long>(issub ? 1u : 0u) << 31) |
@@ -939,7 +1061,12 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
 // 32 (w % 4) + i); ranks > 0 store their partial logits into rank 0's shared
 // memory (distributed shared memory), and after a cluster barrier rank 0 adds
 // the partials in rank order (deterministic) and runs select_token. Splitting
-// K lets a few hundred tokens (decode) still stream X over many SMs.
+// K lets a few hundred tokens (decode) still stream X over many SMs. The
+// partials are laid out [rank - 1][NE / 4][128 tokens][4], so that the 32
+// tokens of a warp store and load 16-byte vectors at consecutive addresses
+// (no bank conflicts). While the TMA and MMA warps run, rank 0's epilogue
+// warps load the selection tables (the delay table too, when small) and
+// each token's home, location and loss.
 // Warp 0 issues the TMA loads (X: 128 x 64 box; W_r: NE x 64 box, rows >= E
 // zero-filled), warp 1 the MMAs; mbarrier ring; bounded waits.
 namespace rt {
@@ -947,16 +1074,20 @@ constexpr int BK = 64;
 constexpr int A_BYTES = 128 * BK * 2;
 constexpr int THREADS = 192;
 // stages of (16 KB + NE x 128 B) in flight per CTA, and the largest cluster,
-// sized so the ring, the partial-logit buffer and the tables fit in 227 KB
+// sized so the ring, the partial logits of ranks 1..S-1, the tables and the
+// staged delay table fit in 227 KB beside the static selection tables
 template <int NE>
-constexpr int stages() { return NE <= 16 ? 8 : (NE <= 32 ? 6 : 4); }
+constexpr int stages() { return NE <= 16 ? 8 : (NE <= 32 ? 7 : 5); }
 template <int NE>
 constexpr int max_split() { return NE <= 16 ? 8 : (NE <= 32 ? 4 : 2); }
 template <int NE>
 constexpr int smem_bytes(int E) {
-  return 1024 + stages<NE>() * (A_BYTES + NE * BK * 2) + 256 + max_split<NE>() * 128 * NE * 4 +
-         8 * E * E;
+  return 1024 + stages<NE>() * (A_BYTES + NE * BK * 2) + 256 +
+         (max_split<NE>() - 1) * 128 * NE * 4 + 8 * E * E + 4 * kDelayStage;
 }
+static_assert(smem_bytes<16>(16) + sizeof(SelSmem) <= 227 * 1024, "router shared memory");
+static_assert(smem_bytes<32>(32) + sizeof(SelSmem) <= 227 * 1024, "router shared memory");
+static_assert(smem_bytes<64>(64) + sizeof(SelSmem) <= 227 * 1024, "router shared memory");
 }  // namespace rt
 
 template <int NE>
@@ -988,9 +1119,11 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
   uint8_t* tiles = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   RouterSmem<NE>& s = *reinterpret_cast<RouterSmem<NE>*>(tiles + STAGES * STAGE_BYTES);
-  float* red = reinterpret_cast<float*>(tiles + STAGES * STAGE_BYTES + 256);  // [split][128][NE]
-  float* s_Q = red + rt::max_split<NE>() * 128 * NE;
+  // partials of ranks 1..split-1: [split - 1][NE / 4][128][4]
+  float* red = reinterpret_cast<float*>(tiles + STAGES * STAGE_BYTES + 256);
+  float* s_Q = red + (rt::max_split<NE>() - 1) * 128 * NE;
   float* s_Cq = s_Q + E * E;
+  float* s_A = s_Cq + E * E;
   __shared__ SelSmem sm;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t rank = split > 1 ? cluster_ctarank() : 0;
@@ -1022,6 +1155,9 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     tmem_relinquish();
   }
   bool tables_ok = true;  // rank 0's epilogue warps load the tables during the main loop
+  const float* Atab = nullptr;
+  int pre_a = 0, pre_s = 0;  // the token's home and location, loaded during the main loop
+  float pre_q = 0.0f;
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -1087,7 +1223,14 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       if (la.H > 1 || la.topk_only) {  // targets only: a selection kernel reads the tables
         if (tid - 64 < 4) sm.kind[tid - 64] = 0;
       } else {
+        const int t = m0 + (warp & 3) * 32 + lane;
+        if (t < T) {
+          pre_a = home[t];
+          pre_s = (loc != nullptr) ? loc[t] : pre_a;  // no state given: first layer (Eq. 36)
+          pre_q = (qhat != nullptr) ? qhat[t] : 0.0f;
+        }
         tables_ok = load_tables_range(tab, E, sm, s_Q, s_Cq, tid - 64, 128);
+        Atab = load_delay_range(tab, E, s_A, tid - 64, 128);
       }
     }
     asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -1111,11 +1254,13 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       }
       tc_fence_before();
       if (rank > 0) {
-        // partial logits of this rank -> red[rank][row][:] in rank 0's shared memory
-        const uint32_t dst = mapa_shared(smem_u32(red + ((size_t)rank * 128 + row) * NE), 0);
+        // partial logits of this rank -> red[rank - 1][c / 4][row][c % 4] in rank 0's
+        // shared memory
+        const uint32_t dst =
+            mapa_shared(smem_u32(red + ((size_t)(rank - 1) * (NE / 4) * 128 + row) * 4), 0);
 #pragma unroll
         for (int c = 0; c < NE; c += 4)
-          asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(dst + c * 4),
+          asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(dst + c * 128 * 4),
                        "f"(lg[c]), "f"(lg[c + 1]), "f"(lg[c + 2]), "f"(lg[c + 3])
                        : "memory");
       }
@@ -1128,22 +1273,35 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     const int row = q * 32 + lane;
     const int t = m0 + row;
     for (int r = 1; r < split; ++r) {
-      const float* src = red + ((size_t)r * 128 + row) * NE;
+      const float4* src = reinterpret_cast<const float4*>(red) + (size_t)(r - 1) * (NE / 4) * 128 + row;
 #pragma unroll
-      for (int c = 0; c < NE; ++c) lg[c] += src[c];
+      for (int c = 0; c < NE; c += 4) {
+        const float4 p = src[(c / 4) * 128];
+        lg[c] += p.x;
+        lg[c + 1] += p.y;
+        lg[c + 2] += p.z;
+        lg[c + 3] += p.w;
+      }
     }
+#pragma unroll
+    for (int e = 0; e < NE; ++e)  // padding past E for select_token
+      if (e >= E) lg[e] = -INFINITY;
     if (t < T && tables_ok) {
       if (logits_out != nullptr) {
 #pragma unroll
         for (int e = 0; e < NE; ++e)  // constant indices keep lg[] in registers
           if (e < E) logits_out[(size_t)t * E + e] = lg[e];
       }
+      // the token's logits into this thread's column of partial slot 0 (read above)
+      float4* col = reinterpret_cast<float4*>(red) + row;
+#pragma unroll
+      for (int c = 0; c < NE; c += 4)
+        col[(c / 4) * 128] = make_float4(lg[c], lg[c + 1], lg[c + 2], lg[c + 3]);
       const int M = reinterpret_cast<const int32_t*>(tab)[2];
       const float qbar = reinterpret_cast<const float*>(tab)[5];
-      const float* gA = reinterpret_cast<const float*>(tab + off_a(E));
-      select_token<NE>(t, lg, E, k, renorm, M, qbar, gA, tab, la, sm, s_Q, s_Cq, home, loc, qhat,
-                       topk_idx, topk_w, chosen_expert, chosen_server, kind_out, kind_count,
-                       la.H > 1 || la.topk_only);
+      select_token(t, ColLogits{col}, E, k, renorm, M, qbar, Atab, tab, la, sm, s_Q, s_Cq, pre_a,
+                   pre_s, pre_q, loc, qhat, topk_idx, topk_w, chosen_expert, chosen_server,
+                   kind_out, kind_count, la.H > 1 || la.topk_only);
     }
     flush_kind_counts(sm, kind_count, counters);
   }
@@ -1266,15 +1424,17 @@ static int route_select_impl(const uint16_t* X, const uint16_t* W_r, const float
     return fail(ORDERMOE_ERR_INVALID_ARG, "route_select: tables buffer smaller than E needs");
   if (T == 0) return ORDERMOE_OK;
   const uint8_t* tb = static_cast<const uint8_t*>(tables);
-  const size_t tab_smem = sizeof(float) * 2 * E * E;
+  const size_t tab_smem = sizeof(float) * 2 * E * E;  // the look-ahead and lane kernels'
+  const size_t sel_smem = tab_smem + sizeof(float) * kDelayStage;  // + the staged delay table
   const int blocks = (T + 127) / 128;
   if (logits_in != nullptr) {
     cudaError_t sel_err = cudaSuccess;
 #define OM_SEL_LAUNCH(EM)                                                                        \
   do {                                                                                           \
+    const size_t lg_smem = sel_smem + sizeof(float) * EM * 128; /* + the logits' chunks */      \
     cudaFuncSetAttribute(select_kernel<EM>, cudaFuncAttributeMaxDynamicSharedMemorySize,         \
-                         (int)tab_smem);                                                         \
-    sel_err = launch_pdl(select_kernel<EM>, dim3(blocks), dim3(128), tab_smem, stream,           \
+                         (int)lg_smem);                                                          \
+    sel_err = launch_pdl(select_kernel<EM>, dim3(blocks), dim3(128), lg_smem, stream,            \
                          logits_in, T, E, k, renorm, tb, home, loc, qhat, logits_out, topk_idx,   \
                          topk_w, chosen_expert, chosen_server, kind, counters, la);              \
   } while (0)
