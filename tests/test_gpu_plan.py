@@ -435,41 +435,101 @@ def test_redundant_plan_at_memory_ratio_two_raises_coverage():
     np.testing.assert_array_equal(reps.cpu().numpy(), ref[2])
 
 
-def test_similarity_full_size_sampled():
-    """The similarity workload: 24 layers x 64 clustered experts, d = 2048,
-    N = 262144 calibration tokens. Checked on sampled expert pairs (the oracle
-    computes the rows of H it needs), plus properties that hold at any size,
-    then the GPU plan's groups and placement."""
+def test_similarity_full_size():
+    """The similarity workload at full size: 24 layers x 64 clustered experts,
+    d = 2048, N = 262144 calibration tokens (Eqs. 3-5), then Alg. 1 on the
+    GPU's own similarities and counts (Eqs. 24-35).
+    - Eq. 3: the GPU's fp32 calibration logits on 512 sampled tokens of two
+      layers against the oracle's fp64 sums;
+    - Eq. 5: the counts of every layer recomputed by the oracle from the GPU's
+      own fp32 logits, bit for bit (the same top-k and tie rule on the same
+      inputs);
+    - Eq. 4: one whole 64 x 64 layer of Sim against the fp64 oracle within
+      2e-5, and sampled expert pairs of two more layers;
+    - Eqs. 24-31: grouping, theta_l, importance and placement of every layer,
+      and (Eqs. 32-35) the replicas and local group coverage at memory ratio
+      2.0, each from the oracle run on the GPU's similarities and counts, bit
+      for bit;
+    - properties at any size: symmetry, |Sim| <= 1, counts summing to N k, the
+      8 router clusters recovered as groups, c.1 and c.2."""
     w = synth.workload("similarity")
-    L, E, d, N = w.L, w.E, w.d, w.n_cal
+    L, E, d, N, M, kf = w.L, w.E, w.d, w.n_cal, w.M, w.k
     Wr = torch.stack([synth.router_weights(E, d, w.n_clusters, seed=500 + l, device=DEV)
                       for l in range(L)])
     Xcal = synth.calibration(N, d, seed=1, device=DEV)
-    sim, counts = gpu_similarity(Wr, Xcal, w.k)
+    sim_t = torch.empty(L, E, E, dtype=torch.float32, device=DEV)
+    counts_t = torch.empty(L, E, dtype=torch.int32, device=DEV)
+    ws = torch.empty(B.ordermoe_similarity_workspace_bytes(L, E, N), dtype=torch.uint8, device=DEV)
+    B.ordermoe_similarity(Wr, Xcal, L, E, d, N, kf, sim_t, counts_t, ws)
+    torch.cuda.synchronize()
+    sim, counts = sim_t.cpu().numpy(), counts_t.cpu().numpy()
+    logits = ws[:N * L * E * 4].view(torch.float32).view(N, L, E).cpu().numpy()
+    del ws
     assert np.allclose(sim, np.transpose(sim, (0, 2, 1)), atol=1e-6)
     assert (np.abs(sim) <= 1 + 1e-6).all()
-    assert (counts.sum(axis=1) == N * w.k).all()
+    assert (counts.sum(axis=1) == N * kf).all()
     rng = np.random.default_rng(0)
     Xb = synth.bits(Xcal)
-    for l in (0, 13, 23):
+    tok = np.sort(rng.choice(N, 512, replace=False))
+    for l in (0, 23):
+        ref = oracle.router_logits(Xb[tok], synth.bits(Wr[l]))
+        np.testing.assert_allclose(logits[tok, l, :], ref, rtol=1e-3, atol=2e-3)
+    for l in range(L):
+        ref = oracle.expert_counts(np.ascontiguousarray(logits[:, l, :]), kf)
+        np.testing.assert_array_equal(counts[l], ref, err_msg="counts of layer %d" % l)
+    del logits
+    np.testing.assert_allclose(sim[7], oracle.similarity(synth.bits(Wr[7]), Xb), atol=2e-5)
+    for l in (0, 23):
         ex = np.sort(rng.choice(E, 3, replace=False))
         ref = oracle.similarity(synth.bits(Wr[l][ex]), Xb)
         np.testing.assert_allclose(sim[l][np.ix_(ex, ex)], ref, atol=2e-5)
-    # the GPU plan: every layer recovers the 8 router clusters (cosine ~0.94
-    # inside a cluster, ~0 across, against theta_l in [0.5, 0.9])
-    p = np.ones((L, E)); C = np.full(w.M, L * E / w.M)
-    group, ng, theta, x, used, st = gpu_place(sim, counts, w.M, p, C, w.theta_min, w.theta_max)
-    assert st == 0 and (ng == w.n_clusters).all()
+    # Alg. 1 on the GPU's similarities and counts, at memory ratio 2.0
+    p = np.ones((L, E)); C = synth.capacities(M, L * E, 2.0, 3)
+    t = lambda a, dt: torch.as_tensor(np.ascontiguousarray(a)).to(device=DEV, dtype=dt)
+    group = torch.empty(L, E, dtype=torch.int32, device=DEV)
+    ng = torch.empty(L, dtype=torch.int32, device=DEV)
+    theta = torch.empty(L, dtype=torch.float32, device=DEV)
+    imp = torch.empty(L, E, dtype=torch.float64, device=DEV)
+    x = torch.empty(L, M, E, dtype=torch.uint8, device=DEV)
+    used = torch.empty(M, dtype=torch.float64, device=DEV)
+    st = torch.empty(1, dtype=torch.int32, device=DEV)
+    gp, gC = t(p, torch.float64), t(C, torch.float64)
+    B.ordermoe_place(sim_t, counts_t, L, E, M, w.theta_min, w.theta_max, w.theta, 0.5, 0.5, 0.5,
+                     0.5, gp, gC, group, ng, theta, imp, x, used, st)
+    torch.cuda.synchronize()
+    got = (group.cpu().numpy(), ng.cpu().numpy(), theta.cpu().numpy(), x.cpu().numpy(),
+           used.cpu().numpy(), int(st.item()))
+    ref = oracle_place_all(sim, counts, M, p, C, w.theta_min, w.theta_max, w.theta)
+    for name, a, b in zip(("group", "n_groups", "theta", "placement", "used", "status"), got, ref):
+        np.testing.assert_array_equal(a, b, err_msg=name)
+    ref_imp = np.stack([oracle.importance(sim[l], counts[l], ref[0][l]) for l in range(L)])
+    np.testing.assert_array_equal(imp.cpu().numpy(), ref_imp)
+    pi = synth.token_shares(synth.homes(8192, M, 3, "zipf1.1"), M)
+    reps = torch.empty(M, dtype=torch.int32, device=DEV)
+    B.ordermoe_replicate(group, imp, gp, gC, t(pi, torch.float64), L, E, M, x, used, reps)
+    cov = torch.empty(L, M, E, dtype=torch.uint8, device=DEV)
+    covered = torch.empty(L, dtype=torch.int32, device=DEV)
+    B.ordermoe_coverage(group, x, L, E, M, cov, covered)
+    torch.cuda.synchronize()
+    rx, rused, rreps = oracle.replicate(ref[0], ref_imp, p, C, pi, ref[3], ref[4])
+    np.testing.assert_array_equal(x.cpu().numpy(), rx)
+    np.testing.assert_array_equal(used.cpu().numpy(), rused)
+    np.testing.assert_array_equal(reps.cpu().numpy(), rreps)
+    gcov = cov.cpu().numpy()
+    for l in range(L):
+        rc = oracle.coverage(rx[l], ref[0][l], E)
+        np.testing.assert_array_equal(gcov[l], rc, err_msg="coverage of layer %d" % l)
+        assert covered[l].item() == int(rc.sum())
+    # what the workload is built to show: the 8 router clusters (cosine ~0.94
+    # inside a cluster, ~0 across, against theta_l in [0.5, 0.9]) become the
+    # groups, every expert placed once (c.2), no server over capacity (c.1)
+    gr = ref[0]
+    assert ref[5] == 0 and (ref[1] == w.n_clusters).all()
     cl = synth.cluster_of(E, w.n_clusters)
     for l in range(L):
-        same = group[l][:, None] == group[l][None, :]
-        np.testing.assert_array_equal(same, cl[:, None] == cl[None, :])
-    assert (x.sum(axis=1) == 1).all()                    # c.2
-    np.testing.assert_allclose(used, np.einsum("lme,le->m", x.astype(float), p))
-    assert (used <= C).all()                              # c.1
-    # same-group dispersion (Eq. 30): servers cover most groups locally
-    cov = np.mean([oracle.coverage(x[l], group[l], w.n_clusters).mean() for l in range(L)])
-    assert cov >= 0.9, cov
+        np.testing.assert_array_equal(gr[l][:, None] == gr[l][None, :], cl[:, None] == cl[None, :])
+    assert (ref[3].sum(axis=1) == 1).all()
+    assert (rused <= C + 1e-9).all()
 
 
 # ------------------------------------------------------------------ whole-layer entry
