@@ -1073,17 +1073,23 @@ namespace rt {
 constexpr int BK = 64;
 constexpr int A_BYTES = 128 * BK * 2;
 constexpr int THREADS = 192;
-// stages of (16 KB + NE x 128 B) in flight per CTA, and the largest cluster,
-// sized so the ring, the partial logits of ranks 1..S-1, the tables and the
-// staged delay table fit in 227 KB beside the static selection tables
+// Only layers of up to 16 experts (NE = 16) select inside the router; for
+// more experts it writes the targets and a selection kernel selects, so the
+// wider instantiations keep no tables and give that space to the X ring.
 template <int NE>
-constexpr int stages() { return NE <= 16 ? 8 : (NE <= 32 ? 7 : 5); }
+constexpr bool selects() { return NE <= 16; }
+// stages of (16 KB + NE x 128 B) in flight per CTA, and the largest cluster,
+// sized so the ring, the partial logits of ranks 1..S-1 and (NE = 16) the
+// tables and the staged delay table fit in 227 KB beside the static
+// selection tables
+template <int NE>
+constexpr int stages() { return NE <= 16 ? 8 : (NE <= 32 ? 8 : 7); }
 template <int NE>
 constexpr int max_split() { return NE <= 16 ? 8 : (NE <= 32 ? 4 : 2); }
 template <int NE>
 constexpr int smem_bytes(int E) {
   return 1024 + stages<NE>() * (A_BYTES + NE * BK * 2) + 256 +
-         (max_split<NE>() - 1) * 128 * NE * 4 + 8 * E * E + 4 * kDelayStage;
+         (max_split<NE>() - 1) * 128 * NE * 4 + (selects<NE>() ? 8 * E * E + 4 * kDelayStage : 0);
 }
 static_assert(smem_bytes<16>(16) + sizeof(SelSmem) <= 227 * 1024, "router shared memory");
 static_assert(smem_bytes<32>(32) + sizeof(SelSmem) <= 227 * 1024, "router shared memory");
@@ -1220,7 +1226,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
     // the selection tables, while the TMA and MMA warps run (named barrier 1:
     // the 128 epilogue threads)
     if (rank == 0) {
-      if (la.H > 1 || la.topk_only) {  // targets only: a selection kernel reads the tables
+      if (!rt::selects<NE>() || la.H > 1 || la.topk_only) {  // targets only: a selection kernel reads the tables
         if (tid - 64 < 4) sm.kind[tid - 64] = 0;
       } else {
         const int t = m0 + (warp & 3) * 32 + lane;
@@ -1301,7 +1307,7 @@ __global__ void __launch_bounds__(rt::THREADS, 1) router_select_kernel(
       const float qbar = reinterpret_cast<const float*>(tab)[5];
       select_token(t, ColLogits{col}, E, k, renorm, M, qbar, Atab, tab, la, sm, s_Q, s_Cq, pre_a,
                    pre_s, pre_q, loc, qhat, topk_idx, topk_w, chosen_expert, chosen_server,
-                   kind_out, kind_count, la.H > 1 || la.topk_only);
+                   kind_out, kind_count, !rt::selects<NE>() || la.H > 1 || la.topk_only);
     }
     flush_kind_counts(sm, kind_count, counters);
   }
