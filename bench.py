@@ -356,7 +356,7 @@ def run_ours(args, dist):
     # batch's copies overlapping its neighbours' compute
     e2e = None
     if not args.no_e2e:
-        E2E_QUEUE = 8
+        E2E_QUEUE = 16
         scratch = torch.empty(B.ordermoe_layer_batches_scratch_bytes(T, E, d, dff, k),
                               dtype=torch.uint8, device=device)
         desc = B.make_layer_desc(T, Wr, W1, W3, W2, tables, k, scratch)

@@ -153,6 +153,53 @@ def test_router_logits_match_oracle(T, d, E):
     np.testing.assert_array_equal(outs[4].cpu().numpy(), kd)
 
 
+@pytest.mark.parametrize("E,k", [(8, 1), (13, 3), (16, 5), (16, 7), (16, 8), (32, 4), (64, 6),
+                                 (64, 8)])
+def test_router_exact_ties_every_list_width(E, k):
+    """Router rows copied in groups of 2 and 3 alternately (each row of a group
+    equal to the group's first), so every logit the tensor-core router
+    computes has bitwise-equal siblings and, for every k, equal logits
+    straddle the k-th rank for some tokens: the top-k (a sorted list of 2, 4,
+    6 or 8 entries; E not a multiple of 4 padded with -inf) must keep the lower
+    index first, as the oracle does on the GPU's own logits (Alg. 2's
+    targets), and the selection from those targets must match bit for bit."""
+    T, d = 300, 512
+    w = synth.workload("tiny", T=T, d=d, E=E, n_clusters=1)
+    inp = synth.layer_inputs(w, seed=9, with_ffn=False)
+    lead, r, size = np.arange(E), 0, 2
+    while r < E:
+        lead[r:r + size] = r
+        r, size = r + size, 5 - size
+    Wr = inp["Wr"][torch.as_tensor(lead)].contiguous()
+    M = w.M
+    sim, group, x = random_tables_case(np.random.default_rng(E + k), E, M, 2)
+    tab = build_tables(sim, group, x, 0.5, 0.05, synth.server_params(M, d, w.dff, 0), DEV)
+    logits = torch.empty(T, E, dtype=torch.float32, device=DEV)
+    outs = [torch.empty(T, k, dtype=dt, device=DEV)
+            for dt in (torch.int32, torch.float32, torch.int32, torch.uint8, torch.uint8)]
+    home = dev(inp["home"])
+    B.ordermoe_route_select(inp["X"].to(DEV), Wr.to(DEV), None, T, E, d, k, 1, tab, home,
+                            home.clone(), torch.zeros(T, device=DEV), logits, *outs)
+    got = logits.cpu().numpy()
+    np.testing.assert_array_equal(got, got[:, lead])
+    np.testing.assert_allclose(got, oracle.router_logits(gbits(inp["X"]), gbits(Wr)), rtol=1e-3,
+                               atol=2e-3)
+    o_idx, o_w = oracle.topk(got, k, 1)
+    np.testing.assert_array_equal(outs[0].cpu().numpy(), o_idx)
+    np.testing.assert_allclose(outs[1].cpu().numpy(), o_w, rtol=1e-5, atol=1e-7)
+    # a tie at the boundary: the k-th and (k + 1)-th logits equal for some token
+    srt = -np.sort(-got, axis=1)
+    assert (srt[:, k - 1] == srt[:, k]).any()
+    sp = synth.server_params(M, d, w.dff, 0)
+    otab = oracle.tables(sim, group, x, 0.5, 0.05, sp.F, sp.B, sp.tau, sp.z, sp.c, sp.omega_T,
+                         sp.omega_Q)
+    h = inp["home"]
+    ch, sv, kd, _, _ = oracle.select(o_idx, otab, h, h.copy(), np.zeros(T, np.float32))
+    np.testing.assert_array_equal(outs[2].cpu().numpy(), ch)
+    np.testing.assert_array_equal(outs[3].cpu().numpy(), sv)
+    np.testing.assert_array_equal(outs[4].cpu().numpy(), kd)
+
+
 # ------------------------------------------------------------------ permutation
 
 @pytest.mark.parametrize("T,k,E,d", [(64, 2, 8, 256), (1000, 6, 64, 64), (1, 1, 1, 8), (333, 3, 7, 40),
