@@ -153,8 +153,8 @@ def test_router_logits_match_oracle(T, d, E):
     np.testing.assert_array_equal(outs[4].cpu().numpy(), kd)
 
 
-@pytest.mark.parametrize("E,k", [(8, 1), (13, 3), (16, 5), (16, 7), (16, 8), (32, 4), (64, 6),
-                                 (64, 8)])
+@pytest.mark.parametrize("E,k", [(8, 1), (13, 3), (16, 5), (16, 7), (16, 8), (24, 3), (32, 4),
+                                 (40, 6), (64, 2), (64, 6), (64, 8)])
 def test_router_exact_ties_every_list_width(E, k):
     """Router rows copied in groups of 2 and 3 alternately (each row of a group
     equal to the group's first), so every logit the tensor-core router
