@@ -937,11 +937,28 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
     const uint8_t* td = tn + (dl - 1) * la.stride;
     const float* Pd = Pn + (size_t)(dl - 1) * E * E;
     for (int k2 = tid; k2 < E; k2 += blockDim.x) cs.qmax1[k2] = qmax_of(td, Pd, k2);
-    for (int i = tid; i < M * E; i += blockDim.x) {
-      const int m2 = i / E, k2 = i - (i / E) * E;
-      cs.U[i] = lookahead_phi<1>(td, la.stride, Pd, E, M, a, m2, k2, 0.0f, qbar);
+    // U[m2][k2] = lookahead_phi<1>(m2, k2, q = 0): the E terms of every entry
+    // (one per next target k') in parallel, then each entry's terms added in
+    // ascending k', skipping P = 0, as lookahead_phi<1> adds them (the same
+    // fp32 value; one thread per entry walked all its terms before)
+    const int per = kLaTerms / E;  // entries per pass
+    for (int base = 0; base < M * E; base += per) {
+      const int ne = min(per, M * E - base);
+      for (int i = tid; i < ne * E; i += blockDim.x) {
+        const int c = base + i / E, kt = i - (i / E) * E;
+        const int m2 = c / E, k2 = c - (c / E) * E;
+        cs.terms[i] = phi_term<1>(td, la.stride, Pd, E, M, a, m2, k2, kt, 0.0f, qbar);
+      }
+      __syncthreads();
+      for (int cl = tid; cl < ne; cl += blockDim.x) {
+        const int c = base + cl, k2 = c - (c / E) * E;
+        float phi = 0.0f;
+        for (int kt = 0; kt < E; ++kt)
+          if (ldt(Pd + (size_t)k2 * E + kt) != 0.0f) phi = __fadd_rn(phi, cs.terms[cl * E + kt]);
+        cs.U[c] = phi;
+      }
+      __syncthreads();
     }
-    __syncthreads();
   }
   if (memo4) {
     // one level up (layer l + 2): Phi^(2) at q = 0, through the U table above
