@@ -134,8 +134,10 @@ int ordermoe_build_tables(const float* sim, const int32_t* group, const uint8_t*
  *              home server with zero loss (the first layer) and the new state
  *              is not written
  *   logits_out [T][E] f32, nullable: the router logits
- *   topk_idx   [T][k] i32  routed (target) experts, rank order
- *   topk_w     [T][k] f32  gate weights of the routed slots
+ *   topk_idx   [T][k] i32  routed (target) experts, rank order: by logit,
+ *              equal logits to the lower expert index
+ *   topk_w     [T][k] f32  gate weights of the routed slots (fp32 softmax
+ *              over all E logits, the terms summed in expert order)
  *   chosen_expert [T][k] i32  executed expert k* per slot (Eq. 43)
  *   chosen_server [T][k] u8   executing server m* per slot
  *   kind       [T][k] u8   0 local exact, 1 local substitute, 2 remote exact,
