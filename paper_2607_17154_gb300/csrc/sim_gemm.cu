@@ -8,11 +8,14 @@
 //     expert-major so that the Gram reads both K-major, and counts each
 //     token's top-k_freq experts of every layer (Eq. 5) in a shared-memory
 //     histogram.
-//   gram_tc_kernel: partial Grams of 128 consecutive rows of H^T (128 / E
-//     layers) over a range of tokens, D = (hi + lo)(hi + lo)^T in fp32 from
-//     four tcgen05 MMAs per K step (hi hi, hi lo, lo hi, lo lo); the epilogue
-//     keeps the diagonal blocks (rows and columns of the same layer: Eq. 4's
-//     inner products). The partials are then reduced in fp64 in a fixed order.
+//   gram_tc_kernel: partial Grams of 64 consecutive rows of H^T (64 / E
+//     layers) over a range of tokens. The 64 hi rows and the same 64 lo rows
+//     form one 128-row tile A, and one tcgen05 MMA per K step accumulates
+//     A A^T, whose four 64 x 64 quadrants are hi hi^T, hi lo^T, lo hi^T and
+//     lo lo^T: the epilogue adds them, (hi hi^T + hi lo^T) + (lo hi^T +
+//     lo lo^T) = (hi + lo)(hi + lo)^T in fp32, and keeps the diagonal blocks
+//     (rows and columns of the same layer: Eq. 4's inner products). The
+//     partials are then reduced in fp64 in a fixed order.
 // Every wait is bounded; a wait that runs out reports ORDERMOE_DEV_WAIT_TIMEOUT,
 // stops the other roles, drains the copies and MMAs in flight and returns.
 #include <mutex>
@@ -54,8 +57,10 @@ constexpr int TMEM_COLS = 512;
 constexpr uint32_t IDESC = idesc_bf16_f32(BM, BN);
 constexpr int MAX_HIST = 4096;  // L * E counters in shared memory
 
-constexpr int G_STAGES = 6;
-constexpr int G_STAGE_BYTES = 2 * BOX_BYTES;  // hi and lo tiles, 128 rows x 64 tokens
+constexpr int G_ROWS = 64;  // rows of H^T per Gram block
+constexpr int G_BOX_BYTES = G_ROWS * BK * 2;
+constexpr int G_STAGES = 12;
+constexpr int G_STAGE_BYTES = 2 * G_BOX_BYTES;  // hi and lo boxes, 64 rows x 64 tokens each
 constexpr int G_TMEM_COLS = 128;
 constexpr uint32_t G_IDESC = idesc_bf16_f32(128, 128);
 
@@ -522,7 +527,22 @@ __global__ void __launch_bounds__(L_THREADS, 1)
   }
 }
 
-// grid (row blocks of 128 rows of H^T, token splits)
+// The AND of v over the 128 epilogue threads (warps 2..5, named barrier 1),
+// returned to all of them: a barrier that every epilogue thread reaches.
+__device__ __forceinline__ bool epi_and(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, 1, 128, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"(static_cast<uint32_t>(v))
+      : "memory");
+  return r != 0;
+}
+
+// grid (row blocks of 64 rows of H^T, token splits)
 __global__ void __launch_bounds__(THREADS, 1)
     gram_tc_kernel(const __grid_constant__ CUtensorMap mapHi, const __grid_constant__ CUtensorMap mapLo,
                    GArgs args) {
@@ -576,8 +596,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         uint8_t* st = tiles + stage * G_STAGE_BYTES;
         mbar_arrive_expect_tx(&s.full[stage], G_STAGE_BYTES);
-        tma_load_2d(st, &mapHi, &s.full[stage], (kb0 + i) * BK, rb * 128);
-        tma_load_2d(st + BOX_BYTES, &mapLo, &s.full[stage], (kb0 + i) * BK, rb * 128);
+        tma_load_2d(st, &mapHi, &s.full[stage], (kb0 + i) * BK, rb * G_ROWS);
+        tma_load_2d(st + G_BOX_BYTES, &mapLo, &s.full[stage], (kb0 + i) * BK, rb * G_ROWS);
         issued_mask |= 1u << stage;
         last_phase_bits = (last_phase_bits & ~(1u << stage)) | (phase << stage);
         if (++stage == G_STAGES) { stage = 0; phase ^= 1u; }
@@ -596,16 +616,12 @@ __global__ void __launch_bounds__(THREADS, 1)
           break;
         }
         tc_fence_after();
-        const uint32_t hi = smem_u32(tiles + stage * G_STAGE_BYTES);
-        const uint32_t lo = hi + BOX_BYTES;
+        // A = [hi; lo] (128 rows, the two boxes back to back), D += A A^T
+        const uint32_t a0 = smem_u32(tiles + stage * G_STAGE_BYTES);
 #pragma unroll
         for (int kk = 0; kk < BK / 16; ++kk) {
-          const uint64_t dh = sdesc_kmajor_sw128(hi + kk * 32);
-          const uint64_t dl = sdesc_kmajor_sw128(lo + kk * 32);
-          mma_bf16(tmem_base, dh, dh, G_IDESC, (i | kk) != 0 ? 1u : 0u);
-          mma_bf16(tmem_base, dh, dl, G_IDESC, 1u);
-          mma_bf16(tmem_base, dl, dh, G_IDESC, 1u);
-          mma_bf16(tmem_base, dl, dl, G_IDESC, 1u);
+          const uint64_t da = sdesc_kmajor_sw128(a0 + kk * 32);
+          mma_bf16(tmem_base, da, da, G_IDESC, (i | kk) != 0 ? 1u : 0u);
         }
         mma_issued = true;
         mma_commit(&s.empty[stage]);
@@ -614,42 +630,58 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (ok) mma_commit(&s.tfull);
     }
   } else {
-    // epilogue: warp q reads TMEM lanes 32 q .. 32 q + 31 (rows of the block)
+    // epilogue: warp q reads TMEM lanes 32 q .. 32 q + 31: rows 0..63 of D
+    // are the hi rows, 64..127 the lo rows of the block's 64 rows of H^T.
+    // Each thread adds its row's two column halves (x hi^T + x lo^T); the lo
+    // threads hand theirs over through shared memory (the consumed ring) and
+    // the hi threads add them: G = (hi hi^T + hi lo^T) + (lo hi^T + lo lo^T).
     const int q = warp & 3;
     const int r = q * 32 + lane;
-    const int gr = rb * 128 + r;
+    const int i = r & (G_ROWS - 1);  // row of the block
+    const int gr = rb * G_ROWS + i;  // row of H^T
     const int E = args.E;
+    const int l = gr / E, ii = gr - l * E;
+    const int c0 = l * E - rb * G_ROWS;  // the layer's first column in the block
+    float* xch = reinterpret_cast<float*>(tiles);  // [64][65] lo-row sums
     bool ok = true;
     if (nkb > 0) {
       ok = __all_sync(0xffffffffu, mbar_wait(&s.tfull, 0, args.limit_ns, abort));
       if (!ok && lane == 0 && !*abort) report(&g_err_simtc, ORDERMOE_DEV_WAIT_TIMEOUT, 23);
       if (!ok) *abort = 1;
     }
-    if (ok && !__any_sync(0xffffffffu, *abort != 0)) {
+    // the same decision in all four epilogue warps (they meet at a barrier below)
+    const bool go = epi_and(ok && *abort == 0);
+    if (go) {
       tc_fence_after();
-      // the columns of this row's layer: E <= 32 -> inside chunk q; E == 64 ->
-      // chunks 2 (q / 2) and 2 (q / 2) + 1 (warp-uniform either way)
-      const int nch = E == 64 ? 2 : 1;
-      const int ch0 = E == 64 ? 2 * (q >> 1) : q;
-      const int l = gr / E, i = gr - l * E;
-      float* dst = args.gpart + (((size_t)l * args.nsplit + split) * 64 + i) * 64;
-      for (int cc = 0; cc < nch; ++cc) {
-        const int ch = ch0 + cc;
-        uint32_t v[32];
+      // the layer's columns: E == 64 -> both 32-column chunks of each half;
+      // E <= 32 -> the chunk q & 1 only (a warp's 32 rows and their layers'
+      // columns lie in the same aligned 32-row range), warp-uniform either way
+      float sum[64];
+#pragma unroll
+      for (int x = 0; x < 64; ++x) sum[x] = 0.0f;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        if (E < 64 && h != (q & 1)) continue;
+        uint32_t v0[32], v1[32];
         if (nkb > 0) {
-          tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + ch * 32, v);
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + h * 32, v0);
+          tmem_ld32(tmem_base + (static_cast<uint32_t>(q * 32) << 16) + 64 + h * 32, v1);
           tmem_ld_wait();
-        } else {
 #pragma unroll
-          for (int x = 0; x < 32; ++x) v[x] = 0u;
+          for (int x = 0; x < 32; ++x)
+            sum[h * 32 + x] = __fadd_rn(__uint_as_float(v0[x]), __uint_as_float(v1[x]));
         }
-        if (gr < args.R) {
+      }
+      if (r >= G_ROWS) {
 #pragma unroll
-          for (int x = 0; x < 32; ++x) {
-            const int col = rb * 128 + ch * 32 + x;
-            if (col / E == l) dst[col - l * E] = __uint_as_float(v[x]);
-          }
-        }
+        for (int x = 0; x < 64; ++x) xch[i * 65 + x] = sum[x];
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (r < G_ROWS && gr < args.R) {
+        float* dst = args.gpart + (((size_t)l * args.nsplit + split) * 64 + ii) * 64;
+#pragma unroll
+        for (int x = 0; x < 64; ++x)
+          if (x >= c0 && x < c0 + E) dst[x - c0] = __fadd_rn(sum[x], xch[i * 65 + x]);
       }
     }
   }
@@ -675,14 +707,14 @@ __global__ void __launch_bounds__(THREADS, 1)
 }
 
 // 2-D bf16 map over [rows][cols] with row pitch ld elements (ld * 2 a multiple
-// of 16 bytes), a 64-column x 128-row box and the 128-byte swizzle; reads past
-// cols or rows return zeros.
+// of 16 bytes), a 64-column x 64-row box (the Gram's) and the 128-byte
+// swizzle; reads past cols or rows return zeros.
 int make_map_ld(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t ld) {
   gg::EncodeTiledFn enc = gg::encode_fn();
   if (!enc) return fail(ORDERMOE_ERR_CUDA, "cuTensorMapEncodeTiled is not available");
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {ld * 2};
-  cuuint32_t box[2] = {BK, 128};
+  cuuint32_t box[2] = {BK, G_ROWS};
   cuuint32_t estr[2] = {1, 1};
   CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -711,7 +743,7 @@ int sim_tc_max_splits() { return 256; }
 // by part.
 int sim_tc_nsplit(int L, int E, int64_t N) {
   const int part = sim_tc_part_layers(E);
-  const int n_rb = ((L < part ? L : part) * E + 127) / 128;
+  const int n_rb = ((L < part ? L : part) * E + sg::G_ROWS - 1) / sg::G_ROWS;
   const int kblocks = static_cast<int>((N + sg::BK - 1) / sg::BK);
   const int sms = num_sms() > 1 ? num_sms() - 1 : 1;  // the pipelined plan keeps one SM free
   int ns = sms / n_rb;
@@ -830,7 +862,7 @@ int sim_tc_launch(const uint16_t* X, int N, const uint16_t* W, int L, int E, int
   ga.nsplit = nsplit;
   ga.gpart = gpart;
   ga.limit_ns = la.limit_ns;
-  gram_tc_kernel<<<dim3((C + 127) / 128, nsplit), THREADS, gsmem, stream>>>(mHi, mLo, ga);
+  gram_tc_kernel<<<dim3((C + G_ROWS - 1) / G_ROWS, nsplit), THREADS, gsmem, stream>>>(mHi, mLo, ga);
   OM_LAUNCHED("gram_tc_kernel");
   return ORDERMOE_OK;
 }
