@@ -749,6 +749,84 @@ __device__ __forceinline__ float phi_term2_memo(const uint8_t* __restrict__ tnex
   return __fmul_rn(p, best);
 }
 
+// An order-preserving map of fp32 onto uint32 (the minimum of the keys is the
+// key of the minimum), so that partial minima can be joined with atomicMin.
+__device__ __forceinline__ uint32_t min_key(float x) {
+  const uint32_t b = __float_as_uint(x);
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float from_min_key(uint32_t key) {
+  return __uint_as_float((key & 0x80000000u) ? (key & 0x7FFFFFFFu) : ~key);
+}
+
+// Pairs (k'', m2) of phi_term2_memo whose Phi^(1) is not in U, listed for a
+// parallel evaluation: code = item << 16 | m2 << 8 | k'' (item: the
+// (candidate, k') term they belong to), A(a, m, m2) + Cq, and the loss q2.
+constexpr int kLaSlow = 512;         // listed pairs per pass
+constexpr int kLaSlowTerms = 2048;   // their Phi^(1) terms per sub-pass
+constexpr size_t kLaSlowBytes = (size_t)kLaSlow * 12 + (size_t)kLaSlowTerms * 4;
+struct LaSlow {
+  uint32_t* code;
+  float* base;
+  float* q2;
+  float* terms;
+};
+
+// phi_term2_memo split in two: the minimum over the pairs whose Phi^(1) is
+// read from U is returned (as a min_key), and each other pair is appended to
+// the list (or, when the list is full, evaluated here). The caller joins the
+// listed pairs' costs into the minimum and multiplies by P(kx -> kt); the
+// minimum of a set does not depend on the order it is taken in, so the term
+// is the same fp32 value.
+__device__ __forceinline__ uint32_t phi_term2_split(const uint8_t* __restrict__ tnext,
+                                                    size_t stride, const float* __restrict__ P,
+                                                    int E, int M, int a, int m, int kx, int kt,
+                                                    float qacc, float qbar, const float* U,
+                                                    const float* qmax1, int item,
+                                                    const LaSlow& slow, int* ns) {
+  const float* Q1 = reinterpret_cast<const float*>(tnext + kOffQtab);
+  const float* C1 = reinterpret_cast<const float*>(tnext + off_cq(E));
+  const float* A1 = reinterpret_cast<const float*>(tnext + off_a(E));
+  const uint32_t* pm1 = reinterpret_cast<const uint32_t*>(tnext + kOffPmask);
+  const unsigned long long* sb1 = reinterpret_cast<const unsigned long long*>(tnext + kOffSubst);
+  float best = INFINITY;
+  unsigned long long cand = ldt(sb1 + kt) | (1ull << kt);
+  while (cand) {
+    const int kk = __ffsll(static_cast<long long>(cand)) - 1;
+    cand &= cand - 1;
+    const bool exact = (kk == kt);
+    float cq = 0.0f, q2 = qacc;
+    if (!exact) {
+      const float qk = ldt(Q1 + kt * E + kk);
+      if (!(__fadd_rn(qacc, qk) <= qbar)) continue;
+      q2 = __fadd_rn(qacc, qk);
+      cq = ldt(C1 + kt * E + kk);
+    }
+    const bool free = __fadd_rn(q2, qmax1[kk]) <= qbar;
+    uint32_t pm = ldt(pm1 + kk);
+    while (pm) {
+      const int m2 = __ffs(pm) - 1;
+      pm &= pm - 1;
+      const float base = __fadd_rn(ldt(A1 + ((size_t)a * M + m) * M + m2), cq);
+      if (free) {
+        best = fminf(best, __fadd_rn(base, U[m2 * E + kk]));
+        continue;
+      }
+      const int e = atomicAdd(ns, 1);
+      if (e < kLaSlow) {
+        slow.code[e] = (static_cast<uint32_t>(item) << 16) | (static_cast<uint32_t>(m2) << 8) |
+                       static_cast<uint32_t>(kk);
+        slow.base[e] = base;
+        slow.q2[e] = q2;
+      } else {
+        best = fminf(best, __fadd_rn(base, lookahead_phi<1>(tnext + stride, stride, P + E * E, E,
+                                                            M, a, m2, kk, q2, qbar)));
+      }
+    }
+  }
+  return min_key(best);
+}
+
 // lookahead_phi<2> with its deepest level read from U / qmax1 as in
 // phi_term2_memo (the same fp32 operations in the same order).
 __device__ float lookahead_phi2_memo(const uint8_t* __restrict__ tnext, size_t stride,
@@ -834,6 +912,13 @@ __host__ __device__ inline size_t la_stage_offset(int E, int H) {
 __host__ __device__ inline size_t la_stage_bytes(int E, int H, size_t stride) {
   return (size_t)(H - 1) * stride + (size_t)(H - 1) * E * E * sizeof(float);
 }
+// H = 3: the pairs listed by phi_term2_split follow the tables (and their
+// shared-memory copy, when there is one); kLaSlowBytes long.
+__host__ __device__ inline size_t la_slow_offset(int E, int H, size_t stride, int staged) {
+  const size_t end = staged ? la_stage_offset(E, H) + la_stage_bytes(E, H, stride)
+                            : 2 * (size_t)E * E * sizeof(float);
+  return (end + 15) & ~size_t(15);
+}
 
 constexpr int kLaThreads = 128;
 constexpr int kLaMaxCand = 65 * 32;  // (target + 64 substitutes) x 32 servers
@@ -848,6 +933,7 @@ struct LaSmem {
   float qmax1[64];            // H = 3, 4: largest substitute loss Phi^(1)(., k2) can consider
   unsigned long long best;
   int n;
+  int ns;                     // H = 3: pairs listed by phi_term2_split
 };
 
 __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
@@ -914,6 +1000,14 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
   float* U2 = s_dyn + 2 * E * E;  // H = 4: Phi^(2)(m2, k2) with every check passing, [32][E]
   float* qmax2 = U2 + 32 * E;     // H = 4: largest loss Phi^(2)(., k2) adds at its level
   float qmaxL1 = -INFINITY;       // H = 4: largest such loss one level deeper
+  LaSlow slow{};                  // H = 3: the listed pairs
+  if (memo) {
+    uint8_t* sp = reinterpret_cast<uint8_t*>(s_dyn) + la_slow_offset(E, 3, la.stride, la.staged);
+    slow.code = reinterpret_cast<uint32_t*>(sp);
+    slow.base = reinterpret_cast<float*>(sp + (size_t)kLaSlow * 4);
+    slow.q2 = slow.base + kLaSlow;
+    slow.terms = slow.q2 + kLaSlow;
+  }
   // the largest substitute loss lookahead_phi<1> on tables tl and transitions Pl
   // can add for expert kx (targets with P(kx -> k') != 0; -inf: none)
   auto qmax_of = [&](const uint8_t* tl, const float* Pl, int kx) {
@@ -1010,25 +1104,71 @@ __global__ void __launch_bounds__(kLaThreads) lookahead_select_kernel(
     const int n = cs.n;
     for (int base = 0; base < n; base += cpp) {
       const int nc = min(cpp, n - base);
-      for (int i = tid; i < nc * E; i += blockDim.x) {
-        const int c = base + i / E, kt = i - (i / E) * E;
-        const uint32_t code = cs.code[c];
-        const int cm = static_cast<int>((code >> 8) & 0xFFu), ck = static_cast<int>(code & 0xFFu);
-        cs.terms[i] = memo    ? phi_term2_memo(tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c],
-                                               qbar, cs.U, cs.qmax1)
-                      : memo4 ? phi_term3_memo(tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c],
+      if (memo) {
+        // H = 3: each (candidate, k') item takes its pairs whose Phi^(1) is in
+        // U and lists the others; the listed pairs' Phi^(1) is then evaluated
+        // with its E terms in parallel and added in ascending k'' as
+        // lookahead_phi<1> adds them, and each pair's cost joins its item's
+        // minimum (a token near its budget has many such pairs, which one
+        // thread used to walk one after another)
+        if (tid == 0) cs.ns = 0;
+        __syncthreads();
+        uint32_t* key = reinterpret_cast<uint32_t*>(cs.terms);
+        for (int i = tid; i < nc * E; i += blockDim.x) {
+          const int c = base + i / E, kt = i - (i / E) * E;
+          const uint32_t code = cs.code[c];
+          const int cm = static_cast<int>((code >> 8) & 0xFFu), ck = static_cast<int>(code & 0xFFu);
+          if (ldt(Pn + (size_t)ck * E + kt) != 0.0f)
+            key[i] = phi_term2_split(tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c], qbar, cs.U,
+                                     cs.qmax1, i, slow, &cs.ns);
+        }
+        __syncthreads();
+        const int ns = min(cs.ns, kLaSlow);
+        const int per2 = kLaSlowTerms / E;
+        for (int sb = 0; sb < ns; sb += per2) {
+          const int ne = min(per2, ns - sb);
+          for (int j = tid; j < ne * E; j += blockDim.x) {
+            const int e = sb + j / E, k3 = j - (j / E) * E;
+            const uint32_t sc = slow.code[e];
+            slow.terms[j] = phi_term<1>(tn + la.stride, la.stride, Pn + E * E, E, M, a,
+                                        static_cast<int>((sc >> 8) & 0xFFu),
+                                        static_cast<int>(sc & 0xFFu), k3, slow.q2[e], qbar);
+          }
+          __syncthreads();
+          for (int el = tid; el < ne; el += blockDim.x) {
+            const uint32_t sc = slow.code[sb + el];
+            const int kk = static_cast<int>(sc & 0xFFu);
+            const float* P2 = Pn + (size_t)E * E + (size_t)kk * E;
+            float phi1 = 0.0f;
+            for (int k3 = 0; k3 < E; ++k3)
+              if (ldt(P2 + k3) != 0.0f) phi1 = __fadd_rn(phi1, slow.terms[el * E + k3]);
+            atomicMin(&key[sc >> 16], min_key(__fadd_rn(slow.base[sb + el], phi1)));
+          }
+          __syncthreads();
+        }
+      } else {
+        for (int i = tid; i < nc * E; i += blockDim.x) {
+          const int c = base + i / E, kt = i - (i / E) * E;
+          const uint32_t code = cs.code[c];
+          const int cm = static_cast<int>((code >> 8) & 0xFFu), ck = static_cast<int>(code & 0xFFu);
+          cs.terms[i] = memo4 ? phi_term3_memo(tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c],
                                                qbar, U2, qmax2, qmaxL1, cs.U, cs.qmax1)
                               : phi_term_h(la.H, tn, la.stride, Pn, E, M, a, cm, ck, kt, cs.qn[c],
                                            qbar);
+        }
+        __syncthreads();
       }
-      __syncthreads();
       for (int cl = tid; cl < nc; cl += blockDim.x) {
         const uint32_t code = cs.code[base + cl];
         const int kk = static_cast<int>(code & 0xFFu), m = static_cast<int>((code >> 8) & 0xFFu);
         const unsigned sub = (code >> 16) & 1u;
         float phi = 0.0f;
-        for (int kt = 0; kt < E; ++kt)
-          if (ldt(Pn + (size_t)kk * E + kt) != 0.0f) phi = __fadd_rn(phi, cs.terms[cl * E + kt]);
+        for (int kt = 0; kt < E; ++kt) {
+          const float p = ldt(Pn + (size_t)kk * E + kt);
+          if (p == 0.0f) continue;
+          const float term = cs.terms[cl * E + kt];
+          phi = __fadd_rn(phi, memo ? __fmul_rn(p, from_min_key(__float_as_uint(term))) : term);
+        }
         const float cost = __fadd_rn(cs.cost0[base + cl], phi);
         const unsigned long long key =
             (static_cast<unsigned long long>(__float_as_uint(cost)) << 32) |
@@ -1398,6 +1538,7 @@ static int launch_lookahead_select(const int32_t* topk_idx, int T, int E, int k,
       la.staged = 1;
     }
   }
+  if (la.H == 3) tab_smem = la_slow_offset(E, 3, la.stride, la.staged) + kLaSlowBytes;
   cudaFuncSetAttribute(lookahead_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                        (int)tab_smem);
   OM_LAUNCH_PDL("lookahead_select_kernel", lookahead_select_kernel, dim3(T), dim3(kLaThreads),
