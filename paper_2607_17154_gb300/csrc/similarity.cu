@@ -374,14 +374,23 @@ __device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float*
         const float v = sv != sv ? -INFINITY : sv;
         if (bg == (1 << 30) || v > bs) { bg = g; bs = v; }
       }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float os = __shfl_xor_sync(0xffffffffu, bs, o);
-        const int og = __shfl_xor_sync(0xffffffffu, bg, o);
-        if (og != (1 << 30) && (bg == (1 << 30) || os > bs || (os == bs && og < bg))) {
-          bs = os;
-          bg = og;
-        }
+      // across the lanes: the largest similarity by an order-preserving 32-bit
+      // key (0: the lane has no dominant; -0 counted as +0, so that equal
+      // similarities are equal keys), then the lowest dominant index among
+      // the lanes that hold it (dominants below 32 before those above)
+      uint32_t key = 0u;
+      if (bg != (1 << 30)) {
+        const uint32_t u = __float_as_uint(bs == 0.0f ? 0.0f : bs);
+        key = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+      }
+      const uint32_t mk = __reduce_max_sync(0xffffffffu, key);
+      const unsigned lo32 = __ballot_sync(0xffffffffu, key == mk && bg < 32);
+      const unsigned hi32 = __ballot_sync(0xffffffffu, key == mk && bg >= 32 && bg != (1 << 30));
+      if (mk == 0u) {
+        bg = 1 << 30;
+      } else {
+        bg = lo32 ? __ffs(lo32) - 1 : __ffs(hi32) - 1 + 32;
+        bs = __uint_as_float((mk & 0x80000000u) ? (mk & 0x7FFFFFFFu) : ~mk);
       }
       if (k > 0) {
         const float s0 = S[j * E + dom[0]];
@@ -405,9 +414,12 @@ __device__ void group_layer(GroupSmem& sm, bool live, int t, int l, const float*
   }
   __syncthreads();
   // Eqs. 27-28
-  double total = 0.0;
+  // the counts' fp64 sum in index order, formed exactly as an integer sum
+  // (every partial sum is an integer below 2^53, so each fp64 addition is exact)
+  long long total_i = 0;
   if (live)
-    for (int e = 0; e < E; ++e) total = __dadd_rn(total, static_cast<double>(cnt[e]));
+    for (int e = 0; e < E; ++e) total_i += cnt[e];
+  const double total = static_cast<double>(total_i);
   if (live && t < E) {
     group[(size_t)l * E + t] = grp[t];
     double sum = 0.0;
