@@ -552,19 +552,23 @@ __device__ int place_layers(PlaceSmem& sm, const int32_t* __restrict__ group,
         gn = grp[jn];
         pn = pls[jn];
       }
-      const double bn = __dadd_rn(b, pj);
-      const bool feas = srv && __double_as_longlong(bn) <= cap_bits;  // bn <= C_m, bn >= 0
-      // eta of this lane's server (lanes past M are no server: 0); at most E <= 64
-      const int et = srv ? min(eta[t * 64 + g], 64) : 0;
-      const double sc = __dadd_rn(a1, l2eta[et]);
-      double a1n = 0.0;
-      if (feas) a1n = __dmul_rn(pp.lambda1, div_rn_markstein(bn, cap, rcap));  // kept if this lane wins
-      unsigned long long key = static_cast<unsigned long long>(__double_as_longlong(sc));
-      // !(sc >= 0) on the bits: a NaN, or a negative value other than -0
-      const unsigned long long mag = key & 0x7FFFFFFFFFFFFFFFull;
-      bad_score |= feas && (mag > 0x7FF0000000000000ull || (key != mag && mag != 0));
-      if (key == 0x8000000000000000ull) key = 0;  // -0 orders like +0
-      if (!feas) key = ~0ull;
+      // the fp64 work on the server lanes only (the other lanes' keys are ~0)
+      double bn = 0.0, a1n = 0.0;
+      unsigned long long key = ~0ull;
+      if (srv) {
+        bn = __dadd_rn(b, pj);
+        const bool feas = __double_as_longlong(bn) <= cap_bits;  // bn <= C_m, bn >= 0
+        const int et = min(eta[t * 64 + g], 64);  // at most E <= 64
+        const double sc = __dadd_rn(a1, l2eta[et]);
+        if (feas) {
+          a1n = __dmul_rn(pp.lambda1, div_rn_markstein(bn, cap, rcap));  // kept if this lane wins
+          unsigned long long ks = static_cast<unsigned long long>(__double_as_longlong(sc));
+          // !(sc >= 0) on the bits: a NaN, or a negative value other than -0
+          const unsigned long long mag = ks & 0x7FFFFFFFFFFFFFFFull;
+          bad_score |= mag > 0x7FF0000000000000ull || (ks != mag && mag != 0);
+          key = (ks == 0x8000000000000000ull) ? 0ull : ks;  // -0 orders like +0
+        }
+      }
       // argmin of the 64-bit keys, ties to the lower server: minimum of the high
       // words, then of the low words among those lanes, then the lowest lane
       const unsigned khi = static_cast<unsigned>(key >> 32), klo = static_cast<unsigned>(key);
