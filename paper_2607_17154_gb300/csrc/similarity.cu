@@ -1002,16 +1002,45 @@ __global__ void __launch_bounds__(32) coverage_kernel(const int32_t* __restrict_
                                                       int32_t* __restrict__ covered) {
   const int l = blockIdx.x;
   const int m = threadIdx.x;
-  unsigned long long bits = 0;
-  if (m < M)
-    for (int j = 0; j < E; ++j) {
-      const int g = group[(size_t)l * E + j];
-      if (g < 0 || g >= E) {
-        report(&g_err_sim, ORDERMOE_DEV_BAD_INDEX, l * E + j);
-        continue;
-      }
-      if (placement[((size_t)l * M + m) * E + j]) bits |= 1ull << g;
+  // the layer's groups, checked once (-1: out of range, reported)
+  __shared__ int gsh[64];
+  for (int j = m; j < E; j += 32) {
+    int g = group[(size_t)l * E + j];
+    if (g < 0 || g >= E) {
+      report(&g_err_sim, ORDERMOE_DEV_BAD_INDEX, l * E + j);
+      g = -1;
     }
+    gsh[j] = g;
+  }
+  __syncwarp();
+  // server m's row of the layer's placement: 16-byte loads where it allows,
+  // all issued before they are used
+  unsigned long long bits = 0;
+  if (m < M) {
+    const uint8_t* row = placement + ((size_t)l * M + m) * E;
+    if ((E & 15) == 0 && (reinterpret_cast<uintptr_t>(row) & 15u) == 0) {
+      uint4 v[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        if (c < E / 16) v[c] = reinterpret_cast<const uint4*>(row)[c];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        if (c >= E / 16) break;
+        const uint32_t w[4] = {v[c].x, v[c].y, v[c].z, v[c].w};
+#pragma unroll
+        for (int q = 0; q < 16; ++q) {
+          const int g = gsh[c * 16 + q];
+          if (((w[q >> 2] >> (8 * (q & 3))) & 0xFFu) != 0u && g >= 0) bits |= 1ull << g;
+        }
+      }
+    } else {
+#pragma unroll 16
+      for (int j = 0; j < E; ++j) {
+        const int g = gsh[j];
+        if (row[j] && g >= 0) bits |= 1ull << g;
+      }
+    }
+  }
   if (m < M && cover != nullptr)
     for (int g = 0; g < E; ++g) cover[((size_t)l * M + m) * E + g] = (bits >> g) & 1ull;
   int n = __popcll(bits);
