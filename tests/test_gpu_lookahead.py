@@ -64,6 +64,12 @@ def stack_tables(rng, L, E, M, qbar, cheap_links):
 
 @pytest.mark.parametrize("E,M,k,H,cheap", [(8, 4, 2, 1, True), (8, 4, 2, 2, True), (8, 4, 2, 3, True),
                                            (16, 4, 3, 3, False), (6, 3, 2, 4, True), (32, 8, 2, 2, True),
+                                           # H = 3 with 8 servers and dear links: about half the
+                                           # tokens have more than 512 pairs in their first slot
+                                           # whose Phi^(1) is not tabulated (up to about 1100), more
+                                           # than the kernel lists (the rest evaluated in place);
+                                           # with 4 servers at most about 215
+                                           (16, 8, 3, 3, False),
                                            # H = 4: the Phi^(2) table used (cheap substitutes) and
                                            # bypassed when budget checks can fail (dear ones)
                                            (8, 4, 2, 4, False), (16, 4, 3, 4, True), (12, 5, 2, 4, False)])
