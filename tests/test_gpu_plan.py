@@ -190,6 +190,36 @@ def test_place_ties_waiting_lists_and_server_counts(L, E, M, scale, frac):
     assert (got[3].sum(axis=1) == 1).all()  # every expert on exactly one server
 
 
+@pytest.mark.parametrize("E", [64, 40, 8])
+def test_group_exact_ties_and_signed_zeros_match_oracle(E):
+    """Similarities drawn from a few exact values give an expert several
+    equally similar dominants (Eqs. 24-26: the scan keeps the lowest
+    dominant); in the last layer (threshold -0.25) the only values are +0, -0
+    and -0.5, so the most similar dominants tie at zero of either sign, which
+    compare equal. Counts tie too (the visiting order: count desc, index asc).
+    Groups, group counts, thresholds and placements bit for bit."""
+    rng = np.random.default_rng(700 + E)
+    L, M = 4, 8
+    sets = [np.array([0.95, 0.95, 0.3, 0.0, -0.0, -0.5], np.float32)] * (L - 1) + \
+        [np.array([0.0, -0.0, -0.5], np.float32)]
+    sims = []
+    for l in range(L):
+        u = rng.choice(sets[l], (E, E)).astype(np.float32)
+        # symmetric by mirroring the upper triangle (a sum would turn -0 into +0)
+        s = np.where(np.triu(np.ones((E, E), bool), 1), u, u.T).astype(np.float32)
+        np.fill_diagonal(s, 1.0)
+        sims.append(s)
+    sim = np.stack(sims)
+    assert np.signbit(sim[L - 1][sim[L - 1] == 0]).any()   # both signs of zero present
+    counts = rng.integers(0, 4, (L, E)).astype(np.int32)
+    p = np.ones((L, E)); C = np.full(M, L * E / M * 1.5)
+    got = gpu_place(sim, counts, M, p, C, theta_min=-0.25, theta_max=0.9)
+    ref = oracle_place_all(sim, counts, M, p, C, theta_min=-0.25, theta_max=0.9)
+    for name, a, b in zip(("group", "n_groups", "theta", "placement", "used", "status"), got, ref):
+        np.testing.assert_array_equal(a, b, err_msg="%s E=%d" % (name, E))
+    assert ref[1][L - 1] < E                                  # experts joined dominants at zero
+
+
 def test_place_with_nan_similarities_matches_oracle():
     """NaN similarities (bad inputs) give the oracle's groups, importances
     (NaN where a group mean meets one), placement order and placement: the
