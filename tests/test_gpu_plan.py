@@ -413,7 +413,7 @@ def test_replicate_largest_shape_and_errors():
     assert code == B.DEV_BAD_VALUE and detail == 2
 
 
-@pytest.mark.parametrize("L,E,M", [(1, 4, 2), (24, 64, 8), (32, 8, 8), (3, 64, 32)])
+@pytest.mark.parametrize("L,E,M", [(1, 4, 2), (24, 64, 8), (32, 8, 8), (3, 64, 32), (5, 48, 6), (4, 40, 3)])
 def test_coverage_bit_exact(L, E, M):
     rng = np.random.default_rng(L + E + M)
     group = rng.integers(0, max(1, E // 3), (L, E)).astype(np.int32)
