@@ -51,6 +51,8 @@ MUTANTS = [
     ("Eq. 4: not normalised", "dot / (norm[i] * norm[j])", "dot"),
     ("Eq. 24: threshold inclusive", "best_s < theta", "best_s <= theta"),
     ("Eq. 25: argmax ties to the later dominant", "if (best_g < 0 || s > best_s)", "if (best_g < 0 || s >= best_s)"),
+    ("Eq. 25: -0 ranked below +0", "if (best_g < 0 || s > best_s)",
+     "if (best_g < 0 || s > best_s || (s == 0.0f && best_s == 0.0f && std::signbit(best_s) && !std::signbit(s)))"),
     ("Eq. 27: representativeness over all experts", "if (group[k] == group[j]) { s += sim[j * E + k]; ++size; }",
      "{ s += sim[j * E + k]; ++size; }"),
     ("Eq. 30: dispersion term dropped", "lambda2 * static_cast<double>(eta)", "0.0"),

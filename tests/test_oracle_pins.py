@@ -913,6 +913,13 @@ def test_group_threshold_is_strict_and_ties_go_to_the_earlier_dominant(orc):
     sim2 = np.array([[1, .1, .6], [.1, 1, .6], [.6, .6, 1]], np.float32)
     g2, K2, dom2 = orc.group(sim2, cnt, 0.3)
     assert K2 == 2 and list(dom2) == [0, 1] and g2[2] == 0
+    # zeros of either sign are equal similarities: 2 is -0 to dominant 0 and +0
+    # to dominant 1 (0 and 1 at -0.5 from each other, threshold -0.25), so the
+    # tie goes to the earlier dominant; with the signs swapped it is the same
+    for z0, z1 in ((-0.0, 0.0), (0.0, -0.0)):
+        sim3 = np.array([[1, -.5, z0], [-.5, 1, z1], [z0, z1, 1]], np.float32)
+        g3, K3, dom3 = orc.group(sim3, cnt, -0.25)
+        assert K3 == 2 and list(dom3) == [0, 1] and g3[2] == 0, (z0, z1, g3)
 
 
 def test_place_disperses_same_group_experts_even_when_load_alone_would_not(orc):
