@@ -123,6 +123,30 @@ MUTANTS = [
      "orc_phi(h - 1, tabs, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar)"),
     ("Eq. 43: cost-to-go ignored",
      "cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, m, kk, qn, qbar);", ""),
+    ("Eq. 40: budget strict", "if (!(q + Qtab[r * E + kk] <= qbar)) continue;      // budget",
+     "if (!(q + Qtab[r * E + kk] < qbar)) continue;      // budget"),
+    ("Eq. 42: budget strict", "if (!(qacc + t1.Qtab[kt * E + kk] <= qbar)) continue;",
+     "if (!(qacc + t1.Qtab[kt * E + kk] < qbar)) continue;"),
+    ("Eq. 42: the most expensive candidate", "if (c < best) best = c;",
+     "if (best == INFINITY || c > best) best = c;"),
+    ("execution type bits swapped", "2 * best_away + best_sub", "2 * best_sub + best_away"),
+    ("tie: substitute before the exact expert", "else if (sub != best_sub) better = sub < best_sub;",
+     "else if (sub != best_sub) better = sub > best_sub;"),
+    ("tie: higher server", "else if (m != best_m) better = m < best_m;",
+     "else if (m != best_m) better = m > best_m;"),
+    ("tie: higher expert", "else better = kk < best_k;", "else better = kk > best_k;"),
+    ("distinct experts: a substitute not marked taken", "taken |= (uint64_t)1 << best_k;", ""),
+    ("Eq. 29: capacity strict", "if (!(b[m] + pl[j] <= C[m])) continue;",
+     "if (!(b[m] + pl[j] < C[m])) continue;"),
+    ("Eq. 30: lambda1 dropped", "lambda1 * (b[m] / C[m])", "(b[m] / C[m])"),
+    ("Eq. 30: dispersion over every expert", "if (g[k] == g[j] && x[m * E + k]) ++eta;",
+     "if (x[m * E + k]) ++eta;"),
+    ("Eq. 31: argmin ties to the later server", "if (best < 0 || score < best_score)",
+     "if (best < 0 || score <= best_score)"),
+    ("waiting list ties to the later server", "if (C[m] - b[m] > C[best] - b[best]) best = m;",
+     "if (C[m] - b[m] >= C[best] - b[best]) best = m;"),
+    ("Eq. 27: mean over all experts' count", "double rho = s / size;", "double rho = s / E;"),
+    ("Eq. 28: frequency not normalised", "count[j] / total : 0.0", "count[j] : 0.0"),
 ]
 
 

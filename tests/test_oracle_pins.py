@@ -580,6 +580,104 @@ def test_theta_endpoints_and_monotone(orc):
     assert th[11] == pytest.approx(0.5 + 0.4 * 12 / 23, abs=1e-7)
 
 
+def hand_tables(orc, E, M, qbar, A, Q=None, Cq=None, subst=None, pmask=None):
+    """Selection tables written by hand (dyadic values, so that sums and ties
+    are exact in fp32): A[a][s][m], Qtab/Cq [E][E], subst bit masks, pmask."""
+    Q = np.zeros((E, E), np.float32) if Q is None else np.asarray(Q, np.float32)
+    Cq = np.zeros((E, E), np.float32) if Cq is None else np.asarray(Cq, np.float32)
+    subst = np.zeros(E, np.uint64) if subst is None else np.asarray(subst, np.uint64)
+    return orc.Tables(np.ascontiguousarray(Q), np.ascontiguousarray(Cq), np.ascontiguousarray(subst),
+                      np.ascontiguousarray(np.asarray(A, np.float32)),
+                      np.ascontiguousarray(np.asarray(pmask, np.uint32)), qbar, E, M)
+
+
+def test_select_budget_is_inclusive(orc):
+    """Eq. 40 admits a substitute when Q_hat + Q <= Qbar: at equality it is
+    feasible. Target 0 sits only on remote server 1 (cost 1); substitute 1 on
+    local server 0 costs Cq = 0.125 and brings the loss from 0.25 to exactly
+    Qbar = 0.5."""
+    E, M = 2, 2
+    A = np.zeros((M, M, M), np.float32); A[0, 0, 1] = 1.0
+    Q = [[0, 0.25], [0.25, 0]]; Cq = [[0, 0.125], [0.125, 0]]
+    tab = hand_tables(orc, E, M, 0.5, A, Q, Cq, subst=[0b10, 0b01], pmask=[0b10, 0b01])
+    ch, sv, kd, loc, q = orc.select(np.array([[0]], np.int32), tab, np.zeros(1, np.uint8),
+                                    np.zeros(1, np.uint8), np.array([0.25], np.float32))
+    assert (ch[0, 0], sv[0, 0], kd[0, 0]) == (1, 0, 1)
+    assert q[0] == np.float32(0.5)
+
+
+def test_select_equal_costs_prefer_the_exact_expert_then_the_lower_substitute(orc):
+    """Ties of Eq. 43's cost: the exact target before a substitute (reading
+    of the tie rule: sub < ...), and among equally cheap substitutes on the same
+    server the lower expert index. Costs are dyadic, so the ties are exact."""
+    E, M = 3, 2
+    # exact target 0 on remote server 1 at 0.5; substitute 1 on local server 0 at 0.25 + Cq 0.25
+    A = np.zeros((M, M, M), np.float32); A[0, 0, 1] = 0.5
+    Cq = np.zeros((E, E), np.float32); Cq[0, 1] = 0.25
+    Q = np.zeros((E, E), np.float32); Q[0, 1] = 0.125
+    A[0, 0, 0] = 0.25
+    tab = hand_tables(orc, E, M, 0.5, A, Q, Cq, subst=[0b010, 0, 0], pmask=[0b10, 0b01, 0b00])
+    ch, sv, kd, _, _ = orc.select(np.array([[0]], np.int32), tab, np.zeros(1, np.uint8),
+                                  np.zeros(1, np.uint8), np.zeros(1, np.float32))
+    assert (ch[0, 0], sv[0, 0], kd[0, 0]) == (0, 1, 2)     # exact, remote: cost 0.5 either way
+    # two substitutes 1 and 2 of target 0 on server 0 at the same cost; the target costs more
+    A2 = np.zeros((M, M, M), np.float32); A2[0, 0, 1] = 1.0
+    Cq2 = np.zeros((E, E), np.float32); Cq2[0, 1] = Cq2[0, 2] = 0.25
+    Q2 = np.zeros((E, E), np.float32); Q2[0, 1] = Q2[0, 2] = 0.125
+    tab2 = hand_tables(orc, E, M, 0.5, A2, Q2, Cq2, subst=[0b110, 0, 0],
+                       pmask=[0b10, 0b01, 0b01])
+    ch, sv, kd, _, _ = orc.select(np.array([[0]], np.int32), tab2, np.zeros(1, np.uint8),
+                                  np.zeros(1, np.uint8), np.zeros(1, np.float32))
+    assert (ch[0, 0], sv[0, 0], kd[0, 0]) == (1, 0, 1)
+
+
+def test_phi_budget_is_inclusive(orc):
+    """Eq. 42 takes the next layer's substitutes under the same rule as Eq. 40:
+    with Q_hat = 0.25 and Q(1 -> 0) = 0.25 the substitute is feasible at
+    Q_hat + Q = Qbar = 0.5. From server 0 the next target 1 runs exactly on
+    server 1 (cost 1) or as substitute 0 on server 0 (cost 0.125), with
+    P(0 -> 1) = 1: Phi^(1) = 0.125."""
+    E, M = 2, 2
+    t0 = hand_tables(orc, E, M, 0.5, np.zeros((M, M, M), np.float32), pmask=[0b01, 0b01])
+    A1 = np.zeros((M, M, M), np.float32); A1[0, 0, 1] = 1.0
+    Q1 = [[0, 0.25], [0.25, 0]]; Cq1 = [[0, 0.125], [0.125, 0]]
+    t1 = hand_tables(orc, E, M, 0.5, A1, Q1, Cq1, subst=[0b10, 0b01], pmask=[0b01, 0b10])
+    P = np.array([[[0, 1], [1, 0]]], np.float32)
+    assert orc.phi(1, [t0, t1], P, 0, 0, 0, 0.25) == 0.125
+    assert orc.phi(1, [t0, t1], P, 0, 0, 0, 0.3) == 1.0     # above the budget: exact only
+
+
+def test_place_load_term_is_weighted_by_lambda1(orc):
+    """Eq. 30's score lambda1 b_m / C_m + lambda2 eta_m with lambda1 = 0.25 and
+    lambda2 = 0.375. Experts in order 0, 1, 2 (p desc, then importance):
+    0 (group 1) -> server 0 (tie at 0, lower server); 1 (group 0) -> server 1
+    (0 against 0.25 * 2/4); 2 (group 0): server 0 scores 0.25 * 0.5 = 0.125,
+    server 1 (C = 1024, one expert of group 0) 0.25/1024 + 0.375 -> server 0.
+    Without the lambda1 weight server 0 would score 0.5 and lose."""
+    group = np.array([[1, 0, 0]], np.int32)
+    imp = np.array([[3.0, 2.0, 1.0]])
+    p = np.array([[2.0, 1.0, 1.0]])
+    C = np.array([4.0, 1024.0])
+    x, used, rc = orc.place(group, imp, p, C, lambda1=0.25, lambda2=0.375)
+    assert rc == 0
+    np.testing.assert_array_equal(x[0], [[1, 0, 1], [0, 1, 0]])
+    np.testing.assert_array_equal(used, [3.0, 1.0])
+
+
+def test_place_waiting_list_ties_go_to_the_lower_server(orc):
+    """Expert 2 (p = 3) fits no server of capacity 2 and waits; experts 0 and 1
+    (p = 2) fill servers 0 and 1. The waiting expert goes to the server with
+    the most room; both have 0, so the lower server takes it (and overflows)."""
+    group = np.array([[0, 1, 2]], np.int32)
+    imp = np.array([[1.0, 1.0, 1.0]])
+    p = np.array([[2.0, 2.0, 3.0]])
+    C = np.array([2.0, 2.0])
+    x, used, rc = orc.place(group, imp, p, C)
+    assert rc == orc.CAPACITY
+    np.testing.assert_array_equal(x[0], [[1, 0, 1], [0, 1, 0]])
+    np.testing.assert_array_equal(used, [5.0, 2.0])
+
+
 def test_group_hand_example(orc):
     # counts order: 2 (9), 0 (7), 4 (5), 1 (3), 3 (1)
     sim = np.array([[1, .9, .2, .1, .3],
