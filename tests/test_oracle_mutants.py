@@ -147,6 +147,28 @@ MUTANTS = [
      "if (C[m] - b[m] >= C[best] - b[best]) best = m;"),
     ("Eq. 27: mean over all experts' count", "double rho = s / size;", "double rho = s / E;"),
     ("Eq. 28: frequency not normalised", "count[j] / total : 0.0", "count[j] : 0.0"),
+    ("Eq. 7: threshold strict", "if (k != r && group[k] == group[r] && s >= theta) bits",
+     "if (k != r && group[k] == group[r] && s > theta) bits"),
+    ("Eq. 18: Sim not clamped", "q = 0.5f * (1.0f - std::min(s, 1.0f));", "q = 0.5f * (1.0f - s);"),
+    ("Eq. 37: compute dropped on the local server", "double dl = comp;", "double dl = 0.0;"),
+    ("Eqs. 15-16: simulator compute dropped", "d = d + (trans + comp);", "d = d + trans;"),
+    ("Eq. 23: delay not normalised", "st += delay[t] / delay_ref[t];", "st += delay[t];"),
+    ("Eq. 23: loss not normalised", "sq += loss[t] / qmax;", "sq += loss[t];"),
+    ("Eq. 45: omega_T not the complement", "out[3] = 1.0 - wq;", "out[3] = omega_T;"),
+    ("Eq. 41: top-1 pairs only", "for (int b : nxt) count[((size_t)l * E + a) * E + b]++;",
+     "if (a == cur[0]) count[((size_t)l * E + a) * E + nxt[0]]++;"),
+    ("Eq. 41: every layer paired with layer 0", "      cur = nxt;\n", "\n"),
+    ("Eq. 42: transition matrix transposed", "const float p = P[(size_t)kx * E + kt];",
+     "const float p = P[(size_t)kt * E + kx];"),
+    ("Eq. 6: one layer takes theta_max", "if (N <= 1) return static_cast<float>(theta_single);",
+     "if (N <= 1) return static_cast<float>(theta_max);"),
+    ("RMSNorm: eps dropped", "std::sqrt(ss / d + eps)", "std::sqrt(ss / d)"),
+    ("SiLU: sign of the exponent", "double silu = g / (1.0 + std::exp(-g));",
+     "double silu = g / (1.0 + std::exp(g));"),
+    ("Eq. 33: importance dropped", "const double benefit = pi[m] * importance[l * E + j] * cover",
+     "const double benefit = pi[m] * 1.0 * cover"),
+    ("Eq. 35: capacity strict", "if (!(used[m] + p[l * E + j] <= C[m])) continue;",
+     "if (!(used[m] + p[l * E + j] < C[m])) continue;"),
 ]
 
 

@@ -145,6 +145,10 @@ def test_tables_quality_terms_closed_forms(orc):
     assert subst[1] == (1 << 3)              # 3: Sim 1.25 >= 0.6
     assert subst[2] == 0                     # alone in group 1
     assert subst[3] == (1 << 0) | (1 << 1)
+    # Eq. 7's threshold is inclusive: a similarity equal to theta qualifies
+    tab2 = orc.tables(sim, group, x, 0.75, 0.25, F, B, tau, 1.0, 1.0, 0.5, 0.5)
+    assert int(tab2.subst[0]) == (1 << 3)    # Sim(0, 3) = 0.75 = theta
+    assert int(tab2.subst[3]) == (1 << 0) | (1 << 1)
 
 
 def test_tables_placement_mask(orc):
@@ -472,6 +476,18 @@ def test_rmsnorm_closed_forms(orc):
     np.testing.assert_array_equal(x[2], np.r_[np.full(8, bits_to_f(bf16_bits([np.sqrt(2.0)]))[0]),
                                               np.zeros(8)].astype(np.float32))
     np.testing.assert_array_equal(x[3], np.r_[[4.0], np.zeros(d - 1)].astype(np.float32))
+
+
+def test_rmsnorm_epsilon_in_the_root(orc):
+    """eps sits inside the root: a zero row stays zero (0 / sqrt(eps)), and a
+    constant row c gives c / sqrt(c^2 + eps): with c = 2^-8 and eps = 2^-16
+    that is 2^-8 / sqrt(2^-15) = sqrt(2) / 2 (1 without eps)."""
+    d = 8
+    h = np.zeros((2, d), np.float32)
+    h[1] = 2.0 ** -8
+    x = bits_to_f(orc.rmsnorm(bf16_bits(h), eps=2.0 ** -16))
+    np.testing.assert_array_equal(x[0], np.zeros(d, np.float32))
+    np.testing.assert_array_equal(x[1], np.full(d, bits_to_f(bf16_bits([np.sqrt(0.5)]))[0]))
 
 
 def test_rmsnorm_scale_invariant_and_unit_rms(orc):
