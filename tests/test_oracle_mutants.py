@@ -16,6 +16,20 @@ import pytest
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 SRC = os.path.join(ROOT, "oracle", "ordermoe_oracle.cpp")
 
+# anchors inside orc_select_lookahead (each occurs once in the source)
+LA_TIE = ("cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, m, kk, qn, qbar);\n"
+          "          const int sub = exact ? 0 : 1;\n          const int away = (m != s) ? 1 : 0;\n"
+          "          bool better;\n          if (!have) better = true;\n"
+          "          else if (cost != best_cost) better = cost < best_cost;\n"
+          "          else if (sub != best_sub) better = sub < best_sub;")
+LA_END = ("      if (!have) return ORC_BAD_ARG;\n      chosen[(int64_t)t * k + j] = best_k;\n"
+          "      server[(int64_t)t * k + j] = static_cast<uint8_t>(best_m);\n"
+          "      kind[(int64_t)t * k + j] = static_cast<uint8_t>(2 * best_away + best_sub);\n"
+          "      if (best_sub) {\n        taken |= (uint64_t)1 << best_k;\n"
+          "        q = q + Qtab[r * E + best_k];\n      }\n      if (j == 0) first_server = best_m;")
+LA_DIST = ("          if ((taken >> kk) & 1u) continue;\n"
+           "          if (!(q + Qtab[r * E + kk] <= qbar)) continue;\n        }\n        const float qn")
+
 # (name, original text, planted mistake)
 MUTANTS = [
     ("router: W transposed", "acc += bf(X, (int64_t)t * d + c) * bf(W, (int64_t)e * d + c);",
@@ -169,6 +183,38 @@ MUTANTS = [
      "const double benefit = pi[m] * 1.0 * cover"),
     ("Eq. 35: capacity strict", "if (!(used[m] + p[l * E + j] <= C[m])) continue;",
      "if (!(used[m] + p[l * E + j] < C[m])) continue;"),
+    ("grouping: visited by increasing count", "return count[a] > count[b]; });",
+     "return count[a] < count[b]; });"),
+    ("grouping: equal counts visited from the higher index",
+     "std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return count[a] > count[b]; });",
+     "std::sort(order.begin(), order.end(), "
+     "[&](int a, int b) { return count[a] > count[b] || (count[a] == count[b] && a > b); });"),
+    ("Eq. 4: a zero-norm pair gets Sim 1", "{ sim[i * E + j] = 0.0f; continue; }",
+     "{ sim[i * E + j] = 1.0f; continue; }"),
+    ("permutation: slot instead of token", "row_token[row] = static_cast<int32_t>(i / k);",
+     "row_token[row] = static_cast<int32_t>(i % k);"),
+    ("gather: the first token's row everywhere", "X + (int64_t)row_token[r] * d",
+     "X + (int64_t)row_token[0] * d"),
+    ("Eq. 23: utility from the means", "out[0] = omega_T * st + omega_Q * sq;",
+     "out[0] = omega_T * tbar + omega_Q * qbar;"),
+    ("Eq. 14: transfers not counted", "trans = z / B[s * M + m] + tau[s * M + m];\n          ++n;",
+     "trans = z / B[s * M + m] + tau[s * M + m];"),
+    ("Eq. 32: unplaced experts cover their group",
+     "if (placement_l[m * E + e]) cover[m * K + group_l[e]] = 1;", "cover[m * K + group_l[e]] = 1;"),
+    ("Eq. 42: future budget from the loss before the substitute",
+     "const float qn = exact ? q : q + Qtab[r * E + kk];", "const float qn = q;"),
+    ("softmax: renormalised over all experts", "for (int j = 0; j < k; ++j) ssel += p[order[j]];",
+     "for (int j = 0; j < E; ++j) ssel += p[order[j]];"),
+] + [
+    # the same rules in the look-ahead's own copy of the selection loop
+    ("look-ahead tie: substitute before the exact expert", LA_TIE,
+     LA_TIE.replace("better = sub < best_sub;", "better = sub > best_sub;")),
+    ("look-ahead Eq. 44: loss not accumulated", LA_END,
+     LA_END.replace("        q = q + Qtab[r * E + best_k];\n", "")),
+    ("look-ahead Eq. 44: location from the last slot", LA_END,
+     LA_END.replace("if (j == 0) first_server = best_m;", "first_server = best_m;")),
+    ("look-ahead: distinct experts ignored", LA_DIST,
+     LA_DIST.replace("          if ((taken >> kk) & 1u) continue;\n", "")),
 ]
 
 

@@ -647,6 +647,27 @@ def test_select_equal_costs_prefer_the_exact_expert_then_the_lower_substitute(or
     assert (ch[0, 0], sv[0, 0], kd[0, 0]) == (1, 0, 1)
 
 
+def test_lookahead_ties_follow_the_myopic_rule(orc):
+    """With P = 0 the cost-to-go is 0 (every term has P = 0), so Eq. 43 with
+    H = 2 takes the same decisions as H = 1, ties included: the exact target
+    before an equally cheap substitute, and the lower of two equally cheap
+    substitutes on one server."""
+    E, M = 3, 2
+    A = np.zeros((M, M, M), np.float32); A[0, 0, 1] = 0.5; A[0, 0, 0] = 0.25
+    Cq = np.zeros((E, E), np.float32); Cq[0, 1] = 0.25
+    Q = np.zeros((E, E), np.float32); Q[0, 1] = 0.125
+    tab = hand_tables(orc, E, M, 0.5, A, Q, Cq, subst=[0b010, 0, 0], pmask=[0b10, 0b01, 0b00])
+    A2 = np.zeros((M, M, M), np.float32); A2[0, 0, 1] = 1.0
+    Cq2 = np.zeros((E, E), np.float32); Cq2[0, 1] = Cq2[0, 2] = 0.25
+    Q2 = np.zeros((E, E), np.float32); Q2[0, 1] = Q2[0, 2] = 0.125
+    tab2 = hand_tables(orc, E, M, 0.5, A2, Q2, Cq2, subst=[0b110, 0, 0], pmask=[0b10, 0b01, 0b01])
+    P = np.zeros((1, E, E), np.float32)
+    z = lambda: (np.zeros(1, np.uint8), np.zeros(1, np.uint8), np.zeros(1, np.float32))
+    for t, want in ((tab, (0, 1, 2)), (tab2, (1, 0, 1))):
+        ch, sv, kd, _, _ = orc.select_lookahead(np.array([[0]], np.int32), [t, t], P, *z())
+        assert (ch[0, 0], sv[0, 0], kd[0, 0]) == want
+
+
 def test_phi_budget_is_inclusive(orc):
     """Eq. 42 takes the next layer's substitutes under the same rule as Eq. 40:
     with Q_hat = 0.25 and Q(1 -> 0) = 0.25 the substitute is feasible at
