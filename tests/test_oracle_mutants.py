@@ -205,6 +205,20 @@ MUTANTS = [
      "const float qn = exact ? q : q + Qtab[r * E + kk];", "const float qn = q;"),
     ("softmax: renormalised over all experts", "for (int j = 0; j < k; ++j) ssel += p[order[j]];",
      "for (int j = 0; j < E; ++j) ssel += p[order[j]];"),
+    ("Eq. 37: links read transposed", "double trans = z / B[s * M + m] + tau[s * M + m];",
+     "double trans = z / B[m * M + s] + tau[m * M + s];"),
+    ("Eq. 41: an empty row spread uniformly",
+     "row > 0.0 ? static_cast<float>(count[((size_t)l * E + a) * E + b] / row) : 0.0f;",
+     "row > 0.0 ? static_cast<float>(count[((size_t)l * E + a) * E + b] / row) : 1.0f / E;"),
+    ("Eq. 4: the diagonal computed, not 1", "if (i == j) { sim[i * E + j] = 1.0f; continue; }", ""),
+    ("Eq. 29: load not updated", "      x[best * E + j] = 1;\n      b[best] += pl[j];\n    }",
+     "      x[best * E + j] = 1;\n    }"),
+    ("waiting list: overflow not reported", "if (b[best] > C[best]) overflow = true;", ""),
+    ("Eq. 34: replicas not counted", "replicas[bm]++;", ""),
+    ("Eq. 45: projected onto [0, inf) only", "wq = std::min(1.0, std::max(0.0, wq));",
+     "wq = std::max(0.0, wq);"),
+    ("Eq. 45: projected onto (-inf, 1] only", "wq = std::min(1.0, std::max(0.0, wq));",
+     "wq = std::min(1.0, wq);"),
 ] + [
     # the same rules in the look-ahead's own copy of the selection loop
     ("look-ahead tie: substitute before the exact expert", LA_TIE,

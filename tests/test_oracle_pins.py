@@ -1076,6 +1076,7 @@ def test_transitions_brute_force(orc):
     N, L, E, kf = 40, 4, 6, 2
     logits = rng.standard_normal((N, L, E)).astype(np.float32)
     logits[0, 1, :] = 0.5                       # ties
+    logits[:, 0, 5] = -10.0                     # expert 5 never in the top-2 at layer 0
     cnt, P = orc.transitions(logits, kf)
     ref = np.zeros((L - 1, E, E), np.int64)
     for n in range(N):
@@ -1087,6 +1088,8 @@ def test_transitions_brute_force(orc):
     rows = ref.sum(axis=2, keepdims=True)
     np.testing.assert_allclose(P, np.where(rows > 0, ref / np.maximum(rows, 1), 0), rtol=1e-7)
     assert cnt.sum() == (L - 1) * N * kf * kf
+    # a row without transitions is 0 (Eq. 41's quotient has no denominator there)
+    assert (cnt[0, 5] == 0).all() and (P[0, 5] == 0).all()
 
 
 def _rand_tables(orc, rng, E, M, kgroups, tau_scale=1.0):
