@@ -219,6 +219,24 @@ MUTANTS = [
      "wq = std::max(0.0, wq);"),
     ("Eq. 45: projected onto (-inf, 1] only", "wq = std::min(1.0, std::max(0.0, wq));",
      "wq = std::min(1.0, wq);"),
+    ("topk: larger logits ranked last", "  if (a != b) return a > b;\n  return ia < ib;",
+     "  if (a != b) return a < b;\n  return ia < ib;"),
+    ("softmax: not normalised", "for (int e = 0; e < E; ++e) p[e] /= s;", ""),
+    ("topk: a NaN logit accepted", "if (std::isnan(l[e])) return ORC_NAN;", ""),
+    ("placement order: size ascending", "if (!same(pl[a], pl[c])) return above(pl[a], pl[c]);",
+     "if (!same(pl[a], pl[c])) return above(pl[c], pl[a]);"),
+    ("placement order: equal keys by the higher index", "      return a < c;\n    });",
+     "      return a > c;\n    });"),
+    ("Eq. 20: loss read from the exact expert's entry",
+     "if (kk != r) q = q + static_cast<double>(Qtab[((size_t)l * E + r) * E + kk]);",
+     "if (kk != r) q = q + static_cast<double>(Qtab[((size_t)l * E + r) * E + r]);"),
+    ("Eq. 23: means over T - 1", "const double tbar = st / T, qbar = sq / T;",
+     "const double tbar = st / (T - 1 > 0 ? T - 1 : 1), qbar = sq / (T - 1 > 0 ? T - 1 : 1);"),
+    ("Eq. 28: no activations give frequency 1", "double f = total > 0.0 ? count[j] / total : 0.0;",
+     "double f = total > 0.0 ? count[j] / total : 1.0;"),
+    ("Eq. 6: theta_min and theta_max swapped",
+     "return static_cast<float>(theta_min + (theta_max - theta_min) * frac);",
+     "return static_cast<float>(theta_max + (theta_min - theta_max) * frac);"),
 ] + [
     # the same rules in the look-ahead's own copy of the selection loop
     ("look-ahead tie: substitute before the exact expert", LA_TIE,

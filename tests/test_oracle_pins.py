@@ -783,6 +783,9 @@ def test_importance_closed_forms(orc):
     I2 = orc.importance(sim, cnt, group, 0.75, 0.25)
     np.testing.assert_allclose(I2, [0.75 * 0.5 + 0.25 * 0.8, 0.75 * 0.25 + 0.25 * 0.8,
                                     0.75 * 0.25 + 0.25 * 1.0], rtol=1e-7)
+    # no activations at all: the frequency term is 0, the importance alpha_r * rho
+    I3 = orc.importance(sim, np.zeros(3, np.int32), group, 0.75, 0.25)
+    np.testing.assert_allclose(I3, [0.25 * 0.8, 0.25 * 0.8, 0.25 * 1.0], rtol=1e-7)
 
 
 def test_place_hand_example_disperses_groups(orc):
