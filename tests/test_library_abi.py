@@ -57,3 +57,21 @@ def test_size_queries_without_gpu(libpath):
     assert B.ordermoe_tables_bytes(65, 4) == 0 and B.ordermoe_tables_bytes(8, 33) == 0
     assert B.ordermoe_dispatch_workspace_bytes(4096, 2, 8) >= 32 * 8 * 4
     assert B.ordermoe_dispatch_workspace_bytes(10, 2, 65) == 0
+
+
+def test_no_cluster_multicast_copies_in_the_kernels():
+    """No bulk copy in the library carries .multicast::cluster: bench.py's
+    replicas run the same kernels on every GPU of a node, so every CTA loads
+    its own boxes. (The tcgen05.commit arrive on both CTAs of a pair is a
+    barrier signal, not a copy, and may multicast.)"""
+    csrc = os.path.join(ROOT, "paper_2607_17154_gb300", "csrc")
+    bad, copies = [], 0
+    for path in sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh"))):
+        text = open(path).read()
+        # PTX strings are split over adjacent literals: join each asm statement first
+        for stmt in re.findall(r"asm\s+volatile\s*\((.*?)\);", text, flags=re.S):
+            ptx = "".join(re.findall(r'"((?:[^"\\]|\\.)*)"', stmt))
+            copies += "cp.async.bulk" in ptx
+            if "cp.async.bulk" in ptx and "multicast::cluster" in ptx:
+                bad.append((os.path.basename(path), ptx[:80]))
+    assert copies > 0 and not bad, (copies, bad)
