@@ -237,6 +237,20 @@ MUTANTS = [
     ("Eq. 6: theta_min and theta_max swapped",
      "return static_cast<float>(theta_min + (theta_max - theta_min) * frac);",
      "return static_cast<float>(theta_max + (theta_min - theta_max) * frac);"),
+    ("router: fp32 running sum",
+     "      double acc = 0.0;\n      for (int c = 0; c < d; ++c) acc += bf(X, (int64_t)t * d + c)",
+     "      float acc = 0.0f;\n      for (int c = 0; c < d; ++c) acc += bf(X, (int64_t)t * d + c)"),
+    ("combine: fp32 running sum",
+     "      double acc = 0.0;\n      for (int j = 0; j < k; ++j) {\n        int64_t row",
+     "      float acc = 0.0f;\n      for (int j = 0; j < k; ++j) {\n        int64_t row"),
+    ("Eq. 3: similarity's H as an fp32 running sum",
+     "      double acc = 0.0;\n      for (int c = 0; c < d; ++c) acc += bf(W, (int64_t)e * d + c) * bf(Xc, n * d + c);",
+     "      float acc = 0.0f;\n      for (int c = 0; c < d; ++c) acc += bf(W, (int64_t)e * d + c) * bf(Xc, n * d + c);"),
+    ("RMSNorm: mean over d - 1", "std::sqrt(ss / d + eps)", "std::sqrt(ss / (d - 1) + eps)"),
+    ("Eq. 5: one slot short", "for (int j = 0; j < kf; ++j) count[order[j]]++;",
+     "for (int j = 0; j + 1 < kf; ++j) count[order[j]]++;"),
+    ("Eq. 37: a transfer on the same server", "        if (s != m) {\n          double trans",
+     "        if (true) {\n          double trans"),
 ] + [
     # the same rules in the look-ahead's own copy of the selection loop
     ("look-ahead tie: substitute before the exact expert", LA_TIE,

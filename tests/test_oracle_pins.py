@@ -44,6 +44,28 @@ def test_router_logits_exact_rational(orc):
             assert got[t, e] == np.float32(float(exact))
 
 
+def test_sums_are_exact_before_their_one_rounding(orc):
+    """The oracle's sums (the router logits and the similarity's H, Eq. 3;
+    the weighted combine of a token's slots) are exact up to their single
+    final rounding: 2^24 + 1 - 2^24 is 1, although a running fp32 sum would
+    lose the 1 to rounding. All inputs are exact in bf16."""
+    big = 2.0 ** 12
+    # router: x . w = 2^24 + 1 - 2^24
+    X = bf16_bits([[big, 1.0, big]]); W = bf16_bits([[big, 1.0, -big]])
+    assert orc.router_logits(X, W)[0, 0] == 1.0
+    # combine: sum_j w_j Y_j with Y = (2^24, 1, -2^24) and unit weights
+    Y = bf16_bits([[2.0 ** 24], [1.0], [-(2.0 ** 24)]])
+    y = orc.combine(Y, np.array([[0, 1, 2]], np.int32), np.ones((1, 3), np.float32))
+    assert bits_to_f(y)[0, 0] == 1.0
+    # similarity: expert 0's activations are (1, 1) only when the cancelling
+    # token keeps its 1; expert 1's are (2^12, 0): Sim = 1 / sqrt(2)
+    Wr = bf16_bits([[big, 1.0, -big], [1.0, 0.0, 0.0]])
+    Xc = bf16_bits([[big, 1.0, big], [0.0, 1.0, 0.0]])
+    sim, H = orc.similarity(Wr, Xc, return_H=True)
+    np.testing.assert_array_equal(H, np.array([[1.0, 1.0], [big, 0.0]], np.float32))
+    assert sim[0, 1] == np.float32(1.0 / np.sqrt(2.0))
+
+
 def test_router_logits_one_hot_tokens_pick_weight_columns(orc):
     rng = np.random.default_rng(2)
     E, d = 3, 11
