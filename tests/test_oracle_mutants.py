@@ -251,6 +251,11 @@ MUTANTS = [
      "for (int j = 0; j + 1 < kf; ++j) count[order[j]]++;"),
     ("Eq. 37: a transfer on the same server", "        if (s != m) {\n          double trans",
      "        if (true) {\n          double trans"),
+    ("Eq. 36: location taken from the home server", "const int s = loc[t];", "const int s = home[t];"),
+    ("Eq. 44: the token's loss restarts at 0", "float q = qhat[t];", "float q = 0.0f;"),
+    ("Eq. 44: loss not written back", "    qhat[t] = q;\n", "\n"),
+    ("Eq. 42: minimum started at 0", "    if (p == 0.0f) continue;\n    float best = INFINITY;",
+     "    if (p == 0.0f) continue;\n    float best = 0.0f;"),
 ] + [
     # the same rules in the look-ahead's own copy of the selection loop
     ("look-ahead tie: substitute before the exact expert", LA_TIE,
