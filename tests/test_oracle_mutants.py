@@ -256,6 +256,17 @@ MUTANTS = [
     ("Eq. 44: loss not written back", "    qhat[t] = q;\n", "\n"),
     ("Eq. 42: minimum started at 0", "    if (p == 0.0f) continue;\n    float best = INFINITY;",
      "    if (p == 0.0f) continue;\n    float best = 0.0f;"),
+    ("Eq. 43: horizon one short",
+     "cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, m, kk, qn, qbar);",
+     "cost = cost + orc_phi(H - 2, tabs.data(), P, E, M, a, m, kk, qn, qbar);"),
+    ("Eq. 42: deeper levels get the loss from before the substitute",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar)",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kk, qacc, qbar)"),
+    ("Eq. 13: transfer time z * B", "double trans = z / B[s * M + m] + tau[s * M + m];",
+     "double trans = z * B[s * M + m] + tau[s * M + m];"),
+    ("Eq. 27: the expert left out of its group's mean",
+     "if (group[k] == group[j]) { s += sim[j * E + k]; ++size; }",
+     "if (group[k] == group[j] && k != j) { s += sim[j * E + k]; ++size; }"),
 ] + [
     # the same rules in the look-ahead's own copy of the selection loop
     ("look-ahead tie: substitute before the exact expert", LA_TIE,

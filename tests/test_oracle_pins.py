@@ -706,6 +706,29 @@ def test_phi_budget_is_inclusive(orc):
     assert orc.phi(1, [t0, t1], P, 0, 0, 0, 0.3) == 1.0     # above the budget: exact only
 
 
+def test_phi_carries_a_substitute_loss_to_the_deeper_level(orc):
+    """Eq. 42 with two future layers, Qbar = 0.5, Q_hat = 0.25. At layer l+1
+    the next target 1 runs exactly on server 1 (cost 1) or as substitute 0 on
+    server 0 (Cq 0.125), which brings the loss to 0.5. At layer l+2 target 1
+    again: exact on server 1 (1 from server 0, 0 from server 1) or substitute 0
+    on server 0 (loss 0.125, free). After the substitute at l+1 the one at l+2
+    no longer fits the budget (0.5 + 0.125 > 0.5), so that path costs
+    0.125 + 1 against 1 + 0 for the exact one: Phi^(2) = 1. Carrying the loss
+    from before the substitute would wrongly let the path cost 0.125."""
+    E, M = 2, 2
+    t0 = hand_tables(orc, E, M, 0.5, np.zeros((M, M, M), np.float32), pmask=[0b01, 0b10])
+    A1 = np.zeros((M, M, M), np.float32); A1[0, 0, 1] = 1.0
+    t1 = hand_tables(orc, E, M, 0.5, A1, Q=[[0, 0], [0.25, 0]], Cq=[[0, 0], [0.125, 0]],
+                     subst=[0, 0b01], pmask=[0b01, 0b10])
+    A2 = np.zeros((M, M, M), np.float32); A2[0, 0, 1] = 1.0; A2[0, 1, 0] = 1.0
+    t2 = hand_tables(orc, E, M, 0.5, A2, Q=[[0, 0], [0.125, 0]], subst=[0, 0b01],
+                     pmask=[0b01, 0b10])
+    P = np.zeros((2, E, E), np.float32)
+    P[0, 0, 1] = 1.0                      # l -> l+1: from expert 0 to target 1
+    P[1, 0, 1] = P[1, 1, 1] = 1.0         # l+1 -> l+2: to target 1
+    assert orc.phi(2, [t0, t1, t2], P, 0, 0, 0, 0.25) == 1.0
+
+
 def test_place_load_term_is_weighted_by_lambda1(orc):
     """Eq. 30's score lambda1 b_m / C_m + lambda2 eta_m with lambda1 = 0.25 and
     lambda2 = 0.375. Experts in order 0, 1, 2 (p desc, then importance):
