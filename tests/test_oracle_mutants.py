@@ -267,6 +267,17 @@ MUTANTS = [
     ("Eq. 27: the expert left out of its group's mean",
      "if (group[k] == group[j]) { s += sim[j * E + k]; ++size; }",
      "if (group[k] == group[j] && k != j) { s += sim[j * E + k]; ++size; }"),
+    ("Eq. 42: deeper levels measured from the home server",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar)",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, a, kk, q2, qbar)"),
+    ("Eq. 42: deeper levels follow the target, not the executed expert",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kk, q2, qbar)",
+     "orc_phi(h - 1, tabs + 1, P + (size_t)E * E, E, M, a, m2, kt, q2, qbar)"),
+    ("Eq. 42: any substitute of the next target", "if (!((t1.subst[kt] >> kk) & 1u)) continue;", ""),
+    ("Eq. 42: any server for the next expert", "if (!((t1.pmask[kk] >> m2) & 1u)) continue;", ""),
+    ("Eq. 43: cost-to-go from the pre-layer location",
+     "cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, m, kk, qn, qbar);",
+     "cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, s, kk, qn, qbar);"),
 ] + [
     # the same rules in the look-ahead's own copy of the selection loop
     ("look-ahead tie: substitute before the exact expert", LA_TIE,

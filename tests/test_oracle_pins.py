@@ -729,6 +729,27 @@ def test_phi_carries_a_substitute_loss_to_the_deeper_level(orc):
     assert orc.phi(2, [t0, t1, t2], P, 0, 0, 0, 0.25) == 1.0
 
 
+def test_phi_continues_from_the_executed_substitute(orc):
+    """Eq. 42 two layers ahead: at layer l+1 the next target 1 runs exactly on
+    server 1 (cost 1) or as substitute 0 on server 0 (Cq 0.125). The layer
+    after follows the transitions of the expert that ran: from 0 to target 0
+    (on server 0, cost 0 from server 0), from 1 to target 1 (on server 1, 0
+    from server 1, 1 from server 0). So the substitute path costs
+    0.125 + 0 and the exact one 1 + 0: Phi^(2) = 0.125. Following the target's
+    row instead (1 -> 1) would cost the substitute path 0.125 + 1."""
+    E, M = 2, 2
+    t0 = hand_tables(orc, E, M, 0.5, np.zeros((M, M, M), np.float32), pmask=[0b01, 0b10])
+    A1 = np.zeros((M, M, M), np.float32); A1[0, 0, 1] = 1.0
+    t1 = hand_tables(orc, E, M, 0.5, A1, Q=[[0, 0], [0.25, 0]], Cq=[[0, 0], [0.125, 0]],
+                     subst=[0, 0b01], pmask=[0b01, 0b10])
+    A2 = np.zeros((M, M, M), np.float32); A2[0, 0, 1] = 1.0; A2[0, 1, 0] = 1.0
+    t2 = hand_tables(orc, E, M, 0.5, A2, pmask=[0b01, 0b10])
+    P = np.zeros((2, E, E), np.float32)
+    P[0, 0, 1] = 1.0                      # l -> l+1: from expert 0 to target 1
+    P[1, 0, 0] = P[1, 1, 1] = 1.0         # l+1 -> l+2: each expert to itself
+    assert orc.phi(2, [t0, t1, t2], P, 0, 0, 0, 0.0) == 0.125
+
+
 def test_place_load_term_is_weighted_by_lambda1(orc):
     """Eq. 30's score lambda1 b_m / C_m + lambda2 eta_m with lambda1 = 0.25 and
     lambda2 = 0.375. Experts in order 0, 1, 2 (p desc, then importance):
