@@ -278,6 +278,14 @@ MUTANTS = [
     ("Eq. 43: cost-to-go from the pre-layer location",
      "cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, m, kk, qn, qbar);",
      "cost = cost + orc_phi(H - 1, tabs.data(), P, E, M, a, s, kk, qn, qbar);"),
+    ("Eq. 32: coverage updated on server 0",
+     "    y[((size_t)bm * L + bl) * E + group[bl * E + bj]] = 1;",
+     "    y[((size_t)0 * L + bl) * E + group[bl * E + bj]] = 1;"),
+    ("Eq. 35: memory charged to server 0", "used[bm] += p[bl * E + bj];", "used[0] += p[bl * E + bj];"),
+    ("Eq. 34: replica not written", "placement[((size_t)bl * M + bm) * E + bj] = 1;", ""),
+    ("Eq. 32: initial coverage from server 0's placement",
+     "if (placement[((size_t)l * M + m) * E + j])\n          y[",
+     "if (placement[((size_t)l * M + 0) * E + j])\n          y["),
 ] + [
     # the same rules in the look-ahead's own copy of the selection loop
     ("look-ahead tie: substitute before the exact expert", LA_TIE,
